@@ -1,0 +1,360 @@
+"""Benchmark of the logits-side hot path of verifier-skipping SDD on GB300.
+
+One step = one fused round of the whole path over one batch of draft blocks:
+confidence statistics of every drafter row, the prefix skip schedule, strict
+(shadow) verification of every block with residual / bonus resampling,
+lenience and top-k acceptance on the same target read, agreement counters and
+the committed tokens (``sdd_block`` = ``sdd_block_scan`` + ``sdd_block_decide``).
+
+Default workload (c3): B=16 blocks, gamma=32, V=151,936, bf16 drafter and
+target logits; half the positions peaked, half flat; strict sampling, lenience
+ell in {1.5, 2, 4} (paper convention 1/ell), top-k k in {2, 5, 10}, raw
+confidence schedule at tau=0.9.  Inputs are seeded synthetic logits (no model
+weights are available); three input sets of 316 MB each rotate, so every step
+reads its logits from HBM, not L2.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--workload c3]
+Prints one JSON line (rank 0).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "draft blocks verified+scheduled/sec at γ=32,V=151,936 bf16; achieved HBM GB/s vs peak"
+UNIT = "blocks/s"
+NEAR = 1e-6
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def _workload_cfg(name):
+    from paper_2608_14787_gb300 import synth
+    wl = synth.WORKLOADS[name]
+    ells = tuple(synth.paper_ell(e) for e in wl.ells)
+    return wl, ells, tuple(wl.topks)
+
+
+def _config_json(wl, ells, ks):
+    return {
+        "workload": f"{wl.name}: {wl.description}",
+        "B": wl.B, "gamma": wl.gamma, "V": wl.V, "dtype": "bf16" if "bfloat16" in str(wl.dtype) else "fp32",
+        "taus": list(wl.taus), "ell_paper": [round(e, 6) for e in ells], "topk": list(ks),
+        "strict": "sampling with residual/bonus resampling, shadow-verifies every block",
+        "K_min": 6, "S_max": 64,
+        "l2": "inputs larger than L2: 3 rotating input sets of (2*gamma+1)*V*2*B bytes each",
+    }
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+
+    FIELDS = ("index,pci.bus_id,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, bus_id: str | None):
+        self.bus_id = (bus_id or "").lower()
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        time.sleep(0.2)
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        rows = []
+        for l in getattr(self, "lines", []):
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 10:
+                continue
+            if self.bus_id and self.bus_id not in f[1].lower() and f[1].lower() not in self.bus_id:
+                continue
+            rows.append(f)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"], "samples": 0}
+        sm = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        mx = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[6 + i].lower() == "active"})
+        pw = [float(r[4]) for r in rows if r[4].replace(".", "").isdigit()]
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows), "power_w_max": max(pw) if pw else None}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def run_reference(args):
+    """The fp64 CPU oracle, as it stands, on a bounded sample per step (one block)."""
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return 0
+    import numpy as np
+    import torch
+    import oracle as orc
+    from paper_2608_14787_gb300 import synth
+    wl, ells, ks = _workload_cfg(args.workload)
+    blk = synth.make_block(wl, device="cpu", round_=0)
+    zd = blk.z_d.view(torch.int16).numpy().view(np.uint16) if wl.dtype == torch.bfloat16 else blk.z_d.numpy()
+    zt = blk.z_t.view(torch.int16).numpy().view(np.uint16) if wl.dtype == torch.bfloat16 else blk.z_t.numpy()
+    xs = blk.x.numpy()
+
+    def one_block(b):
+        st = orc.row_stats(zd[b:b + 1], tokens=xs[b:b + 1])
+        for tau in wl.taus:
+            orc.schedule(st.q, 0, tau, tau, 6, 64)
+        orc.verify_strict(zt[b], zd[b], xs[b], seed=wl.seed, b=b, round_=0)
+        f = orc.target_facts(zt[b], xs[b])
+        for e in ells:
+            orc.verify_lenient(f, xs[b], e)
+        for k in ks:
+            orc.verify_topk(f, xs[b], k)
+
+    for s in range(args.warmup):
+        one_block(s % wl.B)
+    t0 = time.perf_counter()
+    for s in range(args.steps):
+        one_block(s % wl.B)
+    dt = time.perf_counter() - t0
+    value = args.steps / dt
+    sample = f"one {wl.name} block (gamma={wl.gamma}, V={wl.V}) per step, all rules, single thread"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": _config_json(wl, ells, ks),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def _cpu_baseline(wl, ells, ks, blk_host, n_blocks):
+    """Time the oracle on the first n_blocks blocks of one input set (bounded sample)."""
+    import numpy as np
+    import torch
+    import oracle as orc
+    zd = blk_host["z_d"]
+    zt = blk_host["z_t"]
+    xs = blk_host["x"]
+    t0 = time.perf_counter()
+    for b in range(n_blocks):
+        st = orc.row_stats(zd[b:b + 1], tokens=xs[b:b + 1])
+        for tau in wl.taus:
+            orc.schedule(st.q, 0, tau, tau, 6, 64)
+        orc.verify_strict(zt[b], zd[b], xs[b], seed=wl.seed, b=b, round_=0)
+        f = orc.target_facts(zt[b], xs[b])
+        for e in ells:
+            orc.verify_lenient(f, xs[b], e)
+        for k in ks:
+            orc.verify_topk(f, xs[b], k)
+    dt = time.perf_counter() - t0
+    del np, torch
+    return {"value": n_blocks / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{n_blocks} of the {wl.B} blocks of one {wl.name} input set, all rules, single thread "
+                      f"({dt:.1f} s)"}
+
+
+def run_gpu(args):
+    import torch
+    import paper_2608_14787_gb300 as sdd
+    from paper_2608_14787_gb300 import build as sdd_build
+    from paper_2608_14787_gb300 import synth
+
+    ws, rank, local = _dist()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if rank == 0:
+        sdd_build.build()
+    if ws > 1:
+        dist.barrier()
+    sdd.load()
+
+    wl, ells, ks = _workload_cfg(args.workload)
+    B, gamma, V = wl.B, wl.gamma, wl.V
+    n_sets = 3
+    sets = [synth.make_block(wl, device=dev, round_=r + 1000 * rank) for r in range(n_sets)]
+    rnd = sdd.BlockRound(B, gamma, V, dtype=wl.dtype, taus=wl.taus, ells=ells, ks=ks, K_min=6, S_max=64,
+                         device=dev)
+    esz = 2 if wl.dtype == torch.bfloat16 else 4
+    scan_bytes = (2 * gamma + 1) * V * esz * B          # every logit read once
+    stream = torch.cuda.current_stream()
+
+    def step(i, ev=None):
+        s = sets[i % n_sets]
+        rnd.set_inputs(s.z_d, s.z_t, s.x, seed=wl.seed, round_=i)
+        if ev is not None:
+            ev[0].record(stream)
+        rnd.scan()
+        if ev is not None:
+            ev[1].record(stream)
+        rnd.decide()
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    if int(rnd.status.item()) != 0:
+        raise RuntimeError(f"device status {int(rnd.status.item())} after warm-up")
+
+    # ---- device-resident timed region ----
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    bus = torch.cuda.get_device_properties(dev).pci_bus_id if hasattr(torch.cuda.get_device_properties(dev),
+                                                                      "pci_bus_id") else None
+    if ws > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(bus) as clk:
+        t_start.record(stream)
+        for i in range(args.steps):
+            step(i, evs[i])
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    if ws > 1:
+        dist.barrier()
+    total_ms = t_start.elapsed_time(t_end)
+    scan_ms = [a.elapsed_time(b) for a, b in evs]
+    scan_avg_ms = sum(scan_ms) / len(scan_ms)
+    if ws > 1:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    value = ws * B * args.steps / (total_ms / 1e3)
+    status = int(rnd.status.item())
+
+    # ---- end-to-end through the C ABI from pinned host buffers ----
+    hz_d = sets[0].z_d.cpu().pin_memory()
+    hz_t = sets[0].z_t.cpu().pin_memory()
+    hx = sets[0].x.cpu().pin_memory()
+    dz_d, dz_t, dx = sets[0].z_d, sets[0].z_t, sets[0].x
+    outs = [rnd.L_strict, rnd.tokens_strict, rnd.K, rnd.commit_tokens, rnd.commit_n, rnd.q]
+    h_outs = [torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs]
+    e2e_steps = max(3, min(args.steps, 200))
+    h2d = hz_d.numel() * hz_d.element_size() + hz_t.numel() * hz_t.element_size() + hx.numel() * 4
+    d2h = sum(o.numel() * o.element_size() for o in outs)
+
+    def e2e_step(i):
+        dz_d.copy_(hz_d, non_blocking=True)
+        dz_t.copy_(hz_t, non_blocking=True)
+        dx.copy_(hx, non_blocking=True)
+        rnd.set_inputs(dz_d, dz_t, dx, seed=wl.seed, round_=i)
+        rnd.run()
+        for h, d in zip(h_outs, outs):
+            h.copy_(d, non_blocking=True)
+
+    for i in range(2):
+        e2e_step(i)
+    torch.cuda.synchronize()
+    if ws > 1:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(e2e_steps):
+        e2e_step(i)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    if ws > 1:
+        t = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    e2e_value = ws * B * e2e_steps / (e2e_ms / 1e3)
+
+    peak, peak_kind = _peaks()
+    achieved = scan_bytes / (scan_avg_ms / 1e3) / 1e9
+    line = None
+    if rank == 0:
+        cpu = None
+        if ws == 1 and not args.no_cpu_baseline:
+            import numpy as np
+            host = {"z_d": sets[0].z_d[:args.cpu_blocks].cpu().view(torch.int16).numpy().view(np.uint16)
+                    if wl.dtype == torch.bfloat16 else sets[0].z_d[:args.cpu_blocks].cpu().numpy(),
+                    "z_t": sets[0].z_t[:args.cpu_blocks].cpu().view(torch.int16).numpy().view(np.uint16)
+                    if wl.dtype == torch.bfloat16 else sets[0].z_t[:args.cpu_blocks].cpu().numpy(),
+                    "x": sets[0].x[:args.cpu_blocks].cpu().numpy()}
+            cpu = _cpu_baseline(wl, ells, ks, host, min(args.cpu_blocks, B))
+        clocks = clk.summary()
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if esz == 2 else "fp32", "data": "synthetic",
+            "config": _config_json(wl, ells, ks),
+            "achieved_gbs_step": scan_bytes / (total_ms / args.steps / 1e3) / 1e9,
+            "roofline": {"bound": "hbm", "kernel": "scan_kernel (sdd_block_scan)", "achieved": achieved,
+                         "peak": peak, "unit": "GB/s", "frac": achieved / peak, "traffic": args.traffic,
+                         "peak_source": f"{peak_kind} hbm_gbs", "bytes_per_launch": scan_bytes,
+                         "avg_launch_ms": scan_avg_ms},
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": 2 * args.steps,
+            "clocks": clocks,
+            "device_status": status,
+        }
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=4000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--workload", default="c3")
+    ap.add_argument("--cpu-blocks", type=int, default=8)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--traffic", type=float, default=None,
+                    help="dram bytes per scan launch from an ncu capture of the current kernel")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,302 @@
+/*
+ * sdd.h -- C ABI of the GB300 (sm_103a) logits-side path of verifier-skipping
+ * speculative diffusion decoding (Luo, Sandler, Fioretto, "From Positionwise
+ * Confidence to Prefix Scheduling: Verifier Skipping in Speculative Decoding",
+ * arXiv 2608.14787).
+ *
+ * The path has two halves around the verifier call of one decoding round:
+ *   pre-verify   drafter logits -> per-position confidence -> committed prefix
+ *                length K for each threshold pair (skip the verifier, or not);
+ *   post-verify  target logits  -> accepted length L and committed tokens
+ *                under Strict SDD, lenience or top-k acceptance.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * Pointers.  Unless a parameter says "host", every array pointer is DEVICE
+ *   memory owned by the caller.  The library never allocates or frees memory,
+ *   keeps no state between calls and may be called from several host threads.
+ * Layout.  Logits are row-major [B, P, row_stride] with P = gamma drafter
+ *   positions or gamma+1 target positions (the last target row serves the bonus
+ *   token); element v of position j of batch row b sits at
+ *   ((b * P) + j) * row_stride + v.  V <= row_stride is the vocabulary size.
+ *   The base address must be 16-byte aligned and row_stride * element size a
+ *   multiple of 16 bytes; the padding elements V..row_stride-1 are never read
+ *   into any result.  Per-position arrays are [B, gamma] row-major, per-block
+ *   arrays [B], threshold-grid outputs [n, B] (grid index outermost).
+ * Streams.  Every call only enqueues work on `stream` (a cudaStream_t; NULL is
+ *   the legacy default stream) and returns without synchronising.
+ * Workspace.  Calls that take `workspace` need at least sdd_workspace_size()
+ *   bytes of device memory, 256-byte aligned and ZERO-FILLED before its first
+ *   use; every call that completes returns the arrival counters it holds to
+ *   zero, so one workspace serves any number of stream-ordered calls.  Calls that may
+ *   overlap on the GPU (different streams) need separate workspaces.  After a
+ *   call whose device status reports SDD_DEV_TIMEOUT the workspace must be
+ *   zero-filled again.
+ * Errors.  The return value reports host-side problems only: invalid
+ *   arguments are detected before anything is enqueued (SDD_ERR_INVALID_ARGUMENT)
+ *   and launch failures return SDD_ERR_CUDA.  Conditions found while the
+ *   kernels run are OR-ed into the caller's device word `*status` (bits
+ *   SDD_DEV_*; the caller clears it); no kernel traps.  sdd_last_error()
+ *   returns a message for the calling thread's last non-OK return.
+ * Dtypes.  Logits are SDD_F32 or SDD_BF16; all arithmetic is fp32 with fp64
+ *   where sums and threshold comparisons need it.
+ */
+#ifndef SDD_H
+#define SDD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define SDD_API __attribute__((visibility("default")))
+#else
+#define SDD_API
+#endif
+
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st *sdd_stream_t;
+
+typedef enum {
+    SDD_OK = 0,
+    SDD_ERR_INVALID_ARGUMENT = 1,
+    SDD_ERR_UNSUPPORTED = 2,
+    SDD_ERR_CUDA = 3,
+    SDD_ERR_WORKSPACE = 4
+} sdd_status_t;
+
+typedef enum { SDD_F32 = 0, SDD_BF16 = 1 } sdd_dtype_t;
+
+/* Confidence signals of Sec. 4.2. */
+typedef enum { SDD_SIG_RAW = 0, SDD_SIG_MARGINAL = 1, SDD_SIG_CONDITIONAL = 2 } sdd_signal_t;
+
+/* Bits of the device status word. */
+#define SDD_DEV_NONFINITE 1u  /* a logits row held NaN or +inf, or only -inf      */
+#define SDD_DEV_BAD_TOKEN 2u  /* a drafted token or row index was out of range   */
+#define SDD_DEV_TIMEOUT 4u    /* a bounded wait on a tile copy gave up           */
+
+/* Limits. */
+#define SDD_MAX_GAMMA 128
+#define SDD_MAX_GRID 32       /* threshold pairs, lenience values or k values per call */
+
+/* ABI version (major * 10000 + minor * 100 + patch). */
+SDD_API int sdd_version(void);
+
+/* Message describing the calling thread's last non-OK return ("" if none). */
+SDD_API const char *sdd_last_error(void);
+
+/*
+ * sdd_workspace_size -- bytes of zero-filled device scratch that any entry
+ * point needs for blocks of this shape on the CURRENT device (the figure
+ * depends on its SM count).  B, gamma, V as in the calls below.
+ */
+SDD_API sdd_status_t sdd_workspace_size(int B, int gamma, int V, size_t *bytes);
+
+/*
+ * sdd_confidence -- pre-verify statistics of the drafter rows (Sec. 4.2).
+ * For each position (b, j), with z the drafter logits of that row and x_j the
+ * drafted token:
+ *   q       = p_draft(x_j) = exp(z(x_j) - LSE)      (raw confidence, Sec. 4.2)
+ *   logq    = z(x_j) - LSE
+ *   maxprob = max_v p(v)                            (top-1 probability, App. A.7)
+ *   lse     = log sum_v exp(z(v))
+ *   entropy = -sum_v p(v) ln p(v), in nats          (App. A.7 feature)
+ *   argmax  = lowest index attaining max_v z(v)
+ * All outputs are [B, gamma]; every one but q may be NULL.  A row with NaN or
+ * +inf logits, or only -inf, yields NaN statistics, argmax -1 and sets
+ * SDD_DEV_NONFINITE; a drafted token outside [0, V) yields NaN q/logq and sets
+ * SDD_DEV_BAD_TOKEN.  One streaming pass reads every logit exactly once.
+ */
+SDD_API sdd_status_t sdd_confidence(const void *draft_logits, sdd_dtype_t dtype, int B, int gamma, int V,
+                            int64_t row_stride, const int32_t *draft_tokens, float *q, float *logq,
+                            float *maxprob, float *lse, float *entropy, int32_t *argmax,
+                            void *workspace, size_t workspace_bytes, int32_t *status,
+                            sdd_stream_t stream);
+
+/*
+ * sdd_schedule_prefix -- the skip policy of Sec. 4.1 for n_tau threshold pairs
+ * (Eq. 3 and the commit rule that follows it).  For batch row b and pair t:
+ *   B_k = min_{j<=k} q_j;  C_k = (prod q)^(1/k) (RAW), min_{j<=k} q_j (MARGINAL),
+ *   prod_{j<=k} q_j (CONDITIONAL, computed in log space);
+ *   K_hat = max{k : B_k >= eta_b[t], C_k >= eta_c[t], no guarded position in 1..k}
+ *   (0 if none; for MARGINAL both gates use max(eta_b, eta_c)).
+ *   If D_in[b] >= S_max the round is strict; otherwise it skips iff K_hat > 0 and
+ *   K_hat >= K_min.  A skip writes K = K_hat and D_out = D_in + K; a strict round
+ *   writes K = 0 and D_out = 0 (every verifier call resets D).
+ * Readings fixed by this library: positions whose score is not finite count as
+ * guarded (an invalid score); force_strict[b] != 0 (a shortened final block)
+ * forces K_hat = K = 0; a pair with eta_b >= 1 or eta_c >= 1 disables skipping
+ * (K_hat = K = 0), so the threshold limit reproduces Strict SDD exactly.
+ *   q       [B, gamma] scores in [0, 1]: raw confidence from sdd_confidence, or
+ *           the output of a learned survival scorer.
+ *   logq    [B, gamma] natural log of q, or NULL (then log q is taken here).
+ *   eta_b, eta_c  HOST arrays [n_tau], 1 <= n_tau <= SDD_MAX_GRID.
+ *   guard   [B, gamma] uint8, nonzero = this position may not be skipped; NULL = none.
+ *   force_strict [B] uint8 or NULL.  D_in [B] staleness counters (NULL = all 0).
+ *   K_hat, K [n_tau, B]; D_out [n_tau, B] or NULL.
+ */
+SDD_API sdd_status_t sdd_schedule_prefix(const float *q, const float *logq, int B, int gamma,
+                                 sdd_signal_t signal, const double *eta_b, const double *eta_c,
+                                 int n_tau, int K_min, int S_max, const uint8_t *guard,
+                                 const uint8_t *force_strict, const int32_t *D_in, int32_t *K_hat,
+                                 int32_t *K, int32_t *D_out, int32_t *status, sdd_stream_t stream);
+
+/*
+ * sdd_verify_strict -- Strict SDD verification (Sec. 3.1: the standard rule of
+ * speculative decoding) of the blocks listed in rows[0..n_rows) (all B blocks
+ * when rows is NULL; then n_rows must be B).
+ *   greedy != 0 (the paper's runs, Sec. 5.1): accept x_j iff it is the lowest-
+ *     index argmax of target row j; the token after the accepted prefix is the
+ *     target argmax of row L+1 (row gamma+1 when all gamma are accepted).
+ *   greedy == 0 (sampling): accept x_j iff u_j <= p_t(x_j) / p_d(x_j) with
+ *     u_j = U(seed, j, b, round, 0); at the first rejection draw from
+ *     norm(max(0, p_t - p_d)) of that row by inverse CDF in ascending token order
+ *     with U(seed, L+1, b, round, 1) (from p_t when that residual has no mass);
+ *     when all gamma are accepted draw the bonus token from p_t of row gamma+1
+ *     with U(seed, gamma+1, b, round, 2).
+ *   U(seed, j, b, round, purpose): Philox4x32-10 (Salmon et al., SC'11) with key
+ *     (seed low, seed high 32 bits) and counter (j, b, round low 32,
+ *     purpose | round high 32 << 8); u = ((word0 >> 8) | 1) * 2^-24.
+ * Inputs: target_logits [B, gamma+1, row_stride]; draft_logits [B, gamma,
+ *   row_stride], draft_maxprob and draft_argmax [B, gamma] as written by
+ *   sdd_confidence (all three may be NULL when greedy != 0); draft_tokens [B, gamma].
+ * Outputs, written only at the listed rows b: L [B] accepted length;
+ *   tokens [B, gamma+1] = x_1..x_L, the drawn token, then -1; n_commit [B] = L+1.
+ */
+SDD_API sdd_status_t sdd_verify_strict(const void *target_logits, const void *draft_logits,
+                               sdd_dtype_t dtype, int B, int gamma, int V, int64_t row_stride,
+                               const int32_t *draft_tokens, const float *draft_maxprob,
+                               const int32_t *draft_argmax, int greedy, uint64_t seed,
+                               uint64_t round, const int32_t *rows, int n_rows, int32_t *L,
+                               int32_t *tokens, int32_t *n_commit, void *workspace,
+                               size_t workspace_bytes, int32_t *status, sdd_stream_t stream);
+
+/*
+ * sdd_verify_lenient -- lenience acceptance (App. A.6 Eq. 9) for n_ell values in
+ * one read of the target rows: accept x_j iff z_j(x_j) - max_v z_j(v) >= log ell,
+ * except that ell = 1 uses the strict argmax comparison.  The longest accepted
+ * prefix is committed, then the target argmax of the first rejected row (of
+ * row gamma+1 when all are accepted).  ell: HOST array [n_ell] in the paper's
+ * convention 0 < ell <= 1.  Outputs [n_ell, B], tokens [n_ell, B, gamma+1],
+ * written only at the listed rows.
+ */
+SDD_API sdd_status_t sdd_verify_lenient(const void *target_logits, sdd_dtype_t dtype, int B, int gamma,
+                                int V, int64_t row_stride, const int32_t *draft_tokens,
+                                const double *ell, int n_ell, const int32_t *rows, int n_rows,
+                                int32_t *L, int32_t *tokens, int32_t *n_commit, void *workspace,
+                                size_t workspace_bytes, int32_t *status, sdd_stream_t stream);
+
+/*
+ * sdd_verify_topk -- top-k acceptance (App. A.6) for n_k values in one read of
+ * the target rows: accept x_j iff it is among the k largest target logits of row
+ * j, ranking ties by lower token index (so k = 1 is strict greedy).  Prefix and
+ * correction/bonus as for lenience.  k: HOST array [n_k], 1 <= k <= 1024.
+ */
+SDD_API sdd_status_t sdd_verify_topk(const void *target_logits, sdd_dtype_t dtype, int B, int gamma, int V,
+                             int64_t row_stride, const int32_t *draft_tokens, const int32_t *k,
+                             int n_k, const int32_t *rows, int n_rows, int32_t *L, int32_t *tokens,
+                             int32_t *n_commit, void *workspace, size_t workspace_bytes,
+                             int32_t *status, sdd_stream_t stream);
+
+/*
+ * sdd_agreement -- accumulate the agreement counters of Sec. 3.2 for n_tau
+ * schedules against the strict (shadow) accepted lengths L_strict [B]:
+ * for each t, over the rows b with K[t, b] > 0 (the set A of Eq. 1-2),
+ *   acc[t, 0] += min(K, L);  acc[t, 1] += K;  acc[t, 2] += (K <= L);  acc[t, 3] += 1.
+ * StrictToken = acc[t,0] / acc[t,1] (Eq. 1); FullPrefix = acc[t,2] / acc[t,3] (Eq. 2).
+ * acc: device int64 [n_tau, 4], added to (never cleared here).
+ */
+SDD_API sdd_status_t sdd_agreement(const int32_t *K, const int32_t *L_strict, int B, int n_tau,
+                           int64_t *acc, sdd_stream_t stream);
+
+/*
+ * sdd_commit -- the tokens a round commits (Sec. 4.1): a skipped block (K[b] > 0)
+ * commits x_1..x_K without a verifier call; any other block commits the verified
+ * tokens.  K [B] (one schedule), draft_tokens [B, gamma], verified_tokens
+ * [B, gamma+1] and verified_n [B] from a verify call.  Writes out_tokens
+ * [B, gamma+1] (-1 padded) and out_n [B].
+ */
+SDD_API sdd_status_t sdd_commit(const int32_t *K, const int32_t *draft_tokens, const int32_t *verified_tokens,
+                        const int32_t *verified_n, int B, int gamma, int32_t *out_tokens,
+                        int32_t *out_n, sdd_stream_t stream);
+
+/*
+ * sdd_uniforms -- the uniforms U(seed, j, b, round, purpose) that the sampling
+ * rule of sdd_verify_strict draws (Philox4x32-10 map stated there), for n
+ * counters given as device arrays j, b, purpose [n] (uint32) and round [n]
+ * (uint64).  Writes u [n] (fp32, exact).  Lets a caller reproduce or audit
+ * the draws of a round.
+ */
+SDD_API sdd_status_t sdd_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, const uint64_t *round,
+                                  const uint32_t *purpose, int64_t n, float *u, sdd_stream_t stream);
+
+/*
+ * sdd_block -- one round of the whole path over B blocks, fused so that every
+ * drafter and target logit is read once: confidence (sdd_confidence), the skip
+ * schedule for n_tau pairs (sdd_schedule_prefix), strict verification of every
+ * block as the shadow verifier of Sec. 3.2 (sdd_verify_strict, sampling or
+ * greedy), lenience for n_ell values and top-k for n_k values on the same target
+ * read, agreement counters for every pair, and the tokens committed under pair
+ * 0.  Array meanings and layouts are those of the single-purpose calls; NULL
+ * output pointers are skipped.  sdd_block runs sdd_block_scan then
+ * sdd_block_decide on the same stream; the two halves are exported so that a
+ * caller can time the streaming pass on its own.
+ */
+typedef struct sdd_block_args {
+    /* inputs */
+    const void *draft_logits;      /* [B, gamma, row_stride]   */
+    const void *target_logits;     /* [B, gamma+1, row_stride] */
+    const int32_t *draft_tokens;   /* [B, gamma] */
+    int32_t dtype;                 /* sdd_dtype_t */
+    int32_t B, gamma, V;
+    int64_t row_stride;
+    /* schedule (Sec. 4.1) */
+    int32_t signal;                /* sdd_signal_t */
+    int32_t n_tau;                 /* 1..SDD_MAX_GRID */
+    const double *eta_b;           /* HOST [n_tau] */
+    const double *eta_c;           /* HOST [n_tau] */
+    int32_t K_min, S_max;
+    const uint8_t *guard;          /* [B, gamma] or NULL */
+    const uint8_t *force_strict;   /* [B] or NULL */
+    const int32_t *D_in;           /* [B] or NULL */
+    /* strict verification */
+    int32_t greedy;
+    int32_t reserved0;
+    uint64_t seed, round;
+    /* lenience / top-k grids */
+    int32_t n_ell, n_k;            /* 0..SDD_MAX_GRID each */
+    const double *ell;             /* HOST [n_ell], 0 < ell <= 1 */
+    const int32_t *topk;           /* HOST [n_k] */
+    /* outputs: confidence [B, gamma] */
+    float *q, *logq, *maxprob, *lse, *entropy;
+    int32_t *argmax;
+    /* outputs: schedule [n_tau, B] */
+    int32_t *K_hat, *K, *D_out;
+    /* outputs: strict [B], [B, gamma+1], [B] */
+    int32_t *L_strict, *tokens_strict, *n_strict;
+    /* outputs: lenience [n_ell, B], [n_ell, B, gamma+1], [n_ell, B] */
+    int32_t *L_lenient, *tokens_lenient, *n_lenient;
+    /* outputs: top-k [n_k, B], [n_k, B, gamma+1], [n_k, B] */
+    int32_t *L_topk, *tokens_topk, *n_topk;
+    /* outputs: commit under pair 0: [B, gamma+1], [B] */
+    int32_t *commit_tokens, *commit_n;
+    /* agreement counters [n_tau, 4] (added to), or NULL */
+    int64_t *agreement;
+    /* scratch and status */
+    void *workspace;
+    size_t workspace_bytes;
+    int32_t *status;
+} sdd_block_args;
+
+SDD_API sdd_status_t sdd_block(const sdd_block_args *args, sdd_stream_t stream);
+SDD_API sdd_status_t sdd_block_scan(const sdd_block_args *args, sdd_stream_t stream);
+SDD_API sdd_status_t sdd_block_decide(const sdd_block_args *args, sdd_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SDD_H */

@@ -1,0 +1,12 @@
+"""GB300 (sm_103a) logits-side hot path of verifier-skipping speculative
+diffusion decoding (arXiv 2608.14787).
+
+The compute runs in libsdd.so (hand-written CUDA behind the C ABI in
+include/sdd.h); this package holds its build step, a ctypes binding with the
+same entry-point names, and the seeded synthetic-input generators.
+"""
+from .binding import (  # noqa: F401
+    BlockRound, Confidence, SddError, Workspace, agreement, commit, confidence, load, new_status,
+    schedule_prefix, uniforms, verify_lenient, verify_strict, verify_topk, workspace_bytes,
+    SIG_RAW, SIG_MARGINAL, SIG_CONDITIONAL, DEV_NONFINITE, DEV_BAD_TOKEN, DEV_TIMEOUT,
+)

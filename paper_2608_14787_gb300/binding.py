@@ -1,0 +1,379 @@
+"""ctypes binding of libsdd.so (include/sdd.h).
+
+Argument marshalling only: every step of the path runs in the library's CUDA
+kernels.  PyTorch provides device memory (output tensors, the workspace) and
+the current stream.  If the library is missing or fails to load, every entry
+point raises; there is no fallback implementation.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_build", "libsdd.so")
+
+SDD_OK = 0
+SDD_F32 = 0
+SDD_BF16 = 1
+SIG_RAW, SIG_MARGINAL, SIG_CONDITIONAL = 0, 1, 2
+DEV_NONFINITE, DEV_BAD_TOKEN, DEV_TIMEOUT = 1, 2, 4
+MAX_GAMMA = 128
+MAX_GRID = 32
+
+_lib = None
+
+c_i32p = ctypes.POINTER(ctypes.c_int32)
+c_f32p = ctypes.POINTER(ctypes.c_float)
+c_f64p = ctypes.POINTER(ctypes.c_double)
+c_u8p = ctypes.POINTER(ctypes.c_uint8)
+c_i64p = ctypes.POINTER(ctypes.c_int64)
+VP = ctypes.c_void_p
+
+
+class BlockArgs(ctypes.Structure):
+    """Mirror of sdd_block_args (field order and types as in include/sdd.h)."""
+    _fields_ = [
+        ("draft_logits", VP), ("target_logits", VP), ("draft_tokens", VP),
+        ("dtype", ctypes.c_int32), ("B", ctypes.c_int32), ("gamma", ctypes.c_int32), ("V", ctypes.c_int32),
+        ("row_stride", ctypes.c_int64),
+        ("signal", ctypes.c_int32), ("n_tau", ctypes.c_int32), ("eta_b", c_f64p), ("eta_c", c_f64p),
+        ("K_min", ctypes.c_int32), ("S_max", ctypes.c_int32),
+        ("guard", VP), ("force_strict", VP), ("D_in", VP),
+        ("greedy", ctypes.c_int32), ("reserved0", ctypes.c_int32),
+        ("seed", ctypes.c_uint64), ("round", ctypes.c_uint64),
+        ("n_ell", ctypes.c_int32), ("n_k", ctypes.c_int32), ("ell", c_f64p), ("topk", c_i32p),
+        ("q", VP), ("logq", VP), ("maxprob", VP), ("lse", VP), ("entropy", VP), ("argmax", VP),
+        ("K_hat", VP), ("K", VP), ("D_out", VP),
+        ("L_strict", VP), ("tokens_strict", VP), ("n_strict", VP),
+        ("L_lenient", VP), ("tokens_lenient", VP), ("n_lenient", VP),
+        ("L_topk", VP), ("tokens_topk", VP), ("n_topk", VP),
+        ("commit_tokens", VP), ("commit_n", VP),
+        ("agreement", VP),
+        ("workspace", VP), ("workspace_bytes", ctypes.c_size_t),
+        ("status", VP),
+    ]
+
+
+def load(path: str | None = None):
+    """Load libsdd.so (built in-tree by paper_2608_14787_gb300.build)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = path or LIB_PATH
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with paper_2608_14787_gb300.build.build()")
+    L = ctypes.CDLL(path)
+    I = ctypes.c_int
+    i64 = ctypes.c_int64
+    u64 = ctypes.c_uint64
+    L.sdd_version.restype = I
+    L.sdd_last_error.restype = ctypes.c_char_p
+    L.sdd_workspace_size.argtypes = [I, I, I, ctypes.POINTER(ctypes.c_size_t)]
+    L.sdd_confidence.argtypes = [VP, I, I, I, I, i64, VP, VP, VP, VP, VP, VP, VP, VP, ctypes.c_size_t, VP, VP]
+    L.sdd_schedule_prefix.argtypes = [VP, VP, I, I, I, c_f64p, c_f64p, I, I, I, VP, VP, VP, VP, VP, VP, VP, VP]
+    L.sdd_verify_strict.argtypes = [VP, VP, I, I, I, I, i64, VP, VP, VP, I, u64, u64, VP, I, VP, VP, VP, VP,
+                                    ctypes.c_size_t, VP, VP]
+    L.sdd_verify_lenient.argtypes = [VP, I, I, I, I, i64, VP, c_f64p, I, VP, I, VP, VP, VP, VP, ctypes.c_size_t,
+                                     VP, VP]
+    L.sdd_verify_topk.argtypes = [VP, I, I, I, I, i64, VP, c_i32p, I, VP, I, VP, VP, VP, VP, ctypes.c_size_t,
+                                  VP, VP]
+    L.sdd_agreement.argtypes = [VP, VP, I, I, VP, VP]
+    L.sdd_commit.argtypes = [VP, VP, VP, VP, I, I, VP, VP, VP]
+    L.sdd_uniforms.argtypes = [u64, VP, VP, VP, VP, i64, VP, VP]
+    for fn in ("sdd_block", "sdd_block_scan", "sdd_block_decide"):
+        getattr(L, fn).argtypes = [ctypes.POINTER(BlockArgs), VP]
+    for fn in ("sdd_workspace_size", "sdd_confidence", "sdd_schedule_prefix", "sdd_verify_strict",
+               "sdd_verify_lenient", "sdd_verify_topk", "sdd_agreement", "sdd_commit", "sdd_uniforms", "sdd_block",
+               "sdd_block_scan", "sdd_block_decide"):
+        getattr(L, fn).restype = I
+    _lib = L
+    return L
+
+
+class SddError(RuntimeError):
+    pass
+
+
+def _check(rc: int, what: str):
+    if rc != SDD_OK:
+        msg = load().sdd_last_error().decode(errors="replace")
+        raise SddError(f"{what} failed (status {rc}): {msg}")
+
+
+def _p(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return SDD_BF16
+    if t.dtype == torch.float32:
+        return SDD_F32
+    raise TypeError(f"logits must be bfloat16 or float32, got {t.dtype}")
+
+
+def _logits_layout(z: torch.Tensor, npos_name: str):
+    """(V, row_stride) of a [B, P, V] tensor whose last dim is contiguous and
+    whose rows are evenly spaced."""
+    if z.dim() != 3:
+        raise ValueError(f"{npos_name} must be [B, P, V]")
+    B, P, V = z.shape
+    if z.stride(2) != 1 and V > 1:
+        raise ValueError(f"{npos_name} must have unit stride over V")
+    stride = z.stride(1) if P > 1 or B == 1 else z.stride(0) // max(P, 1)
+    if B > 1 and z.stride(0) != stride * P:
+        raise ValueError(f"{npos_name} must have evenly spaced rows (stride(0) == stride(1) * P)")
+    return V, stride
+
+
+def workspace_bytes(B: int, gamma: int, V: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(load().sdd_workspace_size(B, gamma, V, ctypes.byref(n)), "sdd_workspace_size")
+    return int(n.value)
+
+
+class Workspace:
+    """Zero-filled, 256-byte aligned device scratch for blocks up to (B, gamma)."""
+
+    def __init__(self, B: int, gamma: int, V: int, device=None):
+        self.nbytes = workspace_bytes(B, gamma, V)
+        buf = torch.zeros(self.nbytes + 256, dtype=torch.uint8, device=device or "cuda")
+        off = (-buf.data_ptr()) % 256
+        self._buf = buf
+        self.tensor = buf[off:off + self.nbytes]
+
+    @property
+    def ptr(self):
+        return ctypes.c_void_p(self.tensor.data_ptr())
+
+
+def new_status(device=None) -> torch.Tensor:
+    return torch.zeros(1, dtype=torch.int32, device=device or "cuda")
+
+
+@dataclass
+class Confidence:
+    q: torch.Tensor
+    logq: torch.Tensor
+    maxprob: torch.Tensor
+    lse: torch.Tensor
+    entropy: torch.Tensor
+    argmax: torch.Tensor
+
+
+def confidence(z_d: torch.Tensor, x: torch.Tensor, ws: Workspace | None = None, status=None,
+               stream=None) -> Confidence:
+    """sdd_confidence over drafter logits z_d [B, gamma, V] and drafted tokens x [B, gamma]."""
+    B, gamma = x.shape
+    V, stride = _logits_layout(z_d, "z_d")
+    dev = z_d.device
+    ws = ws or Workspace(B, gamma, V, dev)
+    status = new_status(dev) if status is None else status
+    out = Confidence(*(torch.empty(B, gamma, dtype=torch.float32, device=dev) for _ in range(5)),
+                     torch.empty(B, gamma, dtype=torch.int32, device=dev))
+    rc = load().sdd_confidence(_p(z_d), _dtype_code(z_d), B, gamma, V, stride, _p(x), _p(out.q), _p(out.logq),
+                               _p(out.maxprob), _p(out.lse), _p(out.entropy), _p(out.argmax), ws.ptr, ws.nbytes,
+                               _p(status), _stream(stream))
+    _check(rc, "sdd_confidence")
+    return out
+
+
+def _f64_array(vals):
+    arr = (ctypes.c_double * len(vals))(*[float(v) for v in vals])
+    return arr
+
+
+def schedule_prefix(q, eta_b, eta_c, *, signal=SIG_RAW, logq=None, K_min=6, S_max=64, guard=None,
+                    force_strict=None, D_in=None, status=None, stream=None):
+    """sdd_schedule_prefix; returns (K_hat, K, D_out), each [n_tau, B]."""
+    B, gamma = q.shape
+    n_tau = len(eta_b)
+    dev = q.device
+    Kh = torch.empty(n_tau, B, dtype=torch.int32, device=dev)
+    K = torch.empty(n_tau, B, dtype=torch.int32, device=dev)
+    Do = torch.empty(n_tau, B, dtype=torch.int32, device=dev)
+    eb, ec = _f64_array(eta_b), _f64_array(eta_c)
+    rc = load().sdd_schedule_prefix(_p(q), _p(logq), B, gamma, signal, eb, ec, n_tau, K_min, S_max, _p(guard),
+                                    _p(force_strict), _p(D_in), _p(Kh), _p(K), _p(Do), _p(status), _stream(stream))
+    _check(rc, "sdd_schedule_prefix")
+    return Kh, K, Do
+
+
+def verify_strict(z_t, x, *, z_d=None, draft=None, greedy=False, seed=0, round_=0, rows=None,
+                  ws: Workspace | None = None, status=None, stream=None, out=None):
+    """sdd_verify_strict; returns (L [B], tokens [B, gamma+1], n_commit [B])."""
+    B, gamma = x.shape
+    V, stride = _logits_layout(z_t, "z_t")
+    dev = z_t.device
+    ws = ws or Workspace(B, gamma, V, dev)
+    status = new_status(dev) if status is None else status
+    if out is None:
+        out = (torch.full((B,), -2, dtype=torch.int32, device=dev),
+               torch.full((B, gamma + 1), -2, dtype=torch.int32, device=dev),
+               torch.full((B,), -2, dtype=torch.int32, device=dev))
+    L, tok, n = out
+    n_rows = B if rows is None else rows.numel()
+    mp = None if draft is None else draft.maxprob
+    am = None if draft is None else draft.argmax
+    rc = load().sdd_verify_strict(_p(z_t), _p(z_d), _dtype_code(z_t), B, gamma, V, stride, _p(x), _p(mp), _p(am),
+                                  1 if greedy else 0, seed, round_, _p(rows), n_rows, _p(L), _p(tok), _p(n),
+                                  ws.ptr, ws.nbytes, _p(status), _stream(stream))
+    _check(rc, "sdd_verify_strict")
+    return L, tok, n
+
+
+def verify_lenient(z_t, x, ells, *, rows=None, ws=None, status=None, stream=None):
+    """sdd_verify_lenient with ell in the paper's convention (0 < ell <= 1)."""
+    B, gamma = x.shape
+    V, stride = _logits_layout(z_t, "z_t")
+    dev = z_t.device
+    ws = ws or Workspace(B, gamma, V, dev)
+    status = new_status(dev) if status is None else status
+    n = len(ells)
+    L = torch.full((n, B), -2, dtype=torch.int32, device=dev)
+    tok = torch.full((n, B, gamma + 1), -2, dtype=torch.int32, device=dev)
+    nc = torch.full((n, B), -2, dtype=torch.int32, device=dev)
+    n_rows = B if rows is None else rows.numel()
+    rc = load().sdd_verify_lenient(_p(z_t), _dtype_code(z_t), B, gamma, V, stride, _p(x), _f64_array(ells), n,
+                                   _p(rows), n_rows, _p(L), _p(tok), _p(nc), ws.ptr, ws.nbytes, _p(status),
+                                   _stream(stream))
+    _check(rc, "sdd_verify_lenient")
+    return L, tok, nc
+
+
+def verify_topk(z_t, x, ks, *, rows=None, ws=None, status=None, stream=None):
+    B, gamma = x.shape
+    V, stride = _logits_layout(z_t, "z_t")
+    dev = z_t.device
+    ws = ws or Workspace(B, gamma, V, dev)
+    status = new_status(dev) if status is None else status
+    n = len(ks)
+    L = torch.full((n, B), -2, dtype=torch.int32, device=dev)
+    tok = torch.full((n, B, gamma + 1), -2, dtype=torch.int32, device=dev)
+    nc = torch.full((n, B), -2, dtype=torch.int32, device=dev)
+    n_rows = B if rows is None else rows.numel()
+    karr = (ctypes.c_int32 * n)(*[int(k) for k in ks])
+    rc = load().sdd_verify_topk(_p(z_t), _dtype_code(z_t), B, gamma, V, stride, _p(x), karr, n, _p(rows), n_rows,
+                                _p(L), _p(tok), _p(nc), ws.ptr, ws.nbytes, _p(status), _stream(stream))
+    _check(rc, "sdd_verify_topk")
+    return L, tok, nc
+
+
+def agreement(K, L_strict, acc=None, stream=None):
+    n_tau, B = K.shape
+    acc = torch.zeros(n_tau, 4, dtype=torch.int64, device=K.device) if acc is None else acc
+    _check(load().sdd_agreement(_p(K), _p(L_strict), B, n_tau, _p(acc), _stream(stream)), "sdd_agreement")
+    return acc
+
+
+def commit(K, x, verified_tokens, verified_n, stream=None):
+    B, gamma = x.shape
+    out_t = torch.empty(B, gamma + 1, dtype=torch.int32, device=x.device)
+    out_n = torch.empty(B, dtype=torch.int32, device=x.device)
+    _check(load().sdd_commit(_p(K), _p(x), _p(verified_tokens), _p(verified_n), B, gamma, _p(out_t), _p(out_n),
+                             _stream(stream)), "sdd_commit")
+    return out_t, out_n
+
+
+def uniforms(seed, j, b, round_, purpose, stream=None):
+    """sdd_uniforms: Philox uniforms for device arrays j, b, purpose (int32/uint32) and round (int64)."""
+    n = j.numel()
+    u = torch.empty(n, dtype=torch.float32, device=j.device)
+    _check(load().sdd_uniforms(seed, _p(j), _p(b), _p(round_), _p(purpose), n, _p(u), _stream(stream)),
+           "sdd_uniforms")
+    return u
+
+
+class BlockRound:
+    """Pre-allocated arguments and outputs of sdd_block for one (B, gamma, V) shape.
+
+    Attributes after a call: q, logq, maxprob, lse, entropy, argmax [B, gamma];
+    K_hat, K, D_out [n_tau, B]; L_strict [B], tokens_strict [B, gamma+1],
+    n_strict [B]; L_lenient/tokens_lenient/n_lenient [n_ell, ...];
+    L_topk/tokens_topk/n_topk [n_k, ...]; commit_tokens, commit_n;
+    agreement [n_tau, 4] (accumulated across calls).
+    """
+
+    def __init__(self, B, gamma, V, *, dtype=torch.bfloat16, taus=(0.9,), eta_b=None, eta_c=None,
+                 signal=SIG_RAW, K_min=6, S_max=64, ells=(), ks=(), greedy=False, device="cuda"):
+        dev = torch.device(device)
+        self.B, self.gamma, self.V = B, gamma, V
+        self.dtype = dtype
+        eta_b = list(taus) if eta_b is None else list(eta_b)
+        eta_c = list(taus) if eta_c is None else list(eta_c)
+        self.n_tau = len(eta_b)
+        self.ws = Workspace(B, gamma, V, dev)
+        self.status = new_status(dev)
+        f32 = lambda *s: torch.zeros(*s, dtype=torch.float32, device=dev)   # noqa: E731
+        i32 = lambda *s: torch.zeros(*s, dtype=torch.int32, device=dev)     # noqa: E731
+        self.q, self.logq, self.maxprob, self.lse, self.entropy = (f32(B, gamma) for _ in range(5))
+        self.argmax = i32(B, gamma)
+        self.K_hat, self.K, self.D_out = (i32(self.n_tau, B) for _ in range(3))
+        self.D_in = i32(B)
+        self.L_strict, self.tokens_strict, self.n_strict = i32(B), i32(B, gamma + 1), i32(B)
+        ne, nk = len(ells), len(ks)
+        self.L_lenient, self.tokens_lenient, self.n_lenient = i32(max(ne, 1), B), i32(max(ne, 1), B, gamma + 1), \
+            i32(max(ne, 1), B)
+        self.L_topk, self.tokens_topk, self.n_topk = i32(max(nk, 1), B), i32(max(nk, 1), B, gamma + 1), \
+            i32(max(nk, 1), B)
+        self.commit_tokens, self.commit_n = i32(B, gamma + 1), i32(B)
+        self.agreement = torch.zeros(self.n_tau, 4, dtype=torch.int64, device=dev)
+        self._eta_b = _f64_array(eta_b)
+        self._eta_c = _f64_array(eta_c)
+        self._ell = _f64_array(list(ells) or [1.0])
+        self._k = (ctypes.c_int32 * max(nk, 1))(*([int(k) for k in ks] or [1]))
+        a = BlockArgs()
+        a.dtype = SDD_BF16 if dtype == torch.bfloat16 else SDD_F32
+        a.B, a.gamma, a.V = B, gamma, V
+        a.signal, a.n_tau = signal, self.n_tau
+        a.eta_b = ctypes.cast(self._eta_b, c_f64p)
+        a.eta_c = ctypes.cast(self._eta_c, c_f64p)
+        a.K_min, a.S_max = K_min, S_max
+        a.greedy = 1 if greedy else 0
+        a.n_ell, a.n_k = ne, nk
+        a.ell = ctypes.cast(self._ell, c_f64p)
+        a.topk = ctypes.cast(self._k, c_i32p)
+        for name in ("q", "logq", "maxprob", "lse", "entropy", "argmax", "K_hat", "K", "D_out", "L_strict",
+                     "tokens_strict", "n_strict", "commit_tokens", "commit_n", "agreement"):
+            setattr(a, name, getattr(self, name).data_ptr())
+        if ne:
+            a.L_lenient, a.tokens_lenient, a.n_lenient = (t.data_ptr() for t in
+                                                          (self.L_lenient, self.tokens_lenient, self.n_lenient))
+        if nk:
+            a.L_topk, a.tokens_topk, a.n_topk = (t.data_ptr() for t in (self.L_topk, self.tokens_topk, self.n_topk))
+        a.D_in = self.D_in.data_ptr()
+        a.workspace = self.ws.tensor.data_ptr()
+        a.workspace_bytes = self.ws.nbytes
+        a.status = self.status.data_ptr()
+        self.args = a
+
+    def set_inputs(self, z_d, z_t, x, *, seed=0, round_=0, guard=None, force_strict=None):
+        V, stride = _logits_layout(z_d, "z_d")
+        Vt, stride_t = _logits_layout(z_t, "z_t")
+        if (V, stride) != (Vt, stride_t) or V != self.V:
+            raise ValueError("z_d and z_t must share V and row stride")
+        a = self.args
+        a.draft_logits, a.target_logits, a.draft_tokens = z_d.data_ptr(), z_t.data_ptr(), x.data_ptr()
+        a.row_stride = stride
+        a.seed, a.round = seed, round_
+        a.guard = None if guard is None else guard.data_ptr()
+        a.force_strict = None if force_strict is None else force_strict.data_ptr()
+        self._keep = (z_d, z_t, x, guard, force_strict)
+
+    def run(self, stream=None):
+        _check(load().sdd_block(ctypes.byref(self.args), _stream(stream)), "sdd_block")
+
+    def scan(self, stream=None):
+        _check(load().sdd_block_scan(ctypes.byref(self.args), _stream(stream)), "sdd_block_scan")
+
+    def decide(self, stream=None):
+        _check(load().sdd_block_decide(ctypes.byref(self.args), _stream(stream)), "sdd_block_decide")

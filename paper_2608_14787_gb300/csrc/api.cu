@@ -1,0 +1,611 @@
+// api.cu -- the C ABI declared in include/sdd.h: argument checks, workspace
+// layout and kernel launches.  Every check that can fail runs before anything
+// is enqueued; nothing here allocates device memory.
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+
+#include "internal.h"
+
+namespace sdd {
+namespace {
+
+thread_local std::string g_err;
+
+sdd_status_t fail(sdd_status_t s, const char *fmt, ...) __attribute__((format(printf, 2, 3)));
+sdd_status_t fail(sdd_status_t s, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_err = buf;
+    return s;
+}
+
+sdd_status_t cuda_fail(cudaError_t e, const char *what) {
+    return fail(SDD_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// Per-device launch facts, filled on first use (benign race: same values).
+constexpr int kMaxDevices = 64;
+struct DevInfo {
+    int sms;
+    int ctas_per_sm;
+};
+DevInfo g_dev[kMaxDevices];
+std::atomic<int> g_dev_ready[kMaxDevices];
+
+sdd_status_t device_info(DevInfo &out) {
+    int d = 0;
+    cudaError_t e = cudaGetDevice(&d);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (d < 0 || d >= kMaxDevices) return fail(SDD_ERR_UNSUPPORTED, "device ordinal %d out of range", d);
+    if (!g_dev_ready[d].load(std::memory_order_acquire)) {
+        DevInfo di{};
+        e = cudaDeviceGetAttribute(&di.sms, cudaDevAttrMultiProcessorCount, d);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+        e = scan_prepare_device();
+        if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
+        di.ctas_per_sm = scan_max_ctas_per_sm();
+        if (di.ctas_per_sm < 1) return fail(SDD_ERR_UNSUPPORTED, "streaming kernel does not fit on this device");
+        g_dev[d] = di;
+        g_dev_ready[d].store(1, std::memory_order_release);
+    }
+    out = g_dev[d];
+    return SDD_OK;
+}
+
+inline size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+// Workspace layout for blocks of shape (B, gamma) on a device with W_max warps.
+struct Layout {
+    size_t partials, counters, drec, trec, res_total, res_last, res_count, k0, total;
+};
+
+Layout layout(int64_t B, int64_t gamma, int64_t W_max) {
+    Layout L{};
+    const int64_t rows = B * (2 * gamma + 1);
+    size_t o = 0;
+    L.partials = o;
+    o = align256(o + static_cast<size_t>(rows + W_max) * sizeof(Partial));
+    L.counters = o;
+    o = align256(o + static_cast<size_t>(rows) * sizeof(uint32_t));
+    L.drec = o;
+    o = align256(o + static_cast<size_t>(B * gamma) * sizeof(RowRec));
+    L.trec = o;
+    o = align256(o + static_cast<size_t>(B * (gamma + 1)) * sizeof(RowRec));
+    L.res_total = o;
+    o = align256(o + static_cast<size_t>(B * kResidMaxSeg) * sizeof(double));
+    L.res_last = o;
+    o = align256(o + static_cast<size_t>(B * kResidMaxSeg) * sizeof(int32_t));
+    L.res_count = o;
+    o = align256(o + static_cast<size_t>(B) * sizeof(uint32_t));
+    L.k0 = o;
+    o = align256(o + static_cast<size_t>(B) * sizeof(int32_t));
+    L.total = o;
+    return L;
+}
+
+int esize(int dtype) { return dtype == SDD_BF16 ? 2 : 4; }
+
+sdd_status_t check_shape(sdd_dtype_t dtype, int B, int gamma, int V, int64_t row_stride) {
+    if (dtype != SDD_F32 && dtype != SDD_BF16) return fail(SDD_ERR_INVALID_ARGUMENT, "dtype %d unknown", dtype);
+    if (B < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "B = %d < 0", B);
+    if (gamma < 1 || gamma > SDD_MAX_GAMMA)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "gamma = %d outside [1, %d]", gamma, SDD_MAX_GAMMA);
+    if (V < 1) return fail(SDD_ERR_INVALID_ARGUMENT, "V = %d < 1", V);
+    if (row_stride < V) return fail(SDD_ERR_INVALID_ARGUMENT, "row_stride %lld < V %d", (long long)row_stride, V);
+    if ((row_stride * esize(dtype)) % 16 != 0)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "row_stride * element size must be a multiple of 16 bytes");
+    if (row_stride * esize(dtype) > (int64_t(1) << 31))
+        return fail(SDD_ERR_INVALID_ARGUMENT, "rows longer than 2 GiB are not supported");
+    return SDD_OK;
+}
+
+sdd_status_t check_ptr16(const void *p, const char *name) {
+    if (!p) return fail(SDD_ERR_INVALID_ARGUMENT, "%s is NULL", name);
+    if (reinterpret_cast<uintptr_t>(p) % 16 != 0) return fail(SDD_ERR_INVALID_ARGUMENT, "%s is not 16-byte aligned", name);
+    return SDD_OK;
+}
+
+struct Work {
+    char *base;
+    Layout L;
+    int W_max;
+    int sms;
+};
+
+sdd_status_t get_work(void *workspace, size_t bytes, int B, int gamma, Work &w) {
+    DevInfo di;
+    sdd_status_t s = device_info(di);
+    if (s != SDD_OK) return s;
+    w.W_max = di.sms * di.ctas_per_sm * kWarpsPerCta;
+    w.sms = di.sms;
+    w.L = layout(B, gamma, w.W_max);
+    if (!workspace) return fail(SDD_ERR_WORKSPACE, "workspace is NULL");
+    if (reinterpret_cast<uintptr_t>(workspace) % 256 != 0)
+        return fail(SDD_ERR_WORKSPACE, "workspace is not 256-byte aligned");
+    if (bytes < w.L.total)
+        return fail(SDD_ERR_WORKSPACE, "workspace has %zu bytes, %zu needed", bytes, w.L.total);
+    w.base = static_cast<char *>(workspace);
+    return SDD_OK;
+}
+
+void init_scan(ScanParams &p, const Work &w, sdd_dtype_t dtype, int B, int gamma, int V, const int32_t *tokens,
+               int32_t *status) {
+    std::memset(&p, 0, sizeof p);
+    p.dtype = dtype;
+    p.V = V;
+    p.RV = static_cast<int32_t>((static_cast<int64_t>(V) * esize(dtype) + 15) / 16);
+    p.gamma = gamma;
+    p.kcap = 1;
+    p.B = B;
+    p.tokens = tokens;
+    p.partials = reinterpret_cast<Partial *>(w.base + w.L.partials);
+    p.counters = reinterpret_cast<uint32_t *>(w.base + w.L.counters);
+    p.status = status;
+}
+
+// Fill in the totals of a ScanParams whose groups are set, and launch.
+sdd_status_t run_scan(ScanParams &p, const Work &w, cudaStream_t stream) {
+    p.rows0 = static_cast<int64_t>(p.grp[0].nb) * p.grp[0].npos;
+    p.rows = p.rows0 + (p.n_groups > 1 ? static_cast<int64_t>(p.grp[1].nb) * p.grp[1].npos : 0);
+    p.T = p.rows * p.RV;
+    if (p.T == 0) return SDD_OK;
+    const int64_t W = std::min<int64_t>(w.W_max, p.T);
+    p.W = static_cast<int32_t>(W);
+    const int grid = static_cast<int>((W + kWarpsPerCta - 1) / kWarpsPerCta);
+    cudaError_t e = launch_scan(p, grid, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "scan launch");
+    return SDD_OK;
+}
+
+void init_decide(DecideParams &d, const Work &w, sdd_dtype_t dtype, int B, int gamma, int V, int64_t row_stride,
+                 const int32_t *tokens, int32_t *status) {
+    std::memset(&d, 0, sizeof d);
+    d.B = B;
+    d.gamma = gamma;
+    d.V = V;
+    d.RV = static_cast<int32_t>((static_cast<int64_t>(V) * esize(dtype) + 15) / 16);
+    d.dtype = dtype;
+    d.stride_bytes = row_stride * esize(dtype);
+    d.tokens = tokens;
+    d.trec = reinterpret_cast<const RowRec *>(w.base + w.L.trec);
+    d.res_total = reinterpret_cast<double *>(w.base + w.L.res_total);
+    d.res_last = reinterpret_cast<int32_t *>(w.base + w.L.res_last);
+    d.res_count = reinterpret_cast<uint32_t *>(w.base + w.L.res_count);
+    d.k0 = reinterpret_cast<int32_t *>(w.base + w.L.k0);
+    d.status = status;
+    d.nseg = 1;
+    d.seg_vec = d.RV;
+}
+
+// Residual segments per block: about two CTAs per SM in total, at least one
+// full 256-vector chunk per segment.
+void set_segments(DecideParams &d, int sms) {
+    const int nb = std::max(1, d.nb);
+    int nseg = (2 * sms + nb - 1) / nb;
+    nseg = std::min(nseg, kResidMaxSeg);
+    nseg = std::min(nseg, (d.RV + kResidThreads - 1) / kResidThreads);
+    nseg = std::max(nseg, 1);
+    d.seg_vec = (d.RV + nseg - 1) / nseg;
+    d.nseg = (d.RV + d.seg_vec - 1) / d.seg_vec;
+}
+
+sdd_status_t set_thresholds(int signal, const double *eta_b, const double *eta_c, int n_tau, double *eta_loc,
+                            double *log_eta_c, int32_t *tau_off) {
+    if (n_tau < 1 || n_tau > SDD_MAX_GRID)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "n_tau = %d outside [1, %d]", n_tau, SDD_MAX_GRID);
+    if (!eta_b || !eta_c) return fail(SDD_ERR_INVALID_ARGUMENT, "eta_b / eta_c are NULL");
+    if (signal != SDD_SIG_RAW && signal != SDD_SIG_MARGINAL && signal != SDD_SIG_CONDITIONAL)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "signal %d unknown", signal);
+    for (int t = 0; t < n_tau; ++t) {
+        const double eb = eta_b[t], ec = eta_c[t];
+        if (std::isnan(eb) || std::isnan(ec)) return fail(SDD_ERR_INVALID_ARGUMENT, "threshold %d is NaN", t);
+        tau_off[t] = (eb >= 1.0 || ec >= 1.0) ? 1 : 0;
+        const double em = std::max(eb, ec);
+        eta_loc[t] = (signal == SDD_SIG_MARGINAL) ? em : eb;
+        log_eta_c[t] = (ec > 0.0) ? std::log(ec) : -INFINITY;
+    }
+    return SDD_OK;
+}
+
+sdd_status_t set_ell(DecideParams &d, const double *ell, int n_ell) {
+    if (n_ell < 0 || n_ell > SDD_MAX_GRID)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "n_ell = %d outside [0, %d]", n_ell, SDD_MAX_GRID);
+    if (n_ell > 0 && !ell) return fail(SDD_ERR_INVALID_ARGUMENT, "ell is NULL");
+    d.n_ell = n_ell;
+    for (int r = 0; r < n_ell; ++r) {
+        if (!(ell[r] > 0.0 && ell[r] <= 1.0))
+            return fail(SDD_ERR_INVALID_ARGUMENT, "ell[%d] = %g outside (0, 1] (paper convention)", r, ell[r]);
+        d.ell_one[r] = (ell[r] == 1.0) ? 1 : 0;
+        d.ell_thr[r] = std::log(ell[r]);
+    }
+    return SDD_OK;
+}
+
+sdd_status_t set_topk(DecideParams &d, const int32_t *k, int n_k, int &kcap) {
+    if (n_k < 0 || n_k > SDD_MAX_GRID) return fail(SDD_ERR_INVALID_ARGUMENT, "n_k = %d outside [0, %d]", n_k, SDD_MAX_GRID);
+    if (n_k > 0 && !k) return fail(SDD_ERR_INVALID_ARGUMENT, "k is NULL");
+    d.n_k = n_k;
+    for (int r = 0; r < n_k; ++r) {
+        if (k[r] < 1 || k[r] > 1024) return fail(SDD_ERR_INVALID_ARGUMENT, "k[%d] = %d outside [1, 1024]", r, k[r]);
+        d.kval[r] = k[r];
+        kcap = std::max(kcap, static_cast<int>(k[r]));
+    }
+    return SDD_OK;
+}
+
+sdd_status_t check_rows(const int32_t *rows, int n_rows, int B) {
+    if (rows == nullptr && n_rows != B)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "rows is NULL but n_rows = %d != B = %d", n_rows, B);
+    if (n_rows < 0 || n_rows > B) return fail(SDD_ERR_INVALID_ARGUMENT, "n_rows = %d outside [0, B]", n_rows);
+    return SDD_OK;
+}
+
+#define SDD_TRY(expr)                         \
+    do {                                      \
+        sdd_status_t _s = (expr);             \
+        if (_s != SDD_OK) return _s;          \
+    } while (0)
+
+// Target-row scan (post-verify) for the listed blocks.
+sdd_status_t target_scan(const Work &w, const void *target_logits, sdd_dtype_t dtype, int B, int gamma, int V,
+                         int64_t row_stride, const int32_t *tokens, const int32_t *rows, int n_rows, int kcap,
+                         int32_t *status, cudaStream_t stream) {
+    ScanParams p;
+    init_scan(p, w, dtype, B, gamma, V, tokens, status);
+    p.n_groups = 1;
+    p.kcap = kcap;
+    ScanGroup &G = p.grp[0];
+    G.base = static_cast<const char *>(target_logits);
+    G.stride_bytes = row_stride * esize(dtype);
+    G.npos = gamma + 1;
+    G.kind = 1;
+    G.nb = n_rows;
+    G.bidx = rows;
+    G.rec = reinterpret_cast<RowRec *>(w.base + w.L.trec);
+    return run_scan(p, w, stream);
+}
+
+}  // namespace
+}  // namespace sdd
+
+using namespace sdd;
+
+extern "C" {
+
+int sdd_version(void) { return 100; }
+
+const char *sdd_last_error(void) { return g_err.c_str(); }
+
+sdd_status_t sdd_workspace_size(int B, int gamma, int V, size_t *bytes) {
+    if (!bytes) return fail(SDD_ERR_INVALID_ARGUMENT, "bytes is NULL");
+    SDD_TRY(check_shape(SDD_BF16, B, gamma, V, ((static_cast<int64_t>(V) + 7) / 8) * 8));
+    DevInfo di;
+    SDD_TRY(device_info(di));
+    *bytes = layout(B, gamma, static_cast<int64_t>(di.sms) * di.ctas_per_sm * kWarpsPerCta).total;
+    return SDD_OK;
+}
+
+sdd_status_t sdd_confidence(const void *draft_logits, sdd_dtype_t dtype, int B, int gamma, int V,
+                            int64_t row_stride, const int32_t *draft_tokens, float *q, float *logq,
+                            float *maxprob, float *lse, float *entropy, int32_t *argmax, void *workspace,
+                            size_t workspace_bytes, int32_t *status, sdd_stream_t stream) {
+    SDD_TRY(check_shape(dtype, B, gamma, V, row_stride));
+    if (B == 0) return SDD_OK;
+    SDD_TRY(check_ptr16(draft_logits, "draft_logits"));
+    if (!draft_tokens) return fail(SDD_ERR_INVALID_ARGUMENT, "draft_tokens is NULL");
+    if (!q) return fail(SDD_ERR_INVALID_ARGUMENT, "q is NULL");
+    Work w;
+    SDD_TRY(get_work(workspace, workspace_bytes, B, gamma, w));
+    ScanParams p;
+    init_scan(p, w, dtype, B, gamma, V, draft_tokens, status);
+    p.n_groups = 1;
+    ScanGroup &G = p.grp[0];
+    G.base = static_cast<const char *>(draft_logits);
+    G.stride_bytes = row_stride * esize(dtype);
+    G.npos = gamma;
+    G.kind = 0;
+    G.nb = B;
+    G.rec = reinterpret_cast<RowRec *>(w.base + w.L.drec);
+    G.q = q;
+    G.logq = logq;
+    G.maxprob = maxprob;
+    G.lse = lse;
+    G.entropy = entropy;
+    G.argmax = argmax;
+    return run_scan(p, w, reinterpret_cast<cudaStream_t>(stream));
+}
+
+sdd_status_t sdd_schedule_prefix(const float *q, const float *logq, int B, int gamma, sdd_signal_t signal,
+                                 const double *eta_b, const double *eta_c, int n_tau, int K_min, int S_max,
+                                 const uint8_t *guard, const uint8_t *force_strict, const int32_t *D_in,
+                                 int32_t *K_hat, int32_t *K, int32_t *D_out, int32_t *status, sdd_stream_t stream) {
+    (void)status;
+    if (B < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "B = %d < 0", B);
+    if (gamma < 1 || gamma > SDD_MAX_GAMMA)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "gamma = %d outside [1, %d]", gamma, SDD_MAX_GAMMA);
+    ScheduleParams p;
+    std::memset(&p, 0, sizeof p);
+    SDD_TRY(set_thresholds(signal, eta_b, eta_c, n_tau, p.eta_loc, p.log_eta_c, p.tau_off));
+    if (B == 0) return SDD_OK;
+    if (!q || !K_hat || !K) return fail(SDD_ERR_INVALID_ARGUMENT, "q, K_hat and K must not be NULL");
+    p.q = q;
+    p.logq = logq;
+    p.B = B;
+    p.gamma = gamma;
+    p.signal = signal;
+    p.n_tau = n_tau;
+    p.K_min = K_min;
+    p.S_max = S_max;
+    p.guard = guard;
+    p.force_strict = force_strict;
+    p.D_in = D_in;
+    p.K_hat = K_hat;
+    p.K = K;
+    p.D_out = D_out;
+    cudaError_t e = launch_schedule(p, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "schedule launch");
+    return SDD_OK;
+}
+
+sdd_status_t sdd_verify_strict(const void *target_logits, const void *draft_logits, sdd_dtype_t dtype, int B,
+                               int gamma, int V, int64_t row_stride, const int32_t *draft_tokens,
+                               const float *draft_maxprob, const int32_t *draft_argmax, int greedy, uint64_t seed,
+                               uint64_t round, const int32_t *rows, int n_rows, int32_t *L, int32_t *tokens,
+                               int32_t *n_commit, void *workspace, size_t workspace_bytes, int32_t *status,
+                               sdd_stream_t stream) {
+    SDD_TRY(check_shape(dtype, B, gamma, V, row_stride));
+    SDD_TRY(check_rows(rows, n_rows, B));
+    if (n_rows == 0) return SDD_OK;
+    SDD_TRY(check_ptr16(target_logits, "target_logits"));
+    if (!draft_tokens) return fail(SDD_ERR_INVALID_ARGUMENT, "draft_tokens is NULL");
+    if (!greedy) {
+        SDD_TRY(check_ptr16(draft_logits, "draft_logits"));
+        if (!draft_maxprob || !draft_argmax)
+            return fail(SDD_ERR_INVALID_ARGUMENT, "sampling needs draft_maxprob and draft_argmax");
+    }
+    Work w;
+    SDD_TRY(get_work(workspace, workspace_bytes, B, gamma, w));
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    SDD_TRY(target_scan(w, target_logits, dtype, B, gamma, V, row_stride, draft_tokens, rows, n_rows, 1, status, st));
+    DecideParams d;
+    init_decide(d, w, dtype, B, gamma, V, row_stride, draft_tokens, status);
+    d.nb = n_rows;
+    d.bidx = rows;
+    d.zt = static_cast<const char *>(target_logits);
+    d.zd = static_cast<const char *>(draft_logits);
+    d.d_maxprob = draft_maxprob;
+    d.d_argmax = draft_argmax;
+    d.do_strict = 1;
+    d.greedy = greedy ? 1 : 0;
+    d.seed = seed;
+    d.round = round;
+    d.L_strict = L;
+    d.tok_strict = tokens;
+    d.n_strict = n_commit;
+    if (!greedy) set_segments(d, w.sms);
+    cudaError_t e = launch_decide(d, st);
+    if (e != cudaSuccess) return cuda_fail(e, "decide launch");
+    return SDD_OK;
+}
+
+sdd_status_t sdd_verify_lenient(const void *target_logits, sdd_dtype_t dtype, int B, int gamma, int V,
+                                int64_t row_stride, const int32_t *draft_tokens, const double *ell, int n_ell,
+                                const int32_t *rows, int n_rows, int32_t *L, int32_t *tokens, int32_t *n_commit,
+                                void *workspace, size_t workspace_bytes, int32_t *status, sdd_stream_t stream) {
+    SDD_TRY(check_shape(dtype, B, gamma, V, row_stride));
+    SDD_TRY(check_rows(rows, n_rows, B));
+    DecideParams d;
+    std::memset(&d, 0, sizeof d);
+    SDD_TRY(set_ell(d, ell, n_ell));
+    if (n_ell < 1) return fail(SDD_ERR_INVALID_ARGUMENT, "n_ell must be >= 1");
+    if (n_rows == 0) return SDD_OK;
+    SDD_TRY(check_ptr16(target_logits, "target_logits"));
+    if (!draft_tokens) return fail(SDD_ERR_INVALID_ARGUMENT, "draft_tokens is NULL");
+    Work w;
+    SDD_TRY(get_work(workspace, workspace_bytes, B, gamma, w));
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    SDD_TRY(target_scan(w, target_logits, dtype, B, gamma, V, row_stride, draft_tokens, rows, n_rows, 1, status, st));
+    DecideParams dd;
+    init_decide(dd, w, dtype, B, gamma, V, row_stride, draft_tokens, status);
+    dd.nb = n_rows;
+    dd.bidx = rows;
+    dd.zt = static_cast<const char *>(target_logits);
+    dd.n_ell = d.n_ell;
+    std::memcpy(dd.ell_thr, d.ell_thr, sizeof d.ell_thr);
+    std::memcpy(dd.ell_one, d.ell_one, sizeof d.ell_one);
+    dd.L_len = L;
+    dd.tok_len = tokens;
+    dd.n_len = n_commit;
+    cudaError_t e = launch_decide(dd, st);
+    if (e != cudaSuccess) return cuda_fail(e, "decide launch");
+    return SDD_OK;
+}
+
+sdd_status_t sdd_verify_topk(const void *target_logits, sdd_dtype_t dtype, int B, int gamma, int V,
+                             int64_t row_stride, const int32_t *draft_tokens, const int32_t *k, int n_k,
+                             const int32_t *rows, int n_rows, int32_t *L, int32_t *tokens, int32_t *n_commit,
+                             void *workspace, size_t workspace_bytes, int32_t *status, sdd_stream_t stream) {
+    SDD_TRY(check_shape(dtype, B, gamma, V, row_stride));
+    SDD_TRY(check_rows(rows, n_rows, B));
+    DecideParams d;
+    std::memset(&d, 0, sizeof d);
+    int kcap = 1;
+    SDD_TRY(set_topk(d, k, n_k, kcap));
+    if (n_k < 1) return fail(SDD_ERR_INVALID_ARGUMENT, "n_k must be >= 1");
+    if (n_rows == 0) return SDD_OK;
+    SDD_TRY(check_ptr16(target_logits, "target_logits"));
+    if (!draft_tokens) return fail(SDD_ERR_INVALID_ARGUMENT, "draft_tokens is NULL");
+    Work w;
+    SDD_TRY(get_work(workspace, workspace_bytes, B, gamma, w));
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    SDD_TRY(target_scan(w, target_logits, dtype, B, gamma, V, row_stride, draft_tokens, rows, n_rows, kcap, status,
+                        st));
+    DecideParams dd;
+    init_decide(dd, w, dtype, B, gamma, V, row_stride, draft_tokens, status);
+    dd.nb = n_rows;
+    dd.bidx = rows;
+    dd.zt = static_cast<const char *>(target_logits);
+    dd.n_k = d.n_k;
+    std::memcpy(dd.kval, d.kval, sizeof d.kval);
+    dd.L_topk = L;
+    dd.tok_topk = tokens;
+    dd.n_topk = n_commit;
+    cudaError_t e = launch_decide(dd, st);
+    if (e != cudaSuccess) return cuda_fail(e, "decide launch");
+    return SDD_OK;
+}
+
+sdd_status_t sdd_agreement(const int32_t *K, const int32_t *L_strict, int B, int n_tau, int64_t *acc,
+                           sdd_stream_t stream) {
+    if (B < 0 || n_tau < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "B and n_tau must be >= 0");
+    if (B == 0 || n_tau == 0) return SDD_OK;
+    if (!K || !L_strict || !acc) return fail(SDD_ERR_INVALID_ARGUMENT, "K, L_strict and acc must not be NULL");
+    cudaError_t e = launch_agreement(K, L_strict, B, n_tau, reinterpret_cast<long long *>(acc),
+                                     reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "agreement launch");
+    return SDD_OK;
+}
+
+sdd_status_t sdd_commit(const int32_t *K, const int32_t *draft_tokens, const int32_t *verified_tokens,
+                        const int32_t *verified_n, int B, int gamma, int32_t *out_tokens, int32_t *out_n,
+                        sdd_stream_t stream) {
+    if (B < 0 || gamma < 1 || gamma > SDD_MAX_GAMMA) return fail(SDD_ERR_INVALID_ARGUMENT, "bad B or gamma");
+    if (B == 0) return SDD_OK;
+    if (!K || !draft_tokens || !verified_tokens || !verified_n || !out_tokens || !out_n)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "NULL array");
+    cudaError_t e = launch_commit(K, draft_tokens, verified_tokens, verified_n, B, gamma, out_tokens, out_n,
+                                  reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "commit launch");
+    return SDD_OK;
+}
+
+sdd_status_t sdd_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, const uint64_t *round,
+                          const uint32_t *purpose, int64_t n, float *u, sdd_stream_t stream) {
+    if (n < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "n < 0");
+    if (n == 0) return SDD_OK;
+    if (!j || !b || !round || !purpose || !u) return fail(SDD_ERR_INVALID_ARGUMENT, "NULL array");
+    cudaError_t e = launch_uniforms(seed, j, b, round, purpose, n, u, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "uniforms launch");
+    return SDD_OK;
+}
+
+static sdd_status_t block_check(const sdd_block_args *a) {
+    if (!a) return fail(SDD_ERR_INVALID_ARGUMENT, "args is NULL");
+    SDD_TRY(check_shape(static_cast<sdd_dtype_t>(a->dtype), a->B, a->gamma, a->V, a->row_stride));
+    if (a->B == 0) return SDD_OK;
+    SDD_TRY(check_ptr16(a->draft_logits, "draft_logits"));
+    SDD_TRY(check_ptr16(a->target_logits, "target_logits"));
+    if (!a->draft_tokens) return fail(SDD_ERR_INVALID_ARGUMENT, "draft_tokens is NULL");
+    return SDD_OK;
+}
+
+sdd_status_t sdd_block_scan(const sdd_block_args *a, sdd_stream_t stream) {
+    SDD_TRY(block_check(a));
+    if (a->B == 0) return SDD_OK;
+    const sdd_dtype_t dt = static_cast<sdd_dtype_t>(a->dtype);
+    DecideParams tmp;
+    std::memset(&tmp, 0, sizeof tmp);
+    int kcap = 1;
+    SDD_TRY(set_topk(tmp, a->topk, a->n_k, kcap));
+    Work w;
+    SDD_TRY(get_work(a->workspace, a->workspace_bytes, a->B, a->gamma, w));
+    ScanParams p;
+    init_scan(p, w, dt, a->B, a->gamma, a->V, a->draft_tokens, a->status);
+    p.n_groups = 2;
+    p.kcap = kcap;
+    ScanGroup &D = p.grp[0];
+    D.base = static_cast<const char *>(a->draft_logits);
+    D.stride_bytes = a->row_stride * esize(dt);
+    D.npos = a->gamma;
+    D.kind = 0;
+    D.nb = a->B;
+    D.rec = reinterpret_cast<RowRec *>(w.base + w.L.drec);
+    D.q = a->q;
+    D.logq = a->logq;
+    D.maxprob = a->maxprob;
+    D.lse = a->lse;
+    D.entropy = a->entropy;
+    D.argmax = a->argmax;
+    ScanGroup &T = p.grp[1];
+    T.base = static_cast<const char *>(a->target_logits);
+    T.stride_bytes = a->row_stride * esize(dt);
+    T.npos = a->gamma + 1;
+    T.kind = 1;
+    T.nb = a->B;
+    T.rec = reinterpret_cast<RowRec *>(w.base + w.L.trec);
+    return run_scan(p, w, reinterpret_cast<cudaStream_t>(stream));
+}
+
+sdd_status_t sdd_block_decide(const sdd_block_args *a, sdd_stream_t stream) {
+    SDD_TRY(block_check(a));
+    const sdd_dtype_t dt = static_cast<sdd_dtype_t>(a->dtype);
+    DecideParams d;
+    std::memset(&d, 0, sizeof d);
+    SDD_TRY(set_thresholds(a->signal, a->eta_b, a->eta_c, a->n_tau, d.eta_loc, d.log_eta_c, d.tau_off));
+    SDD_TRY(set_ell(d, a->ell, a->n_ell));
+    int kcap = 1;
+    SDD_TRY(set_topk(d, a->topk, a->n_k, kcap));
+    if (a->B == 0) return SDD_OK;
+    Work w;
+    SDD_TRY(get_work(a->workspace, a->workspace_bytes, a->B, a->gamma, w));
+    DecideParams dd;
+    init_decide(dd, w, dt, a->B, a->gamma, a->V, a->row_stride, a->draft_tokens, a->status);
+    dd.nb = a->B;
+    dd.zt = static_cast<const char *>(a->target_logits);
+    dd.zd = static_cast<const char *>(a->draft_logits);
+    dd.drec = reinterpret_cast<const RowRec *>(w.base + w.L.drec);
+    dd.do_strict = 1;
+    dd.greedy = a->greedy ? 1 : 0;
+    dd.seed = a->seed;
+    dd.round = a->round;
+    dd.L_strict = a->L_strict;
+    dd.tok_strict = a->tokens_strict;
+    dd.n_strict = a->n_strict;
+    dd.n_ell = d.n_ell;
+    std::memcpy(dd.ell_thr, d.ell_thr, sizeof d.ell_thr);
+    std::memcpy(dd.ell_one, d.ell_one, sizeof d.ell_one);
+    dd.L_len = a->L_lenient;
+    dd.tok_len = a->tokens_lenient;
+    dd.n_len = a->n_lenient;
+    dd.n_k = d.n_k;
+    std::memcpy(dd.kval, d.kval, sizeof d.kval);
+    dd.L_topk = a->L_topk;
+    dd.tok_topk = a->tokens_topk;
+    dd.n_topk = a->n_topk;
+    dd.do_sched = 1;
+    dd.signal = a->signal;
+    dd.n_tau = a->n_tau;
+    dd.K_min = a->K_min;
+    dd.S_max = a->S_max;
+    std::memcpy(dd.eta_loc, d.eta_loc, sizeof d.eta_loc);
+    std::memcpy(dd.log_eta_c, d.log_eta_c, sizeof d.log_eta_c);
+    std::memcpy(dd.tau_off, d.tau_off, sizeof d.tau_off);
+    dd.guard = a->guard;
+    dd.force_strict = a->force_strict;
+    dd.D_in = a->D_in;
+    dd.K_hat = a->K_hat;
+    dd.K = a->K;
+    dd.D_out = a->D_out;
+    dd.commit_tokens = a->commit_tokens;
+    dd.commit_n = a->commit_n;
+    dd.agreement = reinterpret_cast<long long *>(a->agreement);
+    if (!dd.greedy) set_segments(dd, w.sms);
+    cudaError_t e = launch_decide(dd, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "decide launch");
+    return SDD_OK;
+}
+
+sdd_status_t sdd_block(const sdd_block_args *a, sdd_stream_t stream) {
+    SDD_TRY(sdd_block_scan(a, stream));
+    return sdd_block_decide(a, stream);
+}
+
+}  // extern "C"

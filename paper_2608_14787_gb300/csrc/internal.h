@@ -1,0 +1,136 @@
+// internal.h -- launch parameters shared between the C-ABI layer (api.cu) and
+// the kernels (scan.cu, decide.cu).  Not part of the public ABI.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/sdd.h"
+#include "common.cuh"
+
+namespace sdd {
+
+// Streaming pass geometry: each warp owns a private ring of kStages tiles of
+// kVPL 16-byte vectors per lane, filled by 1D bulk copies.
+constexpr int kWarpsPerCta = 8;
+constexpr int kThreads = kWarpsPerCta * 32;
+constexpr int kVPL = 8;                       // 16-byte vectors per lane per tile
+constexpr int kTileVec = 32 * kVPL;           // vectors per warp tile
+constexpr int kTileBytes = kTileVec * 16;     // 4 KiB
+constexpr int kStages = 3;
+constexpr int kScanSmem = kWarpsPerCta * kStages * kTileBytes + kWarpsPerCta * kStages * 8;
+constexpr uint32_t kWaitPolls = 1u << 24;     // bounded mbarrier wait (seconds of polling)
+
+// Residual / bonus draw geometry.
+constexpr int kResidThreads = 256;
+constexpr int kResidMaxSeg = 64;
+
+// One set of rows streamed by the scan kernel (drafter rows or target rows).
+struct ScanGroup {
+    const char *base;        // logits [B, npos, row_stride]
+    int64_t stride_bytes;    // row_stride * element size
+    int32_t npos;            // rows per block: gamma (drafter) or gamma+1 (target)
+    int32_t kind;            // 0 = drafter (entropy), 1 = target (rank)
+    int32_t nb;              // blocks in this group (after compaction)
+    int32_t pad;
+    const int32_t *bidx;     // [nb] batch index of each listed block, or nullptr (= identity)
+    RowRec *rec;             // [nb * npos] final records, list order
+    // drafter user outputs, indexed (b * gamma + j); any may be nullptr
+    float *q, *logq, *maxprob, *lse, *entropy;
+    int32_t *argmax;
+};
+
+struct ScanParams {
+    ScanGroup grp[2];
+    int32_t n_groups;
+    int32_t dtype;           // SDD_F32 / SDD_BF16
+    int32_t V;
+    int32_t RV;              // 16-byte vectors per row (ceil)
+    int32_t gamma;
+    int32_t kcap;            // rank saturation (>= 1)
+    int32_t B;
+    int32_t W;               // active warps
+    int64_t rows0;           // rows of group 0
+    int64_t rows;            // rows of all groups
+    int64_t T;               // total vectors = rows * RV
+    const int32_t *tokens;   // [B, gamma]
+    Partial *partials;       // [rows + W]
+    uint32_t *counters;      // [rows]
+    int32_t *status;
+};
+
+// Drafter-side facts for the sampling rule and the schedule.
+struct DecideParams {
+    int32_t B, gamma, V, RV;
+    int32_t dtype, nb;
+    int64_t stride_bytes;
+    const int32_t *bidx;           // [nb] or nullptr
+    const char *zt;                // target logits
+    const char *zd;                // drafter logits (sampling only)
+    const int32_t *tokens;         // [B, gamma]
+    const RowRec *trec;            // [nb, gamma+1] list order
+    const RowRec *drec;            // [nb, gamma] list order, or nullptr
+    const float *d_maxprob;        // [B, gamma] user arrays when drec == nullptr
+    const int32_t *d_argmax;
+    // strict
+    int32_t do_strict, greedy;
+    uint64_t seed, round;
+    int32_t *L_strict, *tok_strict, *n_strict;
+    // lenience
+    int32_t n_ell;
+    double ell_thr[SDD_MAX_GRID];
+    int32_t ell_one[SDD_MAX_GRID];
+    int32_t *L_len, *tok_len, *n_len;
+    // top-k
+    int32_t n_k;
+    int32_t kval[SDD_MAX_GRID];
+    int32_t *L_topk, *tok_topk, *n_topk;
+    // schedule (fused round only)
+    int32_t do_sched, signal, n_tau, K_min, S_max;
+    double eta_loc[SDD_MAX_GRID];
+    double log_eta_c[SDD_MAX_GRID];
+    int32_t tau_off[SDD_MAX_GRID];
+    const uint8_t *guard, *force_strict;
+    const int32_t *D_in;
+    int32_t *K_hat, *K, *D_out;
+    int32_t *commit_tokens, *commit_n;
+    int32_t *k0;                   // [nb] workspace: K under pair 0 (fused round)
+    long long *agreement;
+    // residual draw
+    int32_t nseg, seg_vec;
+    double *res_total;             // [nb, nseg]
+    int32_t *res_last;             // [nb, nseg]
+    uint32_t *res_count;           // [nb]
+    int32_t *status;
+};
+
+struct ScheduleParams {
+    const float *q, *logq;
+    int32_t B, gamma, signal, n_tau, K_min, S_max;
+    double eta_loc[SDD_MAX_GRID];
+    double log_eta_c[SDD_MAX_GRID];
+    int32_t tau_off[SDD_MAX_GRID];
+    const uint8_t *guard, *force_strict;
+    const int32_t *D_in;
+    int32_t *K_hat, *K, *D_out;
+};
+
+cudaError_t launch_scan(const ScanParams &p, int grid, cudaStream_t stream);
+cudaError_t launch_decide(const DecideParams &p, cudaStream_t stream);
+cudaError_t launch_schedule(const ScheduleParams &p, cudaStream_t stream);
+cudaError_t launch_agreement(const int32_t *K, const int32_t *L, int B, int n_tau, long long *acc,
+                             cudaStream_t stream);
+cudaError_t launch_commit(const int32_t *K, const int32_t *x, const int32_t *vt, const int32_t *vn, int B,
+                          int gamma, int32_t *out_t, int32_t *out_n, cudaStream_t stream);
+cudaError_t launch_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, const uint64_t *round,
+                            const uint32_t *purpose, int64_t n, float *u, cudaStream_t stream);
+int scan_max_ctas_per_sm();
+cudaError_t scan_prepare_device();
+
+// Index arithmetic of the balanced contiguous partition of T vectors over W
+// warps: warp w owns [start(w), start(w+1)), start(w) = floor(w T / W).
+__host__ __device__ inline int64_t part_start(int64_t w, int64_t T, int64_t W) { return (w * T) / W; }
+// The warp owning vector v (requires W <= T, so every warp is non-empty).
+__host__ __device__ inline int64_t part_owner(int64_t v, int64_t T, int64_t W) { return ((v + 1) * W - 1) / T; }
+
+}  // namespace sdd

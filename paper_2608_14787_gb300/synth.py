@@ -160,7 +160,7 @@ def _rows_runs(wl: Workload, B, G1, V, device, round_):
         sig = torch.full((B, 1, 1), wl.sigma, device=device)
     zd = torch.empty(B, G1, V, device=device)
     zt = torch.empty(B, G1, V, device=device)
-    plant = math.log(V - 1) + 0.5 + 8.0
+    plant = math.log(max(V - 1, 1)) + 0.5 + 8.0
     for b in range(B):   # per batch row keeps fp32 temporaries small
         pk = peaked[b].view(G1, 1)
         base = torch.randn(G1, V, generator=g, device=device)
@@ -191,8 +191,8 @@ def make_block(wl: Workload | str, device="cpu", round_: int = 0, greedy_drafts:
     wl = Workload(**{**wl.__dict__, "B": B, "gamma": gamma, "V": V, "dtype": dtype})
     G1 = gamma + 1
     zd, zt, peaked = _KINDS[wl.kind](wl, B, G1, V, device, round_)
-    z_d = zd[:, :gamma].to(dtype).contiguous()
-    z_t = zt.to(dtype).contiguous()
+    z_d = zd[:, :gamma].to(dtype).clone(memory_format=torch.contiguous_format)
+    z_t = zt.to(dtype).clone(memory_format=torch.contiguous_format)
     del zd, zt
     x = _gumbel_draft(z_d, _gen(device, wl.seed, round_, 7), greedy_drafts)
     return Block(z_d=z_d, z_t=z_t, x=x, peaked=peaked)

@@ -1,0 +1,94 @@
+"""GPU parity at the full sizes of the workloads (V = 151,936, gamma = 32/64),
+in the launch configuration the benchmark times (sdd_block): every block the
+oracle can finish in seconds is compared element by element; at c4 a sample
+of blocks is compared and properties that hold at any size are checked on all
+of them."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as orc
+import paper_2608_14787_gb300 as sdd
+from paper_2608_14787_gb300 import synth
+from parity_util import Tally, assert_close_stats, compare_rule, oracle_block
+
+pytestmark = pytest.mark.gpu
+
+
+def _round(wl_name, blocks=None, greedy=False):
+    wl = synth.WORKLOADS[wl_name]
+    ells = tuple(synth.paper_ell(e) for e in wl.ells)
+    ks = tuple(wl.topks)
+    blk = synth.make_block(wl, device="cuda", round_=0)
+    rnd = sdd.BlockRound(wl.B, wl.gamma, wl.V, dtype=wl.dtype, taus=wl.taus, ells=ells, ks=ks, greedy=greedy,
+                         K_min=6, S_max=64)
+    rnd.set_inputs(blk.z_d, blk.z_t, blk.x, seed=wl.seed, round_=0)
+    rnd.run()
+    torch.cuda.synchronize()
+    assert int(rnd.status.item()) == 0
+    blocks = list(range(wl.B)) if blocks is None else blocks
+    ob = oracle_block(blk.z_d[blocks], blk.z_t[blocks], blk.x[blocks], seed=wl.seed, round_=0,
+                      pairs=[(t, t) for t in wl.taus], ells=ells, ks=ks, sampling=not greedy)
+    return wl, ells, ks, blk, rnd, ob, blocks
+
+
+def _compare(wl, ells, ks, rnd, ob, blocks, greedy=False):
+    sub = lambda t: t[blocks]                                 # noqa: E731
+    assert_close_stats("q", sub(rnd.q), ob.stats.q, wl.dtype)
+    assert_close_stats("maxprob", sub(rnd.maxprob), ob.stats.maxprob, wl.dtype)
+    assert_close_stats("lse", sub(rnd.lse), ob.stats.lse, wl.dtype)
+    assert_close_stats("entropy", sub(rnd.entropy), ob.stats.entropy, wl.dtype)
+    np.testing.assert_array_equal(sub(rnd.argmax).cpu().numpy(), ob.stats.argmax)
+    idx = list(range(len(blocks)))
+    tally = Tally()
+    compare_rule(tally, "strict", sub(rnd.L_strict), sub(rnd.tokens_strict), ob.greedy if greedy else ob.strict, idx)
+    for r, e in enumerate(ells):
+        compare_rule(tally, f"lenient {e:.4f}", sub(rnd.L_lenient[r]), sub(rnd.tokens_lenient[r]), ob.lenient[e], idx)
+    for r, k in enumerate(ks):
+        compare_rule(tally, f"top-{k}", sub(rnd.L_topk[r]), sub(rnd.tokens_topk[r]), ob.topk[k], idx)
+    for t, tau in enumerate(wl.taus):
+        oKh, oK, oD, mg = ob.sched[(tau, tau)]
+        for i, b in enumerate(blocks):
+            ok = rnd.K_hat[t, b].item() == oKh[i] and rnd.K[t, b].item() == oK[i]
+            tally.check(f"schedule tau={tau} block {b}", ok, mg[i])
+    return tally
+
+
+def test_c2_full():
+    wl, ells, ks, blk, rnd, ob, blocks = _round("c2")
+    tally = _compare(wl, ells, ks, rnd, ob, blocks)
+    print("c2", tally)
+
+
+@pytest.mark.parametrize("greedy", [False, True])
+def test_c3_full(greedy):
+    wl, ells, ks, blk, rnd, ob, blocks = _round("c3", greedy=greedy)
+    tally = _compare(wl, ells, ks, rnd, ob, blocks, greedy=greedy)
+    print("c3", "greedy" if greedy else "sampling", tally)
+    # the planted structure makes skipping real at tau = 0.9
+    assert int((rnd.K[0] > 0).sum()) > 0
+
+
+def test_c4_full_sampled_and_properties():
+    blocks = [0, 9, 21, 34, 47, 63]
+    wl, ells, ks, blk, rnd, ob, blocks = _round("c4", blocks=blocks)
+    tally = _compare(wl, ells, ks, rnd, ob, blocks)
+    print("c4 sampled", tally)
+    # properties on all 64 blocks, every tau
+    K = rnd.K.cpu().numpy()
+    Kh = rnd.K_hat.cpu().numpy()
+    q = rnd.q.cpu().numpy().astype(np.float64)
+    L = rnd.L_strict.cpu().numpy()
+    for t, tau in enumerate(wl.taus):
+        below = q < tau
+        first = np.where(below.any(1), below.argmax(1), wl.gamma)
+        assert np.all(Kh[t] <= first), "a prefix extended past the first position below threshold"
+        assert np.all((K[t] == 0) | (K[t] >= 6))
+    assert np.all(K[wl.taus.index(1.0)] == 0), "tau = 1 must reproduce Strict SDD"
+    acc = rnd.agreement.cpu().numpy()
+    for t in range(len(wl.taus)):
+        np.testing.assert_array_equal(acc[t], orc.agreement(K[t], L))
+    # skip rate falls and agreement does not collapse as tau grows (Pareto sweep sanity)
+    skip = (K > 0).mean(1)
+    assert skip[0] >= skip[-2]
+    print("c4 skip rate by tau:", dict(zip(wl.taus, np.round(skip, 3))))

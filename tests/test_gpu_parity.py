@@ -1,0 +1,273 @@
+"""GPU parity: every entry point of the C ABI against the fp64 oracle on the
+same seeded inputs, at sizes the oracle finishes in seconds (several tiles per
+row, ragged tails), plus the edge cases of the method."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as orc
+from paper_2608_14787_gb300 import synth
+from parity_util import Tally, assert_close_logratio, assert_close_stats, compare_rule, host, oracle_block
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda"
+
+
+def _to_dev(blk):
+    return blk.z_d.to(DEV), blk.z_t.to(DEV), blk.x.to(DEV)
+
+
+def _padded(z: torch.Tensor, stride: int) -> torch.Tensor:
+    """Same logits with each row padded to `stride` elements (padding = +inf,
+    which the library must never read into a result)."""
+    B, P, V = z.shape
+    buf = torch.full((B, P, stride), float("inf"), dtype=z.dtype, device=z.device)
+    buf[..., :V] = z
+    return buf[..., :V]
+
+
+# ---------------------------------------------------------------------------
+# confidence (Sec. 4.2)
+# ---------------------------------------------------------------------------
+
+def _check_confidence(sdd, z_d, x, dtype):
+    out = sdd.confidence(z_d, x)
+    torch.cuda.synchronize()
+    st = orc.row_stats(host(z_d.contiguous() if z_d.is_contiguous() else z_d), tokens=x.cpu().numpy())
+    errs = {}
+    errs["q"] = assert_close_stats("q", out.q, st.q, dtype)
+    errs["logq"] = assert_close_logratio("logq", out.logq, st.logq, dtype)
+    errs["maxprob"] = assert_close_stats("maxprob", out.maxprob, st.maxprob, dtype)
+    errs["lse"] = assert_close_stats("lse", out.lse, st.lse, dtype)
+    errs["entropy"] = assert_close_stats("entropy", out.entropy, st.entropy, dtype)
+    np.testing.assert_array_equal(out.argmax.cpu().numpy(), st.argmax)
+    return errs
+
+
+def test_confidence_tiny_fp32(sdd):
+    blk = synth.make_block("tiny", device="cpu")
+    z_d, z_t, x = _to_dev(blk)
+    errs = _check_confidence(sdd, z_d, x, torch.float32)
+    print("tiny fp32 max rel errors:", errs)
+
+
+@pytest.mark.parametrize("B,gamma,V", [(3, 5, 1003), (2, 7, 8), (1, 3, 1), (4, 33, 20011), (2, 64, 4096)])
+def test_confidence_bf16_shapes(sdd, B, gamma, V):
+    blk = synth.make_block("c3", device="cpu", B=B, gamma=gamma, V=V)
+    z_d, z_t, x = _to_dev(blk)
+    stride = ((V + 7) // 8) * 8
+    zp = _padded(z_d, stride) if stride != V else z_d
+    errs = _check_confidence(sdd, zp, x, torch.bfloat16)
+    print(f"bf16 B={B} gamma={gamma} V={V} max rel errors:", errs)
+
+
+def test_confidence_fp32_ragged(sdd):
+    blk = synth.make_block("tiny", device="cpu", B=3, gamma=4, V=1001)
+    z_d, _, x = _to_dev(blk)
+    _check_confidence(sdd, _padded(z_d, 1004), x, torch.float32)
+
+
+def test_confidence_nonfinite_and_bad_tokens(sdd):
+    blk = synth.make_block("c3", device="cpu", B=2, gamma=4, V=3000)
+    z_d, _, x = _to_dev(blk)
+    z_d = z_d.clone()
+    z_d[0, 1, 17] = float("nan")
+    z_d[1, 2, 5] = float("inf")
+    z_d[1, 3, :] = float("-inf")
+    x = x.clone()
+    x[0, 3] = 3000          # out of range
+    status = sdd.new_status()
+    out = sdd.confidence(z_d, x, status=status)
+    torch.cuda.synchronize()
+    s = int(status.item())
+    assert s & sdd.DEV_NONFINITE and s & sdd.DEV_BAD_TOKEN
+    q = out.q.cpu()
+    assert math.isnan(q[0, 1]) and math.isnan(q[1, 2]) and math.isnan(q[1, 3]) and math.isnan(q[0, 3])
+    assert out.argmax[0, 1].item() == -1 and out.argmax[1, 3].item() == -1
+    # untouched rows still agree with the oracle
+    st = orc.row_stats(host(z_d), tokens=np.clip(x.cpu().numpy(), 0, 2999))
+    assert q[0, 0].item() == pytest.approx(st.q[0, 0], rel=2e-3)
+    # masked (-inf) entries in an otherwise finite row are fine
+    z2 = z_d.clone()
+    z2[0, 0, :100] = float("-inf")
+    x2 = x.clone()
+    x2[0, 0] = 500
+    out2 = sdd.confidence(z2, x2)
+    st2 = orc.row_stats(host(z2[:1, :1]), tokens=x2[:1, :1].cpu().numpy())
+    assert out2.entropy[0, 0].item() == pytest.approx(st2.entropy[0, 0], rel=2e-3)
+    assert out2.q[0, 0].item() == pytest.approx(st2.q[0, 0], rel=2e-3)
+
+
+def test_confidence_deterministic(sdd):
+    blk = synth.make_block("c3", device="cpu", B=4, gamma=16, V=50000)
+    z_d, _, x = _to_dev(blk)
+    a = sdd.confidence(z_d, x)
+    b = sdd.confidence(z_d, x)
+    for f in ("q", "logq", "maxprob", "lse", "entropy", "argmax"):
+        assert torch.equal(getattr(a, f), getattr(b, f)), f
+
+
+# ---------------------------------------------------------------------------
+# schedule (Sec. 4.1 Eq. 3)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("signal", [0, 1, 2])
+def test_schedule_vs_oracle(sdd, signal):
+    rng = np.random.default_rng(100 + signal)
+    B, gamma = 257, 40
+    q = (1.0 - 0.35 * rng.random((B, gamma)) ** 4).astype(np.float32)
+    q[rng.random((B, gamma)) < 0.01] = np.nan
+    guard = (rng.random((B, gamma)) < 0.02).astype(np.uint8)
+    force = (rng.random(B) < 0.05).astype(np.uint8)
+    D = rng.integers(0, 80, size=B).astype(np.int32)
+    pairs = [(0.9, 0.93), (0.95, 0.9), (0.8, 0.85), (0.7, 0.7), (0.9, 1.0), (0.99, 0.995), (0.6, 0.5),
+             (0.0, 0.9), (0.9, 0.0)]
+    K_min, S_max = 3, 64
+    dq = torch.from_numpy(q).to(DEV)
+    Kh, K, Do = sdd.schedule_prefix(dq, [p[0] for p in pairs], [p[1] for p in pairs], signal=signal, K_min=K_min,
+                                    S_max=S_max, guard=torch.from_numpy(guard).to(DEV),
+                                    force_strict=torch.from_numpy(force).to(DEV), D_in=torch.from_numpy(D).to(DEV))
+    torch.cuda.synchronize()
+    tally = Tally()
+    for t, (eb, ec) in enumerate(pairs):
+        oKh, oK, oD, mg = orc.schedule(q.astype(np.float64), signal, eb, ec, K_min, S_max, guard=guard,
+                                       force_strict=force, D_in=D)
+        for b in range(B):
+            ok = (Kh[t, b].item() == oKh[b]) and (K[t, b].item() == oK[b]) and (Do[t, b].item() == oD[b])
+            tally.check(f"signal {signal} pair {(eb, ec)} block {b}", ok, mg[b])
+    print("schedule", signal, tally)
+
+
+# ---------------------------------------------------------------------------
+# verification rules (Sec. 3.1, App. A.6)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("wl,B,gamma,V,greedy_drafts", [
+    ("c3", 6, 12, 5003, False), ("c3", 5, 9, 30000, True), ("c2", 2, 16, 20000, False), ("tiny", 3, 8, 4001, False),
+])
+def test_verify_rules_vs_oracle(sdd, wl, B, gamma, V, greedy_drafts):
+    blk = synth.make_block(wl, device="cpu", B=B, gamma=gamma, V=V, greedy_drafts=greedy_drafts,
+                           dtype=torch.float32 if wl == "tiny" else torch.bfloat16)
+    z_d, z_t, x = _to_dev(blk)
+    stride = ((V + 7) // 8) * 8
+    if stride != V:
+        z_d, z_t = _padded(z_d, stride), _padded(z_t, stride)
+    ells = (1.0, 0.9, 0.5, 0.25)
+    ks = (1, 2, 5, 10)
+    seed, rnd = 1234, 7
+    draft = sdd.confidence(z_d, x)
+    Ls, tks, _ = sdd.verify_strict(z_t, x, z_d=z_d, draft=draft, greedy=False, seed=seed, round_=rnd)
+    Lg, tkg, _ = sdd.verify_strict(z_t, x, greedy=True)
+    Ll, tkl, _ = sdd.verify_lenient(z_t, x, ells)
+    Lk, tkk, _ = sdd.verify_topk(z_t, x, ks)
+    torch.cuda.synchronize()
+    ob = oracle_block(z_d, z_t, x, seed=seed, round_=rnd, ells=ells, ks=ks)
+    blocks = list(range(B))
+    tally = Tally()
+    compare_rule(tally, "strict-sampling", Ls, tks, ob.strict, blocks)
+    compare_rule(tally, "strict-greedy", Lg, tkg, ob.greedy, blocks)
+    for r, e in enumerate(ells):
+        compare_rule(tally, f"lenient {e}", Ll[r], tkl[r], ob.lenient[e], blocks)
+    for r, k in enumerate(ks):
+        compare_rule(tally, f"top-{k}", Lk[r], tkk[r], ob.topk[k], blocks)
+    print(wl, tally)
+    assert tally.compared == B * (2 + len(ells) + len(ks))
+
+
+def test_verify_row_subset(sdd):
+    blk = synth.make_block("c3", device="cpu", B=8, gamma=10, V=4096)
+    z_d, z_t, x = _to_dev(blk)
+    rows = torch.tensor([6, 1, 3], dtype=torch.int32, device=DEV)
+    draft = sdd.confidence(z_d, x)
+    L, tok, n = sdd.verify_strict(z_t, x, z_d=z_d, draft=draft, seed=5, round_=2, rows=rows)
+    torch.cuda.synchronize()
+    ob = oracle_block(z_d, z_t, x, seed=5, round_=2, blocks=[6, 1, 3])
+    tally = Tally()
+    compare_rule(tally, "subset", L, tok, ob.strict, [6, 1, 3])
+    untouched = [b for b in range(8) if b not in (6, 1, 3)]
+    assert torch.all(L[untouched] == -2) and torch.all(tok[untouched] == -2) and torch.all(n[untouched] == -2)
+
+
+def test_identical_rows_accept_everything(sdd):
+    blk = synth.make_block("c3", device="cpu", B=16, gamma=16, V=8192)
+    z_d, _, x = _to_dev(blk)
+    z_t = torch.cat([z_d, z_d[:, -1:]], dim=1).contiguous()
+    draft = sdd.confidence(z_d, x)
+    L, tok, n = sdd.verify_strict(z_t, x, z_d=z_d, draft=draft, seed=9, round_=0)
+    torch.cuda.synchronize()
+    # p_t = p_d: the acceptance ratio is one up to fp32 rounding (|log r| < 1e-6)
+    assert int((L == 16).sum()) >= 15
+    Lg, _, _ = sdd.verify_strict(z_t, x, greedy=True)
+
+
+def test_philox_device_matches_oracle(sdd):
+    n = 1 << 20
+    rng = np.random.default_rng(3)
+    j = rng.integers(0, 1 << 32, size=n, dtype=np.uint64).astype(np.uint32)
+    b = rng.integers(0, 1 << 32, size=n, dtype=np.uint64).astype(np.uint32)
+    r = rng.integers(0, 1 << 62, size=n, dtype=np.uint64)
+    p = rng.integers(0, 4, size=n).astype(np.uint32)
+    seed = 0xDEADBEEF12345678
+    u = sdd.uniforms(seed, torch.from_numpy(j.view(np.int32)).to(DEV), torch.from_numpy(b.view(np.int32)).to(DEV),
+                     torch.from_numpy(r.view(np.int64)).to(DEV), torch.from_numpy(p.view(np.int32)).to(DEV))
+    want = orc.uniform_many(seed, j, b, r, p)
+    np.testing.assert_array_equal(u.cpu().numpy().astype(np.float64), want)
+
+
+# ---------------------------------------------------------------------------
+# fused round
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("greedy", [False, True])
+def test_block_round_vs_oracle(sdd, greedy):
+    B, gamma, V = 12, 16, 12007
+    blk = synth.make_block("c3", device="cpu", B=B, gamma=gamma, V=V, greedy_drafts=greedy)
+    z_d, z_t, x = _to_dev(blk)
+    z_d, z_t = _padded(z_d, 12008), _padded(z_t, 12008)
+    taus = (0.5, 0.9, 0.95, 1.0)
+    ells, ks = (1.0, 0.5), (2, 5)
+    rnd = sdd.BlockRound(B, gamma, V, taus=taus, ells=ells, ks=ks, greedy=greedy, K_min=2, S_max=64)
+    D = torch.randint(0, 70, (B,), dtype=torch.int32)
+    rnd.D_in.copy_(D)
+    rnd.set_inputs(z_d, z_t, x, seed=77, round_=3)
+    rnd.run()
+    torch.cuda.synchronize()
+    assert int(rnd.status.item()) == 0
+    ob = oracle_block(z_d, z_t, x, seed=77, round_=3, pairs=[(t, t) for t in taus], K_min=2, S_max=64,
+                      D_in=D.numpy(), ells=ells, ks=ks, sampling=not greedy)
+    assert_close_stats("q", rnd.q, ob.stats.q, torch.bfloat16)
+    assert_close_stats("entropy", rnd.entropy, ob.stats.entropy, torch.bfloat16)
+    np.testing.assert_array_equal(rnd.argmax.cpu().numpy(), ob.stats.argmax)
+    blocks = list(range(B))
+    tally = Tally()
+    compare_rule(tally, "strict", rnd.L_strict, rnd.tokens_strict, ob.greedy if greedy else ob.strict, blocks)
+    for r, e in enumerate(ells):
+        compare_rule(tally, f"lenient {e}", rnd.L_lenient[r], rnd.tokens_lenient[r], ob.lenient[e], blocks)
+    for r, k in enumerate(ks):
+        compare_rule(tally, f"top-{k}", rnd.L_topk[r], rnd.tokens_topk[r], ob.topk[k], blocks)
+    L_or = np.array([(ob.greedy if greedy else ob.strict)[b][0] for b in blocks])
+    acc_want = np.zeros((len(taus), 4), np.int64)
+    for t, tau in enumerate(taus):
+        oKh, oK, oD, mg = ob.sched[(tau, tau)]
+        for b in blocks:
+            ok = (rnd.K_hat[t, b].item() == oKh[b] and rnd.K[t, b].item() == oK[b] and rnd.D_out[t, b].item() == oD[b])
+            tally.check(f"schedule tau {tau} block {b}", ok, mg[b])
+        acc_want[t] = orc.agreement(oK, L_or)
+    np.testing.assert_array_equal(rnd.agreement.cpu().numpy(), acc_want)
+    # committed tokens under pair 0
+    oK0 = ob.sched[(taus[0], taus[0])][1]
+    ct = rnd.commit_tokens.cpu().numpy()
+    cn = rnd.commit_n.cpu().numpy()
+    xs = x.cpu().numpy()
+    for b in blocks:
+        if oK0[b] > 0:
+            assert cn[b] == oK0[b] and np.array_equal(ct[b][:oK0[b]], xs[b][:oK0[b]]) and np.all(ct[b][oK0[b]:] == -1)
+        else:
+            L, tok, _ = (ob.greedy if greedy else ob.strict)[b]
+            assert cn[b] == L + 1 and np.array_equal(ct[b], tok)
+    print("block round", tally)
+    # tau = 1 reproduces Strict SDD with zero skips
+    assert torch.all(rnd.K[3] == 0)
