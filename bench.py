@@ -192,77 +192,12 @@ def _cpu_baseline(wl, ells, ks, blk_host, n_blocks):
                       f"({dt:.1f} s)"}
 
 
-def run_gpu(args):
+def _e2e(args, ws, dev, stream, sets, rnd, wl, B):
+    """The same round end to end through the C ABI: inputs copied from pinned
+    host buffers and results copied back inside the timed region."""
     import torch
-    import paper_2608_14787_gb300 as sdd
-    from paper_2608_14787_gb300 import build as sdd_build
-    from paper_2608_14787_gb300 import synth
-
-    ws, rank, local = _dist()
     if ws > 1:
         import torch.distributed as dist
-        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    if rank == 0:
-        sdd_build.build()
-    if ws > 1:
-        dist.barrier()
-    sdd.load()
-
-    wl, ells, ks = _workload_cfg(args.workload)
-    B, gamma, V = wl.B, wl.gamma, wl.V
-    n_sets = 3
-    sets = [synth.make_block(wl, device=dev, round_=r + 1000 * rank) for r in range(n_sets)]
-    rnd = sdd.BlockRound(B, gamma, V, dtype=wl.dtype, taus=wl.taus, ells=ells, ks=ks, K_min=6, S_max=64,
-                         device=dev)
-    esz = 2 if wl.dtype == torch.bfloat16 else 4
-    scan_bytes = (2 * gamma + 1) * V * esz * B          # every logit read once
-    stream = torch.cuda.current_stream()
-
-    def step(i, ev=None):
-        s = sets[i % n_sets]
-        rnd.set_inputs(s.z_d, s.z_t, s.x, seed=wl.seed, round_=i)
-        if ev is not None:
-            ev[0].record(stream)
-        rnd.scan()
-        if ev is not None:
-            ev[1].record(stream)
-        rnd.decide()
-
-    for i in range(args.warmup):
-        step(i)
-    torch.cuda.synchronize()
-    if int(rnd.status.item()) != 0:
-        raise RuntimeError(f"device status {int(rnd.status.item())} after warm-up")
-
-    # ---- device-resident timed region ----
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    bus = torch.cuda.get_device_properties(dev).pci_bus_id if hasattr(torch.cuda.get_device_properties(dev),
-                                                                      "pci_bus_id") else None
-    if ws > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-    with ClockSampler(bus) as clk:
-        t_start.record(stream)
-        for i in range(args.steps):
-            step(i, evs[i])
-        t_end.record(stream)
-        torch.cuda.synchronize()
-    if ws > 1:
-        dist.barrier()
-    total_ms = t_start.elapsed_time(t_end)
-    scan_ms = [a.elapsed_time(b) for a, b in evs]
-    scan_avg_ms = sum(scan_ms) / len(scan_ms)
-    if ws > 1:
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
-    value = ws * B * args.steps / (total_ms / 1e3)
-    status = int(rnd.status.item())
-
-    # ---- end-to-end through the C ABI from pinned host buffers ----
     hz_d = sets[0].z_d.cpu().pin_memory()
     hz_t = sets[0].z_t.cpu().pin_memory()
     hx = sets[0].x.cpu().pin_memory()
@@ -298,22 +233,98 @@ def run_gpu(args):
         t = torch.tensor([e2e_ms], device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         e2e_ms = float(t.item())
-    e2e_value = ws * B * e2e_steps / (e2e_ms / 1e3)
+    return ws * B * e2e_steps / (e2e_ms / 1e3), h2d, d2h
+
+
+def run_gpu(args):
+    import torch
+    import paper_2608_14787_gb300 as sdd
+    from paper_2608_14787_gb300 import build as sdd_build
+    from paper_2608_14787_gb300 import synth
+
+    ws, rank, local = _dist()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if rank == 0:
+        sdd_build.build()
+    if ws > 1:
+        dist.barrier()
+    sdd.load()
+
+    wl, ells, ks = _workload_cfg(args.workload)
+    B, gamma, V = wl.B, wl.gamma, wl.V
+    n_sets = max(1, args.sets)
+    sets = [synth.make_block(wl, device=dev, round_=r + 1000 * rank) for r in range(n_sets)]
+    rnd = sdd.BlockRound(B, gamma, V, dtype=wl.dtype, taus=wl.taus, ells=ells, ks=ks, K_min=6, S_max=64,
+                         device=dev)
+    esz = 2 if wl.dtype == torch.bfloat16 else 4
+    scan_bytes = (2 * gamma + 1) * V * esz * B          # every logit read once
+    stream = torch.cuda.current_stream()
+
+    def step(i, ev=None):
+        s = sets[i % n_sets]
+        rnd.set_inputs(s.z_d, s.z_t, s.x, seed=wl.seed, round_=i)
+        if ev is not None:
+            ev[0].record(stream)
+        rnd.scan()
+        if ev is not None:
+            ev[1].record(stream)
+        rnd.decide()
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    if int(rnd.status.item()) != 0:
+        raise RuntimeError(f"device status {int(rnd.status.item())} after warm-up")
+
+    # ---- device-resident timed region ----
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    props = torch.cuda.get_device_properties(dev)
+    bus = getattr(props, "pci_bus_id", None)
+    if ws > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(bus) as clk:
+        t_start.record(stream)
+        for i in range(args.steps):
+            step(i, evs[i])
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    if ws > 1:
+        dist.barrier()
+    total_ms = t_start.elapsed_time(t_end)
+    scan_ms = [a.elapsed_time(b) for a, b in evs]
+    scan_avg_ms = sum(scan_ms) / len(scan_ms)
+    if ws > 1:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    value = ws * B * args.steps / (total_ms / 1e3)
+    status = int(rnd.status.item())
+
+    if args.no_e2e:
+        e2e = None
+    else:
+        e2e_value, h2d, d2h = _e2e(args, ws, dev, stream, sets, rnd, wl, B)
+        e2e = {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
     peak, peak_kind = _peaks()
     achieved = scan_bytes / (scan_avg_ms / 1e3) / 1e9
-    line = None
     if rank == 0:
         cpu = None
         if ws == 1 and not args.no_cpu_baseline:
             import numpy as np
-            host = {"z_d": sets[0].z_d[:args.cpu_blocks].cpu().view(torch.int16).numpy().view(np.uint16)
-                    if wl.dtype == torch.bfloat16 else sets[0].z_d[:args.cpu_blocks].cpu().numpy(),
-                    "z_t": sets[0].z_t[:args.cpu_blocks].cpu().view(torch.int16).numpy().view(np.uint16)
-                    if wl.dtype == torch.bfloat16 else sets[0].z_t[:args.cpu_blocks].cpu().numpy(),
-                    "x": sets[0].x[:args.cpu_blocks].cpu().numpy()}
-            cpu = _cpu_baseline(wl, ells, ks, host, min(args.cpu_blocks, B))
-        clocks = clk.summary()
+            nb = min(args.cpu_blocks, B)
+
+            def h(t):
+                t = t[:nb].cpu()
+                return t.view(torch.int16).numpy().view(np.uint16) if t.dtype == torch.bfloat16 else t.numpy()
+            host = {"z_d": h(sets[0].z_d), "z_t": h(sets[0].z_t), "x": sets[0].x[:nb].cpu().numpy()}
+            cpu = _cpu_baseline(wl, ells, ks, host, nb)
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
@@ -325,9 +336,9 @@ def run_gpu(args):
                          "peak_source": f"{peak_kind} hbm_gbs", "bytes_per_launch": scan_bytes,
                          "avg_launch_ms": scan_avg_ms},
             "cpu_baseline": cpu,
-            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "e2e": e2e,
             "gpu_launches": 2 * args.steps,
-            "clocks": clocks,
+            "clocks": clk.summary(),
             "device_status": status,
         }
         print(json.dumps(line), flush=True)
@@ -346,6 +357,8 @@ def main():
     ap.add_argument("--workload", default="c3")
     ap.add_argument("--cpu-blocks", type=int, default=8)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--sets", type=int, default=3, help="rotating input sets (3 x 316 MB exceeds L2)")
     ap.add_argument("--traffic", type=float, default=None,
                     help="dram bytes per scan launch from an ncu capture of the current kernel")
     args = ap.parse_args()

@@ -102,17 +102,19 @@ SDD_API sdd_status_t sdd_workspace_size(int B, int gamma, int V, size_t *bytes);
  *   q       = p_draft(x_j) = exp(z(x_j) - LSE)      (raw confidence, Sec. 4.2)
  *   logq    = z(x_j) - LSE
  *   maxprob = max_v p(v)                            (top-1 probability, App. A.7)
- *   lse     = log sum_v exp(z(v))
+ *   lse     = log sum_v exp(z(v)), in fp64 (the exact normaliser the sampling
+ *             rule of sdd_verify_strict needs)
  *   entropy = -sum_v p(v) ln p(v), in nats          (App. A.7 feature)
  *   argmax  = lowest index attaining max_v z(v)
- * All outputs are [B, gamma]; every one but q may be NULL.  A row with NaN or
+ * All outputs are [B, gamma]; every one but q may be NULL.  Finite logits
+ * below -2^23 are treated as masked (-inf).  A row with NaN or
  * +inf logits, or only -inf, yields NaN statistics, argmax -1 and sets
  * SDD_DEV_NONFINITE; a drafted token outside [0, V) yields NaN q/logq and sets
  * SDD_DEV_BAD_TOKEN.  One streaming pass reads every logit exactly once.
  */
 SDD_API sdd_status_t sdd_confidence(const void *draft_logits, sdd_dtype_t dtype, int B, int gamma, int V,
                             int64_t row_stride, const int32_t *draft_tokens, float *q, float *logq,
-                            float *maxprob, float *lse, float *entropy, int32_t *argmax,
+                            float *maxprob, double *lse, float *entropy, int32_t *argmax,
                             void *workspace, size_t workspace_bytes, int32_t *status,
                             sdd_stream_t stream);
 
@@ -161,15 +163,14 @@ SDD_API sdd_status_t sdd_schedule_prefix(const float *q, const float *logq, int 
  *     (seed low, seed high 32 bits) and counter (j, b, round low 32,
  *     purpose | round high 32 << 8); u = ((word0 >> 8) | 1) * 2^-24.
  * Inputs: target_logits [B, gamma+1, row_stride]; draft_logits [B, gamma,
- *   row_stride], draft_maxprob and draft_argmax [B, gamma] as written by
- *   sdd_confidence (all three may be NULL when greedy != 0); draft_tokens [B, gamma].
+ *   row_stride] and draft_lse [B, gamma] (fp64, as written by sdd_confidence;
+ *   both may be NULL when greedy != 0); draft_tokens [B, gamma].
  * Outputs, written only at the listed rows b: L [B] accepted length;
  *   tokens [B, gamma+1] = x_1..x_L, the drawn token, then -1; n_commit [B] = L+1.
  */
 SDD_API sdd_status_t sdd_verify_strict(const void *target_logits, const void *draft_logits,
                                sdd_dtype_t dtype, int B, int gamma, int V, int64_t row_stride,
-                               const int32_t *draft_tokens, const float *draft_maxprob,
-                               const int32_t *draft_argmax, int greedy, uint64_t seed,
+                               const int32_t *draft_tokens, const double *draft_lse, int greedy, uint64_t seed,
                                uint64_t round, const int32_t *rows, int n_rows, int32_t *L,
                                int32_t *tokens, int32_t *n_commit, void *workspace,
                                size_t workspace_bytes, int32_t *status, sdd_stream_t stream);
@@ -270,8 +271,10 @@ typedef struct sdd_block_args {
     int32_t n_ell, n_k;            /* 0..SDD_MAX_GRID each */
     const double *ell;             /* HOST [n_ell], 0 < ell <= 1 */
     const int32_t *topk;           /* HOST [n_k] */
-    /* outputs: confidence [B, gamma] */
-    float *q, *logq, *maxprob, *lse, *entropy;
+    /* outputs: confidence [B, gamma] (lse in fp64) */
+    float *q, *logq, *maxprob;
+    double *lse;
+    float *entropy;
     int32_t *argmax;
     /* outputs: schedule [n_tau, B] */
     int32_t *K_hat, *K, *D_out;

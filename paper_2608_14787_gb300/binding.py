@@ -75,7 +75,7 @@ def load(path: str | None = None):
     L.sdd_workspace_size.argtypes = [I, I, I, ctypes.POINTER(ctypes.c_size_t)]
     L.sdd_confidence.argtypes = [VP, I, I, I, I, i64, VP, VP, VP, VP, VP, VP, VP, VP, ctypes.c_size_t, VP, VP]
     L.sdd_schedule_prefix.argtypes = [VP, VP, I, I, I, c_f64p, c_f64p, I, I, I, VP, VP, VP, VP, VP, VP, VP, VP]
-    L.sdd_verify_strict.argtypes = [VP, VP, I, I, I, I, i64, VP, VP, VP, I, u64, u64, VP, I, VP, VP, VP, VP,
+    L.sdd_verify_strict.argtypes = [VP, VP, I, I, I, I, i64, VP, VP, I, u64, u64, VP, I, VP, VP, VP, VP,
                                     ctypes.c_size_t, VP, VP]
     L.sdd_verify_lenient.argtypes = [VP, I, I, I, I, i64, VP, c_f64p, I, VP, I, VP, VP, VP, VP, ctypes.c_size_t,
                                      VP, VP]
@@ -178,8 +178,9 @@ def confidence(z_d: torch.Tensor, x: torch.Tensor, ws: Workspace | None = None, 
     dev = z_d.device
     ws = ws or Workspace(B, gamma, V, dev)
     status = new_status(dev) if status is None else status
-    out = Confidence(*(torch.empty(B, gamma, dtype=torch.float32, device=dev) for _ in range(5)),
-                     torch.empty(B, gamma, dtype=torch.int32, device=dev))
+    f32 = lambda: torch.empty(B, gamma, dtype=torch.float32, device=dev)  # noqa: E731
+    out = Confidence(q=f32(), logq=f32(), maxprob=f32(), lse=torch.empty(B, gamma, dtype=torch.float64, device=dev),
+                     entropy=f32(), argmax=torch.empty(B, gamma, dtype=torch.int32, device=dev))
     rc = load().sdd_confidence(_p(z_d), _dtype_code(z_d), B, gamma, V, stride, _p(x), _p(out.q), _p(out.logq),
                                _p(out.maxprob), _p(out.lse), _p(out.entropy), _p(out.argmax), ws.ptr, ws.nbytes,
                                _p(status), _stream(stream))
@@ -222,9 +223,8 @@ def verify_strict(z_t, x, *, z_d=None, draft=None, greedy=False, seed=0, round_=
                torch.full((B,), -2, dtype=torch.int32, device=dev))
     L, tok, n = out
     n_rows = B if rows is None else rows.numel()
-    mp = None if draft is None else draft.maxprob
-    am = None if draft is None else draft.argmax
-    rc = load().sdd_verify_strict(_p(z_t), _p(z_d), _dtype_code(z_t), B, gamma, V, stride, _p(x), _p(mp), _p(am),
+    lse = None if draft is None else draft.lse
+    rc = load().sdd_verify_strict(_p(z_t), _p(z_d), _dtype_code(z_t), B, gamma, V, stride, _p(x), _p(lse),
                                   1 if greedy else 0, seed, round_, _p(rows), n_rows, _p(L), _p(tok), _p(n),
                                   ws.ptr, ws.nbytes, _p(status), _stream(stream))
     _check(rc, "sdd_verify_strict")
@@ -315,7 +315,8 @@ class BlockRound:
         self.status = new_status(dev)
         f32 = lambda *s: torch.zeros(*s, dtype=torch.float32, device=dev)   # noqa: E731
         i32 = lambda *s: torch.zeros(*s, dtype=torch.int32, device=dev)     # noqa: E731
-        self.q, self.logq, self.maxprob, self.lse, self.entropy = (f32(B, gamma) for _ in range(5))
+        self.q, self.logq, self.maxprob, self.entropy = (f32(B, gamma) for _ in range(4))
+        self.lse = torch.zeros(B, gamma, dtype=torch.float64, device=dev)
         self.argmax = i32(B, gamma)
         self.K_hat, self.K, self.D_out = (i32(self.n_tau, B) for _ in range(3))
         self.D_in = i32(B)

@@ -295,7 +295,7 @@ sdd_status_t sdd_workspace_size(int B, int gamma, int V, size_t *bytes) {
 
 sdd_status_t sdd_confidence(const void *draft_logits, sdd_dtype_t dtype, int B, int gamma, int V,
                             int64_t row_stride, const int32_t *draft_tokens, float *q, float *logq,
-                            float *maxprob, float *lse, float *entropy, int32_t *argmax, void *workspace,
+                            float *maxprob, double *lse, float *entropy, int32_t *argmax, void *workspace,
                             size_t workspace_bytes, int32_t *status, sdd_stream_t stream) {
     SDD_TRY(check_shape(dtype, B, gamma, V, row_stride));
     if (B == 0) return SDD_OK;
@@ -357,7 +357,7 @@ sdd_status_t sdd_schedule_prefix(const float *q, const float *logq, int B, int g
 
 sdd_status_t sdd_verify_strict(const void *target_logits, const void *draft_logits, sdd_dtype_t dtype, int B,
                                int gamma, int V, int64_t row_stride, const int32_t *draft_tokens,
-                               const float *draft_maxprob, const int32_t *draft_argmax, int greedy, uint64_t seed,
+                               const double *draft_lse, int greedy, uint64_t seed,
                                uint64_t round, const int32_t *rows, int n_rows, int32_t *L, int32_t *tokens,
                                int32_t *n_commit, void *workspace, size_t workspace_bytes, int32_t *status,
                                sdd_stream_t stream) {
@@ -368,8 +368,7 @@ sdd_status_t sdd_verify_strict(const void *target_logits, const void *draft_logi
     if (!draft_tokens) return fail(SDD_ERR_INVALID_ARGUMENT, "draft_tokens is NULL");
     if (!greedy) {
         SDD_TRY(check_ptr16(draft_logits, "draft_logits"));
-        if (!draft_maxprob || !draft_argmax)
-            return fail(SDD_ERR_INVALID_ARGUMENT, "sampling needs draft_maxprob and draft_argmax");
+        if (!draft_lse) return fail(SDD_ERR_INVALID_ARGUMENT, "sampling needs draft_lse");
     }
     Work w;
     SDD_TRY(get_work(workspace, workspace_bytes, B, gamma, w));
@@ -381,8 +380,7 @@ sdd_status_t sdd_verify_strict(const void *target_logits, const void *draft_logi
     d.bidx = rows;
     d.zt = static_cast<const char *>(target_logits);
     d.zd = static_cast<const char *>(draft_logits);
-    d.d_maxprob = draft_maxprob;
-    d.d_argmax = draft_argmax;
+    d.d_lse = draft_lse;
     d.do_strict = 1;
     d.greedy = greedy ? 1 : 0;
     d.seed = seed;

@@ -16,36 +16,52 @@ namespace sdd {
 // ---------------------------------------------------------------------------
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
-// Every logit is clamped from below to -2^100 (exact in bf16 and fp32).  A
-// masked (-inf) logit then contributes exp(-huge) = 0 to every sum and 0 * y
-// = 0 to the entropy accumulator without ever forming inf - inf or 0 * inf.
-constexpr uint32_t kClampBits = 0xF1800000u;      // -2^100 as fp32 bits
-constexpr uint32_t kClampPairBf16 = 0xF180F180u;  // the same value in both bf16 halves
+constexpr double kLn2d = 0.6931471805599453094;
+constexpr double kLog2ed = 1.4426950408889634074;
+// Every logit is clamped from below to -2^23 (exact in bf16 and fp32).  A
+// masked (-inf) logit then contributes 2^(-huge) = 0 to every sum and 0 * y = 0
+// to the entropy accumulator without ever forming inf - inf or 0 * inf, and
+// every scaling reference (an integer in log2 units, see SoftState) stays an
+// exactly representable fp32 integer.  Finite logits below -2^23 act as masked.
+constexpr uint32_t kClampBits = 0xCB000000u;      // -2^23 as fp32 bits
+constexpr uint32_t kClampPairBf16 = 0xCB00CB00u;  // the same value in both bf16 halves
 constexpr uint32_t kNegInfPairBf16 = 0xFF80FF80u;
 
 __device__ __forceinline__ float clamp_floor() { return __uint_as_float(kClampBits); }
+// ceil(-2^23 * log2(e)) in fp32: the reference of an empty / fully masked state.
+__device__ __forceinline__ float clamp_ref() { return ceilf(clamp_floor() * kLog2e); }
+
+// Exact powers of two 2^k for integer-valued k <= 0 (0 below the normal range).
+__device__ __forceinline__ float pow2f_int(float k) {
+    return (k < -126.f) ? 0.f : __int_as_float((127 + static_cast<int>(k)) << 23);
+}
+__device__ __forceinline__ double pow2d_int(float k) {
+    return (k < -1022.f) ? 0.0 : __longlong_as_double(static_cast<long long>(1023 + static_cast<int>(k)) << 52);
+}
 
 // ---------------------------------------------------------------------------
 // Records exchanged through the workspace
 // ---------------------------------------------------------------------------
-// Partial softmax state of one warp's piece of one row.
+// Partial softmax state of one warp's piece of one row.  Sums are taken
+// relative to an integer reference r in log2 units:
+//   s = sum 2^(z log2(e) - r),  t2 = sum 2^(z log2(e) - r) (z log2(e) - r).
 struct __align__(32) Partial {
-    float m;        // running max (clamped logits)
-    float s;        // sum exp(z - m)
-    float t2;       // sum exp(z - m) * (z - m) * log2(e)   (drafter rows)
+    float m;        // max of the clamped logits of the piece
+    float r;        // integer reference (log2 units), >= m log2(e) up to rounding
+    float t2;       // entropy accumulator (drafter rows)
     int32_t amax;   // lowest index attaining m (INT32_MAX if none)
     int32_t rank;   // saturated count of entries ranked before the drafted token
-    int32_t pad0, pad1, pad2;
+    int32_t pad;
+    double s;
 };
 
 // Final statistics of one row, written by the warp that merges its partials.
 struct __align__(32) RowRec {
+    double lse;     // log sum_v exp(z(v)) in fp64
     float M;        // max of the clamped logits
-    float S;        // sum exp(z - M)
     float g;        // clamped logit of the drafted token (NaN if the row has none)
-    float gap;      // g - M
-    float q;        // drafter rows: exp(g - M) / S
-    float logq;     // drafter rows: (g - M) - ln S
+    float q;        // exp(g - lse)
+    float logq;     // g - lse
     int32_t argmax; // lowest index attaining M, -1 if the row is invalid
     int32_t rank;   // target rows: saturated rank of the drafted token
 };
@@ -183,30 +199,42 @@ __device__ __forceinline__ float philox_uniform(uint64_t seed, uint32_t j, uint3
 enum : uint32_t { kPurposeAccept = 0, kPurposeResid = 1, kPurposeBonus = 2 };
 
 // ---------------------------------------------------------------------------
-// Online-softmax state merge: (m, s, t2) of two disjoint sets of entries.
+// Online-softmax state and its merge.  All rescaling is by exact powers of
+// two (the references are integers), so merging never rounds the scale.
 // ---------------------------------------------------------------------------
 struct SoftState {
-    float m, s, t2;
+    float m, r, t2;
+    double s;
     int32_t amax, rank;
 };
 
+__device__ __forceinline__ SoftState soft_identity() {
+    SoftState z;
+    z.m = clamp_floor();
+    z.r = clamp_ref();
+    z.t2 = 0.f;
+    z.s = 0.0;
+    z.amax = INT32_MAX;
+    z.rank = 0;
+    return z;
+}
+
 __device__ __forceinline__ SoftState soft_merge(SoftState a, SoftState b) {
-    SoftState r;
-    r.m = fmax_nan(a.m, b.m);
-    const float da = (a.m - r.m) * kLog2e, db = (b.m - r.m) * kLog2e;
-    const float sa = (a.m == r.m) ? 1.f : ex2(da);
-    const float sb = (b.m == r.m) ? 1.f : ex2(db);
-    r.s = a.s * sa + b.s * sb;
-    // t2 is relative to m in log2 units: re-basing adds s * (m - M) * log2(e).
-    r.t2 = (a.t2 * sa + (a.s * sa) * da) + (b.t2 * sb + (b.s * sb) * db);
+    SoftState o;
+    o.m = fmax_nan(a.m, b.m);
+    o.r = fmaxf(a.r, b.r);
+    const float ka = a.r - o.r, kb = b.r - o.r;  // integers <= 0
+    // t2 relative to R: 2^k (t2 + k s)
+    o.t2 = pow2f_int(ka) * (a.t2 + ka * static_cast<float>(a.s)) + pow2f_int(kb) * (b.t2 + kb * static_cast<float>(b.s));
+    o.s = a.s * pow2d_int(ka) + b.s * pow2d_int(kb);
     if (b.m > a.m)
-        r.amax = b.amax;
+        o.amax = b.amax;
     else if (b.m < a.m)
-        r.amax = a.amax;
+        o.amax = a.amax;
     else
-        r.amax = min(a.amax, b.amax);
-    r.rank = a.rank + b.rank;
-    return r;
+        o.amax = min(a.amax, b.amax);
+    o.rank = a.rank + b.rank;
+    return o;
 }
 
 __device__ __forceinline__ SoftState soft_warp_reduce(SoftState v) {
@@ -214,8 +242,9 @@ __device__ __forceinline__ SoftState soft_warp_reduce(SoftState v) {
     for (int off = 16; off > 0; off >>= 1) {
         SoftState o;
         o.m = __shfl_xor_sync(0xFFFFFFFFu, v.m, off);
-        o.s = __shfl_xor_sync(0xFFFFFFFFu, v.s, off);
+        o.r = __shfl_xor_sync(0xFFFFFFFFu, v.r, off);
         o.t2 = __shfl_xor_sync(0xFFFFFFFFu, v.t2, off);
+        o.s = __shfl_xor_sync(0xFFFFFFFFu, v.s, off);
         o.amax = __shfl_xor_sync(0xFFFFFFFFu, v.amax, off);
         o.rank = __shfl_xor_sync(0xFFFFFFFFu, v.rank, off);
         // merge in a fixed order (lower lane first) so every lane agrees bitwise

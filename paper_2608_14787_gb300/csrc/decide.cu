@@ -84,17 +84,24 @@ __device__ __forceinline__ float load_logit(const char *rowp, int v) {
 }
 
 // Weights of the sampling draw for the EPV entries of one 16-byte vector.
-//   residual: max(0, p_t(v) - p_d(v)); bonus (zd == nullptr): exp(z_t(v) - M_t).
+//   residual: p_t - p_d = p_d (exp(D(v)) - 1) with the log-ratio
+//             D(v) = (z_t(v) - z_d(v)) - (LSE_t - LSE_d); the LSE difference is
+//             applied as two fp32 terms (hi + lo) and the difference by expm1, so
+//             no cancellation between near-equal p_t and p_d loses precision;
+//             p_d(v) = 2^(z_d(v) log2(e) - r_d) up to the common factor of the row;
+//   bonus (zd_row == nullptr): 2^(z_t(v) log2(e) - r_t).
+// Returns the fp32 sum of the entries in ascending order (the draw and the
+// totals use this same order).
 template <int DT>
-__device__ __forceinline__ double vec_weights(const char *zt_row, const char *zd_row, int vec, int V, float Mt,
-                                              float invSt, float Md, float invSd, float (&w)[8]) {
+__device__ __forceinline__ float vec_weights(const char *zt_row, const char *zd_row, int vec, int V, float nrt,
+                                             float nrd, float d_hi, float d_lo, float (&w)[8]) {
     constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
     const uint4 a = __ldg(reinterpret_cast<const uint4 *>(zt_row) + vec);
     uint4 d = make_uint4(0, 0, 0, 0);
     if (zd_row) d = __ldg(reinterpret_cast<const uint4 *>(zd_row) + vec);
     const uint32_t *ua = reinterpret_cast<const uint32_t *>(&a);
     const uint32_t *ud = reinterpret_cast<const uint32_t *>(&d);
-    double sum = 0.0;
+    float sum = 0.f;
 #pragma unroll
     for (int e = 0; e < EPV; ++e) {
         float zt, zd;
@@ -109,15 +116,14 @@ __device__ __forceinline__ double vec_weights(const char *zt_row, const char *zd
         zd = fmax_nan(zd, clamp_floor());
         float wv;
         if (zd_row) {
-            const float pt = ex2((zt - Mt) * kLog2e) * invSt;
-            const float pd = ex2((zd - Md) * kLog2e) * invSd;
-            wv = fmaxf(pt - pd, 0.f);
+            const float dv = ((zt - zd) - d_hi) - d_lo;
+            wv = (dv > 0.f) ? ex2(fmaf(zd, kLog2e, nrd)) * expm1f(dv) : 0.f;
         } else {
-            wv = ex2((zt - Mt) * kLog2e);
+            wv = ex2(fmaf(zt, kLog2e, nrt));
         }
         if (vec * EPV + e >= V) wv = 0.f;
         w[e] = wv;
-        sum += static_cast<double>(wv);
+        sum += wv;
     }
     return sum;
 }
@@ -144,7 +150,7 @@ __device__ __forceinline__ double block_incl_scan(double v, double *warp_tot, do
 
 struct DrawCtx {
     const char *zt_row, *zd_row;
-    float Mt, invSt, Md, invSd;
+    float nrt, nrd, d_hi, d_lo;
 };
 
 // One pass over vectors [v0, v1) of the draw row.  With find == false returns
@@ -160,11 +166,12 @@ __device__ double draw_pass(const DrawCtx &c, int v0, int v1, int V, bool find, 
     for (int base = v0; base < v1; base += kResidThreads) {
         const int vec = base + threadIdx.x;
         float w[8];
-        double vs = 0.0;
-        if (vec < v1) vs = vec_weights<DT>(c.zt_row, c.zd_row, vec, V, c.Mt, c.invSt, c.Md, c.invSd, w);
+        float vs_f = 0.f;
+        if (vec < v1) vs_f = vec_weights<DT>(c.zt_row, c.zd_row, vec, V, c.nrt, c.nrd, c.d_hi, c.d_lo, w);
         if (vec < v1)
             for (int e = 0; e < EPV; ++e)
                 if (w[e] > 0.f) last_pos = vec * EPV + e;
+        const double vs = static_cast<double>(vs_f);
         double tot;
         const double incl = block_incl_scan(vs, warp_tot, tot);
         if (find) {
@@ -175,12 +182,13 @@ __device__ double draw_pass(const DrawCtx &c, int v0, int v1, int V, bool find, 
             const int tf = *s_first;
             if (tf != INT32_MAX) {
                 if (static_cast<int>(threadIdx.x) == tf) {
-                    double cum = carry + (incl - vs);
+                    const double before = carry + (incl - vs);
+                    float part = 0.f;
                     int pick = -1, lastp = -1;
                     for (int e = 0; e < EPV; ++e) {
                         if (w[e] > 0.f) lastp = vec * EPV + e;
-                        cum += static_cast<double>(w[e]);
-                        if (w[e] > 0.f && cum > target) {
+                        part += w[e];
+                        if (w[e] > 0.f && before + static_cast<double>(part) > target) {
                             pick = vec * EPV + e;
                             break;
                         }
@@ -196,6 +204,24 @@ __device__ double draw_pass(const DrawCtx &c, int v0, int v1, int V, bool find, 
         carry += tot;
     }
     return carry;
+}
+
+// Draw-row context from the two rows' fp64 log-normalisers.
+__device__ __forceinline__ DrawCtx draw_ctx(const char *zt_row, const char *zd_row, double lse_t, double lse_d) {
+    DrawCtx c;
+    c.zt_row = zt_row;
+    c.zd_row = zd_row;
+    c.nrt = -ceilf(static_cast<float>(lse_t * kLog2ed));
+    c.nrd = 0.f;
+    c.d_hi = 0.f;
+    c.d_lo = 0.f;
+    if (zd_row) {
+        c.nrd = -ceilf(static_cast<float>(lse_d * kLog2ed));
+        const double D = lse_t - lse_d;
+        c.d_hi = static_cast<float>(D);
+        c.d_lo = static_cast<float>(D - static_cast<double>(c.d_hi));
+    }
+    return c;
 }
 
 template <int DT>
@@ -215,7 +241,7 @@ __global__ void __launch_bounds__(kResidThreads) decide_kernel(const __grid_cons
     const int32_t *xb = p.tokens + static_cast<int64_t>(b) * gamma;
 
     __shared__ int s_L;              // strict accepted length
-    __shared__ float s_facts[4];     // Mt, St, Md, Sd of the draw row
+    __shared__ double s_lse[2];      // LSE of the target and drafter draw rows
     __shared__ double s_warp[kResidThreads / 32];
     __shared__ int s_first;
     __shared__ double s_tot[kResidMaxSeg];
@@ -233,25 +259,23 @@ __global__ void __launch_bounds__(kResidThreads) decide_kernel(const __grid_cons
                     if (p.greedy) {
                         fail = !(t.rank == 0);
                     } else {
-                        float Md, Sd, gd;
+                        double lse_d;
+                        float gd;
                         if (p.drec) {
                             const RowRec d = p.drec[static_cast<int64_t>(i) * gamma + j];
-                            Md = d.M;
-                            Sd = d.S;
+                            lse_d = d.lse;
                             gd = d.g;
                         } else {
                             const char *zdr = p.zd + (static_cast<int64_t>(b) * gamma + j) * p.stride_bytes;
-                            const int am = __ldg(p.d_argmax + static_cast<int64_t>(b) * gamma + j);
                             const int xj = xb[j];
-                            Sd = 1.f / __ldg(p.d_maxprob + static_cast<int64_t>(b) * gamma + j);
-                            Md = (am >= 0 && am < p.V) ? fmax_nan(load_logit<DT>(zdr, am), clamp_floor()) : nanf_();
+                            lse_d = __ldg(p.d_lse + static_cast<int64_t>(b) * gamma + j);
                             gd = (xj >= 0 && xj < p.V) ? fmax_nan(load_logit<DT>(zdr, xj), clamp_floor()) : nanf_();
                         }
-                        // log p_t(x_j) - log p_d(x_j), both relative to their own row maxima
-                        const float lr = (t.g - t.M) - (gd - Md) - logf(t.S / Sd);
+                        // log r = log p_t(x_j) - log p_d(x_j) = (g_t - g_d) - (LSE_t - LSE_d), in fp64
+                        const double lr = (static_cast<double>(t.g) - static_cast<double>(gd)) - (t.lse - lse_d);
                         const float u = philox_uniform(p.seed, static_cast<uint32_t>(j + 1), static_cast<uint32_t>(b),
                                                        p.round, kPurposeAccept);
-                        const bool acc = (lr >= 0.f) || (u <= expf(lr));
+                        const bool acc = (lr >= 0.0) || (u <= expf(static_cast<float>(lr)));
                         fail = !acc;
                     }
                 }
@@ -283,7 +307,7 @@ __global__ void __launch_bounds__(kResidThreads) decide_kernel(const __grid_cons
                     bool fail = false;
                     if (j < gamma) {
                         const RowRec t = tr[j];
-                        fail = p.ell_one[r] ? !(t.rank == 0) : !(static_cast<double>(t.gap) >= p.ell_thr[r]);
+                        fail = p.ell_one[r] ? !(t.rank == 0) : !(static_cast<double>(t.g - t.M) >= p.ell_thr[r]);
                     }
                     const unsigned bal = __ballot_sync(0xFFFFFFFFu, fail);
                     if (bal) {
@@ -367,33 +391,16 @@ __global__ void __launch_bounds__(kResidThreads) decide_kernel(const __grid_cons
     // ---- sampling: residual (L < gamma) or bonus (L = gamma) inverse-CDF draw ----
     const int L = s_L;
     if (threadIdx.x == 0) {
-        const RowRec t = tr[L];
-        s_facts[0] = t.M;
-        s_facts[1] = t.S;
-        if (L < gamma) {
-            float Md, Sd;
-            if (p.drec) {
-                const RowRec d = p.drec[static_cast<int64_t>(i) * gamma + L];
-                Md = d.M;
-                Sd = d.S;
-            } else {
-                const char *zdr = p.zd + (static_cast<int64_t>(b) * gamma + L) * p.stride_bytes;
-                const int am = __ldg(p.d_argmax + static_cast<int64_t>(b) * gamma + L);
-                Sd = 1.f / __ldg(p.d_maxprob + static_cast<int64_t>(b) * gamma + L);
-                Md = (am >= 0 && am < p.V) ? fmax_nan(load_logit<DT>(zdr, am), clamp_floor()) : nanf_();
-            }
-            s_facts[2] = Md;
-            s_facts[3] = Sd;
-        }
+        s_lse[0] = tr[L].lse;
+        s_lse[1] = 0.0;
+        if (L < gamma)
+            s_lse[1] = p.drec ? p.drec[static_cast<int64_t>(i) * gamma + L].lse
+                              : __ldg(p.d_lse + static_cast<int64_t>(b) * gamma + L);
     }
     __syncthreads();
-    DrawCtx c;
-    c.zt_row = p.zt + (static_cast<int64_t>(b) * (gamma + 1) + L) * p.stride_bytes;
-    c.zd_row = (L < gamma) ? p.zd + (static_cast<int64_t>(b) * gamma + L) * p.stride_bytes : nullptr;
-    c.Mt = s_facts[0];
-    c.invSt = 1.f / s_facts[1];
-    c.Md = (L < gamma) ? s_facts[2] : 0.f;
-    c.invSd = (L < gamma) ? 1.f / s_facts[3] : 0.f;
+    const DrawCtx c = draw_ctx(p.zt + (static_cast<int64_t>(b) * (gamma + 1) + L) * p.stride_bytes,
+                               (L < gamma) ? p.zd + (static_cast<int64_t>(b) * gamma + L) * p.stride_bytes : nullptr,
+                               s_lse[0], s_lse[1]);
     const int v0 = seg * p.seg_vec, v1 = min(p.RV, v0 + p.seg_vec);
     int last_pos, found;
     const double tot = (v0 < v1) ? draw_pass<DT>(c, v0, v1, p.V, false, 0.0, last_pos, found, s_warp, &s_first) : 0.0;

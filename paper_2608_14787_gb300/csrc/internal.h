@@ -36,7 +36,8 @@ struct ScanGroup {
     const int32_t *bidx;     // [nb] batch index of each listed block, or nullptr (= identity)
     RowRec *rec;             // [nb * npos] final records, list order
     // drafter user outputs, indexed (b * gamma + j); any may be nullptr
-    float *q, *logq, *maxprob, *lse, *entropy;
+    float *q, *logq, *maxprob, *entropy;
+    double *lse;
     int32_t *argmax;
 };
 
@@ -70,8 +71,7 @@ struct DecideParams {
     const int32_t *tokens;         // [B, gamma]
     const RowRec *trec;            // [nb, gamma+1] list order
     const RowRec *drec;            // [nb, gamma] list order, or nullptr
-    const float *d_maxprob;        // [B, gamma] user arrays when drec == nullptr
-    const int32_t *d_argmax;
+    const double *d_lse;           // [B, gamma] drafter LSE (user array) when drec == nullptr
     // strict
     int32_t do_strict, greedy;
     uint64_t seed, round;

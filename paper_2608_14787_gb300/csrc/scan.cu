@@ -79,114 +79,152 @@ __device__ __forceinline__ void mask_tail(uint4 &w, int valid) {
 }
 
 template <int DT>
-__device__ __forceinline__ float elem(const uint4 (&w)[kVPL], int i, int e) {
-    const uint32_t *u = reinterpret_cast<const uint32_t *>(&w[i]);
+__device__ __forceinline__ float vec_elem(const uint4 &w, int e) {
+    const uint32_t *u = reinterpret_cast<const uint32_t *>(&w);
     if (DT == SDD_BF16) return (e & 1) ? bf16_hi(u[e >> 1]) : bf16_lo(u[e >> 1]);
     return __uint_as_float(u[e]);
 }
 
-// Process one tile: the lane's vectors are lane, lane+32, ... of the tile.
-template <int DT, bool kTarget>
-__device__ __forceinline__ void process_tile(const uint4 *tile, int n, int k0, int lane, int tail, bool row_end,
-                                             SoftState &st, float g, int tok, int kcap) {
-    constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
-    uint4 w[kVPL];
+// Clamp one vector from below (NaN-propagating).
+template <int DT>
+__device__ __forceinline__ uint4 clamp_vec(uint4 w) {
+    uint32_t *u = reinterpret_cast<uint32_t *>(&w);
+    if (DT == SDD_BF16) {
 #pragma unroll
+        for (int q = 0; q < 4; ++q) u[q] = bf16x2_max_nan(u[q], kClampPairBf16);
+    } else {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) u[q] = __float_as_uint(fmax_nan(__uint_as_float(u[q]), clamp_floor()));
+    }
+    return w;
+}
+
+// A tile that is not full, or that ends a row whose length is not a whole
+// number of vectors, is completed in shared memory with -inf entries so that
+// the hot loop can read every vector of the tile unconditionally.
+template <int DT>
+__device__ __noinline__ void pad_tile(uint4 *tile, int n, int lane, bool row_end, int tail) {
+    const uint4 ninf = (DT == SDD_BF16) ? make_uint4(kNegInfPairBf16, kNegInfPairBf16, kNegInfPairBf16, kNegInfPairBf16)
+                                        : make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u);
+    for (int idx = n + lane; idx < kTileVec; idx += 32) tile[idx] = ninf;
+    if (row_end && tail && lane == ((n - 1) & 31)) {
+        uint4 w = tile[n - 1];
+        mask_tail<DT>(w, tail);
+        tile[n - 1] = w;
+    }
+    __syncwarp();
+}
+
+// Entries of the lane's vectors in a (full, padded) tile that rank before the
+// drafted token tok: value above g, or equal to g at a lower index.
+template <int DT>
+__device__ __noinline__ int count_before(const uint4 *tile, int n, int k0, int lane, float g, int tok) {
+    constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
+    int cnt = 0;
+#pragma unroll 1
     for (int i = 0; i < kVPL; ++i) {
         const int idx = lane + 32 * i;
-        if (idx < n) {
-            w[i] = tile[idx];
-            if (row_end && tail && idx == n - 1) mask_tail<DT>(w[i], tail);
-        } else {
-            w[i] = make_uint4(kNegInfPairBf16, kNegInfPairBf16, kNegInfPairBf16, kNegInfPairBf16);
-            if (DT != SDD_BF16) w[i] = make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u);
+        if (idx >= n) break;
+        const uint4 w = clamp_vec<DT>(tile[idx]);
+#pragma unroll
+        for (int e = 0; e < EPV; ++e) {
+            const float z = vec_elem<DT>(w, e);
+            const int v = (k0 + idx) * EPV + e;
+            cnt += (z > g || (z == g && v < tok)) ? 1 : 0;
         }
     }
-    // clamp from below (NaN-propagating) and take the tile maximum
+    return cnt;
+}
+
+// Resolve a lane's argmax: the first of its entries equal to m inside the tile
+// that starts at vector k0 of the row (re-read from global memory; the row's
+// padding and entries past V are excluded).
+template <int DT>
+__device__ __noinline__ int first_index(const char *rowp, int k0, int lane, int RV, int V, float m) {
+    constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
+#pragma unroll 1
+    for (int i = 0; i < kVPL; ++i) {
+        const int vec = k0 + lane + 32 * i;
+        if (vec >= RV) break;
+        const uint4 w = clamp_vec<DT>(__ldg(reinterpret_cast<const uint4 *>(rowp) + vec));
+#pragma unroll
+        for (int e = 0; e < EPV; ++e)
+            if (vec * EPV + e < V && vec_elem<DT>(w, e) == m) return vec * EPV + e;
+    }
+    return INT32_MAX;
+}
+
+// Process one full tile: the lane's vectors are lane, lane+32, ... of the tile.
+// Sums are relative to the integer reference st.r (log2 units), so a new
+// maximum rescales by an exact power of two.  A new maximum only records the
+// tile (st.amax = k0); the exact index is resolved once at the end of the piece.
+template <int DT>
+__device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lane, SoftState &st) {
+    uint4 w[kVPL];
+#pragma unroll
+    for (int i = 0; i < kVPL; ++i) w[i] = clamp_vec<DT>(tile[lane + 32 * i]);
     float cm;
     if (DT == SDD_BF16) {
         uint32_t mx = kClampPairBf16;
 #pragma unroll
         for (int i = 0; i < kVPL; ++i) {
-            uint32_t *u = reinterpret_cast<uint32_t *>(&w[i]);
+            const uint32_t *u = reinterpret_cast<const uint32_t *>(&w[i]);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                u[q] = bf16x2_max_nan(u[q], kClampPairBf16);
-                mx = bf16x2_max_nan(mx, u[q]);
-            }
+            for (int q = 0; q < 4; ++q) mx = bf16x2_max_nan(mx, u[q]);
         }
         cm = fmax_nan(bf16_lo(mx), bf16_hi(mx));
     } else {
-        const float fl = clamp_floor();
-        cm = fl;
+        cm = clamp_floor();
 #pragma unroll
         for (int i = 0; i < kVPL; ++i) {
-            float *f = reinterpret_cast<float *>(&w[i]);
+            const float *f = reinterpret_cast<const float *>(&w[i]);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                f[q] = fmax_nan(f[q], fl);
-                cm = fmax_nan(cm, f[q]);
-            }
+            for (int q = 0; q < 4; ++q) cm = fmax_nan(cm, f[q]);
         }
     }
-    // a new running maximum: rescale and locate its first occurrence
     if (cm > st.m) {
-        const float d = (st.m - cm) * kLog2e;
-        const float sc = ex2(d);
-        st.t2 = st.t2 * sc + (st.s * sc) * d;
-        st.s *= sc;
+        st.amax = k0;
         st.m = cm;
-        int found = INT32_MAX;
-#pragma unroll
-        for (int i = 0; i < kVPL; ++i)
-#pragma unroll
-            for (int e = 0; e < EPV; ++e)
-                if (found == INT32_MAX && elem<DT>(w, i, e) == cm) found = (k0 + lane + 32 * i) * EPV + e;
-        st.amax = found;
+        const float rn = ceilf(cm * kLog2e);
+        if (rn > st.r) {
+            const float k = st.r - rn;
+            st.t2 = pow2f_int(k) * (st.t2 + k * static_cast<float>(st.s));
+            st.s *= pow2d_int(k);
+            st.r = rn;
+        }
     }
-    // exp-sum (and entropy accumulator for drafter rows) on packed fp32 pairs
-    const f2_t m2 = f2_pack(st.m, st.m);
-    const f2_t l2 = f2_pack(kLog2e, kLog2e);
-    f2_t as = 0ull, at = 0ull;
+    // y = z log2(e) - r; s += 2^y; t2 += 2^y y   (two accumulators each)
+    const float nr = -st.r;
+    float s0 = 0.f, s1 = 0.f, t0 = 0.f, t1 = 0.f;
 #pragma unroll
     for (int i = 0; i < kVPL; ++i) {
         const uint32_t *u = reinterpret_cast<const uint32_t *>(&w[i]);
 #pragma unroll
-        for (int q = 0; q < (DT == SDD_BF16 ? 4 : 2); ++q) {
-            f2_t z2;
-            if (DT == SDD_BF16)
-                z2 = f2_pack(bf16_lo(u[q]), bf16_hi(u[q]));
-            else
-                z2 = f2_pack(__uint_as_float(u[2 * q]), __uint_as_float(u[2 * q + 1]));
-            const f2_t y2 = f2_mul(f2_sub(z2, m2), l2);
-            float y0, y1;
-            f2_unpack(y2, y0, y1);
-            const f2_t e2 = f2_pack(ex2(y0), ex2(y1));
-            as = f2_add(as, e2);
-            if (!kTarget) at = f2_fma(e2, y2, at);
+        for (int q = 0; q < 4; ++q) {
+            if (DT == SDD_BF16) {
+                const float y0 = fmaf(bf16_lo(u[q]), kLog2e, nr);
+                const float y1 = fmaf(bf16_hi(u[q]), kLog2e, nr);
+                const float e0 = ex2(y0), e1 = ex2(y1);
+                s0 += e0;
+                t0 = fmaf(e0, y0, t0);
+                s1 += e1;
+                t1 = fmaf(e1, y1, t1);
+            } else {
+                const float y0 = fmaf(__uint_as_float(u[q]), kLog2e, nr);
+                const float e0 = ex2(y0);
+                if (q & 1) {
+                    s1 += e0;
+                    t1 = fmaf(e0, y0, t1);
+                } else {
+                    s0 += e0;
+                    t0 = fmaf(e0, y0, t0);
+                }
+            }
         }
     }
-    float a0, a1;
-    f2_unpack(as, a0, a1);
-    st.s += a0 + a1;
-    if (!kTarget) {
-        f2_unpack(at, a0, a1);
-        st.t2 += a0 + a1;
-    }
-    // rank of the drafted token (target rows): only tiles that can hold an
-    // entry >= g are inspected, and a lane stops once its count reaches kcap
-    if (kTarget && tok >= 0 && cm >= g && st.rank < kcap) {
-        int cnt = 0;
-#pragma unroll
-        for (int i = 0; i < kVPL; ++i)
-#pragma unroll
-            for (int e = 0; e < EPV; ++e) {
-                const float z = elem<DT>(w, i, e);
-                const int idx = (k0 + lane + 32 * i) * EPV + e;
-                cnt += (z > g || (z == g && idx < tok)) ? 1 : 0;
-            }
-        st.rank += cnt;
-    }
+    st.s += static_cast<double>(s0) + static_cast<double>(s1);
+    st.t2 += t0 + t1;
+    return cm;
 }
 
 // Final results of row r from its merged state (whole warp calls; lane 0 writes).
@@ -201,48 +239,57 @@ __device__ void finalize_row(const ScanParams &p, int64_t r, SoftState st, int l
     const bool has_tok = j < p.gamma;
     int tok = has_tok ? __ldg(p.tokens + static_cast<int64_t>(b) * p.gamma + j) : -1;
     const bool tok_ok = has_tok && tok >= 0 && tok < p.V;
-    const bool valid = b_ok && isfinite(st.m) && st.m > clamp_floor() && isfinite(st.s) && st.s > 0.f;
+    const bool valid = b_ok && isfinite(st.m) && st.m > clamp_floor() && isfinite(st.s) && st.s > 0.0;
     if (lane != 0) return;
-    float g = __int_as_float(0x7FC00000);
+    const float nanf_ = __int_as_float(0x7FC00000);
+    float g = nanf_;
     if (tok_ok) g = fmax_nan(load_logit<DT>(rowp, tok), clamp_floor());
     RowRec rec;
-    const float nanf_ = __int_as_float(0x7FC00000);
+    const int64_t o = static_cast<int64_t>(b) * p.gamma + j;
     if (valid) {
-        const float lnS = logf(st.s);
+        // The lane that held the row maximum M took its term as ex2(y_M) with
+        // y_M = M log2(e) - ceil(M log2(e)) (its reference when M arrived).  On a
+        // peaked row that one term dominates S, so its MUFU approximation error
+        // is replaced by the exact power of two (scaled to the final reference).
+        const float rM = ceilf(st.m * kLog2e);
+        const float yM = fmaf(st.m, kLog2e, -rM);
+        const double S = st.s + (exp2(static_cast<double>(yM)) - static_cast<double>(ex2(yM))) * pow2d_int(rM - st.r);
+        st.s = S;
+        // all in fp64: LSE = r ln2 + ln S (S relative to the reference r)
+        const double lnS = log(st.s);
+        const double lse = static_cast<double>(st.r) * kLn2d + lnS;
+        rec.lse = lse;
         rec.M = st.m;
-        rec.S = st.s;
         rec.g = g;
-        rec.gap = g - st.m;
-        rec.q = ex2((g - st.m) * kLog2e) / st.s;
-        rec.logq = (g - st.m) - lnS;
+        rec.logq = static_cast<float>(static_cast<double>(g) - lse);
+        rec.q = static_cast<float>(exp(static_cast<double>(g) - lse));
         rec.argmax = st.amax;
         rec.rank = min(st.rank, p.kcap);
         if (G.kind == 0 && b_ok) {
-            const int64_t o = static_cast<int64_t>(b) * p.gamma + j;
             if (G.q) G.q[o] = tok_ok ? rec.q : nanf_;
             if (G.logq) G.logq[o] = tok_ok ? rec.logq : nanf_;
-            if (G.maxprob) G.maxprob[o] = 1.f / st.s;
-            if (G.lse) G.lse[o] = st.m + lnS;
-            if (G.entropy) G.entropy[o] = lnS - (st.t2 * kLn2) / st.s;
+            if (G.maxprob) G.maxprob[o] = static_cast<float>(exp(static_cast<double>(st.m) - lse));
+            if (G.lse) G.lse[o] = lse;
+            if (G.entropy) G.entropy[o] = static_cast<float>(lnS - kLn2d * static_cast<double>(st.t2) / st.s);
             if (G.argmax) G.argmax[o] = st.amax;
         }
     } else {
-        rec.M = rec.S = rec.g = rec.gap = rec.q = rec.logq = nanf_;
+        rec.lse = __longlong_as_double(0x7FF8000000000000ll);
+        rec.M = rec.g = rec.q = rec.logq = nanf_;
         rec.argmax = -1;
         rec.rank = INT32_MAX;
         if (G.kind == 0 && b_ok) {
-            const int64_t o = static_cast<int64_t>(b) * p.gamma + j;
             if (G.q) G.q[o] = nanf_;
             if (G.logq) G.logq[o] = nanf_;
             if (G.maxprob) G.maxprob[o] = nanf_;
-            if (G.lse) G.lse[o] = nanf_;
+            if (G.lse) G.lse[o] = rec.lse;
             if (G.entropy) G.entropy[o] = nanf_;
             if (G.argmax) G.argmax[o] = -1;
         }
         if (b_ok) status_or(p.status, SDD_DEV_NONFINITE);
     }
     if (has_tok && !tok_ok) {
-        rec.q = rec.logq = rec.g = rec.gap = nanf_;
+        rec.q = rec.logq = rec.g = nanf_;
         rec.rank = INT32_MAX;
     }
     if ((has_tok && !tok_ok) || !b_ok) status_or(p.status, SDD_DEV_BAD_TOKEN);
@@ -278,7 +325,8 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
     auto issue = [&](int slot) {
         const int n = static_cast<int>(min(static_cast<int64_t>(min(kTileVec, p.RV - pc.k)), v1 - pc.v));
         if (lane == 0) {
-            fence_proxy_async_smem();
+            // the slot's previous contents were consumed into registers before the
+            // warp reached this point (__syncwarp), so the copy may overwrite it
             mbar_arrive_expect_tx(&bars[slot], static_cast<uint32_t>(n) * 16u);
             bulk_g2s(ring + slot * kTileBytes, prow + static_cast<int64_t>(pc.k) * 16, static_cast<uint32_t>(n) * 16u,
                      &bars[slot]);
@@ -294,58 +342,74 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
     };
     for (int s = 0; s < kStages && pc.v < v1; ++s) issue(s);
 
-    SoftState st;
+    SoftState st = soft_identity();
     bool in_piece = false;
-    int kind = 0, tok = -1;
-    float g = 0.f;
+    int tok = -1;          // drafted token of the current target row (-1: none)
+    float g = 0.f;         // its clamped logit
+    bool rank_on = false;  // warp-uniform: the rank of tok is still below kcap
+    int wrank = 0;         // warp-uniform running rank count
+    const char *crow = nullptr;
     int slot = 0;
     bool timed_out = false;
     while (cc.v < v1) {
         const int n = static_cast<int>(min(static_cast<int64_t>(min(kTileVec, p.RV - cc.k)), v1 - cc.v));
         if (!in_piece) {
-            st.m = clamp_floor();
-            st.s = 0.f;
-            st.t2 = 0.f;
-            st.amax = INT32_MAX;
-            st.rank = 0;
+            st = soft_identity();
             int gi, j, b;
             int64_t lr;
             bool ok;
             row_locate(p, cc.r, gi, lr, j, b, ok);
-            kind = p.grp[gi].kind;
+            const ScanGroup &G = p.grp[gi];
+            crow = G.base + (static_cast<int64_t>(b) * G.npos + j) * G.stride_bytes;
             tok = -1;
             g = 0.f;
-            if (kind == 1 && j < p.gamma) {
-                tok = __ldg(p.tokens + static_cast<int64_t>(b) * p.gamma + j);
-                if (tok >= 0 && tok < p.V) {
-                    const char *rowp = p.grp[gi].base + (static_cast<int64_t>(b) * p.grp[gi].npos + j) *
-                                                            p.grp[gi].stride_bytes;
-                    g = fmax_nan(load_logit<DT>(rowp, tok), clamp_floor());
-                } else {
-                    tok = -1;
+            if (G.kind == 1 && j < p.gamma) {
+                const int t = __ldg(p.tokens + static_cast<int64_t>(b) * p.gamma + j);
+                if (t >= 0 && t < p.V) {
+                    tok = t;
+                    g = fmax_nan(load_logit<DT>(crow, t), clamp_floor());
                 }
             }
+            rank_on = tok >= 0;
+            wrank = 0;
             in_piece = true;
         }
         if (!mbar_wait_bounded(&bars[slot], (phase >> slot) & 1u, kWaitPolls)) {
             timed_out = true;
             break;
         }
-        const uint4 *tile = reinterpret_cast<const uint4 *>(ring + slot * kTileBytes);
+        uint4 *tile = reinterpret_cast<uint4 *>(ring + slot * kTileBytes);
         const bool row_end = (cc.k + n == p.RV);
-        if (kind == 1)
-            process_tile<DT, true>(tile, n, cc.k, lane, tail, row_end, st, g, tok, p.kcap);
-        else
-            process_tile<DT, false>(tile, n, cc.k, lane, tail, row_end, st, g, tok, p.kcap);
+        if (n < kTileVec || (row_end && tail)) pad_tile<DT>(tile, n, lane, row_end, tail);
+        const float cm = process_tile<DT>(tile, cc.k, lane, st);
+        if (rank_on) {
+            const bool want = cm >= g;
+            if (__any_sync(0xFFFFFFFFu, want)) {
+                int c = want ? count_before<DT>(tile, n, cc.k, lane, g, tok) : 0;
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1) c += __shfl_xor_sync(0xFFFFFFFFu, c, off);
+                wrank += c;
+                if (wrank >= p.kcap) rank_on = false;
+            }
+        }
         __syncwarp();
         phase ^= 1u << slot;
         pending &= ~(1u << slot);
+        if (n < kTileVec || (row_end && tail)) fence_proxy_async_smem();  // generic writes of pad_tile
         if (pc.v < v1) issue(slot);
         slot = (slot + 1 == kStages) ? 0 : slot + 1;
         cc.v += n;
         cc.k += n;
         if (row_end || cc.v == v1) {
-            // end of this warp's piece of row cc.r
+            // end of this warp's piece of row cc.r: exact argmax of the piece,
+            // then the warp's partial state
+            float M = st.m;
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) M = fmax_nan(M, __shfl_xor_sync(0xFFFFFFFFu, M, off));
+            int idx = INT32_MAX;
+            if (st.m == M && st.amax != INT32_MAX) idx = first_index<DT>(crow, st.amax, lane, p.RV, p.V, M);
+            st.amax = idx;
+            st.rank = (lane == 0) ? wrank : 0;
             SoftState red = soft_warp_reduce(st);
             const int64_t fw = part_owner(cc.r * p.RV, p.T, p.W);
             const int64_t lw = part_owner((cc.r + 1) * p.RV - 1, p.T, p.W);
@@ -355,11 +419,12 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
                 if (lane == 0) {
                     Partial pt;
                     pt.m = red.m;
-                    pt.s = red.s;
+                    pt.r = red.r;
                     pt.t2 = red.t2;
                     pt.amax = red.amax;
                     pt.rank = red.rank;
-                    pt.pad0 = pt.pad1 = pt.pad2 = 0;
+                    pt.pad = 0;
+                    pt.s = red.s;
                     p.partials[cc.r + gw] = pt;
                 }
                 uint32_t old = 0;
@@ -370,18 +435,14 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
                 old = __shfl_sync(0xFFFFFFFFu, old, 0);
                 if (old == static_cast<uint32_t>(lw - fw)) {
                     __threadfence();
-                    SoftState acc;
-                    acc.m = clamp_floor();
-                    acc.s = 0.f;
-                    acc.t2 = 0.f;
-                    acc.amax = INT32_MAX;
-                    acc.rank = 0;
+                    SoftState acc = soft_identity();
                     for (int64_t w = fw + lane; w <= lw; w += 32) {
                         const Partial *pp = p.partials + cc.r + w;
                         SoftState o;
                         o.m = __ldcg(&pp->m);
-                        o.s = __ldcg(&pp->s);
+                        o.r = __ldcg(&pp->r);
                         o.t2 = __ldcg(&pp->t2);
+                        o.s = __ldcg(&pp->s);
                         o.amax = __ldcg(&pp->amax);
                         o.rank = __ldcg(&pp->rank);
                         acc = soft_merge(acc, o);

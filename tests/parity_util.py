@@ -85,24 +85,27 @@ class OracleBlock:
 
 def oracle_block(z_d, z_t, x, *, seed=0, round_=0, pairs=(), signal=0, K_min=6, S_max=64, D_in=None,
                  ells=(), ks=(), blocks=None, sampling=True, guard=None, force_strict=None) -> OracleBlock:
-    """Run the oracle on blocks `blocks` (default all) of the batch."""
-    zd, zt, xx = host(z_d), host(z_t), x.detach().cpu().numpy().astype(np.int32)
-    B = xx.shape[0]
+    """Run the oracle on blocks `blocks` (default all) of the batch.  The
+    tensors always hold the whole batch, so that each block keeps its batch
+    index b (its Philox stream)."""
+    B = x.shape[0]
     blocks = list(range(B)) if blocks is None else list(blocks)
-    st = orc.row_stats(zd[blocks], tokens=xx[blocks])
+    zd, zt = host(z_d[blocks]), host(z_t[blocks])
+    xx = x[blocks].detach().cpu().numpy().astype(np.int32)
+    st = orc.row_stats(zd, tokens=xx)
     facts, strict, greedy = [], [], []
     lenient = {e: [] for e in ells}
     topk = {k: [] for k in ks}
-    for b in blocks:
-        f = orc.target_facts(zt[b], xx[b])
+    for i, b in enumerate(blocks):
+        f = orc.target_facts(zt[i], xx[i])
         facts.append(f)
-        greedy.append(orc.verify_greedy(f, xx[b]))
+        greedy.append(orc.verify_greedy(f, xx[i]))
         if sampling:
-            strict.append(orc.verify_strict(zt[b], zd[b], xx[b], seed=seed, b=b, round_=round_))
+            strict.append(orc.verify_strict(zt[i], zd[i], xx[i], seed=seed, b=b, round_=round_))
         for e in ells:
-            lenient[e].append(orc.verify_lenient(f, xx[b], e))
+            lenient[e].append(orc.verify_lenient(f, xx[i], e))
         for k in ks:
-            topk[k].append(orc.verify_topk(f, xx[b], k))
+            topk[k].append(orc.verify_topk(f, xx[i], k))
     sched = {}
     D = None if D_in is None else np.asarray(D_in)[blocks]
     g = None if guard is None else np.asarray(guard)[blocks]

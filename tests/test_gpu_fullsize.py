@@ -27,7 +27,7 @@ def _round(wl_name, blocks=None, greedy=False):
     torch.cuda.synchronize()
     assert int(rnd.status.item()) == 0
     blocks = list(range(wl.B)) if blocks is None else blocks
-    ob = oracle_block(blk.z_d[blocks], blk.z_t[blocks], blk.x[blocks], seed=wl.seed, round_=0,
+    ob = oracle_block(blk.z_d, blk.z_t, blk.x, blocks=blocks, seed=wl.seed, round_=0,
                       pairs=[(t, t) for t in wl.taus], ells=ells, ks=ks, sampling=not greedy)
     return wl, ells, ks, blk, rnd, ob, blocks
 

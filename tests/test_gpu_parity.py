@@ -271,3 +271,25 @@ def test_block_round_vs_oracle(sdd, greedy):
     print("block round", tally)
     # tau = 1 reproduces Strict SDD with zero skips
     assert torch.all(rnd.K[3] == 0)
+
+
+@pytest.mark.parametrize("sigma", [0.2, 0.05, 0.01])
+def test_strict_sampling_small_residuals(sdd, sigma):
+    """Target = drafter + N(0, sigma): p_t is close to p_d, so the residual mass
+    R of a rejection is small and made of nearly cancelling terms (on peaked
+    positions R is of order 1e-4).  The draws must still match the oracle."""
+    B, gamma, V = 24, 12, 30000
+    blk = synth.make_block("c3", device="cpu", B=B, gamma=gamma, V=V)
+    g = torch.Generator().manual_seed(int(sigma * 10000))
+    zt = blk.z_t.float().clone()
+    zt[:, :gamma] = blk.z_d.float() + sigma * torch.randn(B, gamma, V, generator=g)
+    z_t = zt.to(torch.bfloat16).contiguous().to(DEV)
+    z_d, x = blk.z_d.to(DEV), blk.x.to(DEV)
+    draft = sdd.confidence(z_d, x)
+    tally = Tally()
+    for rnd in range(3):
+        L, tok, _ = sdd.verify_strict(z_t, x, z_d=z_d, draft=draft, seed=17, round_=rnd)
+        torch.cuda.synchronize()
+        ob = oracle_block(z_d, z_t, x, seed=17, round_=rnd)
+        compare_rule(tally, f"strict sigma={sigma} round {rnd}", L, tok, ob.strict, list(range(B)))
+    print("small residuals", sigma, tally)
