@@ -235,6 +235,31 @@ SDD_API sdd_status_t sdd_uniforms(uint64_t seed, const uint32_t *j, const uint32
                                   const uint32_t *purpose, int64_t n, float *u, sdd_stream_t stream);
 
 /*
+ * sdd_confidence_noalloc -- sdd_confidence without a workspace, for callers
+ * that cannot allocate device memory where they need the statistics: code
+ * running inside CUDA stream capture (where cudaMalloc is not allowed),
+ * programs whose device memory is a fixed arena owned by a framework, or host
+ * loops that have no allocator at hand.  The paper has no counterpart; this is
+ * a deployment convenience.
+ * Same arguments, outputs, status bits and results as sdd_confidence, minus
+ * the workspace.  The scratch is one file-scope device array of 672 KiB that
+ * every GPU loading this library holds until the process exits; it serves
+ * B * gamma <= 8192 drafter rows per call (larger batches are rejected with
+ * SDD_ERR_INVALID_ARGUMENT before anything is enqueued).  The first call on a
+ * device looks up the array's device address and the launch geometry for that
+ * device (make that first call, on each device, before any stream capture).
+ * Every call clears the arrival counters it needs on `stream`, then runs the
+ * same streaming kernel as sdd_confidence.  All calls share the one array, so
+ * calls that may overlap on the GPU (different streams, or host threads without
+ * ordering between them) race on it: order them on one stream.  No allocating
+ * routine is called.
+ */
+SDD_API sdd_status_t sdd_confidence_noalloc(const void *draft_logits, sdd_dtype_t dtype, int B, int gamma, int V,
+                                            int64_t row_stride, const int32_t *draft_tokens, float *q, float *logq,
+                                            float *maxprob, double *lse, float *entropy, int32_t *argmax,
+                                            int32_t *status, sdd_stream_t stream);
+
+/*
  * sdd_block -- one round of the whole path over B blocks, fused so that every
  * drafter and target logit is read once: confidence (sdd_confidence), the skip
  * schedule for n_tau pairs (sdd_schedule_prefix), strict verification of every

@@ -84,6 +84,8 @@ def load(path: str | None = None):
     L.sdd_agreement.argtypes = [VP, VP, I, I, VP, VP]
     L.sdd_commit.argtypes = [VP, VP, VP, VP, I, I, VP, VP, VP]
     L.sdd_uniforms.argtypes = [u64, VP, VP, VP, VP, i64, VP, VP]
+    L.sdd_confidence_noalloc.argtypes = [VP, I, I, I, I, i64, VP, VP, VP, VP, VP, VP, VP, VP, VP]
+    L.sdd_confidence_noalloc.restype = I
     for fn in ("sdd_block", "sdd_block_scan", "sdd_block_decide"):
         getattr(L, fn).argtypes = [ctypes.POINTER(BlockArgs), VP]
     for fn in ("sdd_workspace_size", "sdd_confidence", "sdd_schedule_prefix", "sdd_verify_strict",
@@ -185,6 +187,23 @@ def confidence(z_d: torch.Tensor, x: torch.Tensor, ws: Workspace | None = None, 
                                _p(out.maxprob), _p(out.lse), _p(out.entropy), _p(out.argmax), ws.ptr, ws.nbytes,
                                _p(status), _stream(stream))
     _check(rc, "sdd_confidence")
+    return out
+
+
+def confidence_noalloc(z_d: torch.Tensor, x: torch.Tensor, status=None, stream=None) -> Confidence:
+    """sdd_confidence_noalloc: the same statistics as confidence() with the
+    library's fixed scratch instead of a workspace (B * gamma <= 8192)."""
+    B, gamma = x.shape
+    V, stride = _logits_layout(z_d, "z_d")
+    dev = z_d.device
+    status = new_status(dev) if status is None else status
+    f32 = lambda: torch.empty(B, gamma, dtype=torch.float32, device=dev)  # noqa: E731
+    out = Confidence(q=f32(), logq=f32(), maxprob=f32(), lse=torch.empty(B, gamma, dtype=torch.float64, device=dev),
+                     entropy=f32(), argmax=torch.empty(B, gamma, dtype=torch.int32, device=dev))
+    rc = load().sdd_confidence_noalloc(_p(z_d), _dtype_code(z_d), B, gamma, V, stride, _p(x), _p(out.q),
+                                       _p(out.logq), _p(out.maxprob), _p(out.lse), _p(out.entropy), _p(out.argmax),
+                                       _p(status), _stream(stream))
+    _check(rc, "sdd_confidence_noalloc")
     return out
 
 

@@ -274,6 +274,9 @@ sdd_status_t target_scan(const Work &w, const void *target_logits, sdd_dtype_t d
 }
 
 }  // namespace
+
+void set_last_error(const char *msg) { g_err = msg; }
+
 }  // namespace sdd
 
 using namespace sdd;

@@ -125,6 +125,7 @@ cudaError_t launch_commit(const int32_t *K, const int32_t *x, const int32_t *vt,
 cudaError_t launch_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, const uint64_t *round,
                             const uint32_t *purpose, int64_t n, float *u, cudaStream_t stream);
 int scan_max_ctas_per_sm();
+void set_last_error(const char *msg);  // message returned by sdd_last_error()
 cudaError_t scan_prepare_device();
 
 // Index arithmetic of the balanced contiguous partition of T vectors over W
