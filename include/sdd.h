@@ -268,8 +268,11 @@ SDD_API sdd_status_t sdd_confidence_noalloc(const void *draft_logits, sdd_dtype_
  * read, agreement counters for every pair, and the tokens committed under pair
  * 0.  Array meanings and layouts are those of the single-purpose calls; NULL
  * output pointers are skipped.  sdd_block runs sdd_block_scan then
- * sdd_block_decide on the same stream; the two halves are exported so that a
- * caller can time the streaming pass on its own.
+ * sdd_block_decide on the same stream.  sdd_block_scan streams every logit
+ * once and, as each block's last row completes, evaluates that block's rules,
+ * schedule, agreement counters and skip commits; sdd_block_decide completes the
+ * sampling rule's residual / bonus draws (nothing to do when greedy != 0).  The
+ * two halves are exported so that a caller can time the streaming pass alone.
  */
 typedef struct sdd_block_args {
     /* inputs */

@@ -64,29 +64,28 @@ inline size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255);
 
 // Workspace layout for blocks of shape (B, gamma) on a device with W_max warps.
 struct Layout {
-    size_t partials, counters, drec, trec, res_total, res_last, res_count, k0, total;
+    size_t partials, counters, drec, trec, res_total, res_last, res_count, k0, blk_count, blk_L, total;
 };
 
 Layout layout(int64_t B, int64_t gamma, int64_t W_max) {
     Layout L{};
     const int64_t rows = B * (2 * gamma + 1);
     size_t o = 0;
-    L.partials = o;
-    o = align256(o + static_cast<size_t>(rows + W_max) * sizeof(Partial));
-    L.counters = o;
-    o = align256(o + static_cast<size_t>(rows) * sizeof(uint32_t));
-    L.drec = o;
-    o = align256(o + static_cast<size_t>(B * gamma) * sizeof(RowRec));
-    L.trec = o;
-    o = align256(o + static_cast<size_t>(B * (gamma + 1)) * sizeof(RowRec));
-    L.res_total = o;
-    o = align256(o + static_cast<size_t>(B * kResidMaxSeg) * sizeof(double));
-    L.res_last = o;
-    o = align256(o + static_cast<size_t>(B * kResidMaxSeg) * sizeof(int32_t));
-    L.res_count = o;
-    o = align256(o + static_cast<size_t>(B) * sizeof(uint32_t));
-    L.k0 = o;
-    o = align256(o + static_cast<size_t>(B) * sizeof(int32_t));
+    auto take = [&](size_t bytes) {
+        const size_t at = o;
+        o = align256(o + bytes);
+        return at;
+    };
+    L.partials = take(static_cast<size_t>(rows + W_max) * sizeof(Partial));
+    L.counters = take(static_cast<size_t>(rows) * sizeof(uint32_t));
+    L.drec = take(static_cast<size_t>(B * gamma) * sizeof(RowRec));
+    L.trec = take(static_cast<size_t>(B * (gamma + 1)) * sizeof(RowRec));
+    L.res_total = take(static_cast<size_t>(B * kDrawMaxSeg) * sizeof(double));
+    L.res_last = take(static_cast<size_t>(B * kDrawMaxSeg) * sizeof(int32_t));
+    L.res_count = take(static_cast<size_t>(B) * sizeof(uint32_t));
+    L.k0 = take(static_cast<size_t>(B) * sizeof(int32_t));
+    L.blk_count = take(static_cast<size_t>(B) * sizeof(uint32_t));
+    L.blk_L = take(static_cast<size_t>(B) * sizeof(int32_t));
     L.total = o;
     return L;
 }
@@ -165,36 +164,45 @@ sdd_status_t run_scan(ScanParams &p, const Work &w, cudaStream_t stream) {
     return SDD_OK;
 }
 
-void init_decide(DecideParams &d, const Work &w, sdd_dtype_t dtype, int B, int gamma, int V, int64_t row_stride,
-                 const int32_t *tokens, int32_t *status) {
-    std::memset(&d, 0, sizeof d);
+// Block decisions evaluated inside the streaming kernel.
+void init_dec(DecideParams &d, const Work &w, sdd_dtype_t dtype, int B, int gamma, int V, int64_t row_stride,
+              const int32_t *tokens, int rows_per_block) {
+    d.enabled = 1;
+    d.rows_per_block = rows_per_block;
     d.B = B;
     d.gamma = gamma;
     d.V = V;
-    d.RV = static_cast<int32_t>((static_cast<int64_t>(V) * esize(dtype) + 15) / 16);
-    d.dtype = dtype;
     d.stride_bytes = row_stride * esize(dtype);
     d.tokens = tokens;
     d.trec = reinterpret_cast<const RowRec *>(w.base + w.L.trec);
-    d.res_total = reinterpret_cast<double *>(w.base + w.L.res_total);
-    d.res_last = reinterpret_cast<int32_t *>(w.base + w.L.res_last);
-    d.res_count = reinterpret_cast<uint32_t *>(w.base + w.L.res_count);
+    d.blk_count = reinterpret_cast<uint32_t *>(w.base + w.L.blk_count);
+    d.blk_L = reinterpret_cast<int32_t *>(w.base + w.L.blk_L);
     d.k0 = reinterpret_cast<int32_t *>(w.base + w.L.k0);
-    d.status = status;
-    d.nseg = 1;
-    d.seg_vec = d.RV;
 }
 
-// Residual segments per block: about two CTAs per SM in total, at least one
-// full 256-vector chunk per segment.
-void set_segments(DecideParams &d, int sms) {
-    const int nb = std::max(1, d.nb);
-    int nseg = (2 * sms + nb - 1) / nb;
-    nseg = std::min(nseg, kResidMaxSeg);
-    nseg = std::min(nseg, (d.RV + kResidThreads - 1) / kResidThreads);
-    nseg = std::max(nseg, 1);
-    d.seg_vec = (d.RV + nseg - 1) / nseg;
-    d.nseg = (d.RV + d.seg_vec - 1) / d.seg_vec;
+// The sampling draw: segments of whole 256-vector chunks, at most kDrawMaxSeg.
+void init_draw(DrawParams &q, const Work &w, sdd_dtype_t dtype, int B, int gamma, int V, int64_t row_stride,
+               const int32_t *tokens, int nb, const int32_t *bidx, int32_t *status) {
+    std::memset(&q, 0, sizeof q);
+    q.B = B;
+    q.gamma = gamma;
+    q.V = V;
+    q.RV = static_cast<int32_t>((static_cast<int64_t>(V) * esize(dtype) + 15) / 16);
+    q.dtype = dtype;
+    q.nb = nb;
+    q.bidx = bidx;
+    q.stride_bytes = row_stride * esize(dtype);
+    q.tokens = tokens;
+    q.trec = reinterpret_cast<const RowRec *>(w.base + w.L.trec);
+    q.blk_L = reinterpret_cast<const int32_t *>(w.base + w.L.blk_L);
+    q.res_total = reinterpret_cast<double *>(w.base + w.L.res_total);
+    q.res_last = reinterpret_cast<int32_t *>(w.base + w.L.res_last);
+    q.res_count = reinterpret_cast<uint32_t *>(w.base + w.L.res_count);
+    q.status = status;
+    // segments of 2 vectors per thread (more when the row needs > kDrawMaxSeg)
+    const int per_thread = std::max(2, (q.RV + kDrawThreads * kDrawMaxSeg - 1) / (kDrawThreads * kDrawMaxSeg));
+    q.seg_vec = per_thread * kDrawThreads;
+    q.nseg = (q.RV + q.seg_vec - 1) / q.seg_vec;
 }
 
 sdd_status_t set_thresholds(int signal, const double *eta_b, const double *eta_c, int n_tau, double *eta_loc,
@@ -254,10 +262,11 @@ sdd_status_t check_rows(const int32_t *rows, int n_rows, int B) {
         if (_s != SDD_OK) return _s;          \
     } while (0)
 
-// Target-row scan (post-verify) for the listed blocks.
+// Target-row scan (post-verify) for the listed blocks; the block decisions in
+// `dec` run inside the same launch.
 sdd_status_t target_scan(const Work &w, const void *target_logits, sdd_dtype_t dtype, int B, int gamma, int V,
                          int64_t row_stride, const int32_t *tokens, const int32_t *rows, int n_rows, int kcap,
-                         int32_t *status, cudaStream_t stream) {
+                         const DecideParams &dec, int32_t *status, cudaStream_t stream) {
     ScanParams p;
     init_scan(p, w, dtype, B, gamma, V, tokens, status);
     p.n_groups = 1;
@@ -270,6 +279,7 @@ sdd_status_t target_scan(const Work &w, const void *target_logits, sdd_dtype_t d
     G.nb = n_rows;
     G.bidx = rows;
     G.rec = reinterpret_cast<RowRec *>(w.base + w.L.trec);
+    p.dec = dec;
     return run_scan(p, w, stream);
 }
 
@@ -360,10 +370,9 @@ sdd_status_t sdd_schedule_prefix(const float *q, const float *logq, int B, int g
 
 sdd_status_t sdd_verify_strict(const void *target_logits, const void *draft_logits, sdd_dtype_t dtype, int B,
                                int gamma, int V, int64_t row_stride, const int32_t *draft_tokens,
-                               const double *draft_lse, int greedy, uint64_t seed,
-                               uint64_t round, const int32_t *rows, int n_rows, int32_t *L, int32_t *tokens,
-                               int32_t *n_commit, void *workspace, size_t workspace_bytes, int32_t *status,
-                               sdd_stream_t stream) {
+                               const double *draft_lse, int greedy, uint64_t seed, uint64_t round, const int32_t *rows,
+                               int n_rows, int32_t *L, int32_t *tokens, int32_t *n_commit, void *workspace,
+                               size_t workspace_bytes, int32_t *status, sdd_stream_t stream) {
     SDD_TRY(check_shape(dtype, B, gamma, V, row_stride));
     SDD_TRY(check_rows(rows, n_rows, B));
     if (n_rows == 0) return SDD_OK;
@@ -376,12 +385,10 @@ sdd_status_t sdd_verify_strict(const void *target_logits, const void *draft_logi
     Work w;
     SDD_TRY(get_work(workspace, workspace_bytes, B, gamma, w));
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    SDD_TRY(target_scan(w, target_logits, dtype, B, gamma, V, row_stride, draft_tokens, rows, n_rows, 1, status, st));
     DecideParams d;
-    init_decide(d, w, dtype, B, gamma, V, row_stride, draft_tokens, status);
-    d.nb = n_rows;
+    std::memset(&d, 0, sizeof d);
+    init_dec(d, w, dtype, B, gamma, V, row_stride, draft_tokens, gamma + 1);
     d.bidx = rows;
-    d.zt = static_cast<const char *>(target_logits);
     d.zd = static_cast<const char *>(draft_logits);
     d.d_lse = draft_lse;
     d.do_strict = 1;
@@ -391,9 +398,20 @@ sdd_status_t sdd_verify_strict(const void *target_logits, const void *draft_logi
     d.L_strict = L;
     d.tok_strict = tokens;
     d.n_strict = n_commit;
-    if (!greedy) set_segments(d, w.sms);
-    cudaError_t e = launch_decide(d, st);
-    if (e != cudaSuccess) return cuda_fail(e, "decide launch");
+    SDD_TRY(target_scan(w, target_logits, dtype, B, gamma, V, row_stride, draft_tokens, rows, n_rows, 1, d, status, st));
+    if (greedy) return SDD_OK;
+    DrawParams q;
+    init_draw(q, w, dtype, B, gamma, V, row_stride, draft_tokens, n_rows, rows, status);
+    q.zt = static_cast<const char *>(target_logits);
+    q.zd = static_cast<const char *>(draft_logits);
+    q.d_lse = draft_lse;
+    q.seed = seed;
+    q.round = round;
+    q.L_strict = L;
+    q.tok_strict = tokens;
+    q.n_strict = n_commit;
+    cudaError_t e = launch_draw(q, st);
+    if (e != cudaSuccess) return cuda_fail(e, "draw launch");
     return SDD_OK;
 }
 
@@ -412,22 +430,13 @@ sdd_status_t sdd_verify_lenient(const void *target_logits, sdd_dtype_t dtype, in
     if (!draft_tokens) return fail(SDD_ERR_INVALID_ARGUMENT, "draft_tokens is NULL");
     Work w;
     SDD_TRY(get_work(workspace, workspace_bytes, B, gamma, w));
-    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    SDD_TRY(target_scan(w, target_logits, dtype, B, gamma, V, row_stride, draft_tokens, rows, n_rows, 1, status, st));
-    DecideParams dd;
-    init_decide(dd, w, dtype, B, gamma, V, row_stride, draft_tokens, status);
-    dd.nb = n_rows;
-    dd.bidx = rows;
-    dd.zt = static_cast<const char *>(target_logits);
-    dd.n_ell = d.n_ell;
-    std::memcpy(dd.ell_thr, d.ell_thr, sizeof d.ell_thr);
-    std::memcpy(dd.ell_one, d.ell_one, sizeof d.ell_one);
-    dd.L_len = L;
-    dd.tok_len = tokens;
-    dd.n_len = n_commit;
-    cudaError_t e = launch_decide(dd, st);
-    if (e != cudaSuccess) return cuda_fail(e, "decide launch");
-    return SDD_OK;
+    init_dec(d, w, dtype, B, gamma, V, row_stride, draft_tokens, gamma + 1);
+    d.bidx = rows;
+    d.L_len = L;
+    d.tok_len = tokens;
+    d.n_len = n_commit;
+    return target_scan(w, target_logits, dtype, B, gamma, V, row_stride, draft_tokens, rows, n_rows, 1, d, status,
+                       reinterpret_cast<cudaStream_t>(stream));
 }
 
 sdd_status_t sdd_verify_topk(const void *target_logits, sdd_dtype_t dtype, int B, int gamma, int V,
@@ -446,22 +455,13 @@ sdd_status_t sdd_verify_topk(const void *target_logits, sdd_dtype_t dtype, int B
     if (!draft_tokens) return fail(SDD_ERR_INVALID_ARGUMENT, "draft_tokens is NULL");
     Work w;
     SDD_TRY(get_work(workspace, workspace_bytes, B, gamma, w));
-    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    SDD_TRY(target_scan(w, target_logits, dtype, B, gamma, V, row_stride, draft_tokens, rows, n_rows, kcap, status,
-                        st));
-    DecideParams dd;
-    init_decide(dd, w, dtype, B, gamma, V, row_stride, draft_tokens, status);
-    dd.nb = n_rows;
-    dd.bidx = rows;
-    dd.zt = static_cast<const char *>(target_logits);
-    dd.n_k = d.n_k;
-    std::memcpy(dd.kval, d.kval, sizeof d.kval);
-    dd.L_topk = L;
-    dd.tok_topk = tokens;
-    dd.n_topk = n_commit;
-    cudaError_t e = launch_decide(dd, st);
-    if (e != cudaSuccess) return cuda_fail(e, "decide launch");
-    return SDD_OK;
+    init_dec(d, w, dtype, B, gamma, V, row_stride, draft_tokens, gamma + 1);
+    d.bidx = rows;
+    d.L_topk = L;
+    d.tok_topk = tokens;
+    d.n_topk = n_commit;
+    return target_scan(w, target_logits, dtype, B, gamma, V, row_stride, draft_tokens, rows, n_rows, kcap, d, status,
+                       reinterpret_cast<cudaStream_t>(stream));
 }
 
 sdd_status_t sdd_agreement(const int32_t *K, const int32_t *L_strict, int B, int n_tau, int64_t *acc,
@@ -510,12 +510,14 @@ static sdd_status_t block_check(const sdd_block_args *a) {
 
 sdd_status_t sdd_block_scan(const sdd_block_args *a, sdd_stream_t stream) {
     SDD_TRY(block_check(a));
-    if (a->B == 0) return SDD_OK;
     const sdd_dtype_t dt = static_cast<sdd_dtype_t>(a->dtype);
-    DecideParams tmp;
-    std::memset(&tmp, 0, sizeof tmp);
+    DecideParams d;
+    std::memset(&d, 0, sizeof d);
+    SDD_TRY(set_thresholds(a->signal, a->eta_b, a->eta_c, a->n_tau, d.eta_loc, d.log_eta_c, d.tau_off));
+    SDD_TRY(set_ell(d, a->ell, a->n_ell));
     int kcap = 1;
-    SDD_TRY(set_topk(tmp, a->topk, a->n_k, kcap));
+    SDD_TRY(set_topk(d, a->topk, a->n_k, kcap));
+    if (a->B == 0) return SDD_OK;
     Work w;
     SDD_TRY(get_work(a->workspace, a->workspace_bytes, a->B, a->gamma, w));
     ScanParams p;
@@ -542,65 +544,63 @@ sdd_status_t sdd_block_scan(const sdd_block_args *a, sdd_stream_t stream) {
     T.kind = 1;
     T.nb = a->B;
     T.rec = reinterpret_cast<RowRec *>(w.base + w.L.trec);
+    // every rule, the schedule and the agreement counters run in this launch,
+    // by the warp that finalises each block's last row
+    init_dec(d, w, dt, a->B, a->gamma, a->V, a->row_stride, a->draft_tokens, 2 * a->gamma + 1);
+    d.drec = reinterpret_cast<const RowRec *>(w.base + w.L.drec);
+    d.zd = static_cast<const char *>(a->draft_logits);
+    d.do_strict = 1;
+    d.greedy = a->greedy ? 1 : 0;
+    d.seed = a->seed;
+    d.round = a->round;
+    d.L_strict = a->L_strict;
+    d.tok_strict = a->tokens_strict;
+    d.n_strict = a->n_strict;
+    d.L_len = a->L_lenient;
+    d.tok_len = a->tokens_lenient;
+    d.n_len = a->n_lenient;
+    d.L_topk = a->L_topk;
+    d.tok_topk = a->tokens_topk;
+    d.n_topk = a->n_topk;
+    d.do_sched = 1;
+    d.signal = a->signal;
+    d.n_tau = a->n_tau;
+    d.K_min = a->K_min;
+    d.S_max = a->S_max;
+    d.guard = a->guard;
+    d.force_strict = a->force_strict;
+    d.D_in = a->D_in;
+    d.K_hat = a->K_hat;
+    d.K = a->K;
+    d.D_out = a->D_out;
+    d.commit_tokens = a->commit_tokens;
+    d.commit_n = a->commit_n;
+    d.agreement = reinterpret_cast<long long *>(a->agreement);
+    p.dec = d;
     return run_scan(p, w, reinterpret_cast<cudaStream_t>(stream));
 }
 
 sdd_status_t sdd_block_decide(const sdd_block_args *a, sdd_stream_t stream) {
     SDD_TRY(block_check(a));
+    if (a->B == 0 || a->greedy) return SDD_OK;   // greedy rounds are complete after the scan
     const sdd_dtype_t dt = static_cast<sdd_dtype_t>(a->dtype);
-    DecideParams d;
-    std::memset(&d, 0, sizeof d);
-    SDD_TRY(set_thresholds(a->signal, a->eta_b, a->eta_c, a->n_tau, d.eta_loc, d.log_eta_c, d.tau_off));
-    SDD_TRY(set_ell(d, a->ell, a->n_ell));
-    int kcap = 1;
-    SDD_TRY(set_topk(d, a->topk, a->n_k, kcap));
-    if (a->B == 0) return SDD_OK;
     Work w;
     SDD_TRY(get_work(a->workspace, a->workspace_bytes, a->B, a->gamma, w));
-    DecideParams dd;
-    init_decide(dd, w, dt, a->B, a->gamma, a->V, a->row_stride, a->draft_tokens, a->status);
-    dd.nb = a->B;
-    dd.zt = static_cast<const char *>(a->target_logits);
-    dd.zd = static_cast<const char *>(a->draft_logits);
-    dd.drec = reinterpret_cast<const RowRec *>(w.base + w.L.drec);
-    dd.do_strict = 1;
-    dd.greedy = a->greedy ? 1 : 0;
-    dd.seed = a->seed;
-    dd.round = a->round;
-    dd.L_strict = a->L_strict;
-    dd.tok_strict = a->tokens_strict;
-    dd.n_strict = a->n_strict;
-    dd.n_ell = d.n_ell;
-    std::memcpy(dd.ell_thr, d.ell_thr, sizeof d.ell_thr);
-    std::memcpy(dd.ell_one, d.ell_one, sizeof d.ell_one);
-    dd.L_len = a->L_lenient;
-    dd.tok_len = a->tokens_lenient;
-    dd.n_len = a->n_lenient;
-    dd.n_k = d.n_k;
-    std::memcpy(dd.kval, d.kval, sizeof d.kval);
-    dd.L_topk = a->L_topk;
-    dd.tok_topk = a->tokens_topk;
-    dd.n_topk = a->n_topk;
-    dd.do_sched = 1;
-    dd.signal = a->signal;
-    dd.n_tau = a->n_tau;
-    dd.K_min = a->K_min;
-    dd.S_max = a->S_max;
-    std::memcpy(dd.eta_loc, d.eta_loc, sizeof d.eta_loc);
-    std::memcpy(dd.log_eta_c, d.log_eta_c, sizeof d.log_eta_c);
-    std::memcpy(dd.tau_off, d.tau_off, sizeof d.tau_off);
-    dd.guard = a->guard;
-    dd.force_strict = a->force_strict;
-    dd.D_in = a->D_in;
-    dd.K_hat = a->K_hat;
-    dd.K = a->K;
-    dd.D_out = a->D_out;
-    dd.commit_tokens = a->commit_tokens;
-    dd.commit_n = a->commit_n;
-    dd.agreement = reinterpret_cast<long long *>(a->agreement);
-    if (!dd.greedy) set_segments(dd, w.sms);
-    cudaError_t e = launch_decide(dd, reinterpret_cast<cudaStream_t>(stream));
-    if (e != cudaSuccess) return cuda_fail(e, "decide launch");
+    DrawParams q;
+    init_draw(q, w, dt, a->B, a->gamma, a->V, a->row_stride, a->draft_tokens, a->B, nullptr, a->status);
+    q.zt = static_cast<const char *>(a->target_logits);
+    q.zd = static_cast<const char *>(a->draft_logits);
+    q.drec = reinterpret_cast<const RowRec *>(w.base + w.L.drec);
+    q.seed = a->seed;
+    q.round = a->round;
+    q.k0 = reinterpret_cast<const int32_t *>(w.base + w.L.k0);
+    q.L_strict = a->L_strict;
+    q.tok_strict = a->tokens_strict;
+    q.n_strict = a->n_strict;
+    q.commit_tokens = a->commit_tokens;
+    q.commit_n = a->commit_n;
+    cudaError_t e = launch_draw(q, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "draw launch");
     return SDD_OK;
 }
 

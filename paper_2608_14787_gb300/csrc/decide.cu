@@ -1,212 +1,26 @@
-// decide.cu -- the per-block decisions of the path, after the streaming pass.
+// decide.cu -- the kernels that run after (or beside) the streaming pass.
 //
-//  * schedule_block   -- the skip policy of Sec. 4.1 (Eq. 3, K_min, staleness)
-//                        with the three confidence signals of Sec. 4.2.
-//  * decide_kernel    -- acceptance under Strict SDD (Sec. 3.1; greedy, or the
-//                        speculative-sampling rule it cites), lenience (App. A.6
-//                        Eq. 9) and top-k (App. A.6) from the target facts; the
-//                        residual / bonus inverse-CDF draw of the sampling rule
-//                        split over several CTAs per block; and, for a fused
-//                        round, the schedule, the committed tokens and the
-//                        agreement counters of Sec. 3.2 (Eq. 1-2).
-//  * schedule_kernel, agreement_kernel, commit_kernel -- the same pieces as
-//                        stand-alone entry points.
-#include "internal.h"
+//  * draw_kernel      -- the inverse-CDF draw of the speculative-sampling rule
+//                        cited by Sec. 3.1: at the first rejected position the
+//                        residual norm(max(0, p_t - p_d)), or, when the whole
+//                        block is accepted, p_t of the bonus row.  The draw row
+//                        is split into segments, one CTA each; the last segment
+//                        to finish (atomic arrival, no waiting) locates the
+//                        segment holding u * R and rescans it.
+//  * schedule_kernel  -- the skip policy of Sec. 4.1 as a stand-alone call.
+//  * agreement_kernel, commit_kernel, uniforms_kernel -- small stand-alone calls.
+#include "rules.cuh"
 
 namespace sdd {
 
 namespace {
 
-__device__ __forceinline__ float nanf_() { return __int_as_float(0x7FC00000); }
-
-// Skip policy for one block and one threshold pair, by one warp.
-// q, logq (nullable), guard (nullable) point at the block's gamma positions.
-__device__ void schedule_block(int lane, int gamma, const float *q, const float *logq, const uint8_t *guard,
-                               bool off, int D, int signal, double eta_loc, double log_eta_c, int K_min,
-                               int S_max, int &K_hat, int &K, int &D_out) {
-    if (off) {
-        K_hat = 0;
-        K = 0;
-        D_out = 0;
-        return;
-    }
-    // local gate and guards: kb = number of leading positions that pass
-    int kb = gamma;
-    for (int c = 0; c < gamma; c += 32) {
-        const int j = c + lane;
-        bool fail = false;
-        if (j < gamma) {
-            const float qj = q[j];
-            fail = (guard && guard[j]) || !isfinite(qj) || !(static_cast<double>(qj) >= eta_loc);
-        }
-        const unsigned bal = __ballot_sync(0xFFFFFFFFu, fail);
-        if (bal) {
-            kb = c + __ffs(bal) - 1;
-            break;
-        }
-    }
-    int best = 0;
-    if (signal == SDD_SIG_MARGINAL) {
-        best = kb;
-    } else {
-        // prefix sums of ln q in fp64; raw: S_k >= k ln eta_c, conditional: S_k >= ln eta_c
-        double carry = 0.0;
-        for (int c = 0; c < kb; c += 32) {
-            const int j = c + lane;
-            double v = 0.0;
-            if (j < kb) v = logq ? static_cast<double>(logq[j]) : static_cast<double>(logf(q[j]));
-#pragma unroll
-            for (int off2 = 1; off2 < 32; off2 <<= 1) {
-                const double t = __shfl_up_sync(0xFFFFFFFFu, v, off2);
-                if (lane >= off2) v += t;
-            }
-            const double Sk = carry + v;
-            const bool pass = (j < kb) && ((signal == SDD_SIG_RAW) ? (Sk >= static_cast<double>(j + 1) * log_eta_c)
-                                                                    : (Sk >= log_eta_c));
-            const unsigned bal = __ballot_sync(0xFFFFFFFFu, pass);
-            if (bal) best = c + 32 - __clz(bal);
-            carry = __shfl_sync(0xFFFFFFFFu, Sk, 31);
-        }
-    }
-    K_hat = best;
-    K = (D < S_max && best > 0 && best >= K_min) ? best : 0;
-    D_out = (K > 0) ? D + K : 0;
-}
-
-template <int DT>
-__device__ __forceinline__ float load_logit(const char *rowp, int v) {
-    if (DT == SDD_BF16) {
-        const uint16_t h = __ldg(reinterpret_cast<const unsigned short *>(rowp) + v);
-        return __uint_as_float(static_cast<uint32_t>(h) << 16);
-    } else {
-        return __ldg(reinterpret_cast<const float *>(rowp) + v);
-    }
-}
-
-// Weights of the sampling draw for the EPV entries of one 16-byte vector.
-//   residual: p_t - p_d = p_d (exp(D(v)) - 1) with the log-ratio
-//             D(v) = (z_t(v) - z_d(v)) - (LSE_t - LSE_d); the LSE difference is
-//             applied as two fp32 terms (hi + lo) and the difference by expm1, so
-//             no cancellation between near-equal p_t and p_d loses precision;
-//             p_d(v) = 2^(z_d(v) log2(e) - r_d) up to the common factor of the row;
-//   bonus (zd_row == nullptr): 2^(z_t(v) log2(e) - r_t).
-// Returns the fp32 sum of the entries in ascending order (the draw and the
-// totals use this same order).
-template <int DT>
-__device__ __forceinline__ float vec_weights(const char *zt_row, const char *zd_row, int vec, int V, float nrt,
-                                             float nrd, float d_hi, float d_lo, float (&w)[8]) {
-    constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
-    const uint4 a = __ldg(reinterpret_cast<const uint4 *>(zt_row) + vec);
-    uint4 d = make_uint4(0, 0, 0, 0);
-    if (zd_row) d = __ldg(reinterpret_cast<const uint4 *>(zd_row) + vec);
-    const uint32_t *ua = reinterpret_cast<const uint32_t *>(&a);
-    const uint32_t *ud = reinterpret_cast<const uint32_t *>(&d);
-    float sum = 0.f;
-#pragma unroll
-    for (int e = 0; e < EPV; ++e) {
-        float zt, zd;
-        if (DT == SDD_BF16) {
-            zt = (e & 1) ? bf16_hi(ua[e >> 1]) : bf16_lo(ua[e >> 1]);
-            zd = (e & 1) ? bf16_hi(ud[e >> 1]) : bf16_lo(ud[e >> 1]);
-        } else {
-            zt = __uint_as_float(ua[e]);
-            zd = __uint_as_float(ud[e]);
-        }
-        zt = fmax_nan(zt, clamp_floor());
-        zd = fmax_nan(zd, clamp_floor());
-        float wv;
-        if (zd_row) {
-            const float dv = ((zt - zd) - d_hi) - d_lo;
-            wv = (dv > 0.f) ? ex2(fmaf(zd, kLog2e, nrd)) * expm1f(dv) : 0.f;
-        } else {
-            wv = ex2(fmaf(zt, kLog2e, nrt));
-        }
-        if (vec * EPV + e >= V) wv = 0.f;
-        w[e] = wv;
-        sum += wv;
-    }
-    return sum;
-}
-
-// Inclusive block scan of one double per thread (kResidThreads threads).
-__device__ __forceinline__ double block_incl_scan(double v, double *warp_tot, double &block_total) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-        const double t = __shfl_up_sync(0xFFFFFFFFu, v, off);
-        if (lane >= off) v += t;
-    }
-    if (lane == 31) warp_tot[warp] = v;
-    __syncthreads();
-    double base = 0.0, tot = 0.0;
-    for (int w = 0; w < kResidThreads / 32; ++w) {
-        if (w < warp) base += warp_tot[w];
-        tot += warp_tot[w];
-    }
-    __syncthreads();
-    block_total = tot;
-    return base + v;
-}
-
+// Draw-row context: integer references and the hi/lo LSE difference.
 struct DrawCtx {
     const char *zt_row, *zd_row;
     float nrt, nrd, d_hi, d_lo;
 };
 
-// One pass over vectors [v0, v1) of the draw row.  With find == false returns
-// the weight total (and the last positive index); with find == true returns
-// the index of the first entry whose running sum exceeds `target` (or -1).
-template <int DT>
-__device__ double draw_pass(const DrawCtx &c, int v0, int v1, int V, bool find, double target, int &last_pos,
-                            int &found, double *warp_tot, int *s_first) {
-    constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
-    double carry = 0.0;
-    last_pos = -1;
-    found = -1;
-    for (int base = v0; base < v1; base += kResidThreads) {
-        const int vec = base + threadIdx.x;
-        float w[8];
-        float vs_f = 0.f;
-        if (vec < v1) vs_f = vec_weights<DT>(c.zt_row, c.zd_row, vec, V, c.nrt, c.nrd, c.d_hi, c.d_lo, w);
-        if (vec < v1)
-            for (int e = 0; e < EPV; ++e)
-                if (w[e] > 0.f) last_pos = vec * EPV + e;
-        const double vs = static_cast<double>(vs_f);
-        double tot;
-        const double incl = block_incl_scan(vs, warp_tot, tot);
-        if (find) {
-            if (threadIdx.x == 0) *s_first = INT32_MAX;
-            __syncthreads();
-            if (vec < v1 && carry + incl > target) atomicMin(s_first, static_cast<int>(threadIdx.x));
-            __syncthreads();
-            const int tf = *s_first;
-            if (tf != INT32_MAX) {
-                if (static_cast<int>(threadIdx.x) == tf) {
-                    const double before = carry + (incl - vs);
-                    float part = 0.f;
-                    int pick = -1, lastp = -1;
-                    for (int e = 0; e < EPV; ++e) {
-                        if (w[e] > 0.f) lastp = vec * EPV + e;
-                        part += w[e];
-                        if (w[e] > 0.f && before + static_cast<double>(part) > target) {
-                            pick = vec * EPV + e;
-                            break;
-                        }
-                    }
-                    *s_first = (pick >= 0) ? pick : lastp;
-                }
-                __syncthreads();
-                found = *s_first;
-                __syncthreads();
-                return carry;
-            }
-        }
-        carry += tot;
-    }
-    return carry;
-}
-
-// Draw-row context from the two rows' fp64 log-normalisers.
 __device__ __forceinline__ DrawCtx draw_ctx(const char *zt_row, const char *zd_row, double lse_t, double lse_d) {
     DrawCtx c;
     c.zt_row = zt_row;
@@ -224,214 +38,239 @@ __device__ __forceinline__ DrawCtx draw_ctx(const char *zt_row, const char *zd_r
     return c;
 }
 
+// e^x - 1 for x > 0.  Below 0.35 the Taylor polynomial of degree 7 in Horner
+// form (truncation error x^8/8! < 2e-8 relative there); above it 2^(x log2 e)
+// - 1, where the subtraction loses less than a factor 3.4 of relative accuracy.
+__device__ __forceinline__ float expm1_pos(float x) {
+    if (x < 0.35f) {
+        float p = 1.f / 5040.f;
+        p = fmaf(p, x, 1.f / 720.f);
+        p = fmaf(p, x, 1.f / 120.f);
+        p = fmaf(p, x, 1.f / 24.f);
+        p = fmaf(p, x, 1.f / 6.f);
+        p = fmaf(p, x, 0.5f);
+        p = fmaf(p, x, 1.f);
+        return p * x;
+    }
+    return ex2(x * kLog2e) - 1.f;
+}
+
+// Weights of the draw for the EPV entries of one 16-byte vector.
+//   residual: p_t - p_d = p_d (exp(D(v)) - 1) with the log-ratio
+//             D(v) = (z_t(v) - z_d(v)) - (LSE_t - LSE_d); the LSE difference is
+//             applied as two fp32 terms (hi + lo) and the difference by expm1, so
+//             no cancellation between near-equal p_t and p_d loses precision;
+//             p_d(v) = 2^(z_d(v) log2(e) - r_d) up to the common factor of the row;
+//   bonus (zd_row == nullptr): 2^(z_t(v) log2(e) - r_t).
+// Returns the fp32 sum of the entries in ascending order.
 template <int DT>
-__global__ void __launch_bounds__(kResidThreads) decide_kernel(const __grid_constant__ DecideParams p) {
+__device__ __forceinline__ float vec_weights(const DrawCtx &c, uint4 a, uint4 d, int vec, int V, float (&w)[8]) {
     constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
-    const int i = blockIdx.x;     // listed block
-    const int seg = blockIdx.y;   // residual segment
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int gamma = p.gamma;
-    int b = p.bidx ? __ldg(p.bidx + i) : i;
-    const bool b_ok = (b >= 0 && b < p.B);
-    if (!b_ok) {
-        if (seg == 0 && threadIdx.x == 0) status_or(p.status, SDD_DEV_BAD_TOKEN);
-        return;
-    }
-    const RowRec *tr = p.trec + static_cast<int64_t>(i) * (gamma + 1);
-    const int32_t *xb = p.tokens + static_cast<int64_t>(b) * gamma;
-
-    __shared__ int s_L;              // strict accepted length
-    __shared__ double s_lse[2];      // LSE of the target and drafter draw rows
-    __shared__ double s_warp[kResidThreads / 32];
-    __shared__ int s_first;
-    __shared__ double s_tot[kResidMaxSeg];
-    __shared__ int s_last[kResidMaxSeg];
-
-    // ---- acceptance decisions (warp 0) ----
-    if (warp == 0) {
-        int L = gamma;
-        if (p.do_strict) {
-            for (int c = 0; c < gamma; c += 32) {
-                const int j = c + lane;
-                bool fail = false;
-                if (j < gamma) {
-                    const RowRec t = tr[j];
-                    if (p.greedy) {
-                        fail = !(t.rank == 0);
-                    } else {
-                        double lse_d;
-                        float gd;
-                        if (p.drec) {
-                            const RowRec d = p.drec[static_cast<int64_t>(i) * gamma + j];
-                            lse_d = d.lse;
-                            gd = d.g;
-                        } else {
-                            const char *zdr = p.zd + (static_cast<int64_t>(b) * gamma + j) * p.stride_bytes;
-                            const int xj = xb[j];
-                            lse_d = __ldg(p.d_lse + static_cast<int64_t>(b) * gamma + j);
-                            gd = (xj >= 0 && xj < p.V) ? fmax_nan(load_logit<DT>(zdr, xj), clamp_floor()) : nanf_();
-                        }
-                        // log r = log p_t(x_j) - log p_d(x_j) = (g_t - g_d) - (LSE_t - LSE_d), in fp64
-                        const double lr = (static_cast<double>(t.g) - static_cast<double>(gd)) - (t.lse - lse_d);
-                        const float u = philox_uniform(p.seed, static_cast<uint32_t>(j + 1), static_cast<uint32_t>(b),
-                                                       p.round, kPurposeAccept);
-                        const bool acc = (lr >= 0.0) || (u <= expf(static_cast<float>(lr)));
-                        fail = !acc;
-                    }
-                }
-                const unsigned bal = __ballot_sync(0xFFFFFFFFu, fail);
-                if (bal) {
-                    L = c + __ffs(bal) - 1;
-                    break;
-                }
-            }
-            if (lane == 0) s_L = L;
-        }
-        // greedy-family rules are complete here: write them from segment 0
-        if (seg == 0) {
-            auto emit = [&](int32_t *Lp, int32_t *tok, int32_t *np, int Lr) {
-                const int corr = tr[Lr].argmax;
-                if (lane == 0) {
-                    if (Lp) Lp[b] = Lr;
-                    if (np) np[b] = Lr + 1;
-                }
-                if (tok)
-                    for (int j = lane; j <= gamma; j += 32)
-                        tok[static_cast<int64_t>(b) * (gamma + 1) + j] = (j < Lr) ? xb[j] : (j == Lr ? corr : -1);
-            };
-            if (p.do_strict && p.greedy) emit(p.L_strict, p.tok_strict, p.n_strict, L);
-            for (int r = 0; r < p.n_ell; ++r) {
-                int Lr = gamma;
-                for (int c = 0; c < gamma; c += 32) {
-                    const int j = c + lane;
-                    bool fail = false;
-                    if (j < gamma) {
-                        const RowRec t = tr[j];
-                        fail = p.ell_one[r] ? !(t.rank == 0) : !(static_cast<double>(t.g - t.M) >= p.ell_thr[r]);
-                    }
-                    const unsigned bal = __ballot_sync(0xFFFFFFFFu, fail);
-                    if (bal) {
-                        Lr = c + __ffs(bal) - 1;
-                        break;
-                    }
-                }
-                const int64_t o = static_cast<int64_t>(r) * p.B;
-                emit(p.L_len ? p.L_len + o : nullptr, p.tok_len ? p.tok_len + o * (gamma + 1) : nullptr,
-                     p.n_len ? p.n_len + o : nullptr, Lr);
-            }
-            for (int r = 0; r < p.n_k; ++r) {
-                int Lr = gamma;
-                for (int c = 0; c < gamma; c += 32) {
-                    const int j = c + lane;
-                    bool fail = false;
-                    if (j < gamma) fail = !(tr[j].rank < p.kval[r]);
-                    const unsigned bal = __ballot_sync(0xFFFFFFFFu, fail);
-                    if (bal) {
-                        Lr = c + __ffs(bal) - 1;
-                        break;
-                    }
-                }
-                const int64_t o = static_cast<int64_t>(r) * p.B;
-                emit(p.L_topk ? p.L_topk + o : nullptr, p.tok_topk ? p.tok_topk + o * (gamma + 1) : nullptr,
-                     p.n_topk ? p.n_topk + o : nullptr, Lr);
-            }
-            // fused round: schedule, agreement and the tokens of skipped blocks
-            if (p.do_sched) {
-                const RowRec *dr = p.drec + static_cast<int64_t>(i) * gamma;
-                // gather q / logq of the block into registers-by-lane via shared memory is not
-                // needed: schedule_block reads them through these small strided views
-                __shared__ float s_q[SDD_MAX_GAMMA], s_lq[SDD_MAX_GAMMA];
-                for (int j = lane; j < gamma; j += 32) {
-                    s_q[j] = dr[j].q;
-                    s_lq[j] = dr[j].logq;
-                }
-                __syncwarp();
-                const bool force = p.force_strict && p.force_strict[b];
-                const int D = p.D_in ? p.D_in[b] : 0;
-                for (int t = 0; t < p.n_tau; ++t) {
-                    int Kh, K, Do;
-                    schedule_block(lane, gamma, s_q, s_lq,
-                                   p.guard ? p.guard + static_cast<int64_t>(b) * gamma : nullptr,
-                                   force || p.tau_off[t], D, p.signal, p.eta_loc[t], p.log_eta_c[t], p.K_min, p.S_max,
-                                   Kh, K, Do);
-                    if (lane == 0) {
-                        const int64_t o = static_cast<int64_t>(t) * p.B + b;
-                        if (p.K_hat) p.K_hat[o] = Kh;
-                        if (p.K) p.K[o] = K;
-                        if (p.D_out) p.D_out[o] = Do;
-                        if (p.agreement && K > 0 && p.do_strict) {
-                            unsigned long long *a = reinterpret_cast<unsigned long long *>(p.agreement + 4 * t);
-                            atomicAdd(a + 0, static_cast<unsigned long long>(min(K, L)));
-                            atomicAdd(a + 1, static_cast<unsigned long long>(K));
-                            atomicAdd(a + 2, static_cast<unsigned long long>(K <= L ? 1 : 0));
-                            atomicAdd(a + 3, 1ull);
-                        }
-                    }
-                    if (t == 0) {
-                        const bool skip = K > 0;
-                        if (lane == 0) p.k0[i] = K;   // read by the CTA that completes the sampling draw
-                        if (skip || (p.do_strict && p.greedy)) {
-                            // skipped: commit x_1..x_K; greedy strict: the verified tokens
-                            const int Lc = skip ? K : L;
-                            const int corr = skip ? -1 : tr[L].argmax;
-                            if (lane == 0 && p.commit_n) p.commit_n[b] = skip ? K : L + 1;
-                            if (p.commit_tokens)
-                                for (int j = lane; j <= gamma; j += 32)
-                                    p.commit_tokens[static_cast<int64_t>(b) * (gamma + 1) + j] =
-                                        (j < Lc) ? xb[j] : (j == Lc ? corr : -1);
-                        }
-                    }
-                }
-            }
-        }
-    }
-    __syncthreads();
-    if (!p.do_strict || p.greedy) return;
-
-    // ---- sampling: residual (L < gamma) or bonus (L = gamma) inverse-CDF draw ----
-    const int L = s_L;
-    if (threadIdx.x == 0) {
-        s_lse[0] = tr[L].lse;
-        s_lse[1] = 0.0;
-        if (L < gamma)
-            s_lse[1] = p.drec ? p.drec[static_cast<int64_t>(i) * gamma + L].lse
-                              : __ldg(p.d_lse + static_cast<int64_t>(b) * gamma + L);
-    }
-    __syncthreads();
-    const DrawCtx c = draw_ctx(p.zt + (static_cast<int64_t>(b) * (gamma + 1) + L) * p.stride_bytes,
-                               (L < gamma) ? p.zd + (static_cast<int64_t>(b) * gamma + L) * p.stride_bytes : nullptr,
-                               s_lse[0], s_lse[1]);
-    const int v0 = seg * p.seg_vec, v1 = min(p.RV, v0 + p.seg_vec);
-    int last_pos, found;
-    const double tot = (v0 < v1) ? draw_pass<DT>(c, v0, v1, p.V, false, 0.0, last_pos, found, s_warp, &s_first) : 0.0;
-    // publish this segment's total (and last positive entry) and count arrivals
-    int lp = last_pos;
+    const uint32_t *ua = reinterpret_cast<const uint32_t *>(&a);
+    const uint32_t *ud = reinterpret_cast<const uint32_t *>(&d);
+    float sum = 0.f;
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) lp = max(lp, __shfl_xor_sync(0xFFFFFFFFu, lp, off));
-    __shared__ int s_lpw[kResidThreads / 32];
-    if (lane == 0) s_lpw[warp] = lp;
+    for (int e = 0; e < EPV; ++e) {
+        float zt, zd;
+        if (DT == SDD_BF16) {
+            zt = (e & 1) ? bf16_hi(ua[e >> 1]) : bf16_lo(ua[e >> 1]);
+            zd = (e & 1) ? bf16_hi(ud[e >> 1]) : bf16_lo(ud[e >> 1]);
+        } else {
+            zt = __uint_as_float(ua[e]);
+            zd = __uint_as_float(ud[e]);
+        }
+        zt = fmax_nan(zt, clamp_floor());
+        zd = fmax_nan(zd, clamp_floor());
+        float wv;
+        if (c.zd_row) {
+            const float dv = ((zt - zd) - c.d_hi) - c.d_lo;
+            wv = 0.f;
+            if (dv > 0.f) wv = ex2(fmaf(zd, kLog2e, c.nrd)) * expm1_pos(dv);
+        } else {
+            wv = ex2(fmaf(zt, kLog2e, c.nrt));
+        }
+        if (vec * EPV + e >= V) wv = 0.f;
+        w[e] = wv;
+        sum += wv;
+    }
+    return sum;
+}
+
+// Inclusive scan of one fp32 value per thread over the CTA (kDrawThreads).
+// Returns the thread's inclusive value; *total receives the CTA total.
+__device__ __forceinline__ float cta_incl_scan(float v, float *warp_tot, float *total) {
+    constexpr int NW = kDrawThreads / 32;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const float t = __shfl_up_sync(0xFFFFFFFFu, v, off);
+        if (lane >= off) v += t;
+    }
+    if (lane == 31) warp_tot[warp] = v;
     __syncthreads();
-    __shared__ int s_is_last;
-    if (threadIdx.x == 0) {
-        int lpb = -1;
-        for (int w = 0; w < kResidThreads / 32; ++w) lpb = max(lpb, s_lpw[w]);
-        p.res_total[static_cast<int64_t>(i) * p.nseg + seg] = tot;
-        p.res_last[static_cast<int64_t>(i) * p.nseg + seg] = lpb;
-        __threadfence();
-        const uint32_t old = atomicAdd(p.res_count + i, 1u);
-        s_is_last = (old == static_cast<uint32_t>(p.nseg - 1)) ? 1 : 0;
+    if (threadIdx.x < 32) {
+        float t = (lane < NW) ? warp_tot[lane] : 0.f;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const float s = __shfl_up_sync(0xFFFFFFFFu, t, off);
+            if (lane >= off) t += s;
+        }
+        if (lane < NW) warp_tot[NW + lane] = t;   // inclusive prefix of the warp totals
     }
     __syncthreads();
+    const float r = ((warp > 0) ? warp_tot[NW + warp - 1] : 0.f) + v;
+    *total = warp_tot[2 * NW - 1];
+    __syncthreads();
+    return r;
+}
+
+// Sum (fp32, ascending order) of the draw weights of vectors [vb, ve).
+template <int DT>
+__device__ __forceinline__ float run_sum(const DrawCtx &c, int vb, int ve, int V, int &last_pos) {
+    constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
+    float sum = 0.f;
+    for (int v = vb; v < ve; v += 4) {
+        uint4 a[4], d[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int vec = v + k;
+            a[k] = d[k] = make_uint4(0, 0, 0, 0);
+            if (vec < ve) {
+                a[k] = __ldg(reinterpret_cast<const uint4 *>(c.zt_row) + vec);
+                if (c.zd_row) d[k] = __ldg(reinterpret_cast<const uint4 *>(c.zd_row) + vec);
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int vec = v + k;
+            if (vec < ve) {
+                float w[8];
+                vec_weights<DT>(c, a[k], d[k], vec, V, w);
+#pragma unroll
+                for (int e = 0; e < EPV; ++e) {
+                    sum += w[e];
+                    if (w[e] > 0.f) last_pos = vec * EPV + e;
+                }
+            }
+        }
+    }
+    return sum;
+}
+
+// The first entry of vectors [vb, ve) whose running sum, starting at `start`,
+// exceeds `target` (same order and arithmetic as run_sum); -1 if none.
+template <int DT>
+__device__ __forceinline__ int run_find(const DrawCtx &c, int vb, int ve, int V, double start, double target,
+                                        int &last_pos) {
+    constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
+    float sum = 0.f;
+    for (int vec = vb; vec < ve; ++vec) {
+        const uint4 a = __ldg(reinterpret_cast<const uint4 *>(c.zt_row) + vec);
+        const uint4 d = c.zd_row ? __ldg(reinterpret_cast<const uint4 *>(c.zd_row) + vec) : make_uint4(0, 0, 0, 0);
+        float w[8];
+        vec_weights<DT>(c, a, d, vec, V, w);
+#pragma unroll
+        for (int e = 0; e < EPV; ++e) {
+            sum += w[e];
+            if (w[e] > 0.f) {
+                last_pos = vec * EPV + e;
+                if (start + static_cast<double>(sum) > target) return vec * EPV + e;
+            }
+        }
+    }
+    return -1;
+}
+
+// Inverse CDF over vectors [v0, v1) of the draw row, one contiguous run of
+// `vpt` vectors per thread: returns the drawn index (or the last positive
+// entry if rounding leaves none), identical in every thread.
+template <int DT>
+__device__ int cta_find(const DrawCtx &c, int v0, int v1, int vpt, int V, double before, double target,
+                        float *s_warp, int *s_thr, int *s_tok) {
+    const int vb = min(v1, v0 + static_cast<int>(threadIdx.x) * vpt), ve = min(v1, vb + vpt);
+    int lastp = -1;
+    const float ts = run_sum<DT>(c, vb, ve, V, lastp);
+    float tot;
+    const float incl = cta_incl_scan(ts, s_warp, &tot);
+    if (threadIdx.x == 0) *s_thr = INT32_MAX;
+    __syncthreads();
+    const bool mine = (ve > vb) && (before + static_cast<double>(incl) > target);
+    const unsigned bal = __ballot_sync(0xFFFFFFFFu, mine);
+    if ((threadIdx.x & 31) == 0 && bal) atomicMin(s_thr, static_cast<int>(threadIdx.x) + __ffs(bal) - 1);
+    __syncthreads();
+    const int thr = *s_thr;
+    if (thr == INT32_MAX) return -1;
+    if (static_cast<int>(threadIdx.x) == thr) {
+        int lp = -1;
+        const int pick = run_find<DT>(c, vb, ve, V, before + static_cast<double>(incl - ts), target, lp);
+        *s_tok = (pick >= 0) ? pick : lp;
+    }
+    __syncthreads();
+    return *s_tok;
+}
+
+template <int DT>
+__global__ void __launch_bounds__(kDrawThreads) draw_kernel(const __grid_constant__ DrawParams p) {
+    const int i = blockIdx.x;       // listed block
+    const int seg = blockIdx.y;     // segment of the draw row
+    const int gamma = p.gamma;
+    const int b = p.bidx ? __ldg(p.bidx + i) : i;
+    if (b < 0 || b >= p.B) return;  // flagged by the streaming pass
+    __shared__ float s_warp[2 * (kDrawThreads / 32)];
+    __shared__ int s_is_last, s_seg, s_lastp, s_thr, s_tok, s_L;
+    __shared__ double s_target, s_before;
+    __shared__ double s_tot[kDrawMaxSeg];
+    __shared__ int s_last[kDrawMaxSeg];
+    __shared__ DrawCtx s_ctx;
+
+    // the draw row and its context, once per CTA
+    if (threadIdx.x == 0) {
+        const int L = p.blk_L[i];
+        const double lse_t = p.trec[static_cast<int64_t>(i) * (gamma + 1) + L].lse;
+        double lse_d = 0.0;
+        if (L < gamma)
+            lse_d = p.drec ? p.drec[static_cast<int64_t>(i) * gamma + L].lse
+                           : p.d_lse[static_cast<int64_t>(b) * gamma + L];
+        const char *zt_row = p.zt + (static_cast<int64_t>(b) * (gamma + 1) + L) * p.stride_bytes;
+        const char *zd_row = (L < gamma) ? p.zd + (static_cast<int64_t>(b) * gamma + L) * p.stride_bytes : nullptr;
+        s_ctx = draw_ctx(zt_row, zd_row, lse_t, lse_d);
+        s_L = L;
+        s_lastp = -1;
+    }
+    __syncthreads();
+    const DrawCtx c = s_ctx;
+    const int L = s_L;
+    const int vpt = p.seg_vec / kDrawThreads;
+
+    // first pass: this segment's weight total and last positive entry
+    const int v0 = seg * p.seg_vec, v1 = min(p.RV, v0 + p.seg_vec);
+    int last_pos = -1;
+    {
+        const int vb = min(v1, v0 + static_cast<int>(threadIdx.x) * vpt), ve = min(v1, vb + vpt);
+        const float ts = run_sum<DT>(c, vb, ve, p.V, last_pos);
+        float tot;
+        (void)cta_incl_scan(ts, s_warp, &tot);
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) last_pos = max(last_pos, __shfl_xor_sync(0xFFFFFFFFu, last_pos, off));
+        if ((threadIdx.x & 31) == 0) atomicMax(&s_lastp, last_pos);
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            p.res_total[static_cast<int64_t>(i) * p.nseg + seg] = static_cast<double>(tot);
+            p.res_last[static_cast<int64_t>(i) * p.nseg + seg] = s_lastp;
+            __threadfence();
+            const uint32_t old = atomicAdd(p.res_count + i, 1u);
+            s_is_last = (old == static_cast<uint32_t>(p.nseg - 1)) ? 1 : 0;
+        }
+        __syncthreads();
+    }
     if (!s_is_last) return;
     __threadfence();
-    // the last segment to arrive completes the draw for this block
-    if (threadIdx.x < p.nseg) {
-        s_tot[threadIdx.x] = __ldcg(p.res_total + static_cast<int64_t>(i) * p.nseg + threadIdx.x);
-        s_last[threadIdx.x] = __ldcg(p.res_last + static_cast<int64_t>(i) * p.nseg + threadIdx.x);
+    // the last segment to arrive completes the draw: locate the segment holding u * R
+    for (int s = threadIdx.x; s < p.nseg; s += kDrawThreads) {
+        s_tot[s] = __ldcg(p.res_total + static_cast<int64_t>(i) * p.nseg + s);
+        s_last[s] = __ldcg(p.res_last + static_cast<int64_t>(i) * p.nseg + s);
     }
     __syncthreads();
-    __shared__ int s_seg, s_lastp;
-    __shared__ double s_target, s_before;
     if (threadIdx.x == 0) {
         double R = 0.0;
         int lastp = -1;
@@ -443,18 +282,17 @@ __global__ void __launch_bounds__(kResidThreads) decide_kernel(const __grid_cons
         const float u = philox_uniform(p.seed, jj, static_cast<uint32_t>(b), p.round,
                                        (L < gamma) ? kPurposeResid : kPurposeBonus);
         const double target = static_cast<double>(u) * R;
-        int sel = -2;   // -2: none (rounding) -> last positive; -3: no mass
-        double before = 0.0, cum = 0.0;
-        if (!(R > 0.0)) {
-            sel = -3;
-        } else {
+        int sel = (R > 0.0) ? -2 : -3;   // -2: rounding left none (last positive), -3: no mass
+        double cum = 0.0, before = 0.0;
+        if (R > 0.0) {
             for (int s = 0; s < p.nseg; ++s) {
-                if (cum + s_tot[s] > target && s_tot[s] > 0.0) {
+                const double t = s_tot[s];
+                if (t > 0.0 && cum + t > target) {
                     sel = s;
                     before = cum;
                     break;
                 }
-                cum += s_tot[s];
+                cum += t;
             }
         }
         s_seg = sel;
@@ -464,51 +302,43 @@ __global__ void __launch_bounds__(kResidThreads) decide_kernel(const __grid_cons
         p.res_count[i] = 0u;   // leave the workspace zeroed
     }
     __syncthreads();
-    int tok = -1;
+    int tok;
     if (s_seg >= 0) {
         const int sv0 = s_seg * p.seg_vec, sv1 = min(p.RV, sv0 + p.seg_vec);
-        const int lastp = s_lastp;
-        int lp2, fnd;
-        (void)draw_pass<DT>(c, sv0, sv1, p.V, true, s_target - s_before, lp2, fnd, s_warp, &s_first);
-        tok = (fnd >= 0) ? fnd : lastp;
+        tok = cta_find<DT>(c, sv0, sv1, vpt, p.V, s_before, s_target, s_warp, &s_thr, &s_tok);
+        if (tok < 0) tok = s_lastp;
     } else if (s_seg == -2) {
         tok = s_lastp;
     } else {
-        // the residual has no mass (only possible through rounding): draw from p_t of
-        // this row, whole row in this CTA, same inverse-CDF rule
+        // the residual has no mass (only through rounding): draw from p_t of the
+        // same row, whole row in this CTA, same inverse-CDF rule
         DrawCtx ct = c;
         ct.zd_row = nullptr;
-        int lp3, fnd;
-        __syncthreads();
-        const double R = draw_pass<DT>(ct, 0, p.RV, p.V, false, 0.0, lp3, fnd, s_warp, &s_first);
+        const int vrow = (p.RV + kDrawThreads - 1) / kDrawThreads;
+        const int vb = min(p.RV, static_cast<int>(threadIdx.x) * vrow), ve = min(p.RV, vb + vrow);
+        int lp = -1;
+        float tot;
+        (void)cta_incl_scan(run_sum<DT>(ct, vb, ve, p.V, lp), s_warp, &tot);
         const float u = philox_uniform(p.seed, static_cast<uint32_t>(L + 1), static_cast<uint32_t>(b), p.round,
                                        kPurposeResid);
-        if (R > 0.0) {
-            (void)draw_pass<DT>(ct, 0, p.RV, p.V, true, static_cast<double>(u) * R, lp3, fnd, s_warp, &s_first);
-            tok = fnd;
-        }
+        tok = (tot > 0.f) ? cta_find<DT>(ct, 0, p.RV, vrow, p.V, 0.0, static_cast<double>(u) * tot, s_warp, &s_thr, &s_tok)
+                          : -1;
     }
-    if (warp == 0) {
+    if (threadIdx.x < 32) {
+        const int lane = threadIdx.x;
+        const int32_t *xb = p.tokens + static_cast<int64_t>(b) * gamma;
+        const int64_t bo = static_cast<int64_t>(b) * (gamma + 1);
         if (lane == 0) {
             if (p.L_strict) p.L_strict[b] = L;
             if (p.n_strict) p.n_strict[b] = L + 1;
         }
-        if (p.tok_strict)
-            for (int j = lane; j <= gamma; j += 32)
-                p.tok_strict[static_cast<int64_t>(b) * (gamma + 1) + j] = (j < L) ? xb[j] : (j == L ? tok : -1);
-        if (p.do_sched) {
-            // commit under pair 0 when that schedule did not skip this block
-            const int K0 = __ldcg(p.k0 + i);
-            if (K0 == 0) {
-                if (lane == 0 && p.commit_n) p.commit_n[b] = L + 1;
-                if (p.commit_tokens)
-                    for (int j = lane; j <= gamma; j += 32)
-                        p.commit_tokens[static_cast<int64_t>(b) * (gamma + 1) + j] =
-                            (j < L) ? xb[j] : (j == L ? tok : -1);
-            }
+        if (p.tok_strict) write_tokens(lane, gamma, p.tok_strict + bo, xb, L, tok);
+        if (p.k0 && p.k0[i] == 0) {
+            // commit under pair 0: this block was not skipped
+            if (lane == 0 && p.commit_n) p.commit_n[b] = L + 1;
+            if (p.commit_tokens) write_tokens(lane, gamma, p.commit_tokens + bo, xb, L, tok);
         }
     }
-    (void)EPV;
 }
 
 __global__ void schedule_kernel(const __grid_constant__ ScheduleParams p) {
@@ -520,7 +350,7 @@ __global__ void schedule_kernel(const __grid_constant__ ScheduleParams p) {
     const bool force = p.force_strict && p.force_strict[b];
     const int D = p.D_in ? p.D_in[b] : 0;
     int Kh, K, Do;
-    schedule_block(lane, p.gamma, p.q + o, p.logq ? p.logq + o : nullptr, p.guard ? p.guard + o : nullptr,
+    schedule_block(lane, p.gamma, p.q + o, p.logq ? p.logq + o : nullptr, 1, p.guard ? p.guard + o : nullptr,
                    force || p.tau_off[t], D, p.signal, p.eta_loc[t], p.log_eta_c[t], p.K_min, p.S_max, Kh, K, Do);
     if (lane == 0) {
         const int64_t oo = static_cast<int64_t>(t) * p.B + b;
@@ -566,20 +396,13 @@ __global__ void uniforms_kernel(uint64_t seed, const uint32_t *j, const uint32_t
 
 }  // namespace
 
-cudaError_t launch_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, const uint64_t *round,
-                            const uint32_t *purpose, int64_t n, float *u, cudaStream_t stream) {
-    if (n == 0) return cudaSuccess;
-    uniforms_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, stream>>>(seed, j, b, round, purpose, n, u);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_decide(const DecideParams &p, cudaStream_t stream) {
+cudaError_t launch_draw(const DrawParams &p, cudaStream_t stream) {
     if (p.nb == 0) return cudaSuccess;
     const dim3 grid(p.nb, p.nseg);
     if (p.dtype == SDD_BF16)
-        decide_kernel<SDD_BF16><<<grid, kResidThreads, 0, stream>>>(p);
+        draw_kernel<SDD_BF16><<<grid, kDrawThreads, 0, stream>>>(p);
     else
-        decide_kernel<SDD_F32><<<grid, kResidThreads, 0, stream>>>(p);
+        draw_kernel<SDD_F32><<<grid, kDrawThreads, 0, stream>>>(p);
     return cudaGetLastError();
 }
 
@@ -604,6 +427,13 @@ cudaError_t launch_commit(const int32_t *K, const int32_t *x, const int32_t *vt,
     const int64_t n = static_cast<int64_t>(B) * (gamma + 1);
     if (n == 0) return cudaSuccess;
     commit_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, stream>>>(K, x, vt, vn, B, gamma, out_t, out_n);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, const uint64_t *round,
+                            const uint32_t *purpose, int64_t n, float *u, cudaStream_t stream) {
+    if (n == 0) return cudaSuccess;
+    uniforms_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, stream>>>(seed, j, b, round, purpose, n, u);
     return cudaGetLastError();
 }
 

@@ -1,5 +1,5 @@
-// internal.h -- launch parameters shared between the C-ABI layer (api.cu) and
-// the kernels (scan.cu, decide.cu).  Not part of the public ABI.
+// internal.h -- launch parameters shared between the C-ABI layer (api.cu,
+// noalloc.cu) and the kernels (scan.cu, decide.cu).  Not part of the public ABI.
 #pragma once
 
 #include <cstdint>
@@ -21,9 +21,53 @@ constexpr int kStages = 3;
 constexpr int kScanSmem = kWarpsPerCta * kStages * kTileBytes + kWarpsPerCta * kStages * 8;
 constexpr uint32_t kWaitPolls = 1u << 24;     // bounded mbarrier wait (seconds of polling)
 
-// Residual / bonus draw geometry.
-constexpr int kResidThreads = 256;
-constexpr int kResidMaxSeg = 64;
+// Sampling draw geometry: each CTA takes a segment of whole 256-vector chunks
+// of the draw row; at most kDrawMaxSeg segments per block.
+constexpr int kDrawThreads = 256;
+constexpr int kDrawMaxSeg = 128;
+
+// Per-block decisions, evaluated inside the streaming kernel by the warp that
+// finalises a block's last row (rules.cuh).
+struct DecideParams {
+    int32_t enabled;               // run block decisions in the streaming kernel
+    int32_t rows_per_block;        // rows of one block streamed by this launch
+    int32_t B, gamma, V;
+    int32_t pad0;
+    int64_t stride_bytes;
+    const int32_t *bidx;           // [nb] batch index of listed block i, or nullptr
+    const char *zd;                // drafter logits (stand-alone sampling acceptance)
+    const int32_t *tokens;         // [B, gamma]
+    const RowRec *trec;            // [nb, gamma+1] list order
+    const RowRec *drec;            // [nb, gamma] list order, or nullptr
+    const double *d_lse;           // [B, gamma] drafter LSE (user array) when drec == nullptr
+    // strict
+    int32_t do_strict, greedy;
+    uint64_t seed, round;
+    int32_t *L_strict, *tok_strict, *n_strict;
+    // lenience
+    int32_t n_ell;
+    int32_t ell_one[SDD_MAX_GRID];
+    double ell_thr[SDD_MAX_GRID];
+    int32_t *L_len, *tok_len, *n_len;
+    // top-k
+    int32_t n_k;
+    int32_t kval[SDD_MAX_GRID];
+    int32_t *L_topk, *tok_topk, *n_topk;
+    // schedule (fused round)
+    int32_t do_sched, signal, n_tau, K_min, S_max;
+    int32_t tau_off[SDD_MAX_GRID];
+    double eta_loc[SDD_MAX_GRID];
+    double log_eta_c[SDD_MAX_GRID];
+    const uint8_t *guard, *force_strict;
+    const int32_t *D_in;
+    int32_t *K_hat, *K, *D_out;
+    int32_t *commit_tokens, *commit_n;
+    long long *agreement;
+    // workspace
+    uint32_t *blk_count;           // [nb] arrival counters of finalised rows
+    int32_t *blk_L;                // [nb] strict accepted length, for the draw kernel
+    int32_t *k0;                   // [nb] K under pair 0, for the draw kernel
+};
 
 // One set of rows streamed by the scan kernel (drafter rows or target rows).
 struct ScanGroup {
@@ -58,45 +102,25 @@ struct ScanParams {
     Partial *partials;       // [rows + W]
     uint32_t *counters;      // [rows]
     int32_t *status;
+    DecideParams dec;
 };
 
-// Drafter-side facts for the sampling rule and the schedule.
-struct DecideParams {
+// The inverse-CDF draw of the sampling rule (residual or bonus), after the
+// streaming kernel has fixed each block's accepted length.
+struct DrawParams {
     int32_t B, gamma, V, RV;
     int32_t dtype, nb;
     int64_t stride_bytes;
-    const int32_t *bidx;           // [nb] or nullptr
-    const char *zt;                // target logits
-    const char *zd;                // drafter logits (sampling only)
-    const int32_t *tokens;         // [B, gamma]
-    const RowRec *trec;            // [nb, gamma+1] list order
-    const RowRec *drec;            // [nb, gamma] list order, or nullptr
-    const double *d_lse;           // [B, gamma] drafter LSE (user array) when drec == nullptr
-    // strict
-    int32_t do_strict, greedy;
+    const int32_t *bidx;
+    const char *zt, *zd;
+    const int32_t *tokens;
+    const RowRec *trec, *drec;
+    const double *d_lse;
     uint64_t seed, round;
+    const int32_t *blk_L;
+    const int32_t *k0;             // nullptr unless a fused round commits tokens
     int32_t *L_strict, *tok_strict, *n_strict;
-    // lenience
-    int32_t n_ell;
-    double ell_thr[SDD_MAX_GRID];
-    int32_t ell_one[SDD_MAX_GRID];
-    int32_t *L_len, *tok_len, *n_len;
-    // top-k
-    int32_t n_k;
-    int32_t kval[SDD_MAX_GRID];
-    int32_t *L_topk, *tok_topk, *n_topk;
-    // schedule (fused round only)
-    int32_t do_sched, signal, n_tau, K_min, S_max;
-    double eta_loc[SDD_MAX_GRID];
-    double log_eta_c[SDD_MAX_GRID];
-    int32_t tau_off[SDD_MAX_GRID];
-    const uint8_t *guard, *force_strict;
-    const int32_t *D_in;
-    int32_t *K_hat, *K, *D_out;
     int32_t *commit_tokens, *commit_n;
-    int32_t *k0;                   // [nb] workspace: K under pair 0 (fused round)
-    long long *agreement;
-    // residual draw
     int32_t nseg, seg_vec;
     double *res_total;             // [nb, nseg]
     int32_t *res_last;             // [nb, nseg]
@@ -107,16 +131,16 @@ struct DecideParams {
 struct ScheduleParams {
     const float *q, *logq;
     int32_t B, gamma, signal, n_tau, K_min, S_max;
+    int32_t tau_off[SDD_MAX_GRID];
     double eta_loc[SDD_MAX_GRID];
     double log_eta_c[SDD_MAX_GRID];
-    int32_t tau_off[SDD_MAX_GRID];
     const uint8_t *guard, *force_strict;
     const int32_t *D_in;
     int32_t *K_hat, *K, *D_out;
 };
 
 cudaError_t launch_scan(const ScanParams &p, int grid, cudaStream_t stream);
-cudaError_t launch_decide(const DecideParams &p, cudaStream_t stream);
+cudaError_t launch_draw(const DrawParams &p, cudaStream_t stream);
 cudaError_t launch_schedule(const ScheduleParams &p, cudaStream_t stream);
 cudaError_t launch_agreement(const int32_t *K, const int32_t *L, int B, int n_tau, long long *acc,
                              cudaStream_t stream);
@@ -125,8 +149,8 @@ cudaError_t launch_commit(const int32_t *K, const int32_t *x, const int32_t *vt,
 cudaError_t launch_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, const uint64_t *round,
                             const uint32_t *purpose, int64_t n, float *u, cudaStream_t stream);
 int scan_max_ctas_per_sm();
-void set_last_error(const char *msg);  // message returned by sdd_last_error()
 cudaError_t scan_prepare_device();
+void set_last_error(const char *msg);  // message returned by sdd_last_error()
 
 // Index arithmetic of the balanced contiguous partition of T vectors over W
 // warps: warp w owns [start(w), start(w+1)), start(w) = floor(w T / W).

@@ -17,7 +17,7 @@
 // warp at the end of each row piece and publishes a 32-byte partial.  The
 // last warp to finish a row (atomic arrival counter, no waiting) merges the
 // row's partials in a fixed order and writes the row's results.
-#include "internal.h"
+#include "rules.cuh"
 
 namespace sdd {
 
@@ -158,8 +158,19 @@ __device__ __noinline__ int first_index(const char *rowp, int k0, int lane, int 
 // Sums are relative to the integer reference st.r (log2 units), so a new
 // maximum rescales by an exact power of two.  A new maximum only records the
 // tile (st.amax = k0); the exact index is resolved once at the end of the piece.
+// Error-free sum of two fp32 values (Knuth's TwoSum): a + b = s + err exactly.
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &err) {
+    s = a + b;
+    const float bb = s - a;
+    err = (a - (s - bb)) + (b - bb);
+}
+
+// The lane's running exp-sum is kept as an unevaluated fp32 pair (hi, lo)
+// (compensated summation), so the hot loop needs no fp64 arithmetic; the pair
+// is folded into st.s (fp64) at the end of each row piece.
 template <int DT>
-__device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lane, SoftState &st) {
+__device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lane, SoftState &st, float &s_hi,
+                                              float &s_lo) {
     uint4 w[kVPL];
 #pragma unroll
     for (int i = 0; i < kVPL; ++i) w[i] = clamp_vec<DT>(tile[lane + 32 * i]);
@@ -188,8 +199,10 @@ __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lan
         const float rn = ceilf(cm * kLog2e);
         if (rn > st.r) {
             const float k = st.r - rn;
-            st.t2 = pow2f_int(k) * (st.t2 + k * static_cast<float>(st.s));
-            st.s *= pow2d_int(k);
+            const float sc = pow2f_int(k);   // exact power of two (0 below the normal range)
+            st.t2 = sc * (st.t2 + k * (s_hi + s_lo));
+            s_hi *= sc;
+            s_lo *= sc;
             st.r = rn;
         }
     }
@@ -222,7 +235,10 @@ __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lan
             }
         }
     }
-    st.s += static_cast<double>(s0) + static_cast<double>(s1);
+    float e1, e2, h;
+    two_sum(s_hi, s0, h, e1);
+    two_sum(h, s1, s_hi, e2);
+    s_lo += e1 + e2;
     st.t2 += t0 + t1;
     return cm;
 }
@@ -296,6 +312,29 @@ __device__ void finalize_row(const ScanParams &p, int64_t r, SoftState st, int l
     G.rec[lr] = rec;
 }
 
+// A row of list block i is final: count it, and let the warp that completes
+// the block evaluate the block's decisions (rules.cuh).
+template <int DT>
+__device__ __forceinline__ void block_arrive(const ScanParams &p, int64_t r, int lane) {
+    const int gi = (r >= p.rows0) ? 1 : 0;
+    const int64_t lr = gi ? r - p.rows0 : r;
+    const int i = static_cast<int>(lr / p.grp[gi].npos);
+    __syncwarp();
+    uint32_t old = 0;
+    if (lane == 0) {
+        __threadfence();
+        old = atomicAdd(p.dec.blk_count + i, 1u);
+    }
+    old = __shfl_sync(0xFFFFFFFFu, old, 0);
+    if (old == static_cast<uint32_t>(p.dec.rows_per_block - 1)) {
+        __threadfence();
+        __shared__ int s_rule_L[kWarpsPerCta][kMaxRules], s_rule_corr[kWarpsPerCta][kMaxRules];
+        const int w = threadIdx.x >> 5;
+        block_decide<DT>(p.dec, i, lane, s_rule_L[w], s_rule_corr[w]);
+        if (lane == 0) p.dec.blk_count[i] = 0u;   // leave the workspace zeroed
+    }
+}
+
 template <int DT>
 __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant__ ScanParams p) {
     extern __shared__ __align__(128) unsigned char smem[];
@@ -343,6 +382,7 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
     for (int s = 0; s < kStages && pc.v < v1; ++s) issue(s);
 
     SoftState st = soft_identity();
+    float s_hi = 0.f, s_lo = 0.f;   // the lane's exp-sum as an fp32 pair
     bool in_piece = false;
     int tok = -1;          // drafted token of the current target row (-1: none)
     float g = 0.f;         // its clamped logit
@@ -355,6 +395,8 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
         const int n = static_cast<int>(min(static_cast<int64_t>(min(kTileVec, p.RV - cc.k)), v1 - cc.v));
         if (!in_piece) {
             st = soft_identity();
+            s_hi = 0.f;
+            s_lo = 0.f;
             int gi, j, b;
             int64_t lr;
             bool ok;
@@ -381,7 +423,7 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
         uint4 *tile = reinterpret_cast<uint4 *>(ring + slot * kTileBytes);
         const bool row_end = (cc.k + n == p.RV);
         if (n < kTileVec || (row_end && tail)) pad_tile<DT>(tile, n, lane, row_end, tail);
-        const float cm = process_tile<DT>(tile, cc.k, lane, st);
+        const float cm = process_tile<DT>(tile, cc.k, lane, st, s_hi, s_lo);
         if (rank_on) {
             const bool want = cm >= g;
             if (__any_sync(0xFFFFFFFFu, want)) {
@@ -410,11 +452,13 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
             if (st.m == M && st.amax != INT32_MAX) idx = first_index<DT>(crow, st.amax, lane, p.RV, p.V, M);
             st.amax = idx;
             st.rank = (lane == 0) ? wrank : 0;
+            st.s = static_cast<double>(s_hi) + static_cast<double>(s_lo);
             SoftState red = soft_warp_reduce(st);
             const int64_t fw = part_owner(cc.r * p.RV, p.T, p.W);
             const int64_t lw = part_owner((cc.r + 1) * p.RV - 1, p.T, p.W);
             if (fw == lw) {
                 finalize_row<DT>(p, cc.r, red, lane);
+                if (p.dec.enabled) block_arrive<DT>(p, cc.r, lane);
             } else {
                 if (lane == 0) {
                     Partial pt;
@@ -450,6 +494,7 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
                     acc = soft_warp_reduce(acc);
                     if (lane == 0) p.counters[cc.r] = 0u;  // leave the workspace zeroed
                     finalize_row<DT>(p, cc.r, acc, lane);
+                    if (p.dec.enabled) block_arrive<DT>(p, cc.r, lane);
                 }
             }
             in_piece = false;
