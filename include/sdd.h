@@ -27,8 +27,10 @@
  *   the legacy default stream) and returns without synchronising.
  * Workspace.  Calls that take `workspace` need at least sdd_workspace_size()
  *   bytes of device memory, 256-byte aligned and ZERO-FILLED before its first
- *   use; every call that completes returns the arrival counters it holds to
- *   zero, so one workspace serves any number of stream-ordered calls.  Calls that may
+ *   use; it holds the streaming kernel's per-warp partial statistics and the
+ *   sampling draw's per-segment totals and arrival counters.  Every call that
+ *   completes returns those counters to zero, so one workspace serves any
+ *   number of stream-ordered calls.  Calls that may
  *   overlap on the GPU (different streams) need separate workspaces.  After a
  *   call whose device status reports SDD_DEV_TIMEOUT the workspace must be
  *   zero-filled again.
@@ -38,8 +40,13 @@
  *   kernels run are OR-ed into the caller's device word `*status` (bits
  *   SDD_DEV_*; the caller clears it); no kernel traps.  sdd_last_error()
  *   returns a message for the calling thread's last non-OK return.
- * Dtypes.  Logits are SDD_F32 or SDD_BF16; all arithmetic is fp32 with fp64
- *   where sums and threshold comparisons need it.
+ * Dtypes.  Logits are SDD_F32 or SDD_BF16; all arithmetic is fp32, with
+ *   double-float (unevaluated fp32 pairs, about 48 significant bits) where sums,
+ *   log-normalisers and threshold comparisons need more; fp64 results (lse) are
+ *   converted from those pairs.
+ * Kernels.  Each statistics, verification or block call enqueues the
+ *   streaming kernel (one read of the logits) and then the decide kernel
+ *   (row finalisation, decisions, draws) as a programmatic dependent launch.
  */
 #ifndef SDD_H
 #define SDD_H
@@ -242,14 +249,14 @@ SDD_API sdd_status_t sdd_uniforms(uint64_t seed, const uint32_t *j, const uint32
  * loops that have no allocator at hand.  The paper has no counterpart; this is
  * a deployment convenience.
  * Same arguments, outputs, status bits and results as sdd_confidence, minus
- * the workspace.  The scratch is one file-scope device array of 672 KiB that
+ * the workspace.  The scratch is one file-scope device array of 384 KiB that
  * every GPU loading this library holds until the process exits; it serves
  * B * gamma <= 8192 drafter rows per call (larger batches are rejected with
  * SDD_ERR_INVALID_ARGUMENT before anything is enqueued).  The first call on a
  * device looks up the array's device address and the launch geometry for that
  * device (make that first call, on each device, before any stream capture).
- * Every call clears the arrival counters it needs on `stream`, then runs the
- * same streaming kernel as sdd_confidence.  All calls share the one array, so
+ * Every call runs the same streaming and decide kernels as sdd_confidence.  All
+ * calls share the one array, so
  * calls that may overlap on the GPU (different streams, or host threads without
  * ordering between them) race on it: order them on one stream.  No allocating
  * routine is called.
@@ -268,11 +275,13 @@ SDD_API sdd_status_t sdd_confidence_noalloc(const void *draft_logits, sdd_dtype_
  * read, agreement counters for every pair, and the tokens committed under pair
  * 0.  Array meanings and layouts are those of the single-purpose calls; NULL
  * output pointers are skipped.  sdd_block runs sdd_block_scan then
- * sdd_block_decide on the same stream.  sdd_block_scan streams every logit
- * once and, as each block's last row completes, evaluates that block's rules,
- * schedule, agreement counters and skip commits; sdd_block_decide completes the
- * sampling rule's residual / bonus draws (nothing to do when greedy != 0).  The
- * two halves are exported so that a caller can time the streaming pass alone.
+ * sdd_block_decide on the same stream, with the same args.  sdd_block_scan
+ * streams every logit once into per-warp partial statistics (the workspace);
+ * sdd_block_decide finalises every row, evaluates each block's rules,
+ * schedule, agreement counters and commits, and draws the sampling rule's
+ * residual / bonus tokens.  The two halves are exported so that a caller can
+ * time the streaming pass alone; sdd_block_decide must follow the
+ * sdd_block_scan of the same args on the same stream.
  */
 typedef struct sdd_block_args {
     /* inputs */

@@ -35,7 +35,8 @@ sdd_status_t cuda_fail(cudaError_t e, const char *what) {
 constexpr int kMaxDevices = 64;
 struct DevInfo {
     int sms;
-    int ctas_per_sm;
+    int ctas_per_sm;        // streaming kernel
+    int dec_ctas_per_sm;    // decide kernel
 };
 DevInfo g_dev[kMaxDevices];
 std::atomic<int> g_dev_ready[kMaxDevices];
@@ -53,6 +54,8 @@ sdd_status_t device_info(DevInfo &out) {
         if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
         di.ctas_per_sm = scan_max_ctas_per_sm();
         if (di.ctas_per_sm < 1) return fail(SDD_ERR_UNSUPPORTED, "streaming kernel does not fit on this device");
+        di.dec_ctas_per_sm = decide_max_ctas_per_sm();
+        if (di.dec_ctas_per_sm < 1) return fail(SDD_ERR_UNSUPPORTED, "decide kernel does not fit on this device");
         g_dev[d] = di;
         g_dev_ready[d].store(1, std::memory_order_release);
     }
@@ -64,10 +67,10 @@ inline size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255);
 
 // Workspace layout for blocks of shape (B, gamma) on a device with W_max warps.
 struct Layout {
-    size_t partials, counters, drec, trec, res_total, res_last, res_count, k0, blk_count, blk_L, total;
+    size_t partials, res_total, res_pref, res_last, res_count, total;
 };
 
-Layout layout(int64_t B, int64_t gamma, int64_t W_max) {
+Layout layout(int64_t B, int64_t gamma, int64_t W_max, int64_t dec_ctas) {
     Layout L{};
     const int64_t rows = B * (2 * gamma + 1);
     size_t o = 0;
@@ -77,15 +80,11 @@ Layout layout(int64_t B, int64_t gamma, int64_t W_max) {
         return at;
     };
     L.partials = take(static_cast<size_t>(rows + W_max) * sizeof(Partial));
-    L.counters = take(static_cast<size_t>(rows) * sizeof(uint32_t));
-    L.drec = take(static_cast<size_t>(B * gamma) * sizeof(RowRec));
-    L.trec = take(static_cast<size_t>(B * (gamma + 1)) * sizeof(RowRec));
-    L.res_total = take(static_cast<size_t>(B * kDrawMaxSeg) * sizeof(double));
+    L.res_total = take(static_cast<size_t>(B * kDrawMaxSeg) * sizeof(float));
+    // nb * nseg <= max(resident decide CTAs, B) (see init_dec)
+    L.res_pref = take(static_cast<size_t>(std::max(dec_ctas, B)) * kDecThreads * sizeof(float));
     L.res_last = take(static_cast<size_t>(B * kDrawMaxSeg) * sizeof(int32_t));
     L.res_count = take(static_cast<size_t>(B) * sizeof(uint32_t));
-    L.k0 = take(static_cast<size_t>(B) * sizeof(int32_t));
-    L.blk_count = take(static_cast<size_t>(B) * sizeof(uint32_t));
-    L.blk_L = take(static_cast<size_t>(B) * sizeof(int32_t));
     L.total = o;
     return L;
 }
@@ -117,6 +116,7 @@ struct Work {
     Layout L;
     int W_max;
     int sms;
+    int dec_ctas;   // decide-kernel CTAs resident at once on the device
 };
 
 sdd_status_t get_work(void *workspace, size_t bytes, int B, int gamma, Work &w) {
@@ -125,7 +125,8 @@ sdd_status_t get_work(void *workspace, size_t bytes, int B, int gamma, Work &w) 
     if (s != SDD_OK) return s;
     w.W_max = di.sms * di.ctas_per_sm * kWarpsPerCta;
     w.sms = di.sms;
-    w.L = layout(B, gamma, w.W_max);
+    w.dec_ctas = di.sms * di.dec_ctas_per_sm;
+    w.L = layout(B, gamma, w.W_max, w.dec_ctas);
     if (!workspace) return fail(SDD_ERR_WORKSPACE, "workspace is NULL");
     if (reinterpret_cast<uintptr_t>(workspace) % 256 != 0)
         return fail(SDD_ERR_WORKSPACE, "workspace is not 256-byte aligned");
@@ -146,67 +147,59 @@ void init_scan(ScanParams &p, const Work &w, sdd_dtype_t dtype, int B, int gamma
     p.B = B;
     p.tokens = tokens;
     p.partials = reinterpret_cast<Partial *>(w.base + w.L.partials);
-    p.counters = reinterpret_cast<uint32_t *>(w.base + w.L.counters);
     p.status = status;
 }
 
-// Fill in the totals of a ScanParams whose groups are set, and launch.
-sdd_status_t run_scan(ScanParams &p, const Work &w, cudaStream_t stream) {
+// Fill in the totals of a ScanParams whose groups are set.
+void finish_params(ScanParams &p, const Work &w) {
     p.rows0 = static_cast<int64_t>(p.grp[0].nb) * p.grp[0].npos;
     p.rows = p.rows0 + (p.n_groups > 1 ? static_cast<int64_t>(p.grp[1].nb) * p.grp[1].npos : 0);
     p.T = p.rows * p.RV;
+    p.W = static_cast<int32_t>(std::min<int64_t>(w.W_max, p.T));
+}
+
+// The streaming kernel over the rows of p.
+sdd_status_t run_scan(const ScanParams &p, cudaStream_t stream) {
     if (p.T == 0) return SDD_OK;
-    const int64_t W = std::min<int64_t>(w.W_max, p.T);
-    p.W = static_cast<int32_t>(W);
-    const int grid = static_cast<int>((W + kWarpsPerCta - 1) / kWarpsPerCta);
+    const int grid = static_cast<int>((static_cast<int64_t>(p.W) + kWarpsPerCta - 1) / kWarpsPerCta);
     cudaError_t e = launch_scan(p, grid, stream);
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     return SDD_OK;
 }
 
-// Block decisions evaluated inside the streaming kernel.
+// The decide kernel (row finalisation, decisions, draws) behind the streaming kernel.
+sdd_status_t run_decide(const ScanParams &p, cudaStream_t stream) {
+    if (p.T == 0) return SDD_OK;
+    cudaError_t e = launch_decide(p, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "decide launch");
+    return SDD_OK;
+}
+
+// Block decisions and, for the sampling rule, the draw geometry: each of the
+// nb blocks' draw rows is cut into nseg segments of whole kDecThreads-vector
+// chunks, as many as keep nb * nseg CTAs resident in one wave (at least two
+// vectors per thread, at most kDrawMaxSeg segments).
 void init_dec(DecideParams &d, const Work &w, sdd_dtype_t dtype, int B, int gamma, int V, int64_t row_stride,
-              const int32_t *tokens, int rows_per_block) {
+              const int32_t *tokens, int nb) {
     d.enabled = 1;
-    d.rows_per_block = rows_per_block;
     d.B = B;
     d.gamma = gamma;
     d.V = V;
     d.stride_bytes = row_stride * esize(dtype);
     d.tokens = tokens;
-    d.trec = reinterpret_cast<const RowRec *>(w.base + w.L.trec);
-    d.blk_count = reinterpret_cast<uint32_t *>(w.base + w.L.blk_count);
-    d.blk_L = reinterpret_cast<int32_t *>(w.base + w.L.blk_L);
-    d.k0 = reinterpret_cast<int32_t *>(w.base + w.L.k0);
+    d.res_total = reinterpret_cast<float *>(w.base + w.L.res_total);
+    d.res_pref = reinterpret_cast<float *>(w.base + w.L.res_pref);
+    d.res_last = reinterpret_cast<int32_t *>(w.base + w.L.res_last);
+    d.res_count = reinterpret_cast<uint32_t *>(w.base + w.L.res_count);
+    const int RV = static_cast<int>((static_cast<int64_t>(V) * esize(dtype) + 15) / 16);
+    const int want = std::max(1, std::min(kDrawMaxSeg, w.dec_ctas / std::max(nb, 1)));
+    const int per_thread = std::max(2, (RV + kDecThreads * want - 1) / (kDecThreads * want));
+    d.seg_vec = per_thread * kDecThreads;
+    d.nseg = (RV + d.seg_vec - 1) / d.seg_vec;
 }
 
-// The sampling draw: segments of whole 256-vector chunks, at most kDrawMaxSeg.
-void init_draw(DrawParams &q, const Work &w, sdd_dtype_t dtype, int B, int gamma, int V, int64_t row_stride,
-               const int32_t *tokens, int nb, const int32_t *bidx, int32_t *status) {
-    std::memset(&q, 0, sizeof q);
-    q.B = B;
-    q.gamma = gamma;
-    q.V = V;
-    q.RV = static_cast<int32_t>((static_cast<int64_t>(V) * esize(dtype) + 15) / 16);
-    q.dtype = dtype;
-    q.nb = nb;
-    q.bidx = bidx;
-    q.stride_bytes = row_stride * esize(dtype);
-    q.tokens = tokens;
-    q.trec = reinterpret_cast<const RowRec *>(w.base + w.L.trec);
-    q.blk_L = reinterpret_cast<const int32_t *>(w.base + w.L.blk_L);
-    q.res_total = reinterpret_cast<double *>(w.base + w.L.res_total);
-    q.res_last = reinterpret_cast<int32_t *>(w.base + w.L.res_last);
-    q.res_count = reinterpret_cast<uint32_t *>(w.base + w.L.res_count);
-    q.status = status;
-    // segments of 2 vectors per thread (more when the row needs > kDrawMaxSeg)
-    const int per_thread = std::max(2, (q.RV + kDrawThreads * kDrawMaxSeg - 1) / (kDrawThreads * kDrawMaxSeg));
-    q.seg_vec = per_thread * kDrawThreads;
-    q.nseg = (q.RV + q.seg_vec - 1) / q.seg_vec;
-}
-
-sdd_status_t set_thresholds(int signal, const double *eta_b, const double *eta_c, int n_tau, double *eta_loc,
-                            double *log_eta_c, int32_t *tau_off) {
+sdd_status_t set_thresholds(int signal, const double *eta_b, const double *eta_c, int n_tau, df *eta_loc,
+                            df *log_eta_c, int32_t *tau_off) {
     if (n_tau < 1 || n_tau > SDD_MAX_GRID)
         return fail(SDD_ERR_INVALID_ARGUMENT, "n_tau = %d outside [1, %d]", n_tau, SDD_MAX_GRID);
     if (!eta_b || !eta_c) return fail(SDD_ERR_INVALID_ARGUMENT, "eta_b / eta_c are NULL");
@@ -217,8 +210,8 @@ sdd_status_t set_thresholds(int signal, const double *eta_b, const double *eta_c
         if (std::isnan(eb) || std::isnan(ec)) return fail(SDD_ERR_INVALID_ARGUMENT, "threshold %d is NaN", t);
         tau_off[t] = (eb >= 1.0 || ec >= 1.0) ? 1 : 0;
         const double em = std::max(eb, ec);
-        eta_loc[t] = (signal == SDD_SIG_MARGINAL) ? em : eb;
-        log_eta_c[t] = (ec > 0.0) ? std::log(ec) : -INFINITY;
+        eta_loc[t] = df_from_double((signal == SDD_SIG_MARGINAL) ? em : eb);
+        log_eta_c[t] = df_from_double((ec > 0.0) ? std::log(ec) : -INFINITY);
     }
     return SDD_OK;
 }
@@ -232,7 +225,7 @@ sdd_status_t set_ell(DecideParams &d, const double *ell, int n_ell) {
         if (!(ell[r] > 0.0 && ell[r] <= 1.0))
             return fail(SDD_ERR_INVALID_ARGUMENT, "ell[%d] = %g outside (0, 1] (paper convention)", r, ell[r]);
         d.ell_one[r] = (ell[r] == 1.0) ? 1 : 0;
-        d.ell_thr[r] = std::log(ell[r]);
+        d.ell_thr[r] = df_from_double(std::log(ell[r]));
     }
     return SDD_OK;
 }
@@ -278,9 +271,10 @@ sdd_status_t target_scan(const Work &w, const void *target_logits, sdd_dtype_t d
     G.kind = 1;
     G.nb = n_rows;
     G.bidx = rows;
-    G.rec = reinterpret_cast<RowRec *>(w.base + w.L.trec);
     p.dec = dec;
-    return run_scan(p, w, stream);
+    finish_params(p, w);
+    SDD_TRY(run_scan(p, stream));
+    return run_decide(p, stream);
 }
 
 }  // namespace
@@ -302,7 +296,8 @@ sdd_status_t sdd_workspace_size(int B, int gamma, int V, size_t *bytes) {
     SDD_TRY(check_shape(SDD_BF16, B, gamma, V, ((static_cast<int64_t>(V) + 7) / 8) * 8));
     DevInfo di;
     SDD_TRY(device_info(di));
-    *bytes = layout(B, gamma, static_cast<int64_t>(di.sms) * di.ctas_per_sm * kWarpsPerCta).total;
+    *bytes = layout(B, gamma, static_cast<int64_t>(di.sms) * di.ctas_per_sm * kWarpsPerCta,
+                    static_cast<int64_t>(di.sms) * di.dec_ctas_per_sm).total;
     return SDD_OK;
 }
 
@@ -326,14 +321,16 @@ sdd_status_t sdd_confidence(const void *draft_logits, sdd_dtype_t dtype, int B, 
     G.npos = gamma;
     G.kind = 0;
     G.nb = B;
-    G.rec = reinterpret_cast<RowRec *>(w.base + w.L.drec);
     G.q = q;
     G.logq = logq;
     G.maxprob = maxprob;
     G.lse = lse;
     G.entropy = entropy;
     G.argmax = argmax;
-    return run_scan(p, w, reinterpret_cast<cudaStream_t>(stream));
+    finish_params(p, w);
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    SDD_TRY(run_scan(p, st));
+    return run_decide(p, st);
 }
 
 sdd_status_t sdd_schedule_prefix(const float *q, const float *logq, int B, int gamma, sdd_signal_t signal,
@@ -387,8 +384,8 @@ sdd_status_t sdd_verify_strict(const void *target_logits, const void *draft_logi
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     DecideParams d;
     std::memset(&d, 0, sizeof d);
-    init_dec(d, w, dtype, B, gamma, V, row_stride, draft_tokens, gamma + 1);
-    d.bidx = rows;
+    init_dec(d, w, dtype, B, gamma, V, row_stride, draft_tokens, n_rows);
+    d.zt = static_cast<const char *>(target_logits);
     d.zd = static_cast<const char *>(draft_logits);
     d.d_lse = draft_lse;
     d.do_strict = 1;
@@ -398,21 +395,7 @@ sdd_status_t sdd_verify_strict(const void *target_logits, const void *draft_logi
     d.L_strict = L;
     d.tok_strict = tokens;
     d.n_strict = n_commit;
-    SDD_TRY(target_scan(w, target_logits, dtype, B, gamma, V, row_stride, draft_tokens, rows, n_rows, 1, d, status, st));
-    if (greedy) return SDD_OK;
-    DrawParams q;
-    init_draw(q, w, dtype, B, gamma, V, row_stride, draft_tokens, n_rows, rows, status);
-    q.zt = static_cast<const char *>(target_logits);
-    q.zd = static_cast<const char *>(draft_logits);
-    q.d_lse = draft_lse;
-    q.seed = seed;
-    q.round = round;
-    q.L_strict = L;
-    q.tok_strict = tokens;
-    q.n_strict = n_commit;
-    cudaError_t e = launch_draw(q, st);
-    if (e != cudaSuccess) return cuda_fail(e, "draw launch");
-    return SDD_OK;
+    return target_scan(w, target_logits, dtype, B, gamma, V, row_stride, draft_tokens, rows, n_rows, 1, d, status, st);
 }
 
 sdd_status_t sdd_verify_lenient(const void *target_logits, sdd_dtype_t dtype, int B, int gamma, int V,
@@ -430,8 +413,7 @@ sdd_status_t sdd_verify_lenient(const void *target_logits, sdd_dtype_t dtype, in
     if (!draft_tokens) return fail(SDD_ERR_INVALID_ARGUMENT, "draft_tokens is NULL");
     Work w;
     SDD_TRY(get_work(workspace, workspace_bytes, B, gamma, w));
-    init_dec(d, w, dtype, B, gamma, V, row_stride, draft_tokens, gamma + 1);
-    d.bidx = rows;
+    init_dec(d, w, dtype, B, gamma, V, row_stride, draft_tokens, n_rows);
     d.L_len = L;
     d.tok_len = tokens;
     d.n_len = n_commit;
@@ -455,8 +437,7 @@ sdd_status_t sdd_verify_topk(const void *target_logits, sdd_dtype_t dtype, int B
     if (!draft_tokens) return fail(SDD_ERR_INVALID_ARGUMENT, "draft_tokens is NULL");
     Work w;
     SDD_TRY(get_work(workspace, workspace_bytes, B, gamma, w));
-    init_dec(d, w, dtype, B, gamma, V, row_stride, draft_tokens, gamma + 1);
-    d.bidx = rows;
+    init_dec(d, w, dtype, B, gamma, V, row_stride, draft_tokens, n_rows);
     d.L_topk = L;
     d.tok_topk = tokens;
     d.n_topk = n_commit;
@@ -508,7 +489,9 @@ static sdd_status_t block_check(const sdd_block_args *a) {
     return SDD_OK;
 }
 
-sdd_status_t sdd_block_scan(const sdd_block_args *a, sdd_stream_t stream) {
+// The launch parameters of one fused round, from its arguments (both halves
+// of sdd_block build the same ones).  Sets *empty when there is nothing to do.
+static sdd_status_t block_params(const sdd_block_args *a, ScanParams &p, bool *empty) {
     SDD_TRY(block_check(a));
     const sdd_dtype_t dt = static_cast<sdd_dtype_t>(a->dtype);
     DecideParams d;
@@ -517,10 +500,10 @@ sdd_status_t sdd_block_scan(const sdd_block_args *a, sdd_stream_t stream) {
     SDD_TRY(set_ell(d, a->ell, a->n_ell));
     int kcap = 1;
     SDD_TRY(set_topk(d, a->topk, a->n_k, kcap));
-    if (a->B == 0) return SDD_OK;
+    *empty = a->B == 0;
+    if (*empty) return SDD_OK;
     Work w;
     SDD_TRY(get_work(a->workspace, a->workspace_bytes, a->B, a->gamma, w));
-    ScanParams p;
     init_scan(p, w, dt, a->B, a->gamma, a->V, a->draft_tokens, a->status);
     p.n_groups = 2;
     p.kcap = kcap;
@@ -530,7 +513,6 @@ sdd_status_t sdd_block_scan(const sdd_block_args *a, sdd_stream_t stream) {
     D.npos = a->gamma;
     D.kind = 0;
     D.nb = a->B;
-    D.rec = reinterpret_cast<RowRec *>(w.base + w.L.drec);
     D.q = a->q;
     D.logq = a->logq;
     D.maxprob = a->maxprob;
@@ -543,11 +525,8 @@ sdd_status_t sdd_block_scan(const sdd_block_args *a, sdd_stream_t stream) {
     T.npos = a->gamma + 1;
     T.kind = 1;
     T.nb = a->B;
-    T.rec = reinterpret_cast<RowRec *>(w.base + w.L.trec);
-    // every rule, the schedule and the agreement counters run in this launch,
-    // by the warp that finalises each block's last row
-    init_dec(d, w, dt, a->B, a->gamma, a->V, a->row_stride, a->draft_tokens, 2 * a->gamma + 1);
-    d.drec = reinterpret_cast<const RowRec *>(w.base + w.L.drec);
+    init_dec(d, w, dt, a->B, a->gamma, a->V, a->row_stride, a->draft_tokens, a->B);
+    d.zt = static_cast<const char *>(a->target_logits);
     d.zd = static_cast<const char *>(a->draft_logits);
     d.do_strict = 1;
     d.greedy = a->greedy ? 1 : 0;
@@ -577,31 +556,24 @@ sdd_status_t sdd_block_scan(const sdd_block_args *a, sdd_stream_t stream) {
     d.commit_n = a->commit_n;
     d.agreement = reinterpret_cast<long long *>(a->agreement);
     p.dec = d;
-    return run_scan(p, w, reinterpret_cast<cudaStream_t>(stream));
+    finish_params(p, w);
+    return SDD_OK;
+}
+
+sdd_status_t sdd_block_scan(const sdd_block_args *a, sdd_stream_t stream) {
+    ScanParams p;
+    bool empty = false;
+    SDD_TRY(block_params(a, p, &empty));
+    if (empty) return SDD_OK;
+    return run_scan(p, reinterpret_cast<cudaStream_t>(stream));
 }
 
 sdd_status_t sdd_block_decide(const sdd_block_args *a, sdd_stream_t stream) {
-    SDD_TRY(block_check(a));
-    if (a->B == 0 || a->greedy) return SDD_OK;   // greedy rounds are complete after the scan
-    const sdd_dtype_t dt = static_cast<sdd_dtype_t>(a->dtype);
-    Work w;
-    SDD_TRY(get_work(a->workspace, a->workspace_bytes, a->B, a->gamma, w));
-    DrawParams q;
-    init_draw(q, w, dt, a->B, a->gamma, a->V, a->row_stride, a->draft_tokens, a->B, nullptr, a->status);
-    q.zt = static_cast<const char *>(a->target_logits);
-    q.zd = static_cast<const char *>(a->draft_logits);
-    q.drec = reinterpret_cast<const RowRec *>(w.base + w.L.drec);
-    q.seed = a->seed;
-    q.round = a->round;
-    q.k0 = reinterpret_cast<const int32_t *>(w.base + w.L.k0);
-    q.L_strict = a->L_strict;
-    q.tok_strict = a->tokens_strict;
-    q.n_strict = a->n_strict;
-    q.commit_tokens = a->commit_tokens;
-    q.commit_n = a->commit_n;
-    cudaError_t e = launch_draw(q, reinterpret_cast<cudaStream_t>(stream));
-    if (e != cudaSuccess) return cuda_fail(e, "draw launch");
-    return SDD_OK;
+    ScanParams p;
+    bool empty = false;
+    SDD_TRY(block_params(a, p, &empty));
+    if (empty) return SDD_OK;
+    return run_decide(p, reinterpret_cast<cudaStream_t>(stream));
 }
 
 sdd_status_t sdd_block(const sdd_block_args *a, sdd_stream_t stream) {

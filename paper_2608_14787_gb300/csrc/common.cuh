@@ -44,27 +44,125 @@ __device__ __forceinline__ double pow2d_int(float k) {
 // ---------------------------------------------------------------------------
 // Partial softmax state of one warp's piece of one row.  Sums are taken
 // relative to an integer reference r in log2 units:
-//   s = sum 2^(z log2(e) - r),  t2 = sum 2^(z log2(e) - r) (z log2(e) - r).
+//   s = sum 2^(z log2(e) - r)  (kept as an unevaluated fp32 pair sh + sl),
+//   t2 = sum 2^(z log2(e) - r) (z log2(e) - r).
 struct __align__(32) Partial {
     float m;        // max of the clamped logits of the piece
     float r;        // integer reference (log2 units), >= m log2(e) up to rounding
     float t2;       // entropy accumulator (drafter rows)
+    float sh, sl;   // exp-sum as a double-float
     int32_t amax;   // lowest index attaining m (INT32_MAX if none)
-    int32_t rank;   // saturated count of entries ranked before the drafted token
-    int32_t pad;
-    double s;
+    int32_t rank;   // saturated count of entries ranked before the drafted token; -1: token out of range
+    float g;        // clamped logit of the row's drafted token (NaN if the row has none)
 };
 
-// Final statistics of one row, written by the warp that merges its partials.
-struct __align__(32) RowRec {
-    double lse;     // log sum_v exp(z(v)) in fp64
-    float M;        // max of the clamped logits
-    float g;        // clamped logit of the drafted token (NaN if the row has none)
-    float q;        // exp(g - lse)
-    float logq;     // g - lse
-    int32_t argmax; // lowest index attaining M, -1 if the row is invalid
-    int32_t rank;   // target rows: saturated rank of the drafted token
+// ---------------------------------------------------------------------------
+// Double-float arithmetic: a value is an unevaluated pair hi + lo of fp32
+// numbers with |lo| <= ulp(hi) / 2.  Built on the error-free transformations
+// TwoSum (Knuth) and FastTwoSum (Dekker) and on the FMA residual of a product;
+// used wherever the path needs more than fp32 precision, because fp64
+// instructions issue at a small fraction of the fp32 rate on this part.
+// ---------------------------------------------------------------------------
+constexpr float kLn2Hi = 0.693147182464599609375f;    // fp32 nearest ln 2
+constexpr float kLn2Lo = -1.9046542121259336e-09f;    // ln 2 - kLn2Hi
+
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &err) {
+    s = a + b;
+    const float bb = s - a;
+    err = (a - (s - bb)) + (b - bb);
+}
+// Requires |a| >= |b| (or a == 0).
+__device__ __forceinline__ void fast_two_sum(float a, float b, float &s, float &err) {
+    s = a + b;
+    err = b - (s - a);
+}
+
+struct df {
+    float hi, lo;
 };
+
+// A non-finite hi carries lo = 0, so infinities and NaN propagate through hi
+// alone and never form inf - inf in lo.
+__device__ __forceinline__ df df_make(float h, float l) {
+    df r;
+    if (!isfinite(h)) return df{h, 0.f};
+    two_sum(h, l, r.hi, r.lo);   // no ordering precondition: the lo part may exceed a cancelled hi
+    if (!isfinite(r.hi)) r.lo = 0.f;
+    return r;
+}
+__device__ __forceinline__ df df_add(df a, df b) {
+    float s, e;
+    two_sum(a.hi, b.hi, s, e);
+    if (!isfinite(s)) return df{s, 0.f};
+    return df_make(s, e + (a.lo + b.lo));
+}
+__device__ __forceinline__ df df_sub(df a, df b) { return df_add(a, df{-b.hi, -b.lo}); }
+// a - b for two fp32 numbers, exactly.
+__device__ __forceinline__ df df_diff(float a, float b) {
+    df r;
+    two_sum(a, -b, r.hi, r.lo);
+    if (!isfinite(r.hi)) r.lo = 0.f;
+    return r;
+}
+// a * b for an fp32 b (relative error ~2^-46).
+__device__ __forceinline__ df df_mul_f(df a, float b) {
+    const float p = a.hi * b;
+    if (!isfinite(p)) return df{p, 0.f};
+    const float e = fmaf(a.hi, b, -p);
+    return df_make(p, fmaf(a.lo, b, e));
+}
+// a >= b; infinities compare by their hi parts.
+__device__ __forceinline__ bool df_ge(df a, df b) {
+    if (!isfinite(a.hi) || !isfinite(b.hi)) return a.hi >= b.hi;
+    return a.hi > b.hi || (a.hi == b.hi && a.lo >= b.lo);
+}
+// Host-side split of a double into a double-float (exact to ~2^-48 relative).
+__host__ __device__ inline df df_from_double(double x) {
+    df r;
+    r.hi = static_cast<float>(x);
+    r.lo = 0.f;
+    if (r.hi - r.hi == 0.f) r.lo = static_cast<float>(x - static_cast<double>(r.hi));   // hi finite
+    return r;
+}
+
+// Natural logarithm of a positive double-float x = xh + xl with xh normal and
+// 2^-126 < x < 2^126, to about 1e-9 absolute, in fp32 arithmetic only:
+// x = 2^k m (1 + xl / xh) with m in [sqrt(1/2), sqrt(2)), and
+// ln x = k ln 2 + 2 atanh(u),  u = (m - 1 + l) / (m + 1 + l),  l = xl 2^-k,
+// where |u| <= 0.1716 and the series 2 (u + u^3/3 + ... + u^13/13) is exact to
+// 5e-13; its leading term 2u is carried as a double-float (the quotient
+// corrected by its FMA residual), the rest in fp32.
+__device__ __forceinline__ df ln_df(float xh, float xl) {
+    const uint32_t bits = __float_as_uint(xh);
+    int k = static_cast<int>((bits >> 23) & 0xFFu) - 127;
+    float m = __uint_as_float((bits & 0x007FFFFFu) | 0x3F800000u);   // [1, 2)
+    if (m > 1.41421354f) {
+        m *= 0.5f;
+        k += 1;
+    }
+    const float l = xl * __uint_as_float(static_cast<uint32_t>(127 - k) << 23);   // xl 2^-k
+    float fh, fl, dh, dl;
+    two_sum(m - 1.f, l, fh, fl);            // m - 1 is exact
+    two_sum(m, 1.f, dh, dl);
+    dl += l;
+    const float uh = __fdividef(fh, dh);
+    const float res = fmaf(-uh, dh, fh) + (fl - uh * dl);
+    const float ul = __fdividef(res, dh);
+    const float v = uh * uh;
+    float poly = 1.f / 13.f;
+    poly = fmaf(poly, v, 1.f / 11.f);
+    poly = fmaf(poly, v, 1.f / 9.f);
+    poly = fmaf(poly, v, 1.f / 7.f);
+    poly = fmaf(poly, v, 1.f / 5.f);
+    poly = fmaf(poly, v, 1.f / 3.f);
+    const float tail = 2.f * uh * v * poly;
+    const float kf = static_cast<float>(k);
+    const float a = kf * kLn2Hi;
+    const float ae = fmaf(kf, kLn2Hi, -a);
+    float s, e;
+    two_sum(a, 2.f * uh, s, e);
+    return df_make(s, e + ((ae + kf * kLn2Lo) + (2.f * ul + tail)));
+}
 
 // ---------------------------------------------------------------------------
 // Packed fp32 pair arithmetic (sm_100-family f32x2 instructions)
@@ -105,6 +203,19 @@ __device__ __forceinline__ float ex2(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
+}
+
+__device__ __forceinline__ float qnan() { return __int_as_float(0x7FC00000); }
+
+// One logit of a row (bf16 widened exactly to fp32).
+template <int DT>
+__device__ __forceinline__ float logit_at(const char *rowp, int v) {
+    if (DT == SDD_BF16) {
+        const uint16_t h = __ldg(reinterpret_cast<const unsigned short *>(rowp) + v);
+        return __uint_as_float(static_cast<uint32_t>(h) << 16);
+    } else {
+        return __ldg(reinterpret_cast<const float *>(rowp) + v);
+    }
 }
 
 // NaN-propagating maxima: a NaN logit must poison its row, never vanish.
@@ -169,6 +280,32 @@ __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t by
 }
 
 // ---------------------------------------------------------------------------
+// Programmatic dependent launch: a grid launched with the programmatic
+// stream-serialization attribute may be scheduled before the grid ahead of it
+// in the stream completes; griddep_wait() blocks until that grid has completed
+// and its memory operations are visible (a no-op for an ordinary launch).
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Launch `kernel` behind the previous work of `stream` as a programmatic
+// dependent grid (host side).
+template <class Params>
+inline cudaError_t launch_dependent(void (*kernel)(Params), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                                    const Params &p) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, p);
+}
+
+// ---------------------------------------------------------------------------
 // Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11) and the uniform mapping
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
@@ -200,11 +337,12 @@ enum : uint32_t { kPurposeAccept = 0, kPurposeResid = 1, kPurposeBonus = 2 };
 
 // ---------------------------------------------------------------------------
 // Online-softmax state and its merge.  All rescaling is by exact powers of
-// two (the references are integers), so merging never rounds the scale.
+// two (the references are integers), so merging never rounds the scale; the
+// exp-sum stays a double-float throughout.
 // ---------------------------------------------------------------------------
 struct SoftState {
     float m, r, t2;
-    double s;
+    float sh, sl;
     int32_t amax, rank;
 };
 
@@ -213,20 +351,24 @@ __device__ __forceinline__ SoftState soft_identity() {
     z.m = clamp_floor();
     z.r = clamp_ref();
     z.t2 = 0.f;
-    z.s = 0.0;
+    z.sh = 0.f;
+    z.sl = 0.f;
     z.amax = INT32_MAX;
     z.rank = 0;
     return z;
 }
 
-__device__ __forceinline__ SoftState soft_merge(SoftState a, SoftState b) {
+__device__ __forceinline__ SoftState soft_merge(const SoftState &a, const SoftState &b) {
     SoftState o;
     o.m = fmax_nan(a.m, b.m);
     o.r = fmaxf(a.r, b.r);
     const float ka = a.r - o.r, kb = b.r - o.r;  // integers <= 0
-    // t2 relative to R: 2^k (t2 + k s)
-    o.t2 = pow2f_int(ka) * (a.t2 + ka * static_cast<float>(a.s)) + pow2f_int(kb) * (b.t2 + kb * static_cast<float>(b.s));
-    o.s = a.s * pow2d_int(ka) + b.s * pow2d_int(kb);
+    const float pa = pow2f_int(ka), pb = pow2f_int(kb);
+    // t2 relative to the new reference: 2^k (t2 + k s)
+    o.t2 = pa * fmaf(ka, a.sh + a.sl, a.t2) + pb * fmaf(kb, b.sh + b.sl, b.t2);
+    float h, e;
+    two_sum(a.sh * pa, b.sh * pb, h, e);
+    fast_two_sum(h, fmaf(a.sl, pa, fmaf(b.sl, pb, e)), o.sh, o.sl);
     if (b.m > a.m)
         o.amax = b.amax;
     else if (b.m < a.m)
@@ -244,7 +386,8 @@ __device__ __forceinline__ SoftState soft_warp_reduce(SoftState v) {
         o.m = __shfl_xor_sync(0xFFFFFFFFu, v.m, off);
         o.r = __shfl_xor_sync(0xFFFFFFFFu, v.r, off);
         o.t2 = __shfl_xor_sync(0xFFFFFFFFu, v.t2, off);
-        o.s = __shfl_xor_sync(0xFFFFFFFFu, v.s, off);
+        o.sh = __shfl_xor_sync(0xFFFFFFFFu, v.sh, off);
+        o.sl = __shfl_xor_sync(0xFFFFFFFFu, v.sl, off);
         o.amax = __shfl_xor_sync(0xFFFFFFFFu, v.amax, off);
         o.rank = __shfl_xor_sync(0xFFFFFFFFu, v.rank, off);
         // merge in a fixed order (lower lane first) so every lane agrees bitwise

@@ -1,12 +1,23 @@
 // decide.cu -- the kernels that run after (or beside) the streaming pass.
 //
-//  * draw_kernel      -- the inverse-CDF draw of the speculative-sampling rule
-//                        cited by Sec. 3.1: at the first rejected position the
-//                        residual norm(max(0, p_t - p_d)), or, when the whole
-//                        block is accepted, p_t of the bonus row.  The draw row
-//                        is split into segments, one CTA each; the last segment
-//                        to finish (atomic arrival, no waiting) locates the
-//                        segment holding u * R and rescans it.
+//  * decide_kernel    -- one CTA per (listed block, draw segment), launched as
+//                        a programmatic dependent of the streaming grid.
+//                        Phase 1: every CTA finalises all rows of its block,
+//                        one row per thread, into shared memory (rules.cuh).
+//                        Phase 2 (sampling rule): every CTA takes the strict
+//                        accepted length L.  Phase 3: the inverse-CDF draw of
+//                        the speculative-sampling rule cited by Sec. 3.1 --
+//                        at the first rejected position the residual
+//                        norm(max(0, p_t - p_d)), or, when the whole block is
+//                        accepted, p_t of the bonus row: each CTA sums its
+//                        segment of the draw row and publishes its per-thread
+//                        prefix sums; the last to finish (atomic arrival, no
+//                        waiting) locates the segment, then the thread, from
+//                        those sums, and searches that thread's run with one
+//                        warp.  Last, the segment-0 CTA evaluates every other
+//                        rule (lenience, top-k; greedy strict), the skip
+//                        schedule, agreement counters and commits, one warp
+//                        per rule or threshold pair.
 //  * schedule_kernel  -- the skip policy of Sec. 4.1 as a stand-alone call.
 //  * agreement_kernel, commit_kernel, uniforms_kernel -- small stand-alone calls.
 #include "rules.cuh"
@@ -21,19 +32,19 @@ struct DrawCtx {
     float nrt, nrd, d_hi, d_lo;
 };
 
-__device__ __forceinline__ DrawCtx draw_ctx(const char *zt_row, const char *zd_row, double lse_t, double lse_d) {
+__device__ __forceinline__ DrawCtx draw_ctx(const char *zt_row, const char *zd_row, df lse_t, df lse_d) {
     DrawCtx c;
     c.zt_row = zt_row;
     c.zd_row = zd_row;
-    c.nrt = -ceilf(static_cast<float>(lse_t * kLog2ed));
+    c.nrt = -ceilf(lse_t.hi * kLog2e);
     c.nrd = 0.f;
     c.d_hi = 0.f;
     c.d_lo = 0.f;
     if (zd_row) {
-        c.nrd = -ceilf(static_cast<float>(lse_d * kLog2ed));
-        const double D = lse_t - lse_d;
-        c.d_hi = static_cast<float>(D);
-        c.d_lo = static_cast<float>(D - static_cast<double>(c.d_hi));
+        c.nrd = -ceilf(lse_d.hi * kLog2e);
+        const df D = df_sub(lse_t, lse_d);
+        c.d_hi = D.hi;
+        c.d_lo = D.lo;
     }
     return c;
 }
@@ -55,51 +66,89 @@ __device__ __forceinline__ float expm1_pos(float x) {
     return ex2(x * kLog2e) - 1.f;
 }
 
-// Weights of the draw for the EPV entries of one 16-byte vector.
+// Weight of one entry of the draw row (fp32; the product is rounded, never
+// fused into a following sum, so every pass sees the same weight):
 //   residual: p_t - p_d = p_d (exp(D(v)) - 1) with the log-ratio
 //             D(v) = (z_t(v) - z_d(v)) - (LSE_t - LSE_d); the LSE difference is
 //             applied as two fp32 terms (hi + lo) and the difference by expm1, so
 //             no cancellation between near-equal p_t and p_d loses precision;
 //             p_d(v) = 2^(z_d(v) log2(e) - r_d) up to the common factor of the row;
 //   bonus (zd_row == nullptr): 2^(z_t(v) log2(e) - r_t).
-// Returns the fp32 sum of the entries in ascending order.
+// Entries past V weigh 0.
+__device__ __forceinline__ float entry_weight(const DrawCtx &c, float zt, float zd, int v, int V) {
+    zt = fmax_nan(zt, clamp_floor());
+    zd = fmax_nan(zd, clamp_floor());
+    float w;
+    if (c.zd_row) {
+        const float dv = ((zt - zd) - c.d_hi) - c.d_lo;
+        w = (dv > 0.f) ? __fmul_rn(ex2(fmaf(zd, kLog2e, c.nrd)), expm1_pos(dv)) : 0.f;
+    } else {
+        w = ex2(fmaf(zt, kLog2e, c.nrt));
+    }
+    return (v < V) ? w : 0.f;
+}
+
+// Entry e of a 16-byte vector of logits, widened to fp32.
+template <int DT>
+__device__ __forceinline__ float vec_entry(const uint4 &a, int e) {
+    const uint32_t *u = reinterpret_cast<const uint32_t *>(&a);
+    if (DT == SDD_BF16) return (e & 1) ? bf16_hi(u[e >> 1]) : bf16_lo(u[e >> 1]);
+    return __uint_as_float(u[e]);
+}
+
+// Weights of the draw for the EPV entries of one 16-byte vector; returns
+// their fp32 sum in ascending order.
 template <int DT>
 __device__ __forceinline__ float vec_weights(const DrawCtx &c, uint4 a, uint4 d, int vec, int V, float (&w)[8]) {
     constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
-    const uint32_t *ua = reinterpret_cast<const uint32_t *>(&a);
-    const uint32_t *ud = reinterpret_cast<const uint32_t *>(&d);
     float sum = 0.f;
 #pragma unroll
     for (int e = 0; e < EPV; ++e) {
-        float zt, zd;
-        if (DT == SDD_BF16) {
-            zt = (e & 1) ? bf16_hi(ua[e >> 1]) : bf16_lo(ua[e >> 1]);
-            zd = (e & 1) ? bf16_hi(ud[e >> 1]) : bf16_lo(ud[e >> 1]);
-        } else {
-            zt = __uint_as_float(ua[e]);
-            zd = __uint_as_float(ud[e]);
-        }
-        zt = fmax_nan(zt, clamp_floor());
-        zd = fmax_nan(zd, clamp_floor());
-        float wv;
-        if (c.zd_row) {
-            const float dv = ((zt - zd) - c.d_hi) - c.d_lo;
-            wv = 0.f;
-            if (dv > 0.f) wv = ex2(fmaf(zd, kLog2e, c.nrd)) * expm1_pos(dv);
-        } else {
-            wv = ex2(fmaf(zt, kLog2e, c.nrt));
-        }
-        if (vec * EPV + e >= V) wv = 0.f;
-        w[e] = wv;
-        sum += wv;
+        w[e] = entry_weight(c, vec_entry<DT>(a, e), vec_entry<DT>(d, e), vec * EPV + e, V);
+        sum += w[e];
     }
     return sum;
 }
 
-// Inclusive scan of one fp32 value per thread over the CTA (kDrawThreads).
+// The first entry of vectors [vb, ve) at which the running weight sum exceeds
+// rem (a double-float), by one warp: 32 entries at a time, one per lane, a
+// warp prefix sum and a ballot.  If rounding leaves no such entry, the last
+// entry of positive weight; -1 if there is none.
+template <int DT>
+__device__ __forceinline__ int warp_search(const DrawCtx &c, int vb, int ve, int V, df rem, int lane) {
+    constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
+    const int n = (ve - vb) * EPV;
+    float carry = 0.f;
+    int lastp = -1;
+    for (int k0 = 0; k0 < n; k0 += 32) {
+        const int k = k0 + lane;
+        float w = 0.f;
+        if (k < n) {
+            const int vec = vb + k / EPV, e = k % EPV;
+            const uint4 a = __ldg(reinterpret_cast<const uint4 *>(c.zt_row) + vec);
+            const uint4 d = c.zd_row ? __ldg(reinterpret_cast<const uint4 *>(c.zd_row) + vec) : make_uint4(0, 0, 0, 0);
+            w = entry_weight(c, vec_entry<DT>(a, e), vec_entry<DT>(d, e), vec * EPV + e, V);
+        }
+        float run = w;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const float t = __shfl_up_sync(0xFFFFFFFFu, run, off);
+            if (lane >= off) run += t;
+        }
+        run += carry;
+        const unsigned hit = __ballot_sync(0xFFFFFFFFu, w > 0.f && !df_ge(rem, df{run, 0.f}));
+        if (hit) return vb * EPV + k0 + __ffs(hit) - 1;
+        const unsigned pos = __ballot_sync(0xFFFFFFFFu, w > 0.f);
+        if (pos) lastp = vb * EPV + k0 + 31 - __clz(pos);
+        carry = __shfl_sync(0xFFFFFFFFu, run, 31);
+    }
+    return lastp;
+}
+
+// Inclusive scan of one fp32 value per thread over the CTA (kDecThreads).
 // Returns the thread's inclusive value; *total receives the CTA total.
 __device__ __forceinline__ float cta_incl_scan(float v, float *warp_tot, float *total) {
-    constexpr int NW = kDrawThreads / 32;
+    constexpr int NW = kDecThreads / 32;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
@@ -157,11 +206,10 @@ __device__ __forceinline__ float run_sum(const DrawCtx &c, int vb, int ve, int V
     return sum;
 }
 
-// The first entry of vectors [vb, ve) whose running sum, starting at `start`,
-// exceeds `target` (same order and arithmetic as run_sum); -1 if none.
+// The first entry of vectors [vb, ve) whose running sum (same order and
+// arithmetic as run_sum) exceeds rem, a double-float; -1 if none.
 template <int DT>
-__device__ __forceinline__ int run_find(const DrawCtx &c, int vb, int ve, int V, double start, double target,
-                                        int &last_pos) {
+__device__ __forceinline__ int run_find(const DrawCtx &c, int vb, int ve, int V, df rem, int &last_pos) {
     constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
     float sum = 0.f;
     for (int vec = vb; vec < ve; ++vec) {
@@ -174,7 +222,7 @@ __device__ __forceinline__ int run_find(const DrawCtx &c, int vb, int ve, int V,
             sum += w[e];
             if (w[e] > 0.f) {
                 last_pos = vec * EPV + e;
-                if (start + static_cast<double>(sum) > target) return vec * EPV + e;
+                if (!df_ge(rem, df{sum, 0.f})) return vec * EPV + e;
             }
         }
     }
@@ -182,11 +230,12 @@ __device__ __forceinline__ int run_find(const DrawCtx &c, int vb, int ve, int V,
 }
 
 // Inverse CDF over vectors [v0, v1) of the draw row, one contiguous run of
-// `vpt` vectors per thread: returns the drawn index (or the last positive
-// entry if rounding leaves none), identical in every thread.
+// `vpt` vectors per thread: the first entry at which the running sum exceeds
+// rem (a double-float), or the last positive entry if rounding leaves none;
+// identical in every thread.
 template <int DT>
-__device__ int cta_find(const DrawCtx &c, int v0, int v1, int vpt, int V, double before, double target,
-                        float *s_warp, int *s_thr, int *s_tok) {
+__device__ int cta_find(const DrawCtx &c, int v0, int v1, int vpt, int V, df rem, float *s_warp, int *s_thr,
+                        int *s_tok) {
     const int vb = min(v1, v0 + static_cast<int>(threadIdx.x) * vpt), ve = min(v1, vb + vpt);
     int lastp = -1;
     const float ts = run_sum<DT>(c, vb, ve, V, lastp);
@@ -194,7 +243,7 @@ __device__ int cta_find(const DrawCtx &c, int v0, int v1, int vpt, int V, double
     const float incl = cta_incl_scan(ts, s_warp, &tot);
     if (threadIdx.x == 0) *s_thr = INT32_MAX;
     __syncthreads();
-    const bool mine = (ve > vb) && (before + static_cast<double>(incl) > target);
+    const bool mine = (ve > vb) && !df_ge(rem, df{incl, 0.f});
     const unsigned bal = __ballot_sync(0xFFFFFFFFu, mine);
     if ((threadIdx.x & 31) == 0 && bal) atomicMin(s_thr, static_cast<int>(threadIdx.x) + __ffs(bal) - 1);
     __syncthreads();
@@ -202,141 +251,351 @@ __device__ int cta_find(const DrawCtx &c, int v0, int v1, int vpt, int V, double
     if (thr == INT32_MAX) return -1;
     if (static_cast<int>(threadIdx.x) == thr) {
         int lp = -1;
-        const int pick = run_find<DT>(c, vb, ve, V, before + static_cast<double>(incl - ts), target, lp);
+        const int pick = run_find<DT>(c, vb, ve, V, df_sub(rem, df{incl - ts, 0.f}), lp);
         *s_tok = (pick >= 0) ? pick : lp;
     }
     __syncthreads();
     return *s_tok;
 }
 
+// Skip schedule of threshold pair t for a block (Sec. 4.1), by one warp, from
+// the drafter facts: prefix sums of ln q as double-floats, then sched_step
+// chunk by chunk and sched_final.
+__device__ __forceinline__ void sched_pair(const DecideParams &d, const BlockFacts &F, int t, bool force, int D,
+                                           int lane, int &Kh, int &K, int &Do) {
+    Kh = K = Do = 0;
+    if (force || d.tau_off[t]) return;
+    const int gamma = d.gamma;
+    int kb = gamma, best = 0;
+    df carry = df{0.f, 0.f};
+    for (int c = 0; c < gamma && kb >= c; c += 32) {
+        const int j = c + lane;
+        const bool in = j < gamma;
+        const df S = df_add(carry, warp_prefix_df(in ? df{F.d_lq[j], 0.f} : df{0.f, 0.f}, lane));
+        carry.hi = __shfl_sync(0xFFFFFFFFu, S.hi, 31);
+        carry.lo = __shfl_sync(0xFFFFFFFFu, S.lo, 31);
+        sched_step(c, lane, gamma, in, in ? F.d_q[j] : 0.f, in && F.guard[j] != 0, S, d.eta_loc[t], d.log_eta_c[t],
+                   d.signal, kb, best);
+    }
+    Kh = (d.signal == SDD_SIG_MARGINAL) ? kb : best;
+    sched_final(Kh, D, d.K_min, d.S_max, K, Do);
+}
+
 template <int DT>
-__global__ void __launch_bounds__(kDrawThreads) draw_kernel(const __grid_constant__ DrawParams p) {
+__global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_constant__ ScanParams p) {
+    griddep_wait();   // launched behind the streaming grid that wrote the partials
+    const DecideParams &d = p.dec;
     const int i = blockIdx.x;       // listed block
     const int seg = blockIdx.y;     // segment of the draw row
+    const bool leader = seg == 0;   // writes the block's outputs
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    constexpr int NW = kDecThreads / 32;
     const int gamma = p.gamma;
-    const int b = p.bidx ? __ldg(p.bidx + i) : i;
-    if (b < 0 || b >= p.B) return;  // flagged by the streaming pass
-    __shared__ float s_warp[2 * (kDrawThreads / 32)];
-    __shared__ int s_is_last, s_seg, s_lastp, s_thr, s_tok, s_L;
-    __shared__ double s_target, s_before;
-    __shared__ double s_tot[kDrawMaxSeg];
-    __shared__ int s_last[kDrawMaxSeg];
-    __shared__ DrawCtx s_ctx;
 
-    // the draw row and its context, once per CTA
-    if (threadIdx.x == 0) {
-        const int L = p.blk_L[i];
-        const double lse_t = p.trec[static_cast<int64_t>(i) * (gamma + 1) + L].lse;
-        double lse_d = 0.0;
-        if (L < gamma)
-            lse_d = p.drec ? p.drec[static_cast<int64_t>(i) * gamma + L].lse
-                           : p.d_lse[static_cast<int64_t>(b) * gamma + L];
-        const char *zt_row = p.zt + (static_cast<int64_t>(b) * (gamma + 1) + L) * p.stride_bytes;
-        const char *zd_row = (L < gamma) ? p.zd + (static_cast<int64_t>(b) * gamma + L) * p.stride_bytes : nullptr;
-        s_ctx = draw_ctx(zt_row, zd_row, lse_t, lse_d);
-        s_L = L;
-        s_lastp = -1;
+    __shared__ BlockFacts F;
+    __shared__ int s_L[kMaxRules], s_corr[kMaxRules];
+    __shared__ int s_K0, s_force, s_D;
+
+    int gd = -1, gt = -1;
+    for (int gi = 0; gi < p.n_groups; ++gi) {
+        if (p.grp[gi].kind == 0)
+            gd = gi;
+        else
+            gt = gi;
+    }
+    const int32_t *bidx = p.grp[0].bidx;
+    const int b = bidx ? __ldg(bidx + i) : i;
+    if (b < 0 || b >= p.B) {
+        if (leader && tid == 0) status_or(p.status, SDD_DEV_BAD_TOKEN);
+        return;
+    }
+    const bool dec = d.enabled != 0;
+    const bool sampling = dec && d.do_strict && !d.greedy;
+    const bool has_d = gd >= 0;
+    const bool alone_d = !has_d && sampling;   // drafter facts from the caller's LSE
+    const int nd = (has_d || alone_d) ? gamma : 0;
+    const int nt = (gt >= 0) ? gamma + 1 : 0;
+    const int64_t ob = static_cast<int64_t>(b) * gamma;
+    const int64_t bo = static_cast<int64_t>(b) * (gamma + 1);
+
+    // ---- phase 1: facts of every row of the block, one row per thread ----
+    if (dec) {
+        for (int j = tid; j < gamma; j += kDecThreads) {
+            F.x[j] = __ldg(d.tokens + ob + j);
+            F.guard[j] = d.guard ? d.guard[ob + j] : 0;
+        }
+        if (tid == 0) {
+            s_force = d.force_strict ? d.force_strict[b] : 0;
+            s_D = d.D_in ? d.D_in[b] : 0;
+        }
+    }
+    for (int s = tid; s < nd + nt; s += kDecThreads) {
+        if (s < nd) {
+            const int j = s;
+            RowFacts f;
+            if (has_d) {
+                const ScanGroup &G = p.grp[gd];
+                SoftState acc;
+                float g;
+                bool bad;
+                merge_row(p, (gd ? p.rows0 : 0) + static_cast<int64_t>(i) * G.npos + j, acc, g, bad);
+                f = row_final(p, G, j, b, acc, g, bad, leader);
+            } else {
+                // stand-alone acceptance: the caller's drafter LSE and the token's drafter logit
+                f = facts_invalid();
+                f.lse = df_from_double(__ldg(d.d_lse + ob + j));
+                const int xj = __ldg(d.tokens + ob + j);
+                f.g = (xj >= 0 && xj < p.V)
+                          ? fmax_nan(logit_at<DT>(d.zd + (ob + j) * d.stride_bytes, xj), clamp_floor())
+                          : qnan();
+            }
+            put_drafter(F, j, f);
+        } else {
+            const int j = s - nd;
+            const ScanGroup &G = p.grp[gt];
+            SoftState acc;
+            float g;
+            bool bad;
+            merge_row(p, (gt ? p.rows0 : 0) + static_cast<int64_t>(i) * G.npos + j, acc, g, bad);
+            put_target(F, j, row_final(p, G, j, b, acc, g, bad, leader));
+        }
     }
     __syncthreads();
-    const DrawCtx c = s_ctx;
-    const int L = s_L;
-    const int vpt = p.seg_vec / kDrawThreads;
+    if (!dec) return;
+    const bool sched = d.do_sched && has_d;
 
-    // first pass: this segment's weight total and last positive entry
-    const int v0 = seg * p.seg_vec, v1 = min(p.RV, v0 + p.seg_vec);
-    int last_pos = -1;
-    {
-        const int vb = min(v1, v0 + static_cast<int>(threadIdx.x) * vpt), ve = min(v1, vb + vpt);
-        const float ts = run_sum<DT>(c, vb, ve, p.V, last_pos);
-        float tot;
-        (void)cta_incl_scan(ts, s_warp, &tot);
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) last_pos = max(last_pos, __shfl_xor_sync(0xFFFFFFFFu, last_pos, off));
-        if ((threadIdx.x & 31) == 0) atomicMax(&s_lastp, last_pos);
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            p.res_total[static_cast<int64_t>(i) * p.nseg + seg] = static_cast<double>(tot);
-            p.res_last[static_cast<int64_t>(i) * p.nseg + seg] = s_lastp;
-            __threadfence();
-            const uint32_t old = atomicAdd(p.res_count + i, 1u);
-            s_is_last = (old == static_cast<uint32_t>(p.nseg - 1)) ? 1 : 0;
-        }
-        __syncthreads();
-    }
-    if (!s_is_last) return;
-    __threadfence();
-    // the last segment to arrive completes the draw: locate the segment holding u * R
-    for (int s = threadIdx.x; s < p.nseg; s += kDrawThreads) {
-        s_tot[s] = __ldcg(p.res_total + static_cast<int64_t>(i) * p.nseg + s);
-        s_last[s] = __ldcg(p.res_last + static_cast<int64_t>(i) * p.nseg + s);
-    }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        double R = 0.0;
-        int lastp = -1;
-        for (int s = 0; s < p.nseg; ++s) {
-            R += s_tot[s];
-            lastp = max(lastp, s_last[s]);
-        }
-        const uint32_t jj = (L < gamma) ? static_cast<uint32_t>(L + 1) : static_cast<uint32_t>(gamma + 1);
-        const float u = philox_uniform(p.seed, jj, static_cast<uint32_t>(b), p.round,
-                                       (L < gamma) ? kPurposeResid : kPurposeBonus);
-        const double target = static_cast<double>(u) * R;
-        int sel = (R > 0.0) ? -2 : -3;   // -2: rounding left none (last positive), -3: no mass
-        double cum = 0.0, before = 0.0;
-        if (R > 0.0) {
-            for (int s = 0; s < p.nseg; ++s) {
-                const double t = s_tot[s];
-                if (t > 0.0 && cum + t > target) {
-                    sel = s;
-                    before = cum;
-                    break;
-                }
-                cum += t;
+    if (sampling) {
+        // ---- phase 2 (every CTA): the strict accepted length L ----
+        if (warp == 0) {
+            const int L = rule_first_reject(d, F, 0, b, lane);
+            if (lane == 0) {
+                s_L[0] = L;
+                s_corr[0] = F.t_am[L];
             }
         }
-        s_seg = sel;
-        s_target = target;
-        s_before = before;
-        s_lastp = lastp;
-        p.res_count[i] = 0u;   // leave the workspace zeroed
+        __shared__ float s_warp[2 * NW];
+        __shared__ float s_pref[kDecThreads];
+        __shared__ int s_is_last, s_seg, s_lastp, s_thr, s_tok;
+        __shared__ df s_rem;
+        __shared__ float s_tot[kDrawMaxSeg];
+        __shared__ df s_cum[kDrawMaxSeg];
+        __shared__ int s_last[kDrawMaxSeg];
+        if (tid == 0) {
+            s_lastp = -1;
+            s_thr = INT32_MAX;
+        }
+        __syncthreads();
+
+        // ---- phase 3 (every CTA): its segment of the draw row at position L
+        // (the residual row, or the bonus row when every position passed) ----
+        const int L = s_L[0];
+        const char *zt_row = d.zt + (bo + L) * d.stride_bytes;
+        const char *zd_row = (L < gamma) ? d.zd + (ob + L) * d.stride_bytes : nullptr;
+        const DrawCtx c = draw_ctx(zt_row, zd_row, df{F.t_lh[L], F.t_ll[L]},
+                                   (L < gamma) ? df{F.d_lh[L], F.d_ll[L]} : df{0.f, 0.f});
+        const int vpt = d.seg_vec / kDecThreads;
+        const int64_t pair = static_cast<int64_t>(i) * d.nseg + seg;
+        {
+            const int v0 = seg * d.seg_vec, v1 = min(p.RV, v0 + d.seg_vec);
+            const int vb = min(v1, v0 + tid * vpt), ve = min(v1, vb + vpt);
+            int last_pos = -1;
+            const float ts = run_sum<DT>(c, vb, ve, p.V, last_pos);
+            float tot;
+            const float incl = cta_incl_scan(ts, s_warp, &tot);
+            d.res_pref[pair * kDecThreads + tid] = incl;   // this thread's inclusive prefix in the segment
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1)
+                last_pos = max(last_pos, __shfl_xor_sync(0xFFFFFFFFu, last_pos, off));
+            if (lane == 0) atomicMax(&s_lastp, last_pos);
+            __syncthreads();
+            if (tid == 0) {
+                d.res_total[pair] = tot;
+                d.res_last[pair] = s_lastp;
+                // the barrier above orders every thread's prefix store before
+                // this fence, which orders them all before the arrival
+                __threadfence();
+                const uint32_t old = atomicAdd(d.res_count + i, 1u);
+                s_is_last = (old == static_cast<uint32_t>(d.nseg - 1)) ? 1 : 0;
+            }
+            __syncthreads();
+        }
+        if (s_is_last) {
+            // the last segment to arrive completes the draw
+            __threadfence();
+            for (int sg = tid; sg < d.nseg; sg += kDecThreads) {
+                s_tot[sg] = __ldcg(d.res_total + static_cast<int64_t>(i) * d.nseg + sg);
+                s_last[sg] = __ldcg(d.res_last + static_cast<int64_t>(i) * d.nseg + sg);
+            }
+            __syncthreads();
+            if (warp == 0) {
+                // R = sum of the segment totals and their inclusive prefix sums
+                // (double-floats); the first segment whose prefix exceeds u * R
+                df carry = df{0.f, 0.f};
+                int lastp = -1;
+                for (int s0 = 0; s0 < d.nseg; s0 += 32) {
+                    const int sg = s0 + lane;
+                    const float t = (sg < d.nseg) ? s_tot[sg] : 0.f;
+                    const df cum = df_add(carry, warp_prefix_df(df{t, 0.f}, lane));
+                    if (sg < d.nseg) {
+                        s_cum[sg] = cum;
+                        lastp = max(lastp, s_last[sg]);
+                    }
+                    carry.hi = __shfl_sync(0xFFFFFFFFu, cum.hi, 31);
+                    carry.lo = __shfl_sync(0xFFFFFFFFu, cum.lo, 31);
+                }
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1) lastp = max(lastp, __shfl_xor_sync(0xFFFFFFFFu, lastp, off));
+                const df Rm = carry;
+                const uint32_t jj = (L < gamma) ? static_cast<uint32_t>(L + 1) : static_cast<uint32_t>(gamma + 1);
+                const float u = philox_uniform(d.seed, jj, static_cast<uint32_t>(b), d.round,
+                                               (L < gamma) ? kPurposeResid : kPurposeBonus);
+                const df target = df_mul_f(Rm, u);
+                int sel = (Rm.hi > 0.f) ? -2 : -3;   // -2: rounding left none (last positive), -3: no mass
+                if (Rm.hi > 0.f) {
+                    __syncwarp();
+                    for (int s0 = 0; s0 < d.nseg; s0 += 32) {
+                        const int sg = s0 + lane;
+                        const bool hit = (sg < d.nseg) && s_tot[sg] > 0.f && !df_ge(target, s_cum[sg]);
+                        const unsigned bal = __ballot_sync(0xFFFFFFFFu, hit);
+                        if (bal) {
+                            sel = s0 + __ffs(bal) - 1;
+                            break;
+                        }
+                    }
+                }
+                if (lane == 0) {
+                    s_seg = sel;
+                    s_rem = (sel > 0) ? df_sub(target, s_cum[sel - 1]) : target;   // u R minus the mass before sel
+                    s_lastp = lastp;
+                    d.res_count[i] = 0u;   // leave the workspace zeroed
+                }
+            }
+            if (warp == 1 && sched) {
+                // pair 0 decides whether this block commits its verified tokens
+                int Kh, K, Do;
+                sched_pair(d, F, 0, s_force != 0, s_D, lane, Kh, K, Do);
+                if (lane == 0) s_K0 = K;
+            }
+            __syncthreads();
+            int tok;
+            const int sel = s_seg;
+            if (sel >= 0) {
+                // the thread of segment sel whose run holds u R, from the
+                // inclusive prefixes that segment's CTA published
+                const float pv = __ldcg(d.res_pref + (static_cast<int64_t>(i) * d.nseg + sel) * kDecThreads + tid);
+                s_pref[tid] = pv;
+                const df rem = s_rem;
+                const unsigned bal = __ballot_sync(0xFFFFFFFFu, !df_ge(rem, df{pv, 0.f}));
+                if (lane == 0 && bal) atomicMin(&s_thr, warp * 32 + __ffs(bal) - 1);
+                __syncthreads();
+                const int thr = s_thr;
+                if (thr == INT32_MAX) {
+                    tok = s_last[sel];   // rounding: the segment's last positive entry
+                } else {
+                    if (warp == 0) {
+                        const df rem2 = (thr > 0) ? df_sub(rem, df{s_pref[thr - 1], 0.f}) : rem;
+                        const int sv0 = sel * d.seg_vec, sv1 = min(p.RV, sv0 + d.seg_vec);
+                        const int vb = min(sv1, sv0 + thr * vpt), ve = min(sv1, vb + vpt);
+                        const int pick = warp_search<DT>(c, vb, ve, p.V, rem2, lane);
+                        if (lane == 0) s_tok = (pick >= 0) ? pick : s_last[sel];
+                    }
+                    __syncthreads();
+                    tok = s_tok;
+                }
+            } else if (sel == -2) {
+                tok = s_lastp;
+            } else {
+                // the residual has no mass (only through rounding): draw from p_t
+                // of the same row, whole row in this CTA, same inverse-CDF rule
+                DrawCtx ct = c;
+                ct.zd_row = nullptr;
+                const int vrow = (p.RV + kDecThreads - 1) / kDecThreads;
+                const int vb = min(p.RV, tid * vrow), ve = min(p.RV, vb + vrow);
+                int lp = -1;
+                float tot;
+                (void)cta_incl_scan(run_sum<DT>(ct, vb, ve, p.V, lp), s_warp, &tot);
+                const float u = philox_uniform(d.seed, static_cast<uint32_t>(L + 1), static_cast<uint32_t>(b),
+                                               d.round, kPurposeResid);
+                tok = (tot > 0.f)
+                          ? cta_find<DT>(ct, 0, p.RV, vrow, p.V, df_mul_f(df{tot, 0.f}, u), s_warp, &s_thr, &s_tok)
+                          : -1;
+            }
+            if (warp == 0) {
+                if (lane == 0) {
+                    if (d.L_strict) d.L_strict[b] = L;
+                    if (d.n_strict) d.n_strict[b] = L + 1;
+                }
+                if (d.tok_strict) write_tokens(lane, gamma, d.tok_strict + bo, F.x, L, tok);
+                if (sched && s_K0 == 0) {
+                    // commit under pair 0: this block was not skipped
+                    if (lane == 0 && d.commit_n) d.commit_n[b] = L + 1;
+                    if (d.commit_tokens) write_tokens(lane, gamma, d.commit_tokens + bo, F.x, L, tok);
+                }
+            }
+        }
+        if (!leader) return;
+        __syncthreads();
+    }
+
+    // ---- the leader: every other rule (a warp per rule), the schedule (a warp
+    // per threshold pair), agreement counters and the remaining commits ----
+    const int R = 1 + d.n_ell + d.n_k;
+    for (int r = warp; r < R; r += NW) {
+        if (r == 0) {
+            if (!d.do_strict || sampling) continue;   // sampling: completed by the draw
+            const int L = rule_first_reject(d, F, 0, b, lane);
+            if (lane == 0) {
+                s_L[0] = L;
+                s_corr[0] = F.t_am[L];
+                if (d.L_strict) d.L_strict[b] = L;
+                if (d.n_strict) d.n_strict[b] = L + 1;
+            }
+            if (d.tok_strict) write_tokens(lane, gamma, d.tok_strict + bo, F.x, L, F.t_am[L]);
+        } else {
+            const int L = rule_first_reject(d, F, r, b, lane);
+            const int corr = F.t_am[L];   // target argmax at the first rejection, or of the bonus row
+            const bool len = r <= d.n_ell;
+            const int64_t o = static_cast<int64_t>(len ? r - 1 : r - 1 - d.n_ell) * p.B + b;
+            int32_t *Lo = len ? d.L_len : d.L_topk, *no = len ? d.n_len : d.n_topk;
+            int32_t *to = len ? d.tok_len : d.tok_topk;
+            if (lane == 0) {
+                if (Lo) Lo[o] = L;
+                if (no) no[o] = L + 1;
+            }
+            if (to) write_tokens(lane, gamma, to + o * (gamma + 1), F.x, L, corr);
+        }
+    }
+    if (!sched) return;
+    __syncthreads();   // s_L[0] of a greedy strict rule
+    for (int t = warp; t < d.n_tau; t += NW) {
+        int Kh, K, Do;
+        sched_pair(d, F, t, s_force != 0, s_D, lane, Kh, K, Do);
+        if (lane == 0) {
+            if (t == 0) s_K0 = K;
+            const int64_t o = static_cast<int64_t>(t) * p.B + b;
+            if (d.K_hat) d.K_hat[o] = Kh;
+            if (d.K) d.K[o] = K;
+            if (d.D_out) d.D_out[o] = Do;
+            if (d.agreement && K > 0 && d.do_strict) {
+                const int L = s_L[0];
+                unsigned long long *a = reinterpret_cast<unsigned long long *>(d.agreement + 4 * t);
+                atomicAdd(a + 0, static_cast<unsigned long long>(min(K, L)));
+                atomicAdd(a + 1, static_cast<unsigned long long>(K));
+                atomicAdd(a + 2, static_cast<unsigned long long>(K <= L ? 1 : 0));
+                atomicAdd(a + 3, 1ull);
+            }
+        }
     }
     __syncthreads();
-    int tok;
-    if (s_seg >= 0) {
-        const int sv0 = s_seg * p.seg_vec, sv1 = min(p.RV, sv0 + p.seg_vec);
-        tok = cta_find<DT>(c, sv0, sv1, vpt, p.V, s_before, s_target, s_warp, &s_thr, &s_tok);
-        if (tok < 0) tok = s_lastp;
-    } else if (s_seg == -2) {
-        tok = s_lastp;
-    } else {
-        // the residual has no mass (only through rounding): draw from p_t of the
-        // same row, whole row in this CTA, same inverse-CDF rule
-        DrawCtx ct = c;
-        ct.zd_row = nullptr;
-        const int vrow = (p.RV + kDrawThreads - 1) / kDrawThreads;
-        const int vb = min(p.RV, static_cast<int>(threadIdx.x) * vrow), ve = min(p.RV, vb + vrow);
-        int lp = -1;
-        float tot;
-        (void)cta_incl_scan(run_sum<DT>(ct, vb, ve, p.V, lp), s_warp, &tot);
-        const float u = philox_uniform(p.seed, static_cast<uint32_t>(L + 1), static_cast<uint32_t>(b), p.round,
-                                       kPurposeResid);
-        tok = (tot > 0.f) ? cta_find<DT>(ct, 0, p.RV, vrow, p.V, 0.0, static_cast<double>(u) * tot, s_warp, &s_thr, &s_tok)
-                          : -1;
-    }
-    if (threadIdx.x < 32) {
-        const int lane = threadIdx.x;
-        const int32_t *xb = p.tokens + static_cast<int64_t>(b) * gamma;
-        const int64_t bo = static_cast<int64_t>(b) * (gamma + 1);
-        if (lane == 0) {
-            if (p.L_strict) p.L_strict[b] = L;
-            if (p.n_strict) p.n_strict[b] = L + 1;
-        }
-        if (p.tok_strict) write_tokens(lane, gamma, p.tok_strict + bo, xb, L, tok);
-        if (p.k0 && p.k0[i] == 0) {
-            // commit under pair 0: this block was not skipped
-            if (lane == 0 && p.commit_n) p.commit_n[b] = L + 1;
-            if (p.commit_tokens) write_tokens(lane, gamma, p.commit_tokens + bo, xb, L, tok);
+    if (warp == 0) {
+        // tokens committed by a fused round: a skipped block commits x_1..x_K
+        // (pair 0); a greedy strict block its verified tokens
+        const int K0 = s_K0;
+        if (K0 > 0 || (d.do_strict && !sampling)) {
+            const int Lc = (K0 > 0) ? K0 : s_L[0];
+            const int corr = (K0 > 0) ? -1 : s_corr[0];
+            if (lane == 0 && d.commit_n) d.commit_n[b] = (K0 > 0) ? K0 : s_L[0] + 1;
+            if (d.commit_tokens) write_tokens(lane, gamma, d.commit_tokens + bo, F.x, Lc, corr);
         }
     }
 }
@@ -346,12 +605,28 @@ __global__ void schedule_kernel(const __grid_constant__ ScheduleParams p) {
     const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     if (w >= static_cast<int64_t>(p.B) * p.n_tau) return;
     const int t = static_cast<int>(w / p.B), b = static_cast<int>(w % p.B);
-    const int64_t o = static_cast<int64_t>(b) * p.gamma;
+    const int gamma = p.gamma;
+    const int64_t o = static_cast<int64_t>(b) * gamma;
     const bool force = p.force_strict && p.force_strict[b];
     const int D = p.D_in ? p.D_in[b] : 0;
-    int Kh, K, Do;
-    schedule_block(lane, p.gamma, p.q + o, p.logq ? p.logq + o : nullptr, 1, p.guard ? p.guard + o : nullptr,
-                   force || p.tau_off[t], D, p.signal, p.eta_loc[t], p.log_eta_c[t], p.K_min, p.S_max, Kh, K, Do);
+    int Kh = 0, K = 0, Do = 0;
+    if (!(force || p.tau_off[t])) {
+        int kb = gamma, best = 0;
+        df carry = df{0.f, 0.f};
+        for (int c = 0; c < gamma && kb >= c; c += 32) {
+            const int j = c + lane;
+            const bool in = j < gamma;
+            const float qj = in ? p.q[o + j] : 0.f;
+            const float lq = in ? (p.logq ? p.logq[o + j] : logf(qj)) : 0.f;
+            const bool guard_j = in && p.guard && p.guard[o + j];
+            const df S = df_add(carry, warp_prefix_df(df{lq, 0.f}, lane));
+            carry.hi = __shfl_sync(0xFFFFFFFFu, S.hi, 31);
+            carry.lo = __shfl_sync(0xFFFFFFFFu, S.lo, 31);
+            sched_step(c, lane, gamma, in, qj, guard_j, S, p.eta_loc[t], p.log_eta_c[t], p.signal, kb, best);
+        }
+        Kh = (p.signal == SDD_SIG_MARGINAL) ? kb : best;
+        sched_final(Kh, D, p.K_min, p.S_max, K, Do);
+    }
     if (lane == 0) {
         const int64_t oo = static_cast<int64_t>(t) * p.B + b;
         p.K_hat[oo] = Kh;
@@ -396,14 +671,18 @@ __global__ void uniforms_kernel(uint64_t seed, const uint32_t *j, const uint32_t
 
 }  // namespace
 
-cudaError_t launch_draw(const DrawParams &p, cudaStream_t stream) {
-    if (p.nb == 0) return cudaSuccess;
-    const dim3 grid(p.nb, p.nseg);
-    if (p.dtype == SDD_BF16)
-        draw_kernel<SDD_BF16><<<grid, kDrawThreads, 0, stream>>>(p);
-    else
-        draw_kernel<SDD_F32><<<grid, kDrawThreads, 0, stream>>>(p);
-    return cudaGetLastError();
+int decide_max_ctas_per_sm() {
+    int n = 0;
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decide_kernel<SDD_BF16>, kDecThreads, 0);
+    return n;
+}
+
+cudaError_t launch_decide(const ScanParams &p, cudaStream_t stream) {
+    const int nb = p.grp[0].nb;
+    if (nb == 0) return cudaSuccess;
+    const int nseg = (p.dec.enabled && p.dec.do_strict && !p.dec.greedy) ? p.dec.nseg : 1;
+    return launch_dependent(p.dtype == SDD_BF16 ? decide_kernel<SDD_BF16> : decide_kernel<SDD_F32>, dim3(nb, nseg),
+                            dim3(kDecThreads), 0, stream, p);
 }
 
 cudaError_t launch_schedule(const ScheduleParams &p, cudaStream_t stream) {

@@ -21,25 +21,21 @@ constexpr int kStages = 3;
 constexpr int kScanSmem = kWarpsPerCta * kStages * kTileBytes + kWarpsPerCta * kStages * 8;
 constexpr uint32_t kWaitPolls = 1u << 24;     // bounded mbarrier wait (seconds of polling)
 
-// Sampling draw geometry: each CTA takes a segment of whole 256-vector chunks
-// of the draw row; at most kDrawMaxSeg segments per block.
-constexpr int kDrawThreads = 256;
+// Decide kernel geometry: one CTA of kDecThreads per (listed block, draw
+// segment); each draw segment is a run of whole 256-vector chunks of the draw
+// row, at most kDrawMaxSeg per block.
+constexpr int kDecThreads = 256;
 constexpr int kDrawMaxSeg = 128;
 
-// Per-block decisions, evaluated inside the streaming kernel by the warp that
-// finalises a block's last row (rules.cuh).
+// Per-block finalisation and decisions (decide.cu, rules.cuh).  Thresholds
+// are double-floats split on the host from their fp64 values.
 struct DecideParams {
-    int32_t enabled;               // run block decisions in the streaming kernel
-    int32_t rows_per_block;        // rows of one block streamed by this launch
+    int32_t enabled;               // evaluate block decisions after finalising the rows
     int32_t B, gamma, V;
-    int32_t pad0;
     int64_t stride_bytes;
-    const int32_t *bidx;           // [nb] batch index of listed block i, or nullptr
-    const char *zd;                // drafter logits (stand-alone sampling acceptance)
+    const char *zt, *zd;           // target / drafter logits (draw rows, stand-alone acceptance)
     const int32_t *tokens;         // [B, gamma]
-    const RowRec *trec;            // [nb, gamma+1] list order
-    const RowRec *drec;            // [nb, gamma] list order, or nullptr
-    const double *d_lse;           // [B, gamma] drafter LSE (user array) when drec == nullptr
+    const double *d_lse;           // [B, gamma] drafter LSE (user array) when no drafter rows are streamed
     // strict
     int32_t do_strict, greedy;
     uint64_t seed, round;
@@ -47,7 +43,7 @@ struct DecideParams {
     // lenience
     int32_t n_ell;
     int32_t ell_one[SDD_MAX_GRID];
-    double ell_thr[SDD_MAX_GRID];
+    df ell_thr[SDD_MAX_GRID];      // ln(ell)
     int32_t *L_len, *tok_len, *n_len;
     // top-k
     int32_t n_k;
@@ -56,20 +52,23 @@ struct DecideParams {
     // schedule (fused round)
     int32_t do_sched, signal, n_tau, K_min, S_max;
     int32_t tau_off[SDD_MAX_GRID];
-    double eta_loc[SDD_MAX_GRID];
-    double log_eta_c[SDD_MAX_GRID];
+    df eta_loc[SDD_MAX_GRID];
+    df log_eta_c[SDD_MAX_GRID];
     const uint8_t *guard, *force_strict;
     const int32_t *D_in;
     int32_t *K_hat, *K, *D_out;
     int32_t *commit_tokens, *commit_n;
     long long *agreement;
-    // workspace
-    uint32_t *blk_count;           // [nb] arrival counters of finalised rows
-    int32_t *blk_L;                // [nb] strict accepted length, for the draw kernel
-    int32_t *k0;                   // [nb] K under pair 0, for the draw kernel
+    // sampling draw (residual / bonus inverse CDF), workspace
+    int32_t nseg, seg_vec;         // segments per block and vectors per segment
+    float *res_total;              // [nb, nseg]
+    float *res_pref;               // [nb, nseg, kDecThreads] per-thread inclusive prefix sums
+    int32_t *res_last;             // [nb, nseg]
+    uint32_t *res_count;           // [nb] (zero between calls)
 };
 
 // One set of rows streamed by the scan kernel (drafter rows or target rows).
+// Both groups of a launch list the same blocks in the same order.
 struct ScanGroup {
     const char *base;        // logits [B, npos, row_stride]
     int64_t stride_bytes;    // row_stride * element size
@@ -78,7 +77,6 @@ struct ScanGroup {
     int32_t nb;              // blocks in this group (after compaction)
     int32_t pad;
     const int32_t *bidx;     // [nb] batch index of each listed block, or nullptr (= identity)
-    RowRec *rec;             // [nb * npos] final records, list order
     // drafter user outputs, indexed (b * gamma + j); any may be nullptr
     float *q, *logq, *maxprob, *entropy;
     double *lse;
@@ -100,47 +98,26 @@ struct ScanParams {
     int64_t T;               // total vectors = rows * RV
     const int32_t *tokens;   // [B, gamma]
     Partial *partials;       // [rows + W]
-    uint32_t *counters;      // [rows]
     int32_t *status;
     DecideParams dec;
-};
-
-// The inverse-CDF draw of the sampling rule (residual or bonus), after the
-// streaming kernel has fixed each block's accepted length.
-struct DrawParams {
-    int32_t B, gamma, V, RV;
-    int32_t dtype, nb;
-    int64_t stride_bytes;
-    const int32_t *bidx;
-    const char *zt, *zd;
-    const int32_t *tokens;
-    const RowRec *trec, *drec;
-    const double *d_lse;
-    uint64_t seed, round;
-    const int32_t *blk_L;
-    const int32_t *k0;             // nullptr unless a fused round commits tokens
-    int32_t *L_strict, *tok_strict, *n_strict;
-    int32_t *commit_tokens, *commit_n;
-    int32_t nseg, seg_vec;
-    double *res_total;             // [nb, nseg]
-    int32_t *res_last;             // [nb, nseg]
-    uint32_t *res_count;           // [nb]
-    int32_t *status;
 };
 
 struct ScheduleParams {
     const float *q, *logq;
     int32_t B, gamma, signal, n_tau, K_min, S_max;
     int32_t tau_off[SDD_MAX_GRID];
-    double eta_loc[SDD_MAX_GRID];
-    double log_eta_c[SDD_MAX_GRID];
+    df eta_loc[SDD_MAX_GRID];
+    df log_eta_c[SDD_MAX_GRID];
     const uint8_t *guard, *force_strict;
     const int32_t *D_in;
     int32_t *K_hat, *K, *D_out;
 };
 
+// The streaming kernel (grid = warps / kWarpsPerCta CTAs).
 cudaError_t launch_scan(const ScanParams &p, int grid, cudaStream_t stream);
-cudaError_t launch_draw(const DrawParams &p, cudaStream_t stream);
+// The decide kernel over (listed blocks, p.dec.nseg) CTAs, launched as a
+// programmatic dependent of the streaming kernel.
+cudaError_t launch_decide(const ScanParams &p, cudaStream_t stream);
 cudaError_t launch_schedule(const ScheduleParams &p, cudaStream_t stream);
 cudaError_t launch_agreement(const int32_t *K, const int32_t *L, int B, int n_tau, long long *acc,
                              cudaStream_t stream);
@@ -149,6 +126,7 @@ cudaError_t launch_commit(const int32_t *K, const int32_t *x, const int32_t *vt,
 cudaError_t launch_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, const uint64_t *round,
                             const uint32_t *purpose, int64_t n, float *u, cudaStream_t stream);
 int scan_max_ctas_per_sm();
+int decide_max_ctas_per_sm();
 cudaError_t scan_prepare_device();
 void set_last_error(const char *msg);  // message returned by sdd_last_error()
 

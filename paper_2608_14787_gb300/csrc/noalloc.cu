@@ -5,8 +5,7 @@
 // where they need the statistics: code running inside a CUDA graph capture, a
 // framework whose device memory is owned by a fixed arena, or an embedded
 // host loop without an allocator.  This entry point takes no workspace.  Its
-// scratch -- per-warp partial states, per-row arrival counters and per-row
-// records -- lives in one file-scope device array of fixed size that every GPU
+// scratch -- the per-warp partial states of the streaming kernel -- lives in one file-scope device array of fixed size that every GPU
 // which loads this library holds until the process exits.
 #include <algorithm>
 #include <atomic>
@@ -23,9 +22,7 @@ namespace {
 constexpr int kNoAllocMaxRows = 8192;
 constexpr int kNoAllocMaxWarps = 4096;
 constexpr size_t kPartialBytes = static_cast<size_t>(kNoAllocMaxRows + kNoAllocMaxWarps) * sizeof(Partial);
-constexpr size_t kCounterBytes = static_cast<size_t>(kNoAllocMaxRows) * sizeof(uint32_t);
-constexpr size_t kRecordBytes = static_cast<size_t>(kNoAllocMaxRows) * sizeof(RowRec);
-constexpr size_t kScratchBytes = kPartialBytes + kCounterBytes + kRecordBytes;  // 672 KiB
+constexpr size_t kScratchBytes = kPartialBytes;  // 384 KiB
 
 // The scratch.  In host code this name is only a stand-in for the device
 // symbol: its device address comes from cudaGetSymbolAddress below.
@@ -125,7 +122,6 @@ sdd_status_t sdd_confidence_noalloc(const void *draft_logits, sdd_dtype_t dtype,
     p.B = B;
     p.tokens = draft_tokens;
     p.partials = reinterpret_cast<Partial *>(nd.scratch);
-    p.counters = reinterpret_cast<uint32_t *>(nd.scratch + kPartialBytes);
     p.status = status;
     ScanGroup &G = p.grp[0];
     G.base = static_cast<const char *>(draft_logits);
@@ -133,7 +129,6 @@ sdd_status_t sdd_confidence_noalloc(const void *draft_logits, sdd_dtype_t dtype,
     G.npos = gamma;
     G.kind = 0;
     G.nb = B;
-    G.rec = reinterpret_cast<RowRec *>(nd.scratch + kPartialBytes + kCounterBytes);
     G.q = q;
     G.logq = logq;
     G.maxprob = maxprob;
@@ -146,12 +141,10 @@ sdd_status_t sdd_confidence_noalloc(const void *draft_logits, sdd_dtype_t dtype,
     const int64_t W = std::min<int64_t>(nd.W_max, p.T);
     p.W = static_cast<int32_t>(W);
 
-    // The arrival counters must start at zero; the array keeps whatever the
-    // previous call (or an interrupted one) left, so clear them on the stream.
-    cudaError_t e = cudaMemsetAsync(p.counters, 0, static_cast<size_t>(rows) * sizeof(uint32_t), st);
-    if (e != cudaSuccess) return na_fail(SDD_ERR_CUDA, "cudaMemsetAsync: %s", cudaGetErrorString(e));
-    e = launch_scan(p, static_cast<int>((W + kWarpsPerCta - 1) / kWarpsPerCta), st);
+    cudaError_t e = launch_scan(p, static_cast<int>((W + kWarpsPerCta - 1) / kWarpsPerCta), st);
     if (e != cudaSuccess) return na_fail(SDD_ERR_CUDA, "scan launch: %s", cudaGetErrorString(e));
+    e = launch_decide(p, st);   // row finalisation only (no decisions)
+    if (e != cudaSuccess) return na_fail(SDD_ERR_CUDA, "decide launch: %s", cudaGetErrorString(e));
     return SDD_OK;
 }
 

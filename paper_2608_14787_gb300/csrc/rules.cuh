@@ -1,263 +1,261 @@
-// rules.cuh -- warp-level decisions for one block of gamma draft positions,
-// evaluated by the warp that finalises the block's last row (inside the
-// streaming kernel) or by the stand-alone schedule kernel.
+// rules.cuh -- what the decide kernel computes for one block of gamma draft
+// positions once every logit has been streamed:
 //
-//  * schedule_block -- the skip policy of Sec. 4.1: Eq. 3 with the three
-//    confidence signals of Sec. 4.2, then K_min / staleness / guards.
-//  * block_decide   -- Strict SDD (Sec. 3.1: greedy, or the acceptance test of
-//    the speculative-sampling rule it cites), lenience (App. A.6 Eq. 9), top-k
-//    (App. A.6), the schedule of a fused round, the agreement counters of
-//    Sec. 3.2 (Eq. 1-2) and the tokens committed by skipped blocks.
+//  * row finalisation -- merge a row's per-warp partials (warp order), then
+//    LSE as a double-float from an fp32 log, q = p(x_j), log q, maxprob and
+//    entropy (the confidence quantities of Sec. 4.2) and the target facts;
+//  * per-position acceptance tests -- Strict SDD (Sec. 3.1: greedy, or the
+//    speculative-sampling acceptance test it cites), lenience (App. A.6,
+//    Eq. 9), top-k (App. A.6);
+//  * sched_step / sched_final -- the skip policy of Sec. 4.1: the local gate,
+//    then Eq. 3 with the raw / conditional / marginal signals of Sec. 4.2, then
+//    K_min, staleness and guards.
+//
+// Everything here is fp32 or double-float (common.cuh): fp64 instructions
+// issue at a small fraction of the fp32 rate on this part.
 #pragma once
 
 #include "internal.h"
 
 namespace sdd {
 
-__device__ __forceinline__ float qnan() { return __int_as_float(0x7FC00000); }
+// ---------------------------------------------------------------------------
+// Row finalisation
+// ---------------------------------------------------------------------------
+// Facts of one finalised row.
+struct RowFacts {
+    df lse;
+    float M, g, q, logq;
+    int32_t argmax, rank;
+};
 
-// A row record written by another SM during this launch: read through L2.
-__device__ __forceinline__ RowRec load_rec(const RowRec *p) {
+__device__ __forceinline__ RowFacts facts_invalid() {
+    RowFacts f;
+    f.lse = df{qnan(), 0.f};
+    f.M = f.g = f.q = f.logq = qnan();
+    f.argmax = -1;
+    f.rank = INT32_MAX;
+    return f;
+}
+
+// A partial written by the streaming grid: read through L2.
+__device__ __forceinline__ Partial load_partial(const Partial *p) {
     union {
         uint4 v[2];
-        RowRec r;
+        Partial q;
     } u;
     u.v[0] = __ldcg(reinterpret_cast<const uint4 *>(p));
     u.v[1] = __ldcg(reinterpret_cast<const uint4 *>(p) + 1);
-    return u.r;
+    return u.q;
 }
 
-template <int DT>
-__device__ __forceinline__ float logit_at(const char *rowp, int v) {
-    if (DT == SDD_BF16) {
-        const uint16_t h = __ldg(reinterpret_cast<const unsigned short *>(rowp) + v);
-        return __uint_as_float(static_cast<uint32_t>(h) << 16);
-    } else {
-        return __ldg(reinterpret_cast<const float *>(rowp) + v);
-    }
-}
-
-// Skip policy for one block and one threshold pair, by one warp.  q and logq
-// (nullable) are read at q[j * stride] for the block's gamma positions; guard
-// is nullable.
-__device__ __forceinline__ void schedule_block(int lane, int gamma, const float *q, const float *logq, int stride,
-                                               const uint8_t *guard, bool off, int D, int signal, double eta_loc,
-                                               double log_eta_c, int K_min, int S_max, int &K_hat, int &K,
-                                               int &D_out) {
-    if (off) {
-        K_hat = 0;
-        K = 0;
-        D_out = 0;
-        return;
-    }
-    // local gate and guards: kb = number of leading positions that pass
-    int kb = gamma;
-    for (int c = 0; c < gamma; c += 32) {
-        const int j = c + lane;
-        bool fail = false;
-        if (j < gamma) {
-            const float qj = __ldcg(q + static_cast<int64_t>(j) * stride);
-            fail = (guard && guard[j]) || !isfinite(qj) || !(static_cast<double>(qj) >= eta_loc);
-        }
-        const unsigned bal = __ballot_sync(0xFFFFFFFFu, fail);
-        if (bal) {
-            kb = c + __ffs(bal) - 1;
-            break;
-        }
-    }
-    int best = 0;
-    if (signal == SDD_SIG_MARGINAL) {
-        best = kb;
-    } else {
-        // prefix sums of ln q in fp64; raw: S_k >= k ln eta_c, conditional: S_k >= ln eta_c
-        double carry = 0.0;
-        for (int c = 0; c < kb; c += 32) {
-            const int j = c + lane;
-            double v = 0.0;
-            if (j < kb)
-                v = logq ? static_cast<double>(__ldcg(logq + static_cast<int64_t>(j) * stride))
-                         : static_cast<double>(logf(__ldcg(q + static_cast<int64_t>(j) * stride)));
+// Merged state of global row r, whose pieces were streamed by warps fw..lw
+// (partial of warp w at index r + w), merged in warp order, four loads in
+// flight at a time.  The row's first piece carries its token logit; any piece
+// flags an out-of-range token.
+__device__ __forceinline__ void merge_row(const ScanParams &p, int64_t r, SoftState &acc, float &g, bool &tok_bad) {
+    const int64_t fw = part_owner(r * p.RV, p.T, p.W), lw = part_owner((r + 1) * p.RV - 1, p.T, p.W);
+    acc = soft_identity();
+    g = qnan();
+    tok_bad = false;
+    for (int64_t w0 = fw; w0 <= lw; w0 += 4) {
+        Partial pt[4];
 #pragma unroll
-            for (int off2 = 1; off2 < 32; off2 <<= 1) {
-                const double t = __shfl_up_sync(0xFFFFFFFFu, v, off2);
-                if (lane >= off2) v += t;
-            }
-            const double Sk = carry + v;
-            const bool pass = (j < kb) && ((signal == SDD_SIG_RAW) ? (Sk >= static_cast<double>(j + 1) * log_eta_c)
-                                                                    : (Sk >= log_eta_c));
-            const unsigned bal = __ballot_sync(0xFFFFFFFFu, pass);
-            if (bal) best = c + 32 - __clz(bal);
-            carry = __shfl_sync(0xFFFFFFFFu, Sk, 31);
+        for (int u = 0; u < 4; ++u)
+            if (w0 + u <= lw) pt[u] = load_partial(p.partials + r + w0 + u);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            if (w0 + u > lw) break;
+            if (w0 + u == fw) g = pt[u].g;
+            tok_bad |= pt[u].rank < 0;
+            SoftState o;
+            o.m = pt[u].m;
+            o.r = pt[u].r;
+            o.t2 = pt[u].t2;
+            o.sh = pt[u].sh;
+            o.sl = pt[u].sl;
+            o.amax = pt[u].amax;
+            o.rank = max(pt[u].rank, 0);
+            acc = soft_merge(acc, o);
         }
     }
-    K_hat = best;
-    K = (D < S_max && best > 0 && best >= K_min) ? best : 0;
-    D_out = (K > 0) ? D + K : 0;
 }
 
-// First failing position (0-based) of a per-position acceptance predicate,
-// gamma if none fails.
-template <class Accept>
-__device__ __forceinline__ int first_reject(int lane, int gamma, Accept accept) {
+// Final results of position j of block b (group G) from its merged state, by
+// one thread.  `write`: also store the drafter user outputs and raise status
+// flags (one CTA per block does).
+__device__ __forceinline__ RowFacts row_final(const ScanParams &p, const ScanGroup &G, int j, int b,
+                                              const SoftState &acc, float g, bool tok_bad, bool write) {
+    const bool has_tok = j < p.gamma;
+    const bool tok_ok = has_tok && !tok_bad;
+    const float S0 = acc.sh + acc.sl;
+    const bool valid = isfinite(acc.m) && acc.m > clamp_floor() && isfinite(S0) && S0 > 0.f;
+    const int64_t o = static_cast<int64_t>(b) * p.gamma + j;
+    const bool outs = write && G.kind == 0;
+    RowFacts f = facts_invalid();
+    if (valid) {
+        // The lane that held the row maximum M took its term as ex2(y_M) with
+        // y_M = M log2(e) - ceil(M log2(e)) (its reference when M arrived).  On a
+        // peaked row that one term dominates S, so its MUFU error is replaced
+        // by the exact 2^y_M = e0 exp(y_M ln 2 - ln e0) ~ e0 (1 + delta).
+        // ln(S + corr) = ln S + corr / S to 2^-43 (|corr / S| < 2^-21), so the
+        // two logarithms are independent.
+        const float rM = ceilf(acc.m * kLog2e);
+        const float yM = fmaf(acc.m, kLog2e, -rM);
+        const float e0 = ex2(yM);
+        const df ln2 = df{kLn2Hi, kLn2Lo};
+        const df lnS0 = ln_df(acc.sh, acc.sl);
+        const df delta = df_sub(df_mul_f(ln2, yM), ln_df(e0, 0.f));
+        const float corr = e0 * (delta.hi + delta.lo) * pow2f_int(rM - acc.r);
+        const float S = S0 + corr;
+        // LSE = r ln 2 + ln S (S relative to the reference r)
+        const df lnS = df_add(lnS0, df{__fdividef(corr, S0), 0.f});
+        f.lse = df_add(df_mul_f(ln2, acc.r), lnS);
+        f.M = acc.m;
+        f.g = tok_ok ? g : qnan();
+        const df dq = df_sub(df{f.g, 0.f}, f.lse);
+        f.logq = dq.hi + dq.lo;
+        const float eq = expf(dq.hi);
+        f.q = fmaf(eq, dq.lo, eq);
+        f.argmax = acc.amax;
+        f.rank = min(acc.rank, p.kcap);
+        if (outs) {
+            if (G.q) G.q[o] = f.q;
+            if (G.logq) G.logq[o] = f.logq;
+            if (G.maxprob) {
+                const df dm = df_sub(df{acc.m, 0.f}, f.lse);
+                const float em = expf(dm.hi);
+                G.maxprob[o] = fmaf(em, dm.lo, em);
+            }
+            if (G.lse) G.lse[o] = static_cast<double>(f.lse.hi) + static_cast<double>(f.lse.lo);
+            // H = ln S - ln 2 * t2 / S (t2 in log2 units against the same reference)
+            if (G.entropy) G.entropy[o] = (lnS.hi + lnS.lo) - kLn2 * acc.t2 / S;
+            if (G.argmax) G.argmax[o] = acc.amax;
+        }
+    } else {
+        if (outs) {
+            if (G.q) G.q[o] = qnan();
+            if (G.logq) G.logq[o] = qnan();
+            if (G.maxprob) G.maxprob[o] = qnan();
+            if (G.lse) G.lse[o] = __longlong_as_double(0x7FF8000000000000ll);
+            if (G.entropy) G.entropy[o] = qnan();
+            if (G.argmax) G.argmax[o] = -1;
+        }
+        if (write) status_or(p.status, SDD_DEV_NONFINITE);
+    }
+    if (has_tok && !tok_ok) {
+        f.q = f.logq = f.g = qnan();
+        f.rank = INT32_MAX;
+        if (write) status_or(p.status, SDD_DEV_BAD_TOKEN);
+    }
+    return f;
+}
+
+// ---------------------------------------------------------------------------
+// The facts of one block, in shared memory (position j on index j)
+// ---------------------------------------------------------------------------
+struct BlockFacts {
+    // target rows, positions 0..gamma (gamma = bonus row)
+    float t_lh[SDD_MAX_GAMMA + 1], t_ll[SDD_MAX_GAMMA + 1], t_M[SDD_MAX_GAMMA + 1], t_g[SDD_MAX_GAMMA + 1];
+    int32_t t_am[SDD_MAX_GAMMA + 1], t_rk[SDD_MAX_GAMMA + 1];
+    // drafter rows (or, with no drafter rows streamed, the caller's LSE and logit)
+    float d_lh[SDD_MAX_GAMMA], d_ll[SDD_MAX_GAMMA], d_g[SDD_MAX_GAMMA], d_q[SDD_MAX_GAMMA], d_lq[SDD_MAX_GAMMA];
+    int32_t x[SDD_MAX_GAMMA];       // drafted tokens
+    uint8_t guard[SDD_MAX_GAMMA];   // guard flags (0 without a guard array)
+};
+
+__device__ __forceinline__ void put_target(BlockFacts &F, int j, const RowFacts &f) {
+    F.t_lh[j] = f.lse.hi;
+    F.t_ll[j] = f.lse.lo;
+    F.t_M[j] = f.M;
+    F.t_g[j] = f.g;
+    F.t_am[j] = f.argmax;
+    F.t_rk[j] = f.rank;
+}
+__device__ __forceinline__ void put_drafter(BlockFacts &F, int j, const RowFacts &f) {
+    F.d_lh[j] = f.lse.hi;
+    F.d_ll[j] = f.lse.lo;
+    F.d_g[j] = f.g;
+    F.d_q[j] = f.q;
+    F.d_lq[j] = f.logq;
+}
+
+// Rules evaluated per block: rule 0 strict, 1..n_ell lenience, then top-k.
+constexpr int kMaxRules = 1 + 2 * SDD_MAX_GRID;
+
+// Acceptance of draft position j (< gamma) of block b under rule r.
+__device__ __forceinline__ bool rule_accept(const DecideParams &d, const BlockFacts &F, int r, int j, int b) {
+    if (r == 0) {
+        if (d.greedy) return F.t_rk[j] == 0;
+        // speculative sampling: accept iff u <= min(1, p_t(x_j) / p_d(x_j)), with
+        // log r = (g_t - g_d) - (LSE_t - LSE_d)
+        const df lr = df_sub(df_diff(F.t_g[j], F.d_g[j]), df_sub(df{F.t_lh[j], F.t_ll[j]}, df{F.d_lh[j], F.d_ll[j]}));
+        const float u = philox_uniform(d.seed, static_cast<uint32_t>(j + 1), static_cast<uint32_t>(b), d.round,
+                                       kPurposeAccept);
+        return df_ge(lr, df{0.f, 0.f}) || (u <= expf(lr.hi));
+    }
+    if (r <= d.n_ell) {
+        const int e = r - 1;
+        if (d.ell_one[e]) return F.t_rk[j] == 0;
+        return df_ge(df_diff(F.t_g[j], F.t_M[j]), d.ell_thr[e]);   // ln p_t(x_j) - ln max p_t >= ln ell
+    }
+    return F.t_rk[j] < d.kval[r - 1 - d.n_ell];
+}
+
+// First rejected position of rule r (gamma if none), by one warp.
+__device__ __forceinline__ int rule_first_reject(const DecideParams &d, const BlockFacts &F, int r, int b, int lane) {
+    const int gamma = d.gamma;
     for (int c = 0; c < gamma; c += 32) {
         const int j = c + lane;
-        const bool fail = (j < gamma) && !accept(j);
-        const unsigned bal = __ballot_sync(0xFFFFFFFFu, fail);
+        const bool rej = (j < gamma) && !rule_accept(d, F, r, j, b);
+        const unsigned bal = __ballot_sync(0xFFFFFFFFu, rej);
         if (bal) return c + __ffs(bal) - 1;
     }
     return gamma;
 }
 
-// x_1..x_L, then `corr`, then -1, into a [gamma+1] token list.
-__device__ __forceinline__ void write_tokens(int lane, int gamma, int32_t *dst, const int32_t *xb, int L, int corr) {
-    for (int j = lane; j <= gamma; j += 32) dst[j] = (j < L) ? __ldg(xb + j) : (j == L ? corr : -1);
+// x_1..x_L, then `corr`, then -1, into a [gamma+1] token list, by one warp.
+__device__ __forceinline__ void write_tokens(int lane, int gamma, int32_t *dst, const int32_t *x, int L, int corr) {
+    for (int j = lane; j <= gamma; j += 32) dst[j] = (j < L) ? x[j] : (j == L ? corr : -1);
 }
 
-// Rules evaluated together, one chunk of 32 positions at a time: the block's
-// records are read once per chunk and every rule tests its acceptance on them;
-// a rule's correction token (the target argmax at its first rejection) is
-// taken from the lane holding that position.
-constexpr int kMaxRules = 1 + 2 * SDD_MAX_GRID;
+// Inclusive prefix sum of one double-float per lane (lane order).
+__device__ __forceinline__ df warp_prefix_df(df v, int lane) {
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        df t;
+        t.hi = __shfl_up_sync(0xFFFFFFFFu, v.hi, off);
+        t.lo = __shfl_up_sync(0xFFFFFFFFu, v.lo, off);
+        if (lane >= off) v = df_add(t, v);
+    }
+    return v;
+}
 
-template <int DT>
-__device__ void block_decide(const DecideParams &p, int i, int lane, int *s_L, int *s_corr) {
-    const int gamma = p.gamma;
-    const int b = p.bidx ? __ldg(p.bidx + i) : i;
-    if (b < 0 || b >= p.B) return;   // flagged by the streaming pass
-    const RowRec *tr = p.trec + static_cast<int64_t>(i) * (gamma + 1);
-    const int32_t *xb = p.tokens + static_cast<int64_t>(b) * gamma;
-    const int64_t bo = static_cast<int64_t>(b) * (gamma + 1);
-    const bool sampling = p.do_strict && !p.greedy;
-    // rule r: 0 strict, 1..n_ell lenience, then top-k
-    const int n_rules = 1 + p.n_ell + p.n_k;
-    for (int r = lane; r < n_rules; r += 32) s_L[r] = -1;
-    __syncwarp();
-    const int bonus_argmax = load_rec(tr + gamma).argmax;
-    int remaining = (p.do_strict ? 1 : 0) + p.n_ell + p.n_k;
-    for (int c = 0; c < gamma && remaining > 0; c += 32) {
-        const int j = c + lane;
-        const bool in = j < gamma;
-        RowRec t{};
-        if (in) t = load_rec(tr + j);
-        auto settle = [&](int r, bool accept) {
-            if (s_L[r] >= 0) return;
-            const unsigned bal = __ballot_sync(0xFFFFFFFFu, in && !accept);
-            if (bal) {
-                const int f = __ffs(bal) - 1;
-                const int corr = __shfl_sync(0xFFFFFFFFu, t.argmax, f);
-                if (lane == 0) {
-                    s_L[r] = c + f;
-                    s_corr[r] = corr;
-                }
-                __syncwarp();
-                --remaining;
-            }
-        };
-        if (p.do_strict) {
-            bool acc = true;
-            if (in) {
-                if (!sampling) {
-                    acc = t.rank == 0;
-                } else {
-                    double lse_d;
-                    float gd;
-                    if (p.drec) {
-                        const RowRec d = load_rec(p.drec + static_cast<int64_t>(i) * gamma + j);
-                        lse_d = d.lse;
-                        gd = d.g;
-                    } else {
-                        const int xj = __ldg(xb + j);
-                        const char *zdr = p.zd + (static_cast<int64_t>(b) * gamma + j) * p.stride_bytes;
-                        lse_d = __ldg(p.d_lse + static_cast<int64_t>(b) * gamma + j);
-                        gd = (xj >= 0 && xj < p.V) ? fmax_nan(logit_at<DT>(zdr, xj), clamp_floor()) : qnan();
-                    }
-                    // log r = log p_t(x_j) - log p_d(x_j) = (g_t - g_d) - (LSE_t - LSE_d)
-                    const double lr = static_cast<double>(t.g - gd) - (t.lse - lse_d);
-                    const float u = philox_uniform(p.seed, static_cast<uint32_t>(j + 1), static_cast<uint32_t>(b),
-                                                   p.round, kPurposeAccept);
-                    acc = (lr >= 0.0) || (u <= expf(static_cast<float>(lr)));
-                }
-            }
-            settle(0, acc);
-        }
-        for (int r = 0; r < p.n_ell; ++r)
-            settle(1 + r, p.ell_one[r] ? (t.rank == 0) : (static_cast<double>(t.g - t.M) >= p.ell_thr[r]));
-        for (int r = 0; r < p.n_k; ++r) settle(1 + p.n_ell + r, t.rank < p.kval[r]);
-    }
-    __syncwarp();
-    auto rule_L = [&](int r) { return s_L[r] >= 0 ? s_L[r] : gamma; };
-    auto rule_corr = [&](int r) { return s_L[r] >= 0 ? s_corr[r] : bonus_argmax; };
-    // ---- outputs of the rules ----
-    int L = gamma;
-    if (p.do_strict) {
-        L = rule_L(0);
-        if (!sampling) {
-            if (lane == 0) {
-                if (p.L_strict) p.L_strict[b] = L;
-                if (p.n_strict) p.n_strict[b] = L + 1;
-            }
-            if (p.tok_strict) write_tokens(lane, gamma, p.tok_strict + bo, xb, L, rule_corr(0));
-        } else if (lane == 0) {
-            p.blk_L[i] = L;   // the draw kernel completes the block
-        }
-    }
-    for (int r = 0; r < p.n_ell; ++r) {
-        const int Lr = rule_L(1 + r);
-        const int64_t o = static_cast<int64_t>(r) * p.B + b;
-        if (lane == 0) {
-            if (p.L_len) p.L_len[o] = Lr;
-            if (p.n_len) p.n_len[o] = Lr + 1;
-        }
-        if (p.tok_len) write_tokens(lane, gamma, p.tok_len + o * (gamma + 1), xb, Lr, rule_corr(1 + r));
-    }
-    for (int r = 0; r < p.n_k; ++r) {
-        const int Lr = rule_L(1 + p.n_ell + r);
-        const int64_t o = static_cast<int64_t>(r) * p.B + b;
-        if (lane == 0) {
-            if (p.L_topk) p.L_topk[o] = Lr;
-            if (p.n_topk) p.n_topk[o] = Lr + 1;
-        }
-        if (p.tok_topk) write_tokens(lane, gamma, p.tok_topk + o * (gamma + 1), xb, Lr, rule_corr(1 + p.n_ell + r));
-    }
-    // ---- fused round: schedule, agreement, tokens of skipped blocks ----
-    if (p.do_sched) {
-        const RowRec *dr = p.drec + static_cast<int64_t>(i) * gamma;
-        const bool force = p.force_strict && p.force_strict[b];
-        const int D = p.D_in ? p.D_in[b] : 0;
-        const float *qv = &dr->q;
-        const float *lqv = &dr->logq;
-        constexpr int kRecFloats = sizeof(RowRec) / sizeof(float);
-        for (int t = 0; t < p.n_tau; ++t) {
-            int Kh, K, Do;
-            schedule_block(lane, gamma, qv, lqv, kRecFloats, p.guard ? p.guard + static_cast<int64_t>(b) * gamma : nullptr,
-                           force || p.tau_off[t], D, p.signal, p.eta_loc[t], p.log_eta_c[t], p.K_min, p.S_max, Kh, K,
-                           Do);
-            if (lane == 0) {
-                const int64_t o = static_cast<int64_t>(t) * p.B + b;
-                if (p.K_hat) p.K_hat[o] = Kh;
-                if (p.K) p.K[o] = K;
-                if (p.D_out) p.D_out[o] = Do;
-                if (p.agreement && K > 0 && p.do_strict) {
-                    unsigned long long *a = reinterpret_cast<unsigned long long *>(p.agreement + 4 * t);
-                    atomicAdd(a + 0, static_cast<unsigned long long>(min(K, L)));
-                    atomicAdd(a + 1, static_cast<unsigned long long>(K));
-                    atomicAdd(a + 2, static_cast<unsigned long long>(K <= L ? 1 : 0));
-                    atomicAdd(a + 3, 1ull);
-                }
-            }
-            if (t == 0) {
-                if (lane == 0) p.k0[i] = K;   // read by the draw kernel
-                const bool skip = K > 0;
-                if (skip || (p.do_strict && !sampling)) {
-                    // skipped: x_1..x_K; greedy strict: the verified tokens
-                    const int Lc = skip ? K : L;
-                    const int corr = skip ? -1 : rule_corr(0);
-                    if (lane == 0 && p.commit_n) p.commit_n[b] = skip ? K : L + 1;
-                    if (p.commit_tokens) write_tokens(lane, gamma, p.commit_tokens + bo, xb, Lc, corr);
-                }
-            }
-        }
-    }
+// One chunk (positions c .. c+31, this lane's position j = c + lane, `in` iff
+// j < gamma) of the skip policy for one threshold pair.  kb = leading
+// positions passing the local gate so far (gamma while no position failed),
+// best = largest prefix length meeting Eq. 3 so far; both warp-uniform.
+// S = inclusive prefix sum of ln q through position j.
+__device__ __forceinline__ void sched_step(int c, int lane, int gamma, bool in, float qj, bool guard_j, const df &S,
+                                           const df &eta_loc, const df &log_eta_c, int signal, int &kb, int &best) {
+    if (kb < c) return;   // the gate failed in an earlier chunk
+    const bool fail = in && (guard_j || !isfinite(qj) || !df_ge(df{qj, 0.f}, eta_loc));
+    const unsigned bal = __ballot_sync(0xFFFFFFFFu, fail);
+    if (kb == gamma && bal) kb = c + __ffs(bal) - 1;
+    if (signal == SDD_SIG_MARGINAL) return;
+    const int j = c + lane;
+    bool pass = false;
+    if (in && j < kb)
+        pass = (signal == SDD_SIG_RAW) ? df_ge(S, df_mul_f(log_eta_c, static_cast<float>(j + 1)))
+                                       : df_ge(S, log_eta_c);
+    const unsigned bal2 = __ballot_sync(0xFFFFFFFFu, pass);
+    if (bal2) best = c + 32 - __clz(bal2);
+}
+
+// K_min / staleness gate of Sec. 4.1 on a block's K_hat.
+__device__ __forceinline__ void sched_final(int K_hat, int D, int K_min, int S_max, int &K, int &D_out) {
+    K = (D < S_max && K_hat > 0 && K_hat >= K_min) ? K_hat : 0;
+    D_out = (K > 0) ? D + K : 0;
 }
 
 }  // namespace sdd

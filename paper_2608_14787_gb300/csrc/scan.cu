@@ -1,23 +1,25 @@
 // scan.cu -- the streaming pass of the path: one read of every drafter and
-// target logit, producing per-row softmax statistics.
+// target logit, producing per-row partial softmax statistics.
 //
 // What it computes (per row of logits z over the vocabulary):
 //   M = max z, S = sum exp(z - M), T2 = sum exp(z - M) (z - M) log2(e),
 //   the lowest index attaining M, and for target rows the saturated rank of
 //   the drafted token x: #{v : z(v) > z(x)} + #{v < x : z(v) = z(x)}.
-// From these the merging warp derives the quantities of Sec. 4.2 (raw
-// confidence q = p_draft(x_j), LSE, maxprob, entropy) and the target facts that
-// the acceptance rules of Sec. 3.1 and App. A.6 read.
+// From these follow the quantities of Sec. 4.2 (raw confidence q = p_draft(x_j),
+// LSE, maxprob, entropy) and the target facts that the acceptance rules of
+// Sec. 3.1 and App. A.6 read.
 //
 // How: the rows of the call are laid end to end as one sequence of 16-byte
 // vectors, split into contiguous, equal ranges, one per warp (perfect balance,
 // no per-tile scheduling).  Each warp streams its range through a private
 // ring of 4 KiB shared-memory tiles filled by 1D bulk copies (cp.async.bulk +
-// mbarrier), keeps an online-softmax state per lane, reduces it across the
-// warp at the end of each row piece and publishes a 32-byte partial.  The
-// last warp to finish a row (atomic arrival counter, no waiting) merges the
-// row's partials in a fixed order and writes the row's results.
-#include "rules.cuh"
+// mbarrier), keeps an online-softmax state per lane (packed f32x2 arithmetic,
+// exp-sums as double-floats), reduces it across the warp at the end of each
+// row piece and publishes a 32-byte partial.
+// The decide kernel (decide.cu) merges each row's partials and finalises the
+// rows; keeping that out of the streaming kernel keeps this kernel free of
+// register spills.
+#include "internal.h"
 
 namespace sdd {
 
@@ -48,16 +50,6 @@ __device__ __forceinline__ const char *row_base(const ScanParams &p, int64_t r) 
     row_locate(p, r, gi, lr, j, b, ok);
     const ScanGroup &G = p.grp[gi];
     return G.base + (static_cast<int64_t>(b) * G.npos + j) * G.stride_bytes;
-}
-
-template <int DT>
-__device__ __forceinline__ float load_logit(const char *rowp, int v) {
-    if (DT == SDD_BF16) {
-        const uint16_t h = __ldg(reinterpret_cast<const unsigned short *>(rowp) + v);
-        return __uint_as_float(static_cast<uint32_t>(h) << 16);
-    } else {
-        return __ldg(reinterpret_cast<const float *>(rowp) + v);
-    }
 }
 
 // Entries of one 16-byte vector past the end of the row become -inf.
@@ -137,19 +129,26 @@ __device__ __noinline__ int count_before(const uint4 *tile, int n, int k0, int l
 }
 
 // Resolve a lane's argmax: the first of its entries equal to m inside the tile
-// that starts at vector k0 of the row (re-read from global memory; the row's
-// padding and entries past V are excluded).
+// that starts at vector k0 of the row (re-read from global memory, all loads
+// issued before the first compare; the row's padding and entries past V are
+// excluded).
 template <int DT>
 __device__ __noinline__ int first_index(const char *rowp, int k0, int lane, int RV, int V, float m) {
     constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
-#pragma unroll 1
+    uint4 w[kVPL];
+#pragma unroll
+    for (int i = 0; i < kVPL; ++i) {
+        const int vec = k0 + lane + 32 * i;
+        w[i] = (vec < RV) ? __ldg(reinterpret_cast<const uint4 *>(rowp) + vec) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
     for (int i = 0; i < kVPL; ++i) {
         const int vec = k0 + lane + 32 * i;
         if (vec >= RV) break;
-        const uint4 w = clamp_vec<DT>(__ldg(reinterpret_cast<const uint4 *>(rowp) + vec));
+        const uint4 c = clamp_vec<DT>(w[i]);
 #pragma unroll
         for (int e = 0; e < EPV; ++e)
-            if (vec * EPV + e < V && vec_elem<DT>(w, e) == m) return vec * EPV + e;
+            if (vec * EPV + e < V && vec_elem<DT>(c, e) == m) return vec * EPV + e;
     }
     return INT32_MAX;
 }
@@ -158,39 +157,31 @@ __device__ __noinline__ int first_index(const char *rowp, int k0, int lane, int 
 // Sums are relative to the integer reference st.r (log2 units), so a new
 // maximum rescales by an exact power of two.  A new maximum only records the
 // tile (st.amax = k0); the exact index is resolved once at the end of the piece.
-// Error-free sum of two fp32 values (Knuth's TwoSum): a + b = s + err exactly.
-__device__ __forceinline__ void two_sum(float a, float b, float &s, float &err) {
-    s = a + b;
-    const float bb = s - a;
-    err = (a - (s - bb)) + (b - bb);
-}
-
-// The lane's running exp-sum is kept as an unevaluated fp32 pair (hi, lo)
-// (compensated summation), so the hot loop needs no fp64 arithmetic; the pair
-// is folded into st.s (fp64) at the end of each row piece.
-template <int DT>
+// Pairs of entries go through the packed f32x2 pipe: y = z log2(e) - r,
+// s += 2^y and, for drafter rows (ENT), t2 += 2^y y.  Drafter entries are
+// clamped first (so a masked entry adds 0 * finite to t2); target rows need no
+// clamp (2^-inf = 0 and the maximum starts at the clamp value).  The lane's
+// exp-sum is an fp32 pair (s_hi, s_lo) updated by TwoSum once per tile.
+template <int DT, bool ENT>
 __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lane, SoftState &st, float &s_hi,
                                               float &s_lo) {
-    uint4 w[kVPL];
-#pragma unroll
-    for (int i = 0; i < kVPL; ++i) w[i] = clamp_vec<DT>(tile[lane + 32 * i]);
+    // pass 1: the tile maximum (clamp value included)
     float cm;
     if (DT == SDD_BF16) {
         uint32_t mx = kClampPairBf16;
 #pragma unroll
         for (int i = 0; i < kVPL; ++i) {
-            const uint32_t *u = reinterpret_cast<const uint32_t *>(&w[i]);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) mx = bf16x2_max_nan(mx, u[q]);
+            const uint4 w = tile[lane + 32 * i];
+            mx = bf16x2_max_nan(bf16x2_max_nan(mx, w.x), bf16x2_max_nan(w.y, bf16x2_max_nan(w.z, w.w)));
         }
         cm = fmax_nan(bf16_lo(mx), bf16_hi(mx));
     } else {
         cm = clamp_floor();
 #pragma unroll
         for (int i = 0; i < kVPL; ++i) {
-            const float *f = reinterpret_cast<const float *>(&w[i]);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) cm = fmax_nan(cm, f[q]);
+            const uint4 w = tile[lane + 32 * i];
+            cm = fmax_nan(fmax_nan(cm, __uint_as_float(w.x)),
+                          fmax_nan(__uint_as_float(w.y), fmax_nan(__uint_as_float(w.z), __uint_as_float(w.w))));
         }
     }
     if (cm > st.m) {
@@ -200,139 +191,83 @@ __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lan
         if (rn > st.r) {
             const float k = st.r - rn;
             const float sc = pow2f_int(k);   // exact power of two (0 below the normal range)
-            st.t2 = sc * (st.t2 + k * (s_hi + s_lo));
+            if (ENT) st.t2 = sc * fmaf(k, s_hi + s_lo, st.t2);
             s_hi *= sc;
             s_lo *= sc;
             st.r = rn;
         }
     }
-    // y = z log2(e) - r; s += 2^y; t2 += 2^y y   (two accumulators each)
+    // pass 2: the exp-sums, two vectors per step re-read from shared memory
+    // (a bounded register footprint)
     const float nr = -st.r;
-    float s0 = 0.f, s1 = 0.f, t0 = 0.f, t1 = 0.f;
+    const f2_t L2 = f2_pack(kLog2e, kLog2e), NR = f2_pack(nr, nr);
+    f2_t sa = f2_pack(0.f, 0.f), sb = sa, ta = sa, tb = sa;
+    constexpr int PAIRS = (DT == SDD_BF16) ? 4 : 2;   // entry pairs per 16-byte vector
+#pragma unroll 1
+    for (int i = 0; i < kVPL; i += 2) {
+        uint4 w[2];
+        w[0] = tile[lane + 32 * i];
+        w[1] = tile[lane + 32 * (i + 1)];
 #pragma unroll
-    for (int i = 0; i < kVPL; ++i) {
-        const uint32_t *u = reinterpret_cast<const uint32_t *>(&w[i]);
+        for (int h = 0; h < 2; ++h) {
+            if (ENT) w[h] = clamp_vec<DT>(w[h]);
+            const uint32_t *u = reinterpret_cast<const uint32_t *>(&w[h]);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            if (DT == SDD_BF16) {
-                const float y0 = fmaf(bf16_lo(u[q]), kLog2e, nr);
-                const float y1 = fmaf(bf16_hi(u[q]), kLog2e, nr);
-                const float e0 = ex2(y0), e1 = ex2(y1);
-                s0 += e0;
-                t0 = fmaf(e0, y0, t0);
-                s1 += e1;
-                t1 = fmaf(e1, y1, t1);
-            } else {
-                const float y0 = fmaf(__uint_as_float(u[q]), kLog2e, nr);
-                const float e0 = ex2(y0);
+            for (int q = 0; q < PAIRS; ++q) {
+                const f2_t z = (DT == SDD_BF16) ? f2_pack(bf16_lo(u[q]), bf16_hi(u[q]))
+                                                : f2_pack(__uint_as_float(u[2 * q]), __uint_as_float(u[2 * q + 1]));
+                const f2_t y = f2_fma(z, L2, NR);
+                float y0, y1;
+                f2_unpack(y, y0, y1);
+                const f2_t e = f2_pack(ex2(y0), ex2(y1));
                 if (q & 1) {
-                    s1 += e0;
-                    t1 = fmaf(e0, y0, t1);
+                    sb = f2_add(sb, e);
+                    if (ENT) tb = f2_fma(e, y, tb);
                 } else {
-                    s0 += e0;
-                    t0 = fmaf(e0, y0, t0);
+                    sa = f2_add(sa, e);
+                    if (ENT) ta = f2_fma(e, y, ta);
                 }
             }
         }
     }
+    float s0, s1;
+    f2_unpack(f2_add(sa, sb), s0, s1);
     float e1, e2, h;
     two_sum(s_hi, s0, h, e1);
     two_sum(h, s1, s_hi, e2);
     s_lo += e1 + e2;
-    st.t2 += t0 + t1;
+    if (ENT) {
+        float t0, t1;
+        f2_unpack(f2_add(ta, tb), t0, t1);
+        st.t2 += t0 + t1;
+    }
     return cm;
 }
 
-// Final results of row r from its merged state (whole warp calls; lane 0 writes).
-template <int DT>
-__device__ void finalize_row(const ScanParams &p, int64_t r, SoftState st, int lane) {
-    int gi, j, b;
-    int64_t lr;
-    bool b_ok;
-    row_locate(p, r, gi, lr, j, b, b_ok);
-    const ScanGroup &G = p.grp[gi];
-    const char *rowp = G.base + (static_cast<int64_t>(b) * G.npos + j) * G.stride_bytes;
-    const bool has_tok = j < p.gamma;
-    int tok = has_tok ? __ldg(p.tokens + static_cast<int64_t>(b) * p.gamma + j) : -1;
-    const bool tok_ok = has_tok && tok >= 0 && tok < p.V;
-    const bool valid = b_ok && isfinite(st.m) && st.m > clamp_floor() && isfinite(st.s) && st.s > 0.0;
-    if (lane != 0) return;
-    const float nanf_ = __int_as_float(0x7FC00000);
-    float g = nanf_;
-    if (tok_ok) g = fmax_nan(load_logit<DT>(rowp, tok), clamp_floor());
-    RowRec rec;
-    const int64_t o = static_cast<int64_t>(b) * p.gamma + j;
-    if (valid) {
-        // The lane that held the row maximum M took its term as ex2(y_M) with
-        // y_M = M log2(e) - ceil(M log2(e)) (its reference when M arrived).  On a
-        // peaked row that one term dominates S, so its MUFU approximation error
-        // is replaced by the exact power of two (scaled to the final reference).
-        const float rM = ceilf(st.m * kLog2e);
-        const float yM = fmaf(st.m, kLog2e, -rM);
-        const double S = st.s + (exp2(static_cast<double>(yM)) - static_cast<double>(ex2(yM))) * pow2d_int(rM - st.r);
-        st.s = S;
-        // all in fp64: LSE = r ln2 + ln S (S relative to the reference r)
-        const double lnS = log(st.s);
-        const double lse = static_cast<double>(st.r) * kLn2d + lnS;
-        rec.lse = lse;
-        rec.M = st.m;
-        rec.g = g;
-        rec.logq = static_cast<float>(static_cast<double>(g) - lse);
-        rec.q = static_cast<float>(exp(static_cast<double>(g) - lse));
-        rec.argmax = st.amax;
-        rec.rank = min(st.rank, p.kcap);
-        if (G.kind == 0 && b_ok) {
-            if (G.q) G.q[o] = tok_ok ? rec.q : nanf_;
-            if (G.logq) G.logq[o] = tok_ok ? rec.logq : nanf_;
-            if (G.maxprob) G.maxprob[o] = static_cast<float>(exp(static_cast<double>(st.m) - lse));
-            if (G.lse) G.lse[o] = lse;
-            if (G.entropy) G.entropy[o] = static_cast<float>(lnS - kLn2d * static_cast<double>(st.t2) / st.s);
-            if (G.argmax) G.argmax[o] = st.amax;
+// Drafted token of global row r, if the row has one (load issued, not waited on).
+struct RowTok {
+    int t;
+    bool has;
+};
+__device__ __forceinline__ RowTok row_token(const ScanParams &p, int64_t r) {
+    RowTok x{0, false};
+    if (r < p.rows) {
+        int gi, j, b;
+        int64_t lr;
+        bool ok;
+        row_locate(p, r, gi, lr, j, b, ok);
+        if (j < p.gamma) {
+            x.t = __ldg(p.tokens + static_cast<int64_t>(b) * p.gamma + j);
+            x.has = true;
         }
-    } else {
-        rec.lse = __longlong_as_double(0x7FF8000000000000ll);
-        rec.M = rec.g = rec.q = rec.logq = nanf_;
-        rec.argmax = -1;
-        rec.rank = INT32_MAX;
-        if (G.kind == 0 && b_ok) {
-            if (G.q) G.q[o] = nanf_;
-            if (G.logq) G.logq[o] = nanf_;
-            if (G.maxprob) G.maxprob[o] = nanf_;
-            if (G.lse) G.lse[o] = rec.lse;
-            if (G.entropy) G.entropy[o] = nanf_;
-            if (G.argmax) G.argmax[o] = -1;
-        }
-        if (b_ok) status_or(p.status, SDD_DEV_NONFINITE);
     }
-    if (has_tok && !tok_ok) {
-        rec.q = rec.logq = rec.g = nanf_;
-        rec.rank = INT32_MAX;
-    }
-    if ((has_tok && !tok_ok) || !b_ok) status_or(p.status, SDD_DEV_BAD_TOKEN);
-    G.rec[lr] = rec;
+    return x;
 }
-
-// A row of list block i is final: count it, and let the warp that completes
-// the block evaluate the block's decisions (rules.cuh).
+// Clamped logit of row r at its drafted token (NaN if none or out of range).
 template <int DT>
-__device__ __forceinline__ void block_arrive(const ScanParams &p, int64_t r, int lane) {
-    const int gi = (r >= p.rows0) ? 1 : 0;
-    const int64_t lr = gi ? r - p.rows0 : r;
-    const int i = static_cast<int>(lr / p.grp[gi].npos);
-    __syncwarp();
-    uint32_t old = 0;
-    if (lane == 0) {
-        __threadfence();
-        old = atomicAdd(p.dec.blk_count + i, 1u);
-    }
-    old = __shfl_sync(0xFFFFFFFFu, old, 0);
-    if (old == static_cast<uint32_t>(p.dec.rows_per_block - 1)) {
-        __threadfence();
-        __shared__ int s_rule_L[kWarpsPerCta][kMaxRules], s_rule_corr[kWarpsPerCta][kMaxRules];
-        const int w = threadIdx.x >> 5;
-        block_decide<DT>(p.dec, i, lane, s_rule_L[w], s_rule_corr[w]);
-        if (lane == 0) p.dec.blk_count[i] = 0u;   // leave the workspace zeroed
-    }
+__device__ __forceinline__ float token_logit(const ScanParams &p, int64_t r, RowTok x) {
+    if (!x.has || x.t < 0 || x.t >= p.V) return __int_as_float(0x7FC00000);
+    return fmax_nan(logit_at<DT>(row_base(p, r), x.t), clamp_floor());
 }
 
 template <int DT>
@@ -381,12 +316,20 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
     };
     for (int s = 0; s < kStages && pc.v < v1; ++s) issue(s);
 
+    // Drafted tokens and their logits run ahead of the stream: the token two
+    // rows ahead and the logit one row ahead are in flight while the current
+    // piece streams, so no piece start waits on a dependent pair of loads.
+    RowTok tokA = row_token(p, cc.r), tokB = row_token(p, cc.r + 1);
+    float gA = token_logit<DT>(p, cc.r, tokA);
+
     SoftState st = soft_identity();
     float s_hi = 0.f, s_lo = 0.f;   // the lane's exp-sum as an fp32 pair
     bool in_piece = false;
-    int tok = -1;          // drafted token of the current target row (-1: none)
-    float g = 0.f;         // its clamped logit
-    bool rank_on = false;  // warp-uniform: the rank of tok is still below kcap
+    bool ent = false;      // warp-uniform: drafter row (entropy accumulator, clamped entries)
+    int tok = -1;          // drafted token of the current row (-1: none or out of range)
+    bool tok_bad = false;  // the row has a drafted token outside [0, V)
+    float g = 0.f;         // its clamped logit (NaN if none)
+    bool rank_on = false;  // warp-uniform: target row whose token's rank is still below kcap
     int wrank = 0;         // warp-uniform running rank count
     const char *crow = nullptr;
     int slot = 0;
@@ -403,16 +346,16 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
             row_locate(p, cc.r, gi, lr, j, b, ok);
             const ScanGroup &G = p.grp[gi];
             crow = G.base + (static_cast<int64_t>(b) * G.npos + j) * G.stride_bytes;
-            tok = -1;
-            g = 0.f;
-            if (G.kind == 1 && j < p.gamma) {
-                const int t = __ldg(p.tokens + static_cast<int64_t>(b) * p.gamma + j);
-                if (t >= 0 && t < p.V) {
-                    tok = t;
-                    g = fmax_nan(load_logit<DT>(crow, t), clamp_floor());
-                }
-            }
-            rank_on = tok >= 0;
+            ent = G.kind == 0;
+            const bool tok_ok = tokA.has && tokA.t >= 0 && tokA.t < p.V;
+            tok = tok_ok ? tokA.t : -1;
+            tok_bad = tokA.has && !tok_ok;
+            g = gA;
+            // advance the prefetch: logit of the next row, token of the one after
+            gA = token_logit<DT>(p, cc.r + 1, tokB);
+            tokA = tokB;
+            tokB = row_token(p, cc.r + 2);
+            rank_on = !ent && tok >= 0;
             wrank = 0;
             in_piece = true;
         }
@@ -423,7 +366,8 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
         uint4 *tile = reinterpret_cast<uint4 *>(ring + slot * kTileBytes);
         const bool row_end = (cc.k + n == p.RV);
         if (n < kTileVec || (row_end && tail)) pad_tile<DT>(tile, n, lane, row_end, tail);
-        const float cm = process_tile<DT>(tile, cc.k, lane, st, s_hi, s_lo);
+        const float cm = ent ? process_tile<DT, true>(tile, cc.k, lane, st, s_hi, s_lo)
+                             : process_tile<DT, false>(tile, cc.k, lane, st, s_hi, s_lo);
         if (rank_on) {
             const bool want = cm >= g;
             if (__any_sync(0xFFFFFFFFu, want)) {
@@ -452,50 +396,20 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
             if (st.m == M && st.amax != INT32_MAX) idx = first_index<DT>(crow, st.amax, lane, p.RV, p.V, M);
             st.amax = idx;
             st.rank = (lane == 0) ? wrank : 0;
-            st.s = static_cast<double>(s_hi) + static_cast<double>(s_lo);
-            SoftState red = soft_warp_reduce(st);
-            const int64_t fw = part_owner(cc.r * p.RV, p.T, p.W);
-            const int64_t lw = part_owner((cc.r + 1) * p.RV - 1, p.T, p.W);
-            if (fw == lw) {
-                finalize_row<DT>(p, cc.r, red, lane);
-                if (p.dec.enabled) block_arrive<DT>(p, cc.r, lane);
-            } else {
-                if (lane == 0) {
-                    Partial pt;
-                    pt.m = red.m;
-                    pt.r = red.r;
-                    pt.t2 = red.t2;
-                    pt.amax = red.amax;
-                    pt.rank = red.rank;
-                    pt.pad = 0;
-                    pt.s = red.s;
-                    p.partials[cc.r + gw] = pt;
-                }
-                uint32_t old = 0;
-                if (lane == 0) {
-                    __threadfence();
-                    old = atomicAdd(p.counters + cc.r, 1u);
-                }
-                old = __shfl_sync(0xFFFFFFFFu, old, 0);
-                if (old == static_cast<uint32_t>(lw - fw)) {
-                    __threadfence();
-                    SoftState acc = soft_identity();
-                    for (int64_t w = fw + lane; w <= lw; w += 32) {
-                        const Partial *pp = p.partials + cc.r + w;
-                        SoftState o;
-                        o.m = __ldcg(&pp->m);
-                        o.r = __ldcg(&pp->r);
-                        o.t2 = __ldcg(&pp->t2);
-                        o.s = __ldcg(&pp->s);
-                        o.amax = __ldcg(&pp->amax);
-                        o.rank = __ldcg(&pp->rank);
-                        acc = soft_merge(acc, o);
-                    }
-                    acc = soft_warp_reduce(acc);
-                    if (lane == 0) p.counters[cc.r] = 0u;  // leave the workspace zeroed
-                    finalize_row<DT>(p, cc.r, acc, lane);
-                    if (p.dec.enabled) block_arrive<DT>(p, cc.r, lane);
-                }
+            st.sh = s_hi;
+            st.sl = s_lo;
+            const SoftState red = soft_warp_reduce(st);
+            if (lane == 0) {
+                Partial pt;
+                pt.m = red.m;
+                pt.r = red.r;
+                pt.t2 = red.t2;
+                pt.sh = red.sh;
+                pt.sl = red.sl;
+                pt.amax = red.amax;
+                pt.rank = tok_bad ? -1 : red.rank;
+                pt.g = g;
+                p.partials[cc.r + gw] = pt;
             }
             in_piece = false;
             if (row_end) {
