@@ -32,6 +32,10 @@ sys.path.insert(0, ROOT)
 METRIC = "draft blocks verified+scheduled/sec at γ=32,V=151,936 bf16; achieved HBM GB/s vs peak"
 UNIT = "blocks/s"
 NEAR = 1e-6
+# dram__bytes_read.sum + dram__bytes_write.sum of one scan_kernel launch on the
+# c3 workload (318.29 MB + 3.93 MB), from one ncu capture of the kernel as it
+# stands; reported as the roofline's "traffic" for that workload only.
+SCAN_TRAFFIC_C3 = 322_222_336
 
 
 def _peaks():
@@ -362,6 +366,8 @@ def main():
     ap.add_argument("--traffic", type=float, default=None,
                     help="dram bytes per scan launch from an ncu capture of the current kernel")
     args = ap.parse_args()
+    if args.traffic is None and args.workload == "c3":
+        args.traffic = SCAN_TRAFFIC_C3
     if args.warmup < 3:
         args.warmup = 3
     if args.impl == "reference":
