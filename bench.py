@@ -200,6 +200,7 @@ def _e2e(args, ws, dev, stream, sets, rnd, wl, B):
     """The same round end to end through the C ABI: inputs copied from pinned
     host buffers and results copied back inside the timed region."""
     import torch
+    from paper_2608_14787_gb300 import shard
     if ws > 1:
         import torch.distributed as dist
     hz_d = sets[0].z_d.cpu().pin_memory()
@@ -232,11 +233,7 @@ def _e2e(args, ws, dev, stream, sets, rnd, wl, B):
         e2e_step(i)
     e1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
-    if ws > 1:
-        t = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = shard.max_over_ranks(e0.elapsed_time(e1), device=dev)
     return ws * B * e2e_steps / (e2e_ms / 1e3), h2d, d2h
 
 
@@ -244,7 +241,7 @@ def run_gpu(args):
     import torch
     import paper_2608_14787_gb300 as sdd
     from paper_2608_14787_gb300 import build as sdd_build
-    from paper_2608_14787_gb300 import synth
+    from paper_2608_14787_gb300 import shard, synth
 
     ws, rank, local = _dist()
     if ws > 1:
@@ -303,10 +300,7 @@ def run_gpu(args):
     total_ms = t_start.elapsed_time(t_end)
     scan_ms = [a.elapsed_time(b) for a, b in evs]
     scan_avg_ms = sum(scan_ms) / len(scan_ms)
-    if ws > 1:
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = shard.max_over_ranks(total_ms, device=dev)   # blocks shard by rank: no data-path exchange
     value = ws * B * args.steps / (total_ms / 1e3)
     status = int(rnd.status.item())
 
