@@ -16,6 +16,8 @@ marshals numpy arrays into it and composes its steps in the paper's order:
 * ``verify_topk``        -- App. A.6 top-k acceptance.
 * ``agreement``          -- Sec. 3.2 Eq. 1 (StrictToken) and Eq. 2 (FullPrefix).
 * ``philox4x32_10`` / ``uniform`` -- the counter-based uniforms of the sampling rule.
+* ``survival_mlp``       -- the decode-loop workload's stand-in survival scorer
+                            sigmoid(w2 . GELU(W1 h + b1) + b2) (App. A.7 form).
 
 Logit arrays are numpy ``float32`` (fp32 logits) or ``uint16`` (the raw bits of
 bf16 logits); both are converted exactly to fp64 inside the C code.
@@ -98,6 +100,10 @@ def lib():
     L.orc_verify_greedy_family.restype = None
     L.orc_agreement.argtypes = [ip32, ip32, ctypes.c_int, ip64]
     L.orc_agreement.restype = None
+    u16p, f32p, f64p = _P(ctypes.c_uint16), _P(ctypes.c_float), _P(ctypes.c_double)
+    L.orc_survival_mlp.argtypes = [u16p, ctypes.c_int, ctypes.c_int, u16p, f32p, u16p, ctypes.c_double,
+                                   ctypes.c_int, f64p]
+    L.orc_survival_mlp.restype = None
     _lib = L
     return L
 
@@ -315,6 +321,23 @@ def verify_strict(zt_block, zd_block, x, seed: int, b: int, round_: int):
     u_res = uniform(seed, L + 1, b, round_, PURPOSE_RESID)
     u_bonus = uniform(seed, gamma + 1, b, round_, PURPOSE_BONUS)
     return strict_sample_probs(pt, pd, x, u_acc, u_res, u_bonus)
+
+
+def survival_mlp(h_bits, W1_bits, b1, w2_bits, b2: float) -> np.ndarray:
+    """fp64 sigmoid(w2 . GELU(W1 h + b1) + b2) per row of h.  h_bits [M, K] and
+    W1_bits [N, K] / w2_bits [N] are the raw bits of bf16 arrays (uint16), b1 fp32 [N]."""
+    h = np.ascontiguousarray(np.asarray(h_bits, dtype=np.uint16))
+    W1 = np.ascontiguousarray(np.asarray(W1_bits, dtype=np.uint16))
+    w2 = np.ascontiguousarray(np.asarray(w2_bits, dtype=np.uint16))
+    b1 = np.ascontiguousarray(np.asarray(b1, dtype=np.float32))
+    M, K = h.shape
+    N = W1.shape[0]
+    if W1.shape != (N, K) or w2.shape != (N,) or b1.shape != (N,):
+        raise ValueError("shape mismatch")
+    out = np.zeros(M, np.float64)
+    lib().orc_survival_mlp(_ptr(h, ctypes.c_uint16), M, K, _ptr(W1, ctypes.c_uint16), _ptr(b1, ctypes.c_float),
+                           _ptr(w2, ctypes.c_uint16), float(b2), N, _ptr(out, ctypes.c_double))
+    return out
 
 
 def agreement(K, L):

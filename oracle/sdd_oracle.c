@@ -391,3 +391,26 @@ void orc_agreement(const int32_t *K, const int32_t *L, int B, int64_t acc[4]) {
         acc[3] += 1;
     }
 }
+
+/* ------------------------------------------------------------------------ */
+/* Stand-in survival scorer of the decode-loop workload: per position, from   */
+/* the drafter hidden state h (K values), s = sigmoid(w2 . GELU(W1 h + b1) +  */
+/* b2) with N hidden units, GELU(z) = z Phi(z) = z (1 + erf(z / sqrt 2)) / 2. */
+/* The paper's learned scorer (App. A.7) has this form with more layers and   */
+/* trained weights; the stand-in is random-init.  W1 is [N, K] (one row per  */
+/* hidden unit), h is [M, K]; both bf16 bits, converted exactly.             */
+/* ------------------------------------------------------------------------ */
+void orc_survival_mlp(const uint16_t *h, int M, int K, const uint16_t *W1, const float *b1, const uint16_t *w2,
+                      double b2, int N, double *out) {
+    for (int m = 0; m < M; ++m) {
+        double t = b2;
+        for (int n = 0; n < N; ++n) {
+            double z = (double)b1[n];
+            for (int k = 0; k < K; ++k)
+                z += orc_load(W1, ORC_BF16, (int64_t)n * K + k) * orc_load(h, ORC_BF16, (int64_t)m * K + k);
+            const double gelu = 0.5 * z * (1.0 + erf(z / sqrt(2.0)));
+            t += orc_load(w2, ORC_BF16, n) * gelu;
+        }
+        out[m] = 1.0 / (1.0 + exp(-t));
+    }
+}
