@@ -242,6 +242,28 @@ SDD_API sdd_status_t sdd_uniforms(uint64_t seed, const uint32_t *j, const uint32
                                   const uint32_t *purpose, int64_t n, float *u, sdd_stream_t stream);
 
 /*
+ * sdd_survival_mlp -- a learned-style survival score per draft position (the
+ * form of the scorer of App. A.7 with one hidden layer; the decode-loop
+ * workload uses it with random weights as a stand-in for the trained one):
+ *   s[m] = sigmoid(w2 . GELU(W1 h[m] + b1) + b2),  GELU(z) = z Phi(z) (erf form),
+ * for M positions (m = b * gamma + j).  The scores feed sdd_schedule_prefix as q
+ * (the conditional survival signal of Sec. 4.2 treats them as per-position
+ * survival probabilities).  The product W1 h runs on the tensor cores (bf16
+ * inputs, fp32 accumulation).
+ *   h   [M, K] bf16, row-major, 16-byte aligned (drafter hidden states);
+ *       K a positive multiple of SDD_MLP_KSTEP.
+ *   W1  [SDD_MLP_HIDDEN, K] bf16, row-major (one row per hidden unit), 16-byte aligned.
+ *   b1  [SDD_MLP_HIDDEN] fp32; w2 [SDD_MLP_HIDDEN] bf16; b2 a host scalar.
+ *   s   [M] fp32 output.
+ * Needs an sm_10x device (returns SDD_ERR_UNSUPPORTED otherwise).  A bounded
+ * wait that gives up sets SDD_DEV_TIMEOUT in *status (s is then undefined).
+ */
+#define SDD_MLP_HIDDEN 256
+#define SDD_MLP_KSTEP 64
+SDD_API sdd_status_t sdd_survival_mlp(const void *h, int M, int K, const void *W1, const float *b1, const void *w2,
+                                      float b2, float *s, int32_t *status, sdd_stream_t stream);
+
+/*
  * sdd_confidence_noalloc -- sdd_confidence without a workspace, for callers
  * that cannot allocate device memory where they need the statistics: code
  * running inside CUDA stream capture (where cudaMalloc is not allowed),

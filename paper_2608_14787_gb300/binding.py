@@ -86,6 +86,8 @@ def load(path: str | None = None):
     L.sdd_uniforms.argtypes = [u64, VP, VP, VP, VP, i64, VP, VP]
     L.sdd_confidence_noalloc.argtypes = [VP, I, I, I, I, i64, VP, VP, VP, VP, VP, VP, VP, VP, VP]
     L.sdd_confidence_noalloc.restype = I
+    L.sdd_survival_mlp.argtypes = [VP, I, I, VP, VP, VP, ctypes.c_float, VP, VP, VP]
+    L.sdd_survival_mlp.restype = I
     for fn in ("sdd_block", "sdd_block_scan", "sdd_block_decide"):
         getattr(L, fn).argtypes = [ctypes.POINTER(BlockArgs), VP]
     for fn in ("sdd_workspace_size", "sdd_confidence", "sdd_schedule_prefix", "sdd_verify_strict",
@@ -301,6 +303,30 @@ def commit(K, x, verified_tokens, verified_n, stream=None):
     _check(load().sdd_commit(_p(K), _p(x), _p(verified_tokens), _p(verified_n), B, gamma, _p(out_t), _p(out_n),
                              _stream(stream)), "sdd_commit")
     return out_t, out_n
+
+
+MLP_HIDDEN = 256
+MLP_KSTEP = 64
+
+
+def survival_mlp(h, W1, b1, w2, b2: float, *, status=None, stream=None, out=None):
+    """sdd_survival_mlp: sigmoid(w2 . GELU(W1 h + b1) + b2) per row of h.
+    h bf16 [M, K] (or [B, gamma, K]), W1 bf16 [256, K], b1 fp32 [256], w2 bf16 [256];
+    returns fp32 scores shaped like h without its last dimension."""
+    lead = h.shape[:-1]
+    K = h.shape[-1]
+    h2 = h.reshape(-1, K)
+    for t, name, dt in ((h2, "h", torch.bfloat16), (W1, "W1", torch.bfloat16), (w2, "w2", torch.bfloat16),
+                        (b1, "b1", torch.float32)):
+        if t.dtype != dt or not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous CUDA {dt} tensor")
+    if W1.shape != (MLP_HIDDEN, K) or b1.shape != (MLP_HIDDEN,) or w2.shape != (MLP_HIDDEN,):
+        raise ValueError("W1 must be [256, K], b1 and w2 [256]")
+    M = h2.shape[0]
+    s = torch.empty(M, dtype=torch.float32, device=h.device) if out is None else out
+    _check(load().sdd_survival_mlp(_p(h2), M, K, _p(W1), _p(b1), _p(w2), float(b2), _p(s), _p(status),
+                                   _stream(stream)), "sdd_survival_mlp")
+    return s.reshape(lead)
 
 
 def uniforms(seed, j, b, round_, purpose, stream=None):

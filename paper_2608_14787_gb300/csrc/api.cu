@@ -479,6 +479,29 @@ sdd_status_t sdd_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, c
     return SDD_OK;
 }
 
+sdd_status_t sdd_survival_mlp(const void *h, int M, int K, const void *W1, const float *b1, const void *w2, float b2,
+                              float *s, int32_t *status, sdd_stream_t stream) {
+    if (M < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "M = %d < 0", M);
+    if (K < SDD_MLP_KSTEP || K % SDD_MLP_KSTEP != 0)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "K = %d is not a positive multiple of %d", K, SDD_MLP_KSTEP);
+    if (M == 0) return SDD_OK;
+    SDD_TRY(check_ptr16(h, "h"));
+    SDD_TRY(check_ptr16(W1, "W1"));
+    if (!b1 || !w2 || !s) return fail(SDD_ERR_INVALID_ARGUMENT, "b1, w2 and s must not be NULL");
+    int d = 0;
+    cudaError_t e = cudaGetDevice(&d);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    int major = 0, minor = 0;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, d);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, d);
+    if (major != 10) return fail(SDD_ERR_UNSUPPORTED, "tcgen05 scorer needs an sm_10x device (found sm_%d%d)", major, minor);
+    const char *why = nullptr;
+    e = launch_mlp(h, M, K, W1, b1, w2, b2, s, status, reinterpret_cast<cudaStream_t>(stream), &why);
+    if (why) return fail(SDD_ERR_CUDA, "survival scorer: %s", why);
+    if (e != cudaSuccess) return cuda_fail(e, "survival scorer launch");
+    return SDD_OK;
+}
+
 static sdd_status_t block_check(const sdd_block_args *a) {
     if (!a) return fail(SDD_ERR_INVALID_ARGUMENT, "args is NULL");
     SDD_TRY(check_shape(static_cast<sdd_dtype_t>(a->dtype), a->B, a->gamma, a->V, a->row_stride));

@@ -125,6 +125,9 @@ cudaError_t launch_commit(const int32_t *K, const int32_t *x, const int32_t *vt,
                           int gamma, int32_t *out_t, int32_t *out_n, cudaStream_t stream);
 cudaError_t launch_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, const uint64_t *round,
                             const uint32_t *purpose, int64_t n, float *u, cudaStream_t stream);
+// The stand-in survival scorer (mlp.cu); *why names a host-side failure.
+cudaError_t launch_mlp(const void *h, int M, int K, const void *W1, const float *b1, const void *w2, float b2,
+                       float *out, int32_t *status, cudaStream_t stream, const char **why);
 int scan_max_ctas_per_sm();
 int decide_max_ctas_per_sm();
 cudaError_t scan_prepare_device();

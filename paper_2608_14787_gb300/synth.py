@@ -199,11 +199,12 @@ def make_block(wl: Workload | str, device="cpu", round_: int = 0, greedy_drafts:
 
 
 def make_mlp(device="cpu", seed: int = 4, hidden: int = HIDDEN, width: int = MLP_HIDDEN):
-    """Random-init stand-in survival scorer: W1 [hidden, width] bf16, b1 [width] fp32,
-    w2 [width] bf16, b2 scalar fp32."""
+    """Random-init stand-in survival scorer: W1 [width, hidden] bf16 (one row per
+    hidden unit, the Linear layout), b1 [width] fp32, w2 [width] bf16, b2 scalar fp32;
+    W1, b1 ~ U(+-1/sqrt(hidden)), w2, b2 ~ U(+-1/16)."""
     g = _gen(device, seed, 0xA11CE)
     a = 1.0 / math.sqrt(hidden)
-    W1 = ((torch.rand(hidden, width, generator=g, device=device) * 2 - 1) * a).to(torch.bfloat16)
+    W1 = ((torch.rand(width, hidden, generator=g, device=device) * 2 - 1) * a).to(torch.bfloat16)
     b1 = (torch.rand(width, generator=g, device=device) * 2 - 1) * a
     w2 = ((torch.rand(width, generator=g, device=device) * 2 - 1) / 16.0).to(torch.bfloat16)
     b2 = (torch.rand(1, generator=g, device=device) * 2 - 1) / 16.0
