@@ -156,7 +156,8 @@ SDD_API sdd_status_t sdd_schedule_prefix(const float *q, const float *logq, int 
 /*
  * sdd_verify_strict -- Strict SDD verification (Sec. 3.1: the standard rule of
  * speculative decoding) of the blocks listed in rows[0..n_rows) (all B blocks
- * when rows is NULL; then n_rows must be B).
+ * when rows is NULL; then n_rows must be B, or 0 for an empty list, which
+ * enqueues nothing).
  *   greedy != 0 (the paper's runs, Sec. 5.1): accept x_j iff it is the lowest-
  *     index argmax of target row j; the token after the accepted prefix is the
  *     target argmax of row L+1 (row gamma+1 when all gamma are accepted).

@@ -243,6 +243,7 @@ sdd_status_t set_topk(DecideParams &d, const int32_t *k, int n_k, int &kcap) {
 }
 
 sdd_status_t check_rows(const int32_t *rows, int n_rows, int B) {
+    if (n_rows == 0) return SDD_OK;   // nothing to verify: rows may be NULL
     if (rows == nullptr && n_rows != B)
         return fail(SDD_ERR_INVALID_ARGUMENT, "rows is NULL but n_rows = %d != B = %d", n_rows, B);
     if (n_rows < 0 || n_rows > B) return fail(SDD_ERR_INVALID_ARGUMENT, "n_rows = %d outside [0, B]", n_rows);

@@ -1,0 +1,62 @@
+"""The decode loop (raw-confidence policy driving strict verification of the
+blocks it does not skip, a survival-score policy in shadow, D carried across
+rounds, committed tokens) against an oracle replay of the same rounds:
+row statistics -> Eq. 3 schedule with D -> strict sampling on the blocks
+with K = 0 -> commit."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2608_14787_gb300 import synth
+from paper_2608_14787_gb300.loop import DecodeLoop
+
+pytestmark = pytest.mark.gpu
+NEAR = 1e-6
+
+
+def _bits(t):
+    return synth.bf16_bits(t)
+
+
+@pytest.mark.parametrize("B,gamma,V,hidden,rounds", [(6, 8, 3008, 128, 4), (3, 32, 20016, 256, 3)])
+def test_loop_matches_oracle_replay(sdd, orc, B, gamma, V, hidden, rounds):
+    wl = synth.WORKLOADS["c5"]
+    loop = DecodeLoop(B, gamma, V, tau=0.5, tau_mlp=0.3, K_min=2, S_max=6, seed=wl.seed, hidden=hidden)
+    W1, b1, w2 = _bits(loop.W1), loop.b1.cpu().numpy(), _bits(loop.w2)
+    D_raw = np.zeros(B, np.int32)
+    D_mlp = np.zeros(B, np.int32)
+    seen_skip = seen_verify = 0
+    for r in range(rounds):
+        blk = synth.make_block(wl, device="cuda", round_=r, B=B, gamma=gamma, V=V)
+        h = synth.make_hidden(B * gamma, device="cuda", seed=wl.seed, round_=r, hidden=hidden)
+        out = loop.step(blk.z_d, blk.z_t, blk.x, h, round_=r)
+        torch.cuda.synchronize()
+        assert int(loop.status.item()) == 0
+        zd, zt, x = _bits(blk.z_d), _bits(blk.z_t), blk.x.cpu().numpy()
+        # oracle replay of the round
+        st = orc.row_stats(zd, tokens=x)
+        _, K_raw, D_raw, mg_raw = orc.schedule(st.q, orc.SIG_RAW, 0.5, 0.5, 2, 6, D_in=D_raw)
+        s = orc.survival_mlp(_bits(h), W1, b1, w2, loop.b2).reshape(B, gamma)
+        _, K_mlp, D_mlp, mg_mlp = orc.schedule(s, orc.SIG_CONDITIONAL, 0.3, 0.3, 2, 6, D_in=D_mlp)
+        assert (mg_raw >= NEAR).all() and (mg_mlp >= NEAR).all(), "near-threshold row: pick another seed"
+        np.testing.assert_array_equal(out.K_raw.cpu().numpy(), K_raw)
+        np.testing.assert_array_equal(out.K_mlp.cpu().numpy(), K_mlp)
+        np.testing.assert_array_equal(loop.D_raw.cpu().numpy(), D_raw)
+        np.testing.assert_array_equal(loop.D_mlp.cpu().numpy(), D_mlp)
+        L_dev, tok_dev, n_dev = out.L.cpu().numpy(), out.tokens.cpu().numpy(), out.n.cpu().numpy()
+        assert out.n_verified == int((K_raw == 0).sum())
+        for b in range(B):
+            if K_raw[b] > 0:
+                seen_skip += 1
+                want = np.full(gamma + 1, -1, np.int32)
+                want[:K_raw[b]] = x[b, :K_raw[b]]
+                np.testing.assert_array_equal(tok_dev[b], want)
+                assert n_dev[b] == K_raw[b] and L_dev[b] == -2     # the verifier never saw this block
+            else:
+                seen_verify += 1
+                L, tokens, margin = orc.verify_strict(zt[b], zd[b], x[b], seed=wl.seed, b=b, round_=r)
+                assert margin >= NEAR, "near-threshold acceptance: pick another seed"
+                assert L_dev[b] == L
+                np.testing.assert_array_equal(tok_dev[b], tokens)
+                assert n_dev[b] == L + 1
+    assert seen_skip > 0 and seen_verify > 0     # both branches of the loop were exercised
