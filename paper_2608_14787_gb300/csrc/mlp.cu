@@ -17,6 +17,9 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <atomic>
+#include <mutex>
+
 #include "internal.h"
 
 namespace sdd {
@@ -26,7 +29,7 @@ constexpr int kMlpN = 256;           // hidden units = UMMA N
 constexpr int kMlpBM = 128;          // rows per CTA = UMMA M
 constexpr int kMlpBK = 64;           // K per stage: 64 bf16 = one 128-byte swizzle row
 constexpr int kMlpStages = 4;
-constexpr int kMlpThreads = 128;     // warp 0 lane 0: TMA producer; warp 1 lane 0: MMA issuer; all: epilogue
+constexpr int kMlpThreads = 256;     // warp 0 lane 0: TMA producer; warp 1 lane 0: MMA issuer; all: epilogue
 constexpr uint32_t kATileBytes = kMlpBM * kMlpBK * 2;   // 16 KiB
 constexpr uint32_t kBTileBytes = kMlpN * kMlpBK * 2;    // 32 KiB
 constexpr uint32_t kStageBytes = kATileBytes + kBTileBytes;
@@ -97,6 +100,39 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Address of the same shared-memory location in cluster CTA `rank`.
+__device__ __forceinline__ uint32_t map_rank(uint32_t addr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ void st_cluster_v4(uint32_t addr, float a, float b, float c, float d) {
+    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(a), "f"(b), "f"(c), "f"(d)
+                 : "memory");
+}
+
+// Row stride (floats) of a partial accumulator dumped to shared memory: a
+// multiple of 4 for 16-byte accesses, 4 mod 32 so that 8 consecutive rows
+// cover all banks.
+constexpr int kAccStride = kMlpN + 4;
+
+// Grid: (M tiles x S) CTAs in clusters of S along x (S = 1, 2 or 4 splits of
+// K).  CTA rank r of a cluster multiplies K slices [r nk/S, (r+1) nk/S) of its
+// 128-row tile into its own TMEM.  Rows [q R, (q+1) R) of the tile (R = 128/S)
+// are finished by CTA q: once every CTA of the cluster has finished its
+// mainloop (cluster barrier), every CTA pushes its partial of those rows into
+// slot r of CTA q's receive area (distributed shared-memory stores over the
+// idle stage ring); after a second cluster barrier each CTA sums its S slots
+// locally and runs the epilogue.
+template <int S>
 __global__ void __launch_bounds__(kMlpThreads, 1) mlp_kernel(const __grid_constant__ CUtensorMap tmA,
                                                             const __grid_constant__ CUtensorMap tmB,
                                                             const __grid_constant__ MlpParams p) {
@@ -108,9 +144,16 @@ __global__ void __launch_bounds__(kMlpThreads, 1) mlp_kernel(const __grid_consta
     uint64_t *done = empty + kMlpStages;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
     __shared__ int s_abort;
+    __shared__ float s_b1[kMlpN], s_w2[kMlpN];   // epilogue constants, widened once per CTA
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int m0 = blockIdx.x * kMlpBM;
-    const int nk = p.K / kMlpBK;
+    for (int n = tid; n < kMlpN; n += kMlpThreads) {
+        s_b1[n] = __ldg(p.b1 + n);
+        s_w2[n] = __uint_as_float(static_cast<uint32_t>(__ldg(p.w2 + n)) << 16);
+    }
+    const uint32_t rank = (S > 1) ? cluster_rank() : 0u;
+    const int m0 = (blockIdx.x / S) * kMlpBM;
+    const int nk = p.K / kMlpBK / S;           // K slices of this CTA
+    const int kt0 = static_cast<int>(rank) * nk;
 
     if (tid == 0) {
         for (int s = 0; s < kMlpStages; ++s) {
@@ -133,8 +176,8 @@ __global__ void __launch_bounds__(kMlpThreads, 1) mlp_kernel(const __grid_consta
     const uint32_t tmem = *tmem_slot;
 
     if (warp == 0 && lane == 0) {
-        // TMA producer: stage s holds K slice t of the A tile (rows m0..m0+127)
-        // and of the B tile (all 256 hidden units)
+        // TMA producer: stage s holds K slice kt0 + t of the A tile (rows
+        // m0..m0+127) and of the B tile (all 256 hidden units)
         int t = 0;
         for (; t < nk; ++t) {
             const int s = t % kMlpStages;
@@ -145,13 +188,13 @@ __global__ void __launch_bounds__(kMlpThreads, 1) mlp_kernel(const __grid_consta
             }
             mbar_arrive_expect_tx(&full[s], kStageBytes);
             const uint32_t a = smem_addr(smem + s * kStageBytes);
-            tma_load_2d(a, &tmA, t * kMlpBK, m0, smem_addr(&full[s]));
-            tma_load_2d(a + kATileBytes, &tmB, t * kMlpBK, 0, smem_addr(&full[s]));
+            tma_load_2d(a, &tmA, (kt0 + t) * kMlpBK, m0, smem_addr(&full[s]));
+            tma_load_2d(a + kATileBytes, &tmB, (kt0 + t) * kMlpBK, 0, smem_addr(&full[s]));
         }
-        // let every issued load land before the CTA can leave (already true
-        // unless a wait gave up): the last load into each stage
+        // let every issued load land before the ring is reused or the CTA
+        // leaves (already true unless a wait gave up): the last load per stage
         for (int s = 0; s < kMlpStages && s < t; ++s) {
-            const int last = ((t - 1 - s) / kMlpStages) * kMlpStages + s;   // last load issued into stage s
+            const int last = ((t - 1 - s) / kMlpStages) * kMlpStages + s;
             (void)mbar_wait_bounded(&full[s], static_cast<uint32_t>(last / kMlpStages) & 1u, kWaitPolls);
         }
     } else if (warp == 1 && lane == 0) {
@@ -175,30 +218,76 @@ __global__ void __launch_bounds__(kMlpThreads, 1) mlp_kernel(const __grid_consta
     }
     __syncwarp();
 
-    // epilogue: thread (warp w, lane l) owns row 32 w + l of the tile = TMEM lane 32 w + l
-    // warp-uniform, since tcgen05.ld below is a .sync.aligned warp instruction
+    // push the partial accumulator: warp w reads TMEM lanes 32 (w % 4) ..
+    // 32 (w % 4) + 31 (tile rows, all finished by CTA q = 32 (w % 4) / R), columns
+    // half w / 4
     const bool ok = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(done, 0u, kWaitPolls));
     tc_fence_after();
     if (!ok) s_abort = 1;
-    const int row = warp * 32 + lane;
-    float t2 = p.b2;
-    if (ok) {
-        const uint32_t tbase = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    constexpr int R = kMlpBM / S;
+    float *recv = reinterpret_cast<float *>(smem);   // [S slots][R rows][kAccStride], over the idle ring
+    if (S > 1) cluster_sync();   // every CTA's ring is idle before any partial is pushed into it
+    {
+        const int quarter = warp & 3, half = warp >> 2;
+        const int dest = (quarter * 32) / R;
+        const int drow = quarter * 32 - dest * R + lane;
+        const uint32_t local = smem_addr(recv + (static_cast<int>(rank) * R + drow) * kAccStride);
+        const uint32_t dst = (S > 1) ? map_rank(local, static_cast<uint32_t>(dest)) : local;
+        const uint32_t tbase = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
 #pragma unroll 1
-        for (int c = 0; c < kMlpN; c += 32) {
+        for (int c = half * (kMlpN / 2); c < (half + 1) * (kMlpN / 2); c += 32) {
             uint32_t v[32];
-            tmem_ld32(tbase + c, v);
+            if (ok) {
+                tmem_ld32(tbase + c, v);
+            } else {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                const float z = __uint_as_float(v[j]) + __ldg(p.b1 + c + j);
-                const float g = 0.5f * z * (1.f + erff(z * 0.70710678118654752f));
-                const float w = __uint_as_float(static_cast<uint32_t>(__ldg(p.w2 + c + j)) << 16);
-                t2 = fmaf(w, g, t2);
+                for (int j = 0; j < 32; ++j) v[j] = 0u;
             }
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                st_cluster_v4(dst + (c + 4 * j) * 4, __uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                              __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
         }
-        if (m0 + row < p.M) p.out[m0 + row] = 1.f / (1.f + expf(-t2));
     }
     tc_fence_before();
+    if (S > 1)
+        cluster_sync();   // every pushed partial has landed (release / acquire)
+    else
+        __syncthreads();
+
+    // epilogue: the R rows of this CTA, P = kMlpThreads / R threads per row;
+    // thread p of a row takes the 16-byte column chunks p, p + P, p + 2P, ...
+    // (the row's threads read consecutive chunks: no bank conflicts)
+    {
+        constexpr int P = kMlpThreads / R;
+        const int lrow = tid / P;
+        const int pp = tid % P;
+        float t2 = 0.f;
+#pragma unroll 4
+        for (int ch = pp; ch < kMlpN / 4; ch += P) {
+            const int c = 4 * ch;
+            float4 z = *reinterpret_cast<const float4 *>(recv + lrow * kAccStride + c);
+#pragma unroll
+            for (int q = 1; q < S; ++q) {
+                const float4 v = *reinterpret_cast<const float4 *>(recv + (q * R + lrow) * kAccStride + c);
+                z.x += v.x;
+                z.y += v.y;
+                z.z += v.z;
+                z.w += v.w;
+            }
+            const float zz[4] = {z.x, z.y, z.z, z.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int n = c + e;
+                const float u = zz[e] + s_b1[n];
+                const float g = 0.5f * u * (1.f + erff(u * 0.70710678118654752f));
+                t2 = fmaf(s_w2[n], g, t2);
+            }
+        }
+        for (int off = 1; off < P; off <<= 1) t2 += __shfl_xor_sync(0xFFFFFFFFu, t2, off);
+        const int grow = m0 + static_cast<int>(rank) * R + lrow;
+        if (tid % P == 0 && ok && grow < p.M) p.out[grow] = 1.f / (1.f + expf(-(t2 + p.b2)));
+    }
     __syncthreads();
     if (tid == 0 && s_abort) status_or(p.status, SDD_DEV_TIMEOUT);
     if (warp == 0)
@@ -231,6 +320,37 @@ bool make_map(CUtensorMap *map, const void *base, int64_t rows, int K, int box_r
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Encoded maps of recent (address, rows, K) operands: a decode loop passes the
+// same weights every round and often the same hidden-state buffer.
+struct MapCache {
+    struct Entry {
+        const void *base;
+        int64_t rows;
+        int K, box;
+        CUtensorMap map;
+    };
+    static constexpr int kSlots = 8;
+    Entry e[kSlots];
+    int n = 0, next = 0;
+    std::mutex mu;
+    bool get(CUtensorMap *out, const void *base, int64_t rows, int K, int box) {
+        std::lock_guard<std::mutex> g(mu);
+        for (int i = 0; i < n; ++i)
+            if (e[i].base == base && e[i].rows == rows && e[i].K == K && e[i].box == box) {
+                *out = e[i].map;
+                return true;
+            }
+        if (!make_map(out, base, rows, K, box)) return false;
+        e[next] = Entry{base, rows, K, box, *out};
+        next = (next + 1) % kSlots;
+        n = n < kSlots ? n + 1 : n;
+        return true;
+    }
+};
+MapCache g_maps;
+constexpr int kMaxDevices = 64;
+std::atomic<int> g_attr_ready[kMaxDevices];
+
 }  // namespace
 
 cudaError_t launch_mlp(const void *h, int M, int K, const void *W1, const float *b1, const void *w2, float b2,
@@ -238,13 +358,27 @@ cudaError_t launch_mlp(const void *h, int M, int K, const void *W1, const float 
     *why = nullptr;
     if (M == 0) return cudaSuccess;
     CUtensorMap tmA, tmB;
-    if (!make_map(&tmA, h, M, K, kMlpBM) || !make_map(&tmB, W1, kMlpN, K, kMlpN)) {
+    if (!g_maps.get(&tmA, h, M, K, kMlpBM) || !g_maps.get(&tmB, W1, kMlpN, K, kMlpN)) {
         *why = "cuTensorMapEncodeTiled failed";
         return cudaErrorInvalidValue;
     }
-    // per function and device; cheap, so set on every call
-    cudaError_t e = cudaFuncSetAttribute(mlp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMlpSmem);
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) {
+        *why = "device ordinal out of range";
+        return cudaErrorInvalidDevice;
+    }
+    if (!g_attr_ready[dev].load(std::memory_order_acquire)) {
+        for (auto fn : {mlp_kernel<1>, mlp_kernel<2>, mlp_kernel<4>}) {
+            e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kMlpSmem);
+            if (e != cudaSuccess) return e;
+        }
+        g_attr_ready[dev].store(1, std::memory_order_release);
+    }
+    // split K four ways when the slices divide evenly (more SMs, no reloads)
+    const int nk = K / kMlpBK;
+    const int S = (nk % 4 == 0 && nk >= 8) ? 4 : (nk % 2 == 0 && nk >= 4) ? 2 : 1;
     MlpParams p;
     p.M = M;
     p.K = K;
@@ -253,8 +387,21 @@ cudaError_t launch_mlp(const void *h, int M, int K, const void *W1, const float 
     p.b2 = b2;
     p.out = out;
     p.status = status;
-    mlp_kernel<<<(M + kMlpBM - 1) / kMlpBM, kMlpThreads, kMlpSmem, stream>>>(tmA, tmB, p);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(((M + kMlpBM - 1) / kMlpBM) * S);
+    cfg.blockDim = dim3(kMlpThreads);
+    cfg.dynamicSmemBytes = kMlpSmem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = S;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (S == 4) return cudaLaunchKernelEx(&cfg, mlp_kernel<4>, tmA, tmB, p);
+    if (S == 2) return cudaLaunchKernelEx(&cfg, mlp_kernel<2>, tmA, tmB, p);
+    return cudaLaunchKernelEx(&cfg, mlp_kernel<1>, tmA, tmB, p);
 }
 
 }  // namespace sdd
