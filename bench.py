@@ -15,6 +15,10 @@ reads its logits from HBM, not L2.
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--workload c3]
 Prints one JSON line (rank 0).
+
+Other rows of the path, one JSON line each (not the fused-round contract line):
+  python bench.py --component mlp [--steps K]   the survival scorer alone (K launches)
+  python bench.py --component loop [--steps R]  the decode-loop workload (R rounds, default 64)
 """
 from __future__ import annotations
 
@@ -346,6 +350,114 @@ def run_gpu(args):
     return 0
 
 
+def _peak_tflops():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except Exception:
+        return 1900.0, "fallback"
+
+
+def run_component_mlp(args):
+    """The stand-in survival scorer alone (decode-loop batch: 4096 positions,
+    hidden 3584 -> 256 -> 1), device time from CUDA-graph replays of 16 launches
+    over 8 rotating hidden-state buffers (8 x 29 MB > L2)."""
+    import torch
+    import paper_2608_14787_gb300 as sdd
+    from paper_2608_14787_gb300 import build as sdd_build
+    from paper_2608_14787_gb300 import synth
+    sdd_build.build()
+    sdd.load()
+    M, K, N = 128 * 32, synth.HIDDEN, 256
+    W1, b1, w2, b2 = synth.make_mlp(device="cuda", hidden=K)
+    b2 = float(b2.item())
+    hs = [synth.make_hidden(M, device="cuda", round_=r) for r in range(8)]
+    out = torch.empty(M, device="cuda")
+    status = sdd.new_status(torch.device("cuda"))
+    for i in range(max(args.warmup, 3)):
+        sdd.survival_mlp(hs[i % 8], W1, b1, w2, b2, out=out, status=status)
+    torch.cuda.synchronize()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=side):
+        for i in range(16):
+            sdd.survival_mlp(hs[i % 8], W1, b1, w2, b2, out=out, status=status)
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    reps = max(1, args.steps // 16)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(None) as clk:
+        e0.record()
+        for _ in range(reps):
+            g.replay()
+        e1.record()
+        torch.cuda.synchronize()
+    t = e0.elapsed_time(e1) / (reps * 16) / 1e3
+    flops = 2.0 * M * K * N
+    nbytes = M * K * 2 + N * K * 2 + M * 4
+    tpk, tkind = _peak_tflops()
+    hbm, hkind = _peaks()
+    cpu = None
+    if not args.no_cpu_baseline:
+        import numpy as np
+        import oracle as orc
+        rows = 512
+        t0 = time.perf_counter()
+        orc.survival_mlp(synth.bf16_bits(hs[0][:rows]), synth.bf16_bits(W1), b1.cpu().numpy(), synth.bf16_bits(w2), b2)
+        dt = time.perf_counter() - t0
+        cpu = {"value": rows / dt, "unit": "positions/s", "cores": 1, "kind": "oracle",
+               "sample": f"{rows} of the {M} positions, fp64 loops, single thread ({dt:.1f} s)"}
+        del np
+    line = {
+        "component": "a8 survival scorer (sdd_survival_mlp)", "metric": "positions scored/s", "unit": "positions/s",
+        "value": M / t, "us_per_call": t * 1e6, "config": {"M": M, "K": K, "N": N, "dtype": "bf16 in, fp32 acc"},
+        "roofline": {"bound": "hbm", "achieved_gbs": nbytes / t / 1e9, "peak_gbs": hbm, "frac_hbm": nbytes / t / 1e9 / hbm,
+                     "achieved_tflops": flops / t / 1e12, "peak_tflops": tpk,
+                     "frac_tensor": flops / t / 1e12 / tpk, "bytes": nbytes, "flops": flops,
+                     "peak_source": f"{hkind} hbm_gbs / {tkind} bf16_tflops",
+                     "note": "intensity 242 FLOP/B is below the ridge: bytes bound"},
+        "cpu_baseline": cpu, "clocks": clk.summary(), "device_status": int(status.item()),
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_component_loop(args):
+    """The decode-loop workload (B=128, gamma=32, V=151,936 bf16): `--steps`
+    rounds (default 64) of fresh logits and hidden states, generated untimed."""
+    import torch
+    from paper_2608_14787_gb300 import build as sdd_build
+    from paper_2608_14787_gb300 import loop as sdd_loop
+    from paper_2608_14787_gb300 import synth
+    sdd_build.build()
+    rounds = args.steps if args.steps != 4000 else 64
+    with ClockSampler(None) as clk:
+        res = sdd_loop.run(rounds, "c5", warmup=max(2, min(args.warmup, 4)))
+    cpu = None
+    if not args.no_cpu_baseline:
+        import numpy as np
+        import oracle as orc
+        wl = synth.WORKLOADS["c5"]
+        blk = synth.make_block(wl, device="cuda", round_=0, B=1)
+        zd, zt, x = synth.bf16_bits(blk.z_d[0]), synth.bf16_bits(blk.z_t[0]), blk.x[0].cpu().numpy()
+        t0 = time.perf_counter()
+        st = orc.row_stats(zd, tokens=x)
+        orc.schedule(st.q[None], orc.SIG_RAW, 0.9, 0.9, 6, 64)
+        orc.verify_strict(zt, zd, x, seed=wl.seed, b=0, round_=0)
+        dt = time.perf_counter() - t0
+        cpu = {"value": 1.0 / dt, "unit": "blocks/s", "cores": 1, "kind": "oracle",
+               "sample": f"one block of one round (confidence, schedule, strict verification), single thread "
+                         f"({dt:.1f} s)"}
+        del np
+    res.update({"component": "decode loop (c5)", "metric": "blocks/s", "unit": "blocks/s",
+                "value": res["blocks_per_s"], "cpu_baseline": cpu, "clocks": clk.summary()})
+    torch.cuda.synchronize()
+    print(json.dumps(res), flush=True)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -359,7 +471,13 @@ def main():
     ap.add_argument("--sets", type=int, default=3, help="rotating input sets (3 x 316 MB exceeds L2)")
     ap.add_argument("--traffic", type=float, default=None,
                     help="dram bytes per scan launch from an ncu capture of the current kernel")
+    ap.add_argument("--component", default=None, choices=["mlp", "loop"],
+                    help="measure one other row of the path instead of the fused round")
     args = ap.parse_args()
+    if args.component == "mlp":
+        return run_component_mlp(args)
+    if args.component == "loop":
+        return run_component_loop(args)
     if args.traffic is None and args.workload == "c3":
         args.traffic = SCAN_TRAFFIC_C3
     if args.warmup < 3:
