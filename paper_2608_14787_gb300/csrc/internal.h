@@ -21,6 +21,29 @@ constexpr int kStages = 3;
 constexpr int kScanSmem = kWarpsPerCta * kStages * kTileBytes + kWarpsPerCta * kStages * 8;
 constexpr uint32_t kWaitPolls = 1u << 24;     // bounded mbarrier wait (seconds of polling)
 
+// Division by a per-launch constant d >= 1 without the 64-bit integer division
+// routine (a called subroutine, slow on this part): floor(n / d) =
+// umulhi(n, M) >> s with s = floor(log2 d) and M = ceil(2^(64+s) / d), exact for
+// every 0 <= n < 2^53 (M d - 2^(64+s) < d <= 2^(s+1) <= 2^(64+s-53)); a power
+// of two is a plain shift.  Built on the host (make_fastdiv).
+struct FastDiv {
+    uint64_t M;
+    uint32_t s;
+    uint32_t pow2;   // d = 2^s
+};
+
+inline FastDiv make_fastdiv(uint64_t d) {
+    FastDiv f{0, 0, 0};
+    while ((static_cast<uint64_t>(2) << f.s) <= d && f.s < 63) ++f.s;   // s = floor(log2 d)
+    if ((d & (d - 1)) == 0) {
+        f.pow2 = 1;
+        return f;
+    }
+    const unsigned __int128 num = static_cast<unsigned __int128>(1) << (64 + f.s);
+    f.M = static_cast<uint64_t>((num + d - 1) / d);
+    return f;
+}
+
 // Decide kernel geometry: one CTA of kDecThreads per (listed block, draw
 // segment); each draw segment is a run of whole 256-vector chunks of the draw
 // row, at most kDrawMaxSeg per block.
@@ -96,6 +119,7 @@ struct ScanParams {
     int64_t rows0;           // rows of group 0
     int64_t rows;            // rows of all groups
     int64_t T;               // total vectors = rows * RV
+    FastDiv divT, divW, divRV, divNpos[2];   // division by T, W, RV, grp[g].npos
     const int32_t *tokens;   // [B, gamma]
     Partial *partials;       // [rows + W]
     int32_t *status;
@@ -125,6 +149,15 @@ cudaError_t launch_commit(const int32_t *K, const int32_t *x, const int32_t *vt,
                           int gamma, int32_t *out_t, int32_t *out_n, cudaStream_t stream);
 cudaError_t launch_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, const uint64_t *round,
                             const uint32_t *purpose, int64_t n, float *u, cudaStream_t stream);
+// The division constants of a launch whose rows, T and W are set (host).
+// The magic divisions are exact while T * W < 2^53 (run_scan checks it).
+inline void set_divisors(ScanParams &p) {
+    p.divT = make_fastdiv(static_cast<uint64_t>(p.T > 0 ? p.T : 1));
+    p.divW = make_fastdiv(static_cast<uint64_t>(p.W > 0 ? p.W : 1));
+    p.divRV = make_fastdiv(static_cast<uint64_t>(p.RV > 0 ? p.RV : 1));
+    for (int g = 0; g < 2; ++g) p.divNpos[g] = make_fastdiv(static_cast<uint64_t>(p.grp[g].npos > 0 ? p.grp[g].npos : 1));
+}
+
 // The stand-in survival scorer (mlp.cu); *why names a host-side failure.
 cudaError_t launch_mlp(const void *h, int M, int K, const void *W1, const float *b1, const void *w2, float b2,
                        float *out, int32_t *status, cudaStream_t stream, const char **why);
@@ -133,10 +166,18 @@ int decide_max_ctas_per_sm();
 cudaError_t scan_prepare_device();
 void set_last_error(const char *msg);  // message returned by sdd_last_error()
 
+__device__ __forceinline__ int64_t fast_div(int64_t n, const FastDiv &f) {
+    const uint64_t u = static_cast<uint64_t>(n);
+    return static_cast<int64_t>(f.pow2 ? (u >> f.s) : (__umul64hi(u, f.M) >> f.s));
+}
+
 // Index arithmetic of the balanced contiguous partition of T vectors over W
 // warps: warp w owns [start(w), start(w+1)), start(w) = floor(w T / W).
-__host__ __device__ inline int64_t part_start(int64_t w, int64_t T, int64_t W) { return (w * T) / W; }
+// Requires T W < 2^53 (checked by the host).
+__device__ __forceinline__ int64_t part_start(int64_t w, int64_t T, const FastDiv &divW) { return fast_div(w * T, divW); }
 // The warp owning vector v (requires W <= T, so every warp is non-empty).
-__host__ __device__ inline int64_t part_owner(int64_t v, int64_t T, int64_t W) { return ((v + 1) * W - 1) / T; }
+__device__ __forceinline__ int64_t part_owner(int64_t v, int64_t W, const FastDiv &divT) {
+    return fast_div((v + 1) * W - 1, divT);
+}
 
 }  // namespace sdd

@@ -140,6 +140,7 @@ sdd_status_t sdd_confidence_noalloc(const void *draft_logits, sdd_dtype_t dtype,
     p.T = rows * p.RV;
     const int64_t W = std::min<int64_t>(nd.W_max, p.T);
     p.W = static_cast<int32_t>(W);
+    set_divisors(p);
 
     cudaError_t e = launch_scan(p, static_cast<int>((W + kWarpsPerCta - 1) / kWarpsPerCta), st);
     if (e != cudaSuccess) return na_fail(SDD_ERR_CUDA, "scan launch: %s", cudaGetErrorString(e));

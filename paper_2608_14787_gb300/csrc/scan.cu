@@ -36,7 +36,7 @@ __device__ __forceinline__ void row_locate(const ScanParams &p, int64_t r, int &
     gi = (r >= p.rows0) ? 1 : 0;
     lr = gi ? r - p.rows0 : r;
     const ScanGroup &G = p.grp[gi];
-    const int64_t i = lr / G.npos;
+    const int64_t i = fast_div(lr, p.divNpos[gi]);
     j = static_cast<int>(lr - i * G.npos);
     b = G.bidx ? __ldg(G.bidx + i) : static_cast<int>(i);
     b_ok = (b >= 0 && b < p.B);
@@ -288,11 +288,12 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
     }
     __syncwarp();
 
-    const int64_t v0 = part_start(gw, p.T, p.W), v1 = part_start(gw + 1, p.T, p.W);
-    Cursor pc{v0, v0 / p.RV, 0};
+    const int64_t v0 = part_start(gw, p.T, p.divW), v1 = part_start(gw + 1, p.T, p.divW);
+    Cursor pc{v0, fast_div(v0, p.divRV), 0};
     pc.k = static_cast<int32_t>(v0 - pc.r * p.RV);
     Cursor cc = pc;
     const char *prow = row_base(p, pc.r);
+    const uint64_t pol = l2_evict_first_policy();   // the logits are read once
     uint32_t pending = 0;  // slots with a copy in flight
     uint32_t phase = 0;    // parity bit per slot
 
@@ -303,7 +304,7 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
             // warp reached this point (__syncwarp), so the copy may overwrite it
             mbar_arrive_expect_tx(&bars[slot], static_cast<uint32_t>(n) * 16u);
             bulk_g2s(ring + slot * kTileBytes, prow + static_cast<int64_t>(pc.k) * 16, static_cast<uint32_t>(n) * 16u,
-                     &bars[slot]);
+                     &bars[slot], pol);
         }
         pending |= 1u << slot;
         pc.v += n;
