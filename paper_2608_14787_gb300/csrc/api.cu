@@ -67,7 +67,7 @@ inline size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255);
 
 // Workspace layout for blocks of shape (B, gamma) on a device with W_max warps.
 struct Layout {
-    size_t partials, res_total, res_pref, res_last, res_count, total;
+    size_t partials, res_total, res_pref, res_count, total;
 };
 
 Layout layout(int64_t B, int64_t gamma, int64_t W_max, int64_t dec_ctas) {
@@ -83,7 +83,6 @@ Layout layout(int64_t B, int64_t gamma, int64_t W_max, int64_t dec_ctas) {
     L.res_total = take(static_cast<size_t>(B * kDrawMaxSeg) * sizeof(float));
     // nb * nseg <= max(resident decide CTAs, B) (see init_dec)
     L.res_pref = take(static_cast<size_t>(std::max(dec_ctas, B)) * kDecThreads * sizeof(float));
-    L.res_last = take(static_cast<size_t>(B * kDrawMaxSeg) * sizeof(int32_t));
     L.res_count = take(static_cast<size_t>(B) * sizeof(uint32_t));
     L.total = o;
     return L;
@@ -192,7 +191,6 @@ void init_dec(DecideParams &d, const Work &w, sdd_dtype_t dtype, int B, int gamm
     d.tokens = tokens;
     d.res_total = reinterpret_cast<float *>(w.base + w.L.res_total);
     d.res_pref = reinterpret_cast<float *>(w.base + w.L.res_pref);
-    d.res_last = reinterpret_cast<int32_t *>(w.base + w.L.res_last);
     d.res_count = reinterpret_cast<uint32_t *>(w.base + w.L.res_count);
     const int RV = static_cast<int>((static_cast<int64_t>(V) * esize(dtype) + 15) / 16);
     const int want = std::max(1, std::min(kDrawMaxSeg, w.dec_ctas / std::max(nb, 1)));

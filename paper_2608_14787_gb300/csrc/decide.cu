@@ -30,6 +30,7 @@ namespace {
 struct DrawCtx {
     const char *zt_row, *zd_row;
     float nrt, nrd, d_hi, d_lo;
+    f2_t nrt2, nrd2, d_hi2, d_lo2;   // the same constants in both halves of a pair
 };
 
 __device__ __forceinline__ DrawCtx draw_ctx(const char *zt_row, const char *zd_row, df lse_t, df lse_d) {
@@ -46,6 +47,10 @@ __device__ __forceinline__ DrawCtx draw_ctx(const char *zt_row, const char *zd_r
         c.d_hi = D.hi;
         c.d_lo = D.lo;
     }
+    c.nrt2 = f2_pack(c.nrt, c.nrt);
+    c.nrd2 = f2_pack(c.nrd, c.nrd);
+    c.d_hi2 = f2_pack(c.d_hi, c.d_hi);
+    c.d_lo2 = f2_pack(c.d_lo, c.d_lo);
     return c;
 }
 
@@ -88,26 +93,88 @@ __device__ __forceinline__ float entry_weight(const DrawCtx &c, float zt, float 
     return (v < V) ? w : 0.f;
 }
 
-// Entry e of a 16-byte vector of logits, widened to fp32.
-template <int DT>
-__device__ __forceinline__ float vec_entry(const uint4 &a, int e) {
-    const uint32_t *u = reinterpret_cast<const uint32_t *>(&a);
-    if (DT == SDD_BF16) return (e & 1) ? bf16_hi(u[e >> 1]) : bf16_lo(u[e >> 1]);
-    return __uint_as_float(u[e]);
+__device__ __forceinline__ f2_t f2_splat(float v) { return f2_pack(v, v); }
+
+// expm1_pos on both halves of a pair, without branches: the same Taylor
+// polynomial and the same 2^(x log2 e) - 1, each rounded as the scalar form
+// rounds it, the half's range picking the result.
+__device__ __forceinline__ f2_t expm1_pos2(f2_t x) {
+    f2_t p = f2_splat(1.f / 5040.f);
+    p = f2_fma(p, x, f2_splat(1.f / 720.f));
+    p = f2_fma(p, x, f2_splat(1.f / 120.f));
+    p = f2_fma(p, x, f2_splat(1.f / 24.f));
+    p = f2_fma(p, x, f2_splat(1.f / 6.f));
+    p = f2_fma(p, x, f2_splat(0.5f));
+    p = f2_fma(p, x, f2_splat(1.f));
+    p = f2_mul(p, x);
+    float y0, y1, x0, x1, p0, p1;
+    f2_unpack(f2_mul(x, f2_splat(kLog2e)), y0, y1);
+    f2_unpack(x, x0, x1);
+    f2_unpack(p, p0, p1);
+    const f2_t e = f2_sub(f2_pack(ex2(y0), ex2(y1)), f2_splat(1.f));
+    float e0, e1;
+    f2_unpack(e, e0, e1);
+    return f2_pack(x0 < 0.35f ? p0 : e0, x1 < 0.35f ? p1 : e1);
 }
 
-// Weights of the draw for the EPV entries of one 16-byte vector; returns
-// their fp32 sum in ascending order.
-template <int DT>
-__device__ __forceinline__ float vec_weights(const DrawCtx &c, uint4 a, uint4 d, int vec, int V, float (&w)[8]) {
-    constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
-    float sum = 0.f;
-#pragma unroll
-    for (int e = 0; e < EPV; ++e) {
-        w[e] = entry_weight(c, vec_entry<DT>(a, e), vec_entry<DT>(d, e), vec * EPV + e, V);
-        sum += w[e];
+// entry_weight of two entries at once (both below V), through the packed
+// f32x2 pipe: every half is rounded exactly as the scalar form rounds it, so
+// both give the same weights bit for bit.  zt0..zd1 are clamped logits.
+__device__ __forceinline__ void pair_weights(const DrawCtx &c, float zt0, float zt1, float zd0, float zd1, float &w0,
+                                             float &w1) {
+    if (c.zd_row) {
+        const f2_t zd = f2_pack(zd0, zd1);
+        const f2_t dv = f2_sub(f2_sub(f2_sub(f2_pack(zt0, zt1), zd), c.d_hi2), c.d_lo2);
+        float a0, a1, q0, q1, d0, d1;
+        f2_unpack(f2_fma(zd, f2_splat(kLog2e), c.nrd2), a0, a1);
+        f2_unpack(f2_mul(f2_pack(ex2(a0), ex2(a1)), expm1_pos2(dv)), q0, q1);
+        f2_unpack(dv, d0, d1);
+        w0 = (d0 > 0.f) ? q0 : 0.f;
+        w1 = (d1 > 0.f) ? q1 : 0.f;
+    } else {
+        float a0, a1;
+        f2_unpack(f2_fma(f2_pack(zt0, zt1), f2_splat(kLog2e), c.nrt2), a0, a1);
+        w0 = ex2(a0);
+        w1 = ex2(a1);
     }
-    return sum;
+}
+
+// Entry e of a 16-byte vector of logits, widened to fp32.
+// (Word picked by selects: a run-time e never indexes a local array.)
+template <int DT>
+__device__ __forceinline__ float vec_entry(const uint4 &a, int e) {
+    const int k = (DT == SDD_BF16) ? (e >> 1) : e;
+    const uint32_t u = (k < 2) ? ((k == 0) ? a.x : a.y) : ((k == 2) ? a.z : a.w);
+    if (DT == SDD_BF16) return (e & 1) ? bf16_hi(u) : bf16_lo(u);
+    return __uint_as_float(u);
+}
+
+// Weights of the draw for the EPV entries of one 16-byte vector (the values
+// of entry_weight; entries past V weigh 0).
+template <int DT>
+__device__ __forceinline__ void vec_weights(const DrawCtx &c, uint4 a, uint4 d, int vec, int V, float (&w)[8]) {
+    constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
+    const uint32_t *au = reinterpret_cast<const uint32_t *>(&a);
+    const uint32_t *du = reinterpret_cast<const uint32_t *>(&d);
+    if (DT == SDD_BF16) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const uint32_t t2 = bf16x2_max_nan(au[k], kClampPairBf16), d2 = bf16x2_max_nan(du[k], kClampPairBf16);
+            pair_weights(c, bf16_lo(t2), bf16_hi(t2), bf16_lo(d2), bf16_hi(d2), w[2 * k], w[2 * k + 1]);
+        }
+    } else {
+#pragma unroll
+        for (int k = 0; k < 2; ++k)
+            pair_weights(c, fmax_nan(__uint_as_float(au[2 * k]), clamp_floor()),
+                         fmax_nan(__uint_as_float(au[2 * k + 1]), clamp_floor()),
+                         fmax_nan(__uint_as_float(du[2 * k]), clamp_floor()),
+                         fmax_nan(__uint_as_float(du[2 * k + 1]), clamp_floor()), w[2 * k], w[2 * k + 1]);
+    }
+    if (static_cast<int64_t>(vec + 1) * EPV > V) {
+#pragma unroll
+        for (int e = 0; e < EPV; ++e)
+            if (vec * EPV + e >= V) w[e] = 0.f;
+    }
 }
 
 // The first entry of vectors [vb, ve) at which the running weight sum exceeds
@@ -175,7 +242,7 @@ __device__ __forceinline__ float cta_incl_scan(float v, float *warp_tot, float *
 
 // Sum (fp32, ascending order) of the draw weights of vectors [vb, ve).
 template <int DT>
-__device__ __forceinline__ float run_sum(const DrawCtx &c, int vb, int ve, int V, int &last_pos) {
+__device__ __forceinline__ float run_sum(const DrawCtx &c, int vb, int ve, int V) {
     constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
     float sum = 0.f;
     for (int v = vb; v < ve; v += 4) {
@@ -196,10 +263,7 @@ __device__ __forceinline__ float run_sum(const DrawCtx &c, int vb, int ve, int V
                 float w[8];
                 vec_weights<DT>(c, a[k], d[k], vec, V, w);
 #pragma unroll
-                for (int e = 0; e < EPV; ++e) {
-                    sum += w[e];
-                    if (w[e] > 0.f) last_pos = vec * EPV + e;
-                }
+                for (int e = 0; e < EPV; ++e) sum += w[e];
             }
         }
     }
@@ -237,8 +301,7 @@ template <int DT>
 __device__ int cta_find(const DrawCtx &c, int v0, int v1, int vpt, int V, df rem, float *s_warp, int *s_thr,
                         int *s_tok) {
     const int vb = min(v1, v0 + static_cast<int>(threadIdx.x) * vpt), ve = min(v1, vb + vpt);
-    int lastp = -1;
-    const float ts = run_sum<DT>(c, vb, ve, V, lastp);
+    const float ts = run_sum<DT>(c, vb, ve, V);
     float tot;
     const float incl = cta_incl_scan(ts, s_warp, &tot);
     if (threadIdx.x == 0) *s_thr = INT32_MAX;
@@ -372,17 +435,21 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                 s_L[0] = L;
                 s_corr[0] = F.t_am[L];
             }
+        } else if (warp == 1 && sched) {
+            // pair 0 decides whether this block commits its verified tokens
+            int Kh, K, Do;
+            sched_pair(d, F, 0, s_force != 0, s_D, lane, Kh, K, Do);
+            if (lane == 0) s_K0 = K;
         }
         __shared__ float s_warp[2 * NW];
         __shared__ float s_pref[kDecThreads];
-        __shared__ int s_is_last, s_seg, s_lastp, s_thr, s_tok;
+        __shared__ int s_is_last, s_seg, s_thr, s_thr_last, s_tok;
         __shared__ df s_rem;
         __shared__ float s_tot[kDrawMaxSeg];
         __shared__ df s_cum[kDrawMaxSeg];
-        __shared__ int s_last[kDrawMaxSeg];
         if (tid == 0) {
-            s_lastp = -1;
             s_thr = INT32_MAX;
+            s_thr_last = -1;
         }
         __syncthreads();
 
@@ -398,19 +465,12 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
         {
             const int v0 = seg * d.seg_vec, v1 = min(p.RV, v0 + d.seg_vec);
             const int vb = min(v1, v0 + tid * vpt), ve = min(v1, vb + vpt);
-            int last_pos = -1;
-            const float ts = run_sum<DT>(c, vb, ve, p.V, last_pos);
             float tot;
-            const float incl = cta_incl_scan(ts, s_warp, &tot);
+            const float incl = cta_incl_scan(run_sum<DT>(c, vb, ve, p.V), s_warp, &tot);
             d.res_pref[pair * kDecThreads + tid] = incl;   // this thread's inclusive prefix in the segment
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1)
-                last_pos = max(last_pos, __shfl_xor_sync(0xFFFFFFFFu, last_pos, off));
-            if (lane == 0) atomicMax(&s_lastp, last_pos);
             __syncthreads();
             if (tid == 0) {
                 d.res_total[pair] = tot;
-                d.res_last[pair] = s_lastp;
                 // the barrier above orders every thread's prefix store before
                 // this fence, which orders them all before the arrival
                 __threadfence();
@@ -422,35 +482,32 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
         if (s_is_last) {
             // the last segment to arrive completes the draw
             __threadfence();
-            for (int sg = tid; sg < d.nseg; sg += kDecThreads) {
+            for (int sg = tid; sg < d.nseg; sg += kDecThreads)
                 s_tot[sg] = __ldcg(d.res_total + static_cast<int64_t>(i) * d.nseg + sg);
-                s_last[sg] = __ldcg(d.res_last + static_cast<int64_t>(i) * d.nseg + sg);
-            }
             __syncthreads();
             if (warp == 0) {
                 // R = sum of the segment totals and their inclusive prefix sums
                 // (double-floats); the first segment whose prefix exceeds u * R
                 df carry = df{0.f, 0.f};
-                int lastp = -1;
+                int last_seg = -1;   // the last segment of positive mass
                 for (int s0 = 0; s0 < d.nseg; s0 += 32) {
                     const int sg = s0 + lane;
                     const float t = (sg < d.nseg) ? s_tot[sg] : 0.f;
                     const df cum = df_add(carry, warp_prefix_df(df{t, 0.f}, lane));
-                    if (sg < d.nseg) {
-                        s_cum[sg] = cum;
-                        lastp = max(lastp, s_last[sg]);
-                    }
+                    if (sg < d.nseg) s_cum[sg] = cum;
+                    if (t > 0.f) last_seg = sg;
                     carry.hi = __shfl_sync(0xFFFFFFFFu, cum.hi, 31);
                     carry.lo = __shfl_sync(0xFFFFFFFFu, cum.lo, 31);
                 }
 #pragma unroll
-                for (int off = 16; off > 0; off >>= 1) lastp = max(lastp, __shfl_xor_sync(0xFFFFFFFFu, lastp, off));
+                for (int off = 16; off > 0; off >>= 1)
+                    last_seg = max(last_seg, __shfl_xor_sync(0xFFFFFFFFu, last_seg, off));
                 const df Rm = carry;
                 const uint32_t jj = (L < gamma) ? static_cast<uint32_t>(L + 1) : static_cast<uint32_t>(gamma + 1);
                 const float u = philox_uniform(d.seed, jj, static_cast<uint32_t>(b), d.round,
                                                (L < gamma) ? kPurposeResid : kPurposeBonus);
                 const df target = df_mul_f(Rm, u);
-                int sel = (Rm.hi > 0.f) ? -2 : -3;   // -2: rounding left none (last positive), -3: no mass
+                int sel = -1;
                 if (Rm.hi > 0.f) {
                     __syncwarp();
                     for (int s0 = 0; s0 < d.nseg; s0 += 32) {
@@ -464,17 +521,17 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                     }
                 }
                 if (lane == 0) {
-                    s_seg = sel;
-                    s_rem = (sel > 0) ? df_sub(target, s_cum[sel - 1]) : target;   // u R minus the mass before sel
-                    s_lastp = lastp;
+                    if (sel >= 0) {
+                        s_seg = sel;
+                        s_rem = (sel > 0) ? df_sub(target, s_cum[sel - 1]) : target;   // u R minus the mass before sel
+                    } else {
+                        // rounding left no segment (-> the row's last positive
+                        // entry: an infinite remainder), or there is no mass (-1)
+                        s_seg = (Rm.hi > 0.f) ? last_seg : -1;
+                        s_rem = df{__int_as_float(0x7F800000), 0.f};
+                    }
                     d.res_count[i] = 0u;   // leave the workspace zeroed
                 }
-            }
-            if (warp == 1 && sched) {
-                // pair 0 decides whether this block commits its verified tokens
-                int Kh, K, Do;
-                sched_pair(d, F, 0, s_force != 0, s_D, lane, Kh, K, Do);
-                if (lane == 0) s_K0 = K;
             }
             __syncthreads();
             int tok;
@@ -488,22 +545,31 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                 const unsigned bal = __ballot_sync(0xFFFFFFFFu, !df_ge(rem, df{pv, 0.f}));
                 if (lane == 0 && bal) atomicMin(&s_thr, warp * 32 + __ffs(bal) - 1);
                 __syncthreads();
-                const int thr = s_thr;
+                int thr = s_thr;
+                df rem2 = rem;
                 if (thr == INT32_MAX) {
-                    tok = s_last[sel];   // rounding: the segment's last positive entry
-                } else {
-                    if (warp == 0) {
-                        const df rem2 = (thr > 0) ? df_sub(rem, df{s_pref[thr - 1], 0.f}) : rem;
+                    // rounding left no thread: the last thread whose run has
+                    // positive weight (its prefix rose), searched to its end
+                    const bool rose = pv > ((tid > 0) ? s_pref[tid - 1] : 0.f);
+                    const unsigned up = __ballot_sync(0xFFFFFFFFu, rose);
+                    if (lane == 0 && up) atomicMax(&s_thr_last, warp * 32 + 31 - __clz(up));
+                    __syncthreads();
+                    thr = s_thr_last;
+                    rem2 = df{__int_as_float(0x7F800000), 0.f};
+                } else if (thr > 0) {
+                    rem2 = df_sub(rem, df{s_pref[thr - 1], 0.f});
+                }
+                if (warp == 0) {
+                    int pick = -1;
+                    if (thr >= 0) {
                         const int sv0 = sel * d.seg_vec, sv1 = min(p.RV, sv0 + d.seg_vec);
                         const int vb = min(sv1, sv0 + thr * vpt), ve = min(sv1, vb + vpt);
-                        const int pick = warp_search<DT>(c, vb, ve, p.V, rem2, lane);
-                        if (lane == 0) s_tok = (pick >= 0) ? pick : s_last[sel];
+                        pick = warp_search<DT>(c, vb, ve, p.V, rem2, lane);
                     }
-                    __syncthreads();
-                    tok = s_tok;
+                    if (lane == 0) s_tok = pick;
                 }
-            } else if (sel == -2) {
-                tok = s_lastp;
+                __syncthreads();
+                tok = s_tok;
             } else {
                 // the residual has no mass (only through rounding): draw from p_t
                 // of the same row, whole row in this CTA, same inverse-CDF rule
@@ -511,9 +577,8 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                 ct.zd_row = nullptr;
                 const int vrow = (p.RV + kDecThreads - 1) / kDecThreads;
                 const int vb = min(p.RV, tid * vrow), ve = min(p.RV, vb + vrow);
-                int lp = -1;
                 float tot;
-                (void)cta_incl_scan(run_sum<DT>(ct, vb, ve, p.V, lp), s_warp, &tot);
+                (void)cta_incl_scan(run_sum<DT>(ct, vb, ve, p.V), s_warp, &tot);
                 const float u = philox_uniform(d.seed, static_cast<uint32_t>(L + 1), static_cast<uint32_t>(b),
                                                d.round, kPurposeResid);
                 tok = (tot > 0.f)

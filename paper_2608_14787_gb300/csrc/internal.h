@@ -86,7 +86,6 @@ struct DecideParams {
     int32_t nseg, seg_vec;         // segments per block and vectors per segment
     float *res_total;              // [nb, nseg]
     float *res_pref;               // [nb, nseg, kDecThreads] per-thread inclusive prefix sums
-    int32_t *res_last;             // [nb, nseg]
     uint32_t *res_count;           // [nb] (zero between calls)
 };
 
