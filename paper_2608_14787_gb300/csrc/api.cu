@@ -51,6 +51,7 @@ sdd_status_t device_info(DevInfo &out) {
         e = cudaDeviceGetAttribute(&di.sms, cudaDevAttrMultiProcessorCount, d);
         if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
         e = scan_prepare_device();
+        if (e == cudaSuccess) e = decide_prepare_device();
         if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
         di.ctas_per_sm = scan_max_ctas_per_sm();
         if (di.ctas_per_sm < 1) return fail(SDD_ERR_UNSUPPORTED, "streaming kernel does not fit on this device");
@@ -67,7 +68,7 @@ inline size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255);
 
 // Workspace layout for blocks of shape (B, gamma) on a device with W_max warps.
 struct Layout {
-    size_t partials, res_total, res_pref, res_count, total;
+    size_t partials, res_pref, res_count, total;
 };
 
 Layout layout(int64_t B, int64_t gamma, int64_t W_max, int64_t dec_ctas) {
@@ -80,7 +81,6 @@ Layout layout(int64_t B, int64_t gamma, int64_t W_max, int64_t dec_ctas) {
         return at;
     };
     L.partials = take(static_cast<size_t>(rows + W_max) * sizeof(Partial));
-    L.res_total = take(static_cast<size_t>(B * kDrawMaxSeg) * sizeof(float));
     // nb * nseg <= max(resident decide CTAs, B) (see init_dec)
     L.res_pref = take(static_cast<size_t>(std::max(dec_ctas, B)) * kDecThreads * sizeof(float));
     L.res_count = take(static_cast<size_t>(B) * sizeof(uint32_t));
@@ -189,7 +189,6 @@ void init_dec(DecideParams &d, const Work &w, sdd_dtype_t dtype, int B, int gamm
     d.V = V;
     d.stride_bytes = row_stride * esize(dtype);
     d.tokens = tokens;
-    d.res_total = reinterpret_cast<float *>(w.base + w.L.res_total);
     d.res_pref = reinterpret_cast<float *>(w.base + w.L.res_pref);
     d.res_count = reinterpret_cast<uint32_t *>(w.base + w.L.res_count);
     const int RV = static_cast<int>((static_cast<int64_t>(V) * esize(dtype) + 15) / 16);

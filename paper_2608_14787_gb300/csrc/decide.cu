@@ -442,11 +442,10 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
             if (lane == 0) s_K0 = K;
         }
         __shared__ float s_warp[2 * NW];
-        __shared__ float s_pref[kDecThreads];
         __shared__ int s_is_last, s_seg, s_thr, s_thr_last, s_tok;
         __shared__ df s_rem;
-        __shared__ float s_tot[kDrawMaxSeg];
         __shared__ df s_cum[kDrawMaxSeg];
+        extern __shared__ float s_pref_all[];   // [nseg][kDecThreads]: every segment's prefixes (last CTA)
         if (tid == 0) {
             s_thr = INT32_MAX;
             s_thr_last = -1;
@@ -467,23 +466,25 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
             const int vb = min(v1, v0 + tid * vpt), ve = min(v1, vb + vpt);
             float tot;
             const float incl = cta_incl_scan(run_sum<DT>(c, vb, ve, p.V), s_warp, &tot);
+            (void)tot;
             d.res_pref[pair * kDecThreads + tid] = incl;   // this thread's inclusive prefix in the segment
             __syncthreads();
             if (tid == 0) {
-                d.res_total[pair] = tot;
                 // the barrier above orders every thread's prefix store before
-                // this fence, which orders them all before the arrival
-                __threadfence();
-                const uint32_t old = atomicAdd(d.res_count + i, 1u);
+                // this release; the acquire half orders the last arriver's
+                // reads of the other segments' prefixes after their releases
+                const uint32_t old = atom_add_acq_rel_gpu(d.res_count + i, 1u);
                 s_is_last = (old == static_cast<uint32_t>(d.nseg - 1)) ? 1 : 0;
             }
             __syncthreads();
         }
         if (s_is_last) {
-            // the last segment to arrive completes the draw
-            __threadfence();
-            for (int sg = tid; sg < d.nseg; sg += kDecThreads)
-                s_tot[sg] = __ldcg(d.res_total + static_cast<int64_t>(i) * d.nseg + sg);
+            // the last segment to arrive completes the draw: every segment's
+            // prefixes in one round trip (a segment's total is its last prefix)
+            const float4 *src =
+                reinterpret_cast<const float4 *>(d.res_pref + static_cast<int64_t>(i) * d.nseg * kDecThreads);
+            for (int q = tid; q < d.nseg * (kDecThreads / 4); q += kDecThreads) cp_async16(s_pref_all + 4 * q, src + q);
+            cp_async_wait_all();
             __syncthreads();
             if (warp == 0) {
                 // R = sum of the segment totals and their inclusive prefix sums
@@ -492,7 +493,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                 int last_seg = -1;   // the last segment of positive mass
                 for (int s0 = 0; s0 < d.nseg; s0 += 32) {
                     const int sg = s0 + lane;
-                    const float t = (sg < d.nseg) ? s_tot[sg] : 0.f;
+                    const float t = (sg < d.nseg) ? s_pref_all[sg * kDecThreads + kDecThreads - 1] : 0.f;
                     const df cum = df_add(carry, warp_prefix_df(df{t, 0.f}, lane));
                     if (sg < d.nseg) s_cum[sg] = cum;
                     if (t > 0.f) last_seg = sg;
@@ -512,7 +513,8 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                     __syncwarp();
                     for (int s0 = 0; s0 < d.nseg; s0 += 32) {
                         const int sg = s0 + lane;
-                        const bool hit = (sg < d.nseg) && s_tot[sg] > 0.f && !df_ge(target, s_cum[sg]);
+                        const bool hit = (sg < d.nseg) && s_pref_all[sg * kDecThreads + kDecThreads - 1] > 0.f &&
+                                         !df_ge(target, s_cum[sg]);
                         const unsigned bal = __ballot_sync(0xFFFFFFFFu, hit);
                         if (bal) {
                             sel = s0 + __ffs(bal) - 1;
@@ -539,8 +541,8 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
             if (sel >= 0) {
                 // the thread of segment sel whose run holds u R, from the
                 // inclusive prefixes that segment's CTA published
-                const float pv = __ldcg(d.res_pref + (static_cast<int64_t>(i) * d.nseg + sel) * kDecThreads + tid);
-                s_pref[tid] = pv;
+                const float *s_pref = s_pref_all + sel * kDecThreads;
+                const float pv = s_pref[tid];
                 const df rem = s_rem;
                 const unsigned bal = __ballot_sync(0xFFFFFFFFu, !df_ge(rem, df{pv, 0.f}));
                 if (lane == 0 && bal) atomicMin(&s_thr, warp * 32 + __ffs(bal) - 1);
@@ -742,12 +744,22 @@ int decide_max_ctas_per_sm() {
     return n;
 }
 
+// Opt both instantiations in to the prefix staging area of the draw.
+cudaError_t decide_prepare_device() {
+    constexpr int bytes = kDrawMaxSeg * kDecThreads * static_cast<int>(sizeof(float));
+    cudaError_t e = cudaFuncSetAttribute(decide_kernel<SDD_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(decide_kernel<SDD_F32>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+}
+
 cudaError_t launch_decide(const ScanParams &p, cudaStream_t stream) {
     const int nb = p.grp[0].nb;
     if (nb == 0) return cudaSuccess;
-    const int nseg = (p.dec.enabled && p.dec.do_strict && !p.dec.greedy) ? p.dec.nseg : 1;
+    const bool draw = p.dec.enabled && p.dec.do_strict && !p.dec.greedy;
+    const int nseg = draw ? p.dec.nseg : 1;
+    const size_t smem = draw ? static_cast<size_t>(nseg) * kDecThreads * sizeof(float) : 0;
     return launch_dependent(p.dtype == SDD_BF16 ? decide_kernel<SDD_BF16> : decide_kernel<SDD_F32>, dim3(nb, nseg),
-                            dim3(kDecThreads), 0, stream, p);
+                            dim3(kDecThreads), smem, stream, p);
 }
 
 cudaError_t launch_schedule(const ScheduleParams &p, cudaStream_t stream) {

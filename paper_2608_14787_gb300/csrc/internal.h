@@ -17,7 +17,7 @@ constexpr int kThreads = kWarpsPerCta * 32;
 constexpr int kVPL = 8;                       // 16-byte vectors per lane per tile
 constexpr int kTileVec = 32 * kVPL;           // vectors per warp tile
 constexpr int kTileBytes = kTileVec * 16;     // 4 KiB
-constexpr int kStages = 3;
+constexpr int kStages = 2;
 constexpr int kScanSmem = kWarpsPerCta * kStages * kTileBytes + kWarpsPerCta * kStages * 8;
 constexpr uint32_t kWaitPolls = 1u << 24;     // bounded mbarrier wait (seconds of polling)
 
@@ -46,9 +46,10 @@ inline FastDiv make_fastdiv(uint64_t d) {
 
 // Decide kernel geometry: one CTA of kDecThreads per (listed block, draw
 // segment); each draw segment is a run of whole 256-vector chunks of the draw
-// row, at most kDrawMaxSeg per block.
+// row, at most kDrawMaxSeg per block (the last CTA of a block stages every
+// segment's kDecThreads prefixes in shared memory: 1 KiB per segment).
 constexpr int kDecThreads = 256;
-constexpr int kDrawMaxSeg = 128;
+constexpr int kDrawMaxSeg = 64;
 
 // Per-block finalisation and decisions (decide.cu, rules.cuh).  Thresholds
 // are double-floats split on the host from their fp64 values.
@@ -84,7 +85,6 @@ struct DecideParams {
     long long *agreement;
     // sampling draw (residual / bonus inverse CDF), workspace
     int32_t nseg, seg_vec;         // segments per block and vectors per segment
-    float *res_total;              // [nb, nseg]
     float *res_pref;               // [nb, nseg, kDecThreads] per-thread inclusive prefix sums
     uint32_t *res_count;           // [nb] (zero between calls)
 };
@@ -163,6 +163,7 @@ cudaError_t launch_mlp(const void *h, int M, int K, const void *W1, const float 
 int scan_max_ctas_per_sm();
 int decide_max_ctas_per_sm();
 cudaError_t scan_prepare_device();
+cudaError_t decide_prepare_device();
 void set_last_error(const char *msg);  // message returned by sdd_last_error()
 
 __device__ __forceinline__ int64_t fast_div(int64_t n, const FastDiv &f) {
