@@ -229,6 +229,18 @@ __device__ __forceinline__ float fmax_nan(float a, float b) {
     asm("max.NaN.f32 %0, %1, %2;" : "=f"(d) : "f"(a), "f"(b));
     return d;
 }
+// Per-half comparisons of bf16 pairs: each 16-bit half of the result is
+// all ones where the comparison holds, zero elsewhere.
+__device__ __forceinline__ uint32_t bf16x2_gt(uint32_t a, uint32_t b) {
+    uint32_t d;
+    asm("set.gt.u32.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
+}
+__device__ __forceinline__ uint32_t bf16x2_eq(uint32_t a, uint32_t b) {
+    uint32_t d;
+    asm("set.eq.u32.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
+}
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 

@@ -112,6 +112,35 @@ __device__ __noinline__ void pad_tile(uint4 *tile, int n, int lane, bool row_end
 template <int DT>
 __device__ __noinline__ int count_before(const uint4 *tile, int n, int k0, int lane, float g, int tok) {
     constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
+    if (DT == SDD_BF16 && g > clamp_floor()) {
+        // Packed compares, two entries per instruction (g is a bf16 value above
+        // the clamp value, so clamping cannot change a comparison, and padded
+        // entries are -inf).  Entries equal to g rank before the token only at a
+        // lower index: counted one by one, in the rare tiles that hold any.
+        const uint32_t gb = __float_as_uint(g) >> 16, g2 = gb | (gb << 16);
+        int cnt = 0;
+        uint32_t eq = 0;
+#pragma unroll
+        for (int i = 0; i < kVPL; ++i) {
+            const uint4 w = tile[lane + 32 * i];
+            const uint32_t u[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                cnt += __popc(bf16x2_gt(u[q], g2) & 0x00010001u);
+                eq |= bf16x2_eq(u[q], g2);
+            }
+        }
+        if (eq) {
+#pragma unroll 1
+            for (int i = 0; i < kVPL; ++i) {
+                const uint4 w = tile[lane + 32 * i];
+#pragma unroll
+                for (int e = 0; e < EPV; ++e)
+                    cnt += (vec_elem<DT>(w, e) == g && (k0 + lane + 32 * i) * EPV + e < tok) ? 1 : 0;
+            }
+        }
+        return cnt;
+    }
     int cnt = 0;
 #pragma unroll 1
     for (int i = 0; i < kVPL; ++i) {

@@ -293,3 +293,33 @@ def test_strict_sampling_small_residuals(sdd, sigma):
         ob = oracle_block(z_d, z_t, x, seed=17, round_=rnd)
         compare_rule(tally, f"strict sigma={sigma} round {rnd}", L, tok, ob.strict, list(range(B)))
     print("small residuals", sigma, tally)
+
+
+def test_topk_and_greedy_with_tied_logits(sdd):
+    """Ranks with exact ties (App. A.6 top-k, greedy strict): target rows hold a
+    few entries above the drafted token's logit and a dozen exactly equal to it,
+    on both sides of the token, so the index tie-break decides the rank."""
+    B, gamma, V = 4, 6, 6000
+    g = torch.Generator().manual_seed(77)
+    z_t = torch.full((B, gamma + 1, V), -4.0)
+    x = torch.zeros((B, gamma), dtype=torch.int32)
+    for b in range(B):
+        for j in range(gamma + 1):
+            pos = torch.randperm(V, generator=g)[:15]
+            z_t[b, j, pos[:3]] = 2.0 + j % 2       # above the tie level (or two maxima ties)
+            z_t[b, j, pos[3:]] = 1.0 if j % 3 else 2.0 + j % 2
+            if j < gamma:
+                x[b, j] = int(pos[3 + (b * 7 + j * 5) % 12])
+    z_t = z_t.to(torch.bfloat16)
+    z_d = torch.randn((B, gamma, V), generator=g).to(torch.bfloat16)
+    z_d, z_t, x = z_d.to(DEV), z_t.to(DEV), x.to(DEV)
+    ks = (1, 2, 5, 10)
+    Lg, tkg, _ = sdd.verify_strict(z_t, x, greedy=True)
+    Lk, tkk, _ = sdd.verify_topk(z_t, x, ks)
+    torch.cuda.synchronize()
+    ob = oracle_block(z_d, z_t, x, ks=ks, sampling=False)
+    tally = Tally()
+    compare_rule(tally, "strict-greedy", Lg, tkg, ob.greedy, list(range(B)))
+    for r, k in enumerate(ks):
+        compare_rule(tally, f"top-{k}", Lk[r], tkk[r], ob.topk[k], list(range(B)))
+    assert tally.compared == B * (1 + len(ks)) and tally.flagged == 0
