@@ -305,6 +305,9 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t gw = static_cast<int64_t>(blockIdx.x) * kWarpsPerCta + warp;
     if (gw >= p.W) return;
+    // launched as a programmatic dependent of whatever precedes it in the
+    // stream: nothing is read or written before that work has completed
+    griddep_wait();
     constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
     const int tail = p.V % EPV;  // valid entries of the last vector of a row (0 = full)
 
@@ -471,12 +474,11 @@ cudaError_t scan_prepare_device() {
     return cudaFuncSetAttribute(scan_kernel<SDD_F32>, cudaFuncAttributeMaxDynamicSharedMemorySize, kScanSmem);
 }
 
+// The launch overhead of the streaming grid overlaps the tail of the work
+// ahead of it in the stream (the kernel waits for that work to complete).
 cudaError_t launch_scan(const ScanParams &p, int grid, cudaStream_t stream) {
-    if (p.dtype == SDD_BF16)
-        scan_kernel<SDD_BF16><<<grid, kThreads, kScanSmem, stream>>>(p);
-    else
-        scan_kernel<SDD_F32><<<grid, kThreads, kScanSmem, stream>>>(p);
-    return cudaGetLastError();
+    return launch_dependent(p.dtype == SDD_BF16 ? scan_kernel<SDD_BF16> : scan_kernel<SDD_F32>, dim3(grid),
+                            dim3(kThreads), kScanSmem, stream, p);
 }
 
 }  // namespace sdd
