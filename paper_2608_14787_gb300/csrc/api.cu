@@ -154,14 +154,14 @@ void finish_params(ScanParams &p, const Work &w) {
     p.rows0 = static_cast<int64_t>(p.grp[0].nb) * p.grp[0].npos;
     p.rows = p.rows0 + (p.n_groups > 1 ? static_cast<int64_t>(p.grp[1].nb) * p.grp[1].npos : 0);
     p.T = p.rows * p.RV;
-    p.W = static_cast<int32_t>(std::min<int64_t>(w.W_max, p.T));
+    p.W = scan_warps(w.W_max, p.T);
     set_divisors(p);
 }
 
 // The streaming kernel over the rows of p.
 sdd_status_t run_scan(const ScanParams &p, cudaStream_t stream) {
     if (p.T == 0) return SDD_OK;
-    if (static_cast<double>(p.T) * static_cast<double>(p.W) >= 9.007199254740992e15)   // 2^53
+    if (static_cast<double>(p.C) * static_cast<double>(p.W) >= 9.007199254740992e15)   // 2^53
         return fail(SDD_ERR_UNSUPPORTED, "%lld vectors of logits exceed the index arithmetic", (long long)p.T);
     const int grid = static_cast<int>((static_cast<int64_t>(p.W) + kWarpsPerCta - 1) / kWarpsPerCta);
     cudaError_t e = launch_scan(p, grid, stream);

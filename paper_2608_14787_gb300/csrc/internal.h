@@ -2,6 +2,7 @@
 // noalloc.cu) and the kernels (scan.cu, decide.cu).  Not part of the public ABI.
 #pragma once
 
+#include <algorithm>
 #include <cstdint>
 #include <cuda_runtime.h>
 
@@ -12,7 +13,7 @@ namespace sdd {
 
 // Streaming pass geometry: each warp owns a private ring of kStages tiles of
 // kVPL 16-byte vectors per lane, filled by 1D bulk copies.
-constexpr int kWarpsPerCta = 8;
+constexpr int kWarpsPerCta = 16;
 constexpr int kThreads = kWarpsPerCta * 32;
 constexpr int kVPL = 8;                       // 16-byte vectors per lane per tile
 constexpr int kTileVec = 32 * kVPL;           // vectors per warp tile
@@ -118,7 +119,11 @@ struct ScanParams {
     int64_t rows0;           // rows of group 0
     int64_t rows;            // rows of all groups
     int64_t T;               // total vectors = rows * RV
-    FastDiv divT, divW, divRV, divNpos[2];   // division by T, W, RV, grp[g].npos
+    // Cost-balanced partition: a vector of a group-g row costs wt[g] units
+    // (drafter rows carry the entropy work); T0 = rows0 * RV, C = total cost.
+    int32_t wt[2];
+    int64_t T0, C;
+    FastDiv divC, divW, divRV, divNpos[2], divWt[2];   // division by C, W, RV, grp[g].npos, wt[g]
     const int32_t *tokens;   // [B, gamma]
     Partial *partials;       // [rows + W]
     int32_t *status;
@@ -148,10 +153,28 @@ cudaError_t launch_commit(const int32_t *K, const int32_t *x, const int32_t *vt,
                           int gamma, int32_t *out_t, int32_t *out_n, cudaStream_t stream);
 cudaError_t launch_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, const uint64_t *round,
                             const uint32_t *purpose, int64_t n, float *u, cudaStream_t stream);
-// The division constants of a launch whose rows, T and W are set (host).
-// The magic divisions are exact while T * W < 2^53 (run_scan checks it).
+// Relative per-vector cost of streaming a drafter row (online softmax plus
+// the entropy accumulator) and a target row (online softmax plus the rank
+// count), measured on GB300: 10 : 9.
+constexpr int32_t kCostDrafter = 10, kCostTarget = 9;
+
+// Warps of a launch over T vectors with at most W_max warps: at least two
+// vectors per warp, so that with the cost weights every warp's share of the
+// cost holds at least one vector start (no empty warp inside a row).
+inline int32_t scan_warps(int64_t W_max, int64_t T) {
+    return static_cast<int32_t>(std::max<int64_t>(1, std::min<int64_t>(W_max, T / 2)));
+}
+
+// The cost weights and division constants of a launch whose groups, rows, T
+// and W are set (host).  The magic divisions are exact while C * W < 2^53
+// (the callers check it).
 inline void set_divisors(ScanParams &p) {
-    p.divT = make_fastdiv(static_cast<uint64_t>(p.T > 0 ? p.T : 1));
+    const bool mixed = p.n_groups == 2 && p.grp[0].kind != p.grp[1].kind;
+    for (int g = 0; g < 2; ++g) p.wt[g] = mixed ? (p.grp[g].kind == 0 ? kCostDrafter : kCostTarget) : 1;
+    p.T0 = p.rows0 * p.RV;
+    p.C = p.wt[0] * p.T0 + p.wt[1] * (p.T - p.T0);
+    p.divC = make_fastdiv(static_cast<uint64_t>(p.C > 0 ? p.C : 1));
+    for (int g = 0; g < 2; ++g) p.divWt[g] = make_fastdiv(static_cast<uint64_t>(p.wt[g]));
     p.divW = make_fastdiv(static_cast<uint64_t>(p.W > 0 ? p.W : 1));
     p.divRV = make_fastdiv(static_cast<uint64_t>(p.RV > 0 ? p.RV : 1));
     for (int g = 0; g < 2; ++g) p.divNpos[g] = make_fastdiv(static_cast<uint64_t>(p.grp[g].npos > 0 ? p.grp[g].npos : 1));
@@ -171,13 +194,21 @@ __device__ __forceinline__ int64_t fast_div(int64_t n, const FastDiv &f) {
     return static_cast<int64_t>(f.pow2 ? (u >> f.s) : (__umul64hi(u, f.M) >> f.s));
 }
 
-// Index arithmetic of the balanced contiguous partition of T vectors over W
-// warps: warp w owns [start(w), start(w+1)), start(w) = floor(w T / W).
-// Requires T W < 2^53 (checked by the host).
-__device__ __forceinline__ int64_t part_start(int64_t w, int64_t T, const FastDiv &divW) { return fast_div(w * T, divW); }
-// The warp owning vector v (requires W <= T, so every warp is non-empty).
-__device__ __forceinline__ int64_t part_owner(int64_t v, int64_t W, const FastDiv &divT) {
-    return fast_div((v + 1) * W - 1, divT);
+// Index arithmetic of the cost-balanced contiguous partition of the T
+// vectors over W warps.  Vector v occupies the cost interval [cost(v),
+// cost(v+1)) with cost(v) = wt0 min(v, T0) + wt1 max(v - T0, 0); warp w owns
+// the costs [floor(w C / W), floor((w+1) C / W)) and so the vectors whose
+// cost interval starts there: [start(w), start(w+1)) with start(w) the first
+// vector of cost >= floor(w C / W).  Requires C W < 2^53 (checked by the host).
+__device__ __forceinline__ int64_t part_start(const ScanParams &p, int64_t w) {
+    const int64_t c = fast_div(w * p.C, p.divW);
+    const int64_t c0 = p.wt[0] * p.T0;
+    return (c <= c0) ? fast_div(c + p.wt[0] - 1, p.divWt[0]) : p.T0 + fast_div(c - c0 + p.wt[1] - 1, p.divWt[1]);
+}
+// The warp owning vector v.
+__device__ __forceinline__ int64_t part_owner(const ScanParams &p, int64_t v) {
+    const int64_t cost = (v < p.T0) ? p.wt[0] * v : p.wt[0] * p.T0 + p.wt[1] * (v - p.T0);
+    return fast_div((cost + 1) * p.W - 1, p.divC);
 }
 
 }  // namespace sdd

@@ -138,9 +138,11 @@ sdd_status_t sdd_confidence_noalloc(const void *draft_logits, sdd_dtype_t dtype,
     p.rows0 = rows;
     p.rows = rows;
     p.T = rows * p.RV;
-    const int64_t W = std::min<int64_t>(nd.W_max, p.T);
+    const int64_t W = scan_warps(nd.W_max, p.T);
     p.W = static_cast<int32_t>(W);
     set_divisors(p);
+    if (static_cast<double>(p.C) * static_cast<double>(W) >= 9.007199254740992e15)   // 2^53
+        return na_fail(SDD_ERR_UNSUPPORTED, "%lld vectors of logits exceed the index arithmetic", (long long)p.T);
 
     cudaError_t e = launch_scan(p, static_cast<int>((W + kWarpsPerCta - 1) / kWarpsPerCta), st);
     if (e != cudaSuccess) return na_fail(SDD_ERR_CUDA, "scan launch: %s", cudaGetErrorString(e));

@@ -54,7 +54,7 @@ __device__ __forceinline__ Partial load_partial(const Partial *p) {
 // flight at a time.  The row's first piece carries its token logit; any piece
 // flags an out-of-range token.
 __device__ __forceinline__ void merge_row(const ScanParams &p, int64_t r, SoftState &acc, float &g, bool &tok_bad) {
-    const int64_t fw = part_owner(r * p.RV, p.W, p.divT), lw = part_owner((r + 1) * p.RV - 1, p.W, p.divT);
+    const int64_t fw = part_owner(p, r * p.RV), lw = part_owner(p, (r + 1) * p.RV - 1);
     acc = soft_identity();
     g = qnan();
     tok_bad = false;

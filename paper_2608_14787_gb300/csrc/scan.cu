@@ -300,7 +300,7 @@ __device__ __forceinline__ float token_logit(const ScanParams &p, int64_t r, Row
 }
 
 template <int DT>
-__global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant__ ScanParams p) {
+__global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant__ ScanParams p) {
     extern __shared__ __align__(128) unsigned char smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t gw = static_cast<int64_t>(blockIdx.x) * kWarpsPerCta + warp;
@@ -320,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 2) scan_kernel(const __grid_constant
     }
     __syncwarp();
 
-    const int64_t v0 = part_start(gw, p.T, p.divW), v1 = part_start(gw + 1, p.T, p.divW);
+    const int64_t v0 = part_start(p, gw), v1 = part_start(p, gw + 1);
     Cursor pc{v0, fast_div(v0, p.divRV), 0};
     pc.k = static_cast<int32_t>(v0 - pc.r * p.RV);
     Cursor cc = pc;
