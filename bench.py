@@ -38,9 +38,9 @@ UNIT = "blocks/s"
 EV_EVERY = 8   # steps between the event-bracketed launches of the streaming kernel
 NEAR = 1e-6
 # dram__bytes_read.sum + dram__bytes_write.sum of one scan_kernel launch on the
-# c3 workload (318.29 MB + 3.93 MB), from one ncu capture of the kernel as it
+# c3 workload (318.22 MB + 3.34 MB), from one ncu capture of the kernel as it
 # stands; reported as the roofline's "traffic" for that workload only.
-SCAN_TRAFFIC_C3 = 322_222_336
+SCAN_TRAFFIC_C3 = 321_560_320
 
 
 def _peaks():
@@ -60,14 +60,14 @@ def _workload_cfg(name):
     return wl, ells, tuple(wl.topks)
 
 
-def _config_json(wl, ells, ks):
+def _config_json(wl, ells, ks, n_sets=3):
     return {
         "workload": f"{wl.name}: {wl.description}",
         "B": wl.B, "gamma": wl.gamma, "V": wl.V, "dtype": "bf16" if "bfloat16" in str(wl.dtype) else "fp32",
         "taus": list(wl.taus), "ell_paper": [round(e, 6) for e in ells], "topk": list(ks),
         "strict": "sampling with residual/bonus resampling, shadow-verifies every block",
         "K_min": 6, "S_max": 64,
-        "l2": "inputs larger than L2: 3 rotating input sets of (2*gamma+1)*V*2*B bytes each",
+        "l2": f"inputs larger than L2: {n_sets} rotating input set(s) of (2*gamma+1)*V*2*B bytes each",
     }
 
 
@@ -336,7 +336,7 @@ def run_gpu(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if esz == 2 else "fp32", "data": "synthetic",
-            "config": _config_json(wl, ells, ks),
+            "config": _config_json(wl, ells, ks, n_sets),
             "achieved_gbs_step": scan_bytes / (total_ms / args.steps / 1e3) / 1e9,
             "roofline": {"bound": "hbm", "kernel": "scan_kernel (sdd_block_scan)", "achieved": achieved,
                          "peak": peak, "unit": "GB/s", "frac": achieved / peak, "traffic": args.traffic,
