@@ -77,8 +77,10 @@ typedef enum {
 
 typedef enum { SDD_F32 = 0, SDD_BF16 = 1 } sdd_dtype_t;
 
-/* Confidence signals of Sec. 4.2. */
-typedef enum { SDD_SIG_RAW = 0, SDD_SIG_MARGINAL = 1, SDD_SIG_CONDITIONAL = 2 } sdd_signal_t;
+/* Confidence signals of Sec. 4.2, and the confidence-free periodic skipping
+ * baseline of the appendix (its parameters are a period per pair and a skip
+ * length; see sdd_schedule_periodic). */
+typedef enum { SDD_SIG_RAW = 0, SDD_SIG_MARGINAL = 1, SDD_SIG_CONDITIONAL = 2, SDD_SIG_PERIODIC = 3 } sdd_signal_t;
 
 /* Bits of the device status word. */
 #define SDD_DEV_NONFINITE 1u  /* a logits row held NaN or +inf, or only -inf      */
@@ -152,6 +154,28 @@ SDD_API sdd_status_t sdd_schedule_prefix(const float *q, const float *logq, int 
                                  int n_tau, int K_min, int S_max, const uint8_t *guard,
                                  const uint8_t *force_strict, const int32_t *D_in, int32_t *K_hat,
                                  int32_t *K, int32_t *D_out, int32_t *status, sdd_stream_t stream);
+
+/*
+ * sdd_schedule_periodic -- the confidence-free periodic skipping baseline (the
+ * appendix's periodic-skipping paragraph and table): a skip of K_skip tokens is
+ * attempted once every period[t] rounds, all other rounds are strict, and an
+ * attempt meets the same guards as sdd_schedule_prefix.  For batch row b, pair t:
+ *   attempt = (round mod period[t] == period[t] - 1)   (reading: period[t] - 1
+ *             strict rounds precede each attempt; round counts from 0);
+ *   K_hat   = attempt ? min(K_skip, gamma, first guarded position - 1) : 0
+ *             (the prefix stops before a guarded position; force_strict[b]
+ *             forces K_hat = 0);
+ *   then the commit rule of sdd_schedule_prefix: D_in[b] >= S_max forces a
+ *   strict round, otherwise the block skips iff K_hat > 0 and K_hat >= K_min
+ *   (with K_min = K_skip a guarded prefix cancels the attempt).
+ *   period  HOST [n_p], each >= 1, 1 <= n_p <= SDD_MAX_GRID.  K_skip >= 1.
+ *   guard, force_strict, D_in, K_hat, K, D_out: as for sdd_schedule_prefix
+ *   ([n_p, B] outputs).  No scores are read.
+ */
+SDD_API sdd_status_t sdd_schedule_periodic(int B, int gamma, const int32_t *period, int n_p, int K_skip,
+                                           uint64_t round, int K_min, int S_max, const uint8_t *guard,
+                                           const uint8_t *force_strict, const int32_t *D_in, int32_t *K_hat,
+                                           int32_t *K, int32_t *D_out, int32_t *status, sdd_stream_t stream);
 
 /*
  * sdd_verify_strict -- Strict SDD verification (Sec. 3.1: the standard rule of
@@ -317,8 +341,11 @@ typedef struct sdd_block_args {
     /* schedule (Sec. 4.1) */
     int32_t signal;                /* sdd_signal_t */
     int32_t n_tau;                 /* 1..SDD_MAX_GRID */
-    const double *eta_b;           /* HOST [n_tau] */
-    const double *eta_c;           /* HOST [n_tau] */
+    const double *eta_b;           /* HOST [n_tau] (not read for SDD_SIG_PERIODIC) */
+    const double *eta_c;           /* HOST [n_tau] (not read for SDD_SIG_PERIODIC) */
+    const int32_t *period;         /* HOST [n_tau], SDD_SIG_PERIODIC only (else NULL) */
+    int32_t K_skip;                /* SDD_SIG_PERIODIC only */
+    int32_t reserved1;
     int32_t K_min, S_max;
     const uint8_t *guard;          /* [B, gamma] or NULL */
     const uint8_t *force_strict;   /* [B] or NULL */

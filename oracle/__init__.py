@@ -90,6 +90,9 @@ def lib():
     L.orc_schedule.argtypes = [dp, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_double, ctypes.c_double,
                                ctypes.c_int, ctypes.c_int, up8, up8, ip32, ip32, ip32, ip32, dp]
     L.orc_schedule.restype = None
+    L.orc_schedule_periodic.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_uint64,
+                                        ctypes.c_int, ctypes.c_int, up8, up8, ip32, ip32, ip32, ip32]
+    L.orc_schedule_periodic.restype = None
     L.orc_inverse_cdf.argtypes = [dp, ctypes.c_int64, ctypes.c_double, dp]
     L.orc_inverse_cdf.restype = ctypes.c_int64
     L.orc_verify_strict_sample.argtypes = [dp, dp, ip32, ctypes.c_int, ctypes.c_int64, dp, ctypes.c_double,
@@ -214,6 +217,21 @@ def schedule(q, signal, eta_b, eta_c, K_min, S_max, guard=None, force_strict=Non
                        _ptr(Kh, ctypes.c_int32), _ptr(K, ctypes.c_int32), _ptr(Do, ctypes.c_int32),
                        _ptr(mg, ctypes.c_double))
     return Kh, K, Do, mg
+
+
+def schedule_periodic(B, gamma, P, K_skip, round_, K_min, S_max, guard=None, force_strict=None, D_in=None):
+    """Periodic skipping baseline for one period P.  Returns (K_hat, K, D_out)."""
+    g = None if guard is None else np.ascontiguousarray(np.asarray(guard, dtype=np.uint8).reshape(B, gamma))
+    f = None if force_strict is None else np.ascontiguousarray(np.asarray(force_strict, dtype=np.uint8).reshape(B))
+    D = np.zeros(B, np.int32) if D_in is None else np.ascontiguousarray(np.asarray(D_in, dtype=np.int32).reshape(B))
+    Kh = np.zeros(B, np.int32)
+    K = np.zeros(B, np.int32)
+    Do = np.zeros(B, np.int32)
+    lib().orc_schedule_periodic(B, gamma, int(P), int(K_skip), int(round_), int(K_min), int(S_max),
+                                _ptr(g, ctypes.c_uint8) if g is not None else None,
+                                _ptr(f, ctypes.c_uint8) if f is not None else None, _ptr(D, ctypes.c_int32),
+                                _ptr(Kh, ctypes.c_int32), _ptr(K, ctypes.c_int32), _ptr(Do, ctypes.c_int32))
+    return Kh, K, Do
 
 
 # ----------------------------------------------------------------------------

@@ -253,6 +253,39 @@ void orc_schedule(const double *q, int B, int gamma, int signal, double eta_b, d
 }
 
 /* ------------------------------------------------------------------------ */
+/* Periodic skipping baseline (appendix, periodic-skipping paragraph): no    */
+/* confidence.  A skip of K_skip tokens is attempted once every P rounds --  */
+/* in the rounds with round mod P = P - 1 (reading: P - 1 strict rounds      */
+/* precede each attempt) -- and every other round is strict.  The attempt    */
+/* meets the guards of the confidence policy: it cannot cover a guarded      */
+/* position (the prefix ends before the first one), a shortened final block  */
+/* (force_strict) has none, and the commit rule of Sec. 4.1 follows (D >=    */
+/* S_max forces strict; skip iff K_hat > 0 and K_hat >= K_min; D += K or D = */
+/* 0).  Parity pinned by the closed forms in tests/test_oracle_schedule.py.  */
+/* ------------------------------------------------------------------------ */
+void orc_schedule_periodic(int B, int gamma, int P, int K_skip, uint64_t round, int K_min, int S_max,
+                           const uint8_t *guard, const uint8_t *force_strict, const int32_t *D_in,
+                           int32_t *K_hat_out, int32_t *K_out, int32_t *D_out) {
+    int attempt = (round % (uint64_t)P) == (uint64_t)(P - 1);
+    for (int b = 0; b < B; ++b) {
+        int K_hat = 0;
+        if (attempt && !(force_strict && force_strict[b])) {
+            /* longest prefix of length <= min(K_skip, gamma) with no guarded position */
+            int limit = K_skip < gamma ? K_skip : gamma;
+            for (int k = 1; k <= limit; ++k) {
+                if (guard && guard[(int64_t)b * gamma + (k - 1)]) break;
+                K_hat = k;
+            }
+        }
+        int D = D_in ? D_in[b] : 0;
+        int K = (D < S_max && K_hat > 0 && K_hat >= K_min) ? K_hat : 0;
+        K_hat_out[b] = K_hat;
+        K_out[b] = K;
+        if (D_out) D_out[b] = (K > 0) ? D + K : 0;
+    }
+}
+
+/* ------------------------------------------------------------------------ */
 /* Inverse-CDF draw over non-negative weights w[0..V) in ascending index     */
 /* order: the smallest v with sum_{x<=v} w(x) > u * R, R = sum w.  If        */
 /* rounding leaves no such v, the last v with positive weight.  Returns -1   */

@@ -19,7 +19,7 @@ LIB_PATH = os.path.join(_HERE, "_build", "libsdd.so")
 SDD_OK = 0
 SDD_F32 = 0
 SDD_BF16 = 1
-SIG_RAW, SIG_MARGINAL, SIG_CONDITIONAL = 0, 1, 2
+SIG_RAW, SIG_MARGINAL, SIG_CONDITIONAL, SIG_PERIODIC = 0, 1, 2, 3
 DEV_NONFINITE, DEV_BAD_TOKEN, DEV_TIMEOUT = 1, 2, 4
 MAX_GAMMA = 128
 MAX_GRID = 32
@@ -41,6 +41,7 @@ class BlockArgs(ctypes.Structure):
         ("dtype", ctypes.c_int32), ("B", ctypes.c_int32), ("gamma", ctypes.c_int32), ("V", ctypes.c_int32),
         ("row_stride", ctypes.c_int64),
         ("signal", ctypes.c_int32), ("n_tau", ctypes.c_int32), ("eta_b", c_f64p), ("eta_c", c_f64p),
+        ("period", c_i32p), ("K_skip", ctypes.c_int32), ("reserved1", ctypes.c_int32),
         ("K_min", ctypes.c_int32), ("S_max", ctypes.c_int32),
         ("guard", VP), ("force_strict", VP), ("D_in", VP),
         ("greedy", ctypes.c_int32), ("reserved0", ctypes.c_int32),
@@ -75,6 +76,7 @@ def load(path: str | None = None):
     L.sdd_workspace_size.argtypes = [I, I, I, ctypes.POINTER(ctypes.c_size_t)]
     L.sdd_confidence.argtypes = [VP, I, I, I, I, i64, VP, VP, VP, VP, VP, VP, VP, VP, ctypes.c_size_t, VP, VP]
     L.sdd_schedule_prefix.argtypes = [VP, VP, I, I, I, c_f64p, c_f64p, I, I, I, VP, VP, VP, VP, VP, VP, VP, VP]
+    L.sdd_schedule_periodic.argtypes = [I, I, c_i32p, I, I, u64, I, I, VP, VP, VP, VP, VP, VP, VP, VP]
     L.sdd_verify_strict.argtypes = [VP, VP, I, I, I, I, i64, VP, VP, I, u64, u64, VP, I, VP, VP, VP, VP,
                                     ctypes.c_size_t, VP, VP]
     L.sdd_verify_lenient.argtypes = [VP, I, I, I, I, i64, VP, c_f64p, I, VP, I, VP, VP, VP, VP, ctypes.c_size_t,
@@ -90,7 +92,8 @@ def load(path: str | None = None):
     L.sdd_survival_mlp.restype = I
     for fn in ("sdd_block", "sdd_block_scan", "sdd_block_decide"):
         getattr(L, fn).argtypes = [ctypes.POINTER(BlockArgs), VP]
-    for fn in ("sdd_workspace_size", "sdd_confidence", "sdd_schedule_prefix", "sdd_verify_strict",
+    for fn in ("sdd_workspace_size", "sdd_confidence", "sdd_schedule_prefix", "sdd_schedule_periodic",
+               "sdd_verify_strict",
                "sdd_verify_lenient", "sdd_verify_topk", "sdd_agreement", "sdd_commit", "sdd_uniforms", "sdd_block",
                "sdd_block_scan", "sdd_block_decide"):
         getattr(L, fn).restype = I
@@ -230,6 +233,20 @@ def schedule_prefix(q, eta_b, eta_c, *, signal=SIG_RAW, logq=None, K_min=6, S_ma
     return Kh, K, Do
 
 
+def schedule_periodic(B, gamma, periods, *, K_skip=6, round_=0, K_min=6, S_max=64, guard=None, force_strict=None,
+                      D_in=None, status=None, stream=None, device="cuda"):
+    """sdd_schedule_periodic; returns (K_hat, K, D_out), each [n_p, B]."""
+    n_p = len(periods)
+    Kh = torch.empty(n_p, B, dtype=torch.int32, device=device)
+    K = torch.empty(n_p, B, dtype=torch.int32, device=device)
+    Do = torch.empty(n_p, B, dtype=torch.int32, device=device)
+    per = (ctypes.c_int32 * n_p)(*[int(x) for x in periods])
+    rc = load().sdd_schedule_periodic(B, gamma, per, n_p, K_skip, round_, K_min, S_max, _p(guard), _p(force_strict),
+                                      _p(D_in), _p(Kh), _p(K), _p(Do), _p(status), _stream(stream))
+    _check(rc, "sdd_schedule_periodic")
+    return Kh, K, Do
+
+
 def verify_strict(z_t, x, *, z_d=None, draft=None, greedy=False, seed=0, round_=0, rows=None,
                   ws: Workspace | None = None, status=None, stream=None, out=None):
     """sdd_verify_strict; returns (L [B], tokens [B, gamma+1], n_commit [B])."""
@@ -349,10 +366,17 @@ class BlockRound:
     """
 
     def __init__(self, B, gamma, V, *, dtype=torch.bfloat16, taus=(0.9,), eta_b=None, eta_c=None,
-                 signal=SIG_RAW, K_min=6, S_max=64, ells=(), ks=(), greedy=False, device="cuda"):
+                 signal=SIG_RAW, K_min=6, S_max=64, ells=(), ks=(), greedy=False, periods=None, K_skip=6,
+                 device="cuda"):
+        """signal=SIG_PERIODIC schedules the periodic baseline: one pair per entry
+        of `periods` (skip K_skip tokens once every P rounds); taus are unused."""
         dev = torch.device(device)
         self.B, self.gamma, self.V = B, gamma, V
         self.dtype = dtype
+        if signal == SIG_PERIODIC:
+            if not periods:
+                raise ValueError("SIG_PERIODIC needs periods")
+            eta_b = eta_c = [0.0] * len(periods)
         eta_b = list(taus) if eta_b is None else list(eta_b)
         eta_c = list(taus) if eta_c is None else list(eta_c)
         self.n_tau = len(eta_b)
@@ -384,6 +408,10 @@ class BlockRound:
         a.eta_b = ctypes.cast(self._eta_b, c_f64p)
         a.eta_c = ctypes.cast(self._eta_c, c_f64p)
         a.K_min, a.S_max = K_min, S_max
+        if signal == SIG_PERIODIC:
+            self._period = (ctypes.c_int32 * len(periods))(*[int(x) for x in periods])
+            a.period = ctypes.cast(self._period, c_i32p)
+            a.K_skip = int(K_skip)
         a.greedy = 1 if greedy else 0
         a.n_ell, a.n_k = ne, nk
         a.ell = ctypes.cast(self._ell, c_f64p)

@@ -216,6 +216,19 @@ sdd_status_t set_thresholds(int signal, const double *eta_b, const double *eta_c
     return SDD_OK;
 }
 
+// Periods and skip length of the periodic baseline, validated.
+sdd_status_t set_periods(const int32_t *period, int n_p, int K_skip, int32_t *out) {
+    if (n_p < 1 || n_p > SDD_MAX_GRID)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "%d periods outside [1, %d]", n_p, SDD_MAX_GRID);
+    if (!period) return fail(SDD_ERR_INVALID_ARGUMENT, "period is NULL");
+    if (K_skip < 1) return fail(SDD_ERR_INVALID_ARGUMENT, "K_skip = %d < 1", K_skip);
+    for (int t = 0; t < n_p; ++t) {
+        if (period[t] < 1) return fail(SDD_ERR_INVALID_ARGUMENT, "period[%d] = %d < 1", t, period[t]);
+        out[t] = period[t];
+    }
+    return SDD_OK;
+}
+
 sdd_status_t set_ell(DecideParams &d, const double *ell, int n_ell) {
     if (n_ell < 0 || n_ell > SDD_MAX_GRID)
         return fail(SDD_ERR_INVALID_ARGUMENT, "n_ell = %d outside [0, %d]", n_ell, SDD_MAX_GRID);
@@ -353,6 +366,38 @@ sdd_status_t sdd_schedule_prefix(const float *q, const float *logq, int B, int g
     p.gamma = gamma;
     p.signal = signal;
     p.n_tau = n_tau;
+    p.K_min = K_min;
+    p.S_max = S_max;
+    p.guard = guard;
+    p.force_strict = force_strict;
+    p.D_in = D_in;
+    p.K_hat = K_hat;
+    p.K = K;
+    p.D_out = D_out;
+    cudaError_t e = launch_schedule(p, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "schedule launch");
+    return SDD_OK;
+}
+
+sdd_status_t sdd_schedule_periodic(int B, int gamma, const int32_t *period, int n_p, int K_skip, uint64_t round,
+                                   int K_min, int S_max, const uint8_t *guard, const uint8_t *force_strict,
+                                   const int32_t *D_in, int32_t *K_hat, int32_t *K, int32_t *D_out, int32_t *status,
+                                   sdd_stream_t stream) {
+    (void)status;
+    if (B < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "B = %d < 0", B);
+    if (gamma < 1 || gamma > SDD_MAX_GAMMA)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "gamma = %d outside [1, %d]", gamma, SDD_MAX_GAMMA);
+    ScheduleParams p;
+    std::memset(&p, 0, sizeof p);
+    SDD_TRY(set_periods(period, n_p, K_skip, p.period));
+    if (B == 0) return SDD_OK;
+    if (!K_hat || !K) return fail(SDD_ERR_INVALID_ARGUMENT, "K_hat and K must not be NULL");
+    p.B = B;
+    p.gamma = gamma;
+    p.signal = SDD_SIG_PERIODIC;
+    p.n_tau = n_p;
+    p.K_skip = K_skip;
+    p.round = round;
     p.K_min = K_min;
     p.S_max = S_max;
     p.guard = guard;
@@ -520,7 +565,12 @@ static sdd_status_t block_params(const sdd_block_args *a, ScanParams &p, bool *e
     const sdd_dtype_t dt = static_cast<sdd_dtype_t>(a->dtype);
     DecideParams d;
     std::memset(&d, 0, sizeof d);
-    SDD_TRY(set_thresholds(a->signal, a->eta_b, a->eta_c, a->n_tau, d.eta_loc, d.log_eta_c, d.tau_off));
+    if (a->signal == SDD_SIG_PERIODIC) {
+        SDD_TRY(set_periods(a->period, a->n_tau, a->K_skip, d.period));
+        d.K_skip = a->K_skip;
+    } else {
+        SDD_TRY(set_thresholds(a->signal, a->eta_b, a->eta_c, a->n_tau, d.eta_loc, d.log_eta_c, d.tau_off));
+    }
     SDD_TRY(set_ell(d, a->ell, a->n_ell));
     int kcap = 1;
     SDD_TRY(set_topk(d, a->topk, a->n_k, kcap));

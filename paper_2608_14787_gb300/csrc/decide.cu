@@ -329,6 +329,11 @@ __device__ __forceinline__ void sched_pair(const DecideParams &d, const BlockFac
     Kh = K = Do = 0;
     if (force || d.tau_off[t]) return;
     const int gamma = d.gamma;
+    if (d.signal == SDD_SIG_PERIODIC) {
+        Kh = periodic_khat(gamma, d.period[t], d.K_skip, d.round, [&](int j) { return F.guard[j] != 0; }, lane);
+        sched_final(Kh, D, d.K_min, d.S_max, K, Do);
+        return;
+    }
     int kb = gamma, best = 0;
     df carry = df{0.f, 0.f};
     for (int c = 0; c < gamma && kb >= c; c += 32) {
@@ -677,7 +682,13 @@ __global__ void schedule_kernel(const __grid_constant__ ScheduleParams p) {
     const bool force = p.force_strict && p.force_strict[b];
     const int D = p.D_in ? p.D_in[b] : 0;
     int Kh = 0, K = 0, Do = 0;
-    if (!(force || p.tau_off[t])) {
+    if (p.signal == SDD_SIG_PERIODIC) {
+        if (!force) {
+            Kh = periodic_khat(gamma, p.period[t], p.K_skip, p.round,
+                               [&](int j) { return p.guard && p.guard[o + j] != 0; }, lane);
+            sched_final(Kh, D, p.K_min, p.S_max, K, Do);
+        }
+    } else if (!(force || p.tau_off[t])) {
         int kb = gamma, best = 0;
         df carry = df{0.f, 0.f};
         for (int c = 0; c < gamma && kb >= c; c += 32) {

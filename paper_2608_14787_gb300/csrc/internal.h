@@ -76,6 +76,7 @@ struct DecideParams {
     int32_t *L_topk, *tok_topk, *n_topk;
     // schedule (fused round)
     int32_t do_sched, signal, n_tau, K_min, S_max;
+    int32_t period[SDD_MAX_GRID], K_skip;   // SDD_SIG_PERIODIC
     int32_t tau_off[SDD_MAX_GRID];
     df eta_loc[SDD_MAX_GRID];
     df log_eta_c[SDD_MAX_GRID];
@@ -133,6 +134,8 @@ struct ScanParams {
 struct ScheduleParams {
     const float *q, *logq;
     int32_t B, gamma, signal, n_tau, K_min, S_max;
+    int32_t period[SDD_MAX_GRID], K_skip;   // SDD_SIG_PERIODIC
+    uint64_t round;
     int32_t tau_off[SDD_MAX_GRID];
     df eta_loc[SDD_MAX_GRID];
     df log_eta_c[SDD_MAX_GRID];

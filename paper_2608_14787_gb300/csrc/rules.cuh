@@ -252,6 +252,26 @@ __device__ __forceinline__ void sched_step(int c, int lane, int gamma, bool in, 
     if (bal2) best = c + 32 - __clz(bal2);
 }
 
+// K_hat of the periodic skipping baseline (the appendix's confidence-free
+// schedule), by one warp: rounds with round mod period = period - 1 attempt
+// K_skip tokens, every other round none; the prefix stops before the first
+// guarded position (guarded(j) for position j < gamma).
+template <typename Guard>
+__device__ __forceinline__ int periodic_khat(int gamma, int period, int K_skip, uint64_t round, Guard guarded,
+                                             int lane) {
+    if (period < 1 || round % static_cast<uint64_t>(period) != static_cast<uint64_t>(period - 1)) return 0;
+    int kb = gamma;
+    for (int c = 0; c < gamma; c += 32) {
+        const int j = c + lane;
+        const unsigned bal = __ballot_sync(0xFFFFFFFFu, j < gamma && guarded(j));
+        if (bal) {
+            kb = c + __ffs(bal) - 1;
+            break;
+        }
+    }
+    return min(K_skip, kb);
+}
+
 // K_min / staleness gate of Sec. 4.1 on a block's K_hat.
 __device__ __forceinline__ void sched_final(int K_hat, int D, int K_min, int S_max, int &K, int &D_out) {
     K = (D < S_max && K_hat > 0 && K_hat >= K_min) ? K_hat : 0;

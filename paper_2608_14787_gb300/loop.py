@@ -9,7 +9,9 @@ counter D carried across rounds.  The raw-confidence policy drives the round:
 blocks with K = 0 go to the strict verifier (Sec. 3.1), which reads only
 their target rows (row compaction); the committed tokens are x_1..x_K for a
 skipped block and the verified tokens otherwise.  The survival-score policy
-runs in shadow (its decisions and verifier calls saved are counted).
+and the confidence-free periodic baseline of the appendix (a skip of K_min
+tokens once every `period` rounds) run in shadow (their decisions and
+verifier calls saved are counted).
 
 Every step runs in libsdd.so through the binding; this module only sequences
 the calls.  One device-to-host read per round (how many blocks to verify)
@@ -34,6 +36,7 @@ from . import synth
 class RoundOut:
     K_raw: torch.Tensor        # [B] K under raw confidence (drives the round)
     K_mlp: torch.Tensor        # [B] K under the survival score (shadow)
+    K_per: torch.Tensor        # [B] K under the periodic baseline (shadow)
     L: torch.Tensor            # [B] strict accepted length (-2 for skipped blocks)
     tokens: torch.Tensor       # [B, gamma+1] committed tokens (-1 padded)
     n: torch.Tensor            # [B] committed count
@@ -47,6 +50,7 @@ class LoopStats:
     verified: int = 0
     skipped_raw: int = 0
     skipped_mlp: int = 0
+    skipped_per: int = 0
     committed_tokens: int = 0
     device_seconds: float = 0.0
     per_round_verified: list = field(default_factory=list)
@@ -56,16 +60,18 @@ class DecodeLoop:
     """State of one decode loop: workspace, D per policy, scorer weights."""
 
     def __init__(self, B: int, gamma: int, V: int, *, tau: float = 0.9, tau_mlp: float = 0.9, K_min: int = 6,
-                 S_max: int = 64, greedy: bool = False, seed: int = 4, hidden: int = synth.HIDDEN, device="cuda"):
+                 S_max: int = 64, greedy: bool = False, seed: int = 4, hidden: int = synth.HIDDEN, period: int = 4,
+                 device="cuda"):
         self.B, self.gamma, self.V = B, gamma, V
         self.tau, self.tau_mlp, self.K_min, self.S_max = tau, tau_mlp, K_min, S_max
-        self.greedy, self.seed = greedy, seed
+        self.greedy, self.seed, self.period = greedy, seed, period
         dev = torch.device(device)
         self.device = dev
         self.ws = sdd.Workspace(B, gamma, V, dev)
         self.status = sdd.new_status(dev)
         self.D_raw = torch.zeros(B, dtype=torch.int32, device=dev)
         self.D_mlp = torch.zeros(B, dtype=torch.int32, device=dev)
+        self.D_per = torch.zeros(B, dtype=torch.int32, device=dev)
         self.W1, self.b1, self.w2, b2 = synth.make_mlp(device=dev, seed=seed, hidden=hidden)
         self.b2 = float(b2.item())
 
@@ -79,14 +85,17 @@ class DecodeLoop:
         _, K_mlp, D_mlp = sdd.schedule_prefix(s, [self.tau_mlp], [self.tau_mlp], signal=sdd.SIG_CONDITIONAL,
                                               K_min=self.K_min, S_max=self.S_max, D_in=self.D_mlp,
                                               status=self.status)
+        _, K_per, D_per = sdd.schedule_periodic(B, gamma, [self.period], K_skip=max(self.K_min, 1), round_=round_,
+                                                K_min=self.K_min, S_max=self.S_max, D_in=self.D_per,
+                                                status=self.status, device=self.device)
         K = K_raw[0]
         rows = torch.nonzero(K == 0).flatten().to(torch.int32)    # the host's verify decision
         n_rows = int(rows.numel())
         L, tok, n = sdd.verify_strict(z_t, x, z_d=z_d, draft=conf, greedy=self.greedy, seed=self.seed, round_=round_,
                                       rows=rows, ws=self.ws, status=self.status)
         tokens, n_commit = sdd.commit(K, x, tok, n)
-        self.D_raw, self.D_mlp = D_raw[0].contiguous(), D_mlp[0].contiguous()
-        return RoundOut(K_raw=K, K_mlp=K_mlp[0], L=L, tokens=tokens, n=n_commit, n_verified=n_rows)
+        self.D_raw, self.D_mlp, self.D_per = D_raw[0].contiguous(), D_mlp[0].contiguous(), D_per[0].contiguous()
+        return RoundOut(K_raw=K, K_mlp=K_mlp[0], K_per=K_per[0], L=L, tokens=tokens, n=n_commit, n_verified=n_rows)
 
 
 def run(rounds: int = 256, workload: str = "c5", warmup: int = 2, device="cuda") -> dict:
@@ -109,6 +118,7 @@ def run(rounds: int = 256, workload: str = "c5", warmup: int = 2, device="cuda")
         if r < 0:
             loop.D_raw.zero_()
             loop.D_mlp.zero_()
+            loop.D_per.zero_()
             continue
         st.rounds += 1
         st.blocks += B
@@ -117,6 +127,7 @@ def run(rounds: int = 256, workload: str = "c5", warmup: int = 2, device="cuda")
         st.per_round_verified.append(out.n_verified)
         st.skipped_raw += int((out.K_raw > 0).sum().item())
         st.skipped_mlp += int((out.K_mlp > 0).sum().item())
+        st.skipped_per += int((out.K_per > 0).sum().item())
         st.committed_tokens += int(out.n.sum().item())
         del blk, h
     status = int(loop.status.item())
@@ -128,6 +139,8 @@ def run(rounds: int = 256, workload: str = "c5", warmup: int = 2, device="cuda")
         "verifier_calls": st.verified,
         "verifier_calls_saved_raw": st.skipped_raw / max(st.blocks, 1),
         "verifier_calls_saved_mlp_shadow": st.skipped_mlp / max(st.blocks, 1),
+        "verifier_calls_saved_periodic_shadow": st.skipped_per / max(st.blocks, 1),
+        "periodic_P": loop.period,
         "committed_tokens_per_block": st.committed_tokens / max(st.blocks, 1),
         "device_status": status,
     }

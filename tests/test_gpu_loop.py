@@ -21,10 +21,11 @@ def _bits(t):
 @pytest.mark.parametrize("B,gamma,V,hidden,rounds", [(6, 8, 3008, 128, 4), (3, 32, 20016, 256, 3)])
 def test_loop_matches_oracle_replay(sdd, orc, B, gamma, V, hidden, rounds):
     wl = synth.WORKLOADS["c5"]
-    loop = DecodeLoop(B, gamma, V, tau=0.5, tau_mlp=0.3, K_min=2, S_max=6, seed=wl.seed, hidden=hidden)
+    loop = DecodeLoop(B, gamma, V, tau=0.5, tau_mlp=0.3, K_min=2, S_max=6, seed=wl.seed, hidden=hidden, period=2)
     W1, b1, w2 = _bits(loop.W1), loop.b1.cpu().numpy(), _bits(loop.w2)
     D_raw = np.zeros(B, np.int32)
     D_mlp = np.zeros(B, np.int32)
+    D_per = np.zeros(B, np.int32)
     seen_skip = seen_verify = 0
     for r in range(rounds):
         blk = synth.make_block(wl, device="cuda", round_=r, B=B, gamma=gamma, V=V)
@@ -43,6 +44,9 @@ def test_loop_matches_oracle_replay(sdd, orc, B, gamma, V, hidden, rounds):
         np.testing.assert_array_equal(out.K_mlp.cpu().numpy(), K_mlp)
         np.testing.assert_array_equal(loop.D_raw.cpu().numpy(), D_raw)
         np.testing.assert_array_equal(loop.D_mlp.cpu().numpy(), D_mlp)
+        _, K_per, D_per = orc.schedule_periodic(B, gamma, 2, 2, r, 2, 6, D_in=D_per)   # P = 2, K_skip = K_min
+        np.testing.assert_array_equal(out.K_per.cpu().numpy(), K_per)
+        np.testing.assert_array_equal(loop.D_per.cpu().numpy(), D_per)
         L_dev, tok_dev, n_dev = out.L.cpu().numpy(), out.tokens.cpu().numpy(), out.n.cpu().numpy()
         assert out.n_verified == int((K_raw == 0).sum())
         for b in range(B):

@@ -323,3 +323,61 @@ def test_topk_and_greedy_with_tied_logits(sdd):
     for r, k in enumerate(ks):
         compare_rule(tally, f"top-{k}", Lk[r], tkk[r], ob.topk[k], list(range(B)))
     assert tally.compared == B * (1 + len(ks)) and tally.flagged == 0
+
+
+# ---------------------------------------------------------------------------
+# periodic skipping baseline (appendix): stand-alone and in the fused round
+# ---------------------------------------------------------------------------
+
+def test_schedule_periodic_vs_oracle(sdd):
+    B, gamma = 37, 40                     # two warp chunks of positions
+    g = torch.Generator().manual_seed(5)
+    guard = (torch.rand(B, gamma, generator=g) < 0.03).to(torch.uint8)
+    force = (torch.rand(B, generator=g) < 0.1).to(torch.uint8)
+    D = torch.randint(0, 80, (B,), generator=g, dtype=torch.int32)
+    periods = (1, 3, 4, 8)
+    for round_ in range(10):
+        for K_min, K_skip in ((6, 6), (0, 6), (2, 45)):
+            Kh, K, Do = sdd.schedule_periodic(B, gamma, periods, K_skip=K_skip, round_=round_, K_min=K_min,
+                                              S_max=64, guard=guard.to(DEV), force_strict=force.to(DEV),
+                                              D_in=D.to(DEV))
+            torch.cuda.synchronize()
+            for t, P in enumerate(periods):
+                oKh, oK, oD = orc.schedule_periodic(B, gamma, P, K_skip, round_, K_min, 64, guard=guard.numpy(),
+                                                    force_strict=force.numpy(), D_in=D.numpy())
+                np.testing.assert_array_equal(Kh[t].cpu().numpy(), oKh)
+                np.testing.assert_array_equal(K[t].cpu().numpy(), oK)
+                np.testing.assert_array_equal(Do[t].cpu().numpy(), oD)
+
+
+@pytest.mark.parametrize("round_", [2, 3])
+def test_block_round_periodic_vs_oracle(sdd, round_):
+    B, gamma, V = 6, 16, 4096
+    blk = synth.make_block("c3", device="cpu", B=B, gamma=gamma, V=V)
+    z_d, z_t, x = _to_dev(blk)
+    periods = (2, 3, 4)
+    rnd = sdd.BlockRound(B, gamma, V, signal=sdd.SIG_PERIODIC, periods=periods, K_skip=6, K_min=6, S_max=64)
+    D = torch.tensor([0, 5, 60, 64, 70, 10], dtype=torch.int32)
+    rnd.D_in.copy_(D)
+    rnd.set_inputs(z_d, z_t, x, seed=11, round_=round_)
+    rnd.run()
+    torch.cuda.synchronize()
+    assert int(rnd.status.item()) == 0
+    ob = oracle_block(z_d, z_t, x, seed=11, round_=round_)
+    tally = Tally()
+    compare_rule(tally, "strict", rnd.L_strict, rnd.tokens_strict, ob.strict, list(range(B)))
+    xs = x.cpu().numpy()
+    for t, P in enumerate(periods):
+        oKh, oK, oD = orc.schedule_periodic(B, gamma, P, 6, round_, 6, 64, D_in=D.numpy())
+        np.testing.assert_array_equal(rnd.K_hat[t].cpu().numpy(), oKh)
+        np.testing.assert_array_equal(rnd.K[t].cpu().numpy(), oK)
+        np.testing.assert_array_equal(rnd.D_out[t].cpu().numpy(), oD)
+    oK0 = orc.schedule_periodic(B, gamma, periods[0], 6, round_, 6, 64, D_in=D.numpy())[1]
+    ct, cn = rnd.commit_tokens.cpu().numpy(), rnd.commit_n.cpu().numpy()
+    for b in range(B):
+        if oK0[b] > 0:
+            assert cn[b] == 6 and np.array_equal(ct[b][:6], xs[b][:6]) and np.all(ct[b][6:] == -1)
+        else:
+            L, tok, _ = ob.strict[b]
+            assert cn[b] == L + 1 and np.array_equal(ct[b], tok)
+    assert tally.flagged_mismatch == 0

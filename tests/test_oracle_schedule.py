@@ -181,3 +181,58 @@ def test_margin_reports_distance_to_threshold(orc):
     q = np.array([[0.9000004, 0.95, 0.95]])
     _, _, _, mg = orc.schedule(q, MARG, 0.9, 0.9, 0, 64)
     assert mg[0] == pytest.approx(4e-7, rel=1e-3)
+
+
+# ---------------------------------------------------------------------------
+# Periodic skipping baseline (appendix): K_skip tokens once every P rounds
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("P", [1, 3, 4, 8])
+def test_periodic_attempts_once_per_period(orc, P):
+    """Over any P consecutive rounds exactly one attempt; without guards and with
+    staleness far away every attempt skips K_skip tokens and the others are strict."""
+    B, gamma, K_skip = 5, 32, 6
+    for start in range(0, 3 * P):
+        skips = 0
+        for r in range(start, start + P):
+            Kh, K, Do = orc.schedule_periodic(B, gamma, P, K_skip, r, 6, 10**6)
+            assert (Kh == K).all() and len(set(K.tolist())) == 1
+            if K[0] > 0:
+                skips += 1
+                assert K[0] == K_skip and r % P == P - 1
+                assert (Do == K_skip).all()
+            else:
+                assert (Do == 0).all()
+        assert skips == 1
+
+
+def test_periodic_staleness_run_matches_closed_form(orc):
+    """A simulated sequence: D grows by K_skip at every attempt and resets on
+    every strict round, so with S_max >= K_skip every attempt skips and the
+    fraction of verifier calls saved is exactly 1/P."""
+    for P in (3, 4, 8):
+        D = np.zeros(1, np.int32)
+        calls = 0
+        R = 24 * P
+        for r in range(R):
+            Kh, K, Do = orc.schedule_periodic(1, 32, P, 6, r, 6, 64, D_in=D)
+            calls += int(K[0] == 0)
+            D = Do
+        assert calls == R - R // P
+
+
+def test_periodic_guards_kmin_force_and_staleness(orc):
+    B, gamma, P, K_skip = 4, 16, 2, 6
+    guard = np.zeros((B, gamma), np.uint8)
+    guard[1, 2] = 1            # guarded third position: prefix of 2
+    guard[2, 7] = 1            # beyond K_skip: no effect
+    force = np.array([0, 0, 0, 1], np.uint8)
+    D = np.array([0, 0, 0, 0], np.int32)
+    Kh, K, Do = orc.schedule_periodic(B, gamma, P, K_skip, 1, 6, 64, guard=guard, force_strict=force, D_in=D)
+    assert Kh.tolist() == [6, 2, 6, 0] and K.tolist() == [6, 0, 6, 0]     # K_min = 6 cancels the short prefix
+    Kh, K, Do = orc.schedule_periodic(B, gamma, P, K_skip, 1, 0, 64, guard=guard, force_strict=force, D_in=D)
+    assert K.tolist() == [6, 2, 6, 0] and Do.tolist() == [6, 2, 6, 0]
+    Kh, K, Do = orc.schedule_periodic(B, gamma, P, K_skip, 1, 0, 64, D_in=np.array([63, 64, 70, 0], np.int32))
+    assert K.tolist() == [6, 0, 0, 6] and Do.tolist() == [69, 0, 0, 6]   # staleness: D >= S_max forces strict
+    Kh, K, Do = orc.schedule_periodic(B, 4, P, K_skip, 1, 0, 64)            # gamma below K_skip
+    assert K.tolist() == [4] * B
