@@ -83,6 +83,9 @@ def lib():
     L.orc_row_stats.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
                                 ip32, dp, dp, dp, dp, dp, dp, ip32]
     L.orc_row_stats.restype = None
+    L.orc_row_features.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+                                   dp, dp]
+    L.orc_row_features.restype = None
     L.orc_row_probs.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_int64, dp]
     L.orc_row_probs.restype = None
     L.orc_rank.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64]
@@ -181,6 +184,19 @@ def row_stats(z, tokens=None) -> RowStats:
                         *[_ptr(o, ctypes.c_double) for o in outs], _ptr(am, ctypes.c_int32))
     m, lse, q, logq, mp, H = (o.reshape(lead) for o in outs)
     return RowStats(m=m, lse=lse, q=q, logq=logq, maxprob=mp, entropy=H, argmax=am.reshape(lead))
+
+
+def row_features(z):
+    """Probability margin p_(1) - p_(2) and top-5 mass of every row of ``z``
+    ([..., V]), fp64.  Returns (margin, top5) shaped z.shape[:-1]."""
+    z, dt = _logits_arg(z)
+    lead = z.shape[:-1]
+    V = z.shape[-1]
+    n = int(np.prod(lead)) if lead else 1
+    mg = np.zeros(n, np.float64)
+    t5 = np.zeros(n, np.float64)
+    lib().orc_row_features(z.ctypes.data, dt, n, V, V, _ptr(mg, ctypes.c_double), _ptr(t5, ctypes.c_double))
+    return mg.reshape(lead), t5.reshape(lead)
 
 
 def row_probs(z_row) -> np.ndarray:

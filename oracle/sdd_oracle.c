@@ -159,6 +159,61 @@ void orc_row_stats(const void *logits, int dtype, int64_t n_rows, int64_t V, int
     }
 }
 
+/* ------------------------------------------------------------------------ */
+/* Extended pre-verification features of a drafter row (App. A.7's list:    */
+/* probability margin and top-5 probability mass; top-1 probability, its    */
+/* log and the entropy come from orc_row_stats).  With p_(1) >= p_(2) >= ...  */
+/* the probabilities in descending order (ties kept with multiplicity):      */
+/*   margin = p_(1) - p_(2)       (p_(2) = 0 when V = 1)                     */
+/*   top5   = p_(1) + ... + p_(min(5, V))                                   */
+/* Logits are clamped from below at -2^23 as everywhere in the path.  A row  */
+/* with NaN or +inf, or with only -inf, has no distribution: NaN features.   */
+/* Parity pinned in tests/test_oracle_stats.py (closed forms, a library      */
+/* sort + logsumexp).                                                       */
+/* ------------------------------------------------------------------------ */
+void orc_row_features(const void *logits, int dtype, int64_t n_rows, int64_t V, int64_t row_stride,
+                      double *out_margin, double *out_top5) {
+    const double floor_ = -8388608.0; /* -2^23 */
+    for (int64_t r = 0; r < n_rows; ++r) {
+        int64_t base = r * row_stride;
+        double top[5] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY, -INFINITY};
+        double m = -INFINITY;
+        int bad = 0;
+        for (int64_t v = 0; v < V; ++v) {
+            double z = orc_load(logits, dtype, base + v);
+            if (isnan(z) || (isinf(z) && z > 0)) bad = 1;
+            if (z > m) m = z;
+        }
+        if (m == -INFINITY) bad = 1;
+        if (bad) {
+            out_margin[r] = NAN;
+            out_top5[r] = NAN;
+            continue;
+        }
+        double s = 0.0;
+        for (int64_t v = 0; v < V; ++v) {
+            double z = orc_load(logits, dtype, base + v);
+            if (z < floor_) z = floor_;
+            s += exp(z - m);
+            /* insert z into the descending list of the 5 largest values */
+            for (int i = 0; i < 5; ++i) {
+                if (z > top[i]) {
+                    for (int k = 4; k > i; --k) top[k] = top[k - 1];
+                    top[i] = z;
+                    break;
+                }
+            }
+        }
+        double lse = m + log(s);
+        int n = V < 5 ? (int)V : 5;
+        double t5 = 0.0;
+        for (int i = 0; i < n; ++i) t5 += exp(top[i] - lse);
+        double p1 = exp(top[0] - lse), p2 = (V > 1) ? exp(top[1] - lse) : 0.0;
+        out_margin[r] = p1 - p2;
+        out_top5[r] = t5;
+    }
+}
+
 /* Normalised probabilities of one row, p(v) = exp(z(v) - LSE), fp64. */
 void orc_row_probs(const void *logits, int dtype, int64_t V, int64_t offset, double *p) {
     double m = -INFINITY;

@@ -121,3 +121,54 @@ def test_rank_vs_library_sort(orc):
         pos[order] = np.arange(V)
         for t in rng.integers(0, V, size=5):
             assert orc.rank(z, int(t)) == pos[t]
+
+
+# ---------------------------------------------------------------------------
+# Extended features (App. A.7: probability margin, top-5 probability mass)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("V", [1, 3, 5, 6, 1000])
+def test_features_all_equal_row(orc, V):
+    z = np.full((1, V), 2.5, np.float32)
+    mg, t5 = orc.row_features(z)
+    assert mg[0] == pytest.approx(1.0 if V == 1 else 0.0, abs=1e-15)
+    assert t5[0] == pytest.approx(min(5, V) / V, rel=1e-13)
+
+
+@pytest.mark.parametrize("k,V,a", [(1, 100, 3.0), (2, 100, 3.0), (7, 5000, 1.25), (3, 10, -2.0)])
+def test_features_two_level_row(orc, k, V, a):
+    """k entries at level a, V - k at 0: p_hi = e^a / (k e^a + V - k)."""
+    z = np.zeros((1, V), np.float32)
+    z[0, np.random.default_rng(k).choice(V, k, replace=False)] = a
+    mg, t5 = orc.row_features(z)
+    Z = k * math.exp(a) + (V - k)
+    hi, lo = math.exp(a) / Z, 1.0 / Z
+    top = sorted([hi] * k + [lo] * (V - k), reverse=True)
+    assert mg[0] == pytest.approx(top[0] - top[1], rel=1e-12, abs=1e-15)
+    assert t5[0] == pytest.approx(sum(top[:5]), rel=1e-12)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_features_vs_library_sort(orc, dtype):
+    rng = np.random.default_rng(3)
+    R, V = 8, 4003
+    x = (rng.normal(size=(R, V)) * rng.uniform(0.3, 6.0, size=(R, 1))).astype(np.float32)
+    x[2, :40] = x[2].max()            # a tied maximum (margin 0)
+    z, zf = (_bf16_bits(x), _bf16_vals(_bf16_bits(x))) if dtype == "bf16" else (x, x.astype(np.float64))
+    mg, t5 = orc.row_features(z)
+    p = torch.softmax(torch.from_numpy(zf), dim=-1)
+    srt = torch.sort(p, dim=-1, descending=True).values.numpy()
+    np.testing.assert_allclose(mg, srt[:, 0] - srt[:, 1], rtol=1e-11, atol=1e-15)
+    np.testing.assert_allclose(t5, srt[:, :5].sum(-1), rtol=1e-12)
+    assert mg[2] == 0.0
+
+
+def test_features_nonfinite_and_masked(orc):
+    z = np.zeros((4, 50), np.float32)
+    z[0, 3] = np.nan
+    z[1, :] = -np.inf
+    z[2, 10:] = -np.inf                # ten finite entries: top-5 mass 0.5
+    z[3, 7] = np.inf
+    mg, t5 = orc.row_features(z)
+    assert np.isnan(mg[[0, 1, 3]]).all() and np.isnan(t5[[0, 1, 3]]).all()
+    assert mg[2] == 0.0 and t5[2] == pytest.approx(0.5, rel=1e-14)
