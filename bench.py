@@ -19,6 +19,7 @@ Prints one JSON line (rank 0).
 Other rows of the path, one JSON line each (not the fused-round contract line):
   python bench.py --component mlp [--steps K]   the survival scorer alone (K launches)
   python bench.py --component loop [--steps R]  the decode-loop workload (R rounds, default 64)
+  python bench.py --component features          drafter confidence with / without the extended features
 """
 from __future__ import annotations
 
@@ -429,6 +430,65 @@ def run_component_mlp(args):
     return 0
 
 
+def run_component_features(args):
+    """Drafter confidence with and without the extended features (App. A.7:
+    probability margin, top-5 mass) on the drafter half of the c3 workload
+    (16 blocks x 32 rows x 151,936 bf16 = 155.6 MB), 3 rotating input sets
+    (> L2); device time per call (streaming + decide kernels) from CUDA events
+    around `--steps` back-to-back calls."""
+    import torch
+    import paper_2608_14787_gb300 as sdd
+    from paper_2608_14787_gb300 import build as sdd_build
+    from paper_2608_14787_gb300 import synth
+    sdd_build.build()
+    sdd.load()
+    wl = synth.WORKLOADS["c3"]
+    B, gamma, V = wl.B, wl.gamma, wl.V
+    sets = [synth.make_block(wl, device="cuda", round_=r) for r in range(3)]
+    ws = sdd.Workspace(B, gamma, V, torch.device("cuda"))
+    status = sdd.new_status(torch.device("cuda"))
+    steps = max(args.steps // 8, 64)
+
+    def timed(features):
+        for i in range(max(args.warmup, 3)):
+            sdd.confidence(sets[i % 3].z_d, sets[i % 3].x, ws=ws, status=status, features=features)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for i in range(steps):
+            sdd.confidence(sets[i % 3].z_d, sets[i % 3].x, ws=ws, status=status, features=features)
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / steps / 1e3
+    with ClockSampler(None) as clk:
+        t_plain = timed(False)
+        t_feat = timed(True)
+    nbytes = B * gamma * V * 2
+    hbm, hkind = _peaks()
+    cpu = None
+    if not args.no_cpu_baseline:
+        import oracle as orc
+        rows = 16
+        t0 = time.perf_counter()
+        orc.row_features(synth.bf16_bits(sets[0].z_d[0, :rows]))
+        orc.row_stats(synth.bf16_bits(sets[0].z_d[0, :rows]), tokens=sets[0].x[0, :rows].cpu().numpy())
+        dt = time.perf_counter() - t0
+        cpu = {"value": rows / dt, "unit": "rows/s", "cores": 1, "kind": "oracle",
+               "sample": f"{rows} drafter rows of one block, stats + features, single thread ({dt:.2f} s)"}
+    line = {
+        "component": "NEXT-2 extended features (sdd_confidence_features)", "metric": "drafter rows scored/s",
+        "unit": "rows/s", "value": B * gamma / t_feat, "us_per_call": t_feat * 1e6,
+        "us_per_call_without_features": t_plain * 1e6,
+        "config": {"B": B, "gamma": gamma, "V": V, "dtype": "bf16", "rows": B * gamma},
+        "roofline": {"bound": "hbm", "achieved": nbytes / t_feat / 1e9, "peak": hbm, "unit": "GB/s",
+                     "frac": nbytes / t_feat / 1e9 / hbm, "bytes": nbytes, "peak_source": f"{hkind} hbm_gbs",
+                     "note": "whole call (streaming + decide kernels) per launch pair"},
+        "cpu_baseline": cpu, "clocks": clk.summary(), "device_status": int(status.item()),
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_component_loop(args):
     """The decode-loop workload (B=128, gamma=32, V=151,936 bf16): `--steps`
     rounds (default 64) of fresh logits and hidden states, generated untimed."""
@@ -476,13 +536,15 @@ def main():
     ap.add_argument("--sets", type=int, default=3, help="rotating input sets (3 x 316 MB exceeds L2)")
     ap.add_argument("--traffic", type=float, default=None,
                     help="dram bytes per scan launch from an ncu capture of the current kernel")
-    ap.add_argument("--component", default=None, choices=["mlp", "loop"],
+    ap.add_argument("--component", default=None, choices=["mlp", "loop", "features"],
                     help="measure one other row of the path instead of the fused round")
     args = ap.parse_args()
     if args.component == "mlp":
         return run_component_mlp(args)
     if args.component == "loop":
         return run_component_loop(args)
+    if args.component == "features":
+        return run_component_features(args)
     if args.traffic is None and args.workload == "c3":
         args.traffic = SCAN_TRAFFIC_C3
     if args.warmup < 3:

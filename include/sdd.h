@@ -128,6 +128,24 @@ SDD_API sdd_status_t sdd_confidence(const void *draft_logits, sdd_dtype_t dtype,
                             sdd_stream_t stream);
 
 /*
+ * sdd_confidence_features -- sdd_confidence plus two more of the learned
+ * scorer's pre-verification features (App. A.7) from the same single read of
+ * the drafter logits: with p_(1) >= p_(2) >= ... the row's probabilities in
+ * descending order (ties kept with multiplicity),
+ *   margin[b, j] = p_(1) - p_(2)   (p_(2) = 0 when V = 1),
+ *   top5[b, j]   = p_(1) + ... + p_(min(5, V))   (top-5 probability mass),
+ * both fp32 [B, gamma], NaN for a row without a distribution (as q).  The
+ * streaming pass additionally keeps each lane's five largest entries; the
+ * other arguments, outputs and errors are those of sdd_confidence (margin and
+ * top5 must not be NULL).
+ */
+SDD_API sdd_status_t sdd_confidence_features(const void *draft_logits, sdd_dtype_t dtype, int B, int gamma, int V,
+                                             int64_t row_stride, const int32_t *draft_tokens, float *q,
+                                             float *logq, float *maxprob, double *lse, float *entropy,
+                                             int32_t *argmax, float *margin, float *top5, void *workspace,
+                                             size_t workspace_bytes, int32_t *status, sdd_stream_t stream);
+
+/*
  * sdd_schedule_prefix -- the skip policy of Sec. 4.1 for n_tau threshold pairs
  * (Eq. 3 and the commit rule that follows it).  For batch row b and pair t:
  *   B_k = min_{j<=k} q_j;  C_k = (prod q)^(1/k) (RAW), min_{j<=k} q_j (MARGINAL),

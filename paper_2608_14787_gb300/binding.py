@@ -75,6 +75,8 @@ def load(path: str | None = None):
     L.sdd_last_error.restype = ctypes.c_char_p
     L.sdd_workspace_size.argtypes = [I, I, I, ctypes.POINTER(ctypes.c_size_t)]
     L.sdd_confidence.argtypes = [VP, I, I, I, I, i64, VP, VP, VP, VP, VP, VP, VP, VP, ctypes.c_size_t, VP, VP]
+    L.sdd_confidence_features.argtypes = [VP, I, I, I, I, i64, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP,
+                                          ctypes.c_size_t, VP, VP]
     L.sdd_schedule_prefix.argtypes = [VP, VP, I, I, I, c_f64p, c_f64p, I, I, I, VP, VP, VP, VP, VP, VP, VP, VP]
     L.sdd_schedule_periodic.argtypes = [I, I, c_i32p, I, I, u64, I, I, VP, VP, VP, VP, VP, VP, VP, VP]
     L.sdd_verify_strict.argtypes = [VP, VP, I, I, I, I, i64, VP, VP, I, u64, u64, VP, I, VP, VP, VP, VP,
@@ -92,7 +94,8 @@ def load(path: str | None = None):
     L.sdd_survival_mlp.restype = I
     for fn in ("sdd_block", "sdd_block_scan", "sdd_block_decide"):
         getattr(L, fn).argtypes = [ctypes.POINTER(BlockArgs), VP]
-    for fn in ("sdd_workspace_size", "sdd_confidence", "sdd_schedule_prefix", "sdd_schedule_periodic",
+    for fn in ("sdd_workspace_size", "sdd_confidence", "sdd_confidence_features", "sdd_schedule_prefix",
+               "sdd_schedule_periodic",
                "sdd_verify_strict",
                "sdd_verify_lenient", "sdd_verify_topk", "sdd_agreement", "sdd_commit", "sdd_uniforms", "sdd_block",
                "sdd_block_scan", "sdd_block_decide"):
@@ -175,11 +178,14 @@ class Confidence:
     lse: torch.Tensor
     entropy: torch.Tensor
     argmax: torch.Tensor
+    margin: torch.Tensor | None = None   # extended features (confidence(..., features=True))
+    top5: torch.Tensor | None = None
 
 
 def confidence(z_d: torch.Tensor, x: torch.Tensor, ws: Workspace | None = None, status=None,
-               stream=None) -> Confidence:
-    """sdd_confidence over drafter logits z_d [B, gamma, V] and drafted tokens x [B, gamma]."""
+               stream=None, features: bool = False) -> Confidence:
+    """sdd_confidence over drafter logits z_d [B, gamma, V] and drafted tokens x [B, gamma];
+    with features=True sdd_confidence_features (also margin and top5 [B, gamma])."""
     B, gamma = x.shape
     V, stride = _logits_layout(z_d, "z_d")
     dev = z_d.device
@@ -188,6 +194,14 @@ def confidence(z_d: torch.Tensor, x: torch.Tensor, ws: Workspace | None = None, 
     f32 = lambda: torch.empty(B, gamma, dtype=torch.float32, device=dev)  # noqa: E731
     out = Confidence(q=f32(), logq=f32(), maxprob=f32(), lse=torch.empty(B, gamma, dtype=torch.float64, device=dev),
                      entropy=f32(), argmax=torch.empty(B, gamma, dtype=torch.int32, device=dev))
+    if features:
+        out.margin, out.top5 = f32(), f32()
+        rc = load().sdd_confidence_features(_p(z_d), _dtype_code(z_d), B, gamma, V, stride, _p(x), _p(out.q),
+                                            _p(out.logq), _p(out.maxprob), _p(out.lse), _p(out.entropy),
+                                            _p(out.argmax), _p(out.margin), _p(out.top5), ws.ptr, ws.nbytes,
+                                            _p(status), _stream(stream))
+        _check(rc, "sdd_confidence_features")
+        return out
     rc = load().sdd_confidence(_p(z_d), _dtype_code(z_d), B, gamma, V, stride, _p(x), _p(out.q), _p(out.logq),
                                _p(out.maxprob), _p(out.lse), _p(out.entropy), _p(out.argmax), ws.ptr, ws.nbytes,
                                _p(status), _stream(stream))

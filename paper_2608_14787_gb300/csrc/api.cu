@@ -68,7 +68,7 @@ inline size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255);
 
 // Workspace layout for blocks of shape (B, gamma) on a device with W_max warps.
 struct Layout {
-    size_t partials, res_pref, res_count, total;
+    size_t partials, feat, res_pref, res_count, total;
 };
 
 Layout layout(int64_t B, int64_t gamma, int64_t W_max, int64_t dec_ctas) {
@@ -81,6 +81,7 @@ Layout layout(int64_t B, int64_t gamma, int64_t W_max, int64_t dec_ctas) {
         return at;
     };
     L.partials = take(static_cast<size_t>(rows + W_max) * sizeof(Partial));
+    L.feat = take(static_cast<size_t>(rows + W_max) * sizeof(FeatPartial));
     // nb * nseg <= max(resident decide CTAs, B) (see init_dec)
     L.res_pref = take(static_cast<size_t>(std::max(dec_ctas, B)) * kDecThreads * sizeof(float));
     L.res_count = take(static_cast<size_t>(B) * sizeof(uint32_t));
@@ -315,10 +316,12 @@ sdd_status_t sdd_workspace_size(int B, int gamma, int V, size_t *bytes) {
     return SDD_OK;
 }
 
-sdd_status_t sdd_confidence(const void *draft_logits, sdd_dtype_t dtype, int B, int gamma, int V,
-                            int64_t row_stride, const int32_t *draft_tokens, float *q, float *logq,
-                            float *maxprob, double *lse, float *entropy, int32_t *argmax, void *workspace,
-                            size_t workspace_bytes, int32_t *status, sdd_stream_t stream) {
+// The drafter statistics, with the extended features when margin or top5 is set.
+static sdd_status_t confidence_impl(const void *draft_logits, sdd_dtype_t dtype, int B, int gamma, int V,
+                                    int64_t row_stride, const int32_t *draft_tokens, float *q, float *logq,
+                                    float *maxprob, double *lse, float *entropy, int32_t *argmax, float *margin,
+                                    float *top5, void *workspace, size_t workspace_bytes, int32_t *status,
+                                    sdd_stream_t stream) {
     SDD_TRY(check_shape(dtype, B, gamma, V, row_stride));
     if (B == 0) return SDD_OK;
     SDD_TRY(check_ptr16(draft_logits, "draft_logits"));
@@ -341,10 +344,33 @@ sdd_status_t sdd_confidence(const void *draft_logits, sdd_dtype_t dtype, int B, 
     G.lse = lse;
     G.entropy = entropy;
     G.argmax = argmax;
+    if (margin || top5) {
+        G.margin = margin;
+        G.top5 = top5;
+        p.feat = reinterpret_cast<FeatPartial *>(w.base + w.L.feat);
+    }
     finish_params(p, w);
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     SDD_TRY(run_scan(p, st));
     return run_decide(p, st);
+}
+
+sdd_status_t sdd_confidence(const void *draft_logits, sdd_dtype_t dtype, int B, int gamma, int V,
+                            int64_t row_stride, const int32_t *draft_tokens, float *q, float *logq,
+                            float *maxprob, double *lse, float *entropy, int32_t *argmax, void *workspace,
+                            size_t workspace_bytes, int32_t *status, sdd_stream_t stream) {
+    return confidence_impl(draft_logits, dtype, B, gamma, V, row_stride, draft_tokens, q, logq, maxprob, lse, entropy,
+                           argmax, nullptr, nullptr, workspace, workspace_bytes, status, stream);
+}
+
+sdd_status_t sdd_confidence_features(const void *draft_logits, sdd_dtype_t dtype, int B, int gamma, int V,
+                                     int64_t row_stride, const int32_t *draft_tokens, float *q, float *logq,
+                                     float *maxprob, double *lse, float *entropy, int32_t *argmax, float *margin,
+                                     float *top5, void *workspace, size_t workspace_bytes, int32_t *status,
+                                     sdd_stream_t stream) {
+    if (!margin || !top5) return fail(SDD_ERR_INVALID_ARGUMENT, "margin and top5 must not be NULL");
+    return confidence_impl(draft_logits, dtype, B, gamma, V, row_stride, draft_tokens, q, logq, maxprob, lse, entropy,
+                           argmax, margin, top5, workspace, workspace_bytes, status, stream);
 }
 
 sdd_status_t sdd_schedule_prefix(const float *q, const float *logq, int B, int gamma, sdd_signal_t signal,

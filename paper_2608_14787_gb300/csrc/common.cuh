@@ -376,6 +376,13 @@ enum : uint32_t { kPurposeAccept = 0, kPurposeResid = 1, kPurposeBonus = 2 };
 // two (the references are integers), so merging never rounds the scale; the
 // exp-sum stays a double-float throughout.
 // ---------------------------------------------------------------------------
+// The five largest (clamped) logits of a drafter row piece, descending, with
+// multiplicity (-inf where the piece holds fewer): the extended features.
+struct FeatPartial {
+    float top[5];
+    float pad[3];
+};
+
 struct SoftState {
     float m, r, t2;
     float sh, sl;

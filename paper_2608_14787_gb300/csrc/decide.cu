@@ -349,7 +349,9 @@ __device__ __forceinline__ void sched_pair(const DecideParams &d, const BlockFac
     sched_final(Kh, D, d.K_min, d.S_max, K, Do);
 }
 
-template <int DT>
+// FEAT: also the extended features of the drafter rows (a separate
+// instantiation, so that calls without them keep the smaller kernel).
+template <int DT, bool FEAT>
 __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_constant__ ScanParams p) {
     griddep_wait();   // launched behind the streaming grid that wrote the partials
     const DecideParams &d = p.dec;
@@ -406,8 +408,14 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                 SoftState acc;
                 float g;
                 bool bad;
-                merge_row(p, (gd ? p.rows0 : 0) + static_cast<int64_t>(i) * G.npos + j, acc, g, bad);
+                const int64_t r = (gd ? p.rows0 : 0) + static_cast<int64_t>(i) * G.npos + j;
+                merge_row(p, r, acc, g, bad);
                 f = row_final(p, G, j, b, acc, g, bad, leader);
+                if (FEAT && leader) {
+                    float top[5];
+                    feat_merge(p, r, top);
+                    feat_final(G, static_cast<int64_t>(b) * p.gamma + j, top, f.lse);
+                }
             } else {
                 // stand-alone acceptance: the caller's drafter LSE and the token's drafter logit
                 f = facts_invalid();
@@ -751,16 +759,20 @@ __global__ void uniforms_kernel(uint64_t seed, const uint32_t *j, const uint32_t
 
 int decide_max_ctas_per_sm() {
     int n = 0;
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decide_kernel<SDD_BF16>, kDecThreads, 0);
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decide_kernel<SDD_BF16, false>, kDecThreads, 0);
     return n;
 }
 
 // Opt both instantiations in to the prefix staging area of the draw.
 cudaError_t decide_prepare_device() {
     constexpr int bytes = kDrawMaxSeg * kDecThreads * static_cast<int>(sizeof(float));
-    cudaError_t e = cudaFuncSetAttribute(decide_kernel<SDD_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-    if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(decide_kernel<SDD_F32>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    void (*const kernels[])(ScanParams) = {decide_kernel<SDD_BF16, false>, decide_kernel<SDD_F32, false>,
+                                           decide_kernel<SDD_BF16, true>, decide_kernel<SDD_F32, true>};
+    for (auto k : kernels) {
+        const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 cudaError_t launch_decide(const ScanParams &p, cudaStream_t stream) {
@@ -769,7 +781,10 @@ cudaError_t launch_decide(const ScanParams &p, cudaStream_t stream) {
     const bool draw = p.dec.enabled && p.dec.do_strict && !p.dec.greedy;
     const int nseg = draw ? p.dec.nseg : 1;
     const size_t smem = draw ? static_cast<size_t>(nseg) * kDecThreads * sizeof(float) : 0;
-    return launch_dependent(p.dtype == SDD_BF16 ? decide_kernel<SDD_BF16> : decide_kernel<SDD_F32>, dim3(nb, nseg),
+    const bool bf = p.dtype == SDD_BF16, feat = p.feat != nullptr;
+    void (*const k)(ScanParams) = feat ? (bf ? decide_kernel<SDD_BF16, true> : decide_kernel<SDD_F32, true>)
+                                       : (bf ? decide_kernel<SDD_BF16, false> : decide_kernel<SDD_F32, false>);
+    return launch_dependent(k, dim3(nb, nseg),
                             dim3(kDecThreads), smem, stream, p);
 }
 

@@ -105,6 +105,7 @@ struct ScanGroup {
     float *q, *logq, *maxprob, *entropy;
     double *lse;
     int32_t *argmax;
+    float *margin, *top5;    // extended features (only with ScanParams::feat)
 };
 
 struct ScanParams {
@@ -127,6 +128,7 @@ struct ScanParams {
     FastDiv divC, divW, divRV, divNpos[2], divWt[2];   // division by C, W, RV, grp[g].npos, wt[g]
     const int32_t *tokens;   // [B, gamma]
     Partial *partials;       // [rows + W]
+    FeatPartial *feat;       // [rows + W], or nullptr: no extended features
     int32_t *status;
     DecideParams dec;
 };

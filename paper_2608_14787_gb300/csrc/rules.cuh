@@ -151,6 +151,60 @@ __device__ __forceinline__ RowFacts row_final(const ScanParams &p, const ScanGro
     return f;
 }
 
+// The five largest entries of drafter row r (global row index), merged from
+// its pieces' lists, by one thread.  The first four pieces' lists are loaded
+// together (a row rarely has more).
+__device__ __forceinline__ void feat_merge(const ScanParams &p, int64_t r, float (&t)[5]) {
+    const int64_t fw = part_owner(p, r * p.RV), lw = part_owner(p, (r + 1) * p.RV - 1);
+#pragma unroll
+    for (int k = 0; k < 5; ++k) t[k] = -INFINITY;
+    for (int64_t w0 = fw; w0 <= lw; w0 += 4) {
+        uint4 v[4][2];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+            if (w0 + u <= lw) {
+                v[u][0] = __ldcg(reinterpret_cast<const uint4 *>(p.feat + r + w0 + u));
+                v[u][1] = __ldcg(reinterpret_cast<const uint4 *>(p.feat + r + w0 + u) + 1);
+            }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            if (w0 + u > lw) break;
+            const float f[5] = {__uint_as_float(v[u][0].x), __uint_as_float(v[u][0].y), __uint_as_float(v[u][0].z),
+                                __uint_as_float(v[u][0].w), __uint_as_float(v[u][1].x)};
+#pragma unroll
+            for (int i = 0; i < 5; ++i) {
+                float z = f[i];
+#pragma unroll
+                for (int k = 0; k < 5; ++k) {   // insert z into the descending list
+                    const float hi = fmaxf(t[k], z), lo = fminf(t[k], z);
+                    t[k] = hi;
+                    z = lo;
+                }
+            }
+        }
+    }
+}
+
+// Extended features of a drafter row (user index o) from its five largest
+// entries t and LSE: margin = p_(1) - p_(2), top5 = p_(1) + ... + p_(5) (an
+// entry that is not there contributes exp(-inf) = 0), by one thread.
+__device__ __forceinline__ void feat_final(const ScanGroup &G, int64_t o, const float (&t)[5], df lse) {
+    float margin = qnan(), top5 = qnan();
+    if (!isnan(lse.hi)) {
+        float pk[5];
+#pragma unroll
+        for (int k = 0; k < 5; ++k) {
+            const df d = df_sub(df{t[k], 0.f}, lse);
+            const float e = expf(d.hi);
+            pk[k] = (t[k] == -INFINITY) ? 0.f : fmaf(e, d.lo, e);
+        }
+        margin = pk[0] - pk[1];
+        top5 = (((pk[4] + pk[3]) + pk[2]) + pk[1]) + pk[0];
+    }
+    if (G.margin) G.margin[o] = margin;
+    if (G.top5) G.top5[o] = top5;
+}
+
 // ---------------------------------------------------------------------------
 // The facts of one block, in shared memory (position j on index j)
 // ---------------------------------------------------------------------------

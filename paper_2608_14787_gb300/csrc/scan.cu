@@ -191,9 +191,11 @@ __device__ __noinline__ int first_index(const char *rowp, int k0, int lane, int 
 // clamped first (so a masked entry adds 0 * finite to t2); target rows need no
 // clamp (2^-inf = 0 and the maximum starts at the clamp value).  The lane's
 // exp-sum is an fp32 pair (s_hi, s_lo) updated by TwoSum once per tile.
-template <int DT, bool ENT>
+// vmax (FEAT only): the maximum of each of the lane's vectors, kept for the
+// extended features (bf16: as a packed pair, f32: as bits).
+template <int DT, bool ENT, bool FEAT>
 __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lane, SoftState &st, float &s_hi,
-                                              float &s_lo) {
+                                              float &s_lo, uint32_t (&vmax)[kVPL]) {
     // pass 1: the tile maximum (clamp value included)
     float cm;
     if (DT == SDD_BF16) {
@@ -201,7 +203,9 @@ __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lan
 #pragma unroll
         for (int i = 0; i < kVPL; ++i) {
             const uint4 w = tile[lane + 32 * i];
-            mx = bf16x2_max_nan(bf16x2_max_nan(mx, w.x), bf16x2_max_nan(w.y, bf16x2_max_nan(w.z, w.w)));
+            const uint32_t vm = bf16x2_max_nan(bf16x2_max_nan(w.x, w.y), bf16x2_max_nan(w.z, w.w));
+            if (FEAT) vmax[i] = vm;
+            mx = bf16x2_max_nan(mx, vm);
         }
         cm = fmax_nan(bf16_lo(mx), bf16_hi(mx));
     } else {
@@ -209,8 +213,10 @@ __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lan
 #pragma unroll
         for (int i = 0; i < kVPL; ++i) {
             const uint4 w = tile[lane + 32 * i];
-            cm = fmax_nan(fmax_nan(cm, __uint_as_float(w.x)),
-                          fmax_nan(__uint_as_float(w.y), fmax_nan(__uint_as_float(w.z), __uint_as_float(w.w))));
+            const float vm = fmax_nan(fmax_nan(__uint_as_float(w.x), __uint_as_float(w.y)),
+                                      fmax_nan(__uint_as_float(w.z), __uint_as_float(w.w)));
+            if (FEAT) vmax[i] = __float_as_uint(vm);
+            cm = fmax_nan(cm, vm);
         }
     }
     if (cm > st.m) {
@@ -273,6 +279,78 @@ __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lan
     return cm;
 }
 
+// The warp's five largest clamped entries of the piece so far, t[0] >= ... >=
+// t[4] (warp-uniform, with multiplicity), updated with a (full, padded) tile;
+// vmax holds the maxima of the lane's vectors.  Only entries above t[4] change
+// the list (an entry equal to t[4] changes none of its values); on the
+// piece's first tile the list is empty and the candidates are the entries at
+// or above the fifth largest vector maximum of the warp (five entries reach
+// it, so no smaller entry is in the list).  The vectors holding candidates are
+// visited one at a time, every lane reading the visited vector from shared
+// memory, so the list stays identical in all lanes.
+template <int DT>
+__device__ __forceinline__ void top5_tile(const uint4 *tile, int lane, const uint32_t (&vmax)[kVPL], float (&t)[5]) {
+    constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
+    float vm[kVPL];
+#pragma unroll
+    for (int i = 0; i < kVPL; ++i)
+        vm[i] = (DT == SDD_BF16) ? fmaxf(bf16_lo(vmax[i]), bf16_hi(vmax[i])) : __uint_as_float(vmax[i]);
+    const bool first = t[0] == -INFINITY;
+    float thr = t[4];
+    if (first) {
+        // the fifth largest vector maximum of the warp (the lane's largest first)
+        float c[kVPL];
+#pragma unroll
+        for (int i = 0; i < kVPL; ++i) c[i] = vm[i];
+#pragma unroll 1
+        for (int k = 0; k < 5; ++k) {
+            float lm = c[0];
+#pragma unroll
+            for (int i = 1; i < kVPL; ++i) lm = fmaxf(lm, c[i]);
+            asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(thr) : "f"(lm));
+            const int L = __ffs(__ballot_sync(0xFFFFFFFFu, lm == thr)) - 1;
+            if (lane == L) {
+                bool done = false;
+#pragma unroll
+                for (int i = 0; i < kVPL; ++i)
+                    if (!done && c[i] == thr) {
+                        c[i] = -INFINITY;
+                        done = true;
+                    }
+            }
+        }
+    }
+    uint32_t vmask = 0;   // the lane's vectors holding candidates
+#pragma unroll
+    for (int i = 0; i < kVPL; ++i)
+        if (first ? vm[i] >= thr : vm[i] > thr) vmask |= 1u << i;
+#pragma unroll 1
+    for (int guard = 0; guard < 32 * kVPL; ++guard) {
+        const unsigned who = __ballot_sync(0xFFFFFFFFu, vmask != 0);
+        if (!who) break;
+        const int L = __ffs(who) - 1;
+        int iv = 0;
+        if (lane == L) {
+            iv = __ffs(vmask) - 1;
+            vmask &= vmask - 1;
+        }
+        iv = __shfl_sync(0xFFFFFFFFu, iv, L);
+        const uint4 w = clamp_vec<DT>(tile[L + 32 * iv]);
+#pragma unroll
+        for (int e = 0; e < EPV; ++e) {
+            float z = vec_elem<DT>(w, e);
+            if (z > t[4]) {
+#pragma unroll
+                for (int k = 0; k < 5; ++k) {   // insert z into the descending list
+                    const float hi = fmaxf(t[k], z), lo = fminf(t[k], z);
+                    t[k] = hi;
+                    z = lo;
+                }
+            }
+        }
+    }
+}
+
 // Drafted token of global row r, if the row has one (load issued, not waited on).
 struct RowTok {
     int t;
@@ -299,7 +377,9 @@ __device__ __forceinline__ float token_logit(const ScanParams &p, int64_t r, Row
     return fmax_nan(logit_at<DT>(row_base(p, r), x.t), clamp_floor());
 }
 
-template <int DT>
+// FEAT: also the five largest logits of every drafter row piece (extended
+// features); the kernel without it is unchanged.
+template <int DT, bool FEAT>
 __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant__ ScanParams p) {
     extern __shared__ __align__(128) unsigned char smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -356,6 +436,7 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
     float gA = token_logit<DT>(p, cc.r, tokA);
 
     SoftState st = soft_identity();
+    float top[5];          // FEAT: the warp's five largest entries of the piece (drafter rows)
     float s_hi = 0.f, s_lo = 0.f;   // the lane's exp-sum as an fp32 pair
     bool in_piece = false;
     bool ent = false;      // warp-uniform: drafter row (entropy accumulator, clamped entries)
@@ -371,6 +452,10 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
         const int n = static_cast<int>(min(static_cast<int64_t>(min(kTileVec, p.RV - cc.k)), v1 - cc.v));
         if (!in_piece) {
             st = soft_identity();
+            if (FEAT) {
+#pragma unroll
+                for (int k = 0; k < 5; ++k) top[k] = -INFINITY;
+            }
             s_hi = 0.f;
             s_lo = 0.f;
             int gi, j, b;
@@ -399,8 +484,10 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
         uint4 *tile = reinterpret_cast<uint4 *>(ring + slot * kTileBytes);
         const bool row_end = (cc.k + n == p.RV);
         if (n < kTileVec || (row_end && tail)) pad_tile<DT>(tile, n, lane, row_end, tail);
-        const float cm = ent ? process_tile<DT, true>(tile, cc.k, lane, st, s_hi, s_lo)
-                             : process_tile<DT, false>(tile, cc.k, lane, st, s_hi, s_lo);
+        uint32_t vmax[kVPL];
+        const float cm = ent ? process_tile<DT, true, FEAT>(tile, cc.k, lane, st, s_hi, s_lo, vmax)
+                             : process_tile<DT, false, false>(tile, cc.k, lane, st, s_hi, s_lo, vmax);
+        if (FEAT && ent && __any_sync(0xFFFFFFFFu, cm > top[4])) top5_tile<DT>(tile, lane, vmax, top);
         if (rank_on) {
             const bool want = cm >= g;
             if (__any_sync(0xFFFFFFFFu, want)) {
@@ -432,6 +519,13 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
             st.sh = s_hi;
             st.sl = s_lo;
             const SoftState red = soft_warp_reduce(st);
+            if (FEAT && ent && lane == 0) {
+                FeatPartial fp;
+#pragma unroll
+                for (int k = 0; k < 5; ++k) fp.top[k] = top[k];
+                fp.pad[0] = fp.pad[1] = fp.pad[2] = 0.f;
+                p.feat[cc.r + gw] = fp;
+            }
             if (lane == 0) {
                 Partial pt;
                 pt.m = red.m;
@@ -463,22 +557,28 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
 
 int scan_max_ctas_per_sm() {
     int n = 0;
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, scan_kernel<SDD_BF16>, kThreads, kScanSmem);
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, scan_kernel<SDD_BF16, false>, kThreads, kScanSmem);
     return n;
 }
 
 // Opt both instantiations in to their dynamic shared memory on the current device.
 cudaError_t scan_prepare_device() {
-    cudaError_t e = cudaFuncSetAttribute(scan_kernel<SDD_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize, kScanSmem);
-    if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(scan_kernel<SDD_F32>, cudaFuncAttributeMaxDynamicSharedMemorySize, kScanSmem);
+    void (*const kernels[])(ScanParams) = {scan_kernel<SDD_BF16, false>, scan_kernel<SDD_F32, false>,
+                                           scan_kernel<SDD_BF16, true>, scan_kernel<SDD_F32, true>};
+    for (auto k : kernels) {
+        const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kScanSmem);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 // The launch overhead of the streaming grid overlaps the tail of the work
 // ahead of it in the stream (the kernel waits for that work to complete).
 cudaError_t launch_scan(const ScanParams &p, int grid, cudaStream_t stream) {
-    return launch_dependent(p.dtype == SDD_BF16 ? scan_kernel<SDD_BF16> : scan_kernel<SDD_F32>, dim3(grid),
-                            dim3(kThreads), kScanSmem, stream, p);
+    const bool bf = p.dtype == SDD_BF16, feat = p.feat != nullptr;
+    void (*const k)(ScanParams) = feat ? (bf ? scan_kernel<SDD_BF16, true> : scan_kernel<SDD_F32, true>)
+                                       : (bf ? scan_kernel<SDD_BF16, false> : scan_kernel<SDD_F32, false>);
+    return launch_dependent(k, dim3(grid), dim3(kThreads), kScanSmem, stream, p);
 }
 
 }  // namespace sdd

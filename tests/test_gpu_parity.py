@@ -381,3 +381,45 @@ def test_block_round_periodic_vs_oracle(sdd, round_):
             L, tok, _ = ob.strict[b]
             assert cn[b] == L + 1 and np.array_equal(ct[b], tok)
     assert tally.flagged_mismatch == 0
+
+
+# ---------------------------------------------------------------------------
+# extended features (App. A.7): probability margin and top-5 mass
+# ---------------------------------------------------------------------------
+
+def _check_features(sdd, z_d, x, dtype):
+    base = sdd.confidence(z_d, x)
+    out = sdd.confidence(z_d, x, features=True)
+    torch.cuda.synchronize()
+    for f in ("q", "logq", "maxprob", "lse", "entropy", "argmax"):   # the feature pass changes nothing else
+        torch.testing.assert_close(getattr(out, f), getattr(base, f), rtol=0, atol=0, equal_nan=True, msg=f)
+    mg, t5 = orc.row_features(host(z_d.contiguous() if z_d.is_contiguous() else z_d))
+    p1 = orc.row_stats(host(z_d)).maxprob
+    # margin = p1 - p2 cancels: hold it to the tolerance of p1
+    g = out.margin.cpu().double().numpy()
+    both = np.isnan(g) & np.isnan(mg)
+    assert (np.isnan(g) == np.isnan(mg)).all()
+    err = np.abs(g - mg)[~both]
+    assert (err <= (2e-3 if dtype == torch.bfloat16 else 1e-5) * np.abs(p1[~both]) + 1e-7).all(), err.max()
+    assert_close_stats("top5", out.top5, t5, dtype)
+
+
+@pytest.mark.parametrize("B,gamma,V", [(4, 16, 50000), (3, 5, 151936), (2, 33, 4096), (8, 3, 17)])
+def test_features_bf16_vs_oracle(sdd, B, gamma, V):
+    blk = synth.make_block("c3", device="cpu", B=B, gamma=gamma, V=V)
+    z_d, _, x = _to_dev(blk)
+    z_d = z_d.clone()
+    z_d[0, 0, :] = z_d[0, 0].max()                 # a row of ties: margin 0, top5 = 5 / V
+    z_d[0, 1, 5:] = float("-inf")                  # five finite entries
+    if gamma > 2:
+        z_d[0, 2, 3] = float("nan")                # no distribution
+    if V % 8:
+        z_d = _padded(z_d, (V + 7) // 8 * 8)       # 16-byte row stride
+    _check_features(sdd, z_d, x, torch.bfloat16)
+
+
+def test_features_fp32_padded_rows(sdd):
+    blk = synth.make_block("tiny", device="cpu", B=3, gamma=8, V=4001, dtype=torch.float32)
+    z_d, _, x = _to_dev(blk)
+    z_d = _padded(z_d, 4004)
+    _check_features(sdd, z_d, x, torch.float32)
