@@ -110,6 +110,9 @@ def lib():
     L.orc_survival_mlp.argtypes = [u16p, ctypes.c_int, ctypes.c_int, u16p, f32p, u16p, ctypes.c_double,
                                    ctypes.c_int, f64p]
     L.orc_survival_mlp.restype = None
+    L.orc_scorer_deep.argtypes = [u16p, ctypes.c_int, ctypes.c_int, u16p, f32p, u16p, f32p, u16p, f32p, u16p,
+                                  ctypes.c_double, ctypes.c_int, f64p, f64p, f64p]
+    L.orc_scorer_deep.restype = None
     _lib = L
     return L
 
@@ -371,6 +374,29 @@ def survival_mlp(h_bits, W1_bits, b1, w2_bits, b2: float) -> np.ndarray:
     out = np.zeros(M, np.float64)
     lib().orc_survival_mlp(_ptr(h, ctypes.c_uint16), M, K, _ptr(W1, ctypes.c_uint16), _ptr(b1, ctypes.c_float),
                            _ptr(w2, ctypes.c_uint16), float(b2), N, _ptr(out, ctypes.c_double))
+    return out
+
+
+def scorer_deep(x_bits, W1_bits, b1, W2_bits, b2, W3_bits, b3, w4_bits, b4: float) -> np.ndarray:
+    """fp64 sigmoid(w4 . GELU(W3 a2 + b3) + b4), a2 = bf16(GELU(W2 a1 + b2)),
+    a1 = bf16(GELU(W1 x + b1)) per row of x.  x_bits [M, K], W1 [N, K], W2 and W3
+    [N, N], w4 [N]: raw bf16 bits (uint16); biases fp32 [N]."""
+    u16 = lambda a: np.ascontiguousarray(np.asarray(a, dtype=np.uint16))   # noqa: E731
+    f32 = lambda a: np.ascontiguousarray(np.asarray(a, dtype=np.float32))  # noqa: E731
+    x, W1, W2, W3, w4 = u16(x_bits), u16(W1_bits), u16(W2_bits), u16(W3_bits), u16(w4_bits)
+    b1, b2, b3 = f32(b1), f32(b2), f32(b3)
+    M, K = x.shape
+    N = W1.shape[0]
+    if W1.shape != (N, K) or W2.shape != (N, N) or W3.shape != (N, N) or w4.shape != (N,) or \
+            b1.shape != (N,) or b2.shape != (N,) or b3.shape != (N,):
+        raise ValueError("shape mismatch")
+    out = np.zeros(M, np.float64)
+    s1, s2 = np.zeros(N, np.float64), np.zeros(N, np.float64)
+    u16p, f32p, dp = _P(ctypes.c_uint16), _P(ctypes.c_float), _P(ctypes.c_double)
+    lib().orc_scorer_deep(x.ctypes.data_as(u16p), M, K, W1.ctypes.data_as(u16p), b1.ctypes.data_as(f32p),
+                          W2.ctypes.data_as(u16p), b2.ctypes.data_as(f32p), W3.ctypes.data_as(u16p),
+                          b3.ctypes.data_as(f32p), w4.ctypes.data_as(u16p), float(b4), N, out.ctypes.data_as(dp),
+                          s1.ctypes.data_as(dp), s2.ctypes.data_as(dp))
     return out
 
 

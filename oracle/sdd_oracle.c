@@ -502,3 +502,55 @@ void orc_survival_mlp(const uint16_t *h, int M, int K, const uint16_t *W1, const
         out[m] = 1.0 / (1.0 + exp(-t));
     }
 }
+
+/* ------------------------------------------------------------------------ */
+/* The learned scorer's shape (App. A.7): an MLP K -> N -> N -> N -> 1 with   */
+/* GELU hidden layers, on the concatenated input x = [hidden state ; scalar  */
+/* features] (K = 3584 + 19 in the paper), random-init stand-in weights:     */
+/*   a1 = GELU(W1 x + b1), a2 = GELU(W2 a1 + b2), a3 = GELU(W3 a2 + b3),      */
+/*   s  = sigmoid(w4 . a3 + b4).                                             */
+/* a1 and a2 are rounded to bf16 (round to nearest even, from fp32) before   */
+/* the next layer: the tensor-core path consumes them as bf16 operands, so   */
+/* the oracle takes the same rounding (dropout is a training-time op).  W1  */
+/* is [N, K], W2 and W3 [N, N] (one row per output unit), w4 [N]: bf16 bits. */
+/* Pinned in tests/test_oracle_mlp.py (closed forms of single-path nets,     */
+/* hidden-unit permutation invariance, bf16 rounding of the activations).   */
+/* ------------------------------------------------------------------------ */
+static double orc_round_bf16(double v) {
+    float f = (float)v;
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    if ((u & 0x7F800000u) != 0x7F800000u) { /* finite: round to nearest even */
+        u = (u + 0x7FFFu + ((u >> 16) & 1u)) & 0xFFFF0000u;
+    }
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+static double orc_gelu(double z) { return 0.5 * z * (1.0 + erf(z / sqrt(2.0))); }
+
+void orc_scorer_deep(const uint16_t *x, int M, int K, const uint16_t *W1, const float *b1, const uint16_t *W2,
+                     const float *b2, const uint16_t *W3, const float *b3, const uint16_t *w4, double b4, int N,
+                     double *out, double *a1, double *a2) {
+    /* a1, a2: caller scratch of N doubles each */
+    for (int m = 0; m < M; ++m) {
+        for (int n = 0; n < N; ++n) {
+            double z = (double)b1[n];
+            for (int k = 0; k < K; ++k)
+                z += orc_load(W1, ORC_BF16, (int64_t)n * K + k) * orc_load(x, ORC_BF16, (int64_t)m * K + k);
+            a1[n] = orc_round_bf16(orc_gelu(z));
+        }
+        for (int n = 0; n < N; ++n) {
+            double z = (double)b2[n];
+            for (int k = 0; k < N; ++k) z += orc_load(W2, ORC_BF16, (int64_t)n * N + k) * a1[k];
+            a2[n] = orc_round_bf16(orc_gelu(z));
+        }
+        double t = b4;
+        for (int n = 0; n < N; ++n) {
+            double z = (double)b3[n];
+            for (int k = 0; k < N; ++k) z += orc_load(W3, ORC_BF16, (int64_t)n * N + k) * a2[k];
+            t += orc_load(w4, ORC_BF16, n) * orc_gelu(z);
+        }
+        out[m] = 1.0 / (1.0 + exp(-t));
+    }
+}

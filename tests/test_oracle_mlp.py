@@ -82,3 +82,76 @@ def test_hidden_unit_permutation_invariance(orc):
     np.testing.assert_allclose(a, b, rtol=1e-14, atol=0)
     # and the rows are independent: scoring a subset gives the same values
     np.testing.assert_array_equal(orc.survival_mlp(h[3:5], W1, b1, w2, -0.2), a[3:5])
+
+
+# ---------------------------------------------------------------------------
+# The learned scorer's shape (App. A.7): K -> N -> N -> N -> 1, GELU, with the
+# first two layers' activations rounded to bf16 (the tensor-core operands)
+# ---------------------------------------------------------------------------
+
+def _b(a):
+    return torch.from_numpy(np.asarray(a, np.float32)).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+
+
+def _gelu(z):
+    return 0.5 * z * (1.0 + math.erf(z / math.sqrt(2.0)))
+
+
+def _rbf16(v):
+    return float(torch.tensor(float(v), dtype=torch.float32).to(torch.bfloat16).float())
+
+
+def _zeros(N, K):
+    return np.zeros((N, K), np.float32), np.zeros(N, np.float32)
+
+
+def test_deep_zero_weights_closed_form(orc):
+    N, K = 8, 16
+    W, b = _zeros(N, K)
+    b3 = np.linspace(-1.5, 2.0, N).astype(np.float32)
+    w4 = np.linspace(0.5, -0.5, N).astype(np.float32)
+    x = _b(np.random.default_rng(0).normal(size=(3, K)))
+    s = orc.scorer_deep(x, _b(W), b, _b(np.zeros((N, N))), b, _b(np.zeros((N, N))), b3, _b(w4), 0.25)
+    w4r = np.asarray(torch.from_numpy(w4).to(torch.bfloat16).float())
+    t = 0.25 + sum(float(w4r[n]) * _gelu(float(b3[n])) for n in range(N))
+    np.testing.assert_allclose(s, 1.0 / (1.0 + math.exp(-t)), rtol=1e-14)
+
+
+def test_deep_single_path_closed_form_with_bf16_activations(orc):
+    """One weight per layer: s = sigmoid(e GELU(d r(GELU(c r(GELU(a x_j + beta)))))),
+    r = rounding to bf16; every other unit sees GELU(0) = 0."""
+    N, K, j, i, pu, q = 6, 10, 3, 2, 4, 1
+    a, beta, c, d, e = 1.25, 0.3, -0.75, 1.5, 2.0
+    W1, z = _zeros(N, K)
+    W1[i, j] = a
+    b1 = z.copy()
+    b1[i] = beta
+    W2 = np.zeros((N, N), np.float32)
+    W2[pu, i] = c
+    W3 = np.zeros((N, N), np.float32)
+    W3[q, pu] = d
+    w4 = np.zeros(N, np.float32)
+    w4[q] = e
+    x = np.zeros((2, K), np.float32)
+    x[0, j], x[1, j] = 0.6875, -2.5
+    s = orc.scorer_deep(_b(x), _b(W1), b1, _b(W2), z, _b(W3), z, _b(w4), 0.0)
+    for m in range(2):
+        a1 = _rbf16(_gelu(a * x[m, j] + float(np.float32(beta))))
+        a2 = _rbf16(_gelu(c * a1))
+        t = e * _gelu(d * a2)
+        assert s[m] == pytest.approx(1.0 / (1.0 + math.exp(-t)), rel=1e-14)
+        unrounded = 1.0 / (1.0 + math.exp(-e * _gelu(d * _gelu(c * _gelu(a * x[m, j] + float(np.float32(beta)))))))
+        assert abs(s[m] - unrounded) > 1e-9   # the rounding is really applied
+
+
+def test_deep_hidden_unit_permutation_invariance(orc):
+    rng = np.random.default_rng(7)
+    N, K, M = 16, 40, 5
+    x = _b(rng.normal(size=(M, K)))
+    W1, W2, W3 = (rng.normal(size=s) * 0.3 for s in ((N, K), (N, N), (N, N)))
+    b1, b2, b3 = (rng.normal(size=N).astype(np.float32) * 0.2 for _ in range(3))
+    w4 = rng.normal(size=N) * 0.2
+    s0 = orc.scorer_deep(x, _b(W1), b1, _b(W2), b2, _b(W3), b3, _b(w4), -0.1)
+    p1, p2, p3 = rng.permutation(N), rng.permutation(N), rng.permutation(N)
+    s1 = orc.scorer_deep(x, _b(W1[p1]), b1[p1], _b(W2[p2][:, p1]), b2[p2], _b(W3[p3][:, p2]), b3[p3], _b(w4[p3]), -0.1)
+    np.testing.assert_allclose(s1, s0, rtol=1e-12)
