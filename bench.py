@@ -20,6 +20,7 @@ Other rows of the path, one JSON line each (not the fused-round contract line):
   python bench.py --component mlp [--steps K]   the survival scorer alone (K launches)
   python bench.py --component loop [--steps R]  the decode-loop workload (R rounds, default 64)
   python bench.py --component features          drafter confidence with / without the extended features
+  python bench.py --component scorer [--steps K] the deep scorer (K calls)
 """
 from __future__ import annotations
 
@@ -430,6 +431,77 @@ def run_component_mlp(args):
     return 0
 
 
+def run_component_scorer(args):
+    """The deep scorer (learned scorer's shape, App. A.7: (3584 + 19) -> 256 ->
+    256 -> 256 -> 1) on the decode-loop batch (4096 positions), device time from
+    CUDA-graph replays of 16 calls (two launches each) over 8 rotating
+    hidden-state buffers (8 x 29 MB > L2)."""
+    import torch
+    import paper_2608_14787_gb300 as sdd
+    from paper_2608_14787_gb300 import build as sdd_build
+    from paper_2608_14787_gb300 import synth
+    sdd_build.build()
+    sdd.load()
+    M, Kh, N = 128 * 32, synth.HIDDEN, 256
+    w = synth.make_scorer_deep(device="cuda", hidden=Kh)
+    hs = [synth.make_hidden(M, device="cuda", round_=r) for r in range(8)]
+    fs = [synth.make_features(M, device="cuda", round_=r) for r in range(8)]
+    act = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+    out = torch.empty(M, device="cuda")
+    status = sdd.new_status(torch.device("cuda"))
+    for i in range(max(args.warmup, 3)):
+        sdd.scorer_deep(hs[i % 8], fs[i % 8], *w, act=act, out=out, status=status)
+    torch.cuda.synchronize()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=side):
+        for i in range(16):
+            sdd.scorer_deep(hs[i % 8], fs[i % 8], *w, act=act, out=out, status=status)
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    reps = max(1, args.steps // 16)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(None) as clk:
+        e0.record()
+        for _ in range(reps):
+            g.replay()
+        e1.record()
+        torch.cuda.synchronize()
+    t = e0.elapsed_time(e1) / (reps * 16) / 1e3
+    K1 = Kh + N
+    flops = 2.0 * M * (K1 * N + 2 * N * N + N)
+    nbytes = M * K1 * 2 + N * K1 * 2 + 2 * N * N * 2 + 2 * M * N * 2 + M * 4
+    tpk, tkind = _peak_tflops()
+    hbm, hkind = _peaks()
+    cpu = None
+    if not args.no_cpu_baseline:
+        import oracle as orc
+        rows = 128
+        x = torch.cat([hs[0][:rows], fs[0][:rows]], dim=-1)
+        bits = synth.bf16_bits
+        W1, b1, W2, b2, W3, b3, w4, b4 = w
+        t0 = time.perf_counter()
+        orc.scorer_deep(bits(x), bits(W1), b1.cpu().numpy(), bits(W2), b2.cpu().numpy(), bits(W3), b3.cpu().numpy(),
+                        bits(w4), b4)
+        dt = time.perf_counter() - t0
+        cpu = {"value": rows / dt, "unit": "positions/s", "cores": 1, "kind": "oracle",
+               "sample": f"{rows} of the {M} positions, fp64 loops, single thread ({dt:.1f} s)"}
+    line = {
+        "component": "NEXT-2 deep scorer (sdd_scorer_deep)", "metric": "positions scored/s", "unit": "positions/s",
+        "value": M / t, "us_per_call": t * 1e6,
+        "config": {"M": M, "K": f"{Kh} + 256 (19 features, zero padded)", "layers": "3840 -> 256 -> 256 -> 256 -> 1",
+                   "dtype": "bf16 operands, fp32 accumulation"},
+        "roofline": {"bound": "hbm", "achieved_gbs": nbytes / t / 1e9, "peak_gbs": hbm, "frac_hbm": nbytes / t / 1e9 / hbm,
+                     "achieved_tflops": flops / t / 1e12, "peak_tflops": tpk, "frac_tensor": flops / t / 1e12 / tpk,
+                     "bytes": nbytes, "flops": flops, "peak_source": f"{hkind} hbm_gbs / {tkind} bf16_tflops"},
+        "cpu_baseline": cpu, "clocks": clk.summary(), "device_status": int(status.item()),
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_component_features(args):
     """Drafter confidence with and without the extended features (App. A.7:
     probability margin, top-5 mass) on the drafter half of the c3 workload
@@ -536,7 +608,7 @@ def main():
     ap.add_argument("--sets", type=int, default=3, help="rotating input sets (3 x 316 MB exceeds L2)")
     ap.add_argument("--traffic", type=float, default=None,
                     help="dram bytes per scan launch from an ncu capture of the current kernel")
-    ap.add_argument("--component", default=None, choices=["mlp", "loop", "features"],
+    ap.add_argument("--component", default=None, choices=["mlp", "loop", "features", "scorer"],
                     help="measure one other row of the path instead of the fused round")
     args = ap.parse_args()
     if args.component == "mlp":
@@ -545,6 +617,8 @@ def main():
         return run_component_loop(args)
     if args.component == "features":
         return run_component_features(args)
+    if args.component == "scorer":
+        return run_component_scorer(args)
     if args.traffic is None and args.workload == "c3":
         args.traffic = SCAN_TRAFFIC_C3
     if args.warmup < 3:

@@ -307,6 +307,35 @@ SDD_API sdd_status_t sdd_survival_mlp(const void *h, int M, int K, const void *W
                                       float b2, float *s, int32_t *status, sdd_stream_t stream);
 
 /*
+ * sdd_scorer_deep -- the learned scorer's shape of App. A.7 (K -> 256 -> 256 ->
+ * 256 -> 1, GELU hidden layers; dropout is a training-time op) per draft
+ * position, with stand-in weights, on the concatenated input
+ * x[m] = [h[m] ; f[m]] (drafter hidden state and scalar features):
+ *   a1 = bf16(GELU(W1 x + b1)),  a2 = bf16(GELU(W2 a1 + b2)),
+ *   s[m] = sigmoid(w4 . GELU(W3 a2 + b3) + b4).
+ * a1 and a2 are rounded to bf16 (nearest even): the tensor cores take them as
+ * bf16 operands (fp32 accumulation throughout).
+ *   h    [M, Kh] bf16, row-major, 16-byte aligned; Kh a positive multiple of
+ *        SDD_MLP_KSTEP (3584 in the paper).
+ *   f    [M, SDD_MLP_HIDDEN] bf16: the scalar features in the first columns
+ *        (19 in the paper), zeros after them.
+ *   W1   [SDD_MLP_HIDDEN, Kh + SDD_MLP_HIDDEN] bf16 (columns Kh.. weigh f; the
+ *        columns of f's zero padding should be zero too).
+ *   W2, W3 [SDD_MLP_HIDDEN, SDD_MLP_HIDDEN] bf16 (one row per output unit);
+ *   b1, b2, b3 [SDD_MLP_HIDDEN] fp32; w4 [SDD_MLP_HIDDEN] bf16; b4 a host scalar.
+ *   act  [M, SDD_MLP_HIDDEN] bf16 caller scratch (receives a1), 16-byte aligned.
+ *   s    [M] fp32 output.
+ * Two launches on the stream: the first layer (K split over a 4-CTA cluster as
+ * in sdd_survival_mlp), then layers 2 and 3 and the head, one CTA per 128
+ * positions with a2 kept in shared memory.  Needs an sm_10x device; a bounded
+ * wait that gives up sets SDD_DEV_TIMEOUT in *status.
+ */
+SDD_API sdd_status_t sdd_scorer_deep(const void *h, int Kh, const void *f, int M, const void *W1, const float *b1,
+                                     const void *W2, const float *b2, const void *W3, const float *b3,
+                                     const void *w4, float b4, void *act, float *s, int32_t *status,
+                                     sdd_stream_t stream);
+
+/*
  * sdd_confidence_noalloc -- sdd_confidence without a workspace, for callers
  * that cannot allocate device memory where they need the statistics: code
  * running inside CUDA stream capture (where cudaMalloc is not allowed),

@@ -92,6 +92,8 @@ def load(path: str | None = None):
     L.sdd_confidence_noalloc.restype = I
     L.sdd_survival_mlp.argtypes = [VP, I, I, VP, VP, VP, ctypes.c_float, VP, VP, VP]
     L.sdd_survival_mlp.restype = I
+    L.sdd_scorer_deep.argtypes = [VP, I, VP, I, VP, VP, VP, VP, VP, VP, VP, ctypes.c_float, VP, VP, VP, VP]
+    L.sdd_scorer_deep.restype = I
     for fn in ("sdd_block", "sdd_block_scan", "sdd_block_decide"):
         getattr(L, fn).argtypes = [ctypes.POINTER(BlockArgs), VP]
     for fn in ("sdd_workspace_size", "sdd_confidence", "sdd_confidence_features", "sdd_schedule_prefix",
@@ -357,6 +359,27 @@ def survival_mlp(h, W1, b1, w2, b2: float, *, status=None, stream=None, out=None
     s = torch.empty(M, dtype=torch.float32, device=h.device) if out is None else out
     _check(load().sdd_survival_mlp(_p(h2), M, K, _p(W1), _p(b1), _p(w2), float(b2), _p(s), _p(status),
                                    _stream(stream)), "sdd_survival_mlp")
+    return s.reshape(lead)
+
+
+def scorer_deep(h, f, W1, b1, W2, b2, W3, b3, w4, b4, *, act=None, status=None, stream=None, out=None):
+    """sdd_scorer_deep: h [..., Kh] bf16, f [..., 256] bf16 (features, zero padded),
+    W1 [256, Kh + 256], W2 / W3 [256, 256], w4 [256] bf16; b1..b3 fp32 [256], b4 float.
+    Returns s with h's leading shape."""
+    lead = h.shape[:-1]
+    Kh = h.shape[-1]
+    h2 = h.reshape(-1, Kh).contiguous()
+    f2 = f.reshape(-1, f.shape[-1]).contiguous()
+    M = h2.shape[0]
+    if f2.shape != (M, MLP_HIDDEN) or W1.shape != (MLP_HIDDEN, Kh + MLP_HIDDEN):
+        raise ValueError("f must be [M, 256] and W1 [256, Kh + 256]")
+    for t in (W2, W3):
+        if t.shape != (MLP_HIDDEN, MLP_HIDDEN):
+            raise ValueError("W2 and W3 must be [256, 256]")
+    act = torch.empty(M, MLP_HIDDEN, dtype=torch.bfloat16, device=h.device) if act is None else act
+    s = torch.empty(M, dtype=torch.float32, device=h.device) if out is None else out
+    _check(load().sdd_scorer_deep(_p(h2), Kh, _p(f2), M, _p(W1), _p(b1), _p(W2), _p(b2), _p(W3), _p(b3), _p(w4),
+                                  float(b4), _p(act), _p(s), _p(status), _stream(stream)), "sdd_scorer_deep")
     return s.reshape(lead)
 
 

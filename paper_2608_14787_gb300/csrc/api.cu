@@ -574,6 +574,35 @@ sdd_status_t sdd_survival_mlp(const void *h, int M, int K, const void *W1, const
     return SDD_OK;
 }
 
+sdd_status_t sdd_scorer_deep(const void *h, int Kh, const void *f, int M, const void *W1, const float *b1,
+                             const void *W2, const float *b2, const void *W3, const float *b3, const void *w4,
+                             float b4, void *act, float *s, int32_t *status, sdd_stream_t stream) {
+    if (M < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "M = %d < 0", M);
+    if (Kh < SDD_MLP_KSTEP || Kh % SDD_MLP_KSTEP != 0)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "Kh = %d is not a positive multiple of %d", Kh, SDD_MLP_KSTEP);
+    if (M == 0) return SDD_OK;
+    SDD_TRY(check_ptr16(h, "h"));
+    SDD_TRY(check_ptr16(f, "f"));
+    SDD_TRY(check_ptr16(W1, "W1"));
+    SDD_TRY(check_ptr16(W2, "W2"));
+    SDD_TRY(check_ptr16(W3, "W3"));
+    SDD_TRY(check_ptr16(act, "act"));
+    if (!b1 || !b2 || !b3 || !w4 || !s) return fail(SDD_ERR_INVALID_ARGUMENT, "b1, b2, b3, w4 and s must not be NULL");
+    int d = 0;
+    cudaError_t e = cudaGetDevice(&d);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    int major = 0, minor = 0;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, d);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, d);
+    if (major != 10) return fail(SDD_ERR_UNSUPPORTED, "tcgen05 scorer needs an sm_10x device (found sm_%d%d)", major, minor);
+    const char *why = nullptr;
+    e = launch_scorer_deep(h, Kh, f, M, W1, b1, W2, b2, W3, b3, w4, b4, static_cast<uint16_t *>(act), s, status,
+                           reinterpret_cast<cudaStream_t>(stream), &why);
+    if (why) return fail(SDD_ERR_CUDA, "deep scorer: %s", why);
+    if (e != cudaSuccess) return cuda_fail(e, "deep scorer launch");
+    return SDD_OK;
+}
+
 static sdd_status_t block_check(const sdd_block_args *a) {
     if (!a) return fail(SDD_ERR_INVALID_ARGUMENT, "args is NULL");
     SDD_TRY(check_shape(static_cast<sdd_dtype_t>(a->dtype), a->B, a->gamma, a->V, a->row_stride));

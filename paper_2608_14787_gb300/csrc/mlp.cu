@@ -38,10 +38,12 @@ constexpr uint32_t kTmemCols = 256;
 
 struct MlpParams {
     int32_t M, K;
+    int32_t Ka;             // K columns of the first A operand (the rest come from the second)
     const float *b1;        // [256]
-    const uint16_t *w2;     // [256] bf16 bits
+    const uint16_t *w2;     // [256] bf16 bits (head mode)
     float b2;
-    float *out;             // [M]
+    float *out;             // [M] (head mode)
+    uint16_t *act;          // [M, 256] bf16 bits: GELU(W1 x + b1) (activation mode)
     int32_t *status;
 };
 
@@ -119,6 +121,13 @@ __device__ __forceinline__ void st_cluster_v4(uint32_t addr, float a, float b, f
                  : "memory");
 }
 
+// Two fp32 values rounded to bf16 (round to nearest even), packed (a low).
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+    uint32_t d;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(b), "f"(a));
+    return d;
+}
+
 // Row stride (floats) of a partial accumulator dumped to shared memory: a
 // multiple of 4 for 16-byte accesses, 4 mod 32 so that 8 consecutive rows
 // cover all banks.
@@ -132,8 +141,15 @@ constexpr int kAccStride = kMlpN + 4;
 // slot r of CTA q's receive area (distributed shared-memory stores over the
 // idle stage ring); after a second cluster barrier each CTA sums its S slots
 // locally and runs the epilogue.
-template <int S>
+//
+// The A operand is the concatenation [A1 | A2] along K: slices below p.Ka come
+// from tmA, the rest from tmA2 (the scalar features of the deep scorer).
+// HEAD: the epilogue fuses GELU, the w2 dot product and the sigmoid (one
+// float per row); otherwise it writes the layer's activations GELU(z + b1)
+// as bf16 rows of p.act for the next layer.
+template <int S, bool HEAD>
 __global__ void __launch_bounds__(kMlpThreads, 1) mlp_kernel(const __grid_constant__ CUtensorMap tmA,
+                                                            const __grid_constant__ CUtensorMap tmA2,
                                                             const __grid_constant__ CUtensorMap tmB,
                                                             const __grid_constant__ MlpParams p) {
     extern __shared__ unsigned char smem_raw[];
@@ -148,7 +164,7 @@ __global__ void __launch_bounds__(kMlpThreads, 1) mlp_kernel(const __grid_consta
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     for (int n = tid; n < kMlpN; n += kMlpThreads) {
         s_b1[n] = __ldg(p.b1 + n);
-        s_w2[n] = __uint_as_float(static_cast<uint32_t>(__ldg(p.w2 + n)) << 16);
+        s_w2[n] = HEAD ? __uint_as_float(static_cast<uint32_t>(__ldg(p.w2 + n)) << 16) : 0.f;
     }
     const uint32_t rank = (S > 1) ? cluster_rank() : 0u;
     const int m0 = (blockIdx.x / S) * kMlpBM;
@@ -188,8 +204,12 @@ __global__ void __launch_bounds__(kMlpThreads, 1) mlp_kernel(const __grid_consta
             }
             mbar_arrive_expect_tx(&full[s], kStageBytes);
             const uint32_t a = smem_addr(smem + s * kStageBytes);
-            tma_load_2d(a, &tmA, (kt0 + t) * kMlpBK, m0, smem_addr(&full[s]));
-            tma_load_2d(a + kATileBytes, &tmB, (kt0 + t) * kMlpBK, 0, smem_addr(&full[s]));
+            const int k = (kt0 + t) * kMlpBK;
+            if (k < p.Ka)
+                tma_load_2d(a, &tmA, k, m0, smem_addr(&full[s]));
+            else
+                tma_load_2d(a, &tmA2, k - p.Ka, m0, smem_addr(&full[s]));
+            tma_load_2d(a + kATileBytes, &tmB, k, 0, smem_addr(&full[s]));
         }
         // let every issued load land before the ring is reused or the CTA
         // leaves (already true unless a wait gave up): the last load per stage
@@ -262,6 +282,7 @@ __global__ void __launch_bounds__(kMlpThreads, 1) mlp_kernel(const __grid_consta
         constexpr int P = kMlpThreads / R;
         const int lrow = tid / P;
         const int pp = tid % P;
+        const int grow = m0 + static_cast<int>(rank) * R + lrow;
         float t2 = 0.f;
 #pragma unroll 4
         for (int ch = pp; ch < kMlpN / 4; ch += P) {
@@ -276,22 +297,215 @@ __global__ void __launch_bounds__(kMlpThreads, 1) mlp_kernel(const __grid_consta
                 z.w += v.w;
             }
             const float zz[4] = {z.x, z.y, z.z, z.w};
+            float gg[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 const int n = c + e;
                 const float u = zz[e] + s_b1[n];
-                const float g = 0.5f * u * (1.f + erff(u * 0.70710678118654752f));
-                t2 = fmaf(s_w2[n], g, t2);
+                gg[e] = 0.5f * u * (1.f + erff(u * 0.70710678118654752f));
+                if (HEAD) t2 = fmaf(s_w2[n], gg[e], t2);
+            }
+            if (!HEAD && ok && grow < p.M) {
+                // four bf16 activations (round to nearest even) in one 8-byte store
+                const uint32_t lo = pack_bf16x2(gg[0], gg[1]), hi = pack_bf16x2(gg[2], gg[3]);
+                *reinterpret_cast<uint2 *>(p.act + static_cast<int64_t>(grow) * kMlpN + c) = make_uint2(lo, hi);
             }
         }
-        for (int off = 1; off < P; off <<= 1) t2 += __shfl_xor_sync(0xFFFFFFFFu, t2, off);
-        const int grow = m0 + static_cast<int>(rank) * R + lrow;
-        if (tid % P == 0 && ok && grow < p.M) p.out[grow] = 1.f / (1.f + expf(-(t2 + p.b2)));
+        if (HEAD) {
+            for (int off = 1; off < P; off <<= 1) t2 += __shfl_xor_sync(0xFFFFFFFFu, t2, off);
+            if (tid % P == 0 && ok && grow < p.M) p.out[grow] = 1.f / (1.f + expf(-(t2 + p.b2)));
+        }
     }
     __syncthreads();
     if (tid == 0 && s_abort) status_or(p.status, SDD_DEV_TIMEOUT);
     if (warp == 0)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// Layers 2 and 3 and the head of the deep scorer (K -> 256 -> 256 -> 256 -> 1):
+// one CTA per 128-row tile.  The tile's first-layer activations (128 x 256
+// bf16, four 64-column slices with the 128-byte swizzle) and W2 (256 x 256)
+// arrive by TMA; z2 = W2 a1 goes to TMEM columns 0..255; the epilogue writes
+// a2 = bf16(GELU(z2 + b2)) back over a1 in the same swizzled K-major layout
+// (16-byte unit u of row r at r * 128 + (u ^ (r % 8)) * 16 within a slice)
+// while W3 replaces W2; z3 = W3 a2 goes to TMEM columns 256..511; the last
+// epilogue computes sigmoid(w4 . GELU(z3 + b3) + b4) per row.
+// ---------------------------------------------------------------------------
+constexpr uint32_t kTailASlice = kMlpBM * kMlpBK * 2;      // 16 KiB: 128 rows x 64 bf16
+constexpr uint32_t kTailBSlice = kMlpN * kMlpBK * 2;       // 32 KiB: 256 rows x 64 bf16
+constexpr int kTailSlices = kMlpN / kMlpBK;                // 4
+constexpr uint32_t kTailA = kTailSlices * kTailASlice;     // 64 KiB
+constexpr uint32_t kTailB = kTailSlices * kTailBSlice;     // 128 KiB
+constexpr int kTailSmem = kTailA + kTailB + 1024 + 256;
+constexpr uint32_t kTailTmemCols = 512;
+constexpr int kTailThreads = 512;   // 16 warps: four per TMEM lane quarter, 64 columns each
+
+struct TailParams {
+    int32_t M;
+    const float *b2, *b3;      // [256]
+    const uint16_t *w4;        // [256] bf16 bits
+    float b4;
+    float *out;                // [M]
+    int32_t *status;
+};
+
+__global__ void __launch_bounds__(kTailThreads, 1) mlp_tail_kernel(const __grid_constant__ CUtensorMap tmAct,
+                                                                 const __grid_constant__ CUtensorMap tmW2,
+                                                                 const __grid_constant__ CUtensorMap tmW3,
+                                                                 const __grid_constant__ TailParams p) {
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *smem = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                            ~static_cast<uintptr_t>(1023));
+    unsigned char *bufA = smem, *bufB = smem + kTailA;
+    uint64_t *bar = reinterpret_cast<uint64_t *>(smem + kTailA + kTailB);
+    uint64_t *fullA = bar, *fullW2 = bar + 1, *fullW3 = bar + 2, *mma2 = bar + 3, *mma3 = bar + 4;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bar + 5);
+    __shared__ int s_abort;
+    __shared__ float s_b2[kMlpN], s_b3[kMlpN], s_w4[kMlpN];
+    __shared__ float s_part[3][kMlpBM];   // column parts 1..3 of each row's dot product
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int m0 = blockIdx.x * kMlpBM;
+    for (int n = tid; n < kMlpN; n += kTailThreads) {
+        s_b2[n] = __ldg(p.b2 + n);
+        s_b3[n] = __ldg(p.b3 + n);
+        s_w4[n] = __uint_as_float(static_cast<uint32_t>(__ldg(p.w4 + n)) << 16);
+    }
+    if (tid == 0) {
+        for (int i = 0; i < 5; ++i) mbar_init(&bar[i], 1);
+        fence_mbar_init();
+        s_abort = 0;
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(tmem_slot)),
+                     "r"(kTailTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (tid == 0) {
+        mbar_arrive_expect_tx(fullA, kTailA);
+        for (int c = 0; c < kTailSlices; ++c)
+            tma_load_2d(smem_addr(bufA + c * kTailASlice), &tmAct, c * kMlpBK, m0, smem_addr(fullA));
+        mbar_arrive_expect_tx(fullW2, kTailB);
+        for (int c = 0; c < kTailSlices; ++c)
+            tma_load_2d(smem_addr(bufB + c * kTailBSlice), &tmW2, c * kMlpBK, 0, smem_addr(fullW2));
+    } else if (warp == 1 && lane == 0) {
+        const bool okA = mbar_wait_bounded(fullA, 0u, kWaitPolls), okB = mbar_wait_bounded(fullW2, 0u, kWaitPolls);
+        if (okA && okB) {
+            tc_fence_after();
+#pragma unroll 1
+            for (int c = 0; c < kTailSlices; ++c)
+#pragma unroll
+                for (int kk = 0; kk < kMlpBK / 16; ++kk)
+                    umma_f16(tmem, umma_desc_sw128(smem_addr(bufA + c * kTailASlice) + kk * 32),
+                             umma_desc_sw128(smem_addr(bufB + c * kTailBSlice) + kk * 32), (c | kk) != 0 ? 1u : 0u);
+        } else {
+            s_abort = 1;
+        }
+        umma_commit(smem_addr(mma2));   // (arrives at once when nothing was issued)
+    }
+    __syncwarp();
+
+    // layer-2 epilogue: warp w reads TMEM lanes 32 (w % 4) .. + 31 (tile rows),
+    // columns 64 (w / 4) .. + 63
+    const int quarter = warp & 3, part = warp >> 2;
+    const int row = quarter * 32 + lane;
+    const uint32_t tlane = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+    bool ok = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(mma2, 0u, kWaitPolls));
+    tc_fence_after();
+    if (tid == 0 && ok) {
+        // W2 has been read: W3 takes its place
+        mbar_arrive_expect_tx(fullW3, kTailB);
+        for (int c = 0; c < kTailSlices; ++c)
+            tma_load_2d(smem_addr(bufB + c * kTailBSlice), &tmW3, c * kMlpBK, 0, smem_addr(fullW3));
+    }
+#pragma unroll 1
+    for (int cb = 0; cb < 2; ++cb) {
+        const int n0 = part * 64 + cb * 32;
+        uint32_t v[32];
+        if (ok) {
+            tmem_ld32(tlane + n0, v);
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = 0u;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {   // four 16-byte units of 8 activations
+            uint32_t w[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                float g[2];
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int j = u * 8 + q * 2 + e;
+                    const float z = __uint_as_float(v[j]) + s_b2[n0 + j];
+                    g[e] = 0.5f * z * (1.f + erff(z * 0.70710678118654752f));
+                }
+                w[q] = pack_bf16x2(g[0], g[1]);
+            }
+            const int n = n0 + u * 8;                       // first column of the unit
+            const int slice = n / kMlpBK, unit = (n % kMlpBK) / 8;
+            unsigned char *dst = bufA + slice * kTailASlice + row * 128 + ((unit ^ (row & 7)) * 16);
+            *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+    }
+    fence_proxy_async_smem();   // the generic writes of a2, before the tensor cores read them
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+
+    if (warp == 1 && lane == 0) {
+        // (W3 was requested iff ok; its load has landed before the CTA can leave)
+        if (ok && mbar_wait_bounded(fullW3, 0u, kWaitPolls)) {
+            tc_fence_after();
+#pragma unroll 1
+            for (int c = 0; c < kTailSlices; ++c)
+#pragma unroll
+                for (int kk = 0; kk < kMlpBK / 16; ++kk)
+                    umma_f16(tmem + 256, umma_desc_sw128(smem_addr(bufA + c * kTailASlice) + kk * 32),
+                             umma_desc_sw128(smem_addr(bufB + c * kTailBSlice) + kk * 32), (c | kk) != 0 ? 1u : 0u);
+        } else {
+            s_abort = 1;
+        }
+        umma_commit(smem_addr(mma3));
+    }
+    __syncwarp();
+
+    // layer-3 epilogue and head: each thread's dot product over its 64
+    // columns, the four parts of a row added through shared memory
+    ok = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(mma3, 0u, kWaitPolls)) && ok;
+    tc_fence_after();
+    float t = 0.f;
+#pragma unroll 1
+    for (int cb = 0; cb < 2; ++cb) {
+        const int n0 = part * 64 + cb * 32;
+        uint32_t v[32];
+        if (ok) {
+            tmem_ld32(tlane + 256 + n0, v);
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = 0u;
+        }
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            const float z = __uint_as_float(v[j]) + s_b3[n0 + j];
+            t = fmaf(s_w4[n0 + j], 0.5f * z * (1.f + erff(z * 0.70710678118654752f)), t);
+        }
+    }
+    if (part > 0) s_part[part - 1][row] = t;
+    tc_fence_before();
+    __syncthreads();
+    if (part == 0 && ok && m0 + row < p.M)
+        p.out[m0 + row] = 1.f / (1.f + expf(-(((t + s_part[0][row]) + s_part[1][row]) + s_part[2][row] + p.b4)));
+    if (tid == 0 && (s_abort || !ok)) status_or(p.status, SDD_DEV_TIMEOUT);
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTailTmemCols)
+                     : "memory");
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -351,41 +565,49 @@ MapCache g_maps;
 constexpr int kMaxDevices = 64;
 std::atomic<int> g_attr_ready[kMaxDevices];
 
-}  // namespace
-
-cudaError_t launch_mlp(const void *h, int M, int K, const void *W1, const float *b1, const void *w2, float b2,
-                       float *out, int32_t *status, cudaStream_t stream, const char **why) {
-    *why = nullptr;
-    if (M == 0) return cudaSuccess;
-    CUtensorMap tmA, tmB;
-    if (!g_maps.get(&tmA, h, M, K, kMlpBM) || !g_maps.get(&tmB, W1, kMlpN, K, kMlpN)) {
-        *why = "cuTensorMapEncodeTiled failed";
-        return cudaErrorInvalidValue;
-    }
+// Per-device opt-in of every kernel here to its dynamic shared memory.
+cudaError_t mlp_prepare() {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= kMaxDevices) {
-        *why = "device ordinal out of range";
-        return cudaErrorInvalidDevice;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    if (g_attr_ready[dev].load(std::memory_order_acquire)) return cudaSuccess;
+    for (auto fn : {mlp_kernel<1, true>, mlp_kernel<2, true>, mlp_kernel<4, true>, mlp_kernel<1, false>,
+                    mlp_kernel<2, false>, mlp_kernel<4, false>}) {
+        e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kMlpSmem);
+        if (e != cudaSuccess) return e;
     }
-    if (!g_attr_ready[dev].load(std::memory_order_acquire)) {
-        for (auto fn : {mlp_kernel<1>, mlp_kernel<2>, mlp_kernel<4>}) {
-            e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kMlpSmem);
-            if (e != cudaSuccess) return e;
-        }
-        g_attr_ready[dev].store(1, std::memory_order_release);
+    e = cudaFuncSetAttribute(mlp_tail_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kTailSmem);
+    if (e != cudaSuccess) return e;
+    g_attr_ready[dev].store(1, std::memory_order_release);
+    return cudaSuccess;
+}
+
+// The first layer: A = [A1 | A2] (A2 may be absent: Ka = K), W1 [256, K].
+// head: fused GELU / w2 / sigmoid into out; else bf16 activations into act.
+cudaError_t launch_layer1(const void *a1, int Ka, const void *a2, int M, int K, const void *W1, const float *b1,
+                          const void *w2, float b2, float *out, uint16_t *act, bool head, int32_t *status,
+                          cudaStream_t stream, const char **why) {
+    CUtensorMap tmA, tmA2, tmB;
+    if (!g_maps.get(&tmA, a1, M, Ka, kMlpBM) || !g_maps.get(&tmB, W1, kMlpN, K, kMlpN) ||
+        !g_maps.get(&tmA2, a2 ? a2 : a1, M, a2 ? K - Ka : Ka, kMlpBM)) {
+        *why = "cuTensorMapEncodeTiled failed";
+        return cudaErrorInvalidValue;
     }
+    cudaError_t e = mlp_prepare();
+    if (e != cudaSuccess) return e;
     // split K four ways when the slices divide evenly (more SMs, no reloads)
     const int nk = K / kMlpBK;
     const int S = (nk % 4 == 0 && nk >= 8) ? 4 : (nk % 2 == 0 && nk >= 4) ? 2 : 1;
     MlpParams p;
     p.M = M;
     p.K = K;
+    p.Ka = Ka;
     p.b1 = b1;
     p.w2 = static_cast<const uint16_t *>(w2);
     p.b2 = b2;
     p.out = out;
+    p.act = act;
     p.status = status;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(((M + kMlpBM - 1) / kMlpBM) * S);
@@ -399,9 +621,50 @@ cudaError_t launch_mlp(const void *h, int M, int K, const void *W1, const float 
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    if (S == 4) return cudaLaunchKernelEx(&cfg, mlp_kernel<4>, tmA, tmB, p);
-    if (S == 2) return cudaLaunchKernelEx(&cfg, mlp_kernel<2>, tmA, tmB, p);
-    return cudaLaunchKernelEx(&cfg, mlp_kernel<1>, tmA, tmB, p);
+    if (head) {
+        if (S == 4) return cudaLaunchKernelEx(&cfg, mlp_kernel<4, true>, tmA, tmA2, tmB, p);
+        if (S == 2) return cudaLaunchKernelEx(&cfg, mlp_kernel<2, true>, tmA, tmA2, tmB, p);
+        return cudaLaunchKernelEx(&cfg, mlp_kernel<1, true>, tmA, tmA2, tmB, p);
+    }
+    if (S == 4) return cudaLaunchKernelEx(&cfg, mlp_kernel<4, false>, tmA, tmA2, tmB, p);
+    if (S == 2) return cudaLaunchKernelEx(&cfg, mlp_kernel<2, false>, tmA, tmA2, tmB, p);
+    return cudaLaunchKernelEx(&cfg, mlp_kernel<1, false>, tmA, tmA2, tmB, p);
+}
+
+}  // namespace
+
+cudaError_t launch_mlp(const void *h, int M, int K, const void *W1, const float *b1, const void *w2, float b2,
+                       float *out, int32_t *status, cudaStream_t stream, const char **why) {
+    *why = nullptr;
+    if (M == 0) return cudaSuccess;
+    return launch_layer1(h, K, nullptr, M, K, W1, b1, w2, b2, out, nullptr, true, status, stream, why);
+}
+
+cudaError_t launch_scorer_deep(const void *h, int Kh, const void *f, int M, const void *W1, const float *b1,
+                               const void *W2, const float *b2, const void *W3, const float *b3, const void *w4,
+                               float b4, uint16_t *act, float *out, int32_t *status, cudaStream_t stream,
+                               const char **why) {
+    *why = nullptr;
+    if (M == 0) return cudaSuccess;
+    cudaError_t e = launch_layer1(h, Kh, f, M, Kh + kMlpN, W1, b1, nullptr, 0.f, nullptr, act, false, status,
+                                  stream, why);
+    if (e != cudaSuccess || *why) return e;
+    CUtensorMap tmAct, tmW2, tmW3;
+    if (!g_maps.get(&tmAct, act, M, kMlpN, kMlpBM) || !g_maps.get(&tmW2, W2, kMlpN, kMlpN, kMlpN) ||
+        !g_maps.get(&tmW3, W3, kMlpN, kMlpN, kMlpN)) {
+        *why = "cuTensorMapEncodeTiled failed";
+        return cudaErrorInvalidValue;
+    }
+    TailParams p;
+    p.M = M;
+    p.b2 = b2;
+    p.b3 = b3;
+    p.w4 = static_cast<const uint16_t *>(w4);
+    p.b4 = b4;
+    p.out = out;
+    p.status = status;
+    mlp_tail_kernel<<<(M + kMlpBM - 1) / kMlpBM, kTailThreads, kTailSmem, stream>>>(tmAct, tmW2, tmW3, p);
+    return cudaGetLastError();
 }
 
 }  // namespace sdd

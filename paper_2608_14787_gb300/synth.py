@@ -211,6 +211,34 @@ def make_mlp(device="cpu", seed: int = 4, hidden: int = HIDDEN, width: int = MLP
     return W1.contiguous(), b1.contiguous(), w2.contiguous(), b2.contiguous()
 
 
+def make_scorer_deep(device="cpu", seed: int = 5, hidden: int = HIDDEN, n_feat: int = 19, width: int = MLP_HIDDEN):
+    """Random-init stand-in weights of the learned scorer's shape (App. A.7:
+    (hidden + n_feat) -> width -> width -> width -> 1): W1 [width, hidden + width]
+    bf16 whose columns past hidden + n_feat are zero (the feature block is padded
+    to width columns), W2, W3 [width, width] bf16, w4 [width] bf16, b1..b3 fp32,
+    b4 float; U(+-1/sqrt(fan_in)) like a default Linear init."""
+    g = _gen(device, seed, 0xDEE9)
+    u = lambda *s, a: ((torch.rand(*s, generator=g, device=device) * 2 - 1) * a)   # noqa: E731
+    K1 = hidden + n_feat
+    W1 = torch.zeros(width, hidden + width, device=device)
+    W1[:, :K1] = u(width, K1, a=1.0 / math.sqrt(K1))
+    b1 = u(width, a=1.0 / math.sqrt(K1))
+    W2, b2 = u(width, width, a=1.0 / math.sqrt(width)), u(width, a=1.0 / math.sqrt(width))
+    W3, b3 = u(width, width, a=1.0 / math.sqrt(width)), u(width, a=1.0 / math.sqrt(width))
+    w4, b4 = u(width, a=1.0 / math.sqrt(width)), u(1, a=1.0 / math.sqrt(width))
+    bf = lambda t: t.to(torch.bfloat16).contiguous()   # noqa: E731
+    return (bf(W1), b1.contiguous(), bf(W2), b2.contiguous(), bf(W3), b3.contiguous(), bf(w4), float(b4.item()))
+
+
+def make_features(rows: int, device="cpu", seed: int = 5, round_: int = 0, n_feat: int = 19, width: int = MLP_HIDDEN):
+    """Synthetic scalar features [rows, width] bf16: n_feat standard-normal
+    columns, zeros after them (the padded feature block of the deep scorer)."""
+    g = _gen(device, seed, round_, 0xFEA7)
+    f = torch.zeros(rows, width, device=device)
+    f[:, :n_feat] = torch.randn(rows, n_feat, generator=g, device=device)
+    return f.to(torch.bfloat16).contiguous()
+
+
 def make_hidden(rows: int, device="cpu", seed: int = 4, round_: int = 0, hidden: int = HIDDEN):
     g = _gen(device, seed, round_, 0x41DD)
     return torch.randn(rows, hidden, generator=g, device=device).to(torch.bfloat16).contiguous()
