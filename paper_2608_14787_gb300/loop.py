@@ -2,8 +2,10 @@
 
 Every round a batch of B draft blocks of gamma positions is scored twice --
 raw confidence q = p_draft(x_j) from the drafter logits (Sec. 4.2) and a
-learned-style survival score from the drafter hidden states (the scorer form
-of App. A.7; here a random-init stand-in) -- and the prefix schedule of
+learned-style survival score from the drafter hidden states and scalar
+features (the scorer of App. A.7: by default its full shape, (3584 + 19) ->
+256 -> 256 -> 256 -> 1, fed the row statistics the confidence pass also
+returns; here with random-init stand-in weights) -- and the prefix schedule of
 Sec. 4.1 picks K per block for each signal, with each policy's staleness
 counter D carried across rounds.  The raw-confidence policy drives the round:
 blocks with K = 0 go to the strict verifier (Sec. 3.1), which reads only
@@ -61,7 +63,7 @@ class DecodeLoop:
 
     def __init__(self, B: int, gamma: int, V: int, *, tau: float = 0.9, tau_mlp: float = 0.9, K_min: int = 6,
                  S_max: int = 64, greedy: bool = False, seed: int = 4, hidden: int = synth.HIDDEN, period: int = 4,
-                 device="cuda"):
+                 scorer: str = "deep", device="cuda"):
         self.B, self.gamma, self.V = B, gamma, V
         self.tau, self.tau_mlp, self.K_min, self.S_max = tau, tau_mlp, K_min, S_max
         self.greedy, self.seed, self.period = greedy, seed, period
@@ -72,13 +74,43 @@ class DecodeLoop:
         self.D_raw = torch.zeros(B, dtype=torch.int32, device=dev)
         self.D_mlp = torch.zeros(B, dtype=torch.int32, device=dev)
         self.D_per = torch.zeros(B, dtype=torch.int32, device=dev)
-        self.W1, self.b1, self.w2, b2 = synth.make_mlp(device=dev, seed=seed, hidden=hidden)
-        self.b2 = float(b2.item())
+        self.scorer = scorer
+        if scorer == "deep":
+            self.deep = synth.make_scorer_deep(device=dev, seed=seed, hidden=hidden)
+            self.feat = torch.zeros(B * gamma, sdd.MLP_HIDDEN, dtype=torch.bfloat16, device=dev)
+            self.act = torch.empty(B * gamma, sdd.MLP_HIDDEN, dtype=torch.bfloat16, device=dev)
+        elif scorer == "mlp":
+            self.W1, self.b1, self.w2, b2 = synth.make_mlp(device=dev, seed=seed, hidden=hidden)
+            self.b2 = float(b2.item())
+        else:
+            raise ValueError(f"scorer {scorer!r}: 'deep' or 'mlp'")
+
+    def features(self, conf, round_: int) -> torch.Tensor:
+        """The scorer's scalar-feature block [B * gamma, 256] bf16 (19 columns,
+        zeros after them) in the order of App. A.7's list: the diffusion-model
+        quantities (reveal step and rank, parallelism, late reveal, step-0
+        values and their changes, segment position, dataset flags) are not
+        available here and stay zero; the logits-side ones come from the
+        confidence pass: top-1 probability, its log, entropy, its negative,
+        probability margin, top-5 mass; then block position and generated length."""
+        B, gamma = self.B, self.gamma
+        f = self.feat.view(B, gamma, -1)
+        pos = torch.arange(gamma, device=self.device, dtype=torch.float32).view(1, gamma) / gamma
+        cols = {4: conf.maxprob, 5: torch.log(conf.maxprob), 6: conf.entropy, 7: -conf.entropy, 8: conf.margin,
+                9: conf.top5, 14: pos.expand(B, gamma), 15: torch.full((B, gamma), round_ / 256.0, device=self.device)}
+        for c, v in cols.items():
+            f[:, :, c] = v.to(torch.bfloat16)
+        return self.feat
 
     def step(self, z_d, z_t, x, h, round_: int) -> RoundOut:
         B, gamma = self.B, self.gamma
-        conf = sdd.confidence(z_d, x, ws=self.ws, status=self.status)
-        s = sdd.survival_mlp(h, self.W1, self.b1, self.w2, self.b2, status=self.status).reshape(B, gamma)
+        deep = self.scorer == "deep"
+        conf = sdd.confidence(z_d, x, ws=self.ws, status=self.status, features=deep)
+        if deep:
+            s = sdd.scorer_deep(h, self.features(conf, round_), *self.deep, act=self.act,
+                                status=self.status).reshape(B, gamma)
+        else:
+            s = sdd.survival_mlp(h, self.W1, self.b1, self.w2, self.b2, status=self.status).reshape(B, gamma)
         _, K_raw, D_raw = sdd.schedule_prefix(conf.q, [self.tau], [self.tau], signal=sdd.SIG_RAW, logq=conf.logq,
                                               K_min=self.K_min, S_max=self.S_max, D_in=self.D_raw,
                                               status=self.status)
@@ -98,12 +130,12 @@ class DecodeLoop:
         return RoundOut(K_raw=K, K_mlp=K_mlp[0], K_per=K_per[0], L=L, tokens=tokens, n=n_commit, n_verified=n_rows)
 
 
-def run(rounds: int = 256, workload: str = "c5", warmup: int = 2, device="cuda") -> dict:
+def run(rounds: int = 256, workload: str = "c5", warmup: int = 2, scorer: str = "deep", device="cuda") -> dict:
     """The decode-loop workload: `rounds` rounds of fresh synthetic logits and
     hidden states (generated before each round, untimed)."""
     wl = synth.WORKLOADS[workload]
     B, gamma, V = wl.B, wl.gamma, wl.V
-    loop = DecodeLoop(B, gamma, V, tau=wl.taus[0], device=device, seed=wl.seed)
+    loop = DecodeLoop(B, gamma, V, tau=wl.taus[0], device=device, seed=wl.seed, scorer=scorer)
     st = LoopStats()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     for r in range(-warmup, rounds):
@@ -139,6 +171,8 @@ def run(rounds: int = 256, workload: str = "c5", warmup: int = 2, device="cuda")
         "verifier_calls": st.verified,
         "verifier_calls_saved_raw": st.skipped_raw / max(st.blocks, 1),
         "verifier_calls_saved_mlp_shadow": st.skipped_mlp / max(st.blocks, 1),
+        "scorer": "(3584 + 19) -> 256 -> 256 -> 256 -> 1 (sdd_scorer_deep)" if scorer == "deep"
+        else "3584 -> 256 -> 1 (sdd_survival_mlp)",
         "verifier_calls_saved_periodic_shadow": st.skipped_per / max(st.blocks, 1),
         "periodic_P": loop.period,
         "committed_tokens_per_block": st.committed_tokens / max(st.blocks, 1),

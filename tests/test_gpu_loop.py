@@ -18,11 +18,12 @@ def _bits(t):
     return synth.bf16_bits(t)
 
 
+@pytest.mark.parametrize("scorer", ["deep", "mlp"])
 @pytest.mark.parametrize("B,gamma,V,hidden,rounds", [(6, 8, 3008, 128, 4), (3, 32, 20016, 256, 3)])
-def test_loop_matches_oracle_replay(sdd, orc, B, gamma, V, hidden, rounds):
+def test_loop_matches_oracle_replay(sdd, orc, B, gamma, V, hidden, rounds, scorer):
     wl = synth.WORKLOADS["c5"]
-    loop = DecodeLoop(B, gamma, V, tau=0.5, tau_mlp=0.3, K_min=2, S_max=6, seed=wl.seed, hidden=hidden, period=2)
-    W1, b1, w2 = _bits(loop.W1), loop.b1.cpu().numpy(), _bits(loop.w2)
+    loop = DecodeLoop(B, gamma, V, tau=0.5, tau_mlp=0.3, K_min=2, S_max=6, seed=wl.seed, hidden=hidden, period=2,
+                      scorer=scorer)
     D_raw = np.zeros(B, np.int32)
     D_mlp = np.zeros(B, np.int32)
     D_per = np.zeros(B, np.int32)
@@ -37,13 +38,28 @@ def test_loop_matches_oracle_replay(sdd, orc, B, gamma, V, hidden, rounds):
         # oracle replay of the round
         st = orc.row_stats(zd, tokens=x)
         _, K_raw, D_raw, mg_raw = orc.schedule(st.q, orc.SIG_RAW, 0.5, 0.5, 2, 6, D_in=D_raw)
-        s = orc.survival_mlp(_bits(h), W1, b1, w2, loop.b2).reshape(B, gamma)
+        if scorer == "deep":
+            # the scorer on the device's feature block (the features are pinned by their own parity tests)
+            W1, b1, W2, b2, W3, b3, w4, b4 = loop.deep
+            x_in = torch.cat([h, loop.feat], dim=-1)
+            s = orc.scorer_deep(_bits(x_in), _bits(W1), b1.cpu().numpy(), _bits(W2), b2.cpu().numpy(), _bits(W3),
+                                b3.cpu().numpy(), _bits(w4), b4).reshape(B, gamma)
+        else:
+            s = orc.survival_mlp(_bits(h), _bits(loop.W1), loop.b1.cpu().numpy(), _bits(loop.w2),
+                                 loop.b2).reshape(B, gamma)
         _, K_mlp, D_mlp, mg_mlp = orc.schedule(s, orc.SIG_CONDITIONAL, 0.3, 0.3, 2, 6, D_in=D_mlp)
-        assert (mg_raw >= NEAR).all() and (mg_mlp >= NEAR).all(), "near-threshold row: pick another seed"
+        assert (mg_raw >= NEAR).all(), "near-threshold row: pick another seed"
         np.testing.assert_array_equal(out.K_raw.cpu().numpy(), K_raw)
-        np.testing.assert_array_equal(out.K_mlp.cpu().numpy(), K_mlp)
         np.testing.assert_array_equal(loop.D_raw.cpu().numpy(), D_raw)
-        np.testing.assert_array_equal(loop.D_mlp.cpu().numpy(), D_mlp)
+        # the scorer's schedule: rows whose decision lies within the scores'
+        # tolerance of a threshold (a product of up to gamma scores, each within
+        # 3e-4 for the deep scorer, 5e-5 for the one-layer one) are exempt, and
+        # the oracle continues from the device's staleness counters
+        tol = gamma * (3e-4 if scorer == "deep" else 5e-5)
+        sure = mg_mlp >= tol
+        np.testing.assert_array_equal(out.K_mlp.cpu().numpy()[sure], K_mlp[sure])
+        np.testing.assert_array_equal(loop.D_mlp.cpu().numpy()[sure], D_mlp[sure])
+        D_mlp = loop.D_mlp.cpu().numpy().astype(np.int32)
         _, K_per, D_per = orc.schedule_periodic(B, gamma, 2, 2, r, 2, 6, D_in=D_per)   # P = 2, K_skip = K_min
         np.testing.assert_array_equal(out.K_per.cpu().numpy(), K_per)
         np.testing.assert_array_equal(loop.D_per.cpu().numpy(), D_per)
