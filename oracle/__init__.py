@@ -25,6 +25,7 @@ bf16 logits); both are converted exactly to fp64 inside the C code.
 from __future__ import annotations
 
 import ctypes
+import math
 import os
 import subprocess
 from dataclasses import dataclass
@@ -113,6 +114,10 @@ def lib():
     L.orc_scorer_deep.argtypes = [u16p, ctypes.c_int, ctypes.c_int, u16p, f32p, u16p, f32p, u16p, f32p, u16p,
                                   ctypes.c_double, ctypes.c_int, f64p, f64p, f64p]
     L.orc_scorer_deep.restype = None
+    L.orc_permutation_diagnostic.argtypes = [dp, ip32, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_double,
+                                             ctypes.c_double, ctypes.c_int, ctypes.c_uint64, ip64, dp, ip32, ip32,
+                                             ip32, ip32]
+    L.orc_permutation_diagnostic.restype = None
     _lib = L
     return L
 
@@ -398,6 +403,51 @@ def scorer_deep(x_bits, W1_bits, b1, W2_bits, b2, W3_bits, b3, w4_bits, b4: floa
                           b3.ctypes.data_as(f32p), w4.ctypes.data_as(u16p), float(b4), N, out.ctypes.data_as(dp),
                           s1.ctypes.data_as(dp), s2.ctypes.data_as(dp))
     return out
+
+
+def permutation_diagnostic(q, L, signal, eta_b, eta_c, n_rep, seed):
+    """Sums of the feasible prefix lengths: [n_rep] under the permutations, then
+    the logged order (length n_rep + 1)."""
+    q = np.ascontiguousarray(np.asarray(q, dtype=np.float64))
+    B, gamma = q.shape
+    L = np.ascontiguousarray(np.asarray(L, dtype=np.int32).reshape(B))
+    sums = np.zeros(n_rep + 1, np.int64)
+    qp = np.zeros_like(q)
+    lst, kh, k, d = (np.zeros(max(B, 1), np.int32) for _ in range(4))
+    i32 = lambda a: _ptr(a, ctypes.c_int32)   # noqa: E731
+    lib().orc_permutation_diagnostic(_ptr(q, ctypes.c_double), i32(L), B, gamma, int(signal), float(eta_b),
+                                     float(eta_c), int(n_rep), ctypes.c_uint64(int(seed)), _ptr(sums, ctypes.c_int64),
+                                     _ptr(qp, ctypes.c_double), i32(lst), i32(kh), i32(k), i32(d))
+    return sums
+
+
+def position_metrics(q, L, conditional: bool):
+    """Positionwise BCE, position-only baseline BCE and AUROC (fp64, plain
+    loops over the definitions): labels y = 1{L >= j}, j 1-based; blocks with
+    L >= j - 1 only when conditional.  Returns (bce, bce_base, auroc, n_pos, n_neg)."""
+    q = np.asarray(q, dtype=np.float64)
+    L = np.asarray(L, dtype=np.int64)
+    B, gamma = q.shape
+    out = [np.full(gamma, np.nan) for _ in range(3)]
+    npos, nneg = np.zeros(gamma, np.int64), np.zeros(gamma, np.int64)
+    for j in range(gamma):
+        idx = [b for b in range(B) if not conditional or L[b] >= j]
+        if not idx:
+            continue
+        y = [1 if L[b] >= j + 1 else 0 for b in idx]
+        qc = [min(max(q[b, j], 1e-7), 1.0 - 1e-7) for b in idx]
+        n = len(idx)
+        out[0][j] = -sum(math.log(c) if t else math.log1p(-c) for c, t in zip(qc, y)) / n
+        p = sum(y) / n
+        out[1][j] = -(p * math.log(p) + (1 - p) * math.log1p(-p)) if 0.0 < p < 1.0 else 0.0
+        pos = [q[b, j] for b, t in zip(idx, y) if t]
+        neg = [q[b, j] for b, t in zip(idx, y) if not t]
+        npos[j], nneg[j] = len(pos), len(neg)
+        if pos and neg:
+            gt = sum(1 for a in pos for c in neg if a > c)
+            eq = sum(1 for a in pos for c in neg if a == c)
+            out[2][j] = (gt + 0.5 * eq) / (len(pos) * len(neg))
+    return out[0], out[1], out[2], npos, nneg
 
 
 def agreement(K, L):

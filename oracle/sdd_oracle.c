@@ -17,6 +17,7 @@
  * live in tests/test_oracle_*.py.
  */
 #include <math.h>
+#include <stdlib.h>
 #include <stdint.h>
 #include <string.h>
 
@@ -552,5 +553,59 @@ void orc_scorer_deep(const uint16_t *x, int M, int K, const uint16_t *W1, const 
             t += orc_load(w4, ORC_BF16, n) * orc_gelu(z);
         }
         out[m] = 1.0 / (1.0 + exp(-t));
+    }
+}
+
+/* ------------------------------------------------------------------------ */
+/* Permutation diagnostic (Sec. 5, H1 mechanism, Table 1) on logged blocks:  */
+/* scores q[B][gamma] (fp64), strict accepted lengths L[B].  For each        */
+/* repetition r and position j (1-based), the blocks valid at j -- all for   */
+/* the raw and marginal signals, those with L >= j - 1 for the conditional   */
+/* one -- exchange their (score, label) pairs by a uniformly random          */
+/* permutation; the others keep theirs.  The feasible prefix length of every */
+/* block is then K_hat of orc_schedule for (eta_b, eta_c) (the gates before  */
+/* K_min or staleness).  sums[r] = sum of the feasible prefixes under        */
+/* permutation r; sums[n_rep] = the sum in the logged order.                 */
+/* The permutation of (r, j): the valid blocks in index order, shuffled by   */
+/* Fisher-Yates from the top; slot i swaps with floor(w (i+1) / 2^32), w the */
+/* first Philox4x32-10 word of key seed and counter (i, j - 1, r, 3).  The   */
+/* t-th valid block takes the score of the t-th entry of the shuffle.        */
+/* Parity pinned in tests/test_oracle_diag.py (column-constant and identical */
+/* rows are invariant, permutations preserve every column's multiset, a      */
+/* closed form of the independent-position expectation).                    */
+/* ------------------------------------------------------------------------ */
+void orc_permutation_diagnostic(const double *q, const int32_t *L, int B, int gamma, int signal, double eta_b,
+                                double eta_c, int n_rep, uint64_t seed, int64_t *sums, double *qp, int32_t *list,
+                                int32_t *Khat, int32_t *K, int32_t *D) {
+    /* qp: scratch [B * gamma]; list: scratch [B]; Khat, K, D: scratch [B] */
+    for (int r = 0; r <= n_rep; ++r) {
+        for (int b = 0; b < B; ++b)
+            for (int j = 0; j < gamma; ++j) qp[(int64_t)b * gamma + j] = q[(int64_t)b * gamma + j];
+        if (r < n_rep) {
+            for (int j = 0; j < gamma; ++j) {
+                int n = 0;
+                for (int b = 0; b < B; ++b)
+                    if (signal != 2 || L[b] >= j) list[n++] = b;
+                uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+                int32_t *sh = list + 0; /* shuffled in place; the valid order is recomputed below */
+                int32_t *valid = (int32_t *)malloc(sizeof(int32_t) * (n > 0 ? n : 1));
+                for (int t = 0; t < n; ++t) valid[t] = sh[t];
+                for (int i = n - 1; i > 0; --i) {
+                    uint32_t ctr[4] = {(uint32_t)i, (uint32_t)j, (uint32_t)r, 3u}, out[4];
+                    orc_philox4x32_10(ctr, key, out);
+                    int k = (int)(((uint64_t)out[0] * (uint64_t)(i + 1)) >> 32);
+                    int32_t tmp = sh[i];
+                    sh[i] = sh[k];
+                    sh[k] = tmp;
+                }
+                for (int t = 0; t < n; ++t)
+                    qp[(int64_t)valid[t] * gamma + j] = q[(int64_t)sh[t] * gamma + j];
+                free(valid);
+            }
+        }
+        orc_schedule(qp, B, gamma, signal, eta_b, eta_c, 0, 0x7FFFFFFF, NULL, NULL, NULL, Khat, K, D, NULL);
+        int64_t sum = 0;
+        for (int b = 0; b < B; ++b) sum += Khat[b];
+        sums[r] = sum;
     }
 }
