@@ -21,6 +21,7 @@ Other rows of the path, one JSON line each (not the fused-round contract line):
   python bench.py --component loop [--steps R]  the decode-loop workload (R rounds, default 64)
   python bench.py --component features          drafter confidence with / without the extended features
   python bench.py --component scorer [--steps K] the deep scorer (K calls)
+  python bench.py --component diag              the permutation diagnostic (Table 1 settings)
 """
 from __future__ import annotations
 
@@ -502,6 +503,72 @@ def run_component_scorer(args):
     return 0
 
 
+def run_component_diag(args):
+    """NEXT-4: the permutation diagnostic of Sec. 5 (Table 1's settings: 100
+    repetitions; raw (0.90, 0.93), marginal 0.90, conditional (0.90, 0.90)) and
+    the positionwise metrics on a synthetic log: raw confidence and
+    shadow-verified strict L of 32 fused c3 rounds (512 blocks, gamma = 32).
+    The signals all read the raw-confidence log (no trained scorer exists here)."""
+    import numpy as np
+    import torch
+    import paper_2608_14787_gb300 as sdd
+    from paper_2608_14787_gb300 import build as sdd_build
+    from paper_2608_14787_gb300 import synth
+    sdd_build.build()
+    sdd.load()
+    wl = synth.WORKLOADS["c3"]
+    B, gamma, V = wl.B, wl.gamma, wl.V
+    rnd = sdd.BlockRound(B, gamma, V, taus=wl.taus, K_min=6, S_max=64)
+    qs, Ls = [], []
+    for r in range(32):
+        blk = synth.make_block(wl, device="cuda", round_=r)
+        rnd.set_inputs(blk.z_d, blk.z_t, blk.x, seed=wl.seed, round_=r)
+        rnd.run()
+        qs.append(rnd.q.clone())
+        Ls.append(rnd.L_strict.clone())
+        del blk
+    q, L = torch.cat(qs), torch.cat(Ls)
+    torch.cuda.synchronize()
+    nb = q.shape[0]
+    settings = [("raw", 0, 0.90, 0.93), ("marginal", 1, 0.90, 0.90), ("conditional", 2, 0.90, 0.90)]
+    res, times = {}, []
+    with ClockSampler(None) as clk:
+        for name, sig, eb, ec in settings:
+            sdd.permutation_diagnostic(q, L, signal=sig, eta_b=eb, eta_c=ec, n_rep=100, seed=0)   # warm-up
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            sums = sdd.permutation_diagnostic(q, L, signal=sig, eta_b=eb, eta_c=ec, n_rep=100, seed=0)
+            e1.record()
+            torch.cuda.synchronize()
+            times.append(e0.elapsed_time(e1) / 1e3)
+            s = sums.cpu().numpy()
+            res[name] = {"original": float(s[-1]) / nb, "permuted_mean": float(s[:-1].mean()) / nb}
+        bce, base, auc, npos, nneg = sdd.position_metrics(q, L)
+        torch.cuda.synchronize()
+    cpu = None
+    if not args.no_cpu_baseline:
+        import oracle as orc
+        t0 = time.perf_counter()
+        orc.permutation_diagnostic(q.double().cpu().numpy(), L.cpu().numpy(), 0, 0.90, 0.93, 10, 0)
+        dt = time.perf_counter() - t0
+        cpu = {"value": 10 * nb / dt, "unit": "block-repetitions/s", "cores": 1, "kind": "oracle",
+               "sample": f"10 of the 100 repetitions of the raw setting over {nb} blocks ({dt:.2f} s)"}
+    t_mean = sum(times) / len(times)
+    line = {
+        "component": "NEXT-4 permutation diagnostic (sdd_permutation_diagnostic)",
+        "metric": "block-repetitions/s", "unit": "block-repetitions/s", "value": 100 * nb / t_mean,
+        "us_per_call": t_mean * 1e6, "blocks": nb, "gamma": gamma, "repetitions": 100,
+        "feasible_prefix_mean": res,
+        "mean_bce": float(np.nanmean(bce.cpu().numpy())), "mean_bce_position_only": float(np.nanmean(base.cpu().numpy())),
+        "mean_auroc": float(np.nanmean(auc.cpu().numpy())),
+        "note": "synthetic raw-confidence log (32 c3 rounds); the paper's Table 1 needs its HumanEval logs",
+        "cpu_baseline": cpu, "clocks": clk.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_component_features(args):
     """Drafter confidence with and without the extended features (App. A.7:
     probability margin, top-5 mass) on the drafter half of the c3 workload
@@ -608,7 +675,7 @@ def main():
     ap.add_argument("--sets", type=int, default=3, help="rotating input sets (3 x 316 MB exceeds L2)")
     ap.add_argument("--traffic", type=float, default=None,
                     help="dram bytes per scan launch from an ncu capture of the current kernel")
-    ap.add_argument("--component", default=None, choices=["mlp", "loop", "features", "scorer"],
+    ap.add_argument("--component", default=None, choices=["mlp", "loop", "features", "scorer", "diag"],
                     help="measure one other row of the path instead of the fused round")
     args = ap.parse_args()
     if args.component == "mlp":
@@ -619,6 +686,8 @@ def main():
         return run_component_features(args)
     if args.component == "scorer":
         return run_component_scorer(args)
+    if args.component == "diag":
+        return run_component_diag(args)
     if args.traffic is None and args.workload == "c3":
         args.traffic = SCAN_TRAFFIC_C3
     if args.warmup < 3:

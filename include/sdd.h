@@ -196,6 +196,49 @@ SDD_API sdd_status_t sdd_schedule_periodic(int B, int gamma, const int32_t *peri
                                            int32_t *K, int32_t *D_out, int32_t *status, sdd_stream_t stream);
 
 /*
+ * Offline diagnostics over logged blocks: per block b its position scores
+ * q[b, 0..gamma) (fp32, device) and its strict accepted length L[b] (int32,
+ * device; from Strict SDD or the shadow verifier), j below 1-based.
+ *
+ * sdd_permutation_diagnostic -- the permutation test of Sec. 5 (H1 mechanism,
+ * Table 1): n_rep times, at every position j the (score, label) pairs are
+ * permuted across the blocks valid there -- all blocks for RAW and MARGINAL,
+ * those with L >= j - 1 for CONDITIONAL -- which keeps every positionwise
+ * distribution (so every positionwise metric) and breaks the association of
+ * positions within a block; then the feasible prefix length of every block
+ * is recomputed: K_hat of sdd_schedule_prefix for the pair (eta_b, eta_c)
+ * before K_min or staleness.  Permutation r of position j is a Fisher-Yates
+ * shuffle of the valid blocks in index order: slot i (from the top) swaps
+ * with floor(w (i + 1) / 2^32), w the first word of Philox4x32-10 with key
+ * seed and counter (i, j - 1, r, 3) (the map of sdd_uniforms, purpose 3).
+ * Writes sums[r] = sum over blocks of the feasible prefix length under
+ * permutation r (r < n_rep) and sums[n_rep] = that sum in the logged order
+ * (int64, device); the means are sums / B.  Workspace: at least
+ * sdd_permutation_workspace_size(B, gamma, n_rep) bytes (device).  B <= 50000.
+ */
+SDD_API sdd_status_t sdd_permutation_workspace_size(int B, int gamma, int n_rep, size_t *bytes);
+SDD_API sdd_status_t sdd_permutation_diagnostic(const float *q, const int32_t *L, int B, int gamma,
+                                                sdd_signal_t signal, double eta_b, double eta_c, int n_rep,
+                                                uint64_t seed, int64_t *sums, void *workspace,
+                                                size_t workspace_bytes, sdd_stream_t stream);
+
+/*
+ * sdd_position_metrics -- positionwise offline metrics (Sec. 5 H1, App. offline
+ * metrics) of the scores against the labels y = 1{L >= j} at each position j,
+ * over all blocks (conditional = 0: marginal survival, raw confidence) or the
+ * blocks with L >= j - 1 (conditional != 0): for position j (index j - 1)
+ *   bce[j]      = -mean(y ln q' + (1 - y) ln(1 - q')), q' = q clamped to [1e-7, 1 - 1e-7];
+ *   bce_base[j] = the same for the position-only predictor (the positive rate
+ *                 at j on these blocks): -(p ln p + (1 - p) ln(1 - p));
+ *   auroc[j]    = (#{q_pos > q_neg} + #{q_pos = q_neg} / 2) / (n_pos n_neg),
+ *                 NaN without positives or negatives;
+ *   n_pos, n_neg [gamma] int32 (may be NULL).  bce, bce_base, auroc fp64 [gamma], device.
+ */
+SDD_API sdd_status_t sdd_position_metrics(const float *q, const int32_t *L, int B, int gamma, int conditional,
+                                          double *bce, double *bce_base, double *auroc, int32_t *n_pos,
+                                          int32_t *n_neg, sdd_stream_t stream);
+
+/*
  * sdd_verify_strict -- Strict SDD verification (Sec. 3.1: the standard rule of
  * speculative decoding) of the blocks listed in rows[0..n_rows) (all B blocks
  * when rows is NULL; then n_rows must be B, or 0 for an empty list, which

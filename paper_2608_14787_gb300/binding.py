@@ -94,6 +94,13 @@ def load(path: str | None = None):
     L.sdd_survival_mlp.restype = I
     L.sdd_scorer_deep.argtypes = [VP, I, VP, I, VP, VP, VP, VP, VP, VP, VP, ctypes.c_float, VP, VP, VP, VP]
     L.sdd_scorer_deep.restype = I
+    L.sdd_permutation_workspace_size.argtypes = [I, I, I, ctypes.POINTER(ctypes.c_size_t)]
+    L.sdd_permutation_workspace_size.restype = I
+    L.sdd_permutation_diagnostic.argtypes = [VP, VP, I, I, I, ctypes.c_double, ctypes.c_double, I, u64, VP, VP,
+                                             ctypes.c_size_t, VP]
+    L.sdd_permutation_diagnostic.restype = I
+    L.sdd_position_metrics.argtypes = [VP, VP, I, I, I, VP, VP, VP, VP, VP, VP]
+    L.sdd_position_metrics.restype = I
     for fn in ("sdd_block", "sdd_block_scan", "sdd_block_decide"):
         getattr(L, fn).argtypes = [ctypes.POINTER(BlockArgs), VP]
     for fn in ("sdd_workspace_size", "sdd_confidence", "sdd_confidence_features", "sdd_schedule_prefix",
@@ -381,6 +388,37 @@ def scorer_deep(h, f, W1, b1, W2, b2, W3, b3, w4, b4, *, act=None, status=None, 
     _check(load().sdd_scorer_deep(_p(h2), Kh, _p(f2), M, _p(W1), _p(b1), _p(W2), _p(b2), _p(W3), _p(b3), _p(w4),
                                   float(b4), _p(act), _p(s), _p(status), _stream(stream)), "sdd_scorer_deep")
     return s.reshape(lead)
+
+
+def permutation_diagnostic(q, L, *, signal=SIG_RAW, eta_b=0.9, eta_c=0.93, n_rep=100, seed=0, stream=None):
+    """sdd_permutation_diagnostic over logged blocks (q [B, gamma] fp32, L [B]
+    int32): returns the int64 sums [n_rep + 1] of the feasible prefix lengths
+    (the permutations, then the logged order); means are sums / B."""
+    B, gamma = q.shape
+    nbytes = ctypes.c_size_t(0)
+    _check(load().sdd_permutation_workspace_size(B, gamma, n_rep, ctypes.byref(nbytes)),
+           "sdd_permutation_workspace_size")
+    ws = torch.empty(max(int(nbytes.value), 1), dtype=torch.uint8, device=q.device)
+    sums = torch.empty(n_rep + 1, dtype=torch.int64, device=q.device)
+    q = q.contiguous()
+    L = L.to(torch.int32).contiguous()
+    _check(load().sdd_permutation_diagnostic(_p(q), _p(L), B, gamma, signal, float(eta_b), float(eta_c), n_rep, seed,
+                                             _p(sums), _p(ws), ws.numel(), _stream(stream)),
+           "sdd_permutation_diagnostic")
+    return sums
+
+
+def position_metrics(q, L, *, conditional=False, stream=None):
+    """sdd_position_metrics: (bce, bce_base, auroc) fp64 [gamma] and (n_pos, n_neg) int32 [gamma]."""
+    B, gamma = q.shape
+    dev = q.device
+    out = [torch.empty(gamma, dtype=torch.float64, device=dev) for _ in range(3)]
+    cnt = [torch.empty(gamma, dtype=torch.int32, device=dev) for _ in range(2)]
+    q = q.contiguous()
+    L = L.to(torch.int32).contiguous()
+    _check(load().sdd_position_metrics(_p(q), _p(L), B, gamma, 1 if conditional else 0, *(_p(t) for t in out),
+                                       *(_p(t) for t in cnt), _stream(stream)), "sdd_position_metrics")
+    return (*out, *cnt)
 
 
 def uniforms(seed, j, b, round_, purpose, stream=None):

@@ -603,6 +603,58 @@ sdd_status_t sdd_scorer_deep(const void *h, int Kh, const void *f, int M, const 
     return SDD_OK;
 }
 
+sdd_status_t sdd_permutation_workspace_size(int B, int gamma, int n_rep, size_t *bytes) {
+    if (!bytes) return fail(SDD_ERR_INVALID_ARGUMENT, "bytes is NULL");
+    if (B < 0 || gamma < 1 || gamma > SDD_MAX_GAMMA || n_rep < 0)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "B = %d, gamma = %d, n_rep = %d out of range", B, gamma, n_rep);
+    *bytes = align256(static_cast<size_t>(n_rep) * gamma * B * sizeof(int32_t)) +
+             align256(static_cast<size_t>(n_rep + 1) * sizeof(unsigned long long));
+    return SDD_OK;
+}
+
+sdd_status_t sdd_permutation_diagnostic(const float *q, const int32_t *L, int B, int gamma, sdd_signal_t signal,
+                                        double eta_b, double eta_c, int n_rep, uint64_t seed, int64_t *sums,
+                                        void *workspace, size_t workspace_bytes, sdd_stream_t stream) {
+    if (B < 0 || gamma < 1 || gamma > SDD_MAX_GAMMA)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "B = %d / gamma = %d out of range", B, gamma);
+    if (n_rep < 0 || n_rep > 100000) return fail(SDD_ERR_INVALID_ARGUMENT, "n_rep = %d out of range", n_rep);
+    if (B > 50000) return fail(SDD_ERR_UNSUPPORTED, "B = %d logged blocks exceed 50000 (one shared-memory list)", B);
+    df eta_loc, log_eta_c;
+    int32_t off = 0;
+    SDD_TRY(set_thresholds(signal, &eta_b, &eta_c, 1, &eta_loc, &log_eta_c, &off));
+    if (B == 0) return SDD_OK;
+    if (!q || !L || !sums) return fail(SDD_ERR_INVALID_ARGUMENT, "q, L and sums must not be NULL");
+    size_t need = 0;
+    SDD_TRY(sdd_permutation_workspace_size(B, gamma, n_rep, &need));
+    if (!workspace || workspace_bytes < need)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "workspace of %zu bytes < %zu needed", workspace_bytes, need);
+    if (off) {   // a threshold >= 1 disables skipping: every feasible prefix is 0
+        cudaError_t e = cudaMemsetAsync(sums, 0, sizeof(int64_t) * (n_rep + 1), reinterpret_cast<cudaStream_t>(stream));
+        return e == cudaSuccess ? SDD_OK : cuda_fail(e, "memset");
+    }
+    unsigned char *base = static_cast<unsigned char *>(workspace);
+    int32_t *perm = reinterpret_cast<int32_t *>(base);
+    unsigned long long *acc = reinterpret_cast<unsigned long long *>(
+        base + align256(static_cast<size_t>(n_rep) * gamma * B * sizeof(int32_t)));
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e = launch_perm_diag(q, L, B, gamma, signal, eta_loc, log_eta_c, n_rep, seed, perm, acc, st);
+    if (e != cudaSuccess) return cuda_fail(e, "permutation diagnostic launch");
+    e = cudaMemcpyAsync(sums, acc, sizeof(int64_t) * (n_rep + 1), cudaMemcpyDeviceToDevice, st);
+    return e == cudaSuccess ? SDD_OK : cuda_fail(e, "copy");
+}
+
+sdd_status_t sdd_position_metrics(const float *q, const int32_t *L, int B, int gamma, int conditional, double *bce,
+                                  double *bce_base, double *auroc, int32_t *n_pos, int32_t *n_neg,
+                                  sdd_stream_t stream) {
+    if (B < 0 || gamma < 1 || gamma > SDD_MAX_GAMMA)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "B = %d / gamma = %d out of range", B, gamma);
+    if (!q || !L || !bce || !bce_base || !auroc)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "q, L, bce, bce_base and auroc must not be NULL");
+    cudaError_t e = launch_position_metrics(q, L, B, gamma, conditional ? 1 : 0, bce, bce_base, auroc, n_pos, n_neg,
+                                            reinterpret_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? SDD_OK : cuda_fail(e, "position metrics launch");
+}
+
 static sdd_status_t block_check(const sdd_block_args *a) {
     if (!a) return fail(SDD_ERR_INVALID_ARGUMENT, "args is NULL");
     SDD_TRY(check_shape(static_cast<sdd_dtype_t>(a->dtype), a->B, a->gamma, a->V, a->row_stride));

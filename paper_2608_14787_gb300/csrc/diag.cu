@@ -1,0 +1,176 @@
+// diag.cu -- offline diagnostics over logged blocks (scores q [B, gamma] and
+// strict accepted lengths L [B] of Strict SDD / shadow-verified rounds):
+//
+//  * the permutation diagnostic behind Table 1 (Sec. 5, H1 mechanism): at every
+//    position j the (score, label) pairs are permuted across the blocks valid
+//    there (all blocks; for the conditional signal those with L >= j - 1, j
+//    1-based), which keeps every positionwise distribution and breaks the
+//    association of positions within a block; the feasible prefix length
+//    (Eq. 3's gates, before K_min or staleness) is recomputed per block;
+//  * positionwise offline metrics (App. offline metrics): BCE of the scores
+//    against the labels 1{L >= j}, the position-only baseline (the positive
+//    rate at j), and AUROC (Mann-Whitney, ties count one half).
+//
+// perm_build_kernel  -- one CTA per (repetition, position): Fisher-Yates over
+//                       the valid blocks in shared memory, Philox draws.
+// perm_prefix_kernel -- one warp per (repetition, block): the gates of Eq. 3 on
+//                       the permuted scores (the schedule's own arithmetic),
+//                       integer sums per repetition (exact, order-free).
+// metrics_kernel     -- one CTA per position: fp64 BCE sums, integer pair counts.
+#include "rules.cuh"
+
+namespace sdd {
+namespace {
+
+constexpr uint32_t kPurposePerm = 3;
+constexpr int kDiagThreads = 256;
+
+__global__ void __launch_bounds__(kDiagThreads) perm_build_kernel(const int32_t *L, int B, int gamma, int n_rep,
+                                                                  int conditional, uint64_t seed, int32_t *perm) {
+    extern __shared__ int32_t s_list[];   // [B]: the valid blocks, then their shuffle
+    const int r = blockIdx.x / gamma, j = blockIdx.x % gamma;
+    int32_t *row = perm + (static_cast<int64_t>(r) * gamma + j) * B;
+    __shared__ int s_n;
+    if (threadIdx.x == 0) {
+        // the valid blocks in index order (serial: the order defines the draw)
+        int n = 0;
+        for (int b = 0; b < B; ++b)
+            if (!conditional || __ldg(L + b) >= j) s_list[n++] = b;
+        // Fisher-Yates from the top: slot i swaps with k = floor(w (i + 1) / 2^32),
+        // w the first Philox word of counter (i, j, r, purpose)
+        const uint2 key = make_uint2(static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32));
+        for (int i = n - 1; i > 0; --i) {
+            const uint4 o = philox4x32_10(make_uint4(static_cast<uint32_t>(i), static_cast<uint32_t>(j),
+                                                     static_cast<uint32_t>(r), kPurposePerm),
+                                          key);
+            const int k = static_cast<int>((static_cast<uint64_t>(o.x) * static_cast<uint64_t>(i + 1)) >> 32);
+            const int32_t t = s_list[i];
+            s_list[i] = s_list[k];
+            s_list[k] = t;
+        }
+        s_n = n;
+    }
+    __syncthreads();
+    // block b (t-th valid block) takes the score of block s_list[t]; others keep theirs
+    if (threadIdx.x == 0) {
+        int t = 0;
+        for (int b = 0; b < B; ++b) row[b] = (!conditional || __ldg(L + b) >= j) ? s_list[t++] : b;
+    }
+}
+
+__global__ void perm_prefix_kernel(const float *q, const int32_t *perm, int B, int gamma, int n_rep, int signal,
+                                   df eta_loc, df log_eta_c, unsigned long long *sums) {
+    const int lane = threadIdx.x & 31;
+    const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    if (w >= static_cast<int64_t>(n_rep + 1) * B) return;
+    const int r = static_cast<int>(w / B), b = static_cast<int>(w % B);   // r == n_rep: the logged order
+    int kb = gamma, best = 0;
+    df carry = df{0.f, 0.f};
+    for (int c = 0; c < gamma && kb >= c; c += 32) {
+        const int j = c + lane;
+        const bool in = j < gamma;
+        int src = b;
+        if (in && r < n_rep) src = __ldg(perm + (static_cast<int64_t>(r) * gamma + j) * B + b);
+        const float qj = in ? __ldg(q + static_cast<int64_t>(src) * gamma + j) : 0.f;
+        const float lq = in ? logf(qj) : 0.f;
+        const df S = df_add(carry, warp_prefix_df(df{lq, 0.f}, lane));
+        carry.hi = __shfl_sync(0xFFFFFFFFu, S.hi, 31);
+        carry.lo = __shfl_sync(0xFFFFFFFFu, S.lo, 31);
+        sched_step(c, lane, gamma, in, qj, false, S, eta_loc, log_eta_c, signal, kb, best);
+    }
+    const int Kh = (signal == SDD_SIG_MARGINAL) ? kb : best;
+    if (lane == 0) atomicAdd(sums + r, static_cast<unsigned long long>(Kh));
+}
+
+__global__ void __launch_bounds__(kDiagThreads) metrics_kernel(const float *q, const int32_t *L, int B, int gamma,
+                                                               int conditional, double *bce, double *bce_base,
+                                                               double *auroc, int32_t *n_pos, int32_t *n_neg) {
+    const int j = blockIdx.x;
+    __shared__ double s_bce[kDiagThreads];
+    __shared__ unsigned long long s_np[kDiagThreads], s_nn[kDiagThreads], s_gt[kDiagThreads], s_eq[kDiagThreads];
+    double sb = 0.0;
+    unsigned long long np = 0, nn = 0, gt = 0, eq = 0;
+    for (int b = threadIdx.x; b < B; b += kDiagThreads) {
+        const int l = __ldg(L + b);
+        if (conditional && l < j) continue;
+        const bool y = l >= j + 1;
+        const double qc = fmin(fmax(static_cast<double>(__ldg(q + static_cast<int64_t>(b) * gamma + j)), 1e-7),
+                               1.0 - 1e-7);
+        sb -= y ? log(qc) : log1p(-qc);
+        if (y) {
+            ++np;
+            const float qi = __ldg(q + static_cast<int64_t>(b) * gamma + j);
+            for (int k = 0; k < B; ++k) {   // every valid negative
+                const int lk = __ldg(L + k);
+                if ((conditional && lk < j) || lk >= j + 1) continue;
+                const float qk = __ldg(q + static_cast<int64_t>(k) * gamma + j);
+                gt += qi > qk;
+                eq += qi == qk;
+            }
+        } else {
+            ++nn;
+        }
+    }
+    s_bce[threadIdx.x] = sb;
+    s_np[threadIdx.x] = np;
+    s_nn[threadIdx.x] = nn;
+    s_gt[threadIdx.x] = gt;
+    s_eq[threadIdx.x] = eq;
+    __syncthreads();
+    for (int h = kDiagThreads / 2; h > 0; h >>= 1) {   // fixed-order tree: deterministic sums
+        if (threadIdx.x < h) {
+            s_bce[threadIdx.x] += s_bce[threadIdx.x + h];
+            s_np[threadIdx.x] += s_np[threadIdx.x + h];
+            s_nn[threadIdx.x] += s_nn[threadIdx.x + h];
+            s_gt[threadIdx.x] += s_gt[threadIdx.x + h];
+            s_eq[threadIdx.x] += s_eq[threadIdx.x + h];
+        }
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+        const double P = static_cast<double>(s_np[0]), N = static_cast<double>(s_nn[0]), n = P + N;
+        const double nan = __longlong_as_double(0x7FF8000000000000ll);
+        bce[j] = (n > 0) ? s_bce[0] / n : nan;
+        const double pr = (n > 0) ? P / n : nan;
+        bce_base[j] = (n > 0) ? ((pr > 0.0 && pr < 1.0) ? -(pr * log(pr) + (1.0 - pr) * log1p(-pr)) : 0.0) : nan;
+        auroc[j] = (P > 0 && N > 0) ? (static_cast<double>(s_gt[0]) + 0.5 * static_cast<double>(s_eq[0])) / (P * N)
+                                    : nan;
+        if (n_pos) n_pos[j] = static_cast<int32_t>(s_np[0]);
+        if (n_neg) n_neg[j] = static_cast<int32_t>(s_nn[0]);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_perm_diag(const float *q, const int32_t *L, int B, int gamma, int signal, df eta_loc,
+                             df log_eta_c, int n_rep, uint64_t seed, int32_t *perm, unsigned long long *sums,
+                             cudaStream_t stream) {
+    cudaError_t e = cudaMemsetAsync(sums, 0, sizeof(unsigned long long) * (n_rep + 1), stream);
+    if (e != cudaSuccess) return e;
+    const size_t smem = static_cast<size_t>(B) * sizeof(int32_t);
+    if (smem > 48 * 1024) {
+        e = cudaFuncSetAttribute(perm_build_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+    }
+    if (n_rep > 0) {
+        perm_build_kernel<<<n_rep * gamma, 32, smem, stream>>>(L, B, gamma, n_rep, signal == SDD_SIG_CONDITIONAL,
+                                                               seed, perm);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    const int64_t warps = static_cast<int64_t>(n_rep + 1) * B;
+    perm_prefix_kernel<<<static_cast<unsigned>((warps * 32 + 255) / 256), 256, 0, stream>>>(
+        q, perm, B, gamma, n_rep, signal, eta_loc, log_eta_c, sums);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_position_metrics(const float *q, const int32_t *L, int B, int gamma, int conditional, double *bce,
+                                    double *bce_base, double *auroc, int32_t *n_pos, int32_t *n_neg,
+                                    cudaStream_t stream) {
+    metrics_kernel<<<gamma, kDiagThreads, 0, stream>>>(q, L, B, gamma, conditional, bce, bce_base, auroc, n_pos,
+                                                       n_neg);
+    return cudaGetLastError();
+}
+
+}  // namespace sdd

@@ -185,6 +185,15 @@ inline void set_divisors(ScanParams &p) {
     for (int g = 0; g < 2; ++g) p.divNpos[g] = make_fastdiv(static_cast<uint64_t>(p.grp[g].npos > 0 ? p.grp[g].npos : 1));
 }
 
+// Offline diagnostics (diag.cu).  perm: [n_rep, gamma, B] int32 scratch;
+// sums: [n_rep + 1] feasible-prefix sums (the last: the logged order).
+cudaError_t launch_perm_diag(const float *q, const int32_t *L, int B, int gamma, int signal, df eta_loc,
+                             df log_eta_c, int n_rep, uint64_t seed, int32_t *perm, unsigned long long *sums,
+                             cudaStream_t stream);
+cudaError_t launch_position_metrics(const float *q, const int32_t *L, int B, int gamma, int conditional, double *bce,
+                                    double *bce_base, double *auroc, int32_t *n_pos, int32_t *n_neg,
+                                    cudaStream_t stream);
+
 // The stand-in survival scorer (mlp.cu); *why names a host-side failure.
 cudaError_t launch_mlp(const void *h, int M, int K, const void *W1, const float *b1, const void *w2, float b2,
                        float *out, int32_t *status, cudaStream_t stream, const char **why);
