@@ -12,7 +12,9 @@
 //    rate at j), and AUROC (Mann-Whitney, ties count one half).
 //
 // perm_build_kernel  -- one CTA per (repetition, position): Fisher-Yates over
-//                       the valid blocks in shared memory, Philox draws.
+//                       the valid blocks in shared memory (order-preserving
+//                       compaction by ballots; Philox partners drawn in
+//                       parallel, the swaps in order by one thread).
 // perm_prefix_kernel -- one warp per (repetition, block): the gates of Eq. 3 on
 //                       the permuted scores (the schedule's own arithmetic),
 //                       integer sums per repetition (exact, order-free).
@@ -25,36 +27,75 @@ namespace {
 constexpr uint32_t kPurposePerm = 3;
 constexpr int kDiagThreads = 256;
 
+// Rank of block b among the blocks valid at position j (index order), for a
+// chunk of kDiagThreads consecutive blocks starting at c; n: the valid blocks
+// before the chunk, advanced past it.  Every thread of the CTA calls it.
+__device__ __forceinline__ int valid_rank(const int32_t *L, int B, int j, int conditional, int c, int &n,
+                                          int *s_wsum, bool &v) {
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    const int b = c + tid;
+    v = b < B && (!conditional || __ldg(L + b) >= j);
+    const unsigned m = __ballot_sync(0xFFFFFFFFu, v);
+    if (lane == 0) s_wsum[wid] = __popc(m);
+    __syncthreads();
+    int off = n, tot = 0;
+#pragma unroll
+    for (int u = 0; u < kDiagThreads / 32; ++u) {
+        const int x = s_wsum[u];
+        if (u < wid) off += x;
+        tot += x;
+    }
+    __syncthreads();   // s_wsum is rewritten by the next chunk
+    n += tot;
+    return off + __popc(m & ((1u << lane) - 1u));
+}
+
 __global__ void __launch_bounds__(kDiagThreads) perm_build_kernel(const int32_t *L, int B, int gamma, int n_rep,
                                                                   int conditional, uint64_t seed, int32_t *perm) {
-    extern __shared__ int32_t s_list[];   // [B]: the valid blocks, then their shuffle
+    extern __shared__ int32_t s_list[];        // [B]: the valid blocks, then their shuffle
+    __shared__ int32_t s_k[kDiagThreads];      // swap partners of the current batch of slots
+    __shared__ int s_wsum[kDiagThreads / 32];
     const int r = blockIdx.x / gamma, j = blockIdx.x % gamma;
+    const int tid = threadIdx.x;
     int32_t *row = perm + (static_cast<int64_t>(r) * gamma + j) * B;
-    __shared__ int s_n;
-    if (threadIdx.x == 0) {
-        // the valid blocks in index order (serial: the order defines the draw)
-        int n = 0;
-        for (int b = 0; b < B; ++b)
-            if (!conditional || __ldg(L + b) >= j) s_list[n++] = b;
-        // Fisher-Yates from the top: slot i swaps with k = floor(w (i + 1) / 2^32),
-        // w the first Philox word of counter (i, j, r, purpose)
-        const uint2 key = make_uint2(static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32));
-        for (int i = n - 1; i > 0; --i) {
+    // the valid blocks in index order (the order defines the draw)
+    int n = 0;
+    for (int c = 0; c < B; c += kDiagThreads) {
+        bool v;
+        const int t = valid_rank(L, B, j, conditional, c, n, s_wsum, v);
+        if (v) s_list[t] = c + tid;
+    }
+    __syncthreads();
+    // Fisher-Yates from the top: slot i swaps with k = floor(w (i + 1) / 2^32),
+    // w the first Philox word of counter (i, j, r, purpose).  The partners of
+    // kDiagThreads slots are drawn in parallel, the swaps then run in order.
+    const uint2 key = make_uint2(static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32));
+    for (int top = n - 1; top > 0; top -= kDiagThreads) {
+        const int i = top - tid;
+        if (i > 0) {
             const uint4 o = philox4x32_10(make_uint4(static_cast<uint32_t>(i), static_cast<uint32_t>(j),
                                                      static_cast<uint32_t>(r), kPurposePerm),
                                           key);
-            const int k = static_cast<int>((static_cast<uint64_t>(o.x) * static_cast<uint64_t>(i + 1)) >> 32);
-            const int32_t t = s_list[i];
-            s_list[i] = s_list[k];
-            s_list[k] = t;
+            s_k[tid] = static_cast<int32_t>((static_cast<uint64_t>(o.x) * static_cast<uint64_t>(i + 1)) >> 32);
         }
-        s_n = n;
+        __syncthreads();
+        if (tid == 0) {
+            const int cnt = min(kDiagThreads, top);   // slots top, top - 1, ..., top - cnt + 1 (all > 0)
+            for (int u = 0; u < cnt; ++u) {
+                const int a = top - u, k = s_k[u];
+                const int32_t x = s_list[a];
+                s_list[a] = s_list[k];
+                s_list[k] = x;
+            }
+        }
+        __syncthreads();
     }
-    __syncthreads();
-    // block b (t-th valid block) takes the score of block s_list[t]; others keep theirs
-    if (threadIdx.x == 0) {
-        int t = 0;
-        for (int b = 0; b < B; ++b) row[b] = (!conditional || __ldg(L + b) >= j) ? s_list[t++] : b;
+    // block b (the t-th valid block) takes the score of block s_list[t]; others keep theirs
+    n = 0;
+    for (int c = 0; c < B; c += kDiagThreads) {
+        bool v;
+        const int t = valid_rank(L, B, j, conditional, c, n, s_wsum, v);
+        if (c + tid < B) row[c + tid] = v ? s_list[t] : c + tid;
     }
 }
 
@@ -154,7 +195,7 @@ cudaError_t launch_perm_diag(const float *q, const int32_t *L, int B, int gamma,
         if (e != cudaSuccess) return e;
     }
     if (n_rep > 0) {
-        perm_build_kernel<<<n_rep * gamma, 32, smem, stream>>>(L, B, gamma, n_rep, signal == SDD_SIG_CONDITIONAL,
+        perm_build_kernel<<<n_rep * gamma, kDiagThreads, smem, stream>>>(L, B, gamma, n_rep, signal == SDD_SIG_CONDITIONAL,
                                                                seed, perm);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
