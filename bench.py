@@ -381,16 +381,17 @@ def run_component_mlp(args):
     b2 = float(b2.item())
     hs = [synth.make_hidden(M, device="cuda", round_=r) for r in range(8)]
     out = torch.empty(M, device="cuda")
+    ws = sdd.scorer_workspace(M, torch.device("cuda"))
     status = sdd.new_status(torch.device("cuda"))
     for i in range(max(args.warmup, 3)):
-        sdd.survival_mlp(hs[i % 8], W1, b1, w2, b2, out=out, status=status)
+        sdd.survival_mlp(hs[i % 8], W1, b1, w2, b2, out=out, status=status, workspace=ws)
     torch.cuda.synchronize()
     side = torch.cuda.Stream()
     side.wait_stream(torch.cuda.current_stream())
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, stream=side):
         for i in range(16):
-            sdd.survival_mlp(hs[i % 8], W1, b1, w2, b2, out=out, status=status)
+            sdd.survival_mlp(hs[i % 8], W1, b1, w2, b2, out=out, status=status, workspace=ws)
     for _ in range(3):
         g.replay()
     torch.cuda.synchronize()
@@ -449,16 +450,17 @@ def run_component_scorer(args):
     fs = [synth.make_features(M, device="cuda", round_=r) for r in range(8)]
     act = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
     out = torch.empty(M, device="cuda")
+    ws = sdd.scorer_workspace(M, torch.device("cuda"))
     status = sdd.new_status(torch.device("cuda"))
     for i in range(max(args.warmup, 3)):
-        sdd.scorer_deep(hs[i % 8], fs[i % 8], *w, act=act, out=out, status=status)
+        sdd.scorer_deep(hs[i % 8], fs[i % 8], *w, act=act, out=out, status=status, workspace=ws)
     torch.cuda.synchronize()
     side = torch.cuda.Stream()
     side.wait_stream(torch.cuda.current_stream())
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, stream=side):
         for i in range(16):
-            sdd.scorer_deep(hs[i % 8], fs[i % 8], *w, act=act, out=out, status=status)
+            sdd.scorer_deep(hs[i % 8], fs[i % 8], *w, act=act, out=out, status=status, workspace=ws)
     for _ in range(3):
         g.replay()
     torch.cuda.synchronize()

@@ -328,6 +328,15 @@ SDD_API sdd_status_t sdd_uniforms(uint64_t seed, const uint32_t *j, const uint32
                                   const uint32_t *purpose, int64_t n, float *u, sdd_stream_t stream);
 
 /*
+ * sdd_scorer_workspace_size -- bytes of device scratch that sdd_survival_mlp
+ * and sdd_scorer_deep need for M positions (512 KiB per 128 positions: the
+ * first layer's split-K partial accumulators, later the deep scorer's
+ * second-layer activations).  No zero fill is needed; calls that may overlap
+ * on the GPU need separate workspaces.
+ */
+SDD_API sdd_status_t sdd_scorer_workspace_size(int M, size_t *bytes);
+
+/*
  * sdd_survival_mlp -- a learned-style survival score per draft position (the
  * form of the scorer of App. A.7 with one hidden layer; the decode-loop
  * workload uses it with random weights as a stand-in for the trained one):
@@ -341,13 +350,18 @@ SDD_API sdd_status_t sdd_uniforms(uint64_t seed, const uint32_t *j, const uint32
  *   W1  [SDD_MLP_HIDDEN, K] bf16, row-major (one row per hidden unit), 16-byte aligned.
  *   b1  [SDD_MLP_HIDDEN] fp32; w2 [SDD_MLP_HIDDEN] bf16; b2 a host scalar.
  *   s   [M] fp32 output.
- * Needs an sm_10x device (returns SDD_ERR_UNSUPPORTED otherwise).  A bounded
- * wait that gives up sets SDD_DEV_TIMEOUT in *status (s is then undefined).
+ *   workspace  device scratch of sdd_scorer_workspace_size(M) bytes, 16-byte
+ *       aligned (SDD_ERR_INVALID_ARGUMENT if smaller).
+ * One launch: 128-position tiles, K split over a cluster of up to four CTAs
+ * whose partial products meet in the workspace.  Needs an sm_10x device
+ * (returns SDD_ERR_UNSUPPORTED otherwise).  A bounded wait that gives up sets
+ * SDD_DEV_TIMEOUT in *status (s is then undefined).
  */
 #define SDD_MLP_HIDDEN 256
 #define SDD_MLP_KSTEP 64
 SDD_API sdd_status_t sdd_survival_mlp(const void *h, int M, int K, const void *W1, const float *b1, const void *w2,
-                                      float b2, float *s, int32_t *status, sdd_stream_t stream);
+                                      float b2, float *s, void *workspace, size_t workspace_bytes, int32_t *status,
+                                      sdd_stream_t stream);
 
 /*
  * sdd_scorer_deep -- the learned scorer's shape of App. A.7 (K -> 256 -> 256 ->
@@ -368,15 +382,17 @@ SDD_API sdd_status_t sdd_survival_mlp(const void *h, int M, int K, const void *W
  *   b1, b2, b3 [SDD_MLP_HIDDEN] fp32; w4 [SDD_MLP_HIDDEN] bf16; b4 a host scalar.
  *   act  [M, SDD_MLP_HIDDEN] bf16 caller scratch (receives a1), 16-byte aligned.
  *   s    [M] fp32 output.
+ *   workspace  device scratch of sdd_scorer_workspace_size(M) bytes, 16-byte
+ *        aligned (receives the first layer's partials, then a2).
  * Two launches on the stream: the first layer (K split over a 4-CTA cluster as
- * in sdd_survival_mlp), then layers 2 and 3 and the head, one CTA per 128
- * positions with a2 kept in shared memory.  Needs an sm_10x device; a bounded
- * wait that gives up sets SDD_DEV_TIMEOUT in *status.
+ * in sdd_survival_mlp), then layers 2 and 3 and the head, a 4-CTA cluster per
+ * 128 positions (each CTA 64 of the 256 columns of both layers).  Needs an
+ * sm_10x device; a bounded wait that gives up sets SDD_DEV_TIMEOUT in *status.
  */
 SDD_API sdd_status_t sdd_scorer_deep(const void *h, int Kh, const void *f, int M, const void *W1, const float *b1,
                                      const void *W2, const float *b2, const void *W3, const float *b3,
-                                     const void *w4, float b4, void *act, float *s, int32_t *status,
-                                     sdd_stream_t stream);
+                                     const void *w4, float b4, void *act, float *s, void *workspace,
+                                     size_t workspace_bytes, int32_t *status, sdd_stream_t stream);
 
 /*
  * sdd_confidence_noalloc -- sdd_confidence without a workspace, for callers

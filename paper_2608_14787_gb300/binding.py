@@ -90,9 +90,12 @@ def load(path: str | None = None):
     L.sdd_uniforms.argtypes = [u64, VP, VP, VP, VP, i64, VP, VP]
     L.sdd_confidence_noalloc.argtypes = [VP, I, I, I, I, i64, VP, VP, VP, VP, VP, VP, VP, VP, VP]
     L.sdd_confidence_noalloc.restype = I
-    L.sdd_survival_mlp.argtypes = [VP, I, I, VP, VP, VP, ctypes.c_float, VP, VP, VP]
+    L.sdd_scorer_workspace_size.argtypes = [I, ctypes.POINTER(ctypes.c_size_t)]
+    L.sdd_scorer_workspace_size.restype = I
+    L.sdd_survival_mlp.argtypes = [VP, I, I, VP, VP, VP, ctypes.c_float, VP, VP, ctypes.c_size_t, VP, VP]
     L.sdd_survival_mlp.restype = I
-    L.sdd_scorer_deep.argtypes = [VP, I, VP, I, VP, VP, VP, VP, VP, VP, VP, ctypes.c_float, VP, VP, VP, VP]
+    L.sdd_scorer_deep.argtypes = [VP, I, VP, I, VP, VP, VP, VP, VP, VP, VP, ctypes.c_float, VP, VP, VP,
+                                  ctypes.c_size_t, VP, VP]
     L.sdd_scorer_deep.restype = I
     L.sdd_permutation_workspace_size.argtypes = [I, I, I, ctypes.POINTER(ctypes.c_size_t)]
     L.sdd_permutation_workspace_size.restype = I
@@ -349,10 +352,26 @@ MLP_HIDDEN = 256
 MLP_KSTEP = 64
 
 
-def survival_mlp(h, W1, b1, w2, b2: float, *, status=None, stream=None, out=None):
+def scorer_workspace(M, device):
+    """A device workspace for the scorers over M positions (sdd_scorer_workspace_size bytes)."""
+    nbytes = ctypes.c_size_t(0)
+    _check(load().sdd_scorer_workspace_size(int(M), ctypes.byref(nbytes)), "sdd_scorer_workspace_size")
+    return torch.empty(max(nbytes.value, 16), dtype=torch.uint8, device=device)
+
+
+def _scorer_ws(M, device, workspace):
+    if workspace is None:
+        return scorer_workspace(M, device)
+    if workspace.dtype != torch.uint8 or not workspace.is_cuda or not workspace.is_contiguous():
+        raise ValueError("workspace must be a contiguous CUDA uint8 tensor (see scorer_workspace)")
+    return workspace
+
+
+def survival_mlp(h, W1, b1, w2, b2: float, *, status=None, stream=None, out=None, workspace=None):
     """sdd_survival_mlp: sigmoid(w2 . GELU(W1 h + b1) + b2) per row of h.
     h bf16 [M, K] (or [B, gamma, K]), W1 bf16 [256, K], b1 fp32 [256], w2 bf16 [256];
-    returns fp32 scores shaped like h without its last dimension."""
+    returns fp32 scores shaped like h without its last dimension.  `workspace`:
+    from scorer_workspace(M) (allocated per call when omitted)."""
     lead = h.shape[:-1]
     K = h.shape[-1]
     h2 = h.reshape(-1, K)
@@ -364,15 +383,18 @@ def survival_mlp(h, W1, b1, w2, b2: float, *, status=None, stream=None, out=None
         raise ValueError("W1 must be [256, K], b1 and w2 [256]")
     M = h2.shape[0]
     s = torch.empty(M, dtype=torch.float32, device=h.device) if out is None else out
-    _check(load().sdd_survival_mlp(_p(h2), M, K, _p(W1), _p(b1), _p(w2), float(b2), _p(s), _p(status),
-                                   _stream(stream)), "sdd_survival_mlp")
+    ws = _scorer_ws(M, h.device, workspace)
+    _check(load().sdd_survival_mlp(_p(h2), M, K, _p(W1), _p(b1), _p(w2), float(b2), _p(s), _p(ws), ws.numel(),
+                                   _p(status), _stream(stream)), "sdd_survival_mlp")
     return s.reshape(lead)
 
 
-def scorer_deep(h, f, W1, b1, W2, b2, W3, b3, w4, b4, *, act=None, status=None, stream=None, out=None):
+def scorer_deep(h, f, W1, b1, W2, b2, W3, b3, w4, b4, *, act=None, status=None, stream=None, out=None,
+                workspace=None):
     """sdd_scorer_deep: h [..., Kh] bf16, f [..., 256] bf16 (features, zero padded),
     W1 [256, Kh + 256], W2 / W3 [256, 256], w4 [256] bf16; b1..b3 fp32 [256], b4 float.
-    Returns s with h's leading shape."""
+    Returns s with h's leading shape.  `workspace`: from scorer_workspace(M)
+    (allocated per call when omitted)."""
     lead = h.shape[:-1]
     Kh = h.shape[-1]
     h2 = h.reshape(-1, Kh).contiguous()
@@ -385,8 +407,10 @@ def scorer_deep(h, f, W1, b1, W2, b2, W3, b3, w4, b4, *, act=None, status=None, 
             raise ValueError("W2 and W3 must be [256, 256]")
     act = torch.empty(M, MLP_HIDDEN, dtype=torch.bfloat16, device=h.device) if act is None else act
     s = torch.empty(M, dtype=torch.float32, device=h.device) if out is None else out
+    ws = _scorer_ws(M, h.device, workspace)
     _check(load().sdd_scorer_deep(_p(h2), Kh, _p(f2), M, _p(W1), _p(b1), _p(W2), _p(b2), _p(W3), _p(b3), _p(w4),
-                                  float(b4), _p(act), _p(s), _p(status), _stream(stream)), "sdd_scorer_deep")
+                                  float(b4), _p(act), _p(s), _p(ws), ws.numel(), _p(status), _stream(stream)),
+           "sdd_scorer_deep")
     return s.reshape(lead)
 
 

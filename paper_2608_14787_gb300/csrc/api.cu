@@ -551,8 +551,25 @@ sdd_status_t sdd_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, c
     return SDD_OK;
 }
 
+sdd_status_t sdd_scorer_workspace_size(int M, size_t *bytes) {
+    if (!bytes) return fail(SDD_ERR_INVALID_ARGUMENT, "bytes is NULL");
+    if (M < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "M = %d < 0", M);
+    *bytes = mlp_workspace_bytes(M);
+    return SDD_OK;
+}
+
+// The scorers' workspace: present, 16-byte aligned and large enough for M rows.
+static sdd_status_t check_scorer_ws(int M, const void *workspace, size_t workspace_bytes) {
+    SDD_TRY(check_ptr16(workspace, "workspace"));
+    const size_t need = mlp_workspace_bytes(M);
+    if (workspace_bytes < need)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "workspace of %zu bytes < %zu needed", workspace_bytes, need);
+    return SDD_OK;
+}
+
 sdd_status_t sdd_survival_mlp(const void *h, int M, int K, const void *W1, const float *b1, const void *w2, float b2,
-                              float *s, int32_t *status, sdd_stream_t stream) {
+                              float *s, void *workspace, size_t workspace_bytes, int32_t *status,
+                              sdd_stream_t stream) {
     if (M < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "M = %d < 0", M);
     if (K < SDD_MLP_KSTEP || K % SDD_MLP_KSTEP != 0)
         return fail(SDD_ERR_INVALID_ARGUMENT, "K = %d is not a positive multiple of %d", K, SDD_MLP_KSTEP);
@@ -560,6 +577,7 @@ sdd_status_t sdd_survival_mlp(const void *h, int M, int K, const void *W1, const
     SDD_TRY(check_ptr16(h, "h"));
     SDD_TRY(check_ptr16(W1, "W1"));
     if (!b1 || !w2 || !s) return fail(SDD_ERR_INVALID_ARGUMENT, "b1, w2 and s must not be NULL");
+    SDD_TRY(check_scorer_ws(M, workspace, workspace_bytes));
     int d = 0;
     cudaError_t e = cudaGetDevice(&d);
     if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
@@ -568,7 +586,7 @@ sdd_status_t sdd_survival_mlp(const void *h, int M, int K, const void *W1, const
     cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, d);
     if (major != 10) return fail(SDD_ERR_UNSUPPORTED, "tcgen05 scorer needs an sm_10x device (found sm_%d%d)", major, minor);
     const char *why = nullptr;
-    e = launch_mlp(h, M, K, W1, b1, w2, b2, s, status, reinterpret_cast<cudaStream_t>(stream), &why);
+    e = launch_mlp(h, M, K, W1, b1, w2, b2, s, workspace, status, reinterpret_cast<cudaStream_t>(stream), &why);
     if (why) return fail(SDD_ERR_CUDA, "survival scorer: %s", why);
     if (e != cudaSuccess) return cuda_fail(e, "survival scorer launch");
     return SDD_OK;
@@ -576,7 +594,8 @@ sdd_status_t sdd_survival_mlp(const void *h, int M, int K, const void *W1, const
 
 sdd_status_t sdd_scorer_deep(const void *h, int Kh, const void *f, int M, const void *W1, const float *b1,
                              const void *W2, const float *b2, const void *W3, const float *b3, const void *w4,
-                             float b4, void *act, float *s, int32_t *status, sdd_stream_t stream) {
+                             float b4, void *act, float *s, void *workspace, size_t workspace_bytes,
+                             int32_t *status, sdd_stream_t stream) {
     if (M < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "M = %d < 0", M);
     if (Kh < SDD_MLP_KSTEP || Kh % SDD_MLP_KSTEP != 0)
         return fail(SDD_ERR_INVALID_ARGUMENT, "Kh = %d is not a positive multiple of %d", Kh, SDD_MLP_KSTEP);
@@ -588,6 +607,7 @@ sdd_status_t sdd_scorer_deep(const void *h, int Kh, const void *f, int M, const 
     SDD_TRY(check_ptr16(W3, "W3"));
     SDD_TRY(check_ptr16(act, "act"));
     if (!b1 || !b2 || !b3 || !w4 || !s) return fail(SDD_ERR_INVALID_ARGUMENT, "b1, b2, b3, w4 and s must not be NULL");
+    SDD_TRY(check_scorer_ws(M, workspace, workspace_bytes));
     int d = 0;
     cudaError_t e = cudaGetDevice(&d);
     if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
@@ -596,8 +616,8 @@ sdd_status_t sdd_scorer_deep(const void *h, int Kh, const void *f, int M, const 
     cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, d);
     if (major != 10) return fail(SDD_ERR_UNSUPPORTED, "tcgen05 scorer needs an sm_10x device (found sm_%d%d)", major, minor);
     const char *why = nullptr;
-    e = launch_scorer_deep(h, Kh, f, M, W1, b1, W2, b2, W3, b3, w4, b4, static_cast<uint16_t *>(act), s, status,
-                           reinterpret_cast<cudaStream_t>(stream), &why);
+    e = launch_scorer_deep(h, Kh, f, M, W1, b1, W2, b2, W3, b3, w4, b4, static_cast<uint16_t *>(act), s, workspace,
+                           status, reinterpret_cast<cudaStream_t>(stream), &why);
     if (why) return fail(SDD_ERR_CUDA, "deep scorer: %s", why);
     if (e != cudaSuccess) return cuda_fail(e, "deep scorer launch");
     return SDD_OK;

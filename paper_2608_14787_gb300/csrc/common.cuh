@@ -322,6 +322,11 @@ __device__ __forceinline__ uint32_t atom_add_acq_rel_gpu(uint32_t *addr, uint32_
 // and its memory operations are visible (a no-op for an ordinary launch).
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Lets the grid launched behind this one be scheduled once every CTA of this
+// grid has called it or exited (its griddep_wait still waits for completion).
+__device__ __forceinline__ void griddep_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
 
 // Launch `kernel` behind the previous work of `stream` as a programmatic
 // dependent grid (host side).

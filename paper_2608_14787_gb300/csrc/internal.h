@@ -194,14 +194,17 @@ cudaError_t launch_position_metrics(const float *q, const int32_t *L, int B, int
                                     double *bce_base, double *auroc, int32_t *n_pos, int32_t *n_neg,
                                     cudaStream_t stream);
 
+// Device scratch of the scorers (mlp.cu) for M rows: the split-K partials of
+// the first layer, later the deep scorer's second-layer activations.
+size_t mlp_workspace_bytes(int M);
 // The stand-in survival scorer (mlp.cu); *why names a host-side failure.
 cudaError_t launch_mlp(const void *h, int M, int K, const void *W1, const float *b1, const void *w2, float b2,
-                       float *out, int32_t *status, cudaStream_t stream, const char **why);
+                       float *out, void *ws, int32_t *status, cudaStream_t stream, const char **why);
 // The deep scorer (mlp.cu): layer 1 over [h | f] into act, then layers 2, 3 and the head.
 cudaError_t launch_scorer_deep(const void *h, int Kh, const void *f, int M, const void *W1, const float *b1,
                                const void *W2, const float *b2, const void *W3, const float *b3, const void *w4,
-                               float b4, uint16_t *act, float *out, int32_t *status, cudaStream_t stream,
-                               const char **why);
+                               float b4, uint16_t *act, float *out, void *ws, int32_t *status,
+                               cudaStream_t stream, const char **why);
 int scan_max_ctas_per_sm();
 int decide_max_ctas_per_sm();
 cudaError_t scan_prepare_device();

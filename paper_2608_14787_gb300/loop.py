@@ -84,6 +84,7 @@ class DecodeLoop:
             self.b2 = float(b2.item())
         else:
             raise ValueError(f"scorer {scorer!r}: 'deep' or 'mlp'")
+        self.scorer_ws = sdd.scorer_workspace(B * gamma, dev)
 
     def features(self, conf, round_: int) -> torch.Tensor:
         """The scorer's scalar-feature block [B * gamma, 256] bf16 (19 columns,
@@ -107,10 +108,11 @@ class DecodeLoop:
         deep = self.scorer == "deep"
         conf = sdd.confidence(z_d, x, ws=self.ws, status=self.status, features=deep)
         if deep:
-            s = sdd.scorer_deep(h, self.features(conf, round_), *self.deep, act=self.act,
-                                status=self.status).reshape(B, gamma)
+            s = sdd.scorer_deep(h, self.features(conf, round_), *self.deep, act=self.act, status=self.status,
+                                workspace=self.scorer_ws).reshape(B, gamma)
         else:
-            s = sdd.survival_mlp(h, self.W1, self.b1, self.w2, self.b2, status=self.status).reshape(B, gamma)
+            s = sdd.survival_mlp(h, self.W1, self.b1, self.w2, self.b2, status=self.status,
+                                 workspace=self.scorer_ws).reshape(B, gamma)
         _, K_raw, D_raw = sdd.schedule_prefix(conf.q, [self.tau], [self.tau], signal=sdd.SIG_RAW, logq=conf.logq,
                                               K_min=self.K_min, S_max=self.S_max, D_in=self.D_raw,
                                               status=self.status)

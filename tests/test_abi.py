@@ -96,6 +96,26 @@ def test_invalid_arguments_rejected_on_host(lib):
     assert rc == 1 and b"n_rows" in lib.sdd_last_error()
 
 
+def test_scorer_workspace_size_and_check(lib):
+    # 512 KiB per started 128-position tile: four split-K partials of 128 x 256 fp32
+    n = ctypes.c_size_t(0)
+    for M, tiles in ((0, 0), (1, 1), (128, 1), (129, 2), (4096, 32)):
+        assert lib.sdd_scorer_workspace_size(M, ctypes.byref(n)) == 0
+        assert n.value == tiles * 4 * 256 * 128 * 4
+    assert lib.sdd_scorer_workspace_size(-1, ctypes.byref(n)) == 1
+    assert lib.sdd_scorer_workspace_size(4, None) == 1
+    # a workspace one byte short, or missing, is rejected before any CUDA call
+    VP = ctypes.c_void_p
+    need = 2 * 4 * 256 * 128 * 4
+    rc = lib.sdd_survival_mlp(VP(16), 129, 64, VP(16), VP(16), VP(16), 0.0, VP(16), VP(256), need - 1, None, None)
+    assert rc == 1 and b"workspace" in lib.sdd_last_error()
+    rc = lib.sdd_survival_mlp(VP(16), 129, 64, VP(16), VP(16), VP(16), 0.0, VP(16), None, need, None, None)
+    assert rc == 1 and b"workspace" in lib.sdd_last_error()
+    rc = lib.sdd_scorer_deep(VP(16), 64, VP(16), 129, VP(16), VP(16), VP(16), VP(16), VP(16), VP(16), VP(16), 0.0,
+                             VP(16), VP(16), VP(256), need - 1, None, None)
+    assert rc == 1 and b"workspace" in lib.sdd_last_error()
+
+
 def test_empty_batch_is_a_no_op(lib):
     VP = ctypes.c_void_p
     # B = 0 returns before touching the device or the workspace
