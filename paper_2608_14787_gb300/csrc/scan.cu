@@ -232,13 +232,14 @@ __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lan
             st.r = rn;
         }
     }
-    // pass 2: the exp-sums, two vectors per step re-read from shared memory
-    // (a bounded register footprint)
+    // pass 2: the exp-sums, the vectors re-read from shared memory two at a
+    // time; unrolled, so the reads of later steps issue ahead of the
+    // arithmetic of earlier ones
     const float nr = -st.r;
     const f2_t L2 = f2_pack(kLog2e, kLog2e), NR = f2_pack(nr, nr);
     f2_t sa = f2_pack(0.f, 0.f), sb = sa, ta = sa, tb = sa;
     constexpr int PAIRS = (DT == SDD_BF16) ? 4 : 2;   // entry pairs per 16-byte vector
-#pragma unroll 1
+#pragma unroll
     for (int i = 0; i < kVPL; i += 2) {
         uint4 w[2];
         w[0] = tile[lane + 32 * i];
