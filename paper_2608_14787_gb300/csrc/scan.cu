@@ -280,74 +280,127 @@ __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lan
     return cm;
 }
 
-// The warp's five largest clamped entries of the piece so far, t[0] >= ... >=
-// t[4] (warp-uniform, with multiplicity), updated with a (full, padded) tile;
-// vmax holds the maxima of the lane's vectors.  Only entries above t[4] change
-// the list (an entry equal to t[4] changes none of its values); on the
-// piece's first tile the list is empty and the candidates are the entries at
-// or above the fifth largest vector maximum of the warp (five entries reach
-// it, so no smaller entry is in the list).  The vectors holding candidates are
-// visited one at a time, every lane reading the visited vector from shared
-// memory, so the list stays identical in all lanes.
-template <int DT>
-__device__ __forceinline__ void top5_tile(const uint4 *tile, int lane, const uint32_t (&vmax)[kVPL], float (&t)[5]) {
+// Extended features (drafter rows): the five largest clamped entries of a
+// piece, with multiplicity.  A group is one lane's kVPL vectors of one tile.
+// The five largest entries lie in the five groups with the largest maxima:
+// every other group's maximum is at most the fifth largest group maximum,
+// which those five groups' maxima reach, so an entry outside them can only
+// tie the fifth largest entry.  While the piece streams, each lane keeps its
+// five largest tile maxima (order-preserving integer keys) with the tiles'
+// first vectors -- one compare per tile; at the piece's end the warp merges
+// the lanes' lists (five integer max reductions), re-reads the five groups
+// (40 vectors) from global memory and takes their five largest entries.
+__device__ __forceinline__ uint32_t fkey(float f) {
+    const uint32_t u = __float_as_uint(f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float fkey_inv(uint32_t k) {
+    return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
+}
+
+// The lane's tile maximum cm of the tile starting at row vector k0 into its
+// list (ck descending, ct the tiles; key 0 = empty).
+__device__ __forceinline__ void group_update(float cm, int k0, uint32_t (&ck)[5], int (&ct)[5]) {
+    uint32_t key = fkey(cm);
+    if (key <= ck[4]) return;
+    int k = k0;
+#pragma unroll
+    for (int j = 0; j < 5; ++j)
+        if (key > ck[j]) {
+            const uint32_t tk = ck[j];
+            const int tt = ct[j];
+            ck[j] = key;
+            ct[j] = k;
+            key = tk;
+            k = tt;
+        }
+}
+
+// The five largest clamped entries (descending; -inf where the piece has
+// fewer) of the piece [kb, ke) of row rowp, warp-uniform, from the lanes'
+// group lists.  The 40 vectors of the five groups are loaded (two per lane)
+// before `between` runs, so their round trip overlaps whatever it waits on.
+template <int DT, class Between>
+__device__ __forceinline__ void group_top5(const char *rowp, int kb, int ke, int V, int lane, uint32_t (&ck)[5],
+                                           int (&ct)[5], float (&t)[5], Between between) {
     constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
-    float vm[kVPL];
+    // (the rounds are rolled loops shifting their results in: this code runs
+    // once per piece, and its instructions are fetched while L2 is busy)
+    int gl[5], gk[5];   // the five groups: lane and tile
 #pragma unroll
-    for (int i = 0; i < kVPL; ++i)
-        vm[i] = (DT == SDD_BF16) ? fmaxf(bf16_lo(vmax[i]), bf16_hi(vmax[i])) : __uint_as_float(vmax[i]);
-    const bool first = t[0] == -INFINITY;
-    float thr = t[4];
-    if (first) {
-        // the fifth largest vector maximum of the warp (the lane's largest first)
-        float c[kVPL];
-#pragma unroll
-        for (int i = 0; i < kVPL; ++i) c[i] = vm[i];
+    for (int k = 0; k < 5; ++k) {
+        gl[k] = 0;
+        gk[k] = -1;
+        t[k] = -INFINITY;
+    }
 #pragma unroll 1
-        for (int k = 0; k < 5; ++k) {
-            float lm = c[0];
+    for (int k = 0; k < 5; ++k) {
+        const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, ck[0]);
+        const int owner = __ffs(__ballot_sync(0xFFFFFFFFu, ck[0] == m)) - 1;
+        const int tile = __shfl_sync(0xFFFFFFFFu, ct[0], owner);   // -1 when every list is empty
 #pragma unroll
-            for (int i = 1; i < kVPL; ++i) lm = fmaxf(lm, c[i]);
-            asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(thr) : "f"(lm));
-            const int L = __ffs(__ballot_sync(0xFFFFFFFFu, lm == thr)) - 1;
-            if (lane == L) {
-                bool done = false;
+        for (int j = 0; j < 4; ++j) {
+            gl[j] = gl[j + 1];
+            gk[j] = gk[j + 1];
+        }
+        gl[4] = owner;
+        gk[4] = tile;
+        if (lane == owner) {
 #pragma unroll
-                for (int i = 0; i < kVPL; ++i)
-                    if (!done && c[i] == thr) {
-                        c[i] = -INFINITY;
-                        done = true;
-                    }
+            for (int j = 0; j < 4; ++j) {
+                ck[j] = ck[j + 1];
+                ct[j] = ct[j + 1];
             }
+            ck[4] = 0u;
+            ct[4] = -1;
         }
     }
-    uint32_t vmask = 0;   // the lane's vectors holding candidates
+    // vector u (0..39) of the groups: group u / 8, its (u % 8)-th vector;
+    // lane q takes u = q and u = q + 32
+    int vec[2];
+    uint4 w[2];
 #pragma unroll
-    for (int i = 0; i < kVPL; ++i)
-        if (first ? vm[i] >= thr : vm[i] > thr) vmask |= 1u << i;
-#pragma unroll 1
-    for (int guard = 0; guard < 32 * kVPL; ++guard) {
-        const unsigned who = __ballot_sync(0xFFFFFFFFu, vmask != 0);
-        if (!who) break;
-        const int L = __ffs(who) - 1;
-        int iv = 0;
-        if (lane == L) {
-            iv = __ffs(vmask) - 1;
-            vmask &= vmask - 1;
-        }
-        iv = __shfl_sync(0xFFFFFFFFu, iv, L);
-        const uint4 w = clamp_vec<DT>(tile[L + 32 * iv]);
+    for (int h = 0; h < 2; ++h) {
+        const int u = lane + 32 * h;
+        const int g = u >> 3, j = u & 7;
+        int gk_ = -1, gl_ = 0;
 #pragma unroll
-        for (int e = 0; e < EPV; ++e) {
-            float z = vec_elem<DT>(w, e);
-            if (z > t[4]) {
-#pragma unroll
-                for (int k = 0; k < 5; ++k) {   // insert z into the descending list
-                    const float hi = fmaxf(t[k], z), lo = fminf(t[k], z);
-                    t[k] = hi;
-                    z = lo;
-                }
+        for (int k = 0; k < 5; ++k)
+            if (g == k) {
+                gk_ = gk[k];
+                gl_ = gl[k];
             }
+        const int v = (gk_ >= 0) ? gk_ + gl_ + 32 * j : -1;
+        vec[h] = (u < 40 && v >= kb && v < ke) ? v : -1;
+        w[h] = (vec[h] >= 0) ? __ldg(reinterpret_cast<const uint4 *>(rowp) + vec[h]) : make_uint4(0, 0, 0, 0);
+    }
+    between();
+    float e[2 * EPV];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const uint4 c = clamp_vec<DT>(w[h]);
+#pragma unroll
+        for (int j = 0; j < EPV; ++j)
+            e[h * EPV + j] = (vec[h] >= 0 && vec[h] * EPV + j < V) ? vec_elem<DT>(c, j) : -INFINITY;
+    }
+#pragma unroll 1
+    for (int k = 0; k < 5; ++k) {   // five rounds: the warp's largest remaining entry
+        float lm = e[0];
+#pragma unroll
+        for (int j = 1; j < 2 * EPV; ++j) lm = fmaxf(lm, e[j]);
+        const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, fkey(lm));
+#pragma unroll
+        for (int j = 0; j < 4; ++j) t[j] = t[j + 1];
+        t[4] = fkey_inv(m);
+        const int owner = __ffs(__ballot_sync(0xFFFFFFFFu, fkey(lm) == m)) - 1;
+        if (lane == owner) {
+            bool done = false;
+#pragma unroll
+            for (int j = 0; j < 2 * EPV; ++j)
+                if (!done && fkey(e[j]) == m) {
+                    e[j] = -INFINITY;
+                    done = true;
+                }
         }
     }
 }
@@ -437,7 +490,9 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
     float gA = token_logit<DT>(p, cc.r, tokA);
 
     SoftState st = soft_identity();
-    float top[5];          // FEAT: the warp's five largest entries of the piece (drafter rows)
+    uint32_t ck[5];        // FEAT: the lane's five largest tile maxima of the piece (keys) ...
+    int ct[5];             // ... and their tiles' first vectors (drafter rows)
+    int kb = 0;            // FEAT: the piece's first vector in the row
     float s_hi = 0.f, s_lo = 0.f;   // the lane's exp-sum as an fp32 pair
     bool in_piece = false;
     bool ent = false;      // warp-uniform: drafter row (entropy accumulator, clamped entries)
@@ -455,7 +510,11 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
             st = soft_identity();
             if (FEAT) {
 #pragma unroll
-                for (int k = 0; k < 5; ++k) top[k] = -INFINITY;
+                for (int k = 0; k < 5; ++k) {
+                    ck[k] = 0u;
+                    ct[k] = -1;
+                }
+                kb = cc.k;
             }
             s_hi = 0.f;
             s_lo = 0.f;
@@ -486,9 +545,9 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
         const bool row_end = (cc.k + n == p.RV);
         if (n < kTileVec || (row_end && tail)) pad_tile<DT>(tile, n, lane, row_end, tail);
         uint32_t vmax[kVPL];
-        const float cm = ent ? process_tile<DT, true, FEAT>(tile, cc.k, lane, st, s_hi, s_lo, vmax)
+        const float cm = ent ? process_tile<DT, true, false>(tile, cc.k, lane, st, s_hi, s_lo, vmax)
                              : process_tile<DT, false, false>(tile, cc.k, lane, st, s_hi, s_lo, vmax);
-        if (FEAT && ent && __any_sync(0xFFFFFFFFu, cm > top[4])) top5_tile<DT>(tile, lane, vmax, top);
+        if (FEAT && ent) group_update(cm, cc.k, ck, ct);
         if (rank_on) {
             const bool want = cm >= g;
             if (__any_sync(0xFFFFFFFFu, want)) {
@@ -514,18 +573,27 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) M = fmax_nan(M, __shfl_xor_sync(0xFFFFFFFFu, M, off));
             int idx = INT32_MAX;
-            if (st.m == M && st.amax != INT32_MAX) idx = first_index<DT>(crow, st.amax, lane, p.RV, p.V, M);
+            auto resolve = [&]() {
+                if (st.m == M && st.amax != INT32_MAX) idx = first_index<DT>(crow, st.amax, lane, p.RV, p.V, M);
+            };
+            float top[5];
+            if (FEAT && ent)
+                group_top5<DT>(crow, kb, cc.k, p.V, lane, ck, ct, top, resolve);   // (cc.k: the piece's end)
+            else
+                resolve();
             st.amax = idx;
             st.rank = (lane == 0) ? wrank : 0;
             st.sh = s_hi;
             st.sl = s_lo;
             const SoftState red = soft_warp_reduce(st);
-            if (FEAT && ent && lane == 0) {
+            if (FEAT && ent) {
+                if (lane == 0) {
                 FeatPartial fp;
 #pragma unroll
                 for (int k = 0; k < 5; ++k) fp.top[k] = top[k];
                 fp.pad[0] = fp.pad[1] = fp.pad[2] = 0.f;
                 p.feat[cc.r + gw] = fp;
+                }
             }
             if (lane == 0) {
                 Partial pt;
