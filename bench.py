@@ -41,9 +41,9 @@ UNIT = "blocks/s"
 EV_EVERY = 8   # steps between the event-bracketed launches of the streaming kernel
 NEAR = 1e-6
 # dram__bytes_read.sum + dram__bytes_write.sum of one scan_kernel launch on the
-# c3 workload (318.22 MB + 3.34 MB), from one ncu capture of the kernel as it
+# c3 workload (318.23 MB + 3.48 MB), from one ncu capture of the kernel as it
 # stands; reported as the roofline's "traffic" for that workload only.
-SCAN_TRAFFIC_C3 = 321_560_320
+SCAN_TRAFFIC_C3 = 321_710_336
 
 
 def _peaks():

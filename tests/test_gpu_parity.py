@@ -423,3 +423,31 @@ def test_features_fp32_padded_rows(sdd):
     z_d, _, x = _to_dev(blk)
     z_d = _padded(z_d, 4004)
     _check_features(sdd, z_d, x, torch.float32)
+
+
+@pytest.mark.parametrize("V", [151936, 20003])
+def test_features_planted_top5_layouts(sdd, V):
+    """The five largest entries placed where the selection of lane-tile groups
+    (a lane's 8 vectors of one tile) is tested: all five in one 16-byte vector,
+    one per 2048-entry tile, in the row's last (partial) vector, four tied
+    below the maximum in different groups, and a row whose maximum ties six
+    times (one tie outside the five selected groups)."""
+    blk = synth.make_block("c3", device="cpu", B=2, gamma=6, V=V)
+    z_d, _, x = _to_dev(blk)
+    z_d = z_d.clone()
+    top = 30.0
+    r = z_d[0]
+    r[0, 1000:1005] = torch.tensor([top, top - 1, top - 2, top - 3, top - 4])     # one vector (8-aligned start)
+    for k in range(5):
+        r[1, k * 2048 + 37 * k] = top - k                                              # one per tile
+    r[2, V - 5:] = torch.tensor([top - 4, top - 3, top - 2, top - 1, top])        # the row's end
+    r[3, 3] = top
+    for k, pos in enumerate((9000, 17000, 41000 % V, 77000 % V)):
+        r[3, pos] = top - 1                                                          # ties below the max
+    for k in range(6):
+        r[4, 3000 * k + 5] = top                                                     # the maximum six times
+    r[5, :] = r[5].clamp(max=0.0)
+    r[5, 123] = 1.0                                                                  # a single positive entry
+    if V % 8:
+        z_d = _padded(z_d, (V + 7) // 8 * 8)
+    _check_features(sdd, z_d, x, torch.bfloat16)
