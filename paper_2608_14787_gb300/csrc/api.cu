@@ -627,7 +627,7 @@ sdd_status_t sdd_permutation_workspace_size(int B, int gamma, int n_rep, size_t 
     if (!bytes) return fail(SDD_ERR_INVALID_ARGUMENT, "bytes is NULL");
     if (B < 0 || gamma < 1 || gamma > SDD_MAX_GAMMA || n_rep < 0)
         return fail(SDD_ERR_INVALID_ARGUMENT, "B = %d, gamma = %d, n_rep = %d out of range", B, gamma, n_rep);
-    *bytes = align256(static_cast<size_t>(n_rep) * gamma * B * sizeof(int32_t)) +
+    *bytes = align256(static_cast<size_t>(n_rep) * gamma * B * sizeof(float)) +
              align256(static_cast<size_t>(n_rep + 1) * sizeof(unsigned long long));
     return SDD_OK;
 }
@@ -653,11 +653,11 @@ sdd_status_t sdd_permutation_diagnostic(const float *q, const int32_t *L, int B,
         return e == cudaSuccess ? SDD_OK : cuda_fail(e, "memset");
     }
     unsigned char *base = static_cast<unsigned char *>(workspace);
-    int32_t *perm = reinterpret_cast<int32_t *>(base);
+    float *pq = reinterpret_cast<float *>(base);   // the permuted scores, [n_rep][gamma][B]
     unsigned long long *acc = reinterpret_cast<unsigned long long *>(
-        base + align256(static_cast<size_t>(n_rep) * gamma * B * sizeof(int32_t)));
+        base + align256(static_cast<size_t>(n_rep) * gamma * B * sizeof(float)));
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    cudaError_t e = launch_perm_diag(q, L, B, gamma, signal, eta_loc, log_eta_c, n_rep, seed, perm, acc, st);
+    cudaError_t e = launch_perm_diag(q, L, B, gamma, signal, eta_loc, log_eta_c, n_rep, seed, pq, acc, st);
     if (e != cudaSuccess) return cuda_fail(e, "permutation diagnostic launch");
     e = cudaMemcpyAsync(sums, acc, sizeof(int64_t) * (n_rep + 1), cudaMemcpyDeviceToDevice, st);
     return e == cudaSuccess ? SDD_OK : cuda_fail(e, "copy");

@@ -14,7 +14,9 @@
 // perm_build_kernel  -- one CTA per (repetition, position): Fisher-Yates over
 //                       the valid blocks in shared memory (order-preserving
 //                       compaction by ballots; Philox partners drawn in
-//                       parallel, the swaps in order by one thread).
+//                       parallel, the swaps in order by one thread; 64
+//                       threads, so that 32 CTAs interleave on an SM); it
+//                       writes the permuted scores of its position.
 // perm_prefix_kernel -- one warp per (repetition, block): the gates of Eq. 3 on
 //                       the permuted scores (the schedule's own arithmetic),
 //                       integer sums per repetition (exact, order-free).
@@ -26,51 +28,71 @@ namespace {
 
 constexpr uint32_t kPurposePerm = 3;
 constexpr int kDiagThreads = 256;
+// The permutation builder's CTAs are small so that 32 of them share an SM:
+// each spends most of its time in one thread's serial swap loop, and the SM
+// interleaves those loops.
+constexpr int kPermThreads = 64;
 
-// Rank of block b among the blocks valid at position j (index order), for a
-// chunk of kDiagThreads consecutive blocks starting at c; n: the valid blocks
-// before the chunk, advanced past it.  Every thread of the CTA calls it.
-__device__ __forceinline__ int valid_rank(const int32_t *L, int B, int j, int conditional, int c, int &n,
-                                          int *s_wsum, bool &v) {
-    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-    const int b = c + tid;
-    v = b < B && (!conditional || __ldg(L + b) >= j);
-    const unsigned m = __ballot_sync(0xFFFFFFFFu, v);
-    if (lane == 0) s_wsum[wid] = __popc(m);
-    __syncthreads();
-    int off = n, tot = 0;
-#pragma unroll
-    for (int u = 0; u < kDiagThreads / 32; ++u) {
-        const int x = s_wsum[u];
-        if (u < wid) off += x;
-        tot += x;
-    }
-    __syncthreads();   // s_wsum is rewritten by the next chunk
-    n += tot;
-    return off + __popc(m & ((1u << lane) - 1u));
+// Shared memory of the permutation builder for B logged blocks: the block
+// list [B], the validity bits of position j [ceil(B/32) words] and their
+// exclusive prefix popcounts [ceil(B/32)].
+__host__ __device__ inline size_t perm_smem_bytes(int B) {
+    const size_t words = (static_cast<size_t>(B) + 31) / 32;
+    return (static_cast<size_t>(B) + 2 * words) * sizeof(int32_t);
 }
 
-__global__ void __launch_bounds__(kDiagThreads) perm_build_kernel(const int32_t *L, int B, int gamma, int n_rep,
-                                                                  int conditional, uint64_t seed, int32_t *perm) {
-    extern __shared__ int32_t s_list[];        // [B]: the valid blocks, then their shuffle
-    __shared__ int32_t s_k[kDiagThreads];      // swap partners of the current batch of slots
-    __shared__ int s_wsum[kDiagThreads / 32];
+__global__ void __launch_bounds__(kPermThreads) perm_build_kernel(const float *q, const int32_t *L, int B, int gamma,
+                                                                  int n_rep, int conditional, uint64_t seed,
+                                                                  float *pq) {
+    extern __shared__ int32_t s_dyn[];
+    int32_t *s_list = s_dyn;                                               // the valid blocks, then their shuffle
+    uint32_t *s_mask = reinterpret_cast<uint32_t *>(s_dyn + B);            // validity bits
+    int32_t *s_wpre = s_dyn + B + (B + 31) / 32;                           // valid blocks before each word
+    __shared__ __align__(16) int32_t s_k[kPermThreads];   // swap partners of the current batch of slots
+    __shared__ int s_n;
     const int r = blockIdx.x / gamma, j = blockIdx.x % gamma;
-    const int tid = threadIdx.x;
-    int32_t *row = perm + (static_cast<int64_t>(r) * gamma + j) * B;
+    const int tid = threadIdx.x, lane = tid & 31;
+    const int words = (B + 31) / 32;
+    float *row = pq + (static_cast<int64_t>(r) * gamma + j) * B;
+    // validity bits (the loads of several chunks in flight together)
+#pragma unroll 4
+    for (int c = 0; c < B; c += kPermThreads) {
+        const int b = c + tid;
+        const bool v = b < B && (!conditional || __ldg(L + b) >= j);
+        const unsigned m = __ballot_sync(0xFFFFFFFFu, v);
+        if (lane == 0 && b < B) s_mask[b >> 5] = m;   // (b: the warp's first block, a multiple of 32)
+    }
+    __syncthreads();
+    // exclusive prefix popcounts of the words (one warp)
+    if (tid < 32) {
+        int carry = 0;
+        for (int w0 = 0; w0 < words; w0 += 32) {
+            const int w = w0 + lane;
+            const int c = (w < words) ? __popc(s_mask[w]) : 0;
+            int incl = c;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const int t = __shfl_up_sync(0xFFFFFFFFu, incl, off);
+                if (lane >= off) incl += t;
+            }
+            if (w < words) s_wpre[w] = carry + incl - c;
+            carry += __shfl_sync(0xFFFFFFFFu, incl, 31);
+        }
+        if (lane == 0) s_n = carry;
+    }
+    __syncthreads();
+    const int n = s_n;
     // the valid blocks in index order (the order defines the draw)
-    int n = 0;
-    for (int c = 0; c < B; c += kDiagThreads) {
-        bool v;
-        const int t = valid_rank(L, B, j, conditional, c, n, s_wsum, v);
-        if (v) s_list[t] = c + tid;
+    for (int b = tid; b < B; b += kPermThreads) {
+        const uint32_t m = s_mask[b >> 5], bit = 1u << (b & 31);
+        if (m & bit) s_list[s_wpre[b >> 5] + __popc(m & (bit - 1u))] = b;
     }
     __syncthreads();
     // Fisher-Yates from the top: slot i swaps with k = floor(w (i + 1) / 2^32),
     // w the first Philox word of counter (i, j, r, purpose).  The partners of
-    // kDiagThreads slots are drawn in parallel, the swaps then run in order.
+    // kPermThreads slots are drawn in parallel, the swaps then run in order.
     const uint2 key = make_uint2(static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32));
-    for (int top = n - 1; top > 0; top -= kDiagThreads) {
+    for (int top = n - 1; top > 0; top -= kPermThreads) {
         const int i = top - tid;
         if (i > 0) {
             const uint4 o = philox4x32_10(make_uint4(static_cast<uint32_t>(i), static_cast<uint32_t>(j),
@@ -80,26 +102,39 @@ __global__ void __launch_bounds__(kDiagThreads) perm_build_kernel(const int32_t 
         }
         __syncthreads();
         if (tid == 0) {
-            const int cnt = min(kDiagThreads, top);   // slots top, top - 1, ..., top - cnt + 1 (all > 0)
-            for (int u = 0; u < cnt; ++u) {
-                const int a = top - u, k = s_k[u];
-                const int32_t x = s_list[a];
-                s_list[a] = s_list[k];
-                s_list[k] = x;
+            // slots top, top - 1, ..., top - cnt + 1 (all > 0); x carries the
+            // value at slot a, re-read after each swap (which may have written
+            // slot a - 1), so one shared-memory round trip bounds an iteration;
+            // the partners come four at a time
+            const int cnt = min(kPermThreads, top);
+            int32_t x = s_list[top];
+            for (int u = 0; u < cnt; u += 4) {
+                const int4 kk = *reinterpret_cast<const int4 *>(s_k + u);
+                const int ks[4] = {kk.x, kk.y, kk.z, kk.w};
+#pragma unroll
+                for (int h = 0; h < 4; ++h) {
+                    if (u + h >= cnt) break;
+                    const int a = top - u - h, k = ks[h];
+                    const int32_t y = (k == a) ? x : s_list[k];
+                    s_list[k] = x;
+                    s_list[a] = y;
+                    x = s_list[a - 1];
+                }
             }
         }
         __syncthreads();
     }
-    // block b (the t-th valid block) takes the score of block s_list[t]; others keep theirs
-    n = 0;
-    for (int c = 0; c < B; c += kDiagThreads) {
-        bool v;
-        const int t = valid_rank(L, B, j, conditional, c, n, s_wsum, v);
-        if (c + tid < B) row[c + tid] = v ? s_list[t] : c + tid;
+    // block b (the t-th valid block) takes the score of block s_list[t]; others
+    // keep theirs: the permuted scores of position j, gathered here so that the
+    // prefix kernel reads each with one load
+    for (int b = tid; b < B; b += kPermThreads) {
+        const uint32_t m = s_mask[b >> 5], bit = 1u << (b & 31);
+        const int src = (m & bit) ? s_list[s_wpre[b >> 5] + __popc(m & (bit - 1u))] : b;
+        row[b] = __ldg(q + static_cast<int64_t>(src) * gamma + j);
     }
 }
 
-__global__ void perm_prefix_kernel(const float *q, const int32_t *perm, int B, int gamma, int n_rep, int signal,
+__global__ void perm_prefix_kernel(const float *q, const float *pq, int B, int gamma, int n_rep, int signal,
                                    df eta_loc, df log_eta_c, unsigned long long *sums) {
     const int lane = threadIdx.x & 31;
     const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
@@ -110,9 +145,9 @@ __global__ void perm_prefix_kernel(const float *q, const int32_t *perm, int B, i
     for (int c = 0; c < gamma && kb >= c; c += 32) {
         const int j = c + lane;
         const bool in = j < gamma;
-        int src = b;
-        if (in && r < n_rep) src = __ldg(perm + (static_cast<int64_t>(r) * gamma + j) * B + b);
-        const float qj = in ? __ldg(q + static_cast<int64_t>(src) * gamma + j) : 0.f;
+        const float qj = !in ? 0.f
+                         : (r < n_rep) ? __ldg(pq + (static_cast<int64_t>(r) * gamma + j) * B + b)
+                                       : __ldg(q + static_cast<int64_t>(b) * gamma + j);
         const float lq = in ? logf(qj) : 0.f;
         const df S = df_add(carry, warp_prefix_df(df{lq, 0.f}, lane));
         carry.hi = __shfl_sync(0xFFFFFFFFu, S.hi, 31);
@@ -184,25 +219,25 @@ __global__ void __launch_bounds__(kDiagThreads) metrics_kernel(const float *q, c
 }  // namespace
 
 cudaError_t launch_perm_diag(const float *q, const int32_t *L, int B, int gamma, int signal, df eta_loc,
-                             df log_eta_c, int n_rep, uint64_t seed, int32_t *perm, unsigned long long *sums,
+                             df log_eta_c, int n_rep, uint64_t seed, float *pq, unsigned long long *sums,
                              cudaStream_t stream) {
     cudaError_t e = cudaMemsetAsync(sums, 0, sizeof(unsigned long long) * (n_rep + 1), stream);
     if (e != cudaSuccess) return e;
-    const size_t smem = static_cast<size_t>(B) * sizeof(int32_t);
+    const size_t smem = perm_smem_bytes(B);
     if (smem > 48 * 1024) {
         e = cudaFuncSetAttribute(perm_build_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  static_cast<int>(smem));
         if (e != cudaSuccess) return e;
     }
     if (n_rep > 0) {
-        perm_build_kernel<<<n_rep * gamma, kDiagThreads, smem, stream>>>(L, B, gamma, n_rep, signal == SDD_SIG_CONDITIONAL,
-                                                               seed, perm);
+        perm_build_kernel<<<n_rep * gamma, kPermThreads, smem, stream>>>(q, L, B, gamma, n_rep,
+                                                                        signal == SDD_SIG_CONDITIONAL, seed, pq);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
     const int64_t warps = static_cast<int64_t>(n_rep + 1) * B;
     perm_prefix_kernel<<<static_cast<unsigned>((warps * 32 + 255) / 256), 256, 0, stream>>>(
-        q, perm, B, gamma, n_rep, signal, eta_loc, log_eta_c, sums);
+        q, pq, B, gamma, n_rep, signal, eta_loc, log_eta_c, sums);
     return cudaGetLastError();
 }
 

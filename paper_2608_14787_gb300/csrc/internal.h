@@ -188,7 +188,7 @@ inline void set_divisors(ScanParams &p) {
 // Offline diagnostics (diag.cu).  perm: [n_rep, gamma, B] int32 scratch;
 // sums: [n_rep + 1] feasible-prefix sums (the last: the logged order).
 cudaError_t launch_perm_diag(const float *q, const int32_t *L, int B, int gamma, int signal, df eta_loc,
-                             df log_eta_c, int n_rep, uint64_t seed, int32_t *perm, unsigned long long *sums,
+                             df log_eta_c, int n_rep, uint64_t seed, float *pq, unsigned long long *sums,
                              cudaStream_t stream);
 cudaError_t launch_position_metrics(const float *q, const int32_t *L, int B, int gamma, int conditional, double *bce,
                                     double *bce_base, double *auroc, int32_t *n_pos, int32_t *n_neg,
