@@ -328,6 +328,25 @@ SDD_API sdd_status_t sdd_uniforms(uint64_t seed, const uint32_t *j, const uint32
                                   const uint32_t *purpose, int64_t n, float *u, sdd_stream_t stream);
 
 /*
+ * sdd_scorer_features -- the scalar-feature block of the learned scorer's input
+ * (the feature list of App. A.7) for B*gamma drafter positions, in the column
+ * order of that list:
+ *   f [B*gamma, SDD_MLP_HIDDEN] bf16 (round to nearest even), row-major,
+ *     16-byte aligned; every column is written: 4 top-1 probability (maxprob),
+ *     5 its natural log, 6 entropy, 7 its negative, 8 probability margin,
+ *     9 top-5 mass, 14 block position j / gamma, 15 generated length
+ *     round / 256; every other column 0 (the paper's diffusion-model
+ *     quantities -- reveal step and rank, parallelism, step-0 values -- have
+ *     no counterpart here).
+ *   maxprob, entropy, margin, top5 [B, gamma] fp32: the outputs of
+ *     sdd_confidence_features.  round >= 0.
+ * One launch.  The block is the f argument of sdd_scorer_deep.
+ */
+SDD_API sdd_status_t sdd_scorer_features(const float *maxprob, const float *entropy, const float *margin,
+                                         const float *top5, int B, int gamma, int64_t round, void *f,
+                                         sdd_stream_t stream);
+
+/*
  * sdd_scorer_workspace_size -- bytes of device scratch that sdd_survival_mlp
  * and sdd_scorer_deep need for M positions (512 KiB per 128 positions: the
  * first layer's split-K partial accumulators, later the deep scorer's

@@ -90,6 +90,8 @@ def load(path: str | None = None):
     L.sdd_uniforms.argtypes = [u64, VP, VP, VP, VP, i64, VP, VP]
     L.sdd_confidence_noalloc.argtypes = [VP, I, I, I, I, i64, VP, VP, VP, VP, VP, VP, VP, VP, VP]
     L.sdd_confidence_noalloc.restype = I
+    L.sdd_scorer_features.argtypes = [VP, VP, VP, VP, I, I, i64, VP, VP]
+    L.sdd_scorer_features.restype = I
     L.sdd_scorer_workspace_size.argtypes = [I, ctypes.POINTER(ctypes.c_size_t)]
     L.sdd_scorer_workspace_size.restype = I
     L.sdd_survival_mlp.argtypes = [VP, I, I, VP, VP, VP, ctypes.c_float, VP, VP, ctypes.c_size_t, VP, VP]
@@ -350,6 +352,18 @@ def commit(K, x, verified_tokens, verified_n, stream=None):
 
 MLP_HIDDEN = 256
 MLP_KSTEP = 64
+
+
+def scorer_features(conf, round_: int, *, out=None, stream=None):
+    """sdd_scorer_features: the scorer's scalar-feature block [B * gamma, 256] bf16
+    from a Confidence computed with features=True (App. A.7's column order)."""
+    B, gamma = conf.maxprob.shape
+    if conf.margin is None or conf.top5 is None:
+        raise ValueError("the confidence must be computed with features=True")
+    f = torch.empty(B * gamma, MLP_HIDDEN, dtype=torch.bfloat16, device=conf.maxprob.device) if out is None else out
+    _check(load().sdd_scorer_features(_p(conf.maxprob), _p(conf.entropy), _p(conf.margin), _p(conf.top5), B, gamma,
+                                      int(round_), _p(f), _stream(stream)), "sdd_scorer_features")
+    return f
 
 
 def scorer_workspace(M, device):

@@ -551,6 +551,22 @@ sdd_status_t sdd_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, c
     return SDD_OK;
 }
 
+sdd_status_t sdd_scorer_features(const float *maxprob, const float *entropy, const float *margin,
+                                 const float *top5, int B, int gamma, int64_t round, void *f, sdd_stream_t stream) {
+    if (B < 0 || gamma < 1 || gamma > SDD_MAX_GAMMA)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "B = %d / gamma = %d out of range", B, gamma);
+    if (round < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "round = %lld < 0", static_cast<long long>(round));
+    if (B == 0) return SDD_OK;
+    if (!maxprob || !entropy || !margin || !top5)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "maxprob, entropy, margin and top5 must not be NULL");
+    SDD_TRY(check_ptr16(f, "f"));
+    const cudaError_t e =
+        launch_scorer_features(maxprob, entropy, margin, top5, static_cast<int64_t>(B) * gamma, gamma,
+                               static_cast<float>(static_cast<double>(round) / 256.0), static_cast<uint16_t *>(f),
+                               reinterpret_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? SDD_OK : cuda_fail(e, "scorer features launch");
+}
+
 sdd_status_t sdd_scorer_workspace_size(int M, size_t *bytes) {
     if (!bytes) return fail(SDD_ERR_INVALID_ARGUMENT, "bytes is NULL");
     if (M < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "M = %d < 0", M);

@@ -194,6 +194,9 @@ cudaError_t launch_position_metrics(const float *q, const int32_t *L, int B, int
                                     double *bce_base, double *auroc, int32_t *n_pos, int32_t *n_neg,
                                     cudaStream_t stream);
 
+// The learned scorer's scalar-feature block (mlp.cu), bf16 [M, 256].
+cudaError_t launch_scorer_features(const float *maxprob, const float *entropy, const float *margin, const float *top5,
+                                   int64_t M, int gamma, float gen, uint16_t *f, cudaStream_t stream);
 // Device scratch of the scorers (mlp.cu) for M rows: the split-K partials of
 // the first layer, later the deep scorer's second-layer activations.
 size_t mlp_workspace_bytes(int M);

@@ -754,4 +754,45 @@ cudaError_t launch_scorer_deep(const void *h, int Kh, const void *f, int M, cons
     return cudaLaunchKernelEx(&cfg, mlp_tail_kernel, tmAct, tmW2, tmW3, tmAct2, p);
 }
 
+// ---------------------------------------------------------------------------
+// The learned scorer's scalar-feature block (App. A.7's list): one warp per
+// position writes its 256 bf16 columns (lane u: columns 8u .. 8u + 7), zero
+// except the logits-side features and the position ones.
+// ---------------------------------------------------------------------------
+namespace {
+__global__ void scorer_features_kernel(const float *maxprob, const float *entropy, const float *margin,
+                                       const float *top5, int64_t M, int gamma, float gen, uint16_t *f) {
+    const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (w >= M) return;
+    float v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = 0.f;
+    if (lane == 0) {   // columns 4..7: top-1 probability, its log, entropy, its negative
+        const float mp = __ldg(maxprob + w), h = __ldg(entropy + w);
+        v[4] = mp;
+        v[5] = logf(mp);
+        v[6] = h;
+        v[7] = -h;
+    } else if (lane == 1) {   // columns 8, 9: margin, top-5 mass; 14, 15: block position, generated length
+        v[0] = __ldg(margin + w);
+        v[1] = __ldg(top5 + w);
+        v[6] = static_cast<float>(w % gamma) / static_cast<float>(gamma);
+        v[7] = gen;
+    }
+    const uint4 u = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]),
+                               pack_bf16x2(v[6], v[7]));
+    reinterpret_cast<uint4 *>(f + w * kMlpN)[lane] = u;
+}
+}  // namespace
+
+cudaError_t launch_scorer_features(const float *maxprob, const float *entropy, const float *margin, const float *top5,
+                                   int64_t M, int gamma, float gen, uint16_t *f, cudaStream_t stream) {
+    if (M == 0) return cudaSuccess;
+    const int64_t threads = M * 32;
+    scorer_features_kernel<<<static_cast<unsigned>((threads + 255) / 256), 256, 0, stream>>>(
+        maxprob, entropy, margin, top5, M, gamma, gen, f);
+    return cudaGetLastError();
+}
+
 }  // namespace sdd

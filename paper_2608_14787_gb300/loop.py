@@ -87,21 +87,15 @@ class DecodeLoop:
         self.scorer_ws = sdd.scorer_workspace(B * gamma, dev)
 
     def features(self, conf, round_: int) -> torch.Tensor:
-        """The scorer's scalar-feature block [B * gamma, 256] bf16 (19 columns,
-        zeros after them) in the order of App. A.7's list: the diffusion-model
-        quantities (reveal step and rank, parallelism, late reveal, step-0
-        values and their changes, segment position, dataset flags) are not
-        available here and stay zero; the logits-side ones come from the
-        confidence pass: top-1 probability, its log, entropy, its negative,
-        probability margin, top-5 mass; then block position and generated length."""
-        B, gamma = self.B, self.gamma
-        f = self.feat.view(B, gamma, -1)
-        pos = torch.arange(gamma, device=self.device, dtype=torch.float32).view(1, gamma) / gamma
-        cols = {4: conf.maxprob, 5: torch.log(conf.maxprob), 6: conf.entropy, 7: -conf.entropy, 8: conf.margin,
-                9: conf.top5, 14: pos.expand(B, gamma), 15: torch.full((B, gamma), round_ / 256.0, device=self.device)}
-        for c, v in cols.items():
-            f[:, :, c] = v.to(torch.bfloat16)
-        return self.feat
+        """The scorer's scalar-feature block [B * gamma, 256] bf16 (sdd_scorer_features:
+        19 columns in the order of App. A.7's list, zeros after them).  The
+        diffusion-model quantities (reveal step and rank, parallelism, late
+        reveal, step-0 values and their changes, segment position, dataset
+        flags) are not available here and stay zero; the logits-side ones come
+        from the confidence pass: top-1 probability, its log, entropy, its
+        negative, probability margin, top-5 mass; then block position and
+        generated length."""
+        return sdd.scorer_features(conf, round_, out=self.feat)
 
     def step(self, z_d, z_t, x, h, round_: int) -> RoundOut:
         B, gamma = self.B, self.gamma
