@@ -33,12 +33,19 @@ constexpr int kDiagThreads = 256;
 // interleaves those loops.
 constexpr int kPermThreads = 64;
 
+// Lists of at most this many valid blocks are shuffled by the parallel
+// construction below; longer ones by the serial swap loop.
+constexpr int kPermPar = 4096;
+
 // Shared memory of the permutation builder for B logged blocks: the block
 // list [B], the validity bits of position j [ceil(B/32) words] and their
-// exclusive prefix popcounts [ceil(B/32)].
+// exclusive prefix popcounts [ceil(B/32)]; for B <= kPermPar the parallel
+// construction's arrays: one [B] of 32-bit bucket bounds and four [B] of
+// 16-bit indices (small, so that ~23 CTAs share an SM).
 __host__ __device__ inline size_t perm_smem_bytes(int B) {
     const size_t words = (static_cast<size_t>(B) + 31) / 32;
-    return (static_cast<size_t>(B) + 2 * words) * sizeof(int32_t);
+    const size_t par = (B <= kPermPar) ? static_cast<size_t>(B) * (sizeof(int32_t) + 4 * sizeof(int16_t)) : 0;
+    return (static_cast<size_t>(B) + 2 * words) * sizeof(int32_t) + par;
 }
 
 __global__ void __launch_bounds__(kPermThreads) perm_build_kernel(const float *q, const int32_t *L, int B, int gamma,
@@ -88,41 +95,137 @@ __global__ void __launch_bounds__(kPermThreads) perm_build_kernel(const float *q
         if (m & bit) s_list[s_wpre[b >> 5] + __popc(m & (bit - 1u))] = b;
     }
     __syncthreads();
-    // Fisher-Yates from the top: slot i swaps with k = floor(w (i + 1) / 2^32),
-    // w the first Philox word of counter (i, j, r, purpose).  The partners of
-    // kPermThreads slots are drawn in parallel, the swaps then run in order.
+    // Fisher-Yates from the top: slot i swaps with k_i = floor(w (i + 1) / 2^32),
+    // w the first Philox word of counter (i, j, r, purpose), for i = n-1 .. 1.
     const uint2 key = make_uint2(static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32));
-    for (int top = n - 1; top > 0; top -= kPermThreads) {
-        const int i = top - tid;
-        if (i > 0) {
-            const uint4 o = philox4x32_10(make_uint4(static_cast<uint32_t>(i), static_cast<uint32_t>(j),
+    if (n > 1 && n <= kPermPar) {
+        // The same permutation without the serial loop.  Step a moves the
+        // value then at slot a to slot k_a and fixes slot a.  Let P(s) be the
+        // value at slot s just before step s (slot 0: at the end); the last
+        // step before a that wrote slot s is the smallest a' > a with
+        // k_a' = s, and it wrote P(a').  So, with bucket(s) = {a : k_a = s}:
+        //   P(s) = P(min{a' in bucket(s), a' > s}), or the original s_list[s];
+        //   final[a] = P(min{a' in bucket(k_a), a' > a}), or s_list[k_a];
+        //   final[0] = P(0).
+        // P follows the "first step above" chains to their ends (pointer
+        // jumping); buckets come from a counting sort, each sorted by index.
+        int32_t *s_cnt = s_wpre + words;                          // bucket sizes, starts, then ends
+        int16_t *s_kk = reinterpret_cast<int16_t *>(s_cnt + B);   // k_a
+        int16_t *s_bkt = s_kk + B;                                // steps by bucket; later the final list
+        int16_t *s_nxt = s_bkt + B;                               // next step of the bucket above a (-1: none)
+        int16_t *s_ptr = s_nxt + B;                               // chain links, then chain ends
+        __shared__ int32_t s_part[kPermThreads];
+        for (int t = tid; t < n; t += kPermThreads) s_cnt[t] = 0;
+        __syncthreads();
+        for (int a = 1 + tid; a < n; a += kPermThreads) {
+            const uint4 o = philox4x32_10(make_uint4(static_cast<uint32_t>(a), static_cast<uint32_t>(j),
                                                      static_cast<uint32_t>(r), kPurposePerm),
                                           key);
-            s_k[tid] = static_cast<int32_t>((static_cast<uint64_t>(o.x) * static_cast<uint64_t>(i + 1)) >> 32);
+            const int k = static_cast<int>((static_cast<uint64_t>(o.x) * static_cast<uint64_t>(a + 1)) >> 32);
+            s_kk[a] = static_cast<int16_t>(k);
+            atomicAdd(&s_cnt[k], 1);
         }
         __syncthreads();
+        // bucket starts: exclusive prefix of the sizes (chunks per thread)
+        const int chunk = (n + kPermThreads - 1) / kPermThreads;
+        const int c0 = min(n, tid * chunk), c1 = min(n, c0 + chunk);
+        int sum = 0;
+        for (int t = c0; t < c1; ++t) sum += s_cnt[t];
+        s_part[tid] = sum;
+        __syncthreads();
         if (tid == 0) {
-            // slots top, top - 1, ..., top - cnt + 1 (all > 0); x carries the
-            // value at slot a, re-read after each swap (which may have written
-            // slot a - 1), so one shared-memory round trip bounds an iteration;
-            // the partners come four at a time
-            const int cnt = min(kPermThreads, top);
-            int32_t x = s_list[top];
-            for (int u = 0; u < cnt; u += 4) {
-                const int4 kk = *reinterpret_cast<const int4 *>(s_k + u);
-                const int ks[4] = {kk.x, kk.y, kk.z, kk.w};
-#pragma unroll
-                for (int h = 0; h < 4; ++h) {
-                    if (u + h >= cnt) break;
-                    const int a = top - u - h, k = ks[h];
-                    const int32_t y = (k == a) ? x : s_list[k];
-                    s_list[k] = x;
-                    s_list[a] = y;
-                    x = s_list[a - 1];
-                }
+            int run = 0;
+            for (int t = 0; t < kPermThreads; ++t) {
+                const int v = s_part[t];
+                s_part[t] = run;
+                run += v;
             }
         }
         __syncthreads();
+        int run = s_part[tid];
+        for (int t = c0; t < c1; ++t) {
+            const int v = s_cnt[t];
+            s_cnt[t] = run;
+            run += v;
+        }
+        __syncthreads();
+        // scatter (the starts advance to the ends: bucket t is [end(t-1), end(t)))
+        for (int a = 1 + tid; a < n; a += kPermThreads)
+            s_bkt[atomicAdd(&s_cnt[s_kk[a]], 1)] = static_cast<int16_t>(a);
+        __syncthreads();
+        // per slot: its bucket sorted, successors, the first step above the slot
+        for (int t = tid; t < n; t += kPermThreads) {
+            const int b0 = (t > 0) ? s_cnt[t - 1] : 0, b1 = s_cnt[t];
+            for (int u = b0 + 1; u < b1; ++u) {   // insertion sort (buckets hold ~1 step)
+                const int v = s_bkt[u];
+                int w = u - 1;
+                while (w >= b0 && s_bkt[w] > v) {
+                    s_bkt[w + 1] = s_bkt[w];
+                    --w;
+                }
+                s_bkt[w + 1] = static_cast<int16_t>(v);
+            }
+            int above = t;   // the chain ends here when no step above t targets t
+            for (int u = b0; u < b1; ++u) {
+                const int v = s_bkt[u];
+                s_nxt[v] = (u + 1 < b1) ? s_bkt[u + 1] : static_cast<int16_t>(-1);
+                if (above == t && v > t) above = v;
+            }
+            s_ptr[t] = static_cast<int16_t>(above);
+        }
+        __syncthreads();
+        for (int span = 1; span < n; span <<= 1) {   // pointer jumping to the chain ends
+            for (int t = tid; t < n; t += kPermThreads) s_ptr[t] = s_ptr[s_ptr[t]];
+            __syncthreads();
+        }
+        for (int a = tid; a < n; a += kPermThreads) {
+            int v;
+            if (a == 0) {
+                v = s_list[s_ptr[0]];
+            } else {
+                const int na = s_nxt[a];
+                v = (na >= 0) ? s_list[s_ptr[na]] : s_list[s_kk[a]];
+            }
+            s_bkt[a] = static_cast<int16_t>(v);
+        }
+        __syncthreads();
+        for (int a = tid; a < n; a += kPermThreads) s_list[a] = s_bkt[a];
+        __syncthreads();
+    } else {
+        // serial: the partners of kPermThreads slots drawn in parallel, the swaps
+        // then in order
+        for (int top = n - 1; top > 0; top -= kPermThreads) {
+            const int i = top - tid;
+            if (i > 0) {
+                const uint4 o = philox4x32_10(make_uint4(static_cast<uint32_t>(i), static_cast<uint32_t>(j),
+                                                         static_cast<uint32_t>(r), kPurposePerm),
+                                              key);
+                s_k[tid] = static_cast<int32_t>((static_cast<uint64_t>(o.x) * static_cast<uint64_t>(i + 1)) >> 32);
+            }
+            __syncthreads();
+            if (tid == 0) {
+                // slots top, top - 1, ..., top - cnt + 1 (all > 0); x carries the
+                // value at slot a, re-read after each swap (which may have written
+                // slot a - 1), so one shared-memory round trip bounds an iteration;
+                // the partners come four at a time
+                const int cnt = min(kPermThreads, top);
+                int32_t x = s_list[top];
+                for (int u = 0; u < cnt; u += 4) {
+                    const int4 kk = *reinterpret_cast<const int4 *>(s_k + u);
+                    const int ks[4] = {kk.x, kk.y, kk.z, kk.w};
+#pragma unroll
+                    for (int h = 0; h < 4; ++h) {
+                        if (u + h >= cnt) break;
+                        const int a = top - u - h, k = ks[h];
+                        const int32_t y = (k == a) ? x : s_list[k];
+                        s_list[k] = x;
+                        s_list[a] = y;
+                        x = s_list[a - 1];
+                    }
+                }
+            }
+            __syncthreads();
+        }
     }
     // block b (the t-th valid block) takes the score of block s_list[t]; others
     // keep theirs: the permuted scores of position j, gathered here so that the
