@@ -206,7 +206,10 @@ def _cpu_baseline(wl, ells, ks, blk_host, n_blocks):
 
 def _e2e(args, ws, dev, stream, sets, rnd, wl, B):
     """The same round end to end through the C ABI: inputs copied from pinned
-    host buffers and results copied back inside the timed region."""
+    host buffers and results copied back inside the timed region.  Two device
+    input buffers alternate: step i + 1's host-to-device copy (on a copy
+    stream) overlaps step i's round, and a buffer is refilled only after the
+    round that read it (events); every step's copies are inside the region."""
     import torch
     from paper_2608_14787_gb300 import shard
     if ws > 1:
@@ -214,32 +217,55 @@ def _e2e(args, ws, dev, stream, sets, rnd, wl, B):
     hz_d = sets[0].z_d.cpu().pin_memory()
     hz_t = sets[0].z_t.cpu().pin_memory()
     hx = sets[0].x.cpu().pin_memory()
-    dz_d, dz_t, dx = sets[0].z_d, sets[0].z_t, sets[0].x
+    bufs = [(st.z_d, st.z_t, st.x) for st in sets[:2]]
+    if len(bufs) < 2:   # (a single input set: a second device buffer for the copies)
+        bufs.append(tuple(torch.empty_like(t) for t in bufs[0]))
     outs = [rnd.L_strict, rnd.tokens_strict, rnd.K, rnd.commit_tokens, rnd.commit_n, rnd.q]
     h_outs = [torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs]
     e2e_steps = max(3, min(args.steps, 200))
     h2d = hz_d.numel() * hz_d.element_size() + hz_t.numel() * hz_t.element_size() + hx.numel() * 4
     d2h = sum(o.numel() * o.element_size() for o in outs)
+    main = torch.cuda.current_stream()
+    copy = torch.cuda.Stream()
+    ready = [torch.cuda.Event() for _ in range(2)]
+    done = [torch.cuda.Event() for _ in range(2)]
+    for ev in done:
+        ev.record(main)
 
-    def e2e_step(i):
-        dz_d.copy_(hz_d, non_blocking=True)
-        dz_t.copy_(hz_t, non_blocking=True)
-        dx.copy_(hx, non_blocking=True)
+    def issue_copy(i):
+        b = i % 2
+        copy.wait_event(done[b])               # the round that last read this buffer has finished
+        with torch.cuda.stream(copy):
+            for d, h in zip(bufs[b], (hz_d, hz_t, hx)):
+                d.copy_(h, non_blocking=True)
+        ready[b].record(copy)
+
+    def e2e_round(i):
+        b = i % 2
+        main.wait_event(ready[b])
+        dz_d, dz_t, dx = bufs[b]
         rnd.set_inputs(dz_d, dz_t, dx, seed=wl.seed, round_=i)
         rnd.run()
         for h, d in zip(h_outs, outs):
             h.copy_(d, non_blocking=True)
+        done[b].record(main)
 
-    for i in range(2):
-        e2e_step(i)
+    def run(n):
+        copy.wait_stream(main)   # the copies start after everything issued so far (the start event)
+        issue_copy(0)
+        for i in range(n):
+            if i + 1 < n:
+                issue_copy(i + 1)
+            e2e_round(i)
+
+    run(2)
     torch.cuda.synchronize()
     if ws > 1:
         dist.barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for i in range(e2e_steps):
-        e2e_step(i)
-    e1.record(stream)
+    e0.record(main)
+    run(e2e_steps)
+    e1.record(main)
     torch.cuda.synchronize()
     e2e_ms = shard.max_over_ranks(e0.elapsed_time(e1), device=dev)
     return ws * B * e2e_steps / (e2e_ms / 1e3), h2d, d2h
