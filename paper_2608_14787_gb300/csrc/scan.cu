@@ -191,11 +191,10 @@ __device__ __noinline__ int first_index(const char *rowp, int k0, int lane, int 
 // clamped first (so a masked entry adds 0 * finite to t2); target rows need no
 // clamp (2^-inf = 0 and the maximum starts at the clamp value).  The lane's
 // exp-sum is an fp32 pair (s_hi, s_lo) updated by TwoSum once per tile.
-// vmax (FEAT only): the maximum of each of the lane's vectors, kept for the
-// extended features (bf16: as a packed pair, f32: as bits).
-template <int DT, bool ENT, bool FEAT>
+// Returns the lane's tile maximum (clamp value included).
+template <int DT, bool ENT>
 __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lane, SoftState &st, float &s_hi,
-                                              float &s_lo, uint32_t (&vmax)[kVPL]) {
+                                              float &s_lo) {
     // pass 1: the tile maximum (clamp value included)
     float cm;
     if (DT == SDD_BF16) {
@@ -204,7 +203,6 @@ __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lan
         for (int i = 0; i < kVPL; ++i) {
             const uint4 w = tile[lane + 32 * i];
             const uint32_t vm = bf16x2_max_nan(bf16x2_max_nan(w.x, w.y), bf16x2_max_nan(w.z, w.w));
-            if (FEAT) vmax[i] = vm;
             mx = bf16x2_max_nan(mx, vm);
         }
         cm = fmax_nan(bf16_lo(mx), bf16_hi(mx));
@@ -215,7 +213,6 @@ __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lan
             const uint4 w = tile[lane + 32 * i];
             const float vm = fmax_nan(fmax_nan(__uint_as_float(w.x), __uint_as_float(w.y)),
                                       fmax_nan(__uint_as_float(w.z), __uint_as_float(w.w)));
-            if (FEAT) vmax[i] = __float_as_uint(vm);
             cm = fmax_nan(cm, vm);
         }
     }
@@ -544,9 +541,8 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
         uint4 *tile = reinterpret_cast<uint4 *>(ring + slot * kTileBytes);
         const bool row_end = (cc.k + n == p.RV);
         if (n < kTileVec || (row_end && tail)) pad_tile<DT>(tile, n, lane, row_end, tail);
-        uint32_t vmax[kVPL];
-        const float cm = ent ? process_tile<DT, true, false>(tile, cc.k, lane, st, s_hi, s_lo, vmax)
-                             : process_tile<DT, false, false>(tile, cc.k, lane, st, s_hi, s_lo, vmax);
+        const float cm = ent ? process_tile<DT, true>(tile, cc.k, lane, st, s_hi, s_lo)
+                             : process_tile<DT, false>(tile, cc.k, lane, st, s_hi, s_lo);
         if (FEAT && ent) group_update(cm, cc.k, ck, ct);
         if (rank_on) {
             const bool want = cm >= g;
