@@ -10,12 +10,15 @@
 // Sec. 3.1 and App. A.6 read.
 //
 // How: the rows of the call are laid end to end as one sequence of 16-byte
-// vectors, split into contiguous, equal ranges, one per warp (perfect balance,
-// no per-tile scheduling).  Each warp streams its range through a private
-// ring of 4 KiB shared-memory tiles filled by 1D bulk copies (cp.async.bulk +
-// mbarrier), keeps an online-softmax state per lane (packed f32x2 arithmetic,
-// exp-sums as double-floats), reduces it across the warp at the end of each
-// row piece and publishes a 32-byte partial.
+// vectors, split into contiguous ranges of equal cost, one per warp (a drafter
+// vector weighs 10, a target vector 9: the drafter rows' entropy accumulator
+// costs more; no per-tile scheduling).  Each warp streams its range through a
+// private ring of two 4 KiB shared-memory tiles filled by 1D bulk copies
+// (cp.async.bulk + mbarrier), keeps an online-softmax state per lane (packed
+// f32x2 arithmetic, exp-sums as double-floats), reduces it across the warp at
+// the end of each row piece and publishes a 32-byte partial.  The feature
+// instantiation also publishes each drafter row piece's five largest entries
+// (group_update / group_top5 below).
 // The decide kernel (decide.cu) merges each row's partials and finalises the
 // rows; keeping that out of the streaming kernel keeps this kernel free of
 // register spills.
