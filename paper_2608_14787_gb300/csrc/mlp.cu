@@ -1,19 +1,23 @@
-// mlp.cu -- the stand-in survival scorer of the decode-loop workload on the
-// 5th-generation tensor cores:
+// mlp.cu -- the learned-scorer stand-ins of the decode-loop workload on the
+// 5th-generation tensor cores (App. A.7's form, random weights):
 //
-//   s[m] = sigmoid(w2 . GELU(W1 h[m] + b1) + b2),  GELU(z) = z Phi(z) (erf form),
+//   one layer:  s[m] = sigmoid(w2 . GELU(W1 h[m] + b1) + b2),
+//   deep:       a1 = bf16(GELU(W1 [h ; f] + b1)), a2 = bf16(GELU(W2 a1 + b2)),
+//               s[m] = sigmoid(w4 . GELU(W3 a2 + b3) + b4),
+//   GELU(z) = z Phi(z) (erf form), fp32 accumulation throughout,
 //
-// for h [M, K] bf16 (drafter hidden states), W1 [256, K] bf16 (one row per
-// hidden unit), b1 fp32 [256], w2 bf16 [256], b2 fp32 -- the form of the
-// learned scorer of App. A.7 with one hidden layer and random weights.
+// and the scalar-feature block f of the deep scorer's input.
 //
-// One CTA per 128-row tile computes the whole 128 x 256 product W1 h on
-// tcgen05: a four-stage ring of 48 KiB (A tile 128 x 64, B tile 256 x 64, both
-// K-major with the 128-byte swizzle) filled by 2D TMA loads; one thread issues
-// tcgen05.mma.kind::f16 (M = 128, N = 256, K = 16, fp32 accumulate) into a
-// 256-column TMEM accumulator and commits each stage back to the producer;
-// then four warps read their 32 rows from TMEM (tcgen05.ld) and fuse bias,
-// GELU, the w2 dot product and the sigmoid, writing one float per row.
+// First layer (mlp_kernel): a cluster of S = 4 CTAs per 128-row tile splits K;
+// each CTA streams its K quarter through a four-stage ring of 48 KiB (A tile
+// 128 x 64, B tile 256 x 64, K-major, 128-byte swizzle) filled by 2D TMA, one
+// thread issues tcgen05.mma.kind::f16 (M = 128, N = 256, K = 16) into a
+// 256-column TMEM accumulator; the partial accumulators meet through an L2
+// workspace (stores, one cluster barrier, bulk copies) and CTA q finishes
+// output columns [64 q, 64 q + 64) with the fused epilogue.
+// Layers 2-3 of the deep scorer (mlp_tail_kernel): a cluster of four CTAs per
+// tile, each computing 64 output columns of both layers, a2 through the
+// workspace and back by TMA.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
