@@ -9,7 +9,12 @@
 //    Eq. 9), top-k (App. A.6);
 //  * sched_step / sched_final -- the skip policy of Sec. 4.1: the local gate,
 //    then Eq. 3 with the raw / conditional / marginal signals of Sec. 4.2, then
-//    K_min, staleness and guards.
+//    K_min, staleness and guards;
+//  * periodic_khat -- the confidence-free periodic baseline of the appendix's
+//    periodic-skipping paragraph (an attempt every P rounds, same guards);
+//  * feat_merge / feat_final -- the extended features of App. A.7: a drafter
+//    row's five largest entries merged from its pieces' lists, then the
+//    probability margin and the top-5 mass.
 //
 // Everything here is fp32 or double-float (common.cuh): fp64 instructions
 // issue at a small fraction of the fp32 rate on this part.
