@@ -196,20 +196,31 @@ class Confidence:
     top5: torch.Tensor | None = None
 
 
+def confidence_buffers(B: int, gamma: int, device, features: bool = False) -> Confidence:
+    """Output tensors for confidence(..., out=): [B, gamma] each (lse fp64, argmax int32)."""
+    f32 = lambda: torch.empty(B, gamma, dtype=torch.float32, device=device)  # noqa: E731
+    out = Confidence(q=f32(), logq=f32(), maxprob=f32(), lse=torch.empty(B, gamma, dtype=torch.float64, device=device),
+                     entropy=f32(), argmax=torch.empty(B, gamma, dtype=torch.int32, device=device))
+    if features:
+        out.margin, out.top5 = f32(), f32()
+    return out
+
+
 def confidence(z_d: torch.Tensor, x: torch.Tensor, ws: Workspace | None = None, status=None,
-               stream=None, features: bool = False) -> Confidence:
+               stream=None, features: bool = False, out: Confidence | None = None) -> Confidence:
     """sdd_confidence over drafter logits z_d [B, gamma, V] and drafted tokens x [B, gamma];
-    with features=True sdd_confidence_features (also margin and top5 [B, gamma])."""
+    with features=True sdd_confidence_features (also margin and top5 [B, gamma]).
+    `out`: tensors from confidence_buffers (filled and returned) instead of new ones."""
     B, gamma = x.shape
     V, stride = _logits_layout(z_d, "z_d")
     dev = z_d.device
     ws = ws or Workspace(B, gamma, V, dev)
     status = new_status(dev) if status is None else status
-    f32 = lambda: torch.empty(B, gamma, dtype=torch.float32, device=dev)  # noqa: E731
-    out = Confidence(q=f32(), logq=f32(), maxprob=f32(), lse=torch.empty(B, gamma, dtype=torch.float64, device=dev),
-                     entropy=f32(), argmax=torch.empty(B, gamma, dtype=torch.int32, device=dev))
+    if out is None:
+        out = confidence_buffers(B, gamma, dev, features)
+    elif out.q.shape != (B, gamma) or (features and (out.margin is None or out.top5 is None)):
+        raise ValueError("out must come from confidence_buffers(B, gamma, device, features)")
     if features:
-        out.margin, out.top5 = f32(), f32()
         rc = load().sdd_confidence_features(_p(z_d), _dtype_code(z_d), B, gamma, V, stride, _p(x), _p(out.q),
                                             _p(out.logq), _p(out.maxprob), _p(out.lse), _p(out.entropy),
                                             _p(out.argmax), _p(out.margin), _p(out.top5), ws.ptr, ws.nbytes,
@@ -246,14 +257,16 @@ def _f64_array(vals):
 
 
 def schedule_prefix(q, eta_b, eta_c, *, signal=SIG_RAW, logq=None, K_min=6, S_max=64, guard=None,
-                    force_strict=None, D_in=None, status=None, stream=None):
-    """sdd_schedule_prefix; returns (K_hat, K, D_out), each [n_tau, B]."""
+                    force_strict=None, D_in=None, status=None, stream=None, out=None):
+    """sdd_schedule_prefix; returns (K_hat, K, D_out), each [n_tau, B] int32 (`out`:
+    three such tensors to fill instead; D_out must not alias D_in)."""
     B, gamma = q.shape
     n_tau = len(eta_b)
     dev = q.device
-    Kh = torch.empty(n_tau, B, dtype=torch.int32, device=dev)
-    K = torch.empty(n_tau, B, dtype=torch.int32, device=dev)
-    Do = torch.empty(n_tau, B, dtype=torch.int32, device=dev)
+    if out is None:
+        Kh, K, Do = (torch.empty(n_tau, B, dtype=torch.int32, device=dev) for _ in range(3))
+    else:
+        Kh, K, Do = out
     eb, ec = _f64_array(eta_b), _f64_array(eta_c)
     rc = load().sdd_schedule_prefix(_p(q), _p(logq), B, gamma, signal, eb, ec, n_tau, K_min, S_max, _p(guard),
                                     _p(force_strict), _p(D_in), _p(Kh), _p(K), _p(Do), _p(status), _stream(stream))
@@ -262,12 +275,14 @@ def schedule_prefix(q, eta_b, eta_c, *, signal=SIG_RAW, logq=None, K_min=6, S_ma
 
 
 def schedule_periodic(B, gamma, periods, *, K_skip=6, round_=0, K_min=6, S_max=64, guard=None, force_strict=None,
-                      D_in=None, status=None, stream=None, device="cuda"):
-    """sdd_schedule_periodic; returns (K_hat, K, D_out), each [n_p, B]."""
+                      D_in=None, status=None, stream=None, device="cuda", out=None):
+    """sdd_schedule_periodic; returns (K_hat, K, D_out), each [n_p, B] int32 (`out`:
+    three such tensors to fill instead; D_out must not alias D_in)."""
     n_p = len(periods)
-    Kh = torch.empty(n_p, B, dtype=torch.int32, device=device)
-    K = torch.empty(n_p, B, dtype=torch.int32, device=device)
-    Do = torch.empty(n_p, B, dtype=torch.int32, device=device)
+    if out is None:
+        Kh, K, Do = (torch.empty(n_p, B, dtype=torch.int32, device=device) for _ in range(3))
+    else:
+        Kh, K, Do = out
     per = (ctypes.c_int32 * n_p)(*[int(x) for x in periods])
     rc = load().sdd_schedule_periodic(B, gamma, per, n_p, K_skip, round_, K_min, S_max, _p(guard), _p(force_strict),
                                       _p(D_in), _p(Kh), _p(K), _p(Do), _p(status), _stream(stream))
@@ -341,10 +356,14 @@ def agreement(K, L_strict, acc=None, stream=None):
     return acc
 
 
-def commit(K, x, verified_tokens, verified_n, stream=None):
+def commit(K, x, verified_tokens, verified_n, stream=None, out=None):
+    """sdd_commit; returns (tokens [B, gamma+1], n [B]) int32 (`out`: two such tensors to fill)."""
     B, gamma = x.shape
-    out_t = torch.empty(B, gamma + 1, dtype=torch.int32, device=x.device)
-    out_n = torch.empty(B, dtype=torch.int32, device=x.device)
+    if out is None:
+        out_t = torch.empty(B, gamma + 1, dtype=torch.int32, device=x.device)
+        out_n = torch.empty(B, dtype=torch.int32, device=x.device)
+    else:
+        out_t, out_n = out
     _check(load().sdd_commit(_p(K), _p(x), _p(verified_tokens), _p(verified_n), B, gamma, _p(out_t), _p(out_n),
                              _stream(stream)), "sdd_commit")
     return out_t, out_n

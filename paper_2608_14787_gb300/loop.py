@@ -85,6 +85,13 @@ class DecodeLoop:
         else:
             raise ValueError(f"scorer {scorer!r}: 'deep' or 'mlp'")
         self.scorer_ws = sdd.scorer_workspace(B * gamma, dev)
+        # per-round outputs, allocated once: the schedules' (K_hat, K, D_out)
+        # alternate between two sets so that D_out never aliases D_in
+        i32 = lambda *shape: torch.empty(*shape, dtype=torch.int32, device=dev)  # noqa: E731
+        self._conf = sdd.confidence_buffers(B, gamma, dev, features=(scorer == "deep"))
+        self._sched = {p: [(i32(1, B), i32(1, B), i32(1, B)) for _ in range(2)] for p in ("raw", "mlp", "per")}
+        self._commit = (i32(B, gamma + 1), i32(B))
+        self._flip = 0
 
     def features(self, conf, round_: int) -> torch.Tensor:
         """The scorer's scalar-feature block [B * gamma, 256] bf16 (sdd_scorer_features:
@@ -98,9 +105,13 @@ class DecodeLoop:
         return sdd.scorer_features(conf, round_, out=self.feat)
 
     def step(self, z_d, z_t, x, h, round_: int) -> RoundOut:
+        """One round.  The returned tensors (and the loop's D and feature
+        block) live in buffers that the next step reuses."""
         B, gamma = self.B, self.gamma
         deep = self.scorer == "deep"
-        conf = sdd.confidence(z_d, x, ws=self.ws, status=self.status, features=deep)
+        o = self._flip
+        self._flip ^= 1
+        conf = sdd.confidence(z_d, x, ws=self.ws, status=self.status, features=deep, out=self._conf)
         if deep:
             s = sdd.scorer_deep(h, self.features(conf, round_), *self.deep, act=self.act, status=self.status,
                                 workspace=self.scorer_ws).reshape(B, gamma)
@@ -109,20 +120,21 @@ class DecodeLoop:
                                  workspace=self.scorer_ws).reshape(B, gamma)
         _, K_raw, D_raw = sdd.schedule_prefix(conf.q, [self.tau], [self.tau], signal=sdd.SIG_RAW, logq=conf.logq,
                                               K_min=self.K_min, S_max=self.S_max, D_in=self.D_raw,
-                                              status=self.status)
+                                              status=self.status, out=self._sched["raw"][o])
         _, K_mlp, D_mlp = sdd.schedule_prefix(s, [self.tau_mlp], [self.tau_mlp], signal=sdd.SIG_CONDITIONAL,
                                               K_min=self.K_min, S_max=self.S_max, D_in=self.D_mlp,
-                                              status=self.status)
+                                              status=self.status, out=self._sched["mlp"][o])
         _, K_per, D_per = sdd.schedule_periodic(B, gamma, [self.period], K_skip=max(self.K_min, 1), round_=round_,
                                                 K_min=self.K_min, S_max=self.S_max, D_in=self.D_per,
-                                                status=self.status, device=self.device)
+                                                status=self.status, device=self.device,
+                                                out=self._sched["per"][o])
         K = K_raw[0]
         rows = torch.nonzero(K == 0).flatten().to(torch.int32)    # the host's verify decision
         n_rows = int(rows.numel())
         L, tok, n = sdd.verify_strict(z_t, x, z_d=z_d, draft=conf, greedy=self.greedy, seed=self.seed, round_=round_,
                                       rows=rows, ws=self.ws, status=self.status)
-        tokens, n_commit = sdd.commit(K, x, tok, n)
-        self.D_raw, self.D_mlp, self.D_per = D_raw[0].contiguous(), D_mlp[0].contiguous(), D_per[0].contiguous()
+        tokens, n_commit = sdd.commit(K, x, tok, n, out=self._commit)
+        self.D_raw, self.D_mlp, self.D_per = D_raw[0], D_mlp[0], D_per[0]
         return RoundOut(K_raw=K, K_mlp=K_mlp[0], K_per=K_per[0], L=L, tokens=tokens, n=n_commit, n_verified=n_rows)
 
 
