@@ -230,7 +230,8 @@ void orc_row_probs(const void *logits, int dtype, int64_t V, int64_t offset, dou
 
 /* Rank of `token` in one row under the order (larger logit first, then lower
  * index first): #{v : z(v) > z(t)} + #{v < t : z(v) = z(t)}.  Rank 0 is the
- * greedy argmax; "among the k largest target logits" (App. A.6) is rank < k. */
+ * greedy argmax; the top-k rule of App. A.6 (the drafted token is one of the
+ * target's k largest logits) is rank < k. */
 int64_t orc_rank(const void *logits, int dtype, int64_t V, int64_t offset, int64_t token) {
     double g = orc_load(logits, dtype, offset + token);
     int64_t rank = 0;
