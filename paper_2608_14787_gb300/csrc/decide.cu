@@ -409,12 +409,14 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                 float g;
                 bool bad;
                 const int64_t r = (gd ? p.rows0 : 0) + static_cast<int64_t>(i) * G.npos + j;
-                merge_row(p, r, acc, g, bad);
-                f = row_final(p, G, j, b, acc, g, bad, leader);
                 if (FEAT && leader) {
                     float top[5];
-                    feat_merge(p, r, top);
+                    merge_row_t<true>(p, r, acc, g, bad, top);
+                    f = row_final(p, G, j, b, acc, g, bad, leader);
                     feat_final(G, static_cast<int64_t>(b) * p.gamma + j, top, f.lse);
+                } else {
+                    merge_row(p, r, acc, g, bad);
+                    f = row_final(p, G, j, b, acc, g, bad, leader);
                 }
             } else {
                 // stand-alone acceptance: the caller's drafter LSE and the token's drafter logit

@@ -12,9 +12,9 @@
 //    K_min, staleness and guards;
 //  * periodic_khat -- the confidence-free periodic baseline of the appendix's
 //    periodic-skipping paragraph (an attempt every P rounds, same guards);
-//  * feat_merge / feat_final -- the extended features of App. A.7: a drafter
-//    row's five largest entries merged from its pieces' lists, then the
-//    probability margin and the top-5 mass.
+//  * merge_row_t<true> / feat_final -- the extended features of App. A.7: a
+//    drafter row's five largest entries merged from its pieces' lists (loaded
+//    with its partials), then the probability margin and the top-5 mass.
 //
 // Everything here is fp32 or double-float (common.cuh): fp64 instructions
 // issue at a small fraction of the fp32 rate on this part.
@@ -57,17 +57,32 @@ __device__ __forceinline__ Partial load_partial(const Partial *p) {
 // Merged state of global row r, whose pieces were streamed by warps fw..lw
 // (partial of warp w at index r + w), merged in warp order, four loads in
 // flight at a time.  The row's first piece carries its token logit; any piece
-// flags an out-of-range token.
-__device__ __forceinline__ void merge_row(const ScanParams &p, int64_t r, SoftState &acc, float &g, bool &tok_bad) {
+// flags an out-of-range token.  FEAT (drafter rows of the feature call): also
+// the row's five largest entries t, merged from the pieces' lists (p.feat,
+// indexed like the partials) loaded in the same batches.
+template <bool FEAT>
+__device__ __forceinline__ void merge_row_t(const ScanParams &p, int64_t r, SoftState &acc, float &g, bool &tok_bad,
+                                            float (&t)[5]) {
     const int64_t fw = part_owner(p, r * p.RV), lw = part_owner(p, (r + 1) * p.RV - 1);
     acc = soft_identity();
     g = qnan();
     tok_bad = false;
+    if (FEAT) {
+#pragma unroll
+        for (int k = 0; k < 5; ++k) t[k] = -INFINITY;
+    }
     for (int64_t w0 = fw; w0 <= lw; w0 += 4) {
         Partial pt[4];
+        uint4 fv[4][2];   // FEAT: the pieces' top-5 lists, loaded in the same batch
 #pragma unroll
         for (int u = 0; u < 4; ++u)
-            if (w0 + u <= lw) pt[u] = load_partial(p.partials + r + w0 + u);
+            if (w0 + u <= lw) {
+                pt[u] = load_partial(p.partials + r + w0 + u);
+                if (FEAT) {
+                    fv[u][0] = __ldcg(reinterpret_cast<const uint4 *>(p.feat + r + w0 + u));
+                    fv[u][1] = __ldcg(reinterpret_cast<const uint4 *>(p.feat + r + w0 + u) + 1);
+                }
+            }
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
             if (w0 + u > lw) break;
@@ -82,8 +97,27 @@ __device__ __forceinline__ void merge_row(const ScanParams &p, int64_t r, SoftSt
             o.amax = pt[u].amax;
             o.rank = max(pt[u].rank, 0);
             acc = soft_merge(acc, o);
+            if (FEAT) {
+                const float f[5] = {__uint_as_float(fv[u][0].x), __uint_as_float(fv[u][0].y),
+                                    __uint_as_float(fv[u][0].z), __uint_as_float(fv[u][0].w),
+                                    __uint_as_float(fv[u][1].x)};
+#pragma unroll
+                for (int i = 0; i < 5; ++i) {
+                    float z = f[i];
+#pragma unroll
+                    for (int k = 0; k < 5; ++k) {   // insert z into the descending list
+                        const float hi = fmaxf(t[k], z), lo = fminf(t[k], z);
+                        t[k] = hi;
+                        z = lo;
+                    }
+                }
+            }
         }
     }
+}
+__device__ __forceinline__ void merge_row(const ScanParams &p, int64_t r, SoftState &acc, float &g, bool &tok_bad) {
+    float t[5];
+    merge_row_t<false>(p, r, acc, g, tok_bad, t);
 }
 
 // Final results of position j of block b (group G) from its merged state, by
@@ -154,40 +188,6 @@ __device__ __forceinline__ RowFacts row_final(const ScanParams &p, const ScanGro
         if (write) status_or(p.status, SDD_DEV_BAD_TOKEN);
     }
     return f;
-}
-
-// The five largest entries of drafter row r (global row index), merged from
-// its pieces' lists, by one thread.  The first four pieces' lists are loaded
-// together (a row rarely has more).
-__device__ __forceinline__ void feat_merge(const ScanParams &p, int64_t r, float (&t)[5]) {
-    const int64_t fw = part_owner(p, r * p.RV), lw = part_owner(p, (r + 1) * p.RV - 1);
-#pragma unroll
-    for (int k = 0; k < 5; ++k) t[k] = -INFINITY;
-    for (int64_t w0 = fw; w0 <= lw; w0 += 4) {
-        uint4 v[4][2];
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-            if (w0 + u <= lw) {
-                v[u][0] = __ldcg(reinterpret_cast<const uint4 *>(p.feat + r + w0 + u));
-                v[u][1] = __ldcg(reinterpret_cast<const uint4 *>(p.feat + r + w0 + u) + 1);
-            }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            if (w0 + u > lw) break;
-            const float f[5] = {__uint_as_float(v[u][0].x), __uint_as_float(v[u][0].y), __uint_as_float(v[u][0].z),
-                                __uint_as_float(v[u][0].w), __uint_as_float(v[u][1].x)};
-#pragma unroll
-            for (int i = 0; i < 5; ++i) {
-                float z = f[i];
-#pragma unroll
-                for (int k = 0; k < 5; ++k) {   // insert z into the descending list
-                    const float hi = fmaxf(t[k], z), lo = fminf(t[k], z);
-                    t[k] = hi;
-                    z = lo;
-                }
-            }
-        }
-    }
 }
 
 // Extended features of a drafter row (user index o) from its five largest
