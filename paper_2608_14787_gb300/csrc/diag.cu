@@ -33,8 +33,8 @@ constexpr int kDiagThreads = 256;
 // interleaves those loops.
 constexpr int kPermThreads = 64;
 
-// Lists of at most this many valid blocks are shuffled by the parallel
-// construction below; longer ones by the serial swap loop.
+// Logs of at most this many blocks are shuffled by the parallel construction
+// below; longer ones by the serial swap loop.
 constexpr int kPermPar = 4096;
 
 // Shared memory of the permutation builder for B logged blocks: the block
@@ -98,7 +98,7 @@ __global__ void __launch_bounds__(kPermThreads) perm_build_kernel(const float *q
     // Fisher-Yates from the top: slot i swaps with k_i = floor(w (i + 1) / 2^32),
     // w the first Philox word of counter (i, j, r, purpose), for i = n-1 .. 1.
     const uint2 key = make_uint2(static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32));
-    if (n > 1 && n <= kPermPar) {
+    if (n > 1 && B <= kPermPar) {   // (the shared-memory layout follows B, not n)
         // The same permutation without the serial loop.  Step a moves the
         // value then at slot a to slot k_a and fixes slot a.  Let P(s) be the
         // value at slot s just before step s (slot 0: at the end); the last

@@ -32,6 +32,19 @@ def test_permutation_diagnostic_vs_oracle(sdd, orc, signal, eta_b, eta_c):
     assert want[:-1].mean() < want[-1]           # the dependence the permutation breaks
 
 
+@pytest.mark.parametrize("signal", [0, 2])
+def test_permutation_diagnostic_long_log_vs_oracle(sdd, orc, signal):
+    """A log longer than the parallel shuffle's limit (4096 blocks): the serial
+    swap loop, also when few blocks remain valid (conditional signal, late
+    positions)."""
+    q, L = _synthetic_log(4500, 12, 5 + signal)
+    sums = sdd.permutation_diagnostic(torch.from_numpy(q).cuda(), torch.from_numpy(L).cuda(), signal=signal,
+                                      eta_b=0.90, eta_c=0.90, n_rep=3, seed=4)
+    torch.cuda.synchronize()
+    want = orc.permutation_diagnostic(q.astype(np.float64), L, signal, 0.90, 0.90, 3, 4)
+    np.testing.assert_array_equal(sums.cpu().numpy(), want)
+
+
 def test_position_metrics_vs_oracle(sdd, orc):
     q, L = _synthetic_log(300, 16, 5)
     qd, Ld = torch.from_numpy(q).cuda(), torch.from_numpy(L).cuda()
