@@ -69,10 +69,51 @@ def _P(t):
 
 def lib():
     global _lib
-    if _lib is not None:
-        return _lib
-    build()
-    L = ctypes.CDLL(_LIB_PATH)
+    if _lib is None:
+        _lib = _bind(build())
+    return _lib
+
+
+def build_variant(replacements, out_dir: str) -> str:
+    """Compile a copy of the oracle source with each (old, new) text
+    replacement applied (every `old` must occur exactly once) into out_dir.
+    Tests use it to plant a mistake in the oracle and check that a pin fails."""
+    src = open(_SRC).read()
+    for old, new in replacements:
+        if src.count(old) != 1:
+            raise ValueError(f"replacement target must occur once: {old!r}")
+        src = src.replace(old, new)
+    os.makedirs(out_dir, exist_ok=True)
+    c_path = os.path.join(out_dir, "sdd_oracle_variant.c")
+    so_path = os.path.join(out_dir, "liboracle_variant.so")
+    with open(c_path, "w") as f:
+        f.write(src)
+    subprocess.check_call(["gcc", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared", "-std=c11",
+                           "-o", so_path, c_path, "-lm"])
+    return so_path
+
+
+class using_library:
+    """Context manager: route every oracle call through the library at `path`
+    (a variant from build_variant) and restore the real one afterwards."""
+
+    def __init__(self, path: str):
+        self.path = path
+
+    def __enter__(self):
+        global _lib
+        self.saved = lib()
+        _lib = _bind(self.path)
+        return self
+
+    def __exit__(self, *exc):
+        global _lib
+        _lib = self.saved
+        return False
+
+
+def _bind(path: str):
+    L = ctypes.CDLL(path)
     dp, ip32, ip64, up8, up32, up64 = (_P(ctypes.c_double), _P(ctypes.c_int32), _P(ctypes.c_int64),
                                        _P(ctypes.c_uint8), _P(ctypes.c_uint32), _P(ctypes.c_uint64))
     L.orc_philox4x32_10.argtypes = [up32, up32, up32]
@@ -118,7 +159,8 @@ def lib():
                                              ctypes.c_double, ctypes.c_int, ctypes.c_uint64, ip64, dp, ip32, ip32,
                                              ip32, ip32]
     L.orc_permutation_diagnostic.restype = None
-    _lib = L
+    L.orc_shuffle.argtypes = [ctypes.c_int, ctypes.c_uint64, ctypes.c_int, ctypes.c_int, ip32]
+    L.orc_shuffle.restype = None
     return L
 
 
@@ -383,8 +425,8 @@ def survival_mlp(h_bits, W1_bits, b1, w2_bits, b2: float) -> np.ndarray:
 
 
 def scorer_deep(x_bits, W1_bits, b1, W2_bits, b2, W3_bits, b3, w4_bits, b4: float) -> np.ndarray:
-    """fp64 sigmoid(w4 . GELU(W3 a2 + b3) + b4), a2 = bf16(GELU(W2 a1 + b2)),
-    a1 = bf16(GELU(W1 x + b1)) per row of x.  x_bits [M, K], W1 [N, K], W2 and W3
+    """fp64 sigmoid(w4 . GELU(W3 a2 + b3) + b4), a2 = GELU(W2 a1 + b2),
+    a1 = GELU(W1 x + b1) per row of x, every activation in fp64.  x_bits [M, K], W1 [N, K], W2 and W3
     [N, N], w4 [N]: raw bf16 bits (uint16); biases fp32 [N]."""
     u16 = lambda a: np.ascontiguousarray(np.asarray(a, dtype=np.uint16))   # noqa: E731
     f32 = lambda a: np.ascontiguousarray(np.asarray(a, dtype=np.float32))  # noqa: E731
@@ -419,6 +461,14 @@ def permutation_diagnostic(q, L, signal, eta_b, eta_c, n_rep, seed):
                                      float(eta_c), int(n_rep), ctypes.c_uint64(int(seed)), _ptr(sums, ctypes.c_int64),
                                      _ptr(qp, ctypes.c_double), i32(lst), i32(kh), i32(k), i32(d))
     return sums
+
+
+def shuffle(n: int, seed: int, j0: int, r: int) -> np.ndarray:
+    """The diagnostic's Fisher-Yates permutation of 0..n-1 for repetition r
+    and 0-based position j0."""
+    perm = np.zeros(max(n, 1), np.int32)
+    lib().orc_shuffle(int(n), ctypes.c_uint64(int(seed)), int(j0), int(r), _ptr(perm, ctypes.c_int32))
+    return perm[:n]
 
 
 def position_metrics(q, L, conditional: bool):

@@ -104,10 +104,19 @@ void orc_uniform_many(int64_t n, uint64_t seed, const uint32_t *j, const uint32_
 /* Two-pass plain definition: m = max z, LSE = m + ln sum exp(z - m),         */
 /* p(v) = exp(z(v) - LSE), maxprob = exp(m - LSE), H = -sum p ln p,          */
 /* argmax = lowest index attaining m, q = p(token), logq = z(token) - LSE.   */
-/* A row with NaN or +inf anywhere, or with every entry -inf, has no         */
-/* distribution: all its outputs are NaN and argmax is -1.                   */
-/* Pinned by closed forms and by fp64 library softmax/logsumexp/entr.        */
+/* Logits are clamped from below at -2^23 (z <- max(z, -2^23); -inf too), so */
+/* an entry at or below the floor contributes exp(-2^23 - m), which is 0 in  */
+/* fp64 unless the row's maximum m lies within ~745 of the floor.  A row     */
+/* with NaN or +inf anywhere, or whose clamped maximum is the floor itself   */
+/* (every entry -inf or at most -2^23), has no distribution: all its outputs */
+/* are NaN and argmax is -1.                                                 */
+/* Pinned by closed forms, by fp64 library softmax/logsumexp/entr, and by    */
+/* rows below the floor.                                                     */
 /* ------------------------------------------------------------------------ */
+static const double orc_floor = -8388608.0; /* -2^23 */
+
+static double orc_clamp(double z) { return (z < orc_floor) ? orc_floor : z; }
+
 void orc_row_stats(const void *logits, int dtype, int64_t n_rows, int64_t V, int64_t row_stride,
                    const int32_t *tokens, /* [n_rows] or NULL */
                    double *out_m, double *out_lse, double *out_q, double *out_logq,
@@ -120,9 +129,10 @@ void orc_row_stats(const void *logits, int dtype, int64_t n_rows, int64_t V, int
         for (int64_t v = 0; v < V; ++v) {
             double z = orc_load(logits, dtype, base + v);
             if (isnan(z) || (isinf(z) && z > 0)) bad = 1;
+            z = orc_clamp(z);
             if (z > m) { m = z; amax = v; }
         }
-        if (m == -INFINITY) bad = 1;
+        if (!(m > orc_floor)) bad = 1;
         int64_t tok = tokens ? (int64_t)tokens[r] : -1;
         if (tokens && (tok < 0 || tok >= V)) bad = 1;
         if (bad) {
@@ -136,11 +146,11 @@ void orc_row_stats(const void *logits, int dtype, int64_t n_rows, int64_t V, int
             continue;
         }
         double s = 0.0;
-        for (int64_t v = 0; v < V; ++v) s += exp(orc_load(logits, dtype, base + v) - m);
+        for (int64_t v = 0; v < V; ++v) s += exp(orc_clamp(orc_load(logits, dtype, base + v)) - m);
         double lse = m + log(s);
         double H = 0.0;
         for (int64_t v = 0; v < V; ++v) {
-            double z = orc_load(logits, dtype, base + v);
+            double z = orc_clamp(orc_load(logits, dtype, base + v));
             double p = exp(z - lse);
             if (p > 0.0) H -= p * (z - lse);
         }
@@ -150,7 +160,7 @@ void orc_row_stats(const void *logits, int dtype, int64_t n_rows, int64_t V, int
         if (out_entropy) out_entropy[r] = H;
         if (out_argmax) out_argmax[r] = (int32_t)amax;
         if (tokens) {
-            double zt = orc_load(logits, dtype, base + tok);
+            double zt = orc_clamp(orc_load(logits, dtype, base + tok));
             if (out_q) out_q[r] = exp(zt - lse);
             if (out_logq) out_logq[r] = zt - lse;
         } else {
@@ -174,7 +184,6 @@ void orc_row_stats(const void *logits, int dtype, int64_t n_rows, int64_t V, int
 /* ------------------------------------------------------------------------ */
 void orc_row_features(const void *logits, int dtype, int64_t n_rows, int64_t V, int64_t row_stride,
                       double *out_margin, double *out_top5) {
-    const double floor_ = -8388608.0; /* -2^23 */
     for (int64_t r = 0; r < n_rows; ++r) {
         int64_t base = r * row_stride;
         double top[5] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY, -INFINITY};
@@ -183,9 +192,10 @@ void orc_row_features(const void *logits, int dtype, int64_t n_rows, int64_t V, 
         for (int64_t v = 0; v < V; ++v) {
             double z = orc_load(logits, dtype, base + v);
             if (isnan(z) || (isinf(z) && z > 0)) bad = 1;
+            z = orc_clamp(z);
             if (z > m) m = z;
         }
-        if (m == -INFINITY) bad = 1;
+        if (!(m > orc_floor)) bad = 1;
         if (bad) {
             out_margin[r] = NAN;
             out_top5[r] = NAN;
@@ -194,7 +204,7 @@ void orc_row_features(const void *logits, int dtype, int64_t n_rows, int64_t V, 
         double s = 0.0;
         for (int64_t v = 0; v < V; ++v) {
             double z = orc_load(logits, dtype, base + v);
-            if (z < floor_) z = floor_;
+            z = orc_clamp(z);
             s += exp(z - m);
             /* insert z into the descending list of the 5 largest values */
             for (int i = 0; i < 5; ++i) {
@@ -215,17 +225,20 @@ void orc_row_features(const void *logits, int dtype, int64_t n_rows, int64_t V, 
     }
 }
 
-/* Normalised probabilities of one row, p(v) = exp(z(v) - LSE), fp64. */
+/* Normalised probabilities of one row, p(v) = exp(z(v) - LSE) with the     */
+/* logits clamped at -2^23 as above, fp64 (the softmax the strict rule's     */
+/* residual max(0, p_t - p_d) and bonus draw are built from, Sec. 3.1).      */
+/* Pinned against fp64 library softmax on random, peaked and masked rows.   */
 void orc_row_probs(const void *logits, int dtype, int64_t V, int64_t offset, double *p) {
     double m = -INFINITY;
     for (int64_t v = 0; v < V; ++v) {
-        double z = orc_load(logits, dtype, offset + v);
+        double z = orc_clamp(orc_load(logits, dtype, offset + v));
         if (z > m) m = z;
     }
     double s = 0.0;
-    for (int64_t v = 0; v < V; ++v) s += exp(orc_load(logits, dtype, offset + v) - m);
+    for (int64_t v = 0; v < V; ++v) s += exp(orc_clamp(orc_load(logits, dtype, offset + v)) - m);
     double lse = m + log(s);
-    for (int64_t v = 0; v < V; ++v) p[v] = exp(orc_load(logits, dtype, offset + v) - lse);
+    for (int64_t v = 0; v < V; ++v) p[v] = exp(orc_clamp(orc_load(logits, dtype, offset + v)) - lse);
 }
 
 /* Rank of `token` in one row under the order (larger logit first, then lower
@@ -511,24 +524,12 @@ void orc_survival_mlp(const uint16_t *h, int M, int K, const uint16_t *W1, const
 /* features] (K = 3584 + 19 in the paper), random-init stand-in weights:     */
 /*   a1 = GELU(W1 x + b1), a2 = GELU(W2 a1 + b2), a3 = GELU(W3 a2 + b3),      */
 /*   s  = sigmoid(w4 . a3 + b4).                                             */
-/* a1 and a2 are rounded to bf16 (round to nearest even, from fp32) before   */
-/* the next layer: the tensor-core path consumes them as bf16 operands, so   */
-/* the oracle takes the same rounding (dropout is a training-time op).  W1  */
-/* is [N, K], W2 and W3 [N, N] (one row per output unit), w4 [N]: bf16 bits. */
+/* Every activation stays in fp64: the paper fixes no precision for the     */
+/* scorer (dropout is a training-time op and is absent here).  W1 is [N, K], */
+/* W2 and W3 [N, N] (one row per output unit), w4 [N]: bf16 bits.            */
 /* Pinned in tests/test_oracle_mlp.py (closed forms of single-path nets,     */
-/* hidden-unit permutation invariance, bf16 rounding of the activations).   */
+/* zero weights, hidden-unit permutation invariance, a library fp64 chain). */
 /* ------------------------------------------------------------------------ */
-static double orc_round_bf16(double v) {
-    float f = (float)v;
-    uint32_t u;
-    memcpy(&u, &f, sizeof u);
-    if ((u & 0x7F800000u) != 0x7F800000u) { /* finite: round to nearest even */
-        u = (u + 0x7FFFu + ((u >> 16) & 1u)) & 0xFFFF0000u;
-    }
-    memcpy(&f, &u, sizeof f);
-    return (double)f;
-}
-
 static double orc_gelu(double z) { return 0.5 * z * (1.0 + erf(z / sqrt(2.0))); }
 
 void orc_scorer_deep(const uint16_t *x, int M, int K, const uint16_t *W1, const float *b1, const uint16_t *W2,
@@ -540,12 +541,12 @@ void orc_scorer_deep(const uint16_t *x, int M, int K, const uint16_t *W1, const 
             double z = (double)b1[n];
             for (int k = 0; k < K; ++k)
                 z += orc_load(W1, ORC_BF16, (int64_t)n * K + k) * orc_load(x, ORC_BF16, (int64_t)m * K + k);
-            a1[n] = orc_round_bf16(orc_gelu(z));
+            a1[n] = orc_gelu(z);
         }
         for (int n = 0; n < N; ++n) {
             double z = (double)b2[n];
             for (int k = 0; k < N; ++k) z += orc_load(W2, ORC_BF16, (int64_t)n * N + k) * a1[k];
-            a2[n] = orc_round_bf16(orc_gelu(z));
+            a2[n] = orc_gelu(z);
         }
         double t = b4;
         for (int n = 0; n < N; ++n) {
@@ -575,6 +576,24 @@ void orc_scorer_deep(const uint16_t *x, int M, int K, const uint16_t *W1, const 
 /* rows are invariant, permutations preserve every column's multiset, a      */
 /* closed form of the independent-position expectation).                    */
 /* ------------------------------------------------------------------------ */
+/* The shuffle of (r, j) on its own: perm[0..n) starts as 0..n-1 and slot i */
+/* (from n - 1 down to 1) swaps with k = floor(w (i + 1) / 2^32), w the first */
+/* Philox word of counter (i, j0, r, 3), so k is uniform on 0..i (Fisher-    */
+/* Yates; Durstenfeld's in-place form).  j0 = j - 1 is the 0-based position. */
+/* Pinned by a chi-square test over all n! permutations for n <= 4.          */
+void orc_shuffle(int n, uint64_t seed, int j0, int r, int32_t *perm) {
+    uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+    for (int t = 0; t < n; ++t) perm[t] = t;
+    for (int i = n - 1; i > 0; --i) {
+        uint32_t ctr[4] = {(uint32_t)i, (uint32_t)j0, (uint32_t)r, 3u}, out[4];
+        orc_philox4x32_10(ctr, key, out);
+        int k = (int)(((uint64_t)out[0] * (uint64_t)(i + 1)) >> 32);
+        int32_t tmp = perm[i];
+        perm[i] = perm[k];
+        perm[k] = tmp;
+    }
+}
+
 void orc_permutation_diagnostic(const double *q, const int32_t *L, int B, int gamma, int signal, double eta_b,
                                 double eta_c, int n_rep, uint64_t seed, int64_t *sums, double *qp, int32_t *list,
                                 int32_t *Khat, int32_t *K, int32_t *D) {
@@ -587,21 +606,12 @@ void orc_permutation_diagnostic(const double *q, const int32_t *L, int B, int ga
                 int n = 0;
                 for (int b = 0; b < B; ++b)
                     if (signal != 2 || L[b] >= j) list[n++] = b;
-                uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
-                int32_t *sh = list + 0; /* shuffled in place; the valid order is recomputed below */
-                int32_t *valid = (int32_t *)malloc(sizeof(int32_t) * (n > 0 ? n : 1));
-                for (int t = 0; t < n; ++t) valid[t] = sh[t];
-                for (int i = n - 1; i > 0; --i) {
-                    uint32_t ctr[4] = {(uint32_t)i, (uint32_t)j, (uint32_t)r, 3u}, out[4];
-                    orc_philox4x32_10(ctr, key, out);
-                    int k = (int)(((uint64_t)out[0] * (uint64_t)(i + 1)) >> 32);
-                    int32_t tmp = sh[i];
-                    sh[i] = sh[k];
-                    sh[k] = tmp;
-                }
+                int32_t *perm = (int32_t *)malloc(sizeof(int32_t) * (n > 0 ? n : 1));
+                orc_shuffle(n, seed, j, r, perm);
+                /* the t-th valid block takes the score of valid block perm[t] */
                 for (int t = 0; t < n; ++t)
-                    qp[(int64_t)valid[t] * gamma + j] = q[(int64_t)sh[t] * gamma + j];
-                free(valid);
+                    qp[(int64_t)list[t] * gamma + j] = q[(int64_t)list[perm[t]] * gamma + j];
+                free(perm);
             }
         }
         orc_schedule(qp, B, gamma, signal, eta_b, eta_c, 0, 0x7FFFFFFF, NULL, NULL, NULL, Khat, K, D, NULL);

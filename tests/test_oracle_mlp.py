@@ -85,8 +85,8 @@ def test_hidden_unit_permutation_invariance(orc):
 
 
 # ---------------------------------------------------------------------------
-# The learned scorer's shape (App. A.7): K -> N -> N -> N -> 1, GELU, with the
-# first two layers' activations rounded to bf16 (the tensor-core operands)
+# The learned scorer's shape (App. A.7): K -> N -> N -> N -> 1, GELU, every
+# activation in fp64
 # ---------------------------------------------------------------------------
 
 def _b(a):
@@ -117,9 +117,9 @@ def test_deep_zero_weights_closed_form(orc):
     np.testing.assert_allclose(s, 1.0 / (1.0 + math.exp(-t)), rtol=1e-14)
 
 
-def test_deep_single_path_closed_form_with_bf16_activations(orc):
-    """One weight per layer: s = sigmoid(e GELU(d r(GELU(c r(GELU(a x_j + beta)))))),
-    r = rounding to bf16; every other unit sees GELU(0) = 0."""
+def test_deep_single_path_closed_form(orc):
+    """One weight per layer: s = sigmoid(e GELU(d GELU(c GELU(a x_j + beta)))),
+    every other unit sees GELU(0) = 0; the activations are not rounded."""
     N, K, j, i, pu, q = 6, 10, 3, 2, 4, 1
     a, beta, c, d, e = 1.25, 0.3, -0.75, 1.5, 2.0
     W1, z = _zeros(N, K)
@@ -136,12 +136,29 @@ def test_deep_single_path_closed_form_with_bf16_activations(orc):
     x[0, j], x[1, j] = 0.6875, -2.5
     s = orc.scorer_deep(_b(x), _b(W1), b1, _b(W2), z, _b(W3), z, _b(w4), 0.0)
     for m in range(2):
-        a1 = _rbf16(_gelu(a * x[m, j] + float(np.float32(beta))))
-        a2 = _rbf16(_gelu(c * a1))
-        t = e * _gelu(d * a2)
+        t = e * _gelu(d * _gelu(c * _gelu(a * float(x[m, j]) + float(np.float32(beta)))))
         assert s[m] == pytest.approx(1.0 / (1.0 + math.exp(-t)), rel=1e-14)
-        unrounded = 1.0 / (1.0 + math.exp(-e * _gelu(d * _gelu(c * _gelu(a * x[m, j] + float(np.float32(beta)))))))
-        assert abs(s[m] - unrounded) > 1e-9   # the rounding is really applied
+        rounded = e * _gelu(d * _rbf16(_gelu(c * _rbf16(_gelu(a * float(x[m, j]) + float(np.float32(beta)))))))
+        assert abs(s[m] - 1.0 / (1.0 + math.exp(-rounded))) > 1e-9   # no activation is rounded
+
+
+def test_deep_matches_library_chain(orc):
+    """Special case that reduces to library routines: fp64 torch Linear / gelu
+    (erf form) / sigmoid on the same bf16 weights and inputs."""
+    rng = np.random.default_rng(11)
+    M, K, N = 9, 48, 24
+    x = _b(rng.normal(size=(M, K)))
+    W1, W2, W3 = (rng.uniform(-1, 1, s) / math.sqrt(s[1]) for s in ((N, K), (N, N), (N, N)))
+    b1, b2, b3 = (rng.uniform(-0.3, 0.3, N).astype(np.float32) for _ in range(3))
+    w4 = rng.uniform(-1, 1, N) / math.sqrt(N)
+    s = orc.scorer_deep(x, _b(W1), b1, _b(W2), b2, _b(W3), b3, _b(w4), 0.125)
+    v = lambda a: torch.from_numpy(np.asarray(a, np.float32)).to(torch.bfloat16).double()   # noqa: E731
+    F = torch.nn.functional
+    a1 = F.gelu(F.linear(torch.from_numpy(bf16_vals(x)), v(W1), torch.from_numpy(b1).double()))
+    a2 = F.gelu(F.linear(a1, v(W2), torch.from_numpy(b2).double()))
+    a3 = F.gelu(F.linear(a2, v(W3), torch.from_numpy(b3).double()))
+    want = torch.sigmoid(a3 @ v(w4) + 0.125).numpy()
+    np.testing.assert_allclose(s, want, rtol=1e-12, atol=1e-15)
 
 
 def test_deep_hidden_unit_permutation_invariance(orc):
