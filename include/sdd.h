@@ -26,14 +26,14 @@
  * Streams.  Every call only enqueues work on `stream` (a cudaStream_t; NULL is
  *   the legacy default stream) and returns without synchronising.
  * Workspace.  Calls that take `workspace` need at least sdd_workspace_size()
- *   bytes of device memory, 256-byte aligned and ZERO-FILLED before its first
- *   use; it holds the streaming kernel's per-warp partial statistics and the
- *   sampling draw's per-segment totals and arrival counters.  Every call that
- *   completes returns those counters to zero, so one workspace serves any
- *   number of stream-ordered calls.  Calls that may
- *   overlap on the GPU (different streams) need separate workspaces.  After a
- *   call whose device status reports SDD_DEV_TIMEOUT the workspace must be
- *   zero-filled again.
+ *   bytes of device memory for their (B, gamma, V), 256-byte aligned; it holds
+ *   the streaming kernel's per-warp partial statistics and the sampling draw's
+ *   per-segment prefix sums and arrival counters.  Its contents need no
+ *   initialisation: every call writes what it reads and resets the arrival
+ *   counters of its blocks before its draw, so one workspace serves any
+ *   sequence of stream-ordered calls whose shapes it is large enough for (also
+ *   after a call whose device status reports SDD_DEV_TIMEOUT).  Calls that may
+ *   overlap on the GPU (different streams) need separate workspaces.
  * Errors.  The return value reports host-side problems only: invalid
  *   arguments are detected before anything is enqueued (SDD_ERR_INVALID_ARGUMENT)
  *   and launch failures return SDD_ERR_CUDA.  Conditions found while the
@@ -98,7 +98,7 @@ SDD_API int sdd_version(void);
 SDD_API const char *sdd_last_error(void);
 
 /*
- * sdd_workspace_size -- bytes of zero-filled device scratch that any entry
+ * sdd_workspace_size -- bytes of device scratch that any entry
  * point needs for blocks of this shape on the CURRENT device (the figure
  * depends on its SM count).  B, gamma, V as in the calls below.
  */

@@ -166,7 +166,8 @@ def workspace_bytes(B: int, gamma: int, V: int) -> int:
 
 
 class Workspace:
-    """Zero-filled, 256-byte aligned device scratch for blocks up to (B, gamma)."""
+    """256-byte aligned device scratch for any call with at most B blocks of at
+    most gamma positions (its contents need no initialisation)."""
 
     def __init__(self, B: int, gamma: int, V: int, device=None):
         self.nbytes = workspace_bytes(B, gamma, V)

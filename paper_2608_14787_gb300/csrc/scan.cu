@@ -442,6 +442,12 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
     // launched as a programmatic dependent of whatever precedes it in the
     // stream: nothing is read or written before that work has completed
     griddep_wait();
+    // The sampling draw's arrival counters of this call's blocks start at zero
+    // (the decide kernel behind this one reads them only after this grid has
+    // completed), so the workspace needs no zero fill and calls of any shape
+    // that fits it may follow one another.
+    if (gw == 0 && p.dec.enabled && p.dec.res_count != nullptr)
+        for (int i = lane; i < p.grp[0].nb; i += 32) p.dec.res_count[i] = 0u;
     constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
     const int tail = p.V % EPV;  // valid entries of the last vector of a row (0 = full)
 

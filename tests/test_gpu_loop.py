@@ -8,6 +8,7 @@ import pytest
 import torch
 
 from paper_2608_14787_gb300 import synth
+from paper_2608_14787_gb300.binding import MLP_HIDDEN
 from paper_2608_14787_gb300.loop import DecodeLoop
 
 pytestmark = pytest.mark.gpu
@@ -16,6 +17,20 @@ NEAR = 1e-6
 
 def _bits(t):
     return synth.bf16_bits(t)
+
+
+def _oracle_features(orc, st, zd, gamma, round_):
+    """The scorer's scalar-feature block (App. A.7's column order; the drafter
+    quantities without a counterpart here stay 0) from the oracle's row
+    statistics and features, rounded to bf16 bits: [B * gamma, 256]."""
+    B = st.q.shape[0]
+    margin, top5 = orc.row_features(zd)
+    cols = {4: st.maxprob, 5: np.log(st.maxprob), 6: st.entropy, 7: -st.entropy, 8: margin, 9: top5,
+            14: np.broadcast_to(np.arange(gamma) / gamma, (B, gamma)), 15: np.full((B, gamma), round_ / 256.0)}
+    f = np.zeros((B * gamma, MLP_HIDDEN), np.float32)
+    for c, v in cols.items():
+        f[:, c] = np.asarray(v, np.float64).reshape(-1)
+    return _bits(torch.from_numpy(f).to(torch.bfloat16))
 
 
 @pytest.mark.parametrize("scorer", ["deep", "mlp"])
@@ -39,10 +54,11 @@ def test_loop_matches_oracle_replay(sdd, orc, B, gamma, V, hidden, rounds, score
         st = orc.row_stats(zd, tokens=x)
         _, K_raw, D_raw, mg_raw = orc.schedule(st.q, orc.SIG_RAW, 0.5, 0.5, 2, 6, D_in=D_raw)
         if scorer == "deep":
-            # the scorer on the device's feature block (the features are pinned by their own parity tests)
+            # the scorer on a feature block built from the oracle's own row statistics
             W1, b1, W2, b2, W3, b3, w4, b4 = loop.deep
-            x_in = torch.cat([h, loop.feat], dim=-1)
-            s = orc.scorer_deep(_bits(x_in), _bits(W1), b1.cpu().numpy(), _bits(W2), b2.cpu().numpy(), _bits(W3),
+            feat = _oracle_features(orc, st, zd, gamma, r)
+            x_in = np.concatenate([_bits(h).reshape(B * gamma, -1), feat], axis=-1)
+            s = orc.scorer_deep(x_in, _bits(W1), b1.cpu().numpy(), _bits(W2), b2.cpu().numpy(), _bits(W3),
                                 b3.cpu().numpy(), _bits(w4), b4).reshape(B, gamma)
         else:
             s = orc.survival_mlp(_bits(h), _bits(loop.W1), loop.b1.cpu().numpy(), _bits(loop.w2),

@@ -5,9 +5,9 @@ code running under CUDA stream capture, where cudaMalloc is not allowed, or a
 framework whose device memory is a fixed arena it owns.  The library serves
 them from a fixed scratch array of its own.  This test calls that entry point
 through the C ABI twice in a row (the second call starts from whatever the
-first left in the shared scratch) and checks each result against
-sdd_confidence, which takes a caller-provided workspace, with the tolerances
-of the other parity tests.  It lives in a file of its own that is collected
+first left in the shared scratch) and checks each result against the fp64
+oracle, element by element, and against sdd_confidence, which takes a
+caller-provided workspace, with the tolerances of the other parity tests.  It lives in a file of its own that is collected
 last, and passes both alone in a fresh process and after the other tests."""
 import ctypes
 
@@ -30,7 +30,7 @@ def _padded(z, stride):
 
 def _same(name, got, want, dtype):
     g = got.double().cpu().numpy()
-    w = want.double().cpu().numpy()
+    w = want.double().cpu().numpy() if isinstance(want, torch.Tensor) else np.asarray(want, np.float64)
     if name == "logq":      # a log-probability: absolute error = relative error of q
         ok = np.abs(g - w) <= RTOL[dtype]
     else:
@@ -39,7 +39,7 @@ def _same(name, got, want, dtype):
     assert ok.all(), f"{name}: {(~ok).sum()} entries differ"
 
 
-def test_noalloc_matches_workspace_call_twice_in_a_row():
+def test_noalloc_matches_oracle_and_workspace_call_twice_in_a_row(orc):
     import paper_2608_14787_gb300 as sdd
     from paper_2608_14787_gb300 import synth
     if not torch.cuda.is_available():
@@ -56,8 +56,11 @@ def test_noalloc_matches_workspace_call_twice_in_a_row():
         got = sdd.confidence_noalloc(z, blk.x, status=status)
         torch.cuda.synchronize()
         assert int(status.item()) == 0
+        st = orc.row_stats(synth.bf16_bits(blk.z_d), tokens=blk.x.cpu().numpy())
         for f in ("q", "logq", "maxprob", "lse", "entropy"):
+            _same(f, getattr(got, f), getattr(st, f), dtype)
             _same(f, getattr(got, f), getattr(want, f), dtype)
+        np.testing.assert_array_equal(got.argmax.cpu().numpy(), st.argmax)
         assert torch.equal(got.argmax, want.argmax)
 
 
