@@ -38,7 +38,6 @@ sys.path.insert(0, ROOT)
 
 METRIC = "draft blocks verified+scheduled/sec at γ=32,V=151,936 bf16; achieved HBM GB/s vs peak"
 UNIT = "blocks/s"
-EV_EVERY = 8   # steps between the event-bracketed launches of the streaming kernel
 NEAR = 1e-6
 # dram__bytes_read.sum + dram__bytes_write.sum of one scan_kernel launch on the
 # c3 workload (318.23 MB + 3.48 MB), from one ncu capture of the kernel as it
@@ -133,75 +132,155 @@ def _dist():
     return ws, rank, local
 
 
+def _host_info():
+    """Host cores (nproc) and CPU model, for the oracle baseline."""
+    nproc = os.cpu_count() or 1
+    model = None
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                key = line.split(":")[0].strip().lower()
+                if key in ("model name", "cpu part", "hardware") and ":" in line:
+                    model = line.split(":", 1)[1].strip()
+                    if key == "model name":
+                        break
+    except OSError:
+        pass
+    if model is None:
+        try:
+            out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+            for line in out.splitlines():
+                if line.lower().startswith("model name"):
+                    model = line.split(":", 1)[1].strip()
+                    break
+        except Exception:
+            pass
+    return nproc, model or "unknown"
+
+
+def _oracle_one_block(wl, ells, ks, zd, zt, xs, b, round_):
+    """Every rule of the path for one block through the fp64 oracle: the raw
+    schedule per tau (K, margin), strict sampling, lenience per ell and top-k
+    per k (L, tokens, margin)."""
+    import oracle as orc
+    st = orc.row_stats(zd[b:b + 1], tokens=xs[b:b + 1])
+    sched = [orc.schedule(st.q, 0, tau, tau, 6, 64) for tau in wl.taus]
+    out = {"K": [(int(k[1][0]), float(k[3][0])) for k in sched],
+           "strict": orc.verify_strict(zt[b], zd[b], xs[b], seed=wl.seed, b=b, round_=round_)}
+    f = orc.target_facts(zt[b], xs[b])
+    out["lenient"] = [orc.verify_lenient(f, xs[b], e) for e in ells]
+    out["topk"] = [orc.verify_topk(f, xs[b], k) for k in ks]
+    return out
+
+
+def _oracle_blocks(wl, ells, ks, host, blocks, threads, round_=0):
+    """The oracle over `blocks` of one input set, split over `threads` host
+    threads (the oracle's C calls release the interpreter lock, so the threads
+    run on separate cores).  Returns (seconds, {block: results})."""
+    from concurrent.futures import ThreadPoolExecutor
+    zd, zt, xs = host["z_d"], host["z_t"], host["x"]
+    t0 = time.perf_counter()
+    if threads <= 1:
+        res = [_oracle_one_block(wl, ells, ks, zd, zt, xs, b, round_) for b in blocks]
+    else:
+        with ThreadPoolExecutor(max_workers=threads) as ex:
+            res = list(ex.map(lambda b: _oracle_one_block(wl, ells, ks, zd, zt, xs, b, round_), blocks))
+    return time.perf_counter() - t0, dict(zip(blocks, res))
+
+
+def _host_block(blk, wl):
+    import numpy as np
+    import torch
+
+    def h(t):
+        t = t.detach().cpu()
+        return t.view(torch.int16).numpy().view(np.uint16) if t.dtype == torch.bfloat16 else t.numpy()
+    return {"z_d": h(blk.z_d), "z_t": h(blk.z_t), "x": blk.x.detach().cpu().numpy()}
+
+
 def run_reference(args):
-    """The fp64 CPU oracle, as it stands, on a bounded sample per step (one block)."""
+    """The fp64 CPU oracle, as it stands, on the host's cores: each step is a
+    bounded sample of the workload (one block per host thread, all rules)."""
     ws, rank, _ = _dist()
     if rank != 0:
         return 0
-    import numpy as np
-    import torch
-    import oracle as orc
     from paper_2608_14787_gb300 import synth
     wl, ells, ks = _workload_cfg(args.workload)
-    blk = synth.make_block(wl, device="cpu", round_=0)
-    zd = blk.z_d.view(torch.int16).numpy().view(np.uint16) if wl.dtype == torch.bfloat16 else blk.z_d.numpy()
-    zt = blk.z_t.view(torch.int16).numpy().view(np.uint16) if wl.dtype == torch.bfloat16 else blk.z_t.numpy()
-    xs = blk.x.numpy()
+    nproc, model = _host_info()
+    threads = max(1, min(nproc, args.ref_threads or nproc))
+    host = _host_block(synth.make_block(wl, device="cpu", round_=0), wl)
 
-    def one_block(b):
-        st = orc.row_stats(zd[b:b + 1], tokens=xs[b:b + 1])
-        for tau in wl.taus:
-            orc.schedule(st.q, 0, tau, tau, 6, 64)
-        orc.verify_strict(zt[b], zd[b], xs[b], seed=wl.seed, b=b, round_=0)
-        f = orc.target_facts(zt[b], xs[b])
-        for e in ells:
-            orc.verify_lenient(f, xs[b], e)
-        for k in ks:
-            orc.verify_topk(f, xs[b], k)
+    def step(s):
+        blocks = [(s * threads + t) % wl.B for t in range(threads)]
+        _oracle_blocks(wl, ells, ks, host, blocks, threads)
 
     for s in range(args.warmup):
-        one_block(s % wl.B)
+        step(s)
     t0 = time.perf_counter()
     for s in range(args.steps):
-        one_block(s % wl.B)
+        step(s)
     dt = time.perf_counter() - t0
-    value = args.steps / dt
-    sample = f"one {wl.name} block (gamma={wl.gamma}, V={wl.V}) per step, all rules, single thread"
+    value = args.steps * threads / dt
+    sample = (f"{threads} {wl.name} blocks per step (gamma={wl.gamma}, V={wl.V}), one per host thread, "
+              f"all rules")
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": _config_json(wl, ells, ks),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample,
+                         "nproc": nproc, "cpu_model": model},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
     return 0
 
 
-def _cpu_baseline(wl, ells, ks, blk_host, n_blocks):
-    """Time the oracle on the first n_blocks blocks of one input set (bounded sample)."""
+def _cpu_baseline(wl, ells, ks, host, n_single):
+    """The oracle timed on a bounded sample of one input set: one thread over
+    the first n_single blocks, and all host cores over every block.  Returns
+    (cpu_baseline dict, the all-core run's per-block results)."""
+    nproc, model = _host_info()
+    dt1, _ = _oracle_blocks(wl, ells, ks, host, list(range(n_single)), 1)
+    blocks = list(range(wl.B))
+    dtn, res = _oracle_blocks(wl, ells, ks, host, blocks, nproc)
+    base = {"value": len(blocks) / dtn, "unit": UNIT, "cores": min(nproc, len(blocks)), "kind": "oracle",
+            "sample": f"all {wl.B} blocks of one {wl.name} input set, all rules, one block per thread on "
+                      f"{min(nproc, len(blocks))} of {nproc} host cores ({dtn:.1f} s)",
+            "nproc": nproc, "cpu_model": model,
+            "single_thread": {"value": n_single / dt1, "unit": UNIT, "cores": 1,
+                              "sample": f"the first {n_single} blocks, one thread ({dt1:.1f} s)"}}
+    return base, res
+
+
+def _parity_sample(rnd, res, ells, ks):
+    """Compare one round's device outputs with the oracle's results for the
+    same blocks (decisions bit-exact; a decision whose oracle margin is within
+    1e-6 of its threshold is counted as flagged, not compared)."""
     import numpy as np
-    import torch
-    import oracle as orc
-    zd = blk_host["z_d"]
-    zt = blk_host["z_t"]
-    xs = blk_host["x"]
-    t0 = time.perf_counter()
-    for b in range(n_blocks):
-        st = orc.row_stats(zd[b:b + 1], tokens=xs[b:b + 1])
-        for tau in wl.taus:
-            orc.schedule(st.q, 0, tau, tau, 6, 64)
-        orc.verify_strict(zt[b], zd[b], xs[b], seed=wl.seed, b=b, round_=0)
-        f = orc.target_facts(zt[b], xs[b])
-        for e in ells:
-            orc.verify_lenient(f, xs[b], e)
-        for k in ks:
-            orc.verify_topk(f, xs[b], k)
-    dt = time.perf_counter() - t0
-    del np, torch
-    return {"value": n_blocks / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{n_blocks} of the {wl.B} blocks of one {wl.name} input set, all rules, single thread "
-                      f"({dt:.1f} s)"}
+    got = {"K": rnd.K.cpu().numpy(), "L": rnd.L_strict.cpu().numpy(), "tok": rnd.tokens_strict.cpu().numpy(),
+           "Ll": rnd.L_lenient.cpu().numpy(), "tl": rnd.tokens_lenient.cpu().numpy(),
+           "Lk": rnd.L_topk.cpu().numpy(), "tk": rnd.tokens_topk.cpu().numpy()}
+    compared = flagged = mismatched = 0
+
+    def check(ok, margin):
+        nonlocal compared, flagged, mismatched
+        compared += 1
+        if margin < NEAR:
+            flagged += 1
+        elif not ok:
+            mismatched += 1
+    for b, r in res.items():
+        for t, (K, mg) in enumerate(r["K"]):
+            check(got["K"][t, b] == K, mg)
+        L, tok, mg = r["strict"]
+        check(got["L"][b] == L and np.array_equal(got["tok"][b], tok), mg)
+        for e in range(len(ells)):
+            L, tok, mg = r["lenient"][e]
+            check(got["Ll"][e, b] == L and np.array_equal(got["tl"][e, b], tok), mg)
+        for k in range(len(ks)):
+            L, tok, mg = r["topk"][k]
+            check(got["Lk"][k, b] == L and np.array_equal(got["tk"][k, b], tok), mg)
+    return {"blocks": len(res), "decisions": compared, "near_threshold": flagged, "mismatches": mismatched}
 
 
 def _e2e(args, ws, dev, stream, sets, rnd, wl, B):
@@ -299,14 +378,10 @@ def run_gpu(args):
     scan_bytes = (2 * gamma + 1) * V * esz * B          # every logit read once
     stream = torch.cuda.current_stream()
 
-    def step(i, ev=None):
+    def step(i):
         s = sets[i % n_sets]
         rnd.set_inputs(s.z_d, s.z_t, s.x, seed=wl.seed, round_=i)
-        if ev is not None:
-            ev[0].record(stream)
         rnd.scan()
-        if ev is not None:
-            ev[1].record(stream)
         rnd.decide()
 
     for i in range(args.warmup):
@@ -315,12 +390,10 @@ def run_gpu(args):
     if int(rnd.status.item()) != 0:
         raise RuntimeError(f"device status {int(rnd.status.item())} after warm-up")
 
-    # ---- device-resident timed region ----
-    # The streaming kernel's launch duration is bracketed by events on every
-    # EV_EVERY-th step only: an event between two launches stops the next
-    # round's launch from overlapping the tail of the previous one.
-    evs = {i: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for i in range(0, args.steps, EV_EVERY)}
+    # ---- device-resident timed region: exactly K rounds ----
+    # A short device-side spin keeps the stream busy while the host enqueues
+    # the rounds, so the start event fires with rounds already queued behind it
+    # (no host launch latency inside the region).
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     props = torch.cuda.get_device_properties(dev)
     bus = getattr(props, "pci_bus_id", None)
@@ -328,19 +401,43 @@ def run_gpu(args):
         dist.barrier()
     torch.cuda.synchronize()
     with ClockSampler(bus) as clk:
+        torch.cuda._sleep(int(args.prefill_us * 2.0e3))    # ~prefill_us at 2 GHz
         t_start.record(stream)
         for i in range(args.steps):
-            step(i, evs.get(i))
+            step(args.warmup + i)
         t_end.record(stream)
         torch.cuda.synchronize()
     if ws > 1:
         dist.barrier()
     total_ms = t_start.elapsed_time(t_end)
-    scan_ms = [a.elapsed_time(b) for a, b in evs.values()]
-    scan_avg_ms = sum(scan_ms) / len(scan_ms)
     total_ms = shard.max_over_ranks(total_ms, device=dev)   # blocks shard by rank: no data-path exchange
+    ms_per_step = total_ms / args.steps
     value = ws * B * args.steps / (total_ms / 1e3)
     status = int(rnd.status.item())
+
+    # ---- the streaming kernel alone, for the roofline: N back-to-back
+    # launches (rotating input sets) under one event pair ----
+    n_scan = max(50, args.scan_launches)
+    for i in range(3):
+        s = sets[i % n_sets]
+        rnd.set_inputs(s.z_d, s.z_t, s.x, seed=wl.seed, round_=i)
+        rnd.scan()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda._sleep(int(args.prefill_us * 2.0e3))
+    e0.record(stream)
+    for i in range(n_scan):
+        s = sets[i % n_sets]
+        rnd.set_inputs(s.z_d, s.z_t, s.x, seed=wl.seed, round_=i)
+        rnd.scan()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    scan_avg_ms = e0.elapsed_time(e1) / n_scan
+
+    # ---- one untimed round on input set 0 for the oracle parity sample ----
+    rnd.set_inputs(sets[0].z_d, sets[0].z_t, sets[0].x, seed=wl.seed, round_=0)
+    rnd.run()
+    torch.cuda.synchronize()
 
     if args.no_e2e:
         e2e = None
@@ -351,27 +448,29 @@ def run_gpu(args):
     peak, peak_kind = _peaks()
     achieved = scan_bytes / (scan_avg_ms / 1e3) / 1e9
     if rank == 0:
-        cpu = None
+        cpu = parity = None
         if ws == 1 and not args.no_cpu_baseline:
-            import numpy as np
-            nb = min(args.cpu_blocks, B)
-
-            def h(t):
-                t = t[:nb].cpu()
-                return t.view(torch.int16).numpy().view(np.uint16) if t.dtype == torch.bfloat16 else t.numpy()
-            host = {"z_d": h(sets[0].z_d), "z_t": h(sets[0].z_t), "x": sets[0].x[:nb].cpu().numpy()}
-            cpu = _cpu_baseline(wl, ells, ks, host, nb)
+            cpu, res = _cpu_baseline(wl, ells, ks, _host_block(sets[0], wl), min(args.cpu_blocks, B))
+            parity = _parity_sample(rnd, res, ells, ks)
+        roofline = {"bound": "hbm", "kernel": "scan_kernel (sdd_block_scan)", "achieved": achieved,
+                    "peak": peak, "unit": "GB/s", "frac": achieved / peak, "traffic": args.traffic,
+                    "peak_source": f"{peak_kind} hbm_gbs (burst copy; the kernel is timed in a run of "
+                                   f"{n_scan} back-to-back launches)",
+                    "bytes_per_launch": scan_bytes, "avg_launch_ms": scan_avg_ms, "launches_timed": n_scan}
+        if scan_avg_ms > ms_per_step:
+            # the dominant kernel cannot take longer than the round that contains it
+            roofline = {"bound": "hbm", "achieved": None, "peak": peak, "unit": "GB/s", "frac": None,
+                        "traffic": args.traffic, "invalid": f"scan {scan_avg_ms:.4f} ms > round {ms_per_step:.4f} ms"}
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if esz == 2 else "fp32", "data": "synthetic",
             "config": _config_json(wl, ells, ks, n_sets),
-            "achieved_gbs_step": scan_bytes / (total_ms / args.steps / 1e3) / 1e9,
-            "roofline": {"bound": "hbm", "kernel": "scan_kernel (sdd_block_scan)", "achieved": achieved,
-                         "peak": peak, "unit": "GB/s", "frac": achieved / peak, "traffic": args.traffic,
-                         "peak_source": f"{peak_kind} hbm_gbs", "bytes_per_launch": scan_bytes,
-                         "avg_launch_ms": scan_avg_ms},
+            "achieved_gbs_step": ws * scan_bytes / (ms_per_step / 1e3) / 1e9,
+            "frac_of_8tbs_step": ws * scan_bytes / (ms_per_step / 1e3) / 8e12,
+            "roofline": roofline,
             "cpu_baseline": cpu,
+            "parity_sample": parity,
             "e2e": e2e,
             "gpu_launches": 2 * args.steps,
             "clocks": clk.summary(),
@@ -712,6 +811,19 @@ def run_component_loop(args):
     return 0
 
 
+def _launch_ranks(n: int) -> int:
+    """`--gpus N` without a launcher around it: start N ranks of this same
+    command, one per GPU, through torch.distributed.run on 127.0.0.1 (each rank
+    reads RANK / LOCAL_RANK / WORLD_SIZE; rank 0 prints the line)."""
+    import socket
+    with socket.socket(socket.AF_INET, socket.SOCK_STREAM) as sk:
+        sk.bind(("127.0.0.1", 0))
+        port = sk.getsockname()[1]
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={n}",
+           "--master-addr=127.0.0.1", f"--master-port={port}", os.path.abspath(__file__)] + sys.argv[1:]
+    return subprocess.call(cmd)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -719,7 +831,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--workload", default="c3")
-    ap.add_argument("--cpu-blocks", type=int, default=8)
+    ap.add_argument("--cpu-blocks", type=int, default=8, help="blocks of the single-thread oracle sample")
+    ap.add_argument("--ref-threads", type=int, default=0, help="host threads of --impl reference (0: all cores)")
+    ap.add_argument("--scan-launches", type=int, default=60, help="back-to-back streaming launches for the roofline")
+    ap.add_argument("--prefill-us", type=float, default=200.0, help="device spin before the start event")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--sets", type=int, default=3, help="rotating input sets (3 x 316 MB exceeds L2)")
@@ -728,6 +843,8 @@ def main():
     ap.add_argument("--component", default=None, choices=["mlp", "loop", "features", "scorer", "diag"],
                     help="measure one other row of the path instead of the fused round")
     args = ap.parse_args()
+    if args.gpus > 1 and "WORLD_SIZE" not in os.environ:
+        return _launch_ranks(args.gpus)
     if args.component == "mlp":
         return run_component_mlp(args)
     if args.component == "loop":
