@@ -43,6 +43,7 @@ class RoundOut:
     tokens: torch.Tensor       # [B, gamma+1] committed tokens (-1 padded)
     n: torch.Tensor            # [B] committed count
     n_verified: int
+    score: torch.Tensor = None  # [B, gamma] the survival scorer's output
 
 
 @dataclass
@@ -135,7 +136,8 @@ class DecodeLoop:
                                       rows=rows, ws=self.ws, status=self.status)
         tokens, n_commit = sdd.commit(K, x, tok, n, out=self._commit)
         self.D_raw, self.D_mlp, self.D_per = D_raw[0], D_mlp[0], D_per[0]
-        return RoundOut(K_raw=K, K_mlp=K_mlp[0], K_per=K_per[0], L=L, tokens=tokens, n=n_commit, n_verified=n_rows)
+        return RoundOut(K_raw=K, K_mlp=K_mlp[0], K_per=K_per[0], L=L, tokens=tokens, n=n_commit, n_verified=n_rows,
+                        score=s)
 
 
 def run(rounds: int = 256, workload: str = "c5", warmup: int = 2, scorer: str = "deep", device="cuda") -> dict:

@@ -123,3 +123,20 @@ def compare_rule(tally: Tally, name, L_gpu, tok_gpu, oracle_list, blocks):
         ok = (int(L_gpu[b]) == L) and np.array_equal(tok_gpu[b], tok)
         tally.check(f"{name} block {b} (gpu L={int(L_gpu[b])} tok={tok_gpu[b][:L_gpu[b]+1].tolist()[-3:]} ; "
                     f"oracle L={L} tok={tok[:L+1].tolist()[-3:]})", ok, mg)
+
+
+def row_stats_threads(zd, tokens, threads=None):
+    """orc.row_stats over the leading (batch) axis split across host threads
+    (the oracle's C calls release the interpreter lock); same result as one
+    call over the whole array."""
+    import os
+    from concurrent.futures import ThreadPoolExecutor
+    B = zd.shape[0]
+    threads = max(1, min(B, threads or os.cpu_count() or 1))
+    cuts = np.linspace(0, B, threads + 1).astype(int)
+    parts = [(a, b) for a, b in zip(cuts[:-1], cuts[1:]) if b > a]
+    with ThreadPoolExecutor(max_workers=len(parts)) as ex:
+        res = list(ex.map(lambda ab: orc.row_stats(zd[ab[0]:ab[1]], tokens=tokens[ab[0]:ab[1]]), parts))
+    cat = lambda name: np.concatenate([getattr(r, name) for r in res], axis=0)   # noqa: E731
+    return orc.RowStats(m=cat("m"), lse=cat("lse"), q=cat("q"), logq=cat("logq"), maxprob=cat("maxprob"),
+                        entropy=cat("entropy"), argmax=cat("argmax"))

@@ -54,6 +54,23 @@ def _compare(wl, ells, ks, rnd, ob, blocks, greedy=False):
     return tally
 
 
+def test_tiny_full_round():
+    """The tiny workload exactly as stated: B = 1, gamma = 8, V = 32,000 fp32;
+    strict sampling plus the raw-confidence schedule at tau = 0.9, with the
+    committed tokens of the round."""
+    wl, ells, ks, blk, rnd, ob, blocks = _round("tiny")
+    assert (wl.B, wl.gamma, wl.V, wl.dtype) == (1, 8, 32_000, torch.float32) and wl.taus == (0.9,)
+    tally = _compare(wl, ells, ks, rnd, ob, blocks)
+    oK = ob.sched[(0.9, 0.9)][1]
+    L, tok, _ = ob.strict[0]
+    if oK[0] > 0:
+        assert int(rnd.commit_n[0]) == oK[0]
+    else:
+        assert int(rnd.commit_n[0]) == L + 1
+        np.testing.assert_array_equal(rnd.commit_tokens[0].cpu().numpy(), tok)
+    print("tiny", tally)
+
+
 def test_c2_full():
     wl, ells, ks, blk, rnd, ob, blocks = _round("c2")
     tally = _compare(wl, ells, ks, rnd, ob, blocks)

@@ -96,3 +96,78 @@ def test_loop_matches_oracle_replay(sdd, orc, B, gamma, V, hidden, rounds, score
                 np.testing.assert_array_equal(tok_dev[b], tokens)
                 assert n_dev[b] == L + 1
     assert seen_skip > 0 and seen_verify > 0     # both branches of the loop were exercised
+
+
+def test_loop_full_size_decode_workload(sdd, orc):
+    """The decode-loop workload at its stated size (B = 128, gamma = 32,
+    V = 151,936 bf16, hidden 3584, the deep scorer) over three rounds with D
+    carried (Sec. 4.1 loop): every block's K and D under raw confidence
+    against the oracle (rows within 1e-6 of a threshold are flagged and the
+    oracle continues from the device's D there), the strict verification of
+    at least eight verified blocks per round (L and committed tokens), the
+    periodic shadow schedule, and the deep scorer on 64 sampled positions per
+    round."""
+    from parity_util import row_stats_threads
+    wl = synth.WORKLOADS["c5"]
+    B, gamma, V = wl.B, wl.gamma, wl.V
+    loop = DecodeLoop(B, gamma, V, tau=0.9, tau_mlp=0.9, K_min=6, S_max=64, seed=wl.seed, period=4, scorer="deep")
+    D_raw = np.zeros(B, np.int32)
+    D_per = np.zeros(B, np.int32)
+    rng = np.random.default_rng(55)
+    flagged = verified_checked = 0
+    for r in range(3):
+        blk = synth.make_block(wl, device="cuda", round_=r)
+        h = synth.make_hidden(B * gamma, device="cuda", seed=wl.seed, round_=r)
+        out = loop.step(blk.z_d, blk.z_t, blk.x, h, round_=r)
+        torch.cuda.synchronize()
+        assert int(loop.status.item()) == 0
+        zd, x = _bits(blk.z_d), blk.x.cpu().numpy()
+        st = row_stats_threads(zd, x)
+        _, K_raw, D_next, mg = orc.schedule(st.q, orc.SIG_RAW, 0.9, 0.9, 6, 64, D_in=D_raw)
+        K_dev, D_dev = out.K_raw.cpu().numpy(), loop.D_raw.cpu().numpy()
+        sure = mg >= NEAR
+        flagged += int((~sure).sum())
+        np.testing.assert_array_equal(K_dev[sure], K_raw[sure])
+        np.testing.assert_array_equal(D_dev[sure], D_next[sure])
+        D_raw = D_dev.astype(np.int32)
+        _, K_per, D_per = orc.schedule_periodic(B, gamma, 4, 6, r, 6, 64, D_in=D_per)
+        np.testing.assert_array_equal(out.K_per.cpu().numpy(), K_per)
+        np.testing.assert_array_equal(loop.D_per.cpu().numpy(), D_per)
+        # strict verification of verified blocks (K = 0): the first, the last and random ones
+        ver = np.flatnonzero(K_dev == 0)
+        assert out.n_verified == ver.size
+        pick = sorted(set(ver[:2].tolist() + ver[-2:].tolist() +
+                          rng.choice(ver, size=min(6, ver.size), replace=False).tolist())) if ver.size else []
+        assert len(pick) >= min(8, ver.size)
+        zt = _bits(blk.z_t)
+        L_dev, tok_dev, n_dev = out.L.cpu().numpy(), out.tokens.cpu().numpy(), out.n.cpu().numpy()
+        for b in pick:
+            L, tokens, margin = orc.verify_strict(zt[b], zd[b], x[b], seed=wl.seed, b=b, round_=r)
+            if margin < NEAR:
+                flagged += 1
+                continue
+            assert L_dev[b] == L and n_dev[b] == L + 1
+            np.testing.assert_array_equal(tok_dev[b], tokens)
+            verified_checked += 1
+        for b in np.flatnonzero(K_dev > 0)[:8]:
+            want = np.full(gamma + 1, -1, np.int32)
+            want[:K_dev[b]] = x[b, :K_dev[b]]
+            np.testing.assert_array_equal(tok_dev[b], want)
+        # the deep scorer on sampled positions, its features from the oracle's statistics
+        rows = rng.choice(B * gamma, size=64, replace=False)
+        blk_idx, pos = rows // gamma, rows % gamma
+        margin_f, top5 = orc.row_features(zd[blk_idx, pos])
+        cols = {4: st.maxprob[blk_idx, pos], 5: np.log(st.maxprob[blk_idx, pos]), 6: st.entropy[blk_idx, pos],
+                7: -st.entropy[blk_idx, pos], 8: margin_f, 9: top5, 14: pos / gamma, 15: np.full(64, r / 256.0)}
+        f = np.zeros((64, MLP_HIDDEN), np.float32)
+        for c, v in cols.items():
+            f[:, c] = v
+        feat = _bits(torch.from_numpy(f).to(torch.bfloat16))
+        x_in = np.concatenate([_bits(h)[rows], feat], axis=-1)
+        W1, b1, W2, b2, W3, b3, w4, b4 = loop.deep
+        s = orc.scorer_deep(x_in, _bits(W1), b1.cpu().numpy(), _bits(W2), b2.cpu().numpy(), _bits(W3),
+                            b3.cpu().numpy(), _bits(w4), b4)
+        np.testing.assert_allclose(out.score.cpu().numpy().reshape(-1)[rows], s, rtol=0, atol=3e-4)
+        del blk, h
+    assert verified_checked >= 8
+    print(f"decode workload: flagged near-threshold decisions {flagged}, verified blocks compared {verified_checked}")
