@@ -318,6 +318,24 @@ SDD_API sdd_status_t sdd_commit(const int32_t *K, const int32_t *draft_tokens, c
                         int32_t *out_n, sdd_stream_t stream);
 
 /*
+ * sdd_test_wait_hooks -- failure-detection test hooks (the paper has no
+ * counterpart: they test the library's bounded device waits).  They apply to
+ * the streaming kernel of every call this process enqueues afterwards, from
+ * any thread, until changed:
+ *   polls      the number of polls after which a wait for a tile copy gives
+ *              up (each poll may suspend the warp briefly); 0 restores the
+ *              default of 2^24 polls (seconds).  Copies still in flight when a
+ *              warp gives up are always waited for with the default limit.
+ *   drop_copy  nonzero: the first warp of each launch never issues its first
+ *              tile copy, so its wait runs out -- the call returns normally,
+ *              its device status gets SDD_DEV_TIMEOUT, its results are
+ *              undefined, and the context, the workspace and later calls stay
+ *              usable.  0: normal operation.
+ * Returns SDD_OK.  Meant for tests; leave both at 0 in production.
+ */
+SDD_API sdd_status_t sdd_test_wait_hooks(uint32_t polls, int drop_copy);
+
+/*
  * sdd_uniforms -- the uniforms U(seed, j, b, round, purpose) that the sampling
  * rule of sdd_verify_strict draws (Philox4x32-10 map stated there), for n
  * counters given as device arrays j, b, purpose [n] (uint32) and round [n]

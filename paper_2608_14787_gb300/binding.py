@@ -106,6 +106,8 @@ def load(path: str | None = None):
     L.sdd_permutation_diagnostic.restype = I
     L.sdd_position_metrics.argtypes = [VP, VP, I, I, I, VP, VP, VP, VP, VP, VP]
     L.sdd_position_metrics.restype = I
+    L.sdd_test_wait_hooks.argtypes = [ctypes.c_uint32, I]
+    L.sdd_test_wait_hooks.restype = I
     for fn in ("sdd_block", "sdd_block_scan", "sdd_block_decide"):
         getattr(L, fn).argtypes = [ctypes.POINTER(BlockArgs), VP]
     for fn in ("sdd_workspace_size", "sdd_confidence", "sdd_confidence_features", "sdd_schedule_prefix",
@@ -486,6 +488,15 @@ def uniforms(seed, j, b, round_, purpose, stream=None):
     _check(load().sdd_uniforms(seed, _p(j), _p(b), _p(round_), _p(purpose), n, _p(u), _stream(stream)),
            "sdd_uniforms")
     return u
+
+
+def test_wait_hooks(polls: int = 0, drop_copy: bool = False):
+    """sdd_test_wait_hooks: the streaming kernel's ring-wait poll limit (0 =
+    default) and the dropped-first-copy hook, for later calls of this process."""
+    _check(load().sdd_test_wait_hooks(int(polls), 1 if drop_copy else 0), "sdd_test_wait_hooks")
+
+
+test_wait_hooks.__test__ = False   # a library call, not a test
 
 
 class BlockRound:

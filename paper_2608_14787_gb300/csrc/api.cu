@@ -551,6 +551,11 @@ sdd_status_t sdd_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, c
     return SDD_OK;
 }
 
+sdd_status_t sdd_test_wait_hooks(uint32_t polls, int drop_copy) {
+    set_scan_wait_hooks(polls, drop_copy);
+    return SDD_OK;
+}
+
 sdd_status_t sdd_scorer_features(const float *maxprob, const float *entropy, const float *margin,
                                  const float *top5, int B, int gamma, int64_t round, void *f, sdd_stream_t stream) {
     if (B < 0 || gamma < 1 || gamma > SDD_MAX_GAMMA)

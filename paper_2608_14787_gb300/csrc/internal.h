@@ -130,6 +130,8 @@ struct ScanParams {
     Partial *partials;       // [rows + W]
     FeatPartial *feat;       // [rows + W], or nullptr: no extended features
     int32_t *status;
+    uint32_t wait_polls;     // polls of a ring wait before the warp gives up (set at launch)
+    int32_t drop_copy;       // failure-detection test hook: warp 0 never issues its first copy
     DecideParams dec;
 };
 
@@ -148,6 +150,9 @@ struct ScheduleParams {
 
 // The streaming kernel (grid = warps / kWarpsPerCta CTAs).
 cudaError_t launch_scan(const ScanParams &p, int grid, cudaStream_t stream);
+// Failure-detection test hooks of the streaming kernel, read at each launch:
+// the ring waits' poll limit (0 = kWaitPolls) and the dropped first copy.
+void set_scan_wait_hooks(uint32_t polls, int drop_copy);
 // The decide kernel over (listed blocks, p.dec.nseg) CTAs, launched as a
 // programmatic dependent of the streaming kernel.
 cudaError_t launch_decide(const ScanParams &p, cudaStream_t stream);

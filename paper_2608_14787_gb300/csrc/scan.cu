@@ -22,6 +22,8 @@
 // The decide kernel (decide.cu) merges each row's partials and finalises the
 // rows; keeping that out of the streaming kernel keeps this kernel free of
 // register spills.
+#include <atomic>
+
 #include "internal.h"
 
 namespace sdd {
@@ -468,17 +470,24 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
     const uint64_t pol = l2_evict_first_policy();   // the logits are read once
     uint32_t pending = 0;  // slots with a copy in flight
     uint32_t phase = 0;    // parity bit per slot
+    bool drop = p.drop_copy != 0 && gw == 0;   // test hook: this warp's first copy is never issued
 
     auto issue = [&](int slot) {
         const int n = static_cast<int>(min(static_cast<int64_t>(min(kTileVec, p.RV - pc.k)), v1 - pc.v));
-        if (lane == 0) {
+        if (drop) {
+            // nothing will ever complete this slot's barrier: the consumer's
+            // bounded wait runs out (no copy is in flight for the drain)
+            drop = false;
+        } else {
+            if (lane == 0) {
             // the slot's previous contents were consumed into registers before the
             // warp reached this point (__syncwarp), so the copy may overwrite it
-            mbar_arrive_expect_tx(&bars[slot], static_cast<uint32_t>(n) * 16u);
-            bulk_g2s(ring + slot * kTileBytes, prow + static_cast<int64_t>(pc.k) * 16, static_cast<uint32_t>(n) * 16u,
-                     &bars[slot], pol);
+                mbar_arrive_expect_tx(&bars[slot], static_cast<uint32_t>(n) * 16u);
+                bulk_g2s(ring + slot * kTileBytes, prow + static_cast<int64_t>(pc.k) * 16,
+                         static_cast<uint32_t>(n) * 16u, &bars[slot], pol);
+            }
+            pending |= 1u << slot;
         }
-        pending |= 1u << slot;
         pc.v += n;
         pc.k += n;
         if (pc.k == p.RV && pc.v < v1) {
@@ -543,7 +552,8 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
             wrank = 0;
             in_piece = true;
         }
-        if (!mbar_wait_bounded(&bars[slot], (phase >> slot) & 1u, kWaitPolls)) {
+        // warp-uniform outcome: a phase that one lane saw complete is complete for all
+        if (!__any_sync(0xFFFFFFFFu, mbar_wait_bounded(&bars[slot], (phase >> slot) & 1u, p.wait_polls))) {
             timed_out = true;
             break;
         }
@@ -620,8 +630,9 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
         }
     }
     if (timed_out) {
-        status_or(p.status, SDD_DEV_TIMEOUT);
-        // let every copy still in flight land before the CTA's shared memory goes away
+        if (lane == 0) status_or(p.status, SDD_DEV_TIMEOUT);
+        // let every copy still in flight land before the CTA's shared memory
+        // goes away (the full limit, whatever the ring waits were given)
         for (int s = 0; s < kStages; ++s)
             if (pending & (1u << s)) (void)mbar_wait_bounded(&bars[s], (phase >> s) & 1u, kWaitPolls);
     }
@@ -648,11 +659,25 @@ cudaError_t scan_prepare_device() {
 
 // The launch overhead of the streaming grid overlaps the tail of the work
 // ahead of it in the stream (the kernel waits for that work to complete).
+namespace {
+std::atomic<uint32_t> g_wait_polls{0};
+std::atomic<int> g_drop_copy{0};
+}  // namespace
+
+void set_scan_wait_hooks(uint32_t polls, int drop_copy) {
+    g_wait_polls.store(polls, std::memory_order_relaxed);
+    g_drop_copy.store(drop_copy ? 1 : 0, std::memory_order_relaxed);
+}
+
 cudaError_t launch_scan(const ScanParams &p, int grid, cudaStream_t stream) {
     const bool bf = p.dtype == SDD_BF16, feat = p.feat != nullptr;
     void (*const k)(ScanParams) = feat ? (bf ? scan_kernel<SDD_BF16, true> : scan_kernel<SDD_F32, true>)
                                        : (bf ? scan_kernel<SDD_BF16, false> : scan_kernel<SDD_F32, false>);
-    return launch_dependent(k, dim3(grid), dim3(kThreads), kScanSmem, stream, p);
+    ScanParams q = p;
+    const uint32_t polls = g_wait_polls.load(std::memory_order_relaxed);
+    q.wait_polls = polls ? polls : kWaitPolls;
+    q.drop_copy = g_drop_copy.load(std::memory_order_relaxed);
+    return launch_dependent(k, dim3(grid), dim3(kThreads), kScanSmem, stream, q);
 }
 
 }  // namespace sdd
