@@ -252,14 +252,11 @@ def _cpu_baseline(wl, ells, ks, host, n_single):
     return base, res
 
 
-def _parity_sample(rnd, res, ells, ks):
-    """Compare one round's device outputs with the oracle's results for the
-    same blocks (decisions bit-exact; a decision whose oracle margin is within
-    1e-6 of its threshold is counted as flagged, not compared)."""
+def _parity_sample(got, res, ells, ks):
+    """Compare one round's device decisions (host copies) with the oracle's
+    results for the same blocks (bit-exact; a decision whose oracle margin is
+    within 1e-6 of its threshold is counted as flagged, not compared)."""
     import numpy as np
-    got = {"K": rnd.K.cpu().numpy(), "L": rnd.L_strict.cpu().numpy(), "tok": rnd.tokens_strict.cpu().numpy(),
-           "Ll": rnd.L_lenient.cpu().numpy(), "tl": rnd.tokens_lenient.cpu().numpy(),
-           "Lk": rnd.L_topk.cpu().numpy(), "tk": rnd.tokens_topk.cpu().numpy()}
     compared = flagged = mismatched = 0
 
     def check(ok, margin):
@@ -434,10 +431,14 @@ def run_gpu(args):
     torch.cuda.synchronize()
     scan_avg_ms = e0.elapsed_time(e1) / n_scan
 
-    # ---- one untimed round on input set 0 for the oracle parity sample ----
+    # ---- one untimed round on input set 0 for the oracle parity sample (its
+    # decisions are copied out before the end-to-end leg reuses the round) ----
     rnd.set_inputs(sets[0].z_d, sets[0].z_t, sets[0].x, seed=wl.seed, round_=0)
     rnd.run()
     torch.cuda.synchronize()
+    decisions = {"K": rnd.K.cpu().numpy(), "L": rnd.L_strict.cpu().numpy(), "tok": rnd.tokens_strict.cpu().numpy(),
+                 "Ll": rnd.L_lenient.cpu().numpy(), "tl": rnd.tokens_lenient.cpu().numpy(),
+                 "Lk": rnd.L_topk.cpu().numpy(), "tk": rnd.tokens_topk.cpu().numpy()}
 
     if args.no_e2e:
         e2e = None
@@ -451,7 +452,7 @@ def run_gpu(args):
         cpu = parity = None
         if ws == 1 and not args.no_cpu_baseline:
             cpu, res = _cpu_baseline(wl, ells, ks, _host_block(sets[0], wl), min(args.cpu_blocks, B))
-            parity = _parity_sample(rnd, res, ells, ks)
+            parity = _parity_sample(decisions, res, ells, ks)
         roofline = {"bound": "hbm", "kernel": "scan_kernel (sdd_block_scan)", "achieved": achieved,
                     "peak": peak, "unit": "GB/s", "frac": achieved / peak, "traffic": args.traffic,
                     "peak_source": f"{peak_kind} hbm_gbs (burst copy; the kernel is timed in a run of "

@@ -528,6 +528,93 @@ SDD_API sdd_status_t sdd_block(const sdd_block_args *args, sdd_stream_t stream);
 SDD_API sdd_status_t sdd_block_scan(const sdd_block_args *args, sdd_stream_t stream);
 SDD_API sdd_status_t sdd_block_decide(const sdd_block_args *args, sdd_stream_t stream);
 
+/*
+ * Vocabulary-sharded round (a tensor-parallel LM head).  The paper runs its
+ * verifier on one GPU and reads its logits in fp32 (App. A.8); when the
+ * drafter's and verifier's logits are instead split by vocabulary over S
+ * ranks -- rank s holding the contiguous slice [v0_s, v1_s) of every row,
+ * slices in ascending order covering [0, V) -- the same round of sdd_block
+ * runs as follows, with results identical to sdd_block's on the whole rows:
+ *
+ *   1. every rank: sdd_shard_partials on its slice -> one record per row;
+ *   2. exchange: all-gather the records, [S][rows] in slice order;
+ *   3. every rank: sdd_shard_decide -> all of sdd_block's outputs (identical
+ *      on every rank), except, under strict sampling, the token drawn at the
+ *      first rejection or the bonus row, left -1; plus this slice's masses
+ *      of that draw row, [B][2] floats;
+ *   4. (strict sampling) exchange: all-gather the masses, [S][B][2];
+ *   5. (strict sampling) every rank: sdd_shard_draw -> the rank whose slice
+ *      holds the draw writes the token into tokens_strict (and commit_tokens
+ *      when the block is committed); the others write nothing;
+ *   6. (strict sampling) exchange: element-wise MAX all-reduce of
+ *      tokens_strict and commit_tokens (the missing entries are -1).
+ *
+ * A record: the slice's online-softmax state of the row with global indices,
+ * the drafted token's logit when the token lies in the slice, and, for target
+ * rows when the top-k rule runs, the slice's largest logits (value
+ * descending, index ascending) -- the kcap largest of the whole row lie among
+ * them, so the merged rank of the drafted token is exact up to kcap.  Records
+ * are plain bytes: no pointers, the same on every rank.
+ */
+#define SDD_SHARD_KMAX 16
+
+typedef struct sdd_shard_partial {
+    float m;                      /* largest logit of the slice (floored at -2^23) */
+    float r;                      /* integer reference of the sums, in log2 units */
+    float t2;                     /* entropy accumulator relative to r (drafter rows) */
+    float sh, sl;                 /* sum of 2^(z log2(e) - r) over the slice, as hi + lo */
+    int32_t amax;                 /* global index of the slice's first largest logit */
+    float g;                      /* the drafted token's logit if it lies in the slice */
+    int32_t info;                 /* bit 0: token in the slice; bit 1: token outside [0, V);
+                                     bits 8..15: number of candidates */
+    float cz[SDD_SHARD_KMAX];     /* target rows: the slice's largest logits */
+    int32_t cv[SDD_SHARD_KMAX];   /* their global indices */
+} sdd_shard_partial;              /* 160 bytes */
+
+/*
+ * sdd_shard_workspace_size -- bytes of device scratch that sdd_shard_decide
+ * leaves for sdd_shard_draw (per block: the accepted length and the draw
+ * row's log-normalisers): B * 32.
+ */
+SDD_API sdd_status_t sdd_shard_workspace_size(int B, size_t *bytes);
+
+/*
+ * sdd_shard_partials -- step 1.  args as for sdd_block except: draft_logits
+ * and target_logits hold this rank's slice, [B, gamma, row_stride] and
+ * [B, gamma+1, row_stride] with columns 0..(v1-v0-1) = vocabulary entries
+ * v0..v1-1 (v1 - v0 <= row_stride); V is the whole vocabulary; draft_tokens
+ * are global indices; the top-k values (topk, n_k <= SDD_MAX_GRID) fix how
+ * many candidates a record keeps (the largest k, at most SDD_SHARD_KMAX).
+ * Only these fields and status are read.  out: [B*gamma + B*(gamma+1)]
+ * records, drafter rows (b, j) at b*gamma + j, then target rows (b, j) at
+ * B*gamma + b*(gamma+1) + j (device memory).
+ */
+SDD_API sdd_status_t sdd_shard_partials(const sdd_block_args *args, int v0, int v1, sdd_shard_partial *out,
+                                        sdd_stream_t stream);
+
+/*
+ * sdd_shard_decide -- step 3.  args as for sdd_block (outputs included)
+ * except: logits and V as for sdd_shard_partials, workspace = at least
+ * sdd_shard_workspace_size(B) bytes.  all: [n_shards][rows] records of step
+ * 2 (slice order); v0, v1 this rank's slice.  mass: [B][2] floats (device):
+ * this slice's mass of each block's draw row (the residual max(0, p_t - p_d)
+ * at the first rejection, or p_t of the bonus row; then p_t of that row),
+ * written under strict sampling only.  n_shards <= 64.
+ */
+SDD_API sdd_status_t sdd_shard_decide(const sdd_block_args *args, int v0, int v1, int n_shards,
+                                      const sdd_shard_partial *all, float *mass, sdd_stream_t stream);
+
+/*
+ * sdd_shard_draw -- step 5 (strict sampling only).  args, v0, v1, n_shards
+ * as for sdd_shard_decide, the same workspace after it; shard: this rank's
+ * index; mass_all: [n_shards][B][2] floats of step 4.  Locates, in slice order,
+ * the slice holding u R of the inverse-CDF draw (R: the row's total mass) and,
+ * on that slice's rank, the token, written at position L of tokens_strict and,
+ * when the block is committed, of commit_tokens.
+ */
+SDD_API sdd_status_t sdd_shard_draw(const sdd_block_args *args, int v0, int v1, int n_shards, int shard,
+                                    const float *mass_all, sdd_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

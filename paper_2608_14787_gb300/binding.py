@@ -108,6 +108,14 @@ def load(path: str | None = None):
     L.sdd_position_metrics.restype = I
     L.sdd_test_wait_hooks.argtypes = [ctypes.c_uint32, I]
     L.sdd_test_wait_hooks.restype = I
+    L.sdd_shard_workspace_size.argtypes = [I, ctypes.POINTER(ctypes.c_size_t)]
+    L.sdd_shard_workspace_size.restype = I
+    L.sdd_shard_partials.argtypes = [ctypes.POINTER(BlockArgs), I, I, VP, VP]
+    L.sdd_shard_partials.restype = I
+    L.sdd_shard_decide.argtypes = [ctypes.POINTER(BlockArgs), I, I, I, VP, VP, VP]
+    L.sdd_shard_decide.restype = I
+    L.sdd_shard_draw.argtypes = [ctypes.POINTER(BlockArgs), I, I, I, I, VP, VP]
+    L.sdd_shard_draw.restype = I
     for fn in ("sdd_block", "sdd_block_scan", "sdd_block_decide"):
         getattr(L, fn).argtypes = [ctypes.POINTER(BlockArgs), VP]
     for fn in ("sdd_workspace_size", "sdd_confidence", "sdd_confidence_features", "sdd_schedule_prefix",

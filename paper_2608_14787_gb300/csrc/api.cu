@@ -178,6 +178,13 @@ sdd_status_t run_decide(const ScanParams &p, cudaStream_t stream) {
     return SDD_OK;
 }
 
+// The decide kernel of a vocabulary-sharded round (no streaming pass before it).
+sdd_status_t run_decide_shard(const ScanParams &p, cudaStream_t stream) {
+    cudaError_t e = launch_decide(p, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "decide launch");
+    return SDD_OK;
+}
+
 // Block decisions and, for the sampling rule, the draw geometry: each of the
 // nb blocks' draw rows is cut into nseg segments of whole kDecThreads-vector
 // chunks, as many as keep nb * nseg CTAs resident in one wave (at least two
@@ -779,6 +786,223 @@ static sdd_status_t block_params(const sdd_block_args *a, ScanParams &p, bool *e
     d.agreement = reinterpret_cast<long long *>(a->agreement);
     p.dec = d;
     finish_params(p, w);
+    return SDD_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Vocabulary-sharded round
+// ---------------------------------------------------------------------------
+static sdd_status_t shard_check(const sdd_block_args *a, int v0, int v1) {
+    if (!a) return fail(SDD_ERR_INVALID_ARGUMENT, "args is NULL");
+    const sdd_dtype_t dt = static_cast<sdd_dtype_t>(a->dtype);
+    if (dt != SDD_F32 && dt != SDD_BF16) return fail(SDD_ERR_INVALID_ARGUMENT, "dtype %d unknown", a->dtype);
+    if (a->B < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "B = %d < 0", a->B);
+    if (a->gamma < 1 || a->gamma > SDD_MAX_GAMMA)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "gamma = %d outside [1, %d]", a->gamma, SDD_MAX_GAMMA);
+    if (a->V < 1) return fail(SDD_ERR_INVALID_ARGUMENT, "V = %d < 1", a->V);
+    if (v0 < 0 || v1 <= v0 || v1 > a->V)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "slice [%d, %d) is empty or outside [0, V = %d)", v0, v1, a->V);
+    const int w = v1 - v0;
+    if (a->row_stride < w)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "row_stride %lld < slice width %d", (long long)a->row_stride, w);
+    if ((a->row_stride * esize(dt)) % 16 != 0)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "row_stride * element size must be a multiple of 16 bytes");
+    if (a->row_stride * esize(dt) > (int64_t(1) << 31))
+        return fail(SDD_ERR_INVALID_ARGUMENT, "rows longer than 2 GiB are not supported");
+    if (a->B == 0) return SDD_OK;
+    SDD_TRY(check_ptr16(a->draft_logits, "draft_logits"));
+    SDD_TRY(check_ptr16(a->target_logits, "target_logits"));
+    if (!a->draft_tokens) return fail(SDD_ERR_INVALID_ARGUMENT, "draft_tokens is NULL");
+    return SDD_OK;
+}
+
+static sdd_status_t shard_kcap(const sdd_block_args *a, int &kcap) {
+    DecideParams d;
+    std::memset(&d, 0, sizeof d);
+    int kc = 1;
+    SDD_TRY(set_topk(d, a->topk, a->n_k, kc));
+    if (a->n_k > 0 && kc > SDD_SHARD_KMAX)
+        return fail(SDD_ERR_UNSUPPORTED, "top-k with k = %d: the sharded round keeps at most %d candidates", kc,
+                    SDD_SHARD_KMAX);
+    kcap = (a->n_k > 0) ? kc : 0;
+    return SDD_OK;
+}
+
+sdd_status_t sdd_shard_workspace_size(int B, size_t *bytes) {
+    if (!bytes) return fail(SDD_ERR_INVALID_ARGUMENT, "bytes is NULL");
+    if (B < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "B = %d < 0", B);
+    *bytes = static_cast<size_t>(B) * sizeof(ShardDraw);
+    return SDD_OK;
+}
+
+static void shard_geometry(ShardParams &sp, const sdd_block_args *a, int v0, int v1) {
+    std::memset(&sp, 0, sizeof sp);
+    const sdd_dtype_t dt = static_cast<sdd_dtype_t>(a->dtype);
+    sp.zd = static_cast<const char *>(a->draft_logits);
+    sp.zt = static_cast<const char *>(a->target_logits);
+    sp.stride_bytes = a->row_stride * esize(dt);
+    sp.dtype = dt;
+    sp.B = a->B;
+    sp.gamma = a->gamma;
+    sp.Vs = v1 - v0;
+    sp.RVs = static_cast<int32_t>((static_cast<int64_t>(sp.Vs) * esize(dt) + 15) / 16);
+    sp.v0 = v0;
+    sp.V = a->V;
+    sp.tokens = a->draft_tokens;
+    sp.status = a->status;
+}
+
+sdd_status_t sdd_shard_partials(const sdd_block_args *a, int v0, int v1, sdd_shard_partial *out,
+                                sdd_stream_t stream) {
+    SDD_TRY(shard_check(a, v0, v1));
+    int kcap = 0;
+    SDD_TRY(shard_kcap(a, kcap));
+    if (a->B == 0) return SDD_OK;
+    if (!out) return fail(SDD_ERR_INVALID_ARGUMENT, "out is NULL");
+    ShardParams sp;
+    shard_geometry(sp, a, v0, v1);
+    sp.kcap = kcap;
+    sp.out = out;
+    cudaError_t e = launch_shard_partials(sp, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "shard partials launch");
+    return SDD_OK;
+}
+
+static sdd_status_t shard_state_ws(const sdd_block_args *a) {
+    size_t need = 0;
+    SDD_TRY(sdd_shard_workspace_size(a->B, &need));
+    if (!a->workspace) return fail(SDD_ERR_WORKSPACE, "workspace is NULL");
+    if (reinterpret_cast<uintptr_t>(a->workspace) % 16 != 0)
+        return fail(SDD_ERR_WORKSPACE, "workspace is not 16-byte aligned");
+    if (a->workspace_bytes < need)
+        return fail(SDD_ERR_WORKSPACE, "workspace has %zu bytes, %zu needed", a->workspace_bytes, need);
+    return SDD_OK;
+}
+
+sdd_status_t sdd_shard_decide(const sdd_block_args *a, int v0, int v1, int n_shards, const sdd_shard_partial *all,
+                              float *mass, sdd_stream_t stream) {
+    SDD_TRY(shard_check(a, v0, v1));
+    if (n_shards < 1 || n_shards > 64) return fail(SDD_ERR_INVALID_ARGUMENT, "n_shards = %d outside [1, 64]", n_shards);
+    int kcap = 0;
+    SDD_TRY(shard_kcap(a, kcap));
+    const sdd_dtype_t dt = static_cast<sdd_dtype_t>(a->dtype);
+    DecideParams d;
+    std::memset(&d, 0, sizeof d);
+    if (a->signal == SDD_SIG_PERIODIC) {
+        SDD_TRY(set_periods(a->period, a->n_tau, a->K_skip, d.period));
+        d.K_skip = a->K_skip;
+    } else {
+        SDD_TRY(set_thresholds(a->signal, a->eta_b, a->eta_c, a->n_tau, d.eta_loc, d.log_eta_c, d.tau_off));
+    }
+    SDD_TRY(set_ell(d, a->ell, a->n_ell));
+    int kc = 1;
+    SDD_TRY(set_topk(d, a->topk, a->n_k, kc));
+    if (a->B == 0) return SDD_OK;
+    if (!all) return fail(SDD_ERR_INVALID_ARGUMENT, "all is NULL");
+    const bool sampling = !a->greedy;
+    if (sampling && !mass) return fail(SDD_ERR_INVALID_ARGUMENT, "mass is NULL (strict sampling)");
+    SDD_TRY(shard_state_ws(a));
+    ScanParams p;
+    std::memset(&p, 0, sizeof p);
+    p.dtype = dt;
+    p.V = v1 - v0;
+    p.RV = static_cast<int32_t>((static_cast<int64_t>(p.V) * esize(dt) + 15) / 16);
+    p.gamma = a->gamma;
+    p.kcap = std::max(1, kcap);
+    p.B = a->B;
+    p.tokens = a->draft_tokens;
+    p.status = a->status;
+    p.n_groups = 2;
+    ScanGroup &D = p.grp[0];
+    D.base = static_cast<const char *>(a->draft_logits);
+    D.stride_bytes = a->row_stride * esize(dt);
+    D.npos = a->gamma;
+    D.kind = 0;
+    D.nb = a->B;
+    D.q = a->q;
+    D.logq = a->logq;
+    D.maxprob = a->maxprob;
+    D.lse = a->lse;
+    D.entropy = a->entropy;
+    D.argmax = a->argmax;
+    ScanGroup &T = p.grp[1];
+    T.base = static_cast<const char *>(a->target_logits);
+    T.stride_bytes = a->row_stride * esize(dt);
+    T.npos = a->gamma + 1;
+    T.kind = 1;
+    T.nb = a->B;
+    p.rows0 = static_cast<int64_t>(a->B) * a->gamma;
+    p.rows = static_cast<int64_t>(a->B) * (2 * a->gamma + 1);
+    p.shard = all;
+    p.n_shards = n_shards;
+    p.shard_v0 = v0;
+    p.shard_rows = p.rows;
+    d.enabled = 1;
+    d.B = a->B;
+    d.gamma = a->gamma;
+    d.V = p.V;
+    d.stride_bytes = a->row_stride * esize(dt);
+    d.tokens = a->draft_tokens;
+    d.nseg = 1;
+    d.seg_vec = p.RV;
+    d.zt = static_cast<const char *>(a->target_logits);
+    d.zd = static_cast<const char *>(a->draft_logits);
+    d.do_strict = 1;
+    d.greedy = a->greedy ? 1 : 0;
+    d.seed = a->seed;
+    d.round = a->round;
+    d.L_strict = a->L_strict;
+    d.tok_strict = a->tokens_strict;
+    d.n_strict = a->n_strict;
+    d.L_len = a->L_lenient;
+    d.tok_len = a->tokens_lenient;
+    d.n_len = a->n_lenient;
+    d.L_topk = a->L_topk;
+    d.tok_topk = a->tokens_topk;
+    d.n_topk = a->n_topk;
+    d.do_sched = 1;
+    d.signal = a->signal;
+    d.n_tau = a->n_tau;
+    d.K_min = a->K_min;
+    d.S_max = a->S_max;
+    d.guard = a->guard;
+    d.force_strict = a->force_strict;
+    d.D_in = a->D_in;
+    d.K_hat = a->K_hat;
+    d.K = a->K;
+    d.D_out = a->D_out;
+    d.commit_tokens = a->commit_tokens;
+    d.commit_n = a->commit_n;
+    d.agreement = reinterpret_cast<long long *>(a->agreement);
+    d.shard_mass = mass;
+    d.shard_state = static_cast<ShardDraw *>(a->workspace);
+    p.dec = d;
+    DevInfo di;
+    SDD_TRY(device_info(di));   // the kernels' attributes are set on this device
+    return run_decide_shard(p, reinterpret_cast<cudaStream_t>(stream));
+}
+
+sdd_status_t sdd_shard_draw(const sdd_block_args *a, int v0, int v1, int n_shards, int shard, const float *mass_all,
+                            sdd_stream_t stream) {
+    SDD_TRY(shard_check(a, v0, v1));
+    if (n_shards < 1 || n_shards > 64) return fail(SDD_ERR_INVALID_ARGUMENT, "n_shards = %d outside [1, 64]", n_shards);
+    if (shard < 0 || shard >= n_shards)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "shard = %d outside [0, %d)", shard, n_shards);
+    if (a->B == 0 || a->greedy) return SDD_OK;   // only strict sampling draws
+    if (!mass_all) return fail(SDD_ERR_INVALID_ARGUMENT, "mass_all is NULL");
+    SDD_TRY(shard_state_ws(a));
+    ShardParams sp;
+    shard_geometry(sp, a, v0, v1);
+    sp.n_shards = n_shards;
+    sp.shard = shard;
+    sp.mass_all = mass_all;
+    sp.state = static_cast<const ShardDraw *>(a->workspace);
+    sp.seed = a->seed;
+    sp.round = a->round;
+    sp.tok_strict = a->tokens_strict;
+    sp.commit_tokens = a->commit_tokens;
+    cudaError_t e = launch_shard_draw(sp, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "shard draw launch");
     return SDD_OK;
 }
 

@@ -45,7 +45,9 @@ __device__ __forceinline__ double pow2d_int(float k) {
 // Partial softmax state of one warp's piece of one row.  Sums are taken
 // relative to an integer reference r in log2 units:
 //   s = sum 2^(z log2(e) - r)  (kept as an unevaluated fp32 pair sh + sl),
-//   t2 = sum 2^(z log2(e) - r) (z log2(e) - r).
+//   t2 = sum 2^(z log2(e) - r) (z - m) log2(e), against the piece's maximum m
+//   (each term <= 0; the maximum's own term is 0, so on a peaked row t2 stays
+//   small and the entropy ln S' - ln 2 t2 / S involves no cancellation).
 struct __align__(32) Partial {
     float m;        // max of the clamped logits of the piece
     float r;        // integer reference (log2 units), >= m log2(e) up to rounding
@@ -412,8 +414,9 @@ __device__ __forceinline__ SoftState soft_merge(const SoftState &a, const SoftSt
     o.r = fmaxf(a.r, b.r);
     const float ka = a.r - o.r, kb = b.r - o.r;  // integers <= 0
     const float pa = pow2f_int(ka), pb = pow2f_int(kb);
-    // t2 relative to the new reference: 2^k (t2 + k s)
-    o.t2 = pa * fmaf(ka, a.sh + a.sl, a.t2) + pb * fmaf(kb, b.sh + b.sl, b.t2);
+    // t2 against the merged maximum, relative to the new reference:
+    // 2^k (t2 + (m - m') log2(e) s)
+    o.t2 = pa * fmaf((a.m - o.m) * kLog2e, a.sh + a.sl, a.t2) + pb * fmaf((b.m - o.m) * kLog2e, b.sh + b.sl, b.t2);
     float h, e;
     two_sum(a.sh * pa, b.sh * pb, h, e);
     fast_two_sum(h, fmaf(a.sl, pa, fmaf(b.sl, pb, e)), o.sh, o.sl);

@@ -321,6 +321,56 @@ __device__ int cta_find(const DrawCtx &c, int v0, int v1, int vpt, int V, df rem
     return *s_tok;
 }
 
+// Vocabulary-sharded draw: the weight sum of thread tid's run of a draw row of
+// RV vectors cut into one run of ceil(RV / kDecThreads) vectors per thread --
+// the same runs in the decide kernel's slice mass and in the draw, so that
+// both see the same sums bit for bit.
+template <int DT>
+__device__ __forceinline__ float slice_thread_sum(const DrawCtx &c, int RV, int V) {
+    const int vpt = (RV + kDecThreads - 1) / kDecThreads;
+    const int vb = min(RV, static_cast<int>(threadIdx.x) * vpt), ve = min(RV, vb + vpt);
+    return run_sum<DT>(c, vb, ve, V);
+}
+
+// Inverse CDF over a whole draw row of RV vectors by one CTA (the runs of
+// slice_thread_sum): the first entry at which the running sum exceeds rem, or
+// -- when rounding leaves none, or rem is infinite -- the row's last entry of
+// positive weight; -1 if the row has no weight.  Identical in every thread.
+template <int DT>
+__device__ int slice_find(const DrawCtx &c, int RV, int V, df rem, float *s_warp, int *s_thr, int *s_last,
+                          int *s_tok) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int vpt = (RV + kDecThreads - 1) / kDecThreads;
+    const int vb = min(RV, static_cast<int>(threadIdx.x) * vpt), ve = min(RV, vb + vpt);
+    const float ts = run_sum<DT>(c, vb, ve, V);
+    float tot;
+    const float incl = cta_incl_scan(ts, s_warp, &tot);
+    if (threadIdx.x == 0) {
+        *s_thr = INT32_MAX;
+        *s_last = -1;
+        *s_tok = -1;
+    }
+    __syncthreads();
+    const unsigned bal = __ballot_sync(0xFFFFFFFFu, (ve > vb) && !df_ge(rem, df{incl, 0.f}));
+    if (lane == 0 && bal) atomicMin(s_thr, warp * 32 + __ffs(bal) - 1);
+    const unsigned pos = __ballot_sync(0xFFFFFFFFu, ts > 0.f);
+    if (lane == 0 && pos) atomicMax(s_last, warp * 32 + 31 - __clz(pos));
+    __syncthreads();
+    int thr = *s_thr;
+    df r2 = df_sub(rem, df{incl - ts, 0.f});
+    if (thr == INT32_MAX) {
+        thr = *s_last;
+        r2 = df{__int_as_float(0x7F800000), 0.f};
+    }
+    if (static_cast<int>(threadIdx.x) == thr) {
+        int lp = -1;
+        const int pick = run_find<DT>(c, vb, ve, V, r2, lp);
+        *s_tok = (pick >= 0) ? pick : lp;
+    }
+    __syncthreads();
+    return *s_tok;
+}
+
 // Skip schedule of threshold pair t for a block (Sec. 4.1), by one warp, from
 // the drafter facts: prefix sums of ln q as double-floats, then sched_step
 // chunk by chunk and sched_final.
@@ -373,6 +423,8 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
         else
             gt = gi;
     }
+    const PartView pv = part_view(p);
+    if (i >= pv.nb) return;   // (a device block count below the grid's)
     const int32_t *bidx = p.grp[0].bidx;
     const int b = bidx ? __ldg(bidx + i) : i;
     if (b < 0 || b >= p.B) {
@@ -408,14 +460,17 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                 SoftState acc;
                 float g;
                 bool bad;
-                const int64_t r = (gd ? p.rows0 : 0) + static_cast<int64_t>(i) * G.npos + j;
-                if (FEAT && leader) {
+                const int64_t r = (gd ? pv.rows0 : 0) + static_cast<int64_t>(i) * G.npos + j;
+                if (p.shard != nullptr) {
+                    merge_row_shards(p, r, -1, false, acc, g, bad);
+                    f = row_final(p, G, j, b, acc, g, bad, leader);
+                } else if (FEAT && leader) {
                     float top[5];
-                    merge_row_t<true>(p, r, acc, g, bad, top);
+                    merge_row_t<true>(p, pv, r, acc, g, bad, top);
                     f = row_final(p, G, j, b, acc, g, bad, leader);
                     feat_final(G, static_cast<int64_t>(b) * p.gamma + j, top, f.lse);
                 } else {
-                    merge_row(p, r, acc, g, bad);
+                    merge_row(p, pv, r, acc, g, bad);
                     f = row_final(p, G, j, b, acc, g, bad, leader);
                 }
             } else {
@@ -434,7 +489,11 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
             SoftState acc;
             float g;
             bool bad;
-            merge_row(p, (gt ? p.rows0 : 0) + static_cast<int64_t>(i) * G.npos + j, acc, g, bad);
+            const int64_t r = (gt ? pv.rows0 : 0) + static_cast<int64_t>(i) * G.npos + j;
+            if (p.shard != nullptr)
+                merge_row_shards(p, r, (j < gamma) ? __ldg(d.tokens + ob + j) : -1, j < gamma, acc, g, bad);
+            else
+                merge_row(p, pv, r, acc, g, bad);
             put_target(F, j, row_final(p, G, j, b, acc, g, bad, leader));
         }
     }
@@ -467,6 +526,49 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
         }
         __syncthreads();
 
+        if (p.shard != nullptr) {
+            // ---- vocabulary-sharded (one CTA per block): this slice's masses
+            // of the draw row -- the residual (or bonus) weights, then p_t --
+            // for the exchange between ranks; shard_draw_kernel then draws ----
+            const int L = s_L[0];
+            const char *zt_row = d.zt + (bo + L) * d.stride_bytes;
+            const char *zd_row = (L < gamma) ? d.zd + (ob + L) * d.stride_bytes : nullptr;
+            const DrawCtx c = draw_ctx(zt_row, zd_row, df{F.t_lh[L], F.t_ll[L]},
+                                       (L < gamma) ? df{F.d_lh[L], F.d_ll[L]} : df{0.f, 0.f});
+            float tot_r, tot_p;
+            (void)cta_incl_scan(slice_thread_sum<DT>(c, p.RV, p.V), s_warp, &tot_r);
+            if (L < gamma) {
+                DrawCtx ct = c;
+                ct.zd_row = nullptr;
+                (void)cta_incl_scan(slice_thread_sum<DT>(ct, p.RV, p.V), s_warp, &tot_p);
+            } else {
+                tot_p = tot_r;
+            }
+            const bool commit = sched && s_K0 == 0;
+            if (tid == 0) {
+                d.shard_mass[2 * b] = tot_r;
+                d.shard_mass[2 * b + 1] = tot_p;
+                ShardDraw sd;
+                sd.L = L;
+                sd.commit = commit ? 1 : 0;
+                sd.t_lh = F.t_lh[L];
+                sd.t_ll = F.t_ll[L];
+                sd.d_lh = (L < gamma) ? F.d_lh[L] : 0.f;
+                sd.d_ll = (L < gamma) ? F.d_ll[L] : 0.f;
+                sd.pad[0] = sd.pad[1] = 0;
+                d.shard_state[b] = sd;
+            }
+            if (warp == 0) {
+                // the drawn token's place stays -1 until the draw
+                if (lane == 0) {
+                    if (d.L_strict) d.L_strict[b] = L;
+                    if (d.n_strict) d.n_strict[b] = L + 1;
+                    if (commit && d.commit_n) d.commit_n[b] = L + 1;
+                }
+                if (d.tok_strict) write_tokens(lane, gamma, d.tok_strict + bo, F.x, L, -1);
+                if (commit && d.commit_tokens) write_tokens(lane, gamma, d.commit_tokens + bo, F.x, L, -1);
+            }
+        } else {
         // ---- phase 3 (every CTA): its segment of the draw row at position L
         // (the residual row, or the bonus row when every position passed) ----
         const int L = s_L[0];
@@ -615,6 +717,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                 }
             }
         }
+        }
         if (!leader) return;
         __syncthreads();
     }
@@ -679,6 +782,93 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
             if (lane == 0 && d.commit_n) d.commit_n[b] = (K0 > 0) ? K0 : s_L[0] + 1;
             if (d.commit_tokens) write_tokens(lane, gamma, d.commit_tokens + bo, F.x, Lc, corr);
         }
+    }
+}
+
+// Vocabulary-sharded draw, one CTA per block, after every slice's masses of
+// the block's draw row have been exchanged (Sec. 3.1's resampling rule: the
+// inverse CDF in ascending vocabulary order).  Warp 0 takes double-float
+// prefix sums of the slices' masses in slice order and locates u R exactly
+// as the one-GPU draw locates a segment (no residual mass -> p_t of the same
+// row; rounding past the last slice -> the last slice of positive mass, its
+// last positive entry).  Only the rank whose slice holds the draw goes on:
+// it finds the entry in its slice and writes the token at position L.
+constexpr int kMaxShards = 64;
+
+template <int DT>
+__global__ void __launch_bounds__(kDecThreads) shard_draw_kernel(const __grid_constant__ ShardParams sp) {
+    constexpr int NW = kDecThreads / 32;
+    const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int gamma = sp.gamma, S = sp.n_shards;
+    __shared__ float s_warp[2 * NW];
+    __shared__ df s_cum[kMaxShards];
+    __shared__ int s_sel, s_col, s_thr, s_last, s_tok;
+    __shared__ df s_rem;
+    const ShardDraw st = sp.state[b];
+    const int L = st.L;
+    if (warp == 0) {
+        const uint32_t jj = (L < gamma) ? static_cast<uint32_t>(L + 1) : static_cast<uint32_t>(gamma + 1);
+        const float u = philox_uniform(sp.seed, jj, static_cast<uint32_t>(b), sp.round,
+                                       (L < gamma) ? kPurposeResid : kPurposeBonus);
+        int col = 0, last = -1;
+        df R = df{0.f, 0.f};
+        for (int pass = 0; pass < 2; ++pass) {
+            col = pass;
+            df carry = df{0.f, 0.f};
+            last = -1;
+            for (int s0 = 0; s0 < S; s0 += 32) {
+                const int sg = s0 + lane;
+                const float t = (sg < S) ? sp.mass_all[(static_cast<int64_t>(sg) * sp.B + b) * 2 + col] : 0.f;
+                const df cum = df_add(carry, warp_prefix_df(df{t, 0.f}, lane));
+                if (sg < S) s_cum[sg] = cum;
+                if (t > 0.f) last = sg;
+                carry.hi = __shfl_sync(0xFFFFFFFFu, cum.hi, 31);
+                carry.lo = __shfl_sync(0xFFFFFFFFu, cum.lo, 31);
+            }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) last = max(last, __shfl_xor_sync(0xFFFFFFFFu, last, off));
+            R = carry;
+            // the residual has no mass (only through rounding): p_t of the same row
+            if (R.hi > 0.f || L >= gamma) break;
+        }
+        __syncwarp();
+        const df target = df_mul_f(R, u);
+        int sel = -1;
+        if (R.hi > 0.f) {
+            for (int s0 = 0; s0 < S; s0 += 32) {
+                const int sg = s0 + lane;
+                const bool hit = (sg < S) && sp.mass_all[(static_cast<int64_t>(sg) * sp.B + b) * 2 + col] > 0.f &&
+                                 !df_ge(target, s_cum[sg]);
+                const unsigned bal = __ballot_sync(0xFFFFFFFFu, hit);
+                if (bal) {
+                    sel = s0 + __ffs(bal) - 1;
+                    break;
+                }
+            }
+        }
+        if (lane == 0) {
+            s_col = col;
+            if (sel >= 0) {
+                s_sel = sel;
+                s_rem = (sel > 0) ? df_sub(target, s_cum[sel - 1]) : target;
+            } else {
+                s_sel = (R.hi > 0.f) ? last : -1;
+                s_rem = df{__int_as_float(0x7F800000), 0.f};
+            }
+        }
+    }
+    __syncthreads();
+    if (s_sel != sp.shard) return;   // another rank's slice holds this block's draw
+    const int64_t bo = static_cast<int64_t>(b) * (gamma + 1);
+    const char *zt_row = sp.zt + (bo + L) * sp.stride_bytes;
+    const char *zd_row = (L < gamma && s_col == 0) ? sp.zd + (static_cast<int64_t>(b) * gamma + L) * sp.stride_bytes
+                                                   : nullptr;
+    const DrawCtx c = draw_ctx(zt_row, zd_row, df{st.t_lh, st.t_ll}, zd_row ? df{st.d_lh, st.d_ll} : df{0.f, 0.f});
+    const int tok = slice_find<DT>(c, sp.RVs, sp.Vs, s_rem, s_warp, &s_thr, &s_last, &s_tok);
+    if (tid == 0) {
+        const int t = (tok >= 0) ? sp.v0 + tok : -1;
+        if (sp.tok_strict) sp.tok_strict[bo + L] = t;
+        if (st.commit && sp.commit_tokens) sp.commit_tokens[bo + L] = t;
     }
 }
 
@@ -788,6 +978,15 @@ cudaError_t launch_decide(const ScanParams &p, cudaStream_t stream) {
                                        : (bf ? decide_kernel<SDD_BF16, false> : decide_kernel<SDD_F32, false>);
     return launch_dependent(k, dim3(nb, nseg),
                             dim3(kDecThreads), smem, stream, p);
+}
+
+cudaError_t launch_shard_draw(const ShardParams &sp, cudaStream_t stream) {
+    if (sp.B == 0) return cudaSuccess;
+    if (sp.dtype == SDD_BF16)
+        shard_draw_kernel<SDD_BF16><<<sp.B, kDecThreads, 0, stream>>>(sp);
+    else
+        shard_draw_kernel<SDD_F32><<<sp.B, kDecThreads, 0, stream>>>(sp);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_schedule(const ScheduleParams &p, cudaStream_t stream) {

@@ -52,6 +52,16 @@ inline FastDiv make_fastdiv(uint64_t d) {
 constexpr int kDecThreads = 256;
 constexpr int kDrawMaxSeg = 64;
 
+// Vocabulary-sharded draw: what the decide kernel leaves, per block, for the
+// draw that follows the exchange of the slices' draw-row masses (shard.cu).
+struct ShardDraw {
+    int32_t L;          // strict accepted length (the draw row is L, or gamma for the bonus row)
+    int32_t commit;     // the block's verified tokens are committed (pair 0 did not skip it)
+    float t_lh, t_ll;   // LSE of the target draw row (double-float)
+    float d_lh, d_ll;   // LSE of the drafter draw row (residual only)
+    int32_t pad[2];
+};
+
 // Per-block finalisation and decisions (decide.cu, rules.cuh).  Thresholds
 // are double-floats split on the host from their fp64 values.
 struct DecideParams {
@@ -89,6 +99,10 @@ struct DecideParams {
     int32_t nseg, seg_vec;         // segments per block and vectors per segment
     float *res_pref;               // [nb, nseg, kDecThreads] per-thread inclusive prefix sums
     uint32_t *res_count;           // [nb] (zero between calls)
+    // vocabulary-sharded decide: this slice's draw-row masses [B][2] (residual
+    // or bonus weights, then p_t weights) and the per-block draw state
+    float *shard_mass;
+    ShardDraw *shard_state;
 };
 
 // One set of rows streamed by the scan kernel (drafter rows or target rows).
@@ -127,9 +141,19 @@ struct ScanParams {
     int64_t T0, C;
     FastDiv divC, divW, divRV, divNpos[2], divWt[2];   // division by C, W, RV, grp[g].npos, wt[g]
     const int32_t *tokens;   // [B, gamma]
+    // When set, the number of listed blocks is read from this device word at
+    // launch (at most grp[g].nb, which then sizes the grid): rows, T, T0, C
+    // and the active warps follow from it on the device (PartView).
+    const int32_t *nb_dev;
     Partial *partials;       // [rows + W]
     FeatPartial *feat;       // [rows + W], or nullptr: no extended features
     int32_t *status;
+    // vocabulary-sharded decide: the S slices' records [S][rows] replace the
+    // warp partials; V and RV then describe this rank's slice
+    const sdd_shard_partial *shard;
+    int32_t n_shards;
+    int32_t shard_v0;        // first vocabulary index of this rank's slice
+    int64_t shard_rows;      // records per slice (B * (2 gamma + 1))
     uint32_t wait_polls;     // polls of a ring wait before the warp gives up (set at launch)
     int32_t drop_copy;       // failure-detection test hook: warp 0 never issues its first copy
     DecideParams dec;
@@ -157,6 +181,27 @@ void set_scan_wait_hooks(uint32_t polls, int drop_copy);
 // programmatic dependent of the streaming kernel.
 cudaError_t launch_decide(const ScanParams &p, cudaStream_t stream);
 cudaError_t launch_schedule(const ScheduleParams &p, cudaStream_t stream);
+// Vocabulary-sharded path (shard.cu): the slice's per-row records, and the
+// draw once every slice's draw-row mass is known.
+struct ShardParams {
+    const char *zd, *zt;     // this slice of the drafter [B, gamma, .] and target [B, gamma+1, .] logits
+    int64_t stride_bytes;
+    int32_t dtype, B, gamma;
+    int32_t Vs, RVs;         // slice width and its 16-byte vectors
+    int32_t v0, V;           // first index of the slice, full vocabulary
+    int32_t kcap;            // candidates kept per target row (0: none)
+    const int32_t *tokens;   // [B, gamma]
+    sdd_shard_partial *out;  // [B gamma + B (gamma + 1)]
+    int32_t *status;
+    // draw
+    int32_t n_shards, shard;
+    const float *mass_all;   // [n_shards][B][2]
+    const ShardDraw *state;  // [B]
+    uint64_t seed, round;
+    int32_t *tok_strict, *commit_tokens;
+};
+cudaError_t launch_shard_partials(const ShardParams &sp, cudaStream_t stream);
+cudaError_t launch_shard_draw(const ShardParams &sp, cudaStream_t stream);
 cudaError_t launch_agreement(const int32_t *K, const int32_t *L, int B, int n_tau, long long *acc,
                              cudaStream_t stream);
 cudaError_t launch_commit(const int32_t *K, const int32_t *x, const int32_t *vt, const int32_t *vn, int B,
@@ -224,21 +269,67 @@ __device__ __forceinline__ int64_t fast_div(int64_t n, const FastDiv &f) {
     return static_cast<int64_t>(f.pow2 ? (u >> f.s) : (__umul64hi(u, f.M) >> f.s));
 }
 
+// make_fastdiv on the device (a 128-bit division, once per warp).
+__device__ __forceinline__ FastDiv make_fastdiv_dev(uint64_t d) {
+    FastDiv f{0, 63u - static_cast<uint32_t>(__clzll(static_cast<long long>(d))), 0};
+    if ((d & (d - 1)) == 0) {
+        f.pow2 = 1;
+        return f;
+    }
+    const unsigned __int128 num = static_cast<unsigned __int128>(1) << (64 + f.s);
+    f.M = static_cast<uint64_t>((num + d - 1) / d);
+    return f;
+}
+
+// The launch's partition: from the parameters, or -- with a device block
+// count -- computed on the device the way the host computes it.
+struct PartView {
+    int64_t nb, rows0, rows, T, T0, C;
+    int32_t W;
+    FastDiv divC, divW;
+};
+
+__device__ __forceinline__ PartView part_view(const ScanParams &p) {
+    PartView v;
+    if (p.nb_dev == nullptr) {
+        v.nb = p.grp[0].nb;
+        v.rows0 = p.rows0;
+        v.rows = p.rows;
+        v.T = p.T;
+        v.T0 = p.T0;
+        v.C = p.C;
+        v.W = p.W;
+        v.divC = p.divC;
+        v.divW = p.divW;
+        return v;
+    }
+    v.nb = min(max(static_cast<int64_t>(*p.nb_dev), static_cast<int64_t>(0)), static_cast<int64_t>(p.grp[0].nb));
+    v.rows0 = v.nb * p.grp[0].npos;
+    v.rows = v.rows0 + (p.n_groups > 1 ? v.nb * p.grp[1].npos : 0);
+    v.T = v.rows * p.RV;
+    v.T0 = v.rows0 * p.RV;
+    v.C = p.wt[0] * v.T0 + p.wt[1] * (v.T - v.T0);
+    v.W = static_cast<int32_t>(max(static_cast<int64_t>(1), min(static_cast<int64_t>(p.W), v.T / 2)));
+    v.divC = make_fastdiv_dev(static_cast<uint64_t>(v.C > 0 ? v.C : 1));
+    v.divW = make_fastdiv_dev(static_cast<uint64_t>(v.W));
+    return v;
+}
+
 // Index arithmetic of the cost-balanced contiguous partition of the T
 // vectors over W warps.  Vector v occupies the cost interval [cost(v),
 // cost(v+1)) with cost(v) = wt0 min(v, T0) + wt1 max(v - T0, 0); warp w owns
 // the costs [floor(w C / W), floor((w+1) C / W)) and so the vectors whose
 // cost interval starts there: [start(w), start(w+1)) with start(w) the first
 // vector of cost >= floor(w C / W).  Requires C W < 2^53 (checked by the host).
-__device__ __forceinline__ int64_t part_start(const ScanParams &p, int64_t w) {
-    const int64_t c = fast_div(w * p.C, p.divW);
-    const int64_t c0 = p.wt[0] * p.T0;
-    return (c <= c0) ? fast_div(c + p.wt[0] - 1, p.divWt[0]) : p.T0 + fast_div(c - c0 + p.wt[1] - 1, p.divWt[1]);
+__device__ __forceinline__ int64_t part_start(const ScanParams &p, const PartView &v, int64_t w) {
+    const int64_t c = fast_div(w * v.C, v.divW);
+    const int64_t c0 = p.wt[0] * v.T0;
+    return (c <= c0) ? fast_div(c + p.wt[0] - 1, p.divWt[0]) : v.T0 + fast_div(c - c0 + p.wt[1] - 1, p.divWt[1]);
 }
 // The warp owning vector v.
-__device__ __forceinline__ int64_t part_owner(const ScanParams &p, int64_t v) {
-    const int64_t cost = (v < p.T0) ? p.wt[0] * v : p.wt[0] * p.T0 + p.wt[1] * (v - p.T0);
-    return fast_div((cost + 1) * p.W - 1, p.divC);
+__device__ __forceinline__ int64_t part_owner(const ScanParams &p, const PartView &pv, int64_t v) {
+    const int64_t cost = (v < pv.T0) ? p.wt[0] * v : p.wt[0] * pv.T0 + p.wt[1] * (v - pv.T0);
+    return fast_div((cost + 1) * pv.W - 1, pv.divC);
 }
 
 }  // namespace sdd

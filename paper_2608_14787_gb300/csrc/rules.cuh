@@ -61,9 +61,9 @@ __device__ __forceinline__ Partial load_partial(const Partial *p) {
 // the row's five largest entries t, merged from the pieces' lists (p.feat,
 // indexed like the partials) loaded in the same batches.
 template <bool FEAT>
-__device__ __forceinline__ void merge_row_t(const ScanParams &p, int64_t r, SoftState &acc, float &g, bool &tok_bad,
-                                            float (&t)[5]) {
-    const int64_t fw = part_owner(p, r * p.RV), lw = part_owner(p, (r + 1) * p.RV - 1);
+__device__ __forceinline__ void merge_row_t(const ScanParams &p, const PartView &pv, int64_t r, SoftState &acc,
+                                            float &g, bool &tok_bad, float (&t)[5]) {
+    const int64_t fw = part_owner(p, pv, r * p.RV), lw = part_owner(p, pv, (r + 1) * p.RV - 1);
     acc = soft_identity();
     g = qnan();
     tok_bad = false;
@@ -115,9 +115,51 @@ __device__ __forceinline__ void merge_row_t(const ScanParams &p, int64_t r, Soft
         }
     }
 }
-__device__ __forceinline__ void merge_row(const ScanParams &p, int64_t r, SoftState &acc, float &g, bool &tok_bad) {
+__device__ __forceinline__ void merge_row(const ScanParams &p, const PartView &pv, int64_t r, SoftState &acc, float &g,
+                                          bool &tok_bad) {
     float t[5];
-    merge_row_t<false>(p, r, acc, g, tok_bad, t);
+    merge_row_t<false>(p, pv, r, acc, g, tok_bad, t);
+}
+
+// Vocabulary-sharded rows: the merged state of row r from the S slices'
+// records (slice order), the drafted token's logit from the slice that holds
+// it, a token outside [0, V) flagged by any slice, and -- target rows with a
+// token -- its rank among the whole row's logits (entries above it, or equal
+// at a lower index), counted over the union of the slices' largest entries:
+// the kcap largest of the row all lie in that union, so the count is exact
+// up to the saturation at kcap.
+__device__ __forceinline__ void merge_row_shards(const ScanParams &p, int64_t r, int tok, bool rank, SoftState &acc,
+                                                 float &g, bool &tok_bad) {
+    acc = soft_identity();
+    g = qnan();
+    tok_bad = false;
+    for (int s = 0; s < p.n_shards; ++s) {
+        const sdd_shard_partial *rec = p.shard + static_cast<int64_t>(s) * p.shard_rows + r;
+        SoftState o;
+        o.m = rec->m;
+        o.r = rec->r;
+        o.t2 = rec->t2;
+        o.sh = rec->sh;
+        o.sl = rec->sl;
+        o.amax = rec->amax;
+        o.rank = 0;
+        acc = soft_merge(acc, o);
+        const int info = rec->info;
+        if (info & 1) g = rec->g;
+        if (info & 2) tok_bad = true;
+    }
+    if (rank && !tok_bad && !isnan(g)) {
+        int cnt = 0;
+        for (int s = 0; s < p.n_shards; ++s) {
+            const sdd_shard_partial *rec = p.shard + static_cast<int64_t>(s) * p.shard_rows + r;
+            const int nc = min((rec->info >> 8) & 0xFF, SDD_SHARD_KMAX);
+            for (int k = 0; k < nc; ++k) {
+                const float z = rec->cz[k];
+                cnt += (z > g || (z == g && rec->cv[k] < tok)) ? 1 : 0;
+            }
+        }
+        acc.rank = min(cnt, p.kcap);
+    }
 }
 
 // Final results of position j of block b (group G) from its merged state, by
@@ -167,8 +209,20 @@ __device__ __forceinline__ RowFacts row_final(const ScanParams &p, const ScanGro
                 G.maxprob[o] = fmaf(em, dm.lo, em);
             }
             if (G.lse) G.lse[o] = static_cast<double>(f.lse.hi) + static_cast<double>(f.lse.lo);
-            // H = ln S - ln 2 * t2 / S (t2 in log2 units against the same reference)
-            if (G.entropy) G.entropy[o] = (lnS.hi + lnS.lo) - kLn2 * acc.t2 / S;
+            // H = ln S' - ln 2 t2 / S with S' = S 2^-dM the sum against the
+            // row maximum, dM = M log2(e) - r (a double-float: TwoProd and
+            // TwoSum), and t2 already against the maximum: on a peaked row
+            // both terms are small, so nothing cancels
+            if (G.entropy) {
+                const float pm = acc.m * kLog2e;
+                const float pe = fmaf(acc.m, kLog2e, -pm);
+                float dh, dl;
+                two_sum(pm, -acc.r, dh, dl);
+                const df ln2df = df{kLn2Hi, kLn2Lo};
+                const df dMln2 = df_add(df_mul_f(ln2df, dh), df{(dl + pe) * kLn2, 0.f});
+                const df lnSp = df_sub(lnS, dMln2);
+                G.entropy[o] = (lnSp.hi + lnSp.lo) - kLn2 * acc.t2 / S;
+            }
             if (G.argmax) G.argmax[o] = acc.amax;
         }
     } else {

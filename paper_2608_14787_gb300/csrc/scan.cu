@@ -36,10 +36,10 @@ struct Cursor {
     int32_t k;     // vector offset inside the row
 };
 
-__device__ __forceinline__ void row_locate(const ScanParams &p, int64_t r, int &gi, int64_t &lr, int &j, int &b,
-                                           bool &b_ok) {
-    gi = (r >= p.rows0) ? 1 : 0;
-    lr = gi ? r - p.rows0 : r;
+__device__ __forceinline__ void row_locate(const ScanParams &p, const PartView &pv, int64_t r, int &gi, int64_t &lr,
+                                           int &j, int &b, bool &b_ok) {
+    gi = (r >= pv.rows0) ? 1 : 0;
+    lr = gi ? r - pv.rows0 : r;
     const ScanGroup &G = p.grp[gi];
     const int64_t i = fast_div(lr, p.divNpos[gi]);
     j = static_cast<int>(lr - i * G.npos);
@@ -48,11 +48,11 @@ __device__ __forceinline__ void row_locate(const ScanParams &p, int64_t r, int &
     if (!b_ok) b = 0;  // keep every address inside the tensor; the row is flagged at the end
 }
 
-__device__ __forceinline__ const char *row_base(const ScanParams &p, int64_t r) {
+__device__ __forceinline__ const char *row_base(const ScanParams &p, const PartView &pv, int64_t r) {
     int gi, j, b;
     int64_t lr;
     bool ok;
-    row_locate(p, r, gi, lr, j, b, ok);
+    row_locate(p, pv, r, gi, lr, j, b, ok);
     const ScanGroup &G = p.grp[gi];
     return G.base + (static_cast<int64_t>(b) * G.npos + j) * G.stride_bytes;
 }
@@ -192,7 +192,8 @@ __device__ __noinline__ int first_index(const char *rowp, int k0, int lane, int 
 // maximum rescales by an exact power of two.  A new maximum only records the
 // tile (st.amax = k0); the exact index is resolved once at the end of the piece.
 // Pairs of entries go through the packed f32x2 pipe: y = z log2(e) - r,
-// s += 2^y and, for drafter rows (ENT), t2 += 2^y y.  Drafter entries are
+// s += 2^y and, for drafter rows (ENT), t2 += 2^y (z - m) log2(e), m the
+// lane's maximum (so the dominant term of a peaked row adds 0).  Drafter entries are
 // clamped first (so a masked entry adds 0 * finite to t2); target rows need no
 // clamp (2^-inf = 0 and the maximum starts at the clamp value).  The lane's
 // exp-sum is an fp32 pair (s_hi, s_lo) updated by TwoSum once per tile.
@@ -223,12 +224,15 @@ __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lan
     }
     if (cm > st.m) {
         st.amax = k0;
+        // the entropy accumulator is kept against the lane's maximum: a new
+        // maximum shifts it by (m_old - m_new) log2(e) per unit of the sum
+        if (ENT) st.t2 = fmaf((st.m - cm) * kLog2e, s_hi + s_lo, st.t2);
         st.m = cm;
         const float rn = ceilf(cm * kLog2e);
         if (rn > st.r) {
             const float k = st.r - rn;
             const float sc = pow2f_int(k);   // exact power of two (0 below the normal range)
-            if (ENT) st.t2 = sc * fmaf(k, s_hi + s_lo, st.t2);
+            if (ENT) st.t2 *= sc;
             s_hi *= sc;
             s_lo *= sc;
             st.r = rn;
@@ -239,6 +243,10 @@ __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lan
     // arithmetic of earlier ones
     const float nr = -st.r;
     const f2_t L2 = f2_pack(kLog2e, kLog2e), NR = f2_pack(nr, nr);
+    // the lane maximum's own y (the same fma as an entry's): y - DM is an
+    // entry's (z - m) log2(e), exactly 0 for the maximum itself
+    const float dm = fmaf(st.m, kLog2e, nr);
+    const f2_t DM = f2_pack(dm, dm);
     f2_t sa = f2_pack(0.f, 0.f), sb = sa, ta = sa, tb = sa;
     constexpr int PAIRS = (DT == SDD_BF16) ? 4 : 2;   // entry pairs per 16-byte vector
 #pragma unroll
@@ -260,16 +268,44 @@ __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lan
                 const f2_t e = f2_pack(ex2(y0), ex2(y1));
                 if (q & 1) {
                     sb = f2_add(sb, e);
-                    if (ENT) tb = f2_fma(e, y, tb);
+                    if (ENT) tb = f2_fma(e, f2_sub(y, DM), tb);
                 } else {
                     sa = f2_add(sa, e);
-                    if (ENT) ta = f2_fma(e, y, ta);
+                    if (ENT) ta = f2_fma(e, f2_sub(y, DM), ta);
                 }
             }
         }
     }
     float s0, s1;
     f2_unpack(f2_add(sa, sb), s0, s1);
+    if (ENT) {
+        // A tile dominated by one term (the others sum to < 1/16 of it: the
+        // lane holding the peak of a peaked row) loses those others' low bits
+        // next to it, and they make the row's entropy.  The lane re-sums them
+        // among themselves from shared memory (rare: about one lane-tile per
+        // peaked row).
+        const float ycm = fmaf(cm, kLog2e, nr);
+        const float ecm = ex2(ycm);
+        if (s0 + s1 < 1.0625f * ecm && cm > clamp_floor()) {
+            float small = 0.f, nmax = 0.f;
+#pragma unroll 1
+            for (int i = 0; i < kVPL; ++i) {
+                const uint4 w = clamp_vec<DT>(tile[lane + 32 * i]);
+                const uint32_t *u = reinterpret_cast<const uint32_t *>(&w);
+#pragma unroll
+                for (int k = 0; k < 2 * PAIRS; ++k) {
+                    const float z = (DT == SDD_BF16) ? ((k & 1) ? bf16_hi(u[k >> 1]) : bf16_lo(u[k >> 1]))
+                                                     : __uint_as_float(u[k]);
+                    if (z == cm)
+                        nmax += 1.f;
+                    else
+                        small += ex2(fmaf(z, kLog2e, nr));
+                }
+            }
+            s0 = nmax * ecm;   // (nmax <= 64: exact)
+            s1 = small;
+        }
+    }
     float e1, e2, h;
     two_sum(s_hi, s0, h, e1);
     two_sum(h, s1, s_hi, e2);
@@ -412,13 +448,13 @@ struct RowTok {
     int t;
     bool has;
 };
-__device__ __forceinline__ RowTok row_token(const ScanParams &p, int64_t r) {
+__device__ __forceinline__ RowTok row_token(const ScanParams &p, const PartView &pv, int64_t r) {
     RowTok x{0, false};
-    if (r < p.rows) {
+    if (r < pv.rows) {
         int gi, j, b;
         int64_t lr;
         bool ok;
-        row_locate(p, r, gi, lr, j, b, ok);
+        row_locate(p, pv, r, gi, lr, j, b, ok);
         if (j < p.gamma) {
             x.t = __ldg(p.tokens + static_cast<int64_t>(b) * p.gamma + j);
             x.has = true;
@@ -428,9 +464,9 @@ __device__ __forceinline__ RowTok row_token(const ScanParams &p, int64_t r) {
 }
 // Clamped logit of row r at its drafted token (NaN if none or out of range).
 template <int DT>
-__device__ __forceinline__ float token_logit(const ScanParams &p, int64_t r, RowTok x) {
+__device__ __forceinline__ float token_logit(const ScanParams &p, const PartView &pv, int64_t r, RowTok x) {
     if (!x.has || x.t < 0 || x.t >= p.V) return __int_as_float(0x7FC00000);
-    return fmax_nan(logit_at<DT>(row_base(p, r), x.t), clamp_floor());
+    return fmax_nan(logit_at<DT>(row_base(p, pv, r), x.t), clamp_floor());
 }
 
 // FEAT: also the five largest logits of every drafter row piece (extended
@@ -444,12 +480,14 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
     // launched as a programmatic dependent of whatever precedes it in the
     // stream: nothing is read or written before that work has completed
     griddep_wait();
+    const PartView pv = part_view(p);
+    if (gw >= pv.W) return;   // (a device block count can leave warps without work)
     // The sampling draw's arrival counters of this call's blocks start at zero
     // (the decide kernel behind this one reads them only after this grid has
     // completed), so the workspace needs no zero fill and calls of any shape
     // that fits it may follow one another.
     if (gw == 0 && p.dec.enabled && p.dec.res_count != nullptr)
-        for (int i = lane; i < p.grp[0].nb; i += 32) p.dec.res_count[i] = 0u;
+        for (int i = lane; i < pv.nb; i += 32) p.dec.res_count[i] = 0u;
     constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
     const int tail = p.V % EPV;  // valid entries of the last vector of a row (0 = full)
 
@@ -462,11 +500,11 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
     }
     __syncwarp();
 
-    const int64_t v0 = part_start(p, gw), v1 = part_start(p, gw + 1);
+    const int64_t v0 = part_start(p, pv, gw), v1 = part_start(p, pv, gw + 1);
     Cursor pc{v0, fast_div(v0, p.divRV), 0};
     pc.k = static_cast<int32_t>(v0 - pc.r * p.RV);
     Cursor cc = pc;
-    const char *prow = row_base(p, pc.r);
+    const char *prow = row_base(p, pv, pc.r);
     const uint64_t pol = l2_evict_first_policy();   // the logits are read once
     uint32_t pending = 0;  // slots with a copy in flight
     uint32_t phase = 0;    // parity bit per slot
@@ -493,7 +531,7 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
         if (pc.k == p.RV && pc.v < v1) {
             pc.k = 0;
             pc.r += 1;
-            prow = row_base(p, pc.r);
+            prow = row_base(p, pv, pc.r);
         }
     };
     for (int s = 0; s < kStages && pc.v < v1; ++s) issue(s);
@@ -501,8 +539,8 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
     // Drafted tokens and their logits run ahead of the stream: the token two
     // rows ahead and the logit one row ahead are in flight while the current
     // piece streams, so no piece start waits on a dependent pair of loads.
-    RowTok tokA = row_token(p, cc.r), tokB = row_token(p, cc.r + 1);
-    float gA = token_logit<DT>(p, cc.r, tokA);
+    RowTok tokA = row_token(p, pv, cc.r), tokB = row_token(p, pv, cc.r + 1);
+    float gA = token_logit<DT>(p, pv, cc.r, tokA);
 
     SoftState st = soft_identity();
     uint32_t ck[5];        // FEAT: the lane's five largest tile maxima of the piece (keys) ...
@@ -536,7 +574,7 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
             int gi, j, b;
             int64_t lr;
             bool ok;
-            row_locate(p, cc.r, gi, lr, j, b, ok);
+            row_locate(p, pv, cc.r, gi, lr, j, b, ok);
             const ScanGroup &G = p.grp[gi];
             crow = G.base + (static_cast<int64_t>(b) * G.npos + j) * G.stride_bytes;
             ent = G.kind == 0;
@@ -545,9 +583,9 @@ __global__ void __launch_bounds__(kThreads, 1) scan_kernel(const __grid_constant
             tok_bad = tokA.has && !tok_ok;
             g = gA;
             // advance the prefetch: logit of the next row, token of the one after
-            gA = token_logit<DT>(p, cc.r + 1, tokB);
+            gA = token_logit<DT>(p, pv, cc.r + 1, tokB);
             tokA = tokB;
-            tokB = row_token(p, cc.r + 2);
+            tokB = row_token(p, pv, cc.r + 2);
             rank_on = !ent && tok >= 0;
             wrank = 0;
             in_piece = true;

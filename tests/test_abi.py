@@ -123,3 +123,44 @@ def test_empty_batch_is_a_no_op(lib):
                               None) == 0
     assert lib.sdd_commit(None, None, None, None, 0, 4, None, None, None) == 0
     assert lib.sdd_agreement(None, None, 0, 3, None, None) == 0
+
+
+def test_shard_record_layout_matches_c(tmp_path):
+    """sdd_shard_partial is exchanged between ranks as plain bytes: 160 bytes,
+    fields at fixed offsets."""
+    from paper_2608_14787_gb300.vocab_shard import RECORD_BYTES
+    want = {"m": 0, "r": 4, "t2": 8, "sh": 12, "sl": 16, "amax": 20, "g": 24, "info": 28, "cz": 32, "cv": 96}
+    prog = ["#include <stdio.h>", "#include <stddef.h>", f'#include "{HEADER}"', "int main(void) {",
+            'printf("%zu\\n", sizeof(sdd_shard_partial));']
+    for f in want:
+        prog.append(f'printf("%zu\\n", offsetof(sdd_shard_partial, {f}));')
+    prog.append("return 0; }")
+    c = tmp_path / "rec.c"
+    c.write_text("\n".join(prog))
+    exe = tmp_path / "rec"
+    subprocess.check_call(["gcc", "-std=c11", "-o", str(exe), str(c)])
+    vals = [int(x) for x in subprocess.check_output([str(exe)]).split()]
+    assert vals[0] == RECORD_BYTES == 160
+    assert dict(zip(want, vals[1:])) == want
+
+
+def test_shard_arguments_rejected_on_host(lib):
+    from paper_2608_14787_gb300.binding import BlockArgs
+    a = BlockArgs()
+    a.dtype, a.B, a.gamma, a.V, a.row_stride = 1, 2, 4, 1000, 504
+    a.draft_logits = a.target_logits = a.draft_tokens = 256
+    out = ctypes.c_void_p(256)
+    # slice outside [0, V)
+    assert lib.sdd_shard_partials(ctypes.byref(a), 900, 1001, out, None) == 1
+    assert b"slice" in lib.sdd_last_error()
+    # slice wider than the row stride
+    assert lib.sdd_shard_partials(ctypes.byref(a), 0, 600, out, None) == 1
+    # top-k beyond the candidates a record keeps
+    ks = (ctypes.c_int32 * 1)(17)
+    a.n_k, a.topk = 1, ctypes.cast(ks, ctypes.POINTER(ctypes.c_int32))
+    assert lib.sdd_shard_partials(ctypes.byref(a), 0, 500, out, None) == 2
+    # shard index out of range
+    a.n_k = 0
+    assert lib.sdd_shard_draw(ctypes.byref(a), 0, 500, 2, 2, ctypes.c_void_p(256), None) == 1
+    n = ctypes.c_size_t(0)
+    assert lib.sdd_shard_workspace_size(5, ctypes.byref(n)) == 0 and n.value == 5 * 32

@@ -481,3 +481,21 @@ def test_features_planted_top5_layouts(sdd, V):
     if V % 8:
         z_d = _padded(z_d, (V + 7) // 8 * 8)
     _check_features(sdd, z_d, x, torch.bfloat16)
+
+
+def test_entropy_of_peaked_fp32_rows(sdd):
+    """fp32 rows with one token 8 nats above the rest (entropy ~ 6e-3): the
+    entropy is a difference of two terms of order one unless it is accumulated
+    against the row maximum; it must hold the fp32 tolerance (1e-5 relative)
+    in the confidence call and in the fused round."""
+    blk = synth.make_block("c3", device="cpu", B=6, gamma=16, V=20_008, dtype=torch.float32, greedy_drafts=True)
+    z_d, z_t, x = _to_dev(blk)
+    conf = sdd.confidence(z_d, x)
+    rnd = sdd.BlockRound(6, 16, 20_008, dtype=torch.float32, taus=(0.9,), K_min=2)
+    rnd.set_inputs(z_d, z_t, x, seed=1, round_=0)
+    rnd.run()
+    torch.cuda.synchronize()
+    st = orc.row_stats(blk.z_d.numpy(), tokens=blk.x.numpy())
+    assert (st.entropy < 0.05).mean() > 0.25    # the workload's peaked rows
+    assert_close_stats("entropy", conf.entropy, st.entropy, torch.float32)
+    assert_close_stats("entropy", rnd.entropy, st.entropy, torch.float32)

@@ -85,3 +85,67 @@ def test_two_gloo_ranks_sum_to_whole_batch(orc, tmp_path):
     for r in range(WORLD):
         np.testing.assert_array_equal(np.load(tmp_path / f"tot{r}.npy"), want)
         assert np.load(tmp_path / f"max{r}.npy")[0] == 1.5 * WORLD
+
+
+# ---------------------------------------------------------------------------
+# Vocabulary-sharded round: the exchanges between ranks (vocab_shard), with
+# stand-in record bytes (the records themselves come from the GPU kernels and
+# are checked by tests/test_gpu_shard.py)
+# ---------------------------------------------------------------------------
+ROWS = 13
+
+
+def _records(rank):
+    g = torch.Generator().manual_seed(100 + rank)
+    return torch.randint(0, 256, (ROWS * 160,), dtype=torch.uint8, generator=g)
+
+
+def _tokens(rank):
+    # every rank holds -1 at the drawn positions except the rank that drew them
+    t = torch.full((4, 9), -1, dtype=torch.int32)
+    t[:, :3] = torch.arange(12, dtype=torch.int32).view(4, 3)
+    t[rank, 3 + rank] = 1000 + rank
+    return t
+
+
+def _exchange_worker(rank, port, outdir):
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    import torch.distributed as dist
+    from paper_2608_14787_gb300 import vocab_shard
+    dist.init_process_group("gloo", rank=rank, world_size=WORLD)
+    try:
+        allr = vocab_shard._all_gather(_records(rank), WORLD, None)
+        mass = torch.tensor([[rank + 0.5, 2.0 * rank]] * 3, dtype=torch.float32)
+        allm = vocab_shard._all_gather(mass.reshape(-1), WORLD, None).reshape(WORLD, 3, 2)
+        tok = _tokens(rank)
+        vocab_shard._all_reduce_max(tok, None)
+        torch.save({"rec": allr, "mass": allm, "tok": tok}, os.path.join(outdir, f"ex{rank}.pt"))
+        dist.barrier()
+    finally:
+        dist.destroy_process_group()
+
+
+def test_vocab_shard_exchanges_two_gloo_ranks(tmp_path):
+    """All-gather of the record bytes (slice order), of the draw-row masses,
+    and the MAX all-reduce that completes the drawn tokens: every rank ends
+    with the same buffers, equal to the single-process concatenation."""
+    mp.spawn(_exchange_worker, args=(_free_port(), str(tmp_path)), nprocs=WORLD, join=True)
+    want_rec = torch.stack([_records(r) for r in range(WORLD)])
+    want_tok = torch.stack([_tokens(r) for r in range(WORLD)]).amax(dim=0)
+    for r in range(WORLD):
+        got = torch.load(tmp_path / f"ex{r}.pt")
+        assert torch.equal(got["rec"], want_rec)
+        assert torch.equal(got["mass"][1, 0], torch.tensor([1.5, 2.0]))
+        assert torch.equal(got["tok"], want_tok)
+        assert got["tok"][0, 3] == 1000 and got["tok"][1, 4] == 1001
+
+
+def test_slice_bounds_cover_the_vocabulary():
+    from paper_2608_14787_gb300 import vocab_shard
+    for V in (1, 7, 8, 1003, 151_936):
+        for S in (1, 2, 3, 8):
+            b = vocab_shard.slice_bounds(V, S)
+            assert b[0][0] == 0 and b[-1][1] == V
+            assert all(b[i][1] == b[i + 1][0] for i in range(len(b) - 1))
+            assert all(v0 % 8 == 0 and v1 > v0 for v0, v1 in b)
