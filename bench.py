@@ -780,13 +780,14 @@ def run_component_features(args):
 
 def run_component_loop(args):
     """The decode-loop workload (B=128, gamma=32, V=151,936 bf16): `--steps`
-    rounds (default 64) of fresh logits and hidden states, generated untimed."""
+    rounds (default 256, the workload's count), enqueued back to back with no
+    host round trip (inputs: 8 seeded sets generated before the timed region)."""
     import torch
     from paper_2608_14787_gb300 import build as sdd_build
     from paper_2608_14787_gb300 import loop as sdd_loop
     from paper_2608_14787_gb300 import synth
     sdd_build.build()
-    rounds = args.steps if args.steps != 4000 else 64
+    rounds = args.steps if args.steps != 4000 else 256
     with ClockSampler(None) as clk:
         res = sdd_loop.run(rounds, "c5", warmup=max(2, min(args.warmup, 4)))
     cpu = None

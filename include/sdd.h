@@ -269,6 +269,31 @@ SDD_API sdd_status_t sdd_verify_strict(const void *target_logits, const void *dr
                                size_t workspace_bytes, int32_t *status, sdd_stream_t stream);
 
 /*
+ * sdd_select_rows -- the blocks a decode loop sends to the verifier (Sec. 4.1:
+ * every block the skip policy did not skip): rows[0..n) = the indices b with
+ * K[b] == 0 in ascending order, *n_rows = n (K [B], rows [B], n_rows: device).
+ * With sdd_verify_strict_listed this keeps the verifier's row list on the
+ * device, so that a loop round needs no host round trip.
+ */
+SDD_API sdd_status_t sdd_select_rows(const int32_t *K, int B, int32_t *rows, int32_t *n_rows, sdd_stream_t stream);
+
+/*
+ * sdd_verify_strict_listed -- sdd_verify_strict of the blocks rows[0..n) with
+ * the count n read from device memory when the kernels run (*n_rows, at most
+ * B; rows: device [B]), e.g. as written by sdd_select_rows on the same
+ * stream.  The launch covers up to B blocks and the streaming pass splits
+ * the listed blocks' target rows over the warps on the device.  Arguments and
+ * outputs otherwise as sdd_verify_strict (draft_lse required for sampling).
+ */
+SDD_API sdd_status_t sdd_verify_strict_listed(const void *target_logits, const void *draft_logits,
+                                              sdd_dtype_t dtype, int B, int gamma, int V, int64_t row_stride,
+                                              const int32_t *draft_tokens, const double *draft_lse, int greedy,
+                                              uint64_t seed, uint64_t round, const int32_t *rows,
+                                              const int32_t *n_rows, int32_t *L, int32_t *tokens, int32_t *n_commit,
+                                              void *workspace, size_t workspace_bytes, int32_t *status,
+                                              sdd_stream_t stream);
+
+/*
  * sdd_verify_lenient -- lenience acceptance (App. A.6 Eq. 9) for n_ell values in
  * one read of the target rows: accept x_j iff z_j(x_j) - max_v z_j(v) >= log ell,
  * except that ell = 1 uses the strict argmax comparison.  The longest accepted

@@ -108,6 +108,11 @@ def load(path: str | None = None):
     L.sdd_position_metrics.restype = I
     L.sdd_test_wait_hooks.argtypes = [ctypes.c_uint32, I]
     L.sdd_test_wait_hooks.restype = I
+    L.sdd_select_rows.argtypes = [VP, I, VP, VP, VP]
+    L.sdd_select_rows.restype = I
+    L.sdd_verify_strict_listed.argtypes = [VP, VP, I, I, I, I, i64, VP, VP, I, u64, u64, VP, VP, VP, VP, VP, VP,
+                                           ctypes.c_size_t, VP, VP]
+    L.sdd_verify_strict_listed.restype = I
     L.sdd_shard_workspace_size.argtypes = [I, ctypes.POINTER(ctypes.c_size_t)]
     L.sdd_shard_workspace_size.restype = I
     L.sdd_shard_partials.argtypes = [ctypes.POINTER(BlockArgs), I, I, VP, VP]
@@ -320,6 +325,37 @@ def verify_strict(z_t, x, *, z_d=None, draft=None, greedy=False, seed=0, round_=
                                   1 if greedy else 0, seed, round_, _p(rows), n_rows, _p(L), _p(tok), _p(n),
                                   ws.ptr, ws.nbytes, _p(status), _stream(stream))
     _check(rc, "sdd_verify_strict")
+    return L, tok, n
+
+
+def select_rows(K, rows=None, n_rows=None, stream=None):
+    """sdd_select_rows: (rows [B] int32, n_rows [1] int32), both on the device."""
+    B = K.numel()
+    rows = torch.empty(B, dtype=torch.int32, device=K.device) if rows is None else rows
+    n_rows = torch.empty(1, dtype=torch.int32, device=K.device) if n_rows is None else n_rows
+    _check(load().sdd_select_rows(_p(K), B, _p(rows), _p(n_rows), _stream(stream)), "sdd_select_rows")
+    return rows, n_rows
+
+
+def verify_strict_listed(z_t, x, rows, n_rows, *, z_d=None, draft=None, greedy=False, seed=0, round_=0,
+                         ws: Workspace | None = None, status=None, stream=None, out=None):
+    """sdd_verify_strict_listed: the blocks rows[0..n_rows[0]) with the count on the
+    device; returns (L [B], tokens [B, gamma+1], n_commit [B])."""
+    B, gamma = x.shape
+    V, stride = _logits_layout(z_t, "z_t")
+    dev = z_t.device
+    ws = ws or Workspace(B, gamma, V, dev)
+    status = new_status(dev) if status is None else status
+    if out is None:
+        out = (torch.full((B,), -2, dtype=torch.int32, device=dev),
+               torch.full((B, gamma + 1), -2, dtype=torch.int32, device=dev),
+               torch.full((B,), -2, dtype=torch.int32, device=dev))
+    L, tok, n = out
+    lse = None if draft is None else draft.lse
+    rc = load().sdd_verify_strict_listed(_p(z_t), _p(z_d), _dtype_code(z_t), B, gamma, V, stride, _p(x), _p(lse),
+                                         1 if greedy else 0, seed, round_, _p(rows), _p(n_rows), _p(L), _p(tok),
+                                         _p(n), ws.ptr, ws.nbytes, _p(status), _stream(stream))
+    _check(rc, "sdd_verify_strict_listed")
     return L, tok, n
 
 

@@ -281,11 +281,13 @@ sdd_status_t check_rows(const int32_t *rows, int n_rows, int B) {
 // `dec` run inside the same launch.
 sdd_status_t target_scan(const Work &w, const void *target_logits, sdd_dtype_t dtype, int B, int gamma, int V,
                          int64_t row_stride, const int32_t *tokens, const int32_t *rows, int n_rows, int kcap,
-                         const DecideParams &dec, int32_t *status, cudaStream_t stream) {
+                         const DecideParams &dec, int32_t *status, cudaStream_t stream,
+                         const int32_t *nb_dev = nullptr) {
     ScanParams p;
     init_scan(p, w, dtype, B, gamma, V, tokens, status);
     p.n_groups = 1;
     p.kcap = kcap;
+    p.nb_dev = nb_dev;   // the listed-block count, read on the device (n_rows is then its maximum)
     ScanGroup &G = p.grp[0];
     G.base = static_cast<const char *>(target_logits);
     G.stride_bytes = row_stride * esize(dtype);
@@ -475,6 +477,48 @@ sdd_status_t sdd_verify_strict(const void *target_logits, const void *draft_logi
     d.tok_strict = tokens;
     d.n_strict = n_commit;
     return target_scan(w, target_logits, dtype, B, gamma, V, row_stride, draft_tokens, rows, n_rows, 1, d, status, st);
+}
+
+sdd_status_t sdd_verify_strict_listed(const void *target_logits, const void *draft_logits, sdd_dtype_t dtype, int B,
+                                      int gamma, int V, int64_t row_stride, const int32_t *draft_tokens,
+                                      const double *draft_lse, int greedy, uint64_t seed, uint64_t round,
+                                      const int32_t *rows, const int32_t *n_rows, int32_t *L, int32_t *tokens,
+                                      int32_t *n_commit, void *workspace, size_t workspace_bytes, int32_t *status,
+                                      sdd_stream_t stream) {
+    SDD_TRY(check_shape(dtype, B, gamma, V, row_stride));
+    if (B == 0) return SDD_OK;
+    if (!rows || !n_rows) return fail(SDD_ERR_INVALID_ARGUMENT, "rows and n_rows must not be NULL");
+    SDD_TRY(check_ptr16(target_logits, "target_logits"));
+    if (!draft_tokens) return fail(SDD_ERR_INVALID_ARGUMENT, "draft_tokens is NULL");
+    if (!greedy) {
+        SDD_TRY(check_ptr16(draft_logits, "draft_logits"));
+        if (!draft_lse) return fail(SDD_ERR_INVALID_ARGUMENT, "sampling needs draft_lse");
+    }
+    Work w;
+    SDD_TRY(get_work(workspace, workspace_bytes, B, gamma, w));
+    DecideParams d;
+    std::memset(&d, 0, sizeof d);
+    init_dec(d, w, dtype, B, gamma, V, row_stride, draft_tokens, B);
+    d.zt = static_cast<const char *>(target_logits);
+    d.zd = static_cast<const char *>(draft_logits);
+    d.d_lse = draft_lse;
+    d.do_strict = 1;
+    d.greedy = greedy ? 1 : 0;
+    d.seed = seed;
+    d.round = round;
+    d.L_strict = L;
+    d.tok_strict = tokens;
+    d.n_strict = n_commit;
+    return target_scan(w, target_logits, dtype, B, gamma, V, row_stride, draft_tokens, rows, B, 1, d, status,
+                       reinterpret_cast<cudaStream_t>(stream), n_rows);
+}
+
+sdd_status_t sdd_select_rows(const int32_t *K, int B, int32_t *rows, int32_t *n_rows, sdd_stream_t stream) {
+    if (B < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "B = %d < 0", B);
+    if (!rows || !n_rows || (B > 0 && !K)) return fail(SDD_ERR_INVALID_ARGUMENT, "K, rows and n_rows must not be NULL");
+    cudaError_t e = launch_select_rows(K, B, rows, n_rows, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "select rows launch");
+    return SDD_OK;
 }
 
 sdd_status_t sdd_verify_lenient(const void *target_logits, sdd_dtype_t dtype, int B, int gamma, int V,

@@ -980,6 +980,39 @@ cudaError_t launch_decide(const ScanParams &p, cudaStream_t stream) {
                             dim3(kDecThreads), smem, stream, p);
 }
 
+// The blocks that go to the verifier: K[b] == 0, in ascending order, by one
+// CTA (a ballot and a running offset per chunk of 1024).
+__global__ void __launch_bounds__(1024) select_rows_kernel(const int32_t *K, int B, int32_t *rows, int32_t *n_rows) {
+    __shared__ int s_warp[32];
+    __shared__ int s_base;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if (tid == 0) s_base = 0;
+    __syncthreads();
+    for (int c0 = 0; c0 < B; c0 += 1024) {
+        const int b = c0 + tid;
+        const bool sel = b < B && K[b] == 0;
+        const unsigned bal = __ballot_sync(0xFFFFFFFFu, sel);
+        if (lane == 0) s_warp[warp] = __popc(bal);
+        __syncthreads();
+        int before = s_base;
+        for (int w = 0; w < warp; ++w) before += s_warp[w];
+        if (sel) rows[before + __popc(bal & ((1u << lane) - 1u))] = b;
+        __syncthreads();
+        if (tid == 0) {
+            int tot = 0;
+            for (int w = 0; w < 32; ++w) tot += s_warp[w];
+            s_base += tot;
+        }
+        __syncthreads();
+    }
+    if (tid == 0) *n_rows = s_base;
+}
+
+cudaError_t launch_select_rows(const int32_t *K, int B, int32_t *rows, int32_t *n_rows, cudaStream_t stream) {
+    select_rows_kernel<<<1, 1024, 0, stream>>>(K, B, rows, n_rows);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_shard_draw(const ShardParams &sp, cudaStream_t stream) {
     if (sp.B == 0) return cudaSuccess;
     if (sp.dtype == SDD_BF16)

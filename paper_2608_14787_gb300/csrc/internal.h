@@ -204,6 +204,8 @@ cudaError_t launch_shard_partials(const ShardParams &sp, cudaStream_t stream);
 cudaError_t launch_shard_draw(const ShardParams &sp, cudaStream_t stream);
 cudaError_t launch_agreement(const int32_t *K, const int32_t *L, int B, int n_tau, long long *acc,
                              cudaStream_t stream);
+// The batch indices b with K[b] == 0, ascending, and their count (one CTA).
+cudaError_t launch_select_rows(const int32_t *K, int B, int32_t *rows, int32_t *n_rows, cudaStream_t stream);
 cudaError_t launch_commit(const int32_t *K, const int32_t *x, const int32_t *vt, const int32_t *vn, int B,
                           int gamma, int32_t *out_t, int32_t *out_n, cudaStream_t stream);
 cudaError_t launch_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b, const uint64_t *round,

@@ -80,7 +80,7 @@ def test_loop_matches_oracle_replay(sdd, orc, B, gamma, V, hidden, rounds, score
         np.testing.assert_array_equal(out.K_per.cpu().numpy(), K_per)
         np.testing.assert_array_equal(loop.D_per.cpu().numpy(), D_per)
         L_dev, tok_dev, n_dev = out.L.cpu().numpy(), out.tokens.cpu().numpy(), out.n.cpu().numpy()
-        assert out.n_verified == int((K_raw == 0).sum())
+        assert int(out.n_verified.item()) == int((K_raw == 0).sum())
         for b in range(B):
             if K_raw[b] > 0:
                 seen_skip += 1
@@ -135,7 +135,7 @@ def test_loop_full_size_decode_workload(sdd, orc):
         np.testing.assert_array_equal(loop.D_per.cpu().numpy(), D_per)
         # strict verification of verified blocks (K = 0): the first, the last and random ones
         ver = np.flatnonzero(K_dev == 0)
-        assert out.n_verified == ver.size
+        assert int(out.n_verified.item()) == ver.size
         pick = sorted(set(ver[:2].tolist() + ver[-2:].tolist() +
                           rng.choice(ver, size=min(6, ver.size), replace=False).tolist())) if ver.size else []
         assert len(pick) >= min(8, ver.size)

@@ -499,3 +499,31 @@ def test_entropy_of_peaked_fp32_rows(sdd):
     assert (st.entropy < 0.05).mean() > 0.25    # the workload's peaked rows
     assert_close_stats("entropy", conf.entropy, st.entropy, torch.float32)
     assert_close_stats("entropy", rnd.entropy, st.entropy, torch.float32)
+
+
+@pytest.mark.parametrize("frac", [0.0, 0.4, 1.0])
+def test_select_rows_and_listed_verify(sdd, frac):
+    """The verifier's block list selected on the device (K == 0) and verified
+    with its count read there equals sdd_verify_strict on the host list;
+    unlisted blocks keep their previous contents."""
+    B, gamma, V = 21, 10, 6000
+    blk = synth.make_block("c3", device="cpu", B=B, gamma=gamma, V=V)
+    z_d, z_t, x = _to_dev(blk)
+    g = torch.Generator().manual_seed(int(frac * 10))
+    K = torch.where(torch.rand(B, generator=g) < frac, torch.zeros(B, dtype=torch.int32),
+                    torch.randint(1, gamma + 1, (B,), generator=g, dtype=torch.int32)).to(DEV)
+    rows, n = sdd.select_rows(K)
+    draft = sdd.confidence(z_d, x)
+    L, tok, nc = sdd.verify_strict_listed(z_t, x, rows, n, z_d=z_d, draft=draft, seed=4, round_=9)
+    torch.cuda.synchronize()
+    want_rows = torch.nonzero(K == 0).flatten().to(torch.int32)
+    assert int(n.item()) == want_rows.numel()
+    assert torch.equal(rows[:want_rows.numel()], want_rows)
+    if want_rows.numel():
+        L2, tok2, nc2 = sdd.verify_strict(z_t, x, z_d=z_d, draft=draft, seed=4, round_=9, rows=want_rows)
+        torch.cuda.synchronize()
+        assert torch.equal(L, L2) and torch.equal(tok, tok2) and torch.equal(nc, nc2)
+        ob = oracle_block(z_d, z_t, x, seed=4, round_=9, blocks=want_rows.cpu().tolist())
+        compare_rule(Tally(), "listed", L, tok, ob.strict, want_rows.cpu().tolist())
+    skipped = (K != 0).nonzero().flatten()
+    assert torch.all(L[skipped] == -2) and torch.all(tok[skipped] == -2)
