@@ -22,6 +22,7 @@ Other rows of the path, one JSON line each (not the fused-round contract line):
   python bench.py --component features          drafter confidence with / without the extended features
   python bench.py --component scorer [--steps K] the deep scorer (K calls)
   python bench.py --component diag              the permutation diagnostic (Table 1 settings)
+  python bench.py --component shard [--shards S] the vocabulary-sharded round (S ranks in turn on one GPU)
 """
 from __future__ import annotations
 
@@ -708,6 +709,65 @@ def run_component_diag(args):
     return 0
 
 
+def run_component_shard(args):
+    """The vocabulary-sharded round on the benchmark's workload (c3: B=16,
+    gamma=32, V=151,936 bf16, every rule) with S = --shards ranks played in
+    turn on one GPU (vocab_shard.run_local: the exchanges are device-memory
+    concatenations and maxima, timed with the rest): blocks/s of the whole
+    round, and the per-slice partials kernel alone (bytes of one slice's logits
+    over its launch time)."""
+    import torch
+    import paper_2608_14787_gb300 as sdd
+    from paper_2608_14787_gb300 import build as sdd_build
+    from paper_2608_14787_gb300 import synth, vocab_shard
+    sdd_build.build()
+    sdd.load()
+    wl, ells, ks = _workload_cfg("c3")
+    S = args.shards
+    bounds = vocab_shard.slice_bounds(wl.V, S)
+    blk = synth.make_block(wl, device="cuda", round_=0)
+    sd = [vocab_shard.slice_logits(blk.z_d, v0, v1) for v0, v1 in bounds]
+    st = [vocab_shard.slice_logits(blk.z_t, v0, v1) for v0, v1 in bounds]
+    ranks = [vocab_shard.ShardRound(wl.B, wl.gamma, wl.V, v0, v1, taus=wl.taus, ells=ells, ks=ks, K_min=6)
+             for v0, v1 in bounds]
+    for r in range(3):
+        vocab_shard.run_local(ranks, sd, st, blk.x, seed=wl.seed, round_=r)
+    torch.cuda.synchronize()
+    n = max(10, min(args.steps, 200))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(None) as clk:
+        torch.cuda._sleep(int(args.prefill_us * 2.0e3))
+        e0.record()
+        for r in range(n):
+            vocab_shard.run_local(ranks, sd, st, blk.x, seed=wl.seed, round_=r)
+        e1.record()
+        torch.cuda.synchronize()
+    round_ms = e0.elapsed_time(e1) / n
+    # one slice's partials kernel, back to back
+    r0 = ranks[0]
+    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a0.record()
+    for _ in range(50):
+        r0.partials()
+    a1.record()
+    torch.cuda.synchronize()
+    part_ms = a0.elapsed_time(a1) / 50
+    w = bounds[0][1] - bounds[0][0]
+    slice_bytes = wl.B * (2 * wl.gamma + 1) * w * 2
+    peak, kind = _peaks()
+    status = max(int(r.status.item()) for r in ranks)
+    line = {"component": f"vocabulary-sharded round, S = {S} ranks played in turn on one GPU",
+            "metric": "blocks/s", "unit": "blocks/s", "value": wl.B / (round_ms / 1e3), "ms_per_round": round_ms,
+            "config": {"workload": "c3", "B": wl.B, "gamma": wl.gamma, "V": wl.V, "shards": S,
+                       "slices": [list(b) for b in bounds]},
+            "partials_kernel": {"ms": part_ms, "bytes": slice_bytes, "achieved_gbs": slice_bytes / (part_ms / 1e3) / 1e9,
+                                "peak": peak, "frac": slice_bytes / (part_ms / 1e3) / 1e9 / peak,
+                                "peak_source": f"{kind} hbm_gbs"},
+            "clocks": clk.summary(), "device_status": status}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_component_features(args):
     """Drafter confidence with and without the extended features (App. A.7:
     probability margin, top-5 mass) on the drafter half of the c3 workload
@@ -842,7 +902,8 @@ def main():
     ap.add_argument("--sets", type=int, default=3, help="rotating input sets (3 x 316 MB exceeds L2)")
     ap.add_argument("--traffic", type=float, default=None,
                     help="dram bytes per scan launch from an ncu capture of the current kernel")
-    ap.add_argument("--component", default=None, choices=["mlp", "loop", "features", "scorer", "diag"],
+    ap.add_argument("--shards", type=int, default=2, help="--component shard: vocabulary slices")
+    ap.add_argument("--component", default=None, choices=["mlp", "loop", "features", "scorer", "diag", "shard"],
                     help="measure one other row of the path instead of the fused round")
     args = ap.parse_args()
     if args.gpus > 1 and "WORLD_SIZE" not in os.environ:
@@ -857,6 +918,8 @@ def main():
         return run_component_scorer(args)
     if args.component == "diag":
         return run_component_diag(args)
+    if args.component == "shard":
+        return run_component_shard(args)
     if args.traffic is None and args.workload == "c3":
         args.traffic = SCAN_TRAFFIC_C3
     if args.warmup < 3:

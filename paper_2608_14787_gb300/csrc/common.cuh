@@ -448,6 +448,58 @@ __device__ __forceinline__ SoftState soft_warp_reduce(SoftState v) {
     return v;
 }
 
+// ---------------------------------------------------------------------------
+// 16-byte vectors of logits (8 bf16 or 4 fp32 entries)
+// ---------------------------------------------------------------------------
+// Entries of one 16-byte vector past the end of the row become -inf.
+template <int DT>
+__device__ __forceinline__ void mask_tail(uint4 &w, int valid) {
+    uint32_t *u = reinterpret_cast<uint32_t *>(&w);
+    if (DT == SDD_BF16) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+            if (e >= valid) {
+                const uint32_t sh = (e & 1) ? 16u : 0u;
+                u[e >> 1] = (u[e >> 1] & ~(0xFFFFu << sh)) | (0xFF80u << sh);
+            }
+    } else {
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+            if (e >= valid) u[e] = 0xFF800000u;
+    }
+}
+
+// Entry e of a vector for a run-time e: the word is picked by selects, so the
+// vector never has to live in memory to be indexed.
+template <int DT>
+__device__ __forceinline__ float vec_elem_sel(const uint4 &w, int e) {
+    const int k = (DT == SDD_BF16) ? (e >> 1) : e;
+    const uint32_t u = (k < 2) ? ((k == 0) ? w.x : w.y) : ((k == 2) ? w.z : w.w);
+    if (DT == SDD_BF16) return (e & 1) ? bf16_hi(u) : bf16_lo(u);
+    return __uint_as_float(u);
+}
+
+template <int DT>
+__device__ __forceinline__ float vec_elem(const uint4 &w, int e) {
+    const uint32_t *u = reinterpret_cast<const uint32_t *>(&w);
+    if (DT == SDD_BF16) return (e & 1) ? bf16_hi(u[e >> 1]) : bf16_lo(u[e >> 1]);
+    return __uint_as_float(u[e]);
+}
+
+// Clamp one vector from below (NaN-propagating).
+template <int DT>
+__device__ __forceinline__ uint4 clamp_vec(uint4 w) {
+    uint32_t *u = reinterpret_cast<uint32_t *>(&w);
+    if (DT == SDD_BF16) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) u[q] = bf16x2_max_nan(u[q], kClampPairBf16);
+    } else {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) u[q] = __float_as_uint(fmax_nan(__uint_as_float(u[q]), clamp_floor()));
+    }
+    return w;
+}
+
 __device__ __forceinline__ void status_or(int32_t *status, uint32_t bits) {
     if (status) atomicOr(reinterpret_cast<unsigned int *>(status), bits);
 }

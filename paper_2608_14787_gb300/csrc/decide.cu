@@ -399,9 +399,11 @@ __device__ __forceinline__ void sched_pair(const DecideParams &d, const BlockFac
     sched_final(Kh, D, d.K_min, d.S_max, K, Do);
 }
 
-// FEAT: also the extended features of the drafter rows (a separate
-// instantiation, so that calls without them keep the smaller kernel).
-template <int DT, bool FEAT>
+// FEAT: also the extended features of the drafter rows; SHARD: the
+// vocabulary-sharded round (records of S slices instead of warp partials,
+// the draw left to shard_draw_kernel).  Separate instantiations, so that the
+// fused round keeps the smallest kernel.
+template <int DT, bool FEAT, bool SHARD = false>
 __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_constant__ ScanParams p) {
     griddep_wait();   // launched behind the streaming grid that wrote the partials
     const DecideParams &d = p.dec;
@@ -461,7 +463,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                 float g;
                 bool bad;
                 const int64_t r = (gd ? pv.rows0 : 0) + static_cast<int64_t>(i) * G.npos + j;
-                if (p.shard != nullptr) {
+                if (SHARD) {
                     merge_row_shards(p, r, -1, false, acc, g, bad);
                     f = row_final(p, G, j, b, acc, g, bad, leader);
                 } else if (FEAT && leader) {
@@ -490,7 +492,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
             float g;
             bool bad;
             const int64_t r = (gt ? pv.rows0 : 0) + static_cast<int64_t>(i) * G.npos + j;
-            if (p.shard != nullptr)
+            if (SHARD)
                 merge_row_shards(p, r, (j < gamma) ? __ldg(d.tokens + ob + j) : -1, j < gamma, acc, g, bad);
             else
                 merge_row(p, pv, r, acc, g, bad);
@@ -526,7 +528,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
         }
         __syncthreads();
 
-        if (p.shard != nullptr) {
+        if (SHARD) {
             // ---- vocabulary-sharded (one CTA per block): this slice's masses
             // of the draw row -- the residual (or bonus) weights, then p_t --
             // for the exchange between ranks; shard_draw_kernel then draws ----
@@ -959,7 +961,8 @@ int decide_max_ctas_per_sm() {
 cudaError_t decide_prepare_device() {
     constexpr int bytes = kDrawMaxSeg * kDecThreads * static_cast<int>(sizeof(float));
     void (*const kernels[])(ScanParams) = {decide_kernel<SDD_BF16, false>, decide_kernel<SDD_F32, false>,
-                                           decide_kernel<SDD_BF16, true>, decide_kernel<SDD_F32, true>};
+                                           decide_kernel<SDD_BF16, true>, decide_kernel<SDD_F32, true>,
+                                           decide_kernel<SDD_BF16, false, true>, decide_kernel<SDD_F32, false, true>};
     for (auto k : kernels) {
         const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
         if (e != cudaSuccess) return e;
@@ -974,8 +977,10 @@ cudaError_t launch_decide(const ScanParams &p, cudaStream_t stream) {
     const int nseg = draw ? p.dec.nseg : 1;
     const size_t smem = draw ? static_cast<size_t>(nseg) * kDecThreads * sizeof(float) : 0;
     const bool bf = p.dtype == SDD_BF16, feat = p.feat != nullptr;
-    void (*const k)(ScanParams) = feat ? (bf ? decide_kernel<SDD_BF16, true> : decide_kernel<SDD_F32, true>)
-                                       : (bf ? decide_kernel<SDD_BF16, false> : decide_kernel<SDD_F32, false>);
+    void (*const k)(ScanParams) = (p.shard != nullptr)
+                                      ? (bf ? decide_kernel<SDD_BF16, false, true> : decide_kernel<SDD_F32, false, true>)
+                                  : feat ? (bf ? decide_kernel<SDD_BF16, true> : decide_kernel<SDD_F32, true>)
+                                         : (bf ? decide_kernel<SDD_BF16, false> : decide_kernel<SDD_F32, false>);
     return launch_dependent(k, dim3(nb, nseg),
                             dim3(kDecThreads), smem, stream, p);
 }

@@ -57,44 +57,6 @@ __device__ __forceinline__ const char *row_base(const ScanParams &p, const PartV
     return G.base + (static_cast<int64_t>(b) * G.npos + j) * G.stride_bytes;
 }
 
-// Entries of one 16-byte vector past the end of the row become -inf.
-template <int DT>
-__device__ __forceinline__ void mask_tail(uint4 &w, int valid) {
-    uint32_t *u = reinterpret_cast<uint32_t *>(&w);
-    if (DT == SDD_BF16) {
-#pragma unroll
-        for (int e = 0; e < 8; ++e)
-            if (e >= valid) {
-                const uint32_t sh = (e & 1) ? 16u : 0u;
-                u[e >> 1] = (u[e >> 1] & ~(0xFFFFu << sh)) | (0xFF80u << sh);
-            }
-    } else {
-#pragma unroll
-        for (int e = 0; e < 4; ++e)
-            if (e >= valid) u[e] = 0xFF800000u;
-    }
-}
-
-template <int DT>
-__device__ __forceinline__ float vec_elem(const uint4 &w, int e) {
-    const uint32_t *u = reinterpret_cast<const uint32_t *>(&w);
-    if (DT == SDD_BF16) return (e & 1) ? bf16_hi(u[e >> 1]) : bf16_lo(u[e >> 1]);
-    return __uint_as_float(u[e]);
-}
-
-// Clamp one vector from below (NaN-propagating).
-template <int DT>
-__device__ __forceinline__ uint4 clamp_vec(uint4 w) {
-    uint32_t *u = reinterpret_cast<uint32_t *>(&w);
-    if (DT == SDD_BF16) {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) u[q] = bf16x2_max_nan(u[q], kClampPairBf16);
-    } else {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) u[q] = __float_as_uint(fmax_nan(__uint_as_float(u[q]), clamp_floor()));
-    }
-    return w;
-}
 
 // A tile that is not full, or that ends a row whose length is not a whole
 // number of vectors, is completed in shared memory with -inf entries so that
@@ -281,29 +243,43 @@ __device__ __forceinline__ float process_tile(const uint4 *tile, int k0, int lan
     if (ENT) {
         // A tile dominated by one term (the others sum to < 1/16 of it: the
         // lane holding the peak of a peaked row) loses those others' low bits
-        // next to it, and they make the row's entropy.  The lane re-sums them
-        // among themselves from shared memory (rare: about one lane-tile per
-        // peaked row).
-        const float ycm = fmaf(cm, kLog2e, nr);
-        const float ecm = ex2(ycm);
-        if (s0 + s1 < 1.0625f * ecm && cm > clamp_floor()) {
+        // next to it, and they make the row's entropy.  Such a lane's terms
+        // are re-summed by the whole warp -- the maximum counted apart, the
+        // others summed among themselves -- from shared memory (rare: about
+        // one lane-tile per peaked row).
+        const float ecm = ex2(fmaf(cm, kLog2e, nr));
+        unsigned dom = __ballot_sync(0xFFFFFFFFu, s0 + s1 < 1.0625f * ecm && cm > clamp_floor());
+        while (dom) {
+            const int src = __ffs(dom) - 1;
+            dom &= dom - 1;
+            // src's tile maximum and reference (every lane has its own)
+            const float cms = __shfl_sync(0xFFFFFFFFu, cm, src);
+            const float nrs = __shfl_sync(0xFFFFFFFFu, nr, src);
+            // src's 8 vectors, 8 bf16 (or 4 fp32) entries each: lane l takes
+            // entries l and l + 32 of them
+            constexpr int EN = kVPL * 2 * PAIRS;   // entries of one lane-tile
             float small = 0.f, nmax = 0.f;
-#pragma unroll 1
-            for (int i = 0; i < kVPL; ++i) {
-                const uint4 w = clamp_vec<DT>(tile[lane + 32 * i]);
-                const uint32_t *u = reinterpret_cast<const uint32_t *>(&w);
 #pragma unroll
-                for (int k = 0; k < 2 * PAIRS; ++k) {
-                    const float z = (DT == SDD_BF16) ? ((k & 1) ? bf16_hi(u[k >> 1]) : bf16_lo(u[k >> 1]))
-                                                     : __uint_as_float(u[k]);
-                    if (z == cm)
-                        nmax += 1.f;
-                    else
-                        small += ex2(fmaf(z, kLog2e, nr));
-                }
+            for (int t = lane; t < EN; t += 32) {
+                const int i = t / (2 * PAIRS), k = t % (2 * PAIRS);
+                const uint4 w = clamp_vec<DT>(tile[src + 32 * i]);
+                const int wi = (DT == SDD_BF16) ? (k >> 1) : k;   // (word picked by selects, not by index)
+                const uint32_t uw = (wi < 2) ? ((wi == 0) ? w.x : w.y) : ((wi == 2) ? w.z : w.w);
+                const float z = (DT == SDD_BF16) ? ((k & 1) ? bf16_hi(uw) : bf16_lo(uw)) : __uint_as_float(uw);
+                if (z == cms)
+                    nmax += 1.f;
+                else
+                    small += ex2(fmaf(z, kLog2e, nrs));
             }
-            s0 = nmax * ecm;   // (nmax <= 64: exact)
-            s1 = small;
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) {
+                small += __shfl_xor_sync(0xFFFFFFFFu, small, off);
+                nmax += __shfl_xor_sync(0xFFFFFFFFu, nmax, off);
+            }
+            if (lane == src) {
+                s0 = nmax * ecm;   // (nmax <= 64: exact)
+                s1 = small;
+            }
         }
     }
     float e1, e2, h;

@@ -49,6 +49,38 @@ __device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
     return v;
 }
 
+// The rare paths of the per-element work, kept out of line so that the
+// common path is not compiled into predicated copies of them.
+//
+// The first index (ascending) of the value m in one vector whose entries
+// start at index idx0; m is one of them.
+template <int DT>
+__device__ __noinline__ int vector_first_index(uint4 w, int idx0, float m) {
+    constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
+    for (int e = 0; e < EPV; ++e)
+        if (vec_elem_sel<DT>(w, e) == m) return idx0 + e;
+    return INT32_MAX;
+}
+
+struct CandList {
+    int n;       // keys held (at most kl)
+    float thr;   // value of the last key once the list is full, else -inf
+};
+
+// One key into a thread's candidate list (keys descending, kl long, entry k
+// at ck[k * kShardThreads]), inserted from the tail.
+__device__ __noinline__ CandList cand_insert_key(uint64_t *ck, uint64_t key, int kl, CandList c) {
+    int k = min(c.n, kl - 1);   // the slot it takes, moved up past smaller keys
+    while (k > 0 && ck[(k - 1) * kShardThreads] < key) {
+        ck[k * kShardThreads] = ck[(k - 1) * kShardThreads];
+        --k;
+    }
+    ck[k * kShardThreads] = key;
+    c.n = min(c.n + 1, kl);
+    if (c.n == kl) c.thr = cand_value(ck[(kl - 1) * kShardThreads]);
+    return c;
+}
+
 template <int DT, bool CAND>
 __global__ void __launch_bounds__(kShardThreads) shard_partials_kernel(const __grid_constant__ ShardParams sp) {
     constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
@@ -76,58 +108,61 @@ __global__ void __launch_bounds__(kShardThreads) shard_partials_kernel(const __g
     const bool cand = CAND && !drafter;
 
     SoftState st = soft_identity();
-    float mr = clamp_floor();   // running maximum (first index in amax)
     bool nan = false;
     float s_hi = 0.f, s_lo = 0.f;
-    uint64_t ck[SDD_SHARD_KMAX];
-#pragma unroll
-    for (int k = 0; k < SDD_SHARD_KMAX; ++k) ck[k] = 0ull;
+    // target rows: the thread's kcap highest-ranked vectors, ranked by their
+    // maximum (larger first, then lower vector index), keys in descending order
+    // in shared memory, inserted from the tail.  The kcap largest entries of
+    // the slice lie in the slice's kcap highest-ranked vectors (an entry
+    // outside them has kcap vectors ranked above its own, each holding an
+    // entry that ranks before it), so the CTA selects those vectors at the end
+    // and takes the kcap largest of their entries.
+    __shared__ uint64_t s_ck[SDD_SHARD_KMAX][kShardThreads];
+    uint64_t *ck = &s_ck[0][tid];   // entry k at ck[k * kShardThreads]
+    const int kl = cand ? sp.kcap : 0;   // list length
+    CandList cl{0, -INFINITY};
+    constexpr int PAIRS = EPV / 2;
+    const f2_t L2 = f2_pack(kLog2e, kLog2e);
 
     for (int v0 = tid; v0 < sp.RVs; v0 += kShardThreads * kShardU) {
         uint4 w[kShardU];
+        float vm[kShardU];   // each vector's maximum (floored; NaN kept)
 #pragma unroll
         for (int u = 0; u < kShardU; ++u) {
             const int vec = v0 + u * kShardThreads;
-            w[u] = (vec < sp.RVs) ? __ldcs(reinterpret_cast<const uint4 *>(row) + vec) : make_uint4(0, 0, 0, 0);
+            if (vec < sp.RVs) {
+                w[u] = __ldcs(reinterpret_cast<const uint4 *>(row) + vec);
+            } else {
+                const uint32_t ni = (DT == SDD_BF16) ? kNegInfPairBf16 : 0xFF800000u;
+                w[u] = make_uint4(ni, ni, ni, ni);
+            }
         }
-        // the chunk's entries (floored; NaN kept), its maximum and first index
-        float z[kShardU * EPV];
-        bool ok[kShardU * EPV];
         float cm = clamp_floor();
 #pragma unroll
         for (int u = 0; u < kShardU; ++u) {
             const int vec = v0 + u * kShardThreads;
+            if (vec < sp.RVs && (vec + 1) * EPV > sp.Vs) mask_tail<DT>(w[u], sp.Vs - vec * EPV);
+            w[u] = clamp_vec<DT>(w[u]);   // entries past the slice and masked ones: the floor
             const uint32_t *q = reinterpret_cast<const uint32_t *>(&w[u]);
-#pragma unroll
-            for (int e = 0; e < EPV; ++e) {
-                const int i = u * EPV + e;
-                const int idx = vec * EPV + e;
-                ok[i] = vec < sp.RVs && idx < sp.Vs;
-                float x = (DT == SDD_BF16) ? ((e & 1) ? bf16_hi(q[e >> 1]) : bf16_lo(q[e >> 1])) : __uint_as_float(q[e]);
-                x = fmax_nan(x, clamp_floor());
-                z[i] = x;
-                if (ok[i]) {
-                    nan |= isnan(x);
-                    cm = fmax_nan(cm, x);
-                    if (x > mr) {
-                        mr = x;
-                        st.amax = idx;
-                    }
-                    if (cand && !isnan(x)) {
-                        uint64_t key = cand_key(x, sp.v0 + idx);
-                        if (key > ck[SDD_SHARD_KMAX - 1]) {
-#pragma unroll
-                            for (int k = 0; k < SDD_SHARD_KMAX; ++k) {
-                                const uint64_t a = ck[k];
-                                ck[k] = (key > a) ? key : a;
-                                key = (key > a) ? a : key;
-                            }
-                        }
-                    }
-                }
+            if (DT == SDD_BF16) {
+                const uint32_t m2 = bf16x2_max_nan(bf16x2_max_nan(q[0], q[1]), bf16x2_max_nan(q[2], q[3]));
+                vm[u] = fmax_nan(bf16_lo(m2), bf16_hi(m2));
+            } else {
+                vm[u] = fmax_nan(fmax_nan(__uint_as_float(q[0]), __uint_as_float(q[1])),
+                                 fmax_nan(__uint_as_float(q[2]), __uint_as_float(q[3])));
             }
+            cm = fmax_nan(cm, vm[u]);
         }
+        nan |= isnan(cm);
         if (cm > st.m) {
+            // a new maximum (rare): its first index, in the first vector that holds it
+            int us = kShardU - 1;
+#pragma unroll
+            for (int u = kShardU - 2; u >= 0; --u) us = (vm[u] == cm) ? u : us;
+            uint4 ws = w[kShardU - 1];
+#pragma unroll
+            for (int u = kShardU - 2; u >= 0; --u) ws = (u == us) ? w[u] : ws;
+            st.amax = vector_first_index<DT>(ws, (v0 + us * kShardThreads) * EPV, cm);
             // t2 against the maximum (as in the streaming kernel)
             if (drafter) st.t2 = fmaf((st.m - cm) * kLog2e, s_hi + s_lo, st.t2);
             st.m = cm;
@@ -141,25 +176,50 @@ __global__ void __launch_bounds__(kShardThreads) shard_partials_kernel(const __g
                 st.r = rn;
             }
         }
-        const float nr = -st.r;
-        const float dm = fmaf(st.m, kLog2e, nr);
-        float sa = 0.f, ca = 0.f, ta = 0.f;   // compensated (Kahan) exp-sum
+        if (cand) {
 #pragma unroll
-        for (int i = 0; i < kShardU * EPV; ++i) {
-            if (ok[i]) {
-                const float y = fmaf(z[i], kLog2e, nr);
-                const float e = ex2(y);
-                const float yk = e - ca, t = sa + yk;
-                ca = (t - sa) - yk;
-                sa = t;
-                if (drafter) ta = fmaf(e, y - dm, ta);
+            for (int u = 0; u < kShardU; ++u) {
+                const int vec = v0 + u * kShardThreads;
+                // (a vector tying the last key comes later: it ranks after it)
+                if (vm[u] > cl.thr && vec < sp.RVs) cl = cand_insert_key(ck, cand_key(vm[u], vec), kl, cl);
             }
         }
-        float h, e1;
-        two_sum(s_hi, sa, h, e1);
-        s_hi = h;
-        s_lo += e1 - ca;
-        st.t2 += ta;
+        // the exp-sums, two entries at a time (drafter rows: compensated, so
+        // that the small terms of a peaked row survive next to its peak)
+        const float nr = -st.r;
+        const f2_t NR = f2_pack(nr, nr);
+        const float dm = fmaf(st.m, kLog2e, nr);
+        const f2_t DM = f2_pack(dm, dm);
+        f2_t sa = f2_pack(0.f, 0.f), ca = sa, ta = sa;
+#pragma unroll
+        for (int u = 0; u < kShardU; ++u) {
+            const uint32_t *q = reinterpret_cast<const uint32_t *>(&w[u]);
+#pragma unroll
+            for (int h = 0; h < PAIRS; ++h) {
+                const f2_t z = (DT == SDD_BF16) ? f2_pack(bf16_lo(q[h]), bf16_hi(q[h]))
+                                                : f2_pack(__uint_as_float(q[2 * h]), __uint_as_float(q[2 * h + 1]));
+                const f2_t y = f2_fma(z, L2, NR);
+                float y0, y1;
+                f2_unpack(y, y0, y1);
+                const f2_t e = f2_pack(ex2(y0), ex2(y1));
+                if (drafter) {
+                    const f2_t yk = f2_sub(e, ca), t = f2_add(sa, yk);
+                    ca = f2_sub(f2_sub(t, sa), yk);
+                    sa = t;
+                    ta = f2_fma(e, f2_sub(y, DM), ta);
+                } else {
+                    sa = f2_add(sa, e);
+                }
+            }
+        }
+        float a0, a1, c0, c1, t0, t1, h, e1, e2;
+        f2_unpack(sa, a0, a1);
+        f2_unpack(ca, c0, c1);
+        f2_unpack(ta, t0, t1);
+        two_sum(s_hi, a0, h, e1);
+        two_sum(h, a1, s_hi, e2);
+        s_lo += (e1 + e2) - (c0 + c1);
+        st.t2 += t0 + t1;
     }
     if (nan) st.m = qnan();
     st.sh = s_hi;
@@ -171,27 +231,61 @@ __global__ void __launch_bounds__(kShardThreads) shard_partials_kernel(const __g
     const SoftState wst = soft_warp_reduce(st);
     if (lane == 0) s_st[warp] = wst;
 
-    // the slice's kcap largest entries: kcap rounds of a CTA-wide maximum of
-    // the threads' list heads, the winner popping its head
+    // the slice's kcap highest-ranked vectors: kcap rounds of a CTA-wide
+    // maximum of the threads' list heads, the winner popping its head; then
+    // the kcap largest entries of those vectors (one warp, kcap rounds)
     __shared__ uint64_t s_wmax[NW];
     __shared__ uint64_t s_top[SDD_SHARD_KMAX];
+    __shared__ uint64_t s_ent[SDD_SHARD_KMAX * 8];
     const int kc = cand ? sp.kcap : 0;
+    int head = 0;   // the thread's next unselected key
     for (int round = 0; round < kc; ++round) {
-        const uint64_t m = warp_max_u64(ck[0]);
+        const uint64_t mine = (head < cl.n) ? ck[head * kShardThreads] : 0ull;
+        const uint64_t m = warp_max_u64(mine);
         if (lane == 0) s_wmax[warp] = m;
         __syncthreads();
         uint64_t best = 0ull;
 #pragma unroll
         for (int q = 0; q < NW; ++q) best = (s_wmax[q] > best) ? s_wmax[q] : best;
         if (tid == 0) s_top[round] = best;
-        if (best != 0ull && ck[0] == best) {   // keys are unique: one thread pops
-#pragma unroll
-            for (int k = 0; k + 1 < SDD_SHARD_KMAX; ++k) ck[k] = ck[k + 1];
-            ck[SDD_SHARD_KMAX - 1] = 0ull;
-        }
+        if (best != 0ull && mine == best) ++head;   // keys are unique: one thread pops
         __syncthreads();
     }
-    __syncthreads();
+    if (kc > 0) {
+        // the entries of the selected vectors (re-read: kc x 16 bytes), keyed by value and global index
+        if (tid < kc) {
+            const uint64_t vk = s_top[tid];
+            uint4 wv = make_uint4(0, 0, 0, 0);
+            const int vec = (vk != 0ull) ? cand_index(vk) : -1;
+            if (vec >= 0) wv = clamp_vec<DT>(__ldg(reinterpret_cast<const uint4 *>(row) + vec));
+#pragma unroll
+            for (int e = 0; e < EPV; ++e) {
+                const int idx = vec * EPV + e;
+                const float x = vec_elem<DT>(wv, e);
+                s_ent[tid * 8 + e] = (vec >= 0 && idx < sp.Vs && !isnan(x)) ? cand_key(x, sp.v0 + idx) : 0ull;
+            }
+#pragma unroll
+            for (int e = EPV; e < 8; ++e) s_ent[tid * 8 + e] = 0ull;
+        }
+        __syncthreads();
+        if (warp == 0) {
+            const int n = kc * 8;
+            for (int round = 0; round < kc; ++round) {
+                uint64_t mine = 0ull;
+                int at = -1;
+                for (int t = lane; t < n; t += 32)
+                    if (s_ent[t] > mine) {
+                        mine = s_ent[t];
+                        at = t;
+                    }
+                const uint64_t best = warp_max_u64(mine);
+                if (best != 0ull && mine == best) s_ent[at] = 0ull;   // unique keys: one lane takes it
+                if (lane == 0) s_top[round] = best;
+                __syncwarp();
+            }
+        }
+    }
+    __syncthreads();   // (every warp's state in s_st; the selection done)
 
     if (tid == 0) {
         SoftState a = s_st[0];
