@@ -746,6 +746,7 @@ def run_component_shard(args):
     # one slice's partials kernel, back to back
     r0 = ranks[0]
     a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda._sleep(int(2000 * 2.0e3))   # ~2 ms: the 50 launches queue behind it, no host gaps
     a0.record()
     for _ in range(50):
         r0.partials()

@@ -6,11 +6,12 @@
 //    streams its 16-byte vectors (ascending), keeping the online-softmax state
 //    of its entries relative to an integer reference in log2 units (a new
 //    maximum rescales the sums by an exact power of two), the first index of
-//    its maximum, the drafter entropy accumulator, and -- target rows of a
-//    round with the top-k rule -- its SDD_SHARD_KMAX largest entries.  The CTA
-//    merges the threads' states in thread order and selects the slice's kcap
-//    largest entries (value descending, index ascending), then one thread
-//    writes the row's record.  Logits are floored at -2^23 as in the
+//    its maximum and the drafter entropy accumulator; on target rows of a
+//    round with the top-k rule each warp keeps its kcap highest-ranked
+//    vectors in a list held one key per lane.  The CTA merges the threads'
+//    states in thread order and selects the slice's kcap largest entries
+//    (value descending, index ascending), then one thread writes the row's
+//    record.  Logits are floored at -2^23 as in the
 //    streaming kernel; entries past the slice width weigh nothing.
 //
 // The records of all slices are merged, and every rule of the round runs, in
@@ -22,7 +23,11 @@ namespace sdd {
 
 namespace {
 
-constexpr int kShardThreads = 256;
+// One CTA of four warps per row and eight CTAs per SM (64 registers): a c3
+// slice holds 1,040 rows, one wave on 152 SMs.  (256 threads at 4 CTAs per
+// SM: 84 us per half-vocabulary slice, against 58 us.)
+constexpr int kShardThreads = 128;
+constexpr int kShardMinCtas = 8;
 constexpr int kShardU = 4;   // 16-byte vectors per thread in flight
 
 // Order key of a candidate: larger value first, then lower index (an
@@ -62,27 +67,172 @@ __device__ __noinline__ int vector_first_index(uint4 w, int idx0, float m) {
     return INT32_MAX;
 }
 
-struct CandList {
-    int n;       // keys held (at most kl)
-    float thr;   // value of the last key once the list is full, else -inf
+// One key into a warp's candidate list: lane k < kl holds the list's k-th
+// key (descending; 0 = empty), every lane returns its new entry.
+__device__ __forceinline__ uint64_t warp_list_insert(uint64_t lk, uint64_t key, int kl, int lane) {
+    const int pos = __popc(__ballot_sync(0xFFFFFFFFu, lk > key));   // keys ranking before it
+    const uint64_t up = __shfl_up_sync(0xFFFFFFFFu, lk, 1);
+    if (lane < kl && lane > pos) return up;
+    if (lane < kl && lane == pos) return key;
+    return lk;
+}
+
+// The running state of one thread's entries of a row.
+struct ShardAcc {
+    SoftState st;
+    float s_hi, s_lo;   // exp-sum relative to 2^r, as an unevaluated pair
+    bool nan;
+    uint64_t lk;        // candidate rows: this lane's entry of the warp's list
+    float wthr;         // value of the list's last key once full, else -inf
 };
 
-// One key into a thread's candidate list (keys descending, kl long, entry k
-// at ck[k * kShardThreads]), inserted from the tail.
-__device__ __noinline__ CandList cand_insert_key(uint64_t *ck, uint64_t key, int kl, CandList c) {
-    int k = min(c.n, kl - 1);   // the slot it takes, moved up past smaller keys
-    while (k > 0 && ck[(k - 1) * kShardThreads] < key) {
-        ck[k * kShardThreads] = ck[(k - 1) * kShardThreads];
-        --k;
+// One chunk (kShardU vectors per lane, lane-contiguous) of a row.  DRAFT: a
+// drafter row (entropy accumulator, compensated sums); CANDL: a target row
+// of a round with the top-k rule (the warp's candidate list); FULL: every
+// vector of the warp's chunk lies inside the slice and before a ragged last
+// vector (no guards).  Warp-uniform: every lane of the warp runs the same
+// chunk, lanes past the end on floored -inf vectors that weigh nothing.
+template <int DT, bool DRAFT, bool CANDL, bool FULL>
+__device__ __forceinline__ void shard_chunk(const char *row, const ShardParams &sp, int v0, int kl, int lane,
+                                            ShardAcc &a) {
+    constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
+    constexpr int PAIRS = EPV / 2;
+    uint4 w[kShardU];
+    float vm[kShardU];   // each vector's maximum (floored; NaN kept)
+#pragma unroll
+    for (int u = 0; u < kShardU; ++u) {
+        const int vec = v0 + u * kShardThreads;
+        if (FULL || vec < sp.RVs) {
+            w[u] = __ldcs(reinterpret_cast<const uint4 *>(row) + vec);
+        } else {
+            const uint32_t ni = (DT == SDD_BF16) ? kNegInfPairBf16 : 0xFF800000u;
+            w[u] = make_uint4(ni, ni, ni, ni);
+        }
     }
-    ck[k * kShardThreads] = key;
-    c.n = min(c.n + 1, kl);
-    if (c.n == kl) c.thr = cand_value(ck[(kl - 1) * kShardThreads]);
-    return c;
+    float cm = clamp_floor();
+#pragma unroll
+    for (int u = 0; u < kShardU; ++u) {
+        const int vec = v0 + u * kShardThreads;
+        if (!FULL && vec < sp.RVs && (vec + 1) * EPV > sp.Vs) mask_tail<DT>(w[u], sp.Vs - vec * EPV);
+        w[u] = clamp_vec<DT>(w[u]);   // entries past the slice and masked ones: the floor
+        const uint32_t *q = reinterpret_cast<const uint32_t *>(&w[u]);
+        if (DT == SDD_BF16) {
+            const uint32_t m2 = bf16x2_max_nan(bf16x2_max_nan(q[0], q[1]), bf16x2_max_nan(q[2], q[3]));
+            vm[u] = fmax_nan(bf16_lo(m2), bf16_hi(m2));
+        } else {
+            vm[u] = fmax_nan(fmax_nan(__uint_as_float(q[0]), __uint_as_float(q[1])),
+                             fmax_nan(__uint_as_float(q[2]), __uint_as_float(q[3])));
+        }
+        cm = fmax_nan(cm, vm[u]);
+    }
+    a.nan |= isnan(cm);
+    if (cm > a.st.m) {
+        // a new maximum (rare): its first index, in the first vector that holds it
+        int us = kShardU - 1;
+#pragma unroll
+        for (int u = kShardU - 2; u >= 0; --u) us = (vm[u] == cm) ? u : us;
+        uint4 ws = w[kShardU - 1];
+#pragma unroll
+        for (int u = kShardU - 2; u >= 0; --u) ws = (u == us) ? w[u] : ws;
+        a.st.amax = vector_first_index<DT>(ws, (v0 + us * kShardThreads) * EPV, cm);
+        // t2 against the maximum (as in the streaming kernel)
+        if (DRAFT) a.st.t2 = fmaf((a.st.m - cm) * kLog2e, a.s_hi + a.s_lo, a.st.t2);
+        a.st.m = cm;
+        const float rn = ceilf(cm * kLog2e);
+        if (rn > a.st.r) {
+            const float sc = pow2f_int(a.st.r - rn);   // exact power of two (0 below the normal range)
+            if (DRAFT) a.st.t2 *= sc;
+            a.s_hi *= sc;
+            a.s_lo *= sc;
+            a.st.r = rn;
+        }
+    }
+    if (CANDL) {
+#pragma unroll
+        for (int u = 0; u < kShardU; ++u) {
+            const int vec = v0 + u * kShardThreads;
+            // (a vector tying the last key has a larger index: it ranks after it)
+            unsigned pend = __ballot_sync(0xFFFFFFFFu, vm[u] > a.wthr && (FULL || vec < sp.RVs));
+            if (pend) {
+                const uint64_t mine = cand_key(vm[u], vec);
+                while (pend) {
+                    const int src = __ffs(pend) - 1;
+                    pend &= pend - 1;
+                    a.lk = warp_list_insert(a.lk, __shfl_sync(0xFFFFFFFFu, mine, src), kl, lane);
+                }
+                const uint64_t last = __shfl_sync(0xFFFFFFFFu, a.lk, kl - 1);
+                a.wthr = (last != 0ull) ? cand_value(last) : -INFINITY;
+            }
+        }
+    }
+    // the exp-sums, two entries at a time (drafter rows: compensated, so
+    // that the small terms of a peaked row survive next to its peak)
+    const f2_t L2 = f2_pack(kLog2e, kLog2e);
+    const float nr = -a.st.r;
+    const f2_t NR = f2_pack(nr, nr);
+    const float dm = fmaf(a.st.m, kLog2e, nr);
+    const f2_t DM = f2_pack(dm, dm);
+    f2_t sa = f2_pack(0.f, 0.f), ca = sa, ta = sa;
+#pragma unroll
+    for (int u = 0; u < kShardU; ++u) {
+        const uint32_t *q = reinterpret_cast<const uint32_t *>(&w[u]);
+#pragma unroll
+        for (int h = 0; h < PAIRS; ++h) {
+            const f2_t z = (DT == SDD_BF16) ? f2_pack(bf16_lo(q[h]), bf16_hi(q[h]))
+                                            : f2_pack(__uint_as_float(q[2 * h]), __uint_as_float(q[2 * h + 1]));
+            const f2_t y = f2_fma(z, L2, NR);
+            float y0, y1;
+            f2_unpack(y, y0, y1);
+            const f2_t e = f2_pack(ex2(y0), ex2(y1));
+            if (DRAFT) {
+                const f2_t yk = f2_sub(e, ca), t = f2_add(sa, yk);
+                ca = f2_sub(f2_sub(t, sa), yk);
+                sa = t;
+                ta = f2_fma(e, f2_sub(y, DM), ta);
+            } else {
+                sa = f2_add(sa, e);
+            }
+        }
+    }
+    float a0, a1, h, e1, e2;
+    f2_unpack(sa, a0, a1);
+    two_sum(a.s_hi, a0, h, e1);
+    two_sum(h, a1, a.s_hi, e2);
+    if (DRAFT) {
+        float c0, c1, t0, t1;
+        f2_unpack(ca, c0, c1);
+        f2_unpack(ta, t0, t1);
+        a.s_lo += (e1 + e2) - (c0 + c1);
+        a.st.t2 += t0 + t1;
+    } else {
+        a.s_lo += e1 + e2;
+    }
+}
+
+// A thread's part of a row: chunks v0 = tid + c * kShardThreads * kShardU,
+// run while the warp's first lane is inside the row.
+template <int DT, bool DRAFT, bool CANDL>
+__device__ __forceinline__ ShardAcc shard_row(const char *row, const ShardParams &sp, int kl, int tid) {
+    constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
+    const int lane = tid & 31;
+    ShardAcc a;
+    a.st = soft_identity();
+    a.s_hi = a.s_lo = 0.f;
+    a.nan = false;
+    a.lk = 0ull;
+    a.wthr = -INFINITY;
+    const int rvf = (sp.Vs % EPV == 0) ? sp.RVs : sp.RVs - 1;   // vectors wholly inside the slice
+    for (int v0 = tid; v0 - lane < sp.RVs; v0 += kShardThreads * kShardU) {
+        if ((v0 - lane) + 31 + (kShardU - 1) * kShardThreads < rvf)
+            shard_chunk<DT, DRAFT, CANDL, true>(row, sp, v0, kl, lane, a);
+        else
+            shard_chunk<DT, DRAFT, CANDL, false>(row, sp, v0, kl, lane, a);
+    }
+    return a;
 }
 
 template <int DT, bool CAND>
-__global__ void __launch_bounds__(kShardThreads) shard_partials_kernel(const __grid_constant__ ShardParams sp) {
+__global__ void __launch_bounds__(kShardThreads, kShardMinCtas) shard_partials_kernel(const __grid_constant__ ShardParams sp) {
     constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
     constexpr int NW = kShardThreads / 32;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -107,120 +257,21 @@ __global__ void __launch_bounds__(kShardThreads) shard_partials_kernel(const __g
     const bool in_slice = has_tok && !tok_out && tok >= sp.v0 && tok < sp.v0 + sp.Vs;
     const bool cand = CAND && !drafter;
 
-    SoftState st = soft_identity();
-    bool nan = false;
-    float s_hi = 0.f, s_lo = 0.f;
-    // target rows: the thread's kcap highest-ranked vectors, ranked by their
-    // maximum (larger first, then lower vector index), keys in descending order
-    // in shared memory, inserted from the tail.  The kcap largest entries of
-    // the slice lie in the slice's kcap highest-ranked vectors (an entry
-    // outside them has kcap vectors ranked above its own, each holding an
-    // entry that ranks before it), so the CTA selects those vectors at the end
-    // and takes the kcap largest of their entries.
-    __shared__ uint64_t s_ck[SDD_SHARD_KMAX][kShardThreads];
-    uint64_t *ck = &s_ck[0][tid];   // entry k at ck[k * kShardThreads]
+    // target rows: the warp's kcap highest-ranked vectors, ranked by their
+    // maximum (larger first, then lower vector index), held one key per lane
+    // in descending order.  The kcap largest entries of the slice lie in the
+    // slice's kcap highest-ranked vectors (an entry outside them has kcap
+    // vectors ranked above its own, each holding an entry that ranks before
+    // it), so the CTA selects those vectors at the end and takes the kcap
+    // largest of their entries.
     const int kl = cand ? sp.kcap : 0;   // list length
-    CandList cl{0, -INFINITY};
-    constexpr int PAIRS = EPV / 2;
-    const f2_t L2 = f2_pack(kLog2e, kLog2e);
-
-    for (int v0 = tid; v0 < sp.RVs; v0 += kShardThreads * kShardU) {
-        uint4 w[kShardU];
-        float vm[kShardU];   // each vector's maximum (floored; NaN kept)
-#pragma unroll
-        for (int u = 0; u < kShardU; ++u) {
-            const int vec = v0 + u * kShardThreads;
-            if (vec < sp.RVs) {
-                w[u] = __ldcs(reinterpret_cast<const uint4 *>(row) + vec);
-            } else {
-                const uint32_t ni = (DT == SDD_BF16) ? kNegInfPairBf16 : 0xFF800000u;
-                w[u] = make_uint4(ni, ni, ni, ni);
-            }
-        }
-        float cm = clamp_floor();
-#pragma unroll
-        for (int u = 0; u < kShardU; ++u) {
-            const int vec = v0 + u * kShardThreads;
-            if (vec < sp.RVs && (vec + 1) * EPV > sp.Vs) mask_tail<DT>(w[u], sp.Vs - vec * EPV);
-            w[u] = clamp_vec<DT>(w[u]);   // entries past the slice and masked ones: the floor
-            const uint32_t *q = reinterpret_cast<const uint32_t *>(&w[u]);
-            if (DT == SDD_BF16) {
-                const uint32_t m2 = bf16x2_max_nan(bf16x2_max_nan(q[0], q[1]), bf16x2_max_nan(q[2], q[3]));
-                vm[u] = fmax_nan(bf16_lo(m2), bf16_hi(m2));
-            } else {
-                vm[u] = fmax_nan(fmax_nan(__uint_as_float(q[0]), __uint_as_float(q[1])),
-                                 fmax_nan(__uint_as_float(q[2]), __uint_as_float(q[3])));
-            }
-            cm = fmax_nan(cm, vm[u]);
-        }
-        nan |= isnan(cm);
-        if (cm > st.m) {
-            // a new maximum (rare): its first index, in the first vector that holds it
-            int us = kShardU - 1;
-#pragma unroll
-            for (int u = kShardU - 2; u >= 0; --u) us = (vm[u] == cm) ? u : us;
-            uint4 ws = w[kShardU - 1];
-#pragma unroll
-            for (int u = kShardU - 2; u >= 0; --u) ws = (u == us) ? w[u] : ws;
-            st.amax = vector_first_index<DT>(ws, (v0 + us * kShardThreads) * EPV, cm);
-            // t2 against the maximum (as in the streaming kernel)
-            if (drafter) st.t2 = fmaf((st.m - cm) * kLog2e, s_hi + s_lo, st.t2);
-            st.m = cm;
-            const float rn = ceilf(cm * kLog2e);
-            if (rn > st.r) {
-                const float k = st.r - rn;
-                const float sc = pow2f_int(k);   // exact power of two (0 below the normal range)
-                if (drafter) st.t2 *= sc;
-                s_hi *= sc;
-                s_lo *= sc;
-                st.r = rn;
-            }
-        }
-        if (cand) {
-#pragma unroll
-            for (int u = 0; u < kShardU; ++u) {
-                const int vec = v0 + u * kShardThreads;
-                // (a vector tying the last key comes later: it ranks after it)
-                if (vm[u] > cl.thr && vec < sp.RVs) cl = cand_insert_key(ck, cand_key(vm[u], vec), kl, cl);
-            }
-        }
-        // the exp-sums, two entries at a time (drafter rows: compensated, so
-        // that the small terms of a peaked row survive next to its peak)
-        const float nr = -st.r;
-        const f2_t NR = f2_pack(nr, nr);
-        const float dm = fmaf(st.m, kLog2e, nr);
-        const f2_t DM = f2_pack(dm, dm);
-        f2_t sa = f2_pack(0.f, 0.f), ca = sa, ta = sa;
-#pragma unroll
-        for (int u = 0; u < kShardU; ++u) {
-            const uint32_t *q = reinterpret_cast<const uint32_t *>(&w[u]);
-#pragma unroll
-            for (int h = 0; h < PAIRS; ++h) {
-                const f2_t z = (DT == SDD_BF16) ? f2_pack(bf16_lo(q[h]), bf16_hi(q[h]))
-                                                : f2_pack(__uint_as_float(q[2 * h]), __uint_as_float(q[2 * h + 1]));
-                const f2_t y = f2_fma(z, L2, NR);
-                float y0, y1;
-                f2_unpack(y, y0, y1);
-                const f2_t e = f2_pack(ex2(y0), ex2(y1));
-                if (drafter) {
-                    const f2_t yk = f2_sub(e, ca), t = f2_add(sa, yk);
-                    ca = f2_sub(f2_sub(t, sa), yk);
-                    sa = t;
-                    ta = f2_fma(e, f2_sub(y, DM), ta);
-                } else {
-                    sa = f2_add(sa, e);
-                }
-            }
-        }
-        float a0, a1, c0, c1, t0, t1, h, e1, e2;
-        f2_unpack(sa, a0, a1);
-        f2_unpack(ca, c0, c1);
-        f2_unpack(ta, t0, t1);
-        two_sum(s_hi, a0, h, e1);
-        two_sum(h, a1, s_hi, e2);
-        s_lo += (e1 + e2) - (c0 + c1);
-        st.t2 += t0 + t1;
-    }
+    ShardAcc acc = drafter ? shard_row<DT, true, false>(row, sp, 0, tid)
+                           : (cand ? shard_row<DT, false, CAND>(row, sp, kl, tid)
+                                   : shard_row<DT, false, false>(row, sp, 0, tid));
+    SoftState st = acc.st;
+    const uint64_t lk = acc.lk;
+    const bool nan = acc.nan;
+    const float s_hi = acc.s_hi, s_lo = acc.s_lo;
     if (nan) st.m = qnan();
     st.sh = s_hi;
     st.sl = s_lo;
@@ -231,26 +282,34 @@ __global__ void __launch_bounds__(kShardThreads) shard_partials_kernel(const __g
     const SoftState wst = soft_warp_reduce(st);
     if (lane == 0) s_st[warp] = wst;
 
-    // the slice's kcap highest-ranked vectors: kcap rounds of a CTA-wide
-    // maximum of the threads' list heads, the winner popping its head; then
-    // the kcap largest entries of those vectors (one warp, kcap rounds)
-    __shared__ uint64_t s_wmax[NW];
+    // the slice's kcap highest-ranked vectors: the warps' lists in shared
+    // memory, kcap rounds of a warp maximum over them (one warp); then the
+    // kcap largest entries of those vectors (one warp, kcap rounds)
+    __shared__ uint64_t s_wl[NW * SDD_SHARD_KMAX];
     __shared__ uint64_t s_top[SDD_SHARD_KMAX];
     __shared__ uint64_t s_ent[SDD_SHARD_KMAX * 8];
     const int kc = cand ? sp.kcap : 0;
-    int head = 0;   // the thread's next unselected key
-    for (int round = 0; round < kc; ++round) {
-        const uint64_t mine = (head < cl.n) ? ck[head * kShardThreads] : 0ull;
-        const uint64_t m = warp_max_u64(mine);
-        if (lane == 0) s_wmax[warp] = m;
-        __syncthreads();
-        uint64_t best = 0ull;
+    if (lane < kc) s_wl[warp * SDD_SHARD_KMAX + lane] = lk;
+    __syncthreads();
+    if (kc > 0 && warp == 0) {
+        constexpr int PER = (NW * SDD_SHARD_KMAX + 31) / 32;
+        uint64_t mk[PER];
 #pragma unroll
-        for (int q = 0; q < NW; ++q) best = (s_wmax[q] > best) ? s_wmax[q] : best;
-        if (tid == 0) s_top[round] = best;
-        if (best != 0ull && mine == best) ++head;   // keys are unique: one thread pops
-        __syncthreads();
+        for (int t = 0; t < PER; ++t) {
+            const int i = lane + 32 * t;
+            mk[t] = (i < NW * SDD_SHARD_KMAX && (i % SDD_SHARD_KMAX) < kc) ? s_wl[i] : 0ull;
+        }
+        for (int round = 0; round < kc; ++round) {
+            uint64_t mine = 0ull;
+#pragma unroll
+            for (int t = 0; t < PER; ++t) mine = (mk[t] > mine) ? mk[t] : mine;
+            const uint64_t best = warp_max_u64(mine);
+#pragma unroll
+            for (int t = 0; t < PER; ++t) mk[t] = (best != 0ull && mk[t] == best) ? 0ull : mk[t];   // unique keys
+            if (lane == 0) s_top[round] = best;
+        }
     }
+    __syncthreads();
     if (kc > 0) {
         // the entries of the selected vectors (re-read: kc x 16 bytes), keyed by value and global index
         if (tid < kc) {
