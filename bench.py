@@ -13,7 +13,7 @@ confidence schedule at tau=0.9.  Inputs are seeded synthetic logits (no model
 weights are available); three input sets of 316 MB each rotate, so every step
 reads its logits from HBM, not L2.
 
-Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--workload c3]
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--workload c3] [--blocks B]
 Prints one JSON line (rank 0).
 
 Other rows of the path, one JSON line each (not the fused-round contract line):
@@ -56,9 +56,14 @@ def _peaks():
         return 6800.0, "fallback"
 
 
-def _workload_cfg(name):
+def _workload_cfg(name, blocks=None):
+    """A workload by name; `blocks` overrides its batch size B (a sweep of the
+    same rows over more or fewer blocks)."""
     from paper_2608_14787_gb300 import synth
     wl = synth.WORKLOADS[name]
+    if blocks is not None and blocks != wl.B:
+        wl = synth.Workload(**{**wl.__dict__, "B": blocks, "name": f"{wl.name}-B{blocks}",
+                               "description": wl.description.replace(f"B={wl.B},", f"B={blocks},")})
     ells = tuple(synth.paper_ell(e) for e in wl.ells)
     return wl, ells, tuple(wl.topks)
 
@@ -206,7 +211,7 @@ def run_reference(args):
     if rank != 0:
         return 0
     from paper_2608_14787_gb300 import synth
-    wl, ells, ks = _workload_cfg(args.workload)
+    wl, ells, ks = _workload_cfg(args.workload, args.blocks)
     nproc, model = _host_info()
     threads = max(1, min(nproc, args.ref_threads or nproc))
     host = _host_block(synth.make_block(wl, device="cpu", round_=0), wl)
@@ -366,7 +371,7 @@ def run_gpu(args):
         dist.barrier()
     sdd.load()
 
-    wl, ells, ks = _workload_cfg(args.workload)
+    wl, ells, ks = _workload_cfg(args.workload, args.blocks)
     B, gamma, V = wl.B, wl.gamma, wl.V
     n_sets = max(1, args.sets)
     sets = [synth.make_block(wl, device=dev, round_=r + 1000 * rank) for r in range(n_sets)]
@@ -387,6 +392,21 @@ def run_gpu(args):
     torch.cuda.synchronize()
     if int(rnd.status.item()) != 0:
         raise RuntimeError(f"device status {int(rnd.status.item())} after warm-up")
+    graph = None
+    if args.graph:
+        # small rounds outrun the host's launches: the timed rounds replay a
+        # CUDA graph of --graph rounds (the same launches, captured once)
+        if args.steps % args.graph:
+            raise SystemExit("--steps must be a multiple of --graph")
+        side = torch.cuda.Stream(device=dev)
+        side.wait_stream(stream)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=side):
+            for j in range(args.graph):
+                step(args.warmup + j)
+        for _ in range(2):
+            graph.replay()
+        torch.cuda.synchronize()
 
     # ---- device-resident timed region: exactly K rounds ----
     # A short device-side spin keeps the stream busy while the host enqueues
@@ -401,8 +421,12 @@ def run_gpu(args):
     with ClockSampler(bus) as clk:
         torch.cuda._sleep(int(args.prefill_us * 2.0e3))    # ~prefill_us at 2 GHz
         t_start.record(stream)
-        for i in range(args.steps):
-            step(args.warmup + i)
+        if graph is not None:
+            for _ in range(args.steps // args.graph):
+                graph.replay()
+        else:
+            for i in range(args.steps):
+                step(args.warmup + i)
         t_end.record(stream)
         torch.cuda.synchronize()
     if ws > 1:
@@ -467,7 +491,9 @@ def run_gpu(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if esz == 2 else "fp32", "data": "synthetic",
-            "config": _config_json(wl, ells, ks, n_sets),
+            "config": {**_config_json(wl, ells, ks, n_sets),
+                       "launch": (f"CUDA graph of {args.graph} rounds, replayed" if args.graph
+                                  else "one call per kernel, queued behind a device spin")},
             "achieved_gbs_step": ws * scan_bytes / (ms_per_step / 1e3) / 1e9,
             "frac_of_8tbs_step": ws * scan_bytes / (ms_per_step / 1e3) / 8e12,
             "roofline": roofline,
@@ -894,6 +920,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--workload", default="c3")
+    ap.add_argument("--blocks", type=int, default=None, help="override the workload's batch size B")
+    ap.add_argument("--graph", type=int, default=0, help="replay a CUDA graph of this many rounds (small workloads)")
     ap.add_argument("--cpu-blocks", type=int, default=8, help="blocks of the single-thread oracle sample")
     ap.add_argument("--ref-threads", type=int, default=0, help="host threads of --impl reference (0: all cores)")
     ap.add_argument("--scan-launches", type=int, default=60, help="back-to-back streaming launches for the roofline")
@@ -921,7 +949,7 @@ def main():
         return run_component_diag(args)
     if args.component == "shard":
         return run_component_shard(args)
-    if args.traffic is None and args.workload == "c3":
+    if args.traffic is None and args.workload == "c3" and args.blocks in (None, 16):
         args.traffic = SCAN_TRAFFIC_C3
     if args.warmup < 3:
         args.warmup = 3

@@ -155,7 +155,7 @@ void finish_params(ScanParams &p, const Work &w) {
     p.rows0 = static_cast<int64_t>(p.grp[0].nb) * p.grp[0].npos;
     p.rows = p.rows0 + (p.n_groups > 1 ? static_cast<int64_t>(p.grp[1].nb) * p.grp[1].npos : 0);
     p.T = p.rows * p.RV;
-    p.W = scan_warps(w.W_max, p.T);
+    p.W = scan_warps(w.W_max, p.T, p.rows);
     set_divisors(p);
 }
 

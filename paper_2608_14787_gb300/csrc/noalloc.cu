@@ -138,7 +138,7 @@ sdd_status_t sdd_confidence_noalloc(const void *draft_logits, sdd_dtype_t dtype,
     p.rows0 = rows;
     p.rows = rows;
     p.T = rows * p.RV;
-    const int64_t W = scan_warps(nd.W_max, p.T);
+    const int64_t W = scan_warps(nd.W_max, p.T, p.rows);
     p.W = static_cast<int32_t>(W);
     set_divisors(p);
     if (static_cast<double>(p.C) * static_cast<double>(W) >= 9.007199254740992e15)   // 2^53
