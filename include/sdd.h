@@ -39,7 +39,8 @@
  *   and launch failures return SDD_ERR_CUDA.  Conditions found while the
  *   kernels run are OR-ed into the caller's device word `*status` (bits
  *   SDD_DEV_*; the caller clears it); no kernel traps.  sdd_last_error()
- *   returns a message for the calling thread's last non-OK return.
+ *   returns a message for the calling thread's last non-OK return;
+ *   sdd_status_from_device() reads the device word into a return value.
  * Dtypes.  Logits are SDD_F32 or SDD_BF16; all arithmetic is fp32, with
  *   double-float (unevaluated fp32 pairs, about 48 significant bits) where sums,
  *   log-normalisers and threshold comparisons need more; fp64 results (lse) are
@@ -72,7 +73,8 @@ typedef enum {
     SDD_ERR_INVALID_ARGUMENT = 1,
     SDD_ERR_UNSUPPORTED = 2,
     SDD_ERR_CUDA = 3,
-    SDD_ERR_WORKSPACE = 4
+    SDD_ERR_WORKSPACE = 4,
+    SDD_ERR_DEVICE = 5      /* sdd_status_from_device: a device status bit was set */
 } sdd_status_t;
 
 typedef enum { SDD_F32 = 0, SDD_BF16 = 1 } sdd_dtype_t;
@@ -96,6 +98,15 @@ SDD_API int sdd_version(void);
 
 /* Message describing the calling thread's last non-OK return ("" if none). */
 SDD_API const char *sdd_last_error(void);
+
+/* The device status word `status` (int32 in device memory) of the calls
+ * enqueued on `stream` so far, read once they complete (this call
+ * synchronises the stream): *bits (host) receives its SDD_DEV_* bits.
+ * Returns SDD_OK when no bit is set, SDD_ERR_DEVICE when one is (the message
+ * of sdd_last_error() names them), SDD_ERR_CUDA if the read fails,
+ * SDD_ERR_INVALID_ARGUMENT for a NULL pointer.  clear != 0 zeroes the word
+ * after the read (stream-ordered, before this call returns). */
+SDD_API sdd_status_t sdd_status_from_device(int32_t *status, int clear, uint32_t *bits, sdd_stream_t stream);
 
 /*
  * sdd_workspace_size -- bytes of device scratch that any entry

@@ -17,6 +17,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_build", "libsdd.so")
 
 SDD_OK = 0
+SDD_ERR_DEVICE = 5
 SDD_F32 = 0
 SDD_BF16 = 1
 SIG_RAW, SIG_MARGINAL, SIG_CONDITIONAL, SIG_PERIODIC = 0, 1, 2, 3
@@ -107,6 +108,7 @@ def load(path: str | None = None):
     L.sdd_position_metrics.argtypes = [VP, VP, I, I, I, VP, VP, VP, VP, VP, VP]
     L.sdd_position_metrics.restype = I
     L.sdd_test_wait_hooks.argtypes = [ctypes.c_uint32, I]
+    L.sdd_status_from_device.argtypes = [VP, I, ctypes.POINTER(ctypes.c_uint32), VP]
     L.sdd_test_wait_hooks.restype = I
     L.sdd_select_rows.argtypes = [VP, I, VP, VP, VP]
     L.sdd_select_rows.restype = I
@@ -541,6 +543,18 @@ def test_wait_hooks(polls: int = 0, drop_copy: bool = False):
 
 
 test_wait_hooks.__test__ = False   # a library call, not a test
+
+
+def status_from_device(status: torch.Tensor, clear: bool = False, stream=None):
+    """sdd_status_from_device: the SDD_DEV_* bits of a device status word once
+    the stream's calls complete (synchronises the stream); clear=True zeroes
+    the word.  Returns (code, bits): code SDD_OK or SDD_ERR_DEVICE; raises
+    SddError when the read itself fails."""
+    bits = ctypes.c_uint32(0)
+    rc = load().sdd_status_from_device(_p(status), 1 if clear else 0, ctypes.byref(bits), _stream(stream))
+    if rc not in (SDD_OK, SDD_ERR_DEVICE):
+        _check(rc, "sdd_status_from_device")
+    return rc, int(bits.value)
 
 
 class BlockRound:

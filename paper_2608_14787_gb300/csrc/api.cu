@@ -315,6 +315,21 @@ int sdd_version(void) { return 100; }
 
 const char *sdd_last_error(void) { return g_err.c_str(); }
 
+sdd_status_t sdd_status_from_device(int32_t *status, int clear, uint32_t *bits, sdd_stream_t stream) {
+    if (!status || !bits) return fail(SDD_ERR_INVALID_ARGUMENT, "status / bits is NULL");
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    int32_t h = 0;
+    cudaError_t e = cudaMemcpyAsync(&h, status, sizeof h, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && clear) e = cudaMemsetAsync(status, 0, sizeof h, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, "device status read");
+    *bits = static_cast<uint32_t>(h);
+    if (h == 0) return SDD_OK;
+    return fail(SDD_ERR_DEVICE, "device status 0x%x:%s%s%s", static_cast<unsigned>(h),
+                (h & SDD_DEV_NONFINITE) ? " non-finite row" : "", (h & SDD_DEV_BAD_TOKEN) ? " token out of range" : "",
+                (h & SDD_DEV_TIMEOUT) ? " bounded wait expired" : "");
+}
+
 sdd_status_t sdd_workspace_size(int B, int gamma, int V, size_t *bytes) {
     if (!bytes) return fail(SDD_ERR_INVALID_ARGUMENT, "bytes is NULL");
     SDD_TRY(check_shape(SDD_BF16, B, gamma, V, ((static_cast<int64_t>(V) + 7) / 8) * 8));

@@ -96,6 +96,14 @@ def test_invalid_arguments_rejected_on_host(lib):
     assert rc == 1 and b"n_rows" in lib.sdd_last_error()
 
 
+def test_status_from_device_rejects_null_on_host(lib):
+    VP = ctypes.c_void_p
+    bits = ctypes.c_uint32(7)
+    assert lib.sdd_status_from_device(None, 0, ctypes.byref(bits), None) == 1
+    assert b"NULL" in lib.sdd_last_error() and bits.value == 7
+    assert lib.sdd_status_from_device(VP(16), 0, None, None) == 1
+
+
 def test_scorer_workspace_size_and_check(lib):
     # 512 KiB per started 128-position tile: four split-K partials of 128 x 256 fp32
     n = ctypes.c_size_t(0)

@@ -38,8 +38,11 @@ def test_ring_wait_runs_out_and_recovers(sdd, orc, polls):
         sdd.test_wait_hooks(0, drop_copy=False)
     assert int(status.item()) & sdd.DEV_TIMEOUT, int(status.item())
     assert dt < 30.0
+    # the status reader reports it as a return code and clears the word
+    code, bits = sdd.status_from_device(status, clear=True)
+    assert code == sdd.binding.SDD_ERR_DEVICE and bits & sdd.DEV_TIMEOUT
+    assert int(status.item()) == 0 and sdd.status_from_device(status) == (0, 0)
     # the context, the workspace and the library stay usable
-    status.zero_()
     conf = sdd.confidence(blk.z_d, blk.x, ws=ws, status=status)
     torch.cuda.synchronize()
     assert int(status.item()) == 0
@@ -65,5 +68,6 @@ def test_short_limit_without_a_dropped_copy_is_harmless(sdd, orc):
         sdd.test_wait_hooks(0, drop_copy=False)
     st = int(status.item())
     assert st in (0, sdd.DEV_TIMEOUT)
+    assert sdd.status_from_device(status)[1] == st
     if st == 0:
         _check_against_oracle(orc, blk, conf)
