@@ -56,7 +56,7 @@ class DecodeLoop:
 
     def __init__(self, B: int, gamma: int, V: int, *, tau: float = 0.9, tau_mlp: float = 0.9, K_min: int = 6,
                  S_max: int = 64, greedy: bool = False, seed: int = 4, hidden: int = synth.HIDDEN, period: int = 4,
-                 scorer: str = "deep", history: int = 8, device="cuda"):
+                 scorer: str = "deep", history: int = 8, overlap: bool = True, device="cuda"):
         self.B, self.gamma, self.V = B, gamma, V
         self.tau, self.tau_mlp, self.K_min, self.S_max = tau, tau_mlp, K_min, S_max
         self.greedy, self.seed, self.period = greedy, seed, period
@@ -90,6 +90,13 @@ class DecodeLoop:
         self.hist_tokens = i32(H, B, gamma + 1)
         self.hist_n = i32(H, B)
         self.rows = i32(B)
+        # the survival scorer and its shadow schedule need only the confidence
+        # pass: with overlap they run on a second stream beside the raw
+        # schedule and the verifier pass
+        self.overlap = overlap
+        self.side = torch.cuda.Stream(device=dev) if overlap else None
+        self._conf_ready = torch.cuda.Event() if overlap else None
+        self._side_done = torch.cuda.Event() if overlap else None
         self.reset()
 
     def reset(self):
@@ -121,20 +128,33 @@ class DecodeLoop:
             self.hist_vt[k].fill_(-2)
             self.hist_vn[k].fill_(-2)
         self.rounds_run += 1
+        main = torch.cuda.current_stream(self.device)
         conf = sdd.confidence(z_d, x, ws=self.ws, status=self.status, features=deep, out=self._conf)
-        if deep:
-            s = sdd.scorer_deep(h, self.features(conf, round_), *self.deep, act=self.act, status=self.status,
-                                workspace=self.scorer_ws, out=self.score).reshape(B, gamma)
-        else:
-            s = sdd.survival_mlp(h, self.W1, self.b1, self.w2, self.b2, status=self.status,
-                                 workspace=self.scorer_ws, out=self.score).reshape(B, gamma)
         o = lambda p: tuple(t[k] for t in self.hist[p])   # noqa: E731
+
+        def scored():
+            if deep:
+                sc = sdd.scorer_deep(h, self.features(conf, round_), *self.deep, act=self.act, status=self.status,
+                                     workspace=self.scorer_ws, out=self.score).reshape(B, gamma)
+            else:
+                sc = sdd.survival_mlp(h, self.W1, self.b1, self.w2, self.b2, status=self.status,
+                                      workspace=self.scorer_ws, out=self.score).reshape(B, gamma)
+            _, K_m, D_m = sdd.schedule_prefix(sc, [self.tau_mlp], [self.tau_mlp], signal=sdd.SIG_CONDITIONAL,
+                                              K_min=self.K_min, S_max=self.S_max, D_in=self.D_mlp,
+                                              status=self.status, out=o("mlp"))
+            return sc, K_m, D_m
+
+        if self.overlap:
+            self._conf_ready.record(main)
+            self.side.wait_event(self._conf_ready)
+            with torch.cuda.stream(self.side):
+                s, K_mlp, D_mlp = scored()
+                self._side_done.record(self.side)
+        else:
+            s, K_mlp, D_mlp = scored()
         _, K_raw, D_raw = sdd.schedule_prefix(conf.q, [self.tau], [self.tau], signal=sdd.SIG_RAW, logq=conf.logq,
                                               K_min=self.K_min, S_max=self.S_max, D_in=self.D_raw,
                                               status=self.status, out=o("raw"))
-        _, K_mlp, D_mlp = sdd.schedule_prefix(s, [self.tau_mlp], [self.tau_mlp], signal=sdd.SIG_CONDITIONAL,
-                                              K_min=self.K_min, S_max=self.S_max, D_in=self.D_mlp,
-                                              status=self.status, out=o("mlp"))
         _, K_per, D_per = sdd.schedule_periodic(B, gamma, [self.period], K_skip=max(self.K_min, 1), round_=round_,
                                                 K_min=self.K_min, S_max=self.S_max, D_in=self.D_per,
                                                 status=self.status, device=self.device, out=o("per"))
@@ -144,6 +164,11 @@ class DecodeLoop:
                                              seed=self.seed, round_=round_, ws=self.ws, status=self.status,
                                              out=(self.hist_L[k], self.hist_vt[k], self.hist_vn[k]))
         tokens, n_commit = sdd.commit(K, x, tok, n, out=(self.hist_tokens[k], self.hist_n[k]))
+        if self.overlap:
+            # later work on the stream (the next round's confidence pass, which
+            # overwrites what the scorer read; any read of these outputs) comes
+            # after the side stream's
+            main.wait_event(self._side_done)
         self.D_raw, self.D_mlp, self.D_per = D_raw[0], D_mlp[0], D_per[0]
         return RoundOut(K_raw=K, K_mlp=K_mlp[0], K_per=K_per[0], L=L, tokens=tokens, n=n_commit,
                         n_verified=n_rows, score=s)
@@ -169,7 +194,7 @@ class DecodeLoop:
 
 
 def run(rounds: int = 256, workload: str = "c5", warmup: int = 2, scorer: str = "deep", n_sets: int = 8,
-        device="cuda") -> dict:
+        overlap: bool = True, device="cuda") -> dict:
     """The decode-loop workload over `rounds` rounds.  The seeded logits and
     hidden states of `n_sets` rounds are generated first (round r reads set
     r mod n_sets; the rounds still differ by their D, their Philox round index
@@ -180,7 +205,8 @@ def run(rounds: int = 256, workload: str = "c5", warmup: int = 2, scorer: str = 
     reported."""
     wl = synth.WORKLOADS[workload]
     B, gamma, V = wl.B, wl.gamma, wl.V
-    loop = DecodeLoop(B, gamma, V, tau=wl.taus[0], device=device, seed=wl.seed, scorer=scorer, history=rounds)
+    loop = DecodeLoop(B, gamma, V, tau=wl.taus[0], device=device, seed=wl.seed, scorer=scorer, history=rounds,
+                      overlap=overlap)
     sets = [(synth.make_block(wl, device=device, round_=r),
              synth.make_hidden(B * gamma, device=device, seed=wl.seed, round_=r)) for r in range(n_sets)]
     for r in range(warmup):
@@ -222,6 +248,7 @@ def run(rounds: int = 256, workload: str = "c5", warmup: int = 2, scorer: str = 
         "scorer": "(3584 + 19) -> 256 -> 256 -> 256 -> 1 (sdd_scorer_deep)" if scorer == "deep"
         else "3584 -> 256 -> 1 (sdd_survival_mlp)",
         "periodic_P": loop.period,
+        "scorer_stream": "second stream beside the verifier pass" if overlap else "in line",
         "device_status": status,
     }
 
@@ -230,10 +257,11 @@ def main():
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     ap.add_argument("--rounds", type=int, default=256)
     ap.add_argument("--workload", default="c5")
+    ap.add_argument("--no-overlap", action="store_true", help="run the scorer in line on the main stream")
     args = ap.parse_args()
     sdd.load()
     t0 = time.time()
-    res = run(args.rounds, args.workload)
+    res = run(args.rounds, args.workload, overlap=not args.no_overlap)
     res["wall_s"] = time.time() - t0
     print(json.dumps(res), flush=True)
 
