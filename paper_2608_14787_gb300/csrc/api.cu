@@ -199,6 +199,7 @@ void init_dec(DecideParams &d, const Work &w, sdd_dtype_t dtype, int B, int gamm
     d.tokens = tokens;
     d.res_pref = reinterpret_cast<float *>(w.base + w.L.res_pref);
     d.res_count = reinterpret_cast<uint32_t *>(w.base + w.L.res_count);
+    d.dec_ctas = w.dec_ctas;
     const int RV = static_cast<int>((static_cast<int64_t>(V) * esize(dtype) + 15) / 16);
     const int want = std::max(1, std::min(kDrawMaxSeg, w.dec_ctas / std::max(nb, 1)));
     const int per_thread = std::max(2, (RV + kDecThreads * want - 1) / (kDecThreads * want));

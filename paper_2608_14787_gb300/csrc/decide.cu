@@ -403,12 +403,43 @@ __device__ __forceinline__ void sched_pair(const DecideParams &d, const BlockFac
 // vocabulary-sharded round (records of S slices instead of warp partials,
 // the draw left to shard_draw_kernel).  Separate instantiations, so that the
 // fused round keeps the smallest kernel.
+// Draw geometry of one CTA: its listed block i, its segment of the draw row,
+// the block's segment count and vectors per segment.  From the host's
+// (blocks x segments) grid, or -- when the block count lives on the device
+// and the call draws -- from a one-dimensional grid of max(resident CTAs, B)
+// CTAs cut on the device into (listed block, segment) pairs the way the host
+// cuts its grid (init_dec), so that few listed blocks get more segments.
+struct DecGeom {
+    int i, seg, nseg, seg_vec;
+};
+__device__ __forceinline__ DecGeom dec_geom(const ScanParams &p, const PartView &pv, bool draw) {
+    DecGeom g;
+    if (p.nb_dev == nullptr || !draw) {
+        g.i = blockIdx.x;
+        g.seg = blockIdx.y;
+        g.nseg = p.dec.nseg;
+        g.seg_vec = p.dec.seg_vec;
+        return g;
+    }
+    const int nb = static_cast<int>(max(pv.nb, static_cast<int64_t>(1)));
+    const int want = max(1, min(kDrawMaxSeg, min(p.dec.dec_ctas, static_cast<int>(gridDim.x)) / nb));
+    const int per_thread = max(2, (p.RV + kDecThreads * want - 1) / (kDecThreads * want));
+    g.seg_vec = per_thread * kDecThreads;
+    g.nseg = (p.RV + g.seg_vec - 1) / g.seg_vec;
+    g.i = static_cast<int>(blockIdx.x) / g.nseg;
+    g.seg = static_cast<int>(blockIdx.x) % g.nseg;
+    return g;
+}
+
 template <int DT, bool FEAT, bool SHARD = false>
 __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_constant__ ScanParams p) {
     griddep_wait();   // launched behind the streaming grid that wrote the partials
     const DecideParams &d = p.dec;
-    const int i = blockIdx.x;       // listed block
-    const int seg = blockIdx.y;     // segment of the draw row
+    const PartView pv = part_view(p);
+    const DecGeom geo = dec_geom(p, pv, d.enabled && d.do_strict && !d.greedy && !SHARD);
+    const int i = geo.i;            // listed block
+    const int seg = geo.seg;        // segment of the draw row
+    const int nseg = geo.nseg, seg_vec = geo.seg_vec;
     const bool leader = seg == 0;   // writes the block's outputs
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     constexpr int NW = kDecThreads / 32;
@@ -425,7 +456,6 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
         else
             gt = gi;
     }
-    const PartView pv = part_view(p);
     if (i >= pv.nb) return;   // (a device block count below the grid's)
     const int32_t *bidx = p.grp[0].bidx;
     const int b = bidx ? __ldg(bidx + i) : i;
@@ -578,10 +608,10 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
         const char *zd_row = (L < gamma) ? d.zd + (ob + L) * d.stride_bytes : nullptr;
         const DrawCtx c = draw_ctx(zt_row, zd_row, df{F.t_lh[L], F.t_ll[L]},
                                    (L < gamma) ? df{F.d_lh[L], F.d_ll[L]} : df{0.f, 0.f});
-        const int vpt = d.seg_vec / kDecThreads;
-        const int64_t pair = static_cast<int64_t>(i) * d.nseg + seg;
+        const int vpt = seg_vec / kDecThreads;
+        const int64_t pair = static_cast<int64_t>(i) * nseg + seg;
         {
-            const int v0 = seg * d.seg_vec, v1 = min(p.RV, v0 + d.seg_vec);
+            const int v0 = seg * seg_vec, v1 = min(p.RV, v0 + seg_vec);
             const int vb = min(v1, v0 + tid * vpt), ve = min(v1, vb + vpt);
             float tot;
             const float incl = cta_incl_scan(run_sum<DT>(c, vb, ve, p.V), s_warp, &tot);
@@ -593,7 +623,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                 // this release; the acquire half orders the last arriver's
                 // reads of the other segments' prefixes after their releases
                 const uint32_t old = atom_add_acq_rel_gpu(d.res_count + i, 1u);
-                s_is_last = (old == static_cast<uint32_t>(d.nseg - 1)) ? 1 : 0;
+                s_is_last = (old == static_cast<uint32_t>(nseg - 1)) ? 1 : 0;
             }
             __syncthreads();
         }
@@ -601,8 +631,8 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
             // the last segment to arrive completes the draw: every segment's
             // prefixes in one round trip (a segment's total is its last prefix)
             const float4 *src =
-                reinterpret_cast<const float4 *>(d.res_pref + static_cast<int64_t>(i) * d.nseg * kDecThreads);
-            for (int q = tid; q < d.nseg * (kDecThreads / 4); q += kDecThreads) cp_async16(s_pref_all + 4 * q, src + q);
+                reinterpret_cast<const float4 *>(d.res_pref + static_cast<int64_t>(i) * nseg * kDecThreads);
+            for (int q = tid; q < nseg * (kDecThreads / 4); q += kDecThreads) cp_async16(s_pref_all + 4 * q, src + q);
             cp_async_wait_all();
             __syncthreads();
             if (warp == 0) {
@@ -610,11 +640,11 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                 // (double-floats); the first segment whose prefix exceeds u * R
                 df carry = df{0.f, 0.f};
                 int last_seg = -1;   // the last segment of positive mass
-                for (int s0 = 0; s0 < d.nseg; s0 += 32) {
+                for (int s0 = 0; s0 < nseg; s0 += 32) {
                     const int sg = s0 + lane;
-                    const float t = (sg < d.nseg) ? s_pref_all[sg * kDecThreads + kDecThreads - 1] : 0.f;
+                    const float t = (sg < nseg) ? s_pref_all[sg * kDecThreads + kDecThreads - 1] : 0.f;
                     const df cum = df_add(carry, warp_prefix_df(df{t, 0.f}, lane));
-                    if (sg < d.nseg) s_cum[sg] = cum;
+                    if (sg < nseg) s_cum[sg] = cum;
                     if (t > 0.f) last_seg = sg;
                     carry.hi = __shfl_sync(0xFFFFFFFFu, cum.hi, 31);
                     carry.lo = __shfl_sync(0xFFFFFFFFu, cum.lo, 31);
@@ -630,9 +660,9 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                 int sel = -1;
                 if (Rm.hi > 0.f) {
                     __syncwarp();
-                    for (int s0 = 0; s0 < d.nseg; s0 += 32) {
+                    for (int s0 = 0; s0 < nseg; s0 += 32) {
                         const int sg = s0 + lane;
-                        const bool hit = (sg < d.nseg) && s_pref_all[sg * kDecThreads + kDecThreads - 1] > 0.f &&
+                        const bool hit = (sg < nseg) && s_pref_all[sg * kDecThreads + kDecThreads - 1] > 0.f &&
                                          !df_ge(target, s_cum[sg]);
                         const unsigned bal = __ballot_sync(0xFFFFFFFFu, hit);
                         if (bal) {
@@ -683,7 +713,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                 if (warp == 0) {
                     int pick = -1;
                     if (thr >= 0) {
-                        const int sv0 = sel * d.seg_vec, sv1 = min(p.RV, sv0 + d.seg_vec);
+                        const int sv0 = sel * seg_vec, sv1 = min(p.RV, sv0 + seg_vec);
                         const int vb = min(sv1, sv0 + thr * vpt), ve = min(sv1, vb + vpt);
                         pick = warp_search<DT>(c, vb, ve, p.V, rem2, lane);
                     }
@@ -974,15 +1004,17 @@ cudaError_t launch_decide(const ScanParams &p, cudaStream_t stream) {
     const int nb = p.grp[0].nb;
     if (nb == 0) return cudaSuccess;
     const bool draw = p.dec.enabled && p.dec.do_strict && !p.dec.greedy;
-    const int nseg = draw ? p.dec.nseg : 1;
+    // a device block count: a one-dimensional grid cut on the device (dec_geom)
+    const bool dev_geom = draw && p.nb_dev != nullptr && p.shard == nullptr;
+    const int nseg = draw ? (dev_geom ? std::min(kDrawMaxSeg, std::max(p.dec.dec_ctas, 1)) : p.dec.nseg) : 1;
     const size_t smem = draw ? static_cast<size_t>(nseg) * kDecThreads * sizeof(float) : 0;
+    const dim3 grid = dev_geom ? dim3(static_cast<unsigned>(std::max(p.dec.dec_ctas, nb))) : dim3(nb, nseg);
     const bool bf = p.dtype == SDD_BF16, feat = p.feat != nullptr;
     void (*const k)(ScanParams) = (p.shard != nullptr)
                                       ? (bf ? decide_kernel<SDD_BF16, false, true> : decide_kernel<SDD_F32, false, true>)
                                   : feat ? (bf ? decide_kernel<SDD_BF16, true> : decide_kernel<SDD_F32, true>)
                                          : (bf ? decide_kernel<SDD_BF16, false> : decide_kernel<SDD_F32, false>);
-    return launch_dependent(k, dim3(nb, nseg),
-                            dim3(kDecThreads), smem, stream, p);
+    return launch_dependent(k, grid, dim3(kDecThreads), smem, stream, p);
 }
 
 // The blocks that go to the verifier: K[b] == 0, in ascending order, by one

@@ -97,6 +97,7 @@ struct DecideParams {
     long long *agreement;
     // sampling draw (residual / bonus inverse CDF), workspace
     int32_t nseg, seg_vec;         // segments per block and vectors per segment
+    int32_t dec_ctas;              // decide CTAs resident at once (the draw's one-wave budget)
     float *res_pref;               // [nb, nseg, kDecThreads] per-thread inclusive prefix sums
     uint32_t *res_count;           // [nb] (zero between calls)
     // vocabulary-sharded decide: this slice's draw-row masses [B][2] (residual

@@ -90,9 +90,9 @@ class DecodeLoop:
         self.hist_tokens = i32(H, B, gamma + 1)
         self.hist_n = i32(H, B)
         self.rows = i32(B)
-        # the survival scorer and its shadow schedule need only the confidence
-        # pass: with overlap they run on a second stream beside the raw
-        # schedule and the verifier pass
+        # the survival scorer and the two shadow schedules (scorer, periodic)
+        # need only the confidence pass: with overlap they run on a second
+        # stream beside the raw schedule and the verifier pass
         self.overlap = overlap
         self.side = torch.cuda.Stream(device=dev) if overlap else None
         self._conf_ready = torch.cuda.Event() if overlap else None
@@ -142,22 +142,22 @@ class DecodeLoop:
             _, K_m, D_m = sdd.schedule_prefix(sc, [self.tau_mlp], [self.tau_mlp], signal=sdd.SIG_CONDITIONAL,
                                               K_min=self.K_min, S_max=self.S_max, D_in=self.D_mlp,
                                               status=self.status, out=o("mlp"))
-            return sc, K_m, D_m
+            _, K_p, D_p = sdd.schedule_periodic(B, gamma, [self.period], K_skip=max(self.K_min, 1), round_=round_,
+                                                K_min=self.K_min, S_max=self.S_max, D_in=self.D_per,
+                                                status=self.status, device=self.device, out=o("per"))
+            return sc, K_m, D_m, K_p, D_p
 
         if self.overlap:
             self._conf_ready.record(main)
             self.side.wait_event(self._conf_ready)
             with torch.cuda.stream(self.side):
-                s, K_mlp, D_mlp = scored()
+                s, K_mlp, D_mlp, K_per, D_per = scored()
                 self._side_done.record(self.side)
         else:
-            s, K_mlp, D_mlp = scored()
+            s, K_mlp, D_mlp, K_per, D_per = scored()
         _, K_raw, D_raw = sdd.schedule_prefix(conf.q, [self.tau], [self.tau], signal=sdd.SIG_RAW, logq=conf.logq,
                                               K_min=self.K_min, S_max=self.S_max, D_in=self.D_raw,
                                               status=self.status, out=o("raw"))
-        _, K_per, D_per = sdd.schedule_periodic(B, gamma, [self.period], K_skip=max(self.K_min, 1), round_=round_,
-                                                K_min=self.K_min, S_max=self.S_max, D_in=self.D_per,
-                                                status=self.status, device=self.device, out=o("per"))
         K = K_raw[0]
         rows, n_rows = sdd.select_rows(K, rows=self.rows, n_rows=self.hist_n_rows[k])
         L, tok, n = sdd.verify_strict_listed(z_t, x, rows, n_rows, z_d=z_d, draft=conf, greedy=self.greedy,
