@@ -399,10 +399,6 @@ __device__ __forceinline__ void sched_pair(const DecideParams &d, const BlockFac
     sched_final(Kh, D, d.K_min, d.S_max, K, Do);
 }
 
-// FEAT: also the extended features of the drafter rows; SHARD: the
-// vocabulary-sharded round (records of S slices instead of warp partials,
-// the draw left to shard_draw_kernel).  Separate instantiations, so that the
-// fused round keeps the smallest kernel.
 // Draw geometry of one CTA: its listed block i, its segment of the draw row,
 // the block's segment count and vectors per segment.  From the host's
 // (blocks x segments) grid, or -- when the block count lives on the device
@@ -431,6 +427,10 @@ __device__ __forceinline__ DecGeom dec_geom(const ScanParams &p, const PartView 
     return g;
 }
 
+// FEAT: also the extended features of the drafter rows; SHARD: the
+// vocabulary-sharded round (records of S slices instead of warp partials,
+// the draw left to shard_draw_kernel).  Separate instantiations, so that the
+// fused round keeps the smallest kernel.
 template <int DT, bool FEAT, bool SHARD = false>
 __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_constant__ ScanParams p) {
     griddep_wait();   // launched behind the streaming grid that wrote the partials
