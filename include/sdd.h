@@ -609,8 +609,12 @@ typedef struct sdd_shard_partial {
 
 /*
  * sdd_shard_workspace_size -- bytes of device scratch that sdd_shard_decide
- * leaves for sdd_shard_draw (per block: the accepted length and the draw
- * row's log-normalisers): B * 32.
+ * leaves for sdd_shard_draw: per block the accepted length and the draw row's
+ * log-normalisers (32 bytes), an arrival counter, and for up to 64 segments
+ * of this slice's draw row their p_t masses and per-thread prefix sums
+ * (256 floats each); about 66 KiB per block.  Zero-filled once before its
+ * first use (every sdd_shard_decide leaves its counters at zero again);
+ * 16-byte aligned.
  */
 SDD_API sdd_status_t sdd_shard_workspace_size(int B, size_t *bytes);
 

@@ -888,10 +888,38 @@ static sdd_status_t shard_kcap(const sdd_block_args *a, int &kcap) {
     return SDD_OK;
 }
 
+// The sharded round's workspace: per block the draw state, the draw's
+// arrival counter, each draw segment's p_t mass and each segment's per-thread
+// prefix sums (at most kDrawMaxSeg segments of kDecThreads runs per block).
+struct ShardWs {
+    size_t state, count, ptot, pref, total;
+};
+static ShardWs shard_ws_layout(int B) {
+    auto up = [](size_t v, size_t a) { return (v + a - 1) / a * a; };
+    const size_t b = static_cast<size_t>(B);
+    ShardWs w;
+    w.state = 0;
+    w.count = up(b * sizeof(ShardDraw), 16);
+    w.ptot = up(w.count + b * sizeof(uint32_t), 16);
+    w.pref = up(w.ptot + b * kDrawMaxSeg * sizeof(float), 16);
+    w.total = w.pref + b * kDrawMaxSeg * kDecThreads * sizeof(float);
+    return w;
+}
+
+// Draw segments of a slice's draw rows (RV vectors) for B blocks, cut the way
+// init_dec cuts one-GPU draw rows: as many as keep B * nseg decide CTAs
+// resident at once, at least two vectors per thread, at most kDrawMaxSeg.
+static void shard_segments(int B, int RV, int dec_ctas, int32_t &nseg, int32_t &seg_vec) {
+    const int want = std::max(1, std::min(kDrawMaxSeg, dec_ctas / std::max(B, 1)));
+    const int per_thread = std::max(2, (RV + kDecThreads * want - 1) / (kDecThreads * want));
+    seg_vec = per_thread * kDecThreads;
+    nseg = (RV + seg_vec - 1) / seg_vec;
+}
+
 sdd_status_t sdd_shard_workspace_size(int B, size_t *bytes) {
     if (!bytes) return fail(SDD_ERR_INVALID_ARGUMENT, "bytes is NULL");
     if (B < 0) return fail(SDD_ERR_INVALID_ARGUMENT, "B = %d < 0", B);
-    *bytes = static_cast<size_t>(B) * sizeof(ShardDraw);
+    *bytes = shard_ws_layout(B).total;
     return SDD_OK;
 }
 
@@ -1003,8 +1031,15 @@ sdd_status_t sdd_shard_decide(const sdd_block_args *a, int v0, int v1, int n_sha
     d.V = p.V;
     d.stride_bytes = a->row_stride * esize(dt);
     d.tokens = a->draft_tokens;
-    d.nseg = 1;
-    d.seg_vec = p.RV;
+    DevInfo di;
+    SDD_TRY(device_info(di));   // the kernels' attributes are set on this device
+    const ShardWs L = shard_ws_layout(a->B);
+    char *ws = static_cast<char *>(a->workspace);
+    d.dec_ctas = di.sms * di.dec_ctas_per_sm;
+    shard_segments(a->B, p.RV, d.dec_ctas, d.nseg, d.seg_vec);
+    d.res_pref = reinterpret_cast<float *>(ws + L.pref);
+    d.res_count = reinterpret_cast<uint32_t *>(ws + L.count);
+    d.shard_ptot = reinterpret_cast<float *>(ws + L.ptot);
     d.zt = static_cast<const char *>(a->target_logits);
     d.zd = static_cast<const char *>(a->draft_logits);
     d.do_strict = 1;
@@ -1035,10 +1070,8 @@ sdd_status_t sdd_shard_decide(const sdd_block_args *a, int v0, int v1, int n_sha
     d.commit_n = a->commit_n;
     d.agreement = reinterpret_cast<long long *>(a->agreement);
     d.shard_mass = mass;
-    d.shard_state = static_cast<ShardDraw *>(a->workspace);
+    d.shard_state = reinterpret_cast<ShardDraw *>(ws + L.state);
     p.dec = d;
-    DevInfo di;
-    SDD_TRY(device_info(di));   // the kernels' attributes are set on this device
     return run_decide_shard(p, reinterpret_cast<cudaStream_t>(stream));
 }
 
@@ -1056,7 +1089,13 @@ sdd_status_t sdd_shard_draw(const sdd_block_args *a, int v0, int v1, int n_shard
     sp.n_shards = n_shards;
     sp.shard = shard;
     sp.mass_all = mass_all;
-    sp.state = static_cast<const ShardDraw *>(a->workspace);
+    DevInfo di;
+    SDD_TRY(device_info(di));   // the kernels' attributes are set on this device
+    const ShardWs L = shard_ws_layout(a->B);
+    const char *ws = static_cast<const char *>(a->workspace);
+    sp.state = reinterpret_cast<const ShardDraw *>(ws + L.state);
+    sp.res_pref = reinterpret_cast<const float *>(ws + L.pref);
+    shard_segments(a->B, sp.RVs, di.sms * di.dec_ctas_per_sm, sp.nseg, sp.seg_vec);
     sp.seed = a->seed;
     sp.round = a->round;
     sp.tok_strict = a->tokens_strict;

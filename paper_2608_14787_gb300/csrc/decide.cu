@@ -399,6 +399,86 @@ __device__ __forceinline__ void sched_pair(const DecideParams &d, const BlockFac
     sched_final(Kh, D, d.K_min, d.S_max, K, Do);
 }
 
+// The draw's last step over staged segment prefixes: s_pref_all holds nseg
+// segments' per-thread inclusive prefix sums ([nseg][kDecThreads]; a
+// segment's total is its last prefix).
+//
+// segment_cum (warp 0): the segments' cumulative totals as double-floats
+// into s_cum; returns the total, and in last_seg the last segment of
+// positive mass (-1: none).
+__device__ __forceinline__ df segment_cum(const float *s_pref_all, int nseg, df *s_cum, int lane, int &last_seg) {
+    df carry = df{0.f, 0.f};
+    last_seg = -1;
+    for (int s0 = 0; s0 < nseg; s0 += 32) {
+        const int sg = s0 + lane;
+        const float t = (sg < nseg) ? s_pref_all[sg * kDecThreads + kDecThreads - 1] : 0.f;
+        const df cum = df_add(carry, warp_prefix_df(df{t, 0.f}, lane));
+        if (sg < nseg) s_cum[sg] = cum;
+        if (t > 0.f) last_seg = sg;
+        carry.hi = __shfl_sync(0xFFFFFFFFu, cum.hi, 31);
+        carry.lo = __shfl_sync(0xFFFFFFFFu, cum.lo, 31);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) last_seg = max(last_seg, __shfl_xor_sync(0xFFFFFFFFu, last_seg, off));
+    return carry;
+}
+
+// segment_pick (warp 0, after segment_cum and a __syncwarp): the first
+// segment of positive mass whose cumulative total exceeds target; -1 if
+// rounding leaves none.
+__device__ __forceinline__ int segment_pick(const float *s_pref_all, int nseg, const df *s_cum, df target, int lane) {
+    for (int s0 = 0; s0 < nseg; s0 += 32) {
+        const int sg = s0 + lane;
+        const bool hit = (sg < nseg) && s_pref_all[sg * kDecThreads + kDecThreads - 1] > 0.f &&
+                         !df_ge(target, s_cum[sg]);
+        const unsigned bal = __ballot_sync(0xFFFFFFFFu, hit);
+        if (bal) return s0 + __ffs(bal) - 1;
+    }
+    return -1;
+}
+
+// segment_find (every thread of the CTA): the entry of segment sel (vectors
+// [sel seg_vec, ...) of a row of RV vectors, kDecThreads runs of
+// seg_vec / kDecThreads vectors) at which the running sum exceeds rem, a
+// double-float measured from the segment's start: the thread from the
+// segment's prefixes, the entry by warp 0 (warp_search).  When rounding
+// leaves no thread, the last thread whose run has positive weight, searched
+// to its end.  *s_thr must be INT32_MAX and *s_thr_last -1 on entry.
+template <int DT>
+__device__ int segment_find(const DrawCtx &c, const float *s_pref_all, int sel, df rem, int seg_vec, int RV, int V,
+                            int *s_thr, int *s_thr_last, int *s_tok) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int vpt = seg_vec / kDecThreads;
+    const float *s_pref = s_pref_all + sel * kDecThreads;
+    const float pv = s_pref[tid];
+    const unsigned bal = __ballot_sync(0xFFFFFFFFu, !df_ge(rem, df{pv, 0.f}));
+    if (lane == 0 && bal) atomicMin(s_thr, warp * 32 + __ffs(bal) - 1);
+    __syncthreads();
+    int thr = *s_thr;
+    df rem2 = rem;
+    if (thr == INT32_MAX) {
+        const bool rose = pv > ((tid > 0) ? s_pref[tid - 1] : 0.f);
+        const unsigned up = __ballot_sync(0xFFFFFFFFu, rose);
+        if (lane == 0 && up) atomicMax(s_thr_last, warp * 32 + 31 - __clz(up));
+        __syncthreads();
+        thr = *s_thr_last;
+        rem2 = df{__int_as_float(0x7F800000), 0.f};
+    } else if (thr > 0) {
+        rem2 = df_sub(rem, df{s_pref[thr - 1], 0.f});
+    }
+    if (warp == 0) {
+        int pick = -1;
+        if (thr >= 0) {
+            const int sv0 = sel * seg_vec, sv1 = min(RV, sv0 + seg_vec);
+            const int vb = min(sv1, sv0 + thr * vpt), ve = min(sv1, vb + vpt);
+            pick = warp_search<DT>(c, vb, ve, V, rem2, lane);
+        }
+        if (lane == 0) *s_tok = pick;
+    }
+    __syncthreads();
+    return *s_tok;
+}
+
 // Draw geometry of one CTA: its listed block i, its segment of the draw row,
 // the block's segment count and vectors per segment.  From the host's
 // (blocks x segments) grid, or -- when the block count lives on the device
@@ -559,46 +639,81 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
         __syncthreads();
 
         if (SHARD) {
-            // ---- vocabulary-sharded (one CTA per block): this slice's masses
-            // of the draw row -- the residual (or bonus) weights, then p_t --
-            // for the exchange between ranks; shard_draw_kernel then draws ----
+            // ---- vocabulary-sharded: this CTA's segment of this slice's draw
+            // row -- the residual (or bonus) weights' per-thread prefixes,
+            // published for shard_draw_kernel, and the segment's p_t mass; the
+            // last segment to arrive sums the segments' masses in order into
+            // this slice's masses for the exchange between ranks ----
             const int L = s_L[0];
             const char *zt_row = d.zt + (bo + L) * d.stride_bytes;
             const char *zd_row = (L < gamma) ? d.zd + (ob + L) * d.stride_bytes : nullptr;
             const DrawCtx c = draw_ctx(zt_row, zd_row, df{F.t_lh[L], F.t_ll[L]},
                                        (L < gamma) ? df{F.d_lh[L], F.d_ll[L]} : df{0.f, 0.f});
+            const int vpt = seg_vec / kDecThreads;
+            const int sv0 = seg * seg_vec, sv1 = min(p.RV, sv0 + seg_vec);
+            const int vb = min(sv1, sv0 + tid * vpt), ve = min(sv1, vb + vpt);
             float tot_r, tot_p;
-            (void)cta_incl_scan(slice_thread_sum<DT>(c, p.RV, p.V), s_warp, &tot_r);
+            const float incl = cta_incl_scan(run_sum<DT>(c, vb, ve, p.V), s_warp, &tot_r);
+            d.res_pref[(static_cast<int64_t>(b) * kDrawMaxSeg + seg) * kDecThreads + tid] = incl;
             if (L < gamma) {
                 DrawCtx ct = c;
                 ct.zd_row = nullptr;
-                (void)cta_incl_scan(slice_thread_sum<DT>(ct, p.RV, p.V), s_warp, &tot_p);
+                (void)cta_incl_scan(run_sum<DT>(ct, vb, ve, p.V), s_warp, &tot_p);
             } else {
                 tot_p = tot_r;
             }
-            const bool commit = sched && s_K0 == 0;
+            if (tid == 0) d.shard_ptot[static_cast<int64_t>(b) * kDrawMaxSeg + seg] = tot_p;
+            __syncthreads();
             if (tid == 0) {
-                d.shard_mass[2 * b] = tot_r;
-                d.shard_mass[2 * b + 1] = tot_p;
-                ShardDraw sd;
-                sd.L = L;
-                sd.commit = commit ? 1 : 0;
-                sd.t_lh = F.t_lh[L];
-                sd.t_ll = F.t_ll[L];
-                sd.d_lh = (L < gamma) ? F.d_lh[L] : 0.f;
-                sd.d_ll = (L < gamma) ? F.d_ll[L] : 0.f;
-                sd.pad[0] = sd.pad[1] = 0;
-                d.shard_state[b] = sd;
+                // (as in the one-GPU draw: release of this segment's stores,
+                // acquire of the others' for the last arriver)
+                const uint32_t old = atom_add_acq_rel_gpu(d.res_count + b, 1u);
+                s_is_last = (old == static_cast<uint32_t>(nseg - 1)) ? 1 : 0;
             }
-            if (warp == 0) {
-                // the drawn token's place stays -1 until the draw
-                if (lane == 0) {
-                    if (d.L_strict) d.L_strict[b] = L;
-                    if (d.n_strict) d.n_strict[b] = L + 1;
-                    if (commit && d.commit_n) d.commit_n[b] = L + 1;
+            __syncthreads();
+            if (s_is_last && warp == 0) {
+                df cr = df{0.f, 0.f}, cp = df{0.f, 0.f};
+                for (int s0 = 0; s0 < nseg; s0 += 32) {
+                    const int sg = s0 + lane;
+                    const int64_t at = static_cast<int64_t>(b) * kDrawMaxSeg + sg;
+                    const float tr = (sg < nseg) ? __ldcg(d.res_pref + at * kDecThreads + kDecThreads - 1) : 0.f;
+                    const float tq = (sg < nseg) ? __ldcg(d.shard_ptot + at) : 0.f;
+                    const df xr = df_add(cr, warp_prefix_df(df{tr, 0.f}, lane));
+                    const df xq = df_add(cp, warp_prefix_df(df{tq, 0.f}, lane));
+                    cr.hi = __shfl_sync(0xFFFFFFFFu, xr.hi, 31);
+                    cr.lo = __shfl_sync(0xFFFFFFFFu, xr.lo, 31);
+                    cp.hi = __shfl_sync(0xFFFFFFFFu, xq.hi, 31);
+                    cp.lo = __shfl_sync(0xFFFFFFFFu, xq.lo, 31);
                 }
-                if (d.tok_strict) write_tokens(lane, gamma, d.tok_strict + bo, F.x, L, -1);
-                if (commit && d.commit_tokens) write_tokens(lane, gamma, d.commit_tokens + bo, F.x, L, -1);
+                if (lane == 0) {
+                    d.shard_mass[2 * b] = cr.hi + cr.lo;
+                    d.shard_mass[2 * b + 1] = cp.hi + cp.lo;
+                    d.res_count[b] = 0u;   // leave the counter at zero for the next call
+                }
+            }
+            if (leader) {
+                const bool commit = sched && s_K0 == 0;
+                if (tid == 0) {
+                    ShardDraw sd;
+                    sd.L = L;
+                    sd.commit = commit ? 1 : 0;
+                    sd.t_lh = F.t_lh[L];
+                    sd.t_ll = F.t_ll[L];
+                    sd.d_lh = (L < gamma) ? F.d_lh[L] : 0.f;
+                    sd.d_ll = (L < gamma) ? F.d_ll[L] : 0.f;
+                    sd.pad[0] = sd.pad[1] = 0;
+                    d.shard_state[b] = sd;
+                }
+                if (warp == 0) {
+                    // the drawn token's place stays -1 until the draw
+                    if (lane == 0) {
+                        if (d.L_strict) d.L_strict[b] = L;
+                        if (d.n_strict) d.n_strict[b] = L + 1;
+                        if (commit && d.commit_n) d.commit_n[b] = L + 1;
+                    }
+                    if (d.tok_strict) write_tokens(lane, gamma, d.tok_strict + bo, F.x, L, -1);
+                    if (commit && d.commit_tokens) write_tokens(lane, gamma, d.commit_tokens + bo, F.x, L, -1);
+                }
             }
         } else {
         // ---- phase 3 (every CTA): its segment of the draw row at position L
@@ -638,21 +753,8 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
             if (warp == 0) {
                 // R = sum of the segment totals and their inclusive prefix sums
                 // (double-floats); the first segment whose prefix exceeds u * R
-                df carry = df{0.f, 0.f};
-                int last_seg = -1;   // the last segment of positive mass
-                for (int s0 = 0; s0 < nseg; s0 += 32) {
-                    const int sg = s0 + lane;
-                    const float t = (sg < nseg) ? s_pref_all[sg * kDecThreads + kDecThreads - 1] : 0.f;
-                    const df cum = df_add(carry, warp_prefix_df(df{t, 0.f}, lane));
-                    if (sg < nseg) s_cum[sg] = cum;
-                    if (t > 0.f) last_seg = sg;
-                    carry.hi = __shfl_sync(0xFFFFFFFFu, cum.hi, 31);
-                    carry.lo = __shfl_sync(0xFFFFFFFFu, cum.lo, 31);
-                }
-#pragma unroll
-                for (int off = 16; off > 0; off >>= 1)
-                    last_seg = max(last_seg, __shfl_xor_sync(0xFFFFFFFFu, last_seg, off));
-                const df Rm = carry;
+                int last_seg;   // the last segment of positive mass
+                const df Rm = segment_cum(s_pref_all, nseg, s_cum, lane, last_seg);
                 const uint32_t jj = (L < gamma) ? static_cast<uint32_t>(L + 1) : static_cast<uint32_t>(gamma + 1);
                 const float u = philox_uniform(d.seed, jj, static_cast<uint32_t>(b), d.round,
                                                (L < gamma) ? kPurposeResid : kPurposeBonus);
@@ -660,16 +762,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
                 int sel = -1;
                 if (Rm.hi > 0.f) {
                     __syncwarp();
-                    for (int s0 = 0; s0 < nseg; s0 += 32) {
-                        const int sg = s0 + lane;
-                        const bool hit = (sg < nseg) && s_pref_all[sg * kDecThreads + kDecThreads - 1] > 0.f &&
-                                         !df_ge(target, s_cum[sg]);
-                        const unsigned bal = __ballot_sync(0xFFFFFFFFu, hit);
-                        if (bal) {
-                            sel = s0 + __ffs(bal) - 1;
-                            break;
-                        }
-                    }
+                    sel = segment_pick(s_pref_all, nseg, s_cum, target, lane);
                 }
                 if (lane == 0) {
                     if (sel >= 0) {
@@ -689,38 +782,8 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const __grid_consta
             const int sel = s_seg;
             if (sel >= 0) {
                 // the thread of segment sel whose run holds u R, from the
-                // inclusive prefixes that segment's CTA published
-                const float *s_pref = s_pref_all + sel * kDecThreads;
-                const float pv = s_pref[tid];
-                const df rem = s_rem;
-                const unsigned bal = __ballot_sync(0xFFFFFFFFu, !df_ge(rem, df{pv, 0.f}));
-                if (lane == 0 && bal) atomicMin(&s_thr, warp * 32 + __ffs(bal) - 1);
-                __syncthreads();
-                int thr = s_thr;
-                df rem2 = rem;
-                if (thr == INT32_MAX) {
-                    // rounding left no thread: the last thread whose run has
-                    // positive weight (its prefix rose), searched to its end
-                    const bool rose = pv > ((tid > 0) ? s_pref[tid - 1] : 0.f);
-                    const unsigned up = __ballot_sync(0xFFFFFFFFu, rose);
-                    if (lane == 0 && up) atomicMax(&s_thr_last, warp * 32 + 31 - __clz(up));
-                    __syncthreads();
-                    thr = s_thr_last;
-                    rem2 = df{__int_as_float(0x7F800000), 0.f};
-                } else if (thr > 0) {
-                    rem2 = df_sub(rem, df{s_pref[thr - 1], 0.f});
-                }
-                if (warp == 0) {
-                    int pick = -1;
-                    if (thr >= 0) {
-                        const int sv0 = sel * seg_vec, sv1 = min(p.RV, sv0 + seg_vec);
-                        const int vb = min(sv1, sv0 + thr * vpt), ve = min(sv1, vb + vpt);
-                        pick = warp_search<DT>(c, vb, ve, p.V, rem2, lane);
-                    }
-                    if (lane == 0) s_tok = pick;
-                }
-                __syncthreads();
-                tok = s_tok;
+                // inclusive prefixes that segment's CTA published, then the entry
+                tok = segment_find<DT>(c, s_pref_all, sel, s_rem, seg_vec, p.RV, p.V, &s_thr, &s_thr_last, &s_tok);
             } else {
                 // the residual has no mass (only through rounding): draw from p_t
                 // of the same row, whole row in this CTA, same inverse-CDF rule
@@ -834,8 +897,14 @@ __global__ void __launch_bounds__(kDecThreads) shard_draw_kernel(const __grid_co
     const int gamma = sp.gamma, S = sp.n_shards;
     __shared__ float s_warp[2 * NW];
     __shared__ df s_cum[kMaxShards];
-    __shared__ int s_sel, s_col, s_thr, s_last, s_tok;
-    __shared__ df s_rem;
+    __shared__ df s_cseg[kDrawMaxSeg];
+    __shared__ int s_sel, s_col, s_thr, s_last, s_tok, s_seg;
+    __shared__ df s_rem, s_rem2;
+    extern __shared__ float s_pref_all[];   // [nseg][kDecThreads]: the decide's prefixes of this slice's draw row
+    if (tid == 0) {
+        s_thr = INT32_MAX;
+        s_last = -1;
+    }
     const ShardDraw st = sp.state[b];
     const int L = st.L;
     if (warp == 0) {
@@ -896,7 +965,41 @@ __global__ void __launch_bounds__(kDecThreads) shard_draw_kernel(const __grid_co
     const char *zd_row = (L < gamma && s_col == 0) ? sp.zd + (static_cast<int64_t>(b) * gamma + L) * sp.stride_bytes
                                                    : nullptr;
     const DrawCtx c = draw_ctx(zt_row, zd_row, df{st.t_lh, st.t_ll}, zd_row ? df{st.d_lh, st.d_ll} : df{0.f, 0.f});
-    const int tok = slice_find<DT>(c, sp.RVs, sp.Vs, s_rem, s_warp, &s_thr, &s_last, &s_tok);
+    int tok;
+    if (s_col == 0) {
+        // the residual (or bonus) weights: the segment, thread and entry from
+        // the prefixes sdd_shard_decide published (the sums this slice's
+        // mass was made of), as the one-GPU draw locates its token
+        const float4 *src =
+            reinterpret_cast<const float4 *>(sp.res_pref + static_cast<int64_t>(b) * kDrawMaxSeg * kDecThreads);
+        for (int q = tid; q < sp.nseg * (kDecThreads / 4); q += kDecThreads) cp_async16(s_pref_all + 4 * q, src + q);
+        cp_async_wait_all();
+        __syncthreads();
+        if (warp == 0) {
+            int last_seg;
+            (void)segment_cum(s_pref_all, sp.nseg, s_cseg, lane, last_seg);
+            __syncwarp();
+            const df rem = s_rem;
+            const int sel = segment_pick(s_pref_all, sp.nseg, s_cseg, rem, lane);
+            if (lane == 0) {
+                if (sel >= 0) {
+                    s_seg = sel;
+                    s_rem2 = (sel > 0) ? df_sub(rem, s_cseg[sel - 1]) : rem;
+                } else {
+                    // rounding (or an infinite remainder): the slice's last positive entry
+                    s_seg = last_seg;
+                    s_rem2 = df{__int_as_float(0x7F800000), 0.f};
+                }
+            }
+        }
+        __syncthreads();
+        tok = (s_seg >= 0) ? segment_find<DT>(c, s_pref_all, s_seg, s_rem2, sp.seg_vec, sp.RVs, sp.Vs, &s_thr, &s_last,
+                                              &s_tok)
+                           : -1;
+    } else {
+        // p_t of the row (the residual had no mass, only through rounding): the whole slice here
+        tok = slice_find<DT>(c, sp.RVs, sp.Vs, s_rem, s_warp, &s_thr, &s_last, &s_tok);
+    }
     if (tid == 0) {
         const int t = (tok >= 0) ? sp.v0 + tok : -1;
         if (sp.tok_strict) sp.tok_strict[bo + L] = t;
@@ -997,6 +1100,11 @@ cudaError_t decide_prepare_device() {
         const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
         if (e != cudaSuccess) return e;
     }
+    void (*const draws[])(ShardParams) = {shard_draw_kernel<SDD_BF16>, shard_draw_kernel<SDD_F32>};
+    for (auto k : draws) {
+        const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        if (e != cudaSuccess) return e;
+    }
     return cudaSuccess;
 }
 
@@ -1052,10 +1160,11 @@ cudaError_t launch_select_rows(const int32_t *K, int B, int32_t *rows, int32_t *
 
 cudaError_t launch_shard_draw(const ShardParams &sp, cudaStream_t stream) {
     if (sp.B == 0) return cudaSuccess;
+    const size_t smem = static_cast<size_t>(sp.nseg) * kDecThreads * sizeof(float);
     if (sp.dtype == SDD_BF16)
-        shard_draw_kernel<SDD_BF16><<<sp.B, kDecThreads, 0, stream>>>(sp);
+        shard_draw_kernel<SDD_BF16><<<sp.B, kDecThreads, smem, stream>>>(sp);
     else
-        shard_draw_kernel<SDD_F32><<<sp.B, kDecThreads, 0, stream>>>(sp);
+        shard_draw_kernel<SDD_F32><<<sp.B, kDecThreads, smem, stream>>>(sp);
     return cudaGetLastError();
 }
 

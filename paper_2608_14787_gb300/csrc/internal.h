@@ -104,6 +104,7 @@ struct DecideParams {
     // or bonus weights, then p_t weights) and the per-block draw state
     float *shard_mass;
     ShardDraw *shard_state;
+    float *shard_ptot;             // [B][kDrawMaxSeg] each draw segment's p_t mass (this slice)
 };
 
 // One set of rows streamed by the scan kernel (drafter rows or target rows).
@@ -198,6 +199,8 @@ struct ShardParams {
     int32_t n_shards, shard;
     const float *mass_all;   // [n_shards][B][2]
     const ShardDraw *state;  // [B]
+    const float *res_pref;   // [B][kDrawMaxSeg][kDecThreads] the decide's per-thread prefixes of the draw row
+    int32_t nseg, seg_vec;   // its segments of the slice's draw row
     uint64_t seed, round;
     int32_t *tok_strict, *commit_tokens;
 };

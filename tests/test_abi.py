@@ -171,4 +171,8 @@ def test_shard_arguments_rejected_on_host(lib):
     a.n_k = 0
     assert lib.sdd_shard_draw(ctypes.byref(a), 0, 500, 2, 2, ctypes.c_void_p(256), None) == 1
     n = ctypes.c_size_t(0)
-    assert lib.sdd_shard_workspace_size(5, ctypes.byref(n)) == 0 and n.value == 5 * 32
+    # per block: the 32-byte draw state, a counter, 64 segments' p_t masses and
+    # 64 x 256 per-thread prefixes (each region 16-byte aligned)
+    up = lambda v: (v + 15) // 16 * 16   # noqa: E731
+    want = up(up(up(5 * 32) + 5 * 4) + 5 * 64 * 4) + 5 * 64 * 256 * 4
+    assert lib.sdd_shard_workspace_size(5, ctypes.byref(n)) == 0 and n.value == want
