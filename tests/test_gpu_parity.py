@@ -527,3 +527,29 @@ def test_select_rows_and_listed_verify(sdd, frac):
         compare_rule(Tally(), "listed", L, tok, ob.strict, want_rows.cpu().tolist())
     skipped = (K != 0).nonzero().flatten()
     assert torch.all(L[skipped] == -2) and torch.all(tok[skipped] == -2)
+
+
+def test_listed_verify_few_blocks_full_vocabulary(sdd):
+    """Two of 24 blocks listed at V = 151,936: the decide grid, cut on the
+    device from the count, gives each listed block many draw segments (38),
+    the same cut as a host list of those two blocks; the results equal
+    sdd_verify_strict's on the host list bit for bit, and the oracle's."""
+    B, gamma, V = 24, 8, 151_936
+    blk = synth.make_block("c3", device="cpu", B=B, gamma=gamma, V=V)
+    z_d, z_t, x = _to_dev(blk)
+    K = torch.full((B,), 3, dtype=torch.int32)
+    K[5] = 0
+    K[17] = 0
+    K = K.to(DEV)
+    rows, n = sdd.select_rows(K)
+    draft = sdd.confidence(z_d, x)
+    L, tok, nc = sdd.verify_strict_listed(z_t, x, rows, n, z_d=z_d, draft=draft, seed=11, round_=3)
+    want_rows = torch.tensor([5, 17], dtype=torch.int32, device=DEV)
+    L2, tok2, nc2 = sdd.verify_strict(z_t, x, z_d=z_d, draft=draft, seed=11, round_=3, rows=want_rows)
+    torch.cuda.synchronize()
+    assert int(n.item()) == 2
+    assert torch.equal(L, L2) and torch.equal(tok, tok2) and torch.equal(nc, nc2)
+    ob = oracle_block(z_d, z_t, x, seed=11, round_=3, blocks=[5, 17])
+    compare_rule(Tally(), "listed, few blocks", L, tok, ob.strict, [5, 17])
+    others = [b for b in range(B) if b not in (5, 17)]
+    assert torch.all(L[others] == -2) and torch.all(tok[others] == -2)
