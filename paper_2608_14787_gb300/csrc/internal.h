@@ -138,10 +138,13 @@ struct ScanParams {
     int64_t rows;            // rows of all groups
     int64_t T;               // total vectors = rows * RV
     // Cost-balanced partition: a vector of a group-g row costs wt[g] units
-    // (drafter rows carry the entropy work); T0 = rows0 * RV, C = total cost.
+    // (drafter rows carry the entropy work), and the first vector of every row
+    // R more (a piece's end and the next piece's start); P[g] = wt[g] RV + R is
+    // a whole row's cost; T0 = rows0 * RV, C = total cost.
     int32_t wt[2];
+    int64_t R, P[2];
     int64_t T0, C;
-    FastDiv divC, divW, divRV, divNpos[2], divWt[2];   // division by C, W, RV, grp[g].npos, wt[g]
+    FastDiv divC, divW, divRV, divNpos[2], divWt[2], divP[2];   // division by C, W, RV, grp[g].npos, wt[g], P[g]
     const int32_t *tokens;   // [B, gamma]
     // When set, the number of listed blocks is read from this device word at
     // launch (at most grp[g].nb, which then sizes the grid): rows, T, T0, C
@@ -218,6 +221,13 @@ cudaError_t launch_uniforms(uint64_t seed, const uint32_t *j, const uint32_t *b,
 // the entropy accumulator) and a target row (online softmax plus the rank
 // count), measured on GB300: 10 : 9.
 constexpr int32_t kCostDrafter = 10, kCostTarget = 9;
+// Extra cost of a row's first vector, in vectors of the heavier group: the
+// end of a warp's piece of a row (exact argmax re-read, reduction, partial)
+// and the next piece's start.  Per-warp globaltimer stamps (one 16-block
+// round): warps whose range crosses a row boundary ended 3.2 us after those
+// whose range does not.  Measured on GB300 (16-block round, back to back):
+// 0 -> 69.08 us, 200 -> 68.68, 400 -> 68.62, 700 -> 69.21.
+constexpr int64_t kRowStartVec = 400;
 
 // Warps of a launch over T vectors in `rows` rows with at most W_max warps:
 // at least two vectors per warp, so that with the cost weights every warp's
@@ -241,10 +251,22 @@ __host__ __device__ inline int32_t scan_warps(int64_t W_max, int64_t T, int64_t 
 inline void set_divisors(ScanParams &p) {
     const bool mixed = p.n_groups == 2 && p.grp[0].kind != p.grp[1].kind;
     for (int g = 0; g < 2; ++g) p.wt[g] = mixed ? (p.grp[g].kind == 0 ? kCostDrafter : kCostTarget) : 1;
+    const int64_t wmax = std::max(p.wt[0], p.wt[1]), wmin = std::min(p.wt[0], p.wt[1]);
+    // The row-start cost must leave every warp at least one vector start: a
+    // warp's share of the cost, at least a row's cost over kPiecesPerRow
+    // (scan_warps; also for a smaller device block count), has to exceed the
+    // largest single vector's cost R + wmax: wmin RV + R >= kPiecesPerRow
+    // (R + 2 wmax).  Rows too short for that (and too short to be cut at all)
+    // get no row-start cost.
+    int64_t R = kRowStartVec * wmax;
+    if (p.RV < 2 * kPiecesPerRow || wmin * p.RV + R < kPiecesPerRow * (R + 2 * wmax)) R = 0;
+    p.R = R;
+    for (int g = 0; g < 2; ++g) p.P[g] = p.wt[g] * p.RV + R;
     p.T0 = p.rows0 * p.RV;
-    p.C = p.wt[0] * p.T0 + p.wt[1] * (p.T - p.T0);
+    p.C = p.rows0 * p.P[0] + (p.rows - p.rows0) * p.P[1];
     p.divC = make_fastdiv(static_cast<uint64_t>(p.C > 0 ? p.C : 1));
     for (int g = 0; g < 2; ++g) p.divWt[g] = make_fastdiv(static_cast<uint64_t>(p.wt[g]));
+    for (int g = 0; g < 2; ++g) p.divP[g] = make_fastdiv(static_cast<uint64_t>(p.P[g] > 0 ? p.P[g] : 1));
     p.divW = make_fastdiv(static_cast<uint64_t>(p.W > 0 ? p.W : 1));
     p.divRV = make_fastdiv(static_cast<uint64_t>(p.RV > 0 ? p.RV : 1));
     for (int g = 0; g < 2; ++g) p.divNpos[g] = make_fastdiv(static_cast<uint64_t>(p.grp[g].npos > 0 ? p.grp[g].npos : 1));
@@ -323,7 +345,7 @@ __device__ __forceinline__ PartView part_view(const ScanParams &p) {
     v.rows = v.rows0 + (p.n_groups > 1 ? v.nb * p.grp[1].npos : 0);
     v.T = v.rows * p.RV;
     v.T0 = v.rows0 * p.RV;
-    v.C = p.wt[0] * v.T0 + p.wt[1] * (v.T - v.T0);
+    v.C = v.rows0 * p.P[0] + (v.rows - v.rows0) * p.P[1];
     v.W = scan_warps(p.W, v.T, v.rows);
     v.divC = make_fastdiv_dev(static_cast<uint64_t>(v.C > 0 ? v.C : 1));
     v.divW = make_fastdiv_dev(static_cast<uint64_t>(v.W));
@@ -332,18 +354,30 @@ __device__ __forceinline__ PartView part_view(const ScanParams &p) {
 
 // Index arithmetic of the cost-balanced contiguous partition of the T
 // vectors over W warps.  Vector v occupies the cost interval [cost(v),
-// cost(v+1)) with cost(v) = wt0 min(v, T0) + wt1 max(v - T0, 0); warp w owns
-// the costs [floor(w C / W), floor((w+1) C / W)) and so the vectors whose
+// cost(v+1)): a group-g vector costs wt[g] and a row's first vector R more,
+// so cost(v) = (whole rows before v's row) + (R + k wt[g] for the k >= 1
+// vectors of v's row before it, 0 for k = 0), rows of group 0 first.  Warp w
+// owns the costs [floor(w C / W), floor((w+1) C / W)) and so the vectors whose
 // cost interval starts there: [start(w), start(w+1)) with start(w) the first
 // vector of cost >= floor(w C / W).  Requires C W < 2^53 (checked by the host).
 __device__ __forceinline__ int64_t part_start(const ScanParams &p, const PartView &v, int64_t w) {
     const int64_t c = fast_div(w * v.C, v.divW);
-    const int64_t c0 = p.wt[0] * v.T0;
-    return (c <= c0) ? fast_div(c + p.wt[0] - 1, p.divWt[0]) : v.T0 + fast_div(c - c0 + p.wt[1] - 1, p.divWt[1]);
+    const int64_t c0 = v.rows0 * p.P[0];   // the cost of group 0
+    const int g = (c <= c0) ? 0 : 1;
+    const int64_t cg = g ? c - c0 : c;
+    const int64_t r = fast_div(cg, p.divP[g]);   // whole rows of the group before it
+    const int64_t rem = cg - r * p.P[g];
+    int64_t k = 0;
+    if (rem > 0) k = (rem <= p.R) ? 1 : fast_div(rem - p.R + p.wt[g] - 1, p.divWt[g]);
+    return (g ? v.T0 : 0) + r * p.RV + k;
 }
 // The warp owning vector v.
 __device__ __forceinline__ int64_t part_owner(const ScanParams &p, const PartView &pv, int64_t v) {
-    const int64_t cost = (v < pv.T0) ? p.wt[0] * v : p.wt[0] * pv.T0 + p.wt[1] * (v - pv.T0);
+    const int g = (v < pv.T0) ? 0 : 1;
+    const int64_t u = g ? v - pv.T0 : v;
+    const int64_t r = fast_div(u, p.divRV);
+    const int64_t k = u - r * p.RV;
+    const int64_t cost = (g ? pv.rows0 * p.P[0] : 0) + r * p.P[g] + (k > 0 ? p.R + k * p.wt[g] : 0);
     return fast_div((cost + 1) * pv.W - 1, pv.divC);
 }
 

@@ -50,45 +50,103 @@ def test_partition_of_the_64x64_workload():
         assert fast_div(v % (64 * 129), fN) == (v % (64 * 129)) // 65
 
 
-def _weighted(T0, T1, W, w0, w1):
+def _weighted(T0, T1, W, w0, w1, RV=None, R=0):
     """The cost-balanced partition of the streaming kernel (part_start /
-    part_owner in csrc/internal.h), emulated with the same magic divisions."""
-    T, C = T0 + T1, w0 * T0 + w1 * T1
-    fW, fC, f0, f1 = make_fastdiv(W), make_fastdiv(C), make_fastdiv(w0), make_fastdiv(w1)
+    part_owner in csrc/internal.h), emulated with the same magic divisions:
+    rows of RV vectors (group 0: T0 vectors, then group 1: T1), a group-g
+    vector costing w_g and a row's first vector R more."""
+    RV = RV or 1
+    rows0, rows1 = T0 // RV, T1 // RV
+    assert rows0 * RV == T0 and rows1 * RV == T1
+    P = (w0 * RV + R, w1 * RV + R)
+    wt = (w0, w1)
+    T, C = T0 + T1, rows0 * P[0] + rows1 * P[1]
+    fW, fC, fRV = make_fastdiv(W), make_fastdiv(C), make_fastdiv(RV)
+    fWt = (make_fastdiv(w0), make_fastdiv(w1))
+    fP = (make_fastdiv(P[0]), make_fastdiv(P[1]))
+    c0 = rows0 * P[0]
 
     def start(w):
         c = fast_div(w * C, fW)
-        return fast_div(c + w0 - 1, f0) if c <= w0 * T0 else T0 + fast_div(c - w0 * T0 + w1 - 1, f1)
+        g = 0 if c <= c0 else 1
+        cg = c - c0 if g else c
+        r = fast_div(cg, fP[g])
+        rem = cg - r * P[g]
+        k = 0
+        if rem > 0:
+            k = 1 if rem <= R else fast_div(rem - R + wt[g] - 1, fWt[g])
+        return (T0 if g else 0) + r * RV + k
 
     def owner(v):
-        cost = w0 * v if v < T0 else w0 * T0 + w1 * (v - T0)
+        g = 0 if v < T0 else 1
+        u = v - T0 if g else v
+        r = fast_div(u, fRV)
+        k = u - r * RV
+        cost = (c0 if g else 0) + r * P[g] + (R + k * wt[g] if k > 0 else 0)
         return fast_div((cost + 1) * W - 1, fC)
-    return T, start, owner
+
+    def cost(v):   # plain definition: the costs of the vectors before v
+        tot = 0
+        for g, (lo, hi) in enumerate(((0, T0), (T0, T))):
+            for x in range(lo, min(v, hi)):
+                tot += wt[g] + (R if (x - lo) % RV == 0 else 0)
+        return tot
+    return T, start, owner, cost, C
 
 
 def test_cost_weighted_partition():
     rng = np.random.default_rng(2)
-    cases = [(16 * 32 * 18992, 16 * 33 * 18992, 2432, 10, 9),   # the 16 x 32 block workload, drafter rows first
-             (16 * 33 * 18992, 16 * 32 * 18992, 2432, 9, 10),   # target rows first
-             (5 * 1001, 0, 37, 1, 1), (3, 4, 3, 10, 9), (8, 9, 8, 10, 9)]
+    cases = [(16 * 32 * 18992, 16 * 33 * 18992, 2432, 10, 9, 18992, 0),   # the 16 x 32 block workload
+             (16 * 33 * 18992, 16 * 32 * 18992, 2432, 9, 10, 18992, 0),   # target rows first
+             (5 * 1001, 0, 37, 1, 1, 1001, 0), (3, 4, 3, 10, 9, 1, 0), (8, 9, 8, 10, 9, 1, 0),
+             (16 * 32 * 18992, 16 * 33 * 18992, 2432, 10, 9, 18992, 4000)]   # with a row-start cost
     for _ in range(20):
         T0, T1 = int(rng.integers(1, 50000)), int(rng.integers(1, 50000))
-        cases.append((T0, T1, int(rng.integers(1, (T0 + T1) // 2 + 1)), 10, 9))
-    for T0, T1, W, w0, w1 in cases:
-        if (w0, w1) != (1, 1):
+        cases.append((T0, T1, int(rng.integers(1, (T0 + T1) // 2 + 1)), 10, 9, 1, 0))
+    for _ in range(20):
+        # rows with a row-start cost inside the bound that set_divisors keeps
+        # (wmin RV + R >= 16 (R + 2 wmax)); W at most 16 per row
+        RV = int(rng.integers(32, 3000))
+        rows0, rows1 = int(rng.integers(1, 12)), int(rng.integers(0, 12))
+        R = int(rng.integers(0, max(1, (9 * RV - 16 * 20) // 15)))
+        W = int(rng.integers(1, 16 * (rows0 + rows1) + 1))
+        cases.append((rows0 * RV, rows1 * RV, W, 10, 9, RV, R))
+    for T0, T1, W, w0, w1, RV, R in cases:
+        if (w0, w1) != (1, 1) and R == 0:
             W = max(1, min(W, (T0 + T1) // 2))   # scan_warps: at least two vectors per warp
-        T, start, owner = _weighted(T0, T1, W, w0, w1)
+        T, start, owner, _, _ = _weighted(T0, T1, W, w0, w1, RV, R)
         s = [start(w) for w in range(W + 1)]
         assert s[0] == 0 and s[W] == T
-        assert all(s[w + 1] > s[w] for w in range(W)), "empty warp"
+        assert all(s[w + 1] > s[w] for w in range(W)), ("empty warp", T0, T1, W, RV, R)
         probe = set(rng.integers(0, T, 2000).tolist()) | {x for x in s[:-1]} | {x - 1 for x in s[1:]}
         for v in probe:
             w = owner(int(v))
             assert s[w] <= v < s[w + 1], (T0, T1, W, v, w)
     # balance: each warp's cost is within one vector's cost of C / W
     T0, T1, W = 16 * 32 * 18992, 16 * 33 * 18992, 2432
-    T, start, owner = _weighted(T0, T1, W, 10, 9)
-    cost = lambda v: 10 * min(v, T0) + 9 * max(v - T0, 0)
-    per = [cost(start(w + 1)) - cost(start(w)) for w in range(W)]
-    C = cost(T)
-    assert max(per) - min(per) <= 2 * 10 and abs(sum(per) - C) == 0
+    for R in (0, 4000):
+        T, start, owner, _, C = _weighted(T0, T1, W, 10, 9, 18992, R)
+        cost = lambda v: (10 * min(v, T0) + 9 * max(v - T0, 0)
+                          + R * (-(-min(v, T0) // 18992) + -(-max(v - T0, 0) // 18992)))
+        per = [cost(start(w + 1)) - cost(start(w)) for w in range(W)]
+        assert max(per) - min(per) <= 2 * (10 + R) and sum(per) == C
+
+
+def test_partition_cost_against_its_definition():
+    """cost(v) in part_owner equals the plain sum of the vectors' costs."""
+    rng = np.random.default_rng(5)
+    for _ in range(30):
+        RV = int(rng.integers(1, 40))
+        rows0, rows1 = int(rng.integers(0, 5)), int(rng.integers(0, 5))
+        if rows0 + rows1 == 0:
+            continue
+        R = int(rng.integers(0, 50))
+        T0, T1 = rows0 * RV, rows1 * RV
+        T, start, owner, cost, C = _weighted(T0, T1, 1, 10, 9, RV, R)
+        assert cost(T) == C
+        for w_ in (2, 3, 7):
+            T, start, owner, cost, C = _weighted(T0, T1, w_, 10, 9, RV, R)
+            for v in range(T):
+                # the owner of v: the warp whose cost interval holds cost(v)
+                w = owner(v)
+                assert (w * C) // w_ <= cost(v) < ((w + 1) * C) // w_, (RV, R, v)
