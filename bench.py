@@ -18,7 +18,7 @@ Prints one JSON line (rank 0).
 
 Other rows of the path, one JSON line each (not the fused-round contract line):
   python bench.py --component mlp [--steps K]   the survival scorer alone (K launches)
-  python bench.py --component loop [--steps R]  the decode-loop workload (R rounds, default 64)
+  python bench.py --component loop [--steps R]  the decode-loop workload (R rounds, default 256)
   python bench.py --component features          drafter confidence with / without the extended features
   python bench.py --component scorer [--steps K] the deep scorer (K calls)
   python bench.py --component diag              the permutation diagnostic (Table 1 settings)
