@@ -360,11 +360,11 @@ def run_gpu(args):
     from paper_2608_14787_gb300 import shard, synth
 
     ws, rank, local = _dist()
+    torch.cuda.set_device(local)   # before the process group: NCCL binds each rank to its current device
+    dev = torch.device("cuda", local)
     if ws > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
     if rank == 0:
         sdd_build.build()
     if ws > 1:
