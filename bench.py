@@ -490,7 +490,9 @@ def run_gpu(args):
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if esz == 2 else "fp32", "data": "synthetic",
+            # the arithmetic of the path: fp32 with double-float (fp32 pairs) sums
+            # and normalisers; the logits' storage type is config.dtype
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {**_config_json(wl, ells, ks, n_sets),
                        "launch": (f"CUDA graph of {args.graph} rounds, replayed" if args.graph
                                   else "one call per kernel, queued behind a device spin")},
