@@ -115,6 +115,25 @@ def test_sharded_greedy_and_ragged_fp32():
     _same_as_one_gpu(ranks, blk, taus, ells, ks, True, 7, 1, 2, ob)
 
 
+def test_sharded_rounds_reuse_their_workspaces():
+    """The same ranks (workspaces, arrival counters) serve two rounds in a
+    row: the draw's counters are left at zero by every call, so the second
+    round matches the oracle as the first does."""
+    blk = synth.make_block("c3", device="cuda", B=5, gamma=12, V=40_000, round_=9)
+    taus, ells, ks = (0.6,), (0.5,), (3,)
+    bounds = vocab_shard.slice_bounds(40_000, 3)
+    ranks = [vocab_shard.ShardRound(5, 12, 40_000, v0, v1, dtype=blk.z_d.dtype, taus=taus, ells=ells, ks=ks, K_min=2)
+             for v0, v1 in bounds]
+    sd = [vocab_shard.slice_logits(blk.z_d, v0, v1) for v0, v1 in bounds]
+    st = [vocab_shard.slice_logits(blk.z_t, v0, v1) for v0, v1 in bounds]
+    for seed, round_ in ((7, 1), (8, 2)):
+        vocab_shard.run_local(ranks, sd, st, blk.x, seed=seed, round_=round_)
+        torch.cuda.synchronize()
+        for r in ranks:
+            assert int(r.status.item()) == 0
+        _compare_with_oracle(ranks[0], blk, taus, ells, ks, False, seed, round_, 2)
+
+
 def test_sharded_bonus_draw_identical_rows():
     """p_t = p_d: every position accepts and the bonus token is drawn from p_t
     of row gamma + 1 across the slices (Sec. 3.1)."""
