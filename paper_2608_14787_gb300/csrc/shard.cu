@@ -24,8 +24,9 @@ namespace sdd {
 namespace {
 
 // One CTA of four warps per row and eight CTAs per SM (64 registers): a c3
-// slice holds 1,040 rows, one wave on 152 SMs.  (256 threads at 4 CTAs per
-// SM: 84 us per half-vocabulary slice, against 58 us.)
+// slice holds 1,040 rows, one wave on 152 SMs.  (With 256-thread CTAs, four
+// per SM, and per-thread candidate lists in shared memory, a half-vocabulary
+// slice took 84 us; as here, ~55 us.)
 constexpr int kShardThreads = 128;
 constexpr int kShardMinCtas = 8;
 constexpr int kShardU = 4;   // 16-byte vectors per thread in flight
