@@ -565,6 +565,36 @@ SDD_API sdd_status_t sdd_block_scan(const sdd_block_args *args, sdd_stream_t str
 SDD_API sdd_status_t sdd_block_decide(const sdd_block_args *args, sdd_stream_t stream);
 
 /*
+ * sdd_block_pipelined -- rounds of sdd_block over independent batches, two at
+ * a time in one launch: the streaming pass of `next` and, on the same SMs,
+ * the decide work (sdd_block_decide's) of `prev`, whose streaming pass ran
+ * in the previous sdd_block_pipelined call on this stream.  The decide work
+ * of a round is latency-bound (row finalisation, the rules, the sampling
+ * draw); beside the next round's streaming pass it costs little of the
+ * memory bandwidth, instead of leaving the memory system idle behind its own
+ * pass.  A sequence of rounds r_0 .. r_n on one stream runs as
+ *     sdd_block_pipelined(&r_0, NULL), sdd_block_pipelined(&r_1, &r_0), ...,
+ *     sdd_block_pipelined(&r_n, &r_(n-1)), sdd_block_pipelined(NULL, &r_n);
+ * the outputs of r_i are complete when the work of the call that names it as
+ * prev has completed.
+ *   next -- args as for sdd_block (NULL: decide prev only, the last call).
+ *   prev -- the args that were `next` in the previous call on this stream,
+ *           unchanged, with their inputs still in place (the draw reads two
+ *           of its rows again) and its workspace untouched since (NULL: the
+ *           first call).  Its streaming pass must have been made by this
+ *           call: the pipelined pass divides the rows among warps
+ *           differently from sdd_block_scan.
+ * next and prev must use different workspaces and different output arrays.
+ * Results are those of sdd_block on the same args: the same decisions and
+ * tokens (outside the 1e-6 near-threshold band of the float comparisons) and
+ * the same statistics up to rounding (the rows' pieces differ).
+ * Errors: SDD_ERR_INVALID_ARGUMENT for both NULL, a shared workspace or any
+ * error of sdd_block's arguments; as sdd_block otherwise.
+ */
+SDD_API sdd_status_t sdd_block_pipelined(const sdd_block_args *next, const sdd_block_args *prev,
+                                         sdd_stream_t stream);
+
+/*
  * Vocabulary-sharded round (a tensor-parallel LM head).  The paper runs its
  * verifier on one GPU and reads its logits in fp32 (App. A.8); when the
  * drafter's and verifier's logits are instead split by vocabulary over S

@@ -6,7 +6,7 @@ include/sdd.h); this package holds its build step, a ctypes binding with the
 same entry-point names, and the seeded synthetic-input generators.
 """
 from .binding import (  # noqa: F401
-    BlockRound, Confidence, SddError, Workspace, agreement, commit, confidence, confidence_buffers, confidence_noalloc,
+    BlockRound, Confidence, SddError, Workspace, agreement, block_pipelined, commit, confidence, confidence_buffers, confidence_noalloc,
     load, new_status,
     permutation_diagnostic, position_metrics, schedule_periodic, schedule_prefix, scorer_deep, scorer_features, scorer_workspace,
     select_rows, status_from_device, survival_mlp, test_wait_hooks, uniforms, verify_lenient, verify_strict, verify_strict_listed,

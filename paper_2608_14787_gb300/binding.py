@@ -125,6 +125,8 @@ def load(path: str | None = None):
     L.sdd_shard_draw.restype = I
     for fn in ("sdd_block", "sdd_block_scan", "sdd_block_decide"):
         getattr(L, fn).argtypes = [ctypes.POINTER(BlockArgs), VP]
+    L.sdd_block_pipelined.argtypes = [ctypes.POINTER(BlockArgs), ctypes.POINTER(BlockArgs), VP]
+    L.sdd_block_pipelined.restype = I
     for fn in ("sdd_workspace_size", "sdd_confidence", "sdd_confidence_features", "sdd_schedule_prefix",
                "sdd_schedule_periodic",
                "sdd_verify_strict",
@@ -653,3 +655,15 @@ class BlockRound:
 
     def decide(self, stream=None):
         _check(load().sdd_block_decide(ctypes.byref(self.args), _stream(stream)), "sdd_block_decide")
+
+
+def block_pipelined(nxt, prev, stream=None):
+    """sdd_block_pipelined: the streaming pass of BlockRound `nxt` and the
+    decide work of BlockRound `prev` (streamed by the previous call on this
+    stream) in one launch; either may be None (the first and the last call of
+    a sequence).  The two rounds must be different BlockRound objects."""
+    if nxt is not None and nxt is prev:
+        raise ValueError("next and prev must be different BlockRound objects")
+    a = None if nxt is None else ctypes.byref(nxt.args)
+    b = None if prev is None else ctypes.byref(prev.args)
+    _check(load().sdd_block_pipelined(a, b, _stream(stream)), "sdd_block_pipelined")

@@ -52,6 +52,7 @@ sdd_status_t device_info(DevInfo &out) {
         if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
         e = scan_prepare_device();
         if (e == cudaSuccess) e = decide_prepare_device();
+        if (e == cudaSuccess) e = pipe_prepare_device();
         if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
         di.ctas_per_sm = scan_max_ctas_per_sm();
         if (di.ctas_per_sm < 1) return fail(SDD_ERR_UNSUPPORTED, "streaming kernel does not fit on this device");
@@ -185,10 +186,19 @@ sdd_status_t run_decide_shard(const ScanParams &p, cudaStream_t stream) {
     return SDD_OK;
 }
 
-// Block decisions and, for the sampling rule, the draw geometry: each of the
-// nb blocks' draw rows is cut into nseg segments of whole kDecThreads-vector
-// chunks, as many as keep nb * nseg CTAs resident in one wave (at least two
-// vectors per thread, at most kDrawMaxSeg segments).
+// The draw geometry of nb blocks over `budget` decide teams of nt threads:
+// each draw row of RV vectors is cut into nseg segments of whole nt-vector chunks, as
+// many as keep nb * nseg teams within the budget (at least two vectors per
+// thread, at most kDrawMaxSeg segments).
+void draw_segments(int RV, int nb, int budget, int nt, int32_t &nseg, int32_t &seg_vec) {
+    const int want = std::max(1, std::min(kDrawMaxSeg, budget / std::max(nb, 1)));
+    const int per_thread = std::max(2, (RV + nt * want - 1) / (nt * want));
+    seg_vec = per_thread * nt;
+    nseg = (RV + seg_vec - 1) / seg_vec;
+}
+
+// Block decisions and, for the sampling rule, the draw geometry over the
+// decide CTAs resident in one wave.
 void init_dec(DecideParams &d, const Work &w, sdd_dtype_t dtype, int B, int gamma, int V, int64_t row_stride,
               const int32_t *tokens, int nb) {
     d.enabled = 1;
@@ -201,10 +211,7 @@ void init_dec(DecideParams &d, const Work &w, sdd_dtype_t dtype, int B, int gamm
     d.res_count = reinterpret_cast<uint32_t *>(w.base + w.L.res_count);
     d.dec_ctas = w.dec_ctas;
     const int RV = static_cast<int>((static_cast<int64_t>(V) * esize(dtype) + 15) / 16);
-    const int want = std::max(1, std::min(kDrawMaxSeg, w.dec_ctas / std::max(nb, 1)));
-    const int per_thread = std::max(2, (RV + kDecThreads * want - 1) / (kDecThreads * want));
-    d.seg_vec = per_thread * kDecThreads;
-    d.nseg = (RV + d.seg_vec - 1) / d.seg_vec;
+    draw_segments(RV, nb, w.dec_ctas, kDecThreads, d.nseg, d.seg_vec);
 }
 
 sdd_status_t set_thresholds(int signal, const double *eta_b, const double *eta_c, int n_tau, df *eta_loc,
@@ -1124,6 +1131,42 @@ sdd_status_t sdd_block_decide(const sdd_block_args *a, sdd_stream_t stream) {
 sdd_status_t sdd_block(const sdd_block_args *a, sdd_stream_t stream) {
     SDD_TRY(sdd_block_scan(a, stream));
     return sdd_block_decide(a, stream);
+}
+
+// A pipelined round's launch parameters: sdd_block's, streamed by warps
+// kPipeWarps..15 of each CTA (the same when the round is streamed and when it
+// is decided).
+static sdd_status_t pipe_params(const sdd_block_args *a, ScanParams &p, bool *empty) {
+    SDD_TRY(block_params(a, p, empty));
+    if (*empty) return SDD_OK;
+    Work w;
+    SDD_TRY(get_work(a->workspace, a->workspace_bytes, a->B, a->gamma, w));
+    const int wpc = kWarpsPerCta - kPipeWarps;
+    p.W = scan_warps(w.W_max / kWarpsPerCta * wpc, p.T, p.rows);
+    set_divisors(p);
+    p.warp0 = kPipeWarps;
+    p.wpc = wpc;
+    return SDD_OK;
+}
+
+sdd_status_t sdd_block_pipelined(const sdd_block_args *next, const sdd_block_args *prev, sdd_stream_t stream) {
+    if (!next && !prev) return fail(SDD_ERR_INVALID_ARGUMENT, "next and prev are both NULL");
+    if (next && prev && next->B > 0 && prev->B > 0 && next->workspace == prev->workspace)
+        return fail(SDD_ERR_INVALID_ARGUMENT, "next and prev share a workspace");
+    ScanParams pn, pp;
+    bool en = true, ep = true;
+    if (next) SDD_TRY(pipe_params(next, pn, &en));
+    if (prev) SDD_TRY(pipe_params(prev, pp, &ep));
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (en) return ep ? SDD_OK : run_decide(pp, st);   // the last round of a sequence: decide only
+    if (static_cast<double>(pn.C) * static_cast<double>(pn.W) >= 9.007199254740992e15)   // 2^53
+        return fail(SDD_ERR_UNSUPPORTED, "%lld vectors of logits exceed the index arithmetic", (long long)pn.T);
+    const int grid = static_cast<int>((static_cast<int64_t>(pn.W) + pn.wpc - 1) / pn.wpc);
+    // prev's draw segments over this grid's CTAs, one (block, segment) item each
+    if (!ep) draw_segments(pp.RV, pp.grp[0].nb, grid, kPipeTeam, pp.dec.nseg, pp.dec.seg_vec);
+    const cudaError_t e = launch_pipe(&pn, ep ? nullptr : &pp, grid, st);
+    if (e != cudaSuccess) return cuda_fail(e, "pipelined round launch");
+    return SDD_OK;
 }
 
 }  // extern "C"

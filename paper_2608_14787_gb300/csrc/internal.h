@@ -19,7 +19,9 @@ constexpr int kVPL = 8;                       // 16-byte vectors per lane per ti
 constexpr int kTileVec = 32 * kVPL;           // vectors per warp tile
 constexpr int kTileBytes = kTileVec * 16;     // 4 KiB
 constexpr int kStages = 2;
-constexpr int kScanSmem = kWarpsPerCta * kStages * kTileBytes + kWarpsPerCta * kStages * 8;
+// Shared memory of the rings of `warps` streaming warps with `stages` tiles each.
+constexpr int ring_bytes(int stages, int warps) { return warps * stages * (kTileBytes + 8); }
+constexpr int kScanSmem = ring_bytes(kStages, kWarpsPerCta);
 constexpr uint32_t kWaitPolls = 1u << 24;     // bounded mbarrier wait (seconds of polling)
 
 // Division by a per-launch constant d >= 1 without the 64-bit integer division
@@ -145,6 +147,11 @@ struct ScanParams {
     int64_t R, P[2];
     int64_t T0, C;
     FastDiv divC, divW, divRV, divNpos[2], divWt[2], divP[2];   // division by C, W, RV, grp[g].npos, wt[g], P[g]
+    // The streaming warps of a CTA: warps warp0 .. warp0 + wpc - 1, global
+    // streaming warp blockIdx.x * wpc + (warp - warp0) (set_divisors: all 16;
+    // the pipelined round: warps 4-15, warps 0-3 run the previous round's
+    // decide work).
+    int32_t warp0, wpc;
     const int32_t *tokens;   // [B, gamma]
     // When set, the number of listed blocks is read from this device word at
     // launch (at most grp[g].nb, which then sizes the grid): rows, T, T0, C
@@ -185,6 +192,9 @@ void set_scan_wait_hooks(uint32_t polls, int drop_copy);
 // The decide kernel over (listed blocks, p.dec.nseg) CTAs, launched as a
 // programmatic dependent of the streaming kernel.
 cudaError_t launch_decide(const ScanParams &p, cudaStream_t stream);
+// The pipelined round (pipe.cu): next's streaming pass over `grid` CTAs and,
+// on warps 0-3 of the same CTAs, prev's decide work (either may be null).
+cudaError_t launch_pipe(const ScanParams *next, const ScanParams *prev, int grid, cudaStream_t stream);
 cudaError_t launch_schedule(const ScheduleParams &p, cudaStream_t stream);
 // Vocabulary-sharded path (shard.cu): the slice's per-row records, and the
 // draw once every slice's draw-row mass is known.
@@ -245,9 +255,16 @@ __host__ __device__ inline int32_t scan_warps(int64_t W_max, int64_t T, int64_t 
     return static_cast<int32_t>(w > 1 ? w : 1);
 }
 
+// The pipelined round (sdd_block_pipelined): warps 0-3 of every CTA (a team
+// of kPipeTeam threads) run the previous round's decide work while warps
+// 4-15 stream (twelve streaming warps keep an SM's share of the memory
+// bandwidth nearly whole, eight do not).
+constexpr int kPipeTeam = 128;
+constexpr int kPipeWarps = kPipeTeam / 32;
+
 // The cost weights and division constants of a launch whose groups, rows, T
-// and W are set (host).  The magic divisions are exact while C * W < 2^53
-// (the callers check it).
+// and W are set (host), all 16 warps of a CTA streaming.  The magic divisions
+// are exact while C * W < 2^53 (the callers check it).
 inline void set_divisors(ScanParams &p) {
     const bool mixed = p.n_groups == 2 && p.grp[0].kind != p.grp[1].kind;
     for (int g = 0; g < 2; ++g) p.wt[g] = mixed ? (p.grp[g].kind == 0 ? kCostDrafter : kCostTarget) : 1;
@@ -270,6 +287,8 @@ inline void set_divisors(ScanParams &p) {
     p.divW = make_fastdiv(static_cast<uint64_t>(p.W > 0 ? p.W : 1));
     p.divRV = make_fastdiv(static_cast<uint64_t>(p.RV > 0 ? p.RV : 1));
     for (int g = 0; g < 2; ++g) p.divNpos[g] = make_fastdiv(static_cast<uint64_t>(p.grp[g].npos > 0 ? p.grp[g].npos : 1));
+    p.warp0 = 0;
+    p.wpc = kWarpsPerCta;
 }
 
 // Offline diagnostics (diag.cu).  perm: [n_rep, gamma, B] int32 scratch;
@@ -299,6 +318,7 @@ int scan_max_ctas_per_sm();
 int decide_max_ctas_per_sm();
 cudaError_t scan_prepare_device();
 cudaError_t decide_prepare_device();
+cudaError_t pipe_prepare_device();
 void set_last_error(const char *msg);  // message returned by sdd_last_error()
 
 __device__ __forceinline__ int64_t fast_div(int64_t n, const FastDiv &f) {

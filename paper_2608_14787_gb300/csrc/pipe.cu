@@ -1,0 +1,145 @@
+// pipe.cu -- the pipelined round (sdd_block_pipelined): one launch that
+// streams round n's logits and, on the same SMs, finishes round n-1.
+//
+// A round of the fused path is a streaming pass (every logit once, HBM-bound)
+// followed by the decide work (row finalisation, the acceptance rules, the
+// schedule, the sampling draw), which is latency-bound: behind its own
+// streaming pass it leaves the memory system idle for most of its ~12 us.
+// Rounds over independent batches need not wait for one another, so here the
+// decide work of round n-1 runs beside the streaming pass of round n: in every
+// CTA, warps 0-3 do one (block, draw segment) item of round n-1's decide work
+// (decide_cta with a team of kPipeTeam threads and its barrier over those
+// threads only) while warps 4-15 stream round n, the rows divided among
+// twelve warps per CTA.  Measured on GB300 (16 blocks of 32 positions, V =
+// 151,936 bf16, back to back): 63.9 us per round against 68.8 us for the
+// streaming and decide kernels in turn.  Twelve streaming warps keep most of
+// an SM's share of the memory bandwidth, eight do not: a team of eight decide
+// warps (which then streamed a share cut to its decide time) gave 71-75 us;
+// under the concurrent stream a decide item takes ~27 us (43 us for the
+// teams that also locate the draw), all of it before the streaming ends.
+// Round n-1's partials were written by the previous launch on the stream,
+// which has completed when this grid passes griddepcontrol.wait.
+#include <algorithm>
+#include <atomic>
+#include <cstring>
+
+#include "scan.cuh"
+#include "decide.cuh"
+
+namespace sdd {
+
+namespace {
+
+struct PipeParams {
+    ScanParams next;    // the round streamed by this launch (unused when has_next == 0)
+    ScanParams prev;    // the round decided by this launch (unused when has_prev == 0)
+    int32_t has_next, has_prev;
+    int32_t n_items;    // decide items of prev: blocks x draw segments
+    int32_t stage;      // a team stages its draw segment in shared memory
+};
+
+// Warps 0-3 (kPipeTeam threads): prev's decide items of this CTA.  Out of
+// line, so that its register allocation stays apart from the streaming loop's.
+template <int DT>
+__device__ __noinline__ void pipe_decide(const PipeParams &pp, float *s_pref_all) {
+    const ScanParams &p = pp.prev;
+    const PartView pv = part_view(p);
+    // after the segments' prefixes: the staged draw segment (16-byte aligned)
+    uint4 *s_stage = pp.stage ? reinterpret_cast<uint4 *>(s_pref_all + p.dec.nseg * kPipeTeam) : nullptr;
+    for (int item = blockIdx.x; item < pp.n_items; item += gridDim.x) {
+        const DecGeom geo{item / p.dec.nseg, item % p.dec.nseg, p.dec.nseg, p.dec.seg_vec};
+        decide_cta<DT, false, false, kPipeTeam>(p, pv, geo, s_pref_all, s_stage);
+        dec_sync<kPipeTeam>();   // the team's shared memory serves its next item
+    }
+}
+
+// The streaming warps' rings, indexed by streaming warp (twelve per CTA):
+// two stages each, as in the streaming kernel (three measured slower here
+// too: 64.5 against 63.9 us per round).
+constexpr int kPipeStages = 2;
+constexpr int kPipeRings = ring_bytes(kPipeStages, kWarpsPerCta - kPipeWarps);
+
+// DTN, DTP: the logits' types of next and prev (rounds of either type may
+// follow one another).
+template <int DTN, int DTP>
+__global__ void __launch_bounds__(kThreads, 1) pipe_kernel(const __grid_constant__ PipeParams pp) {
+    extern __shared__ __align__(128) unsigned char smem[];
+    // behind the previous launch on the stream (it streamed prev)
+    griddep_wait();
+    if (pp.has_prev && threadIdx.x < kPipeTeam)
+        pipe_decide<DTP>(pp, reinterpret_cast<float *>(smem + kPipeRings));   // [nseg][kPipeTeam] after the rings
+    const int warp = threadIdx.x >> 5;
+    if (pp.has_next && warp >= pp.next.warp0) {
+        const int64_t gw = static_cast<int64_t>(blockIdx.x) * pp.next.wpc + (warp - pp.next.warp0);
+        if (gw < pp.next.W)
+            scan_warp<DTN, false, kPipeStages>(pp.next, smem, gw, warp - pp.next.warp0, pp.next.wpc);
+    }
+}
+
+using PipeKernel = void (*)(PipeParams);
+const PipeKernel kPipeKernels[2][2] = {{pipe_kernel<SDD_F32, SDD_F32>, pipe_kernel<SDD_F32, SDD_BF16>},
+                                       {pipe_kernel<SDD_BF16, SDD_F32>, pipe_kernel<SDD_BF16, SDD_BF16>}};
+
+// The dynamic shared memory a pipelined launch may use on this device (the
+// per-block opt-in limit less the kernels' static shared memory).
+std::atomic<int> g_pipe_smem{0};
+
+}  // namespace
+
+cudaError_t pipe_prepare_device() {
+    int dev = 0, optin = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    size_t stat = 0;
+    for (const auto &row : kPipeKernels)
+        for (PipeKernel k : row) {
+            cudaFuncAttributes fa;
+            if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, k);
+            if (e == cudaSuccess) stat = std::max(stat, fa.sharedSizeBytes);
+        }
+    if (e != cudaSuccess) return e;
+    const int dyn = optin - static_cast<int>(stat);
+    for (const auto &row : kPipeKernels)
+        for (PipeKernel k : row) {
+            e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+            if (e != cudaSuccess) return e;
+        }
+    g_pipe_smem.store(dyn, std::memory_order_relaxed);
+    return cudaSuccess;
+}
+
+// grid: the streaming grid of next (or, without next, enough CTAs for the
+// decide items); prev->dec.nseg / seg_vec: the draw segments of prev's blocks
+// over that grid (one item per CTA while they fit).
+cudaError_t launch_pipe(const ScanParams *next, const ScanParams *prev, int grid, cudaStream_t stream) {
+    PipeParams pp;
+    std::memset(&pp, 0, sizeof pp);
+    if (next) {
+        pp.next = *next;
+        pp.has_next = 1;
+        pp.next.wait_polls = kWaitPolls;
+    }
+    size_t smem = kPipeRings;
+    if (prev) {
+        pp.prev = *prev;
+        pp.has_prev = 1;
+        const bool draw = prev->dec.enabled && prev->dec.do_strict && !prev->dec.greedy;
+        const int nseg = draw ? prev->dec.nseg : 1;
+        pp.prev.dec.nseg = nseg;
+        pp.n_items = prev->grp[0].nb * nseg;
+        if (draw) {
+            smem += static_cast<size_t>(nseg) * kPipeTeam * sizeof(float);
+            // both draw rows' segments, when they fit beside the rings
+            const size_t stage = 2 * static_cast<size_t>(prev->dec.seg_vec) * 16;
+            if (smem + stage <= static_cast<size_t>(g_pipe_smem.load(std::memory_order_relaxed))) {
+                smem += stage;
+                pp.stage = 1;
+            }
+        }
+    }
+    if (grid <= 0) return cudaSuccess;
+    const int dn = (next ? next->dtype : prev->dtype) == SDD_BF16, dp = (prev ? prev->dtype : next->dtype) == SDD_BF16;
+    return launch_dependent(kPipeKernels[dn][dp], dim3(grid), dim3(kThreads), smem, stream, pp);
+}
+
+}  // namespace sdd

@@ -176,3 +176,17 @@ def test_shard_arguments_rejected_on_host(lib):
     up = lambda v: (v + 15) // 16 * 16   # noqa: E731
     want = up(up(up(5 * 32) + 5 * 4) + 5 * 64 * 4) + 5 * 64 * 256 * 4
     assert lib.sdd_shard_workspace_size(5, ctypes.byref(n)) == 0 and n.value == want
+
+
+def test_pipelined_arguments_rejected_on_host(lib):
+    from paper_2608_14787_gb300.binding import BlockArgs
+    assert lib.sdd_block_pipelined(None, None, None) == 1
+    assert b"both NULL" in lib.sdd_last_error()
+    a, b = BlockArgs(), BlockArgs()
+    for x in (a, b):
+        x.dtype, x.B, x.gamma, x.V, x.row_stride = 1, 2, 4, 1000, 1000
+        x.draft_logits = x.target_logits = x.draft_tokens = 256
+        x.workspace = 4096
+    # two rounds in flight cannot share one workspace
+    assert lib.sdd_block_pipelined(ctypes.byref(a), ctypes.byref(b), None) == 1
+    assert b"workspace" in lib.sdd_last_error()
