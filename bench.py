@@ -4,7 +4,11 @@ One step = one fused round of the whole path over one batch of draft blocks:
 confidence statistics of every drafter row, the prefix skip schedule, strict
 (shadow) verification of every block with residual / bonus resampling,
 lenience and top-k acceptance on the same target read, agreement counters and
-the committed tokens (``sdd_block`` = ``sdd_block_scan`` + ``sdd_block_decide``).
+the committed tokens.  Rounds over independent batches are pipelined
+(``sdd_block_pipelined``): each launch streams one round's logits and, on four
+warps of every CTA, finishes the round before; K steps are K launches and one
+closing decide.  The same rounds run unpipelined (``sdd_block_scan`` then
+``sdd_block_decide``) are reported beside them.
 
 Default workload (c3): B=16 blocks, gamma=32, V=151,936, bf16 drafter and
 target logits; half the positions peaked, half flat; strict sampling, lenience
@@ -40,10 +44,12 @@ sys.path.insert(0, ROOT)
 METRIC = "draft blocks verified+scheduled/sec at γ=32,V=151,936 bf16; achieved HBM GB/s vs peak"
 UNIT = "blocks/s"
 NEAR = 1e-6
-# dram__bytes_read.sum + dram__bytes_write.sum of one scan_kernel launch on the
-# c3 workload (318,294,528 B + 3,656,960 B), from one ncu capture of the kernel
-# as it stands; reported as the roofline's "traffic" for that workload only.
+# dram__bytes_read.sum + dram__bytes_write.sum of one launch on the c3
+# workload, from one ncu capture of the kernel as it stands; reported as the
+# "traffic" of that workload's rooflines only: the streaming kernel
+# (318,294,528 B + 3,656,960 B) and the pipelined round's kernel.
 SCAN_TRAFFIC_C3 = 321_951_488
+PIPE_TRAFFIC_C3 = None
 
 
 def _peaks():
@@ -375,12 +381,98 @@ def run_gpu(args):
     B, gamma, V = wl.B, wl.gamma, wl.V
     n_sets = max(1, args.sets)
     sets = [synth.make_block(wl, device=dev, round_=r + 1000 * rank) for r in range(n_sets)]
-    rnd = sdd.BlockRound(B, gamma, V, dtype=wl.dtype, taus=wl.taus, ells=ells, ks=ks, K_min=6, S_max=64,
-                         device=dev)
+    pair = tuple(sdd.BlockRound(B, gamma, V, dtype=wl.dtype, taus=wl.taus, ells=ells, ks=ks, K_min=6, S_max=64,
+                                device=dev) for _ in range(2))
+    rnd = pair[0]
     esz = 2 if wl.dtype == torch.bfloat16 else 4
     scan_bytes = (2 * gamma + 1) * V * esz * B          # every logit read once
+    draw_bytes = 2 * V * esz * B                         # the decide's two draw rows per block
     stream = torch.cuda.current_stream()
+    props = torch.cuda.get_device_properties(dev)
+    bus = getattr(props, "pci_bus_id", None)
 
+    # A step is one round over one batch.  Rounds over independent batches are
+    # pipelined (sdd_block_pipelined): launch i streams round i and, on four
+    # warps of each CTA, finishes round i - 1; a last call finishes the last
+    # round.  K steps = K launches + that last call, all inside the region.
+    def pstep(i):
+        r = pair[i % 2]
+        s = sets[i % n_sets]
+        r.set_inputs(s.z_d, s.z_t, s.x, seed=wl.seed, round_=i)
+        sdd.block_pipelined(r, pair[(i - 1) % 2] if i > 0 else None)
+
+    def pflush(i_last):
+        sdd.block_pipelined(None, pair[i_last % 2])
+
+    def pipelined_region(k, first):
+        """k pipelined steps (rounds first .. first + k - 1) and the closing
+        decide under one event pair; also an event before the closing decide
+        (the k launches' own span)."""
+        t0, t_mid, t1 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+        torch.cuda._sleep(int(args.prefill_us * 2.0e3))    # ~prefill_us at 2 GHz: rounds queue behind it
+        t0.record(stream)
+        for i in range(k):
+            pstep(first + i)
+        t_mid.record(stream)
+        pflush(first + k - 1)
+        t1.record(stream)
+        torch.cuda.synchronize()
+        return t0.elapsed_time(t1), t0.elapsed_time(t_mid)
+
+    graph = None
+    if args.graph:
+        # small rounds outrun the host's launches: the timed steps replay a CUDA
+        # graph of --graph pipelined steps (an even number, so that a replay's
+        # first launch finishes the round the previous replay streamed last)
+        if args.graph % 2 or args.steps % args.graph:
+            raise SystemExit("--graph must be even and divide --steps")
+        for i in range(args.warmup):
+            pstep(i)
+        side = torch.cuda.Stream(device=dev)
+        side.wait_stream(stream)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=side):
+            for j in range(args.graph):
+                pstep(args.warmup + j)
+        for _ in range(2):
+            graph.replay()
+        last = args.warmup + args.graph - 1
+
+        def pipelined_region(k, first):   # noqa: F811 -- the graph's rounds replayed
+            t0, t_mid, t1 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+            torch.cuda._sleep(int(args.prefill_us * 2.0e3))
+            t0.record(stream)
+            for _ in range(k // args.graph):
+                graph.replay()
+            t_mid.record(stream)
+            pflush(last)
+            t1.record(stream)
+            torch.cuda.synchronize()
+            return t0.elapsed_time(t1), t0.elapsed_time(t_mid)
+    else:
+        for i in range(args.warmup):
+            pstep(i)
+        pflush(args.warmup - 1)
+    torch.cuda.synchronize()
+    if int(rnd.status.item()) | int(pair[1].status.item()):
+        raise RuntimeError("device status set after warm-up")
+
+    # ---- device-resident timed region: exactly K rounds ----
+    if ws > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(bus) as clk:
+        total_ms, launches_ms = pipelined_region(args.steps, 0)
+    if ws > 1:
+        dist.barrier()
+    total_ms = shard.max_over_ranks(total_ms, device=dev)   # blocks shard by rank: no data-path exchange
+    ms_per_step = total_ms / args.steps
+    value = ws * B * args.steps / (total_ms / 1e3)
+    pipe_avg_ms = launches_ms / args.steps                # one pipelined launch, back to back
+    status = int(rnd.status.item()) | int(pair[1].status.item())
+
+    # ---- the same rounds unpipelined: sdd_block_scan then sdd_block_decide
+    # per round (each round complete before the next one's streaming pass) ----
     def step(i):
         s = sets[i % n_sets]
         rnd.set_inputs(s.z_d, s.z_t, s.x, seed=wl.seed, round_=i)
@@ -390,55 +482,21 @@ def run_gpu(args):
     for i in range(args.warmup):
         step(i)
     torch.cuda.synchronize()
-    if int(rnd.status.item()) != 0:
-        raise RuntimeError(f"device status {int(rnd.status.item())} after warm-up")
-    graph = None
-    if args.graph:
-        # small rounds outrun the host's launches: the timed rounds replay a
-        # CUDA graph of --graph rounds (the same launches, captured once)
-        if args.steps % args.graph:
-            raise SystemExit("--steps must be a multiple of --graph")
-        side = torch.cuda.Stream(device=dev)
-        side.wait_stream(stream)
-        graph = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(graph, stream=side):
-            for j in range(args.graph):
-                step(args.warmup + j)
-        for _ in range(2):
-            graph.replay()
+    u0, u1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(bus) as uclk:
+        torch.cuda._sleep(int(args.prefill_us * 2.0e3))
+        u0.record(stream)
+        for i in range(args.steps):
+            step(args.warmup + i)
+        u1.record(stream)
         torch.cuda.synchronize()
+    u_ms = shard.max_over_ranks(u0.elapsed_time(u1), device=dev)
+    unpipelined = {"value": ws * B * args.steps / (u_ms / 1e3), "unit": UNIT, "ms_per_step": u_ms / args.steps,
+                   "launches": 2 * args.steps, "clocks": uclk.summary(),
+                   "what": "sdd_block_scan + sdd_block_decide per round, rounds in series"}
 
-    # ---- device-resident timed region: exactly K rounds ----
-    # A short device-side spin keeps the stream busy while the host enqueues
-    # the rounds, so the start event fires with rounds already queued behind it
-    # (no host launch latency inside the region).
-    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    props = torch.cuda.get_device_properties(dev)
-    bus = getattr(props, "pci_bus_id", None)
-    if ws > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-    with ClockSampler(bus) as clk:
-        torch.cuda._sleep(int(args.prefill_us * 2.0e3))    # ~prefill_us at 2 GHz
-        t_start.record(stream)
-        if graph is not None:
-            for _ in range(args.steps // args.graph):
-                graph.replay()
-        else:
-            for i in range(args.steps):
-                step(args.warmup + i)
-        t_end.record(stream)
-        torch.cuda.synchronize()
-    if ws > 1:
-        dist.barrier()
-    total_ms = t_start.elapsed_time(t_end)
-    total_ms = shard.max_over_ranks(total_ms, device=dev)   # blocks shard by rank: no data-path exchange
-    ms_per_step = total_ms / args.steps
-    value = ws * B * args.steps / (total_ms / 1e3)
-    status = int(rnd.status.item())
-
-    # ---- the streaming kernel alone, for the roofline: N back-to-back
-    # launches (rotating input sets) under one event pair ----
+    # ---- the streaming kernel alone: N back-to-back launches (rotating input
+    # sets) under one event pair ----
     n_scan = max(50, args.scan_launches)
     for i in range(3):
         s = sets[i % n_sets]
@@ -456,10 +514,11 @@ def run_gpu(args):
     torch.cuda.synchronize()
     scan_avg_ms = e0.elapsed_time(e1) / n_scan
 
-    # ---- one untimed round on input set 0 for the oracle parity sample (its
-    # decisions are copied out before the end-to-end leg reuses the round) ----
-    rnd.set_inputs(sets[0].z_d, sets[0].z_t, sets[0].x, seed=wl.seed, round_=0)
-    rnd.run()
+    # ---- one untimed pipelined round on input set 0 for the oracle parity
+    # sample (its decisions are copied out before the end-to-end leg) ----
+    pair[0].set_inputs(sets[0].z_d, sets[0].z_t, sets[0].x, seed=wl.seed, round_=0)
+    sdd.block_pipelined(pair[0], None)
+    sdd.block_pipelined(None, pair[0])
     torch.cuda.synchronize()
     decisions = {"K": rnd.K.cpu().numpy(), "L": rnd.L_strict.cpu().numpy(), "tok": rnd.tokens_strict.cpu().numpy(),
                  "Ll": rnd.L_lenient.cpu().numpy(), "tl": rnd.tokens_lenient.cpu().numpy(),
@@ -472,21 +531,24 @@ def run_gpu(args):
         e2e = {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
     peak, peak_kind = _peaks()
-    achieved = scan_bytes / (scan_avg_ms / 1e3) / 1e9
+    pipe_bytes = scan_bytes + draw_bytes
+    achieved = pipe_bytes / (pipe_avg_ms / 1e3) / 1e9
+    scan_achieved = scan_bytes / (scan_avg_ms / 1e3) / 1e9
     if rank == 0:
         cpu = parity = None
         if ws == 1 and not args.no_cpu_baseline:
             cpu, res = _cpu_baseline(wl, ells, ks, _host_block(sets[0], wl), min(args.cpu_blocks, B))
             parity = _parity_sample(decisions, res, ells, ks)
-        roofline = {"bound": "hbm", "kernel": "scan_kernel (sdd_block_scan)", "achieved": achieved,
+        roofline = {"bound": "hbm", "kernel": "pipe_kernel (sdd_block_pipelined)", "achieved": achieved,
                     "peak": peak, "unit": "GB/s", "frac": achieved / peak, "traffic": args.traffic,
-                    "peak_source": f"{peak_kind} hbm_gbs (burst copy; the kernel is timed in a run of "
-                                   f"{n_scan} back-to-back launches)",
-                    "bytes_per_launch": scan_bytes, "avg_launch_ms": scan_avg_ms, "launches_timed": n_scan}
-        if scan_avg_ms > ms_per_step:
-            # the dominant kernel cannot take longer than the round that contains it
+                    "peak_source": f"{peak_kind} hbm_gbs (burst copy)",
+                    "bytes_per_launch": pipe_bytes, "avg_launch_ms": pipe_avg_ms,
+                    "launches_timed": args.steps,
+                    "bytes": "every logit of round i once + the two draw rows per block of round i - 1"}
+        if pipe_avg_ms > ms_per_step:
+            # the dominant kernel cannot take longer than the step that contains it
             roofline = {"bound": "hbm", "achieved": None, "peak": peak, "unit": "GB/s", "frac": None,
-                        "traffic": args.traffic, "invalid": f"scan {scan_avg_ms:.4f} ms > round {ms_per_step:.4f} ms"}
+                        "traffic": args.traffic, "invalid": f"launch {pipe_avg_ms:.4f} ms > step {ms_per_step:.4f} ms"}
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
@@ -494,15 +556,24 @@ def run_gpu(args):
             # and normalisers; the logits' storage type is config.dtype
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {**_config_json(wl, ells, ks, n_sets),
-                       "launch": (f"CUDA graph of {args.graph} rounds, replayed" if args.graph
-                                  else "one call per kernel, queued behind a device spin")},
+                       "launch": ("pipelined rounds (sdd_block_pipelined): K launches each streaming one round "
+                                  "and finishing the one before, + one closing decide, "
+                                  + (f"as replays of a CUDA graph of {args.graph} launches" if args.graph
+                                     else "queued behind a device spin"))},
             "achieved_gbs_step": ws * scan_bytes / (ms_per_step / 1e3) / 1e9,
             "frac_of_8tbs_step": ws * scan_bytes / (ms_per_step / 1e3) / 8e12,
             "roofline": roofline,
+            "roofline_scan_kernel": {"bound": "hbm", "kernel": "scan_kernel (sdd_block_scan)",
+                                     "achieved": scan_achieved, "peak": peak, "unit": "GB/s",
+                                     "frac": scan_achieved / peak,
+                                     "traffic": SCAN_TRAFFIC_C3 if args.c3 else None,
+                                     "bytes_per_launch": scan_bytes, "avg_launch_ms": scan_avg_ms,
+                                     "launches_timed": n_scan},
+            "round_unpipelined": unpipelined,
             "cpu_baseline": cpu,
             "parity_sample": parity,
             "e2e": e2e,
-            "gpu_launches": 2 * args.steps,
+            "gpu_launches": args.steps + 1,
             "clocks": clk.summary(),
             "device_status": status,
         }
@@ -952,7 +1023,8 @@ def main():
     if args.component == "shard":
         return run_component_shard(args)
     if args.traffic is None and args.workload == "c3" and args.blocks in (None, 16):
-        args.traffic = SCAN_TRAFFIC_C3
+        args.traffic = PIPE_TRAFFIC_C3
+    args.c3 = args.workload == "c3" and args.blocks in (None, 16)
     if args.warmup < 3:
         args.warmup = 3
     if args.impl == "reference":
