@@ -47,9 +47,10 @@ NEAR = 1e-6
 # dram__bytes_read.sum + dram__bytes_write.sum of one launch on the c3
 # workload, from one ncu capture of the kernel as it stands; reported as the
 # "traffic" of that workload's rooflines only: the streaming kernel
-# (318,294,528 B + 3,656,960 B) and the pipelined round's kernel.
+# (318,294,528 B + 3,656,960 B) and the pipelined round's kernel
+# (328,085,248 B + 3,866,880 B, three rotating input sets).
 SCAN_TRAFFIC_C3 = 321_951_488
-PIPE_TRAFFIC_C3 = None
+PIPE_TRAFFIC_C3 = 331_952_128
 
 
 def _peaks():
@@ -387,6 +388,10 @@ def run_gpu(args):
     esz = 2 if wl.dtype == torch.bfloat16 else 4
     scan_bytes = (2 * gamma + 1) * V * esz * B          # every logit read once
     draw_bytes = 2 * V * esz * B                         # the decide's two draw rows per block
+    # (the library runs rounds of at most 768 MiB of logits in the pipelined
+    # kernel, larger ones as its streaming and decide kernels; rows padded to
+    # 16 bytes)
+    pipelined_kernel = (2 * gamma + 1) * B * (-(-V * esz // 16) * 16) <= (768 << 20)
     stream = torch.cuda.current_stream()
     props = torch.cuda.get_device_properties(dev)
     bus = getattr(props, "pci_bus_id", None)
@@ -545,6 +550,14 @@ def run_gpu(args):
                     "bytes_per_launch": pipe_bytes, "avg_launch_ms": pipe_avg_ms,
                     "launches_timed": args.steps,
                     "bytes": "every logit of round i once + the two draw rows per block of round i - 1"}
+        if not pipelined_kernel:
+            # rounds above the pipelined kernel's size run as the streaming and
+            # decide kernels: the streaming kernel dominates
+            roofline = {"bound": "hbm", "kernel": "scan_kernel (sdd_block_pipelined on a large round)",
+                        "achieved": scan_achieved, "peak": peak, "unit": "GB/s", "frac": scan_achieved / peak,
+                        "traffic": None, "peak_source": f"{peak_kind} hbm_gbs (burst copy)",
+                        "bytes_per_launch": scan_bytes, "avg_launch_ms": scan_avg_ms, "launches_timed": n_scan}
+            pipe_avg_ms = scan_avg_ms
         if pipe_avg_ms > ms_per_step:
             # the dominant kernel cannot take longer than the step that contains it
             roofline = {"bound": "hbm", "achieved": None, "peak": peak, "unit": "GB/s", "frac": None,
@@ -556,9 +569,11 @@ def run_gpu(args):
             # and normalisers; the logits' storage type is config.dtype
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {**_config_json(wl, ells, ks, n_sets),
-                       "launch": ("pipelined rounds (sdd_block_pipelined): K launches each streaming one round "
+                       "launch": ("pipelined rounds (sdd_block_pipelined): K calls each streaming one round "
                                   "and finishing the one before, + one closing decide, "
-                                  + (f"as replays of a CUDA graph of {args.graph} launches" if args.graph
+                                  + ("in one launch per call (pipe_kernel), " if pipelined_kernel else
+                                     "as the decide and streaming kernels (a round above 768 MiB), ")
+                                  + (f"as replays of a CUDA graph of {args.graph} calls" if args.graph
                                      else "queued behind a device spin"))},
             "achieved_gbs_step": ws * scan_bytes / (ms_per_step / 1e3) / 1e9,
             "frac_of_8tbs_step": ws * scan_bytes / (ms_per_step / 1e3) / 8e12,
@@ -573,7 +588,7 @@ def run_gpu(args):
             "cpu_baseline": cpu,
             "parity_sample": parity,
             "e2e": e2e,
-            "gpu_launches": args.steps + 1,
+            "gpu_launches": (args.steps + 1) if pipelined_kernel else 2 * args.steps,
             "clocks": clk.summary(),
             "device_status": status,
         }

@@ -1133,12 +1133,21 @@ sdd_status_t sdd_block(const sdd_block_args *a, sdd_stream_t stream) {
     return sdd_block_decide(a, stream);
 }
 
+// Rounds of at most this many bytes of logits run in the pipelined kernel;
+// larger ones stream on all sixteen warps of each CTA (sdd_block_scan) and are
+// decided by the decide kernel in the next call.  Measured on GB300 (c3 rows,
+// blocks/s pipelined against unpipelined): B = 16 (316 MB) 251.1 k / 233.2 k,
+// B = 32 (632 MB) 278.6 k / 275.2 k, B = 64 (1.26 GB) 290.9 k / 296.9 k: the
+// decide kernel's fixed tail matters less as the round grows, while twelve
+// streaming warps reach ~0.9 of the copy peak against sixteen's ~1.0.
+constexpr int64_t kPipeMaxBytes = int64_t(768) << 20;
+
 // A pipelined round's launch parameters: sdd_block's, streamed by warps
-// kPipeWarps..15 of each CTA (the same when the round is streamed and when it
-// is decided).
+// kPipeWarps..15 of each CTA when the round is at most kPipeMaxBytes (the same
+// when the round is streamed and when it is decided).
 static sdd_status_t pipe_params(const sdd_block_args *a, ScanParams &p, bool *empty) {
     SDD_TRY(block_params(a, p, empty));
-    if (*empty) return SDD_OK;
+    if (*empty || p.T * 16 > kPipeMaxBytes) return SDD_OK;
     Work w;
     SDD_TRY(get_work(a->workspace, a->workspace_bytes, a->B, a->gamma, w));
     const int wpc = kWarpsPerCta - kPipeWarps;
@@ -1159,6 +1168,11 @@ sdd_status_t sdd_block_pipelined(const sdd_block_args *next, const sdd_block_arg
     if (prev) SDD_TRY(pipe_params(prev, pp, &ep));
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     if (en) return ep ? SDD_OK : run_decide(pp, st);   // the last round of a sequence: decide only
+    if (pn.wpc == kWarpsPerCta) {
+        // a large round: prev's decide kernel, then next's streaming kernel
+        if (!ep) SDD_TRY(run_decide(pp, st));
+        return run_scan(pn, st);
+    }
     if (static_cast<double>(pn.C) * static_cast<double>(pn.W) >= 9.007199254740992e15)   // 2^53
         return fail(SDD_ERR_UNSUPPORTED, "%lld vectors of logits exceed the index arithmetic", (long long)pn.T);
     const int grid = static_cast<int>((static_cast<int64_t>(pn.W) + pn.wpc - 1) / pn.wpc);

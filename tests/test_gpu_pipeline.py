@@ -30,46 +30,53 @@ def _padded(z: torch.Tensor, stride: int) -> torch.Tensor:
 class _Round:
     """One round of a sequence: its inputs, its BlockRound and its rules."""
 
-    def __init__(self, rnd, blk, seed, round_, taus, ells, ks, greedy, K_min, S_max, D):
+    def __init__(self, rnd, blk, seed, round_, taus, ells, ks, greedy, K_min, S_max, D, sample=None):
         self.rnd, self.blk = rnd, blk
         self.seed, self.round_ = seed, round_
         self.taus, self.ells, self.ks, self.greedy = taus, ells, ks, greedy
         self.K_min, self.S_max, self.D = K_min, S_max, D
+        self.sample = sample
 
 
 def _check(r: _Round, tally: Tally):
+    """Round r's outputs against the oracle: every block, or the blocks in
+    r.sample (then without the batch-wide agreement counters)."""
     rnd, blk = r.rnd, r.blk
     dtype = blk.z_d.dtype
     assert int(rnd.status.item()) == 0
+    blocks = list(range(blk.x.shape[0])) if r.sample is None else list(r.sample)
     ob = oracle_block(blk.z_d, blk.z_t, blk.x, seed=r.seed, round_=r.round_, pairs=[(t, t) for t in r.taus],
-                      K_min=r.K_min, S_max=r.S_max, D_in=r.D.numpy(), ells=r.ells, ks=r.ks, sampling=not r.greedy)
-    assert_close_stats("q", rnd.q, ob.stats.q, dtype)
-    assert_close_stats("lse", rnd.lse, ob.stats.lse, dtype)
-    assert_close_stats("entropy", rnd.entropy, ob.stats.entropy, dtype)
-    np.testing.assert_array_equal(rnd.argmax.cpu().numpy(), ob.stats.argmax)
-    blocks = list(range(blk.x.shape[0]))
+                      K_min=r.K_min, S_max=r.S_max, D_in=r.D.numpy(), ells=r.ells, ks=r.ks, sampling=not r.greedy,
+                      blocks=blocks)
+    sub = lambda t: t[blocks]   # noqa: E731
+    assert_close_stats("q", sub(rnd.q), ob.stats.q, dtype)
+    assert_close_stats("lse", sub(rnd.lse), ob.stats.lse, dtype)
+    assert_close_stats("entropy", sub(rnd.entropy), ob.stats.entropy, dtype)
+    np.testing.assert_array_equal(sub(rnd.argmax).cpu().numpy(), ob.stats.argmax)
+    idx = list(range(len(blocks)))
     strict = ob.greedy if r.greedy else ob.strict
-    compare_rule(tally, "strict", rnd.L_strict, rnd.tokens_strict, strict, blocks)
+    compare_rule(tally, "strict", sub(rnd.L_strict), sub(rnd.tokens_strict), strict, idx)
     for i, e in enumerate(r.ells):
-        compare_rule(tally, f"lenient {e:.4f}", rnd.L_lenient[i], rnd.tokens_lenient[i], ob.lenient[e], blocks)
+        compare_rule(tally, f"lenient {e:.4f}", sub(rnd.L_lenient[i]), sub(rnd.tokens_lenient[i]), ob.lenient[e], idx)
     for i, k in enumerate(r.ks):
-        compare_rule(tally, f"top-{k}", rnd.L_topk[i], rnd.tokens_topk[i], ob.topk[k], blocks)
-    L_or = np.array([strict[b][0] for b in blocks])
+        compare_rule(tally, f"top-{k}", sub(rnd.L_topk[i]), sub(rnd.tokens_topk[i]), ob.topk[k], idx)
+    L_or = np.array([strict[i][0] for i in idx])
     acc_want = np.zeros((len(r.taus), 4), np.int64)
     for t, tau in enumerate(r.taus):
         oKh, oK, oD, mg = ob.sched[(tau, tau)]
-        for b in blocks:
-            ok = (rnd.K_hat[t, b].item() == oKh[b] and rnd.K[t, b].item() == oK[b] and rnd.D_out[t, b].item() == oD[b])
-            tally.check(f"schedule tau {tau} block {b}", ok, mg[b])
+        for i, b in enumerate(blocks):
+            ok = (rnd.K_hat[t, b].item() == oKh[i] and rnd.K[t, b].item() == oK[i] and rnd.D_out[t, b].item() == oD[i])
+            tally.check(f"schedule tau {tau} block {b}", ok, mg[i])
         acc_want[t] = orc.agreement(oK, L_or)
-    np.testing.assert_array_equal(rnd.agreement.cpu().numpy(), acc_want)
+    if r.sample is None:
+        np.testing.assert_array_equal(rnd.agreement.cpu().numpy(), acc_want)
     oK0 = ob.sched[(r.taus[0], r.taus[0])][1]
     ct, cn, xs = rnd.commit_tokens.cpu().numpy(), rnd.commit_n.cpu().numpy(), blk.x.cpu().numpy()
-    for b in blocks:
-        if oK0[b] > 0:
-            assert cn[b] == oK0[b] and np.array_equal(ct[b][:oK0[b]], xs[b][:oK0[b]]) and np.all(ct[b][oK0[b]:] == -1)
+    for i, b in enumerate(blocks):
+        if oK0[i] > 0:
+            assert cn[b] == oK0[i] and np.array_equal(ct[b][:oK0[i]], xs[b][:oK0[i]]) and np.all(ct[b][oK0[i]:] == -1)
         else:
-            L, tok, _ = strict[b]
+            L, tok, _ = strict[i]
             assert cn[b] == L + 1 and np.array_equal(ct[b], tok)
 
 
@@ -150,6 +157,27 @@ def test_pipelined_mixed_shapes_and_more_blocks_than_ctas():
         rounds.append(_Round(rnd, blk, 3 + i, i, taus, ells, ks, False, 0, 64, D))
     tally = _run_sequence(rounds)
     print("pipelined mixed shapes", tally)
+
+
+def test_pipelined_large_and_small_rounds_alternate():
+    """Rounds above 768 MiB of logits (48 blocks of the 16-block workload's
+    rows: 948 MB) stream on all sixteen warps and are decided by the decide
+    kernel; smaller ones run in the pipelined kernel.  A sequence alternating
+    the two hands each kind of round to the other kind of call; sampled
+    blocks of the large rounds and every block of the small one against the
+    oracle."""
+    wl = synth.WORKLOADS["c3"]
+    ells = tuple(synth.paper_ell(e) for e in wl.ells)
+    ks = tuple(wl.topks)
+    rounds = []
+    for i, B in enumerate((48, 16, 48)):
+        rnd = sdd.BlockRound(B, wl.gamma, wl.V, dtype=wl.dtype, taus=wl.taus, ells=ells, ks=ks, K_min=6, S_max=64)
+        blk = synth.make_block(wl, device=DEV, B=B, round_=i)
+        sample = None if B == 16 else (0, 13, 30, 47)
+        rounds.append(_Round(rnd, blk, wl.seed, i, wl.taus, ells, ks, False, 6, 64,
+                             torch.zeros(B, dtype=torch.int32), sample=sample))
+    tally = _run_sequence(rounds)
+    print("pipelined large / small", tally)
 
 
 def test_pipelined_rejects_one_round_as_both():
