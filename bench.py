@@ -388,10 +388,10 @@ def run_gpu(args):
     esz = 2 if wl.dtype == torch.bfloat16 else 4
     scan_bytes = (2 * gamma + 1) * V * esz * B          # every logit read once
     draw_bytes = 2 * V * esz * B                         # the decide's two draw rows per block
-    # (the library runs rounds of at most 768 MiB of logits in the pipelined
+    # (the library runs rounds of at most 512 MiB of logits in the pipelined
     # kernel, larger ones as its streaming and decide kernels; rows padded to
     # 16 bytes)
-    pipelined_kernel = (2 * gamma + 1) * B * (-(-V * esz // 16) * 16) <= (768 << 20)
+    pipelined_kernel = (2 * gamma + 1) * B * (-(-V * esz // 16) * 16) <= (512 << 20)
     stream = torch.cuda.current_stream()
     props = torch.cuda.get_device_properties(dev)
     bus = getattr(props, "pci_bus_id", None)
@@ -572,7 +572,7 @@ def run_gpu(args):
                        "launch": ("pipelined rounds (sdd_block_pipelined): K calls each streaming one round "
                                   "and finishing the one before, + one closing decide, "
                                   + ("in one launch per call (pipe_kernel), " if pipelined_kernel else
-                                     "as the decide and streaming kernels (a round above 768 MiB), ")
+                                     "as the decide and streaming kernels (a round above 512 MiB), ")
                                   + (f"as replays of a CUDA graph of {args.graph} calls" if args.graph
                                      else "queued behind a device spin"))},
             "achieved_gbs_step": ws * scan_bytes / (ms_per_step / 1e3) / 1e9,

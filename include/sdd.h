@@ -584,7 +584,7 @@ SDD_API sdd_status_t sdd_block_decide(const sdd_block_args *args, sdd_stream_t s
  *           first call).  Its streaming pass must have been made by this
  *           call: the pipelined pass divides the rows among warps
  *           differently from sdd_block_scan.
- * Rounds of more than 768 MiB of logits, whose decide work is a small part of
+ * Rounds of more than 512 MiB of logits, whose decide work is a small part of
  * their time, run as sdd_block_scan (in the call that names them as next) and
  * sdd_block_decide (in the call that names them as prev) instead.
  * next and prev must use different workspaces and different output arrays.

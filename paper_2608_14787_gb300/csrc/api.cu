@@ -1135,12 +1135,13 @@ sdd_status_t sdd_block(const sdd_block_args *a, sdd_stream_t stream) {
 
 // Rounds of at most this many bytes of logits run in the pipelined kernel;
 // larger ones stream on all sixteen warps of each CTA (sdd_block_scan) and are
-// decided by the decide kernel in the next call.  Measured on GB300 (c3 rows,
-// blocks/s pipelined against unpipelined): B = 16 (316 MB) 251.1 k / 233.2 k,
-// B = 32 (632 MB) 278.6 k / 275.2 k, B = 64 (1.26 GB) 290.9 k / 296.9 k: the
-// decide kernel's fixed tail matters less as the round grows, while twelve
-// streaming warps reach ~0.9 of the copy peak against sixteen's ~1.0.
-constexpr int64_t kPipeMaxBytes = int64_t(768) << 20;
+// decided by the decide kernel in the next call.  Measured on GB300 (rows of
+// 32 positions over V = 151,936 bf16, blocks/s pipelined kernel / two
+// kernels): B = 16 (316 MB) 257 k / 232 k, B = 24 (474 MB) 274.5 k / 257.4 k,
+// B = 32 (632 MB) 254.9 k / 272.4 k, B = 40 (790 MB) 256.5 k / 282.4 k: the
+// decide kernel's fixed tail matters less as the round grows, while fourteen
+// streaming warps and the decide work beside them trail sixteen warps alone.
+constexpr int64_t kPipeMaxBytes = int64_t(512) << 20;
 
 // A pipelined round's launch parameters: sdd_block's, streamed by warps
 // kPipeWarps..15 of each CTA when the round is at most kPipeMaxBytes (the same

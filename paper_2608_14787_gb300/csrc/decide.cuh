@@ -275,14 +275,14 @@ __device__ __forceinline__ float run_sum(const DrawCtx &c, int vb, int ve, int V
     return sum;
 }
 
-// run_sum over a segment staged in shared memory: st / sd hold the draw
-// rows' vectors [v0, v0 + n) (sd unused for the bonus row); vectors [lb, le)
-// of the segment, the same order and arithmetic as run_sum.
+// run_sum over a chunk staged in shared memory, added to sum: st / sd hold
+// the draw rows' vectors [v0, v0 + n) (sd unused for the bonus row); vectors
+// [lb, le) of the chunk (none when lb >= le), the same order and arithmetic
+// as run_sum.
 template <int DT>
 __device__ __forceinline__ float stage_sum(const DrawCtx &c, const uint4 *st, const uint4 *sd, int lb, int le,
-                                           int v0, int V) {
+                                           int v0, int V, float sum) {
     constexpr int EPV = (DT == SDD_BF16) ? 8 : 4;
-    float sum = 0.f;
     for (int v = lb; v < le; ++v) {
         const uint4 a = st[v];
         const uint4 d = c.zd_row ? sd[v] : make_uint4(0, 0, 0, 0);
@@ -538,16 +538,16 @@ __device__ __forceinline__ DecGeom dec_geom(const ScanParams &p, const PartView 
 // (listed block, draw segment) pair geo, after the streaming pass over p's
 // rows has completed.  s_pref_all: nseg * NT floats of shared memory
 // (the last segment to arrive stages every segment's prefixes there);
-// s_stage: 2 * seg_vec vectors of shared memory for the team's segment of
-// both draw rows, or null (the segment is read from global memory).  Every
+// s_stage: 2 * stage_vec vectors of shared memory through which the team
+// reads its segment of both draw rows, or null (read from global memory).  Every
 // return is taken by the whole team.  FEAT: also the extended features of the
 // drafter rows; SHARD: the vocabulary-sharded round (records of S slices
 // instead of warp partials, the draw left to shard_draw_kernel).
 template <int DT, bool FEAT, bool SHARD, int NT = kDecThreads>
 __device__ __forceinline__ void decide_cta(const ScanParams &p, const PartView &pv, const DecGeom &geo,
-                                           float *s_pref_all, uint4 *s_stage = nullptr) {
+                                           float *s_pref_all, uint4 *s_stage = nullptr, int stage_vec = 0) {
     static_assert(!SHARD || NT == kDecThreads, "the sharded round's layouts assume kDecThreads");
-    static_assert(NT % 32 == 0 && NT >= SDD_MAX_GAMMA, "one drafted position per thread");
+    static_assert(NT % 32 == 0 && 2 * NT >= SDD_MAX_GAMMA, "at most two drafted positions per thread");
     const DecideParams &d = p.dec;
     const int i = geo.i;            // listed block
     const int seg = geo.seg;        // segment of the draw row
@@ -586,14 +586,18 @@ __device__ __forceinline__ void decide_cta(const ScanParams &p, const PartView &
 
     // ---- phase 1: facts of every row of the block, one row per thread ----
     // the drafted tokens, guard flags and the block's schedule inputs (gamma <=
-    // NT: one position per thread) are loaded in the same batch as
+    // 2 NT: at most two positions per thread) are loaded in the same batch as
     // the rows' partials below and stored after them: one round trip
-    int32_t xj = 0, force_b = 0, D_b = 0;
-    uint8_t gj = 0;
+    int32_t xj[2] = {0, 0}, force_b = 0, D_b = 0;
+    uint8_t gj[2] = {0, 0};
     if (dec) {
-        if (tid < gamma) {
-            xj = __ldg(d.tokens + ob + tid);
-            gj = d.guard ? d.guard[ob + tid] : 0;
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const int j = tid + k * NT;
+            if (j < gamma) {
+                xj[k] = __ldg(d.tokens + ob + j);
+                gj[k] = d.guard ? d.guard[ob + j] : 0;
+            }
         }
         if (tid == 0) {
             force_b = d.force_strict ? d.force_strict[b] : 0;
@@ -647,9 +651,13 @@ __device__ __forceinline__ void decide_cta(const ScanParams &p, const PartView &
         }
     }
     if (dec) {
-        if (tid < gamma) {
-            F.x[tid] = xj;
-            F.guard[tid] = gj;
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const int j = tid + k * NT;
+            if (j < gamma) {
+                F.x[j] = xj[k];
+                F.guard[j] = gj[k];
+            }
         }
         if (tid == 0) {
             s_force = force_b;
@@ -776,18 +784,25 @@ __device__ __forceinline__ void decide_cta(const ScanParams &p, const PartView &
             const int vb = min(v1, v0 + tid * vpt), ve = min(v1, vb + vpt);
             float ts;
             if (s_stage) {
-                // the segment of both draw rows into shared memory first: one
-                // round trip for all of it (under a concurrent streaming pass
-                // each dependent round trip is long)
-                const uint4 *gt = reinterpret_cast<const uint4 *>(zt_row) + v0;
-                const uint4 *gdr = zd_row ? reinterpret_cast<const uint4 *>(zd_row) + v0 : nullptr;
-                for (int q = tid; q < v1 - v0; q += NT) {
-                    cp_async16(s_stage + q, gt + q);
-                    if (gdr) cp_async16(s_stage + seg_vec + q, gdr + q);
+                // the segment of both draw rows through shared memory in
+                // chunks of stage_vec vectors: one round trip per chunk (under
+                // a concurrent streaming pass each dependent round trip is
+                // long); every thread sums its run chunk by chunk, in order
+                ts = 0.f;
+                const uint4 *gt = reinterpret_cast<const uint4 *>(zt_row);
+                const uint4 *gdr = zd_row ? reinterpret_cast<const uint4 *>(zd_row) : nullptr;
+                for (int c0 = v0; c0 < v1; c0 += stage_vec) {
+                    const int c1 = min(v1, c0 + stage_vec);
+                    for (int q = tid; q < c1 - c0; q += NT) {
+                        cp_async16(s_stage + q, gt + c0 + q);
+                        if (gdr) cp_async16(s_stage + stage_vec + q, gdr + c0 + q);
+                    }
+                    cp_async_wait_all();
+                    dec_sync<NT>();
+                    ts = stage_sum<DT>(c, s_stage, s_stage + stage_vec, max(vb, c0) - c0, min(ve, c1) - c0, c0,
+                                       p.V, ts);
+                    dec_sync<NT>();   // (the next chunk overwrites the stage)
                 }
-                cp_async_wait_all();
-                dec_sync<NT>();
-                ts = stage_sum<DT>(c, s_stage, s_stage + seg_vec, vb - v0, ve - v0, v0, p.V);
             } else {
                 ts = run_sum<DT>(c, vb, ve, p.V);
             }
@@ -876,14 +891,20 @@ __device__ __forceinline__ void decide_cta(const ScanParams &p, const PartView &
             }
         }
         }
-        if (!leader) return;
+        if (SHARD && !leader) return;
         dec_sync<NT>();
     }
 
-    // ---- the leader: every other rule (a warp per rule), the schedule (a warp
-    // per threshold pair), agreement counters and the remaining commits ----
+    // ---- every other rule (a warp per rule), the schedule (a warp per
+    // threshold pair) and the agreement counters: under the sampling rule the
+    // block's draw segments share these tasks round robin (every team holds
+    // the block's facts), otherwise the one team takes them all; then the
+    // leader writes the remaining commits ----
     const int R = 1 + d.n_ell + d.n_k;
-    for (int r = warp; r < R; r += NW) {
+    const int S = (sampling && !SHARD) ? nseg : 1, me = (sampling && !SHARD) ? seg : 0;
+    for (int ir = warp;; ir += NW) {
+        const int r = me + ir * S;   // this team's share of the rules
+        if (r >= R) break;
         if (r == 0) {
             if (!d.do_strict || sampling) continue;   // sampling: completed by the draw
             const int L = rule_first_reject(d, F, 0, b, lane);
@@ -910,7 +931,10 @@ __device__ __forceinline__ void decide_cta(const ScanParams &p, const PartView &
     }
     if (!sched) return;
     dec_sync<NT>();   // s_L[0] of a greedy strict rule
-    for (int t = warp; t < d.n_tau; t += NW) {
+    const int t0 = ((me - R) % S + S) % S;   // pair t goes to team (R + t) mod S
+    for (int it = warp;; it += NW) {
+        const int t = t0 + it * S;
+        if (t >= d.n_tau) break;
         int Kh, K, Do;
         sched_pair(d, F, t, s_force != 0, s_D, lane, Kh, K, Do);
         if (lane == 0) {
@@ -929,6 +953,7 @@ __device__ __forceinline__ void decide_cta(const ScanParams &p, const PartView &
             }
         }
     }
+    if (!leader) return;
     dec_sync<NT>();
     if (warp == 0) {
         // tokens committed by a fused round: a skipped block commits x_1..x_K

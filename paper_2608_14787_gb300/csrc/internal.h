@@ -149,8 +149,8 @@ struct ScanParams {
     FastDiv divC, divW, divRV, divNpos[2], divWt[2], divP[2];   // division by C, W, RV, grp[g].npos, wt[g], P[g]
     // The streaming warps of a CTA: warps warp0 .. warp0 + wpc - 1, global
     // streaming warp blockIdx.x * wpc + (warp - warp0) (set_divisors: all 16;
-    // the pipelined round: warps 4-15, warps 0-3 run the previous round's
-    // decide work).
+    // the pipelined round: warps kPipeWarps-15, the others run the previous
+    // round's decide work).
     int32_t warp0, wpc;
     const int32_t *tokens;   // [B, gamma]
     // When set, the number of listed blocks is read from this device word at
@@ -193,7 +193,7 @@ void set_scan_wait_hooks(uint32_t polls, int drop_copy);
 // programmatic dependent of the streaming kernel.
 cudaError_t launch_decide(const ScanParams &p, cudaStream_t stream);
 // The pipelined round (pipe.cu): next's streaming pass over `grid` CTAs and,
-// on warps 0-3 of the same CTAs, prev's decide work (either may be null).
+// on warps 0-1 of the same CTAs, prev's decide work (either may be null).
 cudaError_t launch_pipe(const ScanParams *next, const ScanParams *prev, int grid, cudaStream_t stream);
 cudaError_t launch_schedule(const ScheduleParams &p, cudaStream_t stream);
 // Vocabulary-sharded path (shard.cu): the slice's per-row records, and the
@@ -255,11 +255,10 @@ __host__ __device__ inline int32_t scan_warps(int64_t W_max, int64_t T, int64_t 
     return static_cast<int32_t>(w > 1 ? w : 1);
 }
 
-// The pipelined round (sdd_block_pipelined): warps 0-3 of every CTA (a team
+// The pipelined round (sdd_block_pipelined): warps 0-1 of every CTA (a team
 // of kPipeTeam threads) run the previous round's decide work while warps
-// 4-15 stream (twelve streaming warps keep an SM's share of the memory
-// bandwidth nearly whole, eight do not).
-constexpr int kPipeTeam = 128;
+// 2-15 stream.
+constexpr int kPipeTeam = 64;
 constexpr int kPipeWarps = kPipeTeam / 32;
 
 // The cost weights and division constants of a launch whose groups, rows, T

@@ -7,16 +7,16 @@
 // streaming pass it leaves the memory system idle for most of its ~12 us.
 // Rounds over independent batches need not wait for one another, so here the
 // decide work of round n-1 runs beside the streaming pass of round n: in every
-// CTA, warps 0-3 do one (block, draw segment) item of round n-1's decide work
+// CTA, warps 0-1 do one (block, draw segment) item of round n-1's decide work
 // (decide_cta with a team of kPipeTeam threads and its barrier over those
-// threads only) while warps 4-15 stream round n, the rows divided among
-// twelve warps per CTA.  Measured on GB300 (16 blocks of 32 positions, V =
-// 151,936 bf16, back to back): 63.9 us per round against 68.8 us for the
-// streaming and decide kernels in turn.  Twelve streaming warps keep most of
-// an SM's share of the memory bandwidth, eight do not: a team of eight decide
-// warps (which then streamed a share cut to its decide time) gave 71-75 us;
-// under the concurrent stream a decide item takes ~27 us (43 us for the
-// teams that also locate the draw), all of it before the streaming ends.
+// threads only) while warps 2-15 stream round n, the rows divided among
+// fourteen warps per CTA.  Measured on GB300 (16 blocks of 32 positions, V =
+// 151,936 bf16, back to back): 62.7 us per round against 69.0 us for the
+// streaming and decide kernels in turn.  A team of eight decide warps beside
+// eight streaming warps (which then streamed a share cut to its decide time)
+// gave 71-75 us, four decide warps beside twelve 63.5-64.0 us; with two, a
+// decide item takes ~41 us under the concurrent stream, still before the
+// streaming warps end.
 // Round n-1's partials were written by the previous launch on the stream,
 // which has completed when this grid passes griddepcontrol.wait.
 #include <algorithm>
@@ -35,25 +35,25 @@ struct PipeParams {
     ScanParams prev;    // the round decided by this launch (unused when has_prev == 0)
     int32_t has_next, has_prev;
     int32_t n_items;    // decide items of prev: blocks x draw segments
-    int32_t stage;      // a team stages its draw segment in shared memory
+    int32_t stage_vec;  // vectors per row of a team's staged chunk of its draw segment (0: none)
 };
 
-// Warps 0-3 (kPipeTeam threads): prev's decide items of this CTA.  Out of
+// Warps 0-1 (kPipeTeam threads): prev's decide items of this CTA.  Out of
 // line, so that its register allocation stays apart from the streaming loop's.
 template <int DT>
 __device__ __noinline__ void pipe_decide(const PipeParams &pp, float *s_pref_all) {
     const ScanParams &p = pp.prev;
     const PartView pv = part_view(p);
     // after the segments' prefixes: the staged draw segment (16-byte aligned)
-    uint4 *s_stage = pp.stage ? reinterpret_cast<uint4 *>(s_pref_all + p.dec.nseg * kPipeTeam) : nullptr;
+    uint4 *s_stage = pp.stage_vec ? reinterpret_cast<uint4 *>(s_pref_all + p.dec.nseg * kPipeTeam) : nullptr;
     for (int item = blockIdx.x; item < pp.n_items; item += gridDim.x) {
         const DecGeom geo{item / p.dec.nseg, item % p.dec.nseg, p.dec.nseg, p.dec.seg_vec};
-        decide_cta<DT, false, false, kPipeTeam>(p, pv, geo, s_pref_all, s_stage);
+        decide_cta<DT, false, false, kPipeTeam>(p, pv, geo, s_pref_all, s_stage, pp.stage_vec);
         dec_sync<kPipeTeam>();   // the team's shared memory serves its next item
     }
 }
 
-// The streaming warps' rings, indexed by streaming warp (twelve per CTA):
+// The streaming warps' rings, indexed by streaming warp (fourteen per CTA):
 // two stages each, as in the streaming kernel (three measured slower here
 // too: 64.5 against 63.9 us per round).
 constexpr int kPipeStages = 2;
@@ -66,14 +66,16 @@ __global__ void __launch_bounds__(kThreads, 1) pipe_kernel(const __grid_constant
     extern __shared__ __align__(128) unsigned char smem[];
     // behind the previous launch on the stream (it streamed prev)
     griddep_wait();
-    if (pp.has_prev && threadIdx.x < kPipeTeam)
-        pipe_decide<DTP>(pp, reinterpret_cast<float *>(smem + kPipeRings));   // [nseg][kPipeTeam] after the rings
-    const int warp = threadIdx.x >> 5;
-    if (pp.has_next && warp >= pp.next.warp0) {
-        const int64_t gw = static_cast<int64_t>(blockIdx.x) * pp.next.wpc + (warp - pp.next.warp0);
-        if (gw < pp.next.W)
-            scan_warp<DTN, false, kPipeStages>(pp.next, smem, gw, warp - pp.next.warp0, pp.next.wpc);
+    if (threadIdx.x < kPipeTeam) {
+        if (pp.has_prev) pipe_decide<DTP>(pp, reinterpret_cast<float *>(smem + kPipeRings));   // after the rings
+        return;
     }
+    // (next.warp0 == kPipeWarps, next.wpc == kWarpsPerCta - kPipeWarps: compile-time here)
+    constexpr int kStreamWarps = kWarpsPerCta - kPipeWarps;
+    const int warp = threadIdx.x >> 5;
+    const int64_t gw = static_cast<int64_t>(blockIdx.x) * kStreamWarps + (warp - kPipeWarps);
+    if (pp.has_next && gw < pp.next.W)
+        scan_warp<DTN, false, kPipeStages>(pp.next, smem, gw, warp - kPipeWarps, kStreamWarps);
 }
 
 using PipeKernel = void (*)(PipeParams);
@@ -129,11 +131,13 @@ cudaError_t launch_pipe(const ScanParams *next, const ScanParams *prev, int grid
         pp.n_items = prev->grp[0].nb * nseg;
         if (draw) {
             smem += static_cast<size_t>(nseg) * kPipeTeam * sizeof(float);
-            // both draw rows' segments, when they fit beside the rings
-            const size_t stage = 2 * static_cast<size_t>(prev->dec.seg_vec) * 16;
-            if (smem + stage <= static_cast<size_t>(g_pipe_smem.load(std::memory_order_relaxed))) {
-                smem += stage;
-                pp.stage = 1;
+            // chunks of both draw rows' segments in the shared memory left
+            // beside the rings (the whole segment when it fits)
+            const size_t room = static_cast<size_t>(g_pipe_smem.load(std::memory_order_relaxed)) - smem;
+            const int chunk = static_cast<int>(std::min<size_t>(prev->dec.seg_vec, room / 32));
+            if (chunk >= kPipeTeam) {
+                pp.stage_vec = chunk;
+                smem += 2 * static_cast<size_t>(chunk) * 16;
             }
         }
     }

@@ -160,7 +160,7 @@ def test_pipelined_mixed_shapes_and_more_blocks_than_ctas():
 
 
 def test_pipelined_large_and_small_rounds_alternate():
-    """Rounds above 768 MiB of logits (48 blocks of the 16-block workload's
+    """Rounds above 512 MiB of logits (48 blocks of the 16-block workload's
     rows: 948 MB) stream on all sixteen warps and are decided by the decide
     kernel; smaller ones run in the pipelined kernel.  A sequence alternating
     the two hands each kind of round to the other kind of call; sampled
