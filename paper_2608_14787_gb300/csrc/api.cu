@@ -1153,7 +1153,7 @@ static sdd_status_t pipe_params(const sdd_block_args *a, ScanParams &p, bool *em
     SDD_TRY(get_work(a->workspace, a->workspace_bytes, a->B, a->gamma, w));
     const int wpc = kWarpsPerCta - kPipeWarps;
     p.W = scan_warps(w.W_max / kWarpsPerCta * wpc, p.T, p.rows);
-    set_divisors(p);
+    set_divisors(p, kPipeCostDrafter, kPipeCostTarget);
     p.warp0 = kPipeWarps;
     p.wpc = wpc;
     return SDD_OK;

@@ -260,13 +260,19 @@ __host__ __device__ inline int32_t scan_warps(int64_t W_max, int64_t T, int64_t 
 // 2-15 stream.
 constexpr int kPipeTeam = 64;
 constexpr int kPipeWarps = kPipeTeam / 32;
+// The pipelined pass's cost weights (drafter, target vector), as kCostDrafter
+// and kCostTarget for the streaming kernel: on fourteen warps beside the
+// decide work the drafter rows' entropy work weighs more (GB300, 16-block
+// round: 10 : 9 62.3 us, 21 : 18 61.2, 11 : 9 61.5, 23 : 18 62.2, 12 : 9 63.5;
+// with 10 : 9 the CTAs streaming drafter rows ended ~2.5 us after the others).
+constexpr int32_t kPipeCostDrafter = 21, kPipeCostTarget = 18;
 
 // The cost weights and division constants of a launch whose groups, rows, T
 // and W are set (host), all 16 warps of a CTA streaming.  The magic divisions
 // are exact while C * W < 2^53 (the callers check it).
-inline void set_divisors(ScanParams &p) {
+inline void set_divisors(ScanParams &p, int32_t cost_drafter = kCostDrafter, int32_t cost_target = kCostTarget) {
     const bool mixed = p.n_groups == 2 && p.grp[0].kind != p.grp[1].kind;
-    for (int g = 0; g < 2; ++g) p.wt[g] = mixed ? (p.grp[g].kind == 0 ? kCostDrafter : kCostTarget) : 1;
+    for (int g = 0; g < 2; ++g) p.wt[g] = mixed ? (p.grp[g].kind == 0 ? cost_drafter : cost_target) : 1;
     const int64_t wmax = std::max(p.wt[0], p.wt[1]), wmin = std::min(p.wt[0], p.wt[1]);
     // The row-start cost must leave every warp at least one vector start: a
     // warp's share of the cost, at least a row's cost over kPiecesPerRow
