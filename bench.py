@@ -48,9 +48,9 @@ NEAR = 1e-6
 # workload, from one ncu capture of the kernel as it stands; reported as the
 # "traffic" of that workload's rooflines only: the streaming kernel
 # (318,294,528 B + 3,656,960 B) and the pipelined round's kernel
-# (328,375,296 B + 3,593,728 B, three rotating input sets).
+# (328,386,304 B + 3,987,968 B, three rotating input sets).
 SCAN_TRAFFIC_C3 = 321_951_488
-PIPE_TRAFFIC_C3 = 331_969_024
+PIPE_TRAFFIC_C3 = 332_374_272
 
 
 def _peaks():
