@@ -12,10 +12,11 @@
 // accepted, p_t of the bonus row: each team sums its segment of the draw row
 // and publishes its per-thread prefix sums; the last to finish (atomic
 // arrival, no waiting) locates the segment, then the thread, from those sums,
-// and searches that thread's run with one warp.  Last, the segment-0 team
-// evaluates every other rule (lenience, top-k; greedy strict), the skip
-// schedule, agreement counters and commits, one warp per rule or threshold
-// pair.
+// and searches that thread's run with one warp.  Last, every other rule
+// (lenience, top-k; greedy strict), the skip schedule and the agreement
+// counters, one warp per rule or threshold pair, shared round robin by the
+// block's segment teams under the sampling rule; the segment-0 team writes
+// the commits.
 #pragma once
 
 #include "rules.cuh"
