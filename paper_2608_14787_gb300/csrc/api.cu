@@ -1151,10 +1151,12 @@ static sdd_status_t pipe_params(const sdd_block_args *a, ScanParams &p, bool *em
     if (*empty || p.T * 16 > kPipeMaxBytes) return SDD_OK;
     Work w;
     SDD_TRY(get_work(a->workspace, a->workspace_bytes, a->B, a->gamma, w));
-    const int wpc = kWarpsPerCta - kPipeWarps;
+    // the decide team beside this round's streaming pass (warps 0 .. warp0-1)
+    const int team_warps = (p.T * 16 <= kPipeSmallBytes ? kPipeTeamSmall : kPipeTeam) / 32;
+    const int wpc = kWarpsPerCta - team_warps;
     p.W = scan_warps(w.W_max / kWarpsPerCta * wpc, p.T, p.rows);
     set_divisors(p, kPipeCostDrafter, kPipeCostTarget);
-    p.warp0 = kPipeWarps;
+    p.warp0 = team_warps;
     p.wpc = wpc;
     return SDD_OK;
 }
@@ -1178,7 +1180,7 @@ sdd_status_t sdd_block_pipelined(const sdd_block_args *next, const sdd_block_arg
         return fail(SDD_ERR_UNSUPPORTED, "%lld vectors of logits exceed the index arithmetic", (long long)pn.T);
     const int grid = static_cast<int>((static_cast<int64_t>(pn.W) + pn.wpc - 1) / pn.wpc);
     // prev's draw segments over this grid's CTAs, one (block, segment) item each
-    if (!ep) draw_segments(pp.RV, pp.grp[0].nb, grid, kPipeTeam, pp.dec.nseg, pp.dec.seg_vec);
+    if (!ep) draw_segments(pp.RV, pp.grp[0].nb, grid, 32 * pn.warp0, pp.dec.nseg, pp.dec.seg_vec);
     const cudaError_t e = launch_pipe(&pn, ep ? nullptr : &pp, grid, st);
     if (e != cudaSuccess) return cuda_fail(e, "pipelined round launch");
     return SDD_OK;

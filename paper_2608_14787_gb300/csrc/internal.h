@@ -20,7 +20,7 @@ constexpr int kTileVec = 32 * kVPL;           // vectors per warp tile
 constexpr int kTileBytes = kTileVec * 16;     // 4 KiB
 constexpr int kStages = 2;
 // Shared memory of the rings of `warps` streaming warps with `stages` tiles each.
-constexpr int ring_bytes(int stages, int warps) { return warps * stages * (kTileBytes + 8); }
+__host__ __device__ constexpr int ring_bytes(int stages, int warps) { return warps * stages * (kTileBytes + 8); }
 constexpr int kScanSmem = ring_bytes(kStages, kWarpsPerCta);
 constexpr uint32_t kWaitPolls = 1u << 24;     // bounded mbarrier wait (seconds of polling)
 
@@ -193,7 +193,8 @@ void set_scan_wait_hooks(uint32_t polls, int drop_copy);
 // programmatic dependent of the streaming kernel.
 cudaError_t launch_decide(const ScanParams &p, cudaStream_t stream);
 // The pipelined round (pipe.cu): next's streaming pass over `grid` CTAs and,
-// on warps 0-1 of the same CTAs, prev's decide work (either may be null).
+// on the first next->warp0 warps of the same CTAs, prev's decide work (prev
+// may be null).
 cudaError_t launch_pipe(const ScanParams *next, const ScanParams *prev, int grid, cudaStream_t stream);
 cudaError_t launch_schedule(const ScheduleParams &p, cudaStream_t stream);
 // Vocabulary-sharded path (shard.cu): the slice's per-row records, and the
@@ -255,11 +256,16 @@ __host__ __device__ inline int32_t scan_warps(int64_t W_max, int64_t T, int64_t 
     return static_cast<int32_t>(w > 1 ? w : 1);
 }
 
-// The pipelined round (sdd_block_pipelined): warps 0-1 of every CTA (a team
-// of kPipeTeam threads) run the previous round's decide work while warps
-// 2-15 stream.
-constexpr int kPipeTeam = 64;
-constexpr int kPipeWarps = kPipeTeam / 32;
+// The pipelined round (sdd_block_pipelined): the first warps of every CTA (a
+// team of 64 threads, or 128 after a round of at most kPipeSmallBytes of
+// logits) run the previous round's decide work while the others stream.  A
+// round that small is latency-bound: its decide items are few and each takes
+// longer than its streaming pass (GB300, one 32 x 151,936 bf16 block: 23.8
+// us per round with a 128-thread team, 27.9 us with 64; one 8 x 32,000 fp32
+// block: 22.8 / 24.2 us), while at 16 blocks the two more streaming warps
+// win (61.2 against 63.5 us).
+constexpr int kPipeTeam = 64, kPipeTeamSmall = 128;
+constexpr int64_t kPipeSmallBytes = int64_t(64) << 20;
 // The pipelined pass's cost weights (drafter, target vector), as kCostDrafter
 // and kCostTarget for the streaming kernel: on fourteen warps beside the
 // decide work the drafter rows' entropy work weighs more (GB300, 16-block
