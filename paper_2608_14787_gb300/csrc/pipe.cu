@@ -7,16 +7,16 @@
 // streaming pass it leaves the memory system idle for most of its ~12 us.
 // Rounds over independent batches need not wait for one another, so here the
 // decide work of round n-1 runs beside the streaming pass of round n: in every
-// CTA, warps 0-1 do one (block, draw segment) item of round n-1's decide work
-// (decide_cta with a team of kPipeTeam threads and its barrier over those
-// threads only) while warps 2-15 stream round n, the rows divided among
-// fourteen warps per CTA.  Measured on GB300 (16 blocks of 32 positions, V =
-// 151,936 bf16, back to back): 62.7 us per round against 69.0 us for the
-// streaming and decide kernels in turn.  A team of eight decide warps beside
-// eight streaming warps (which then streamed a share cut to its decide time)
-// gave 71-75 us, four decide warps beside twelve 63.5-64.0 us; with two, a
-// decide item takes ~41 us under the concurrent stream, still before the
-// streaming warps end.
+// CTA, the first warps (a team of kPipeTeam = 64 threads; kPipeTeamSmall =
+// 128 when round n is a small, latency-bound one) do one (block, draw
+// segment) item of round n-1's decide work (decide_cta, its barrier over the
+// team only) while the other warps stream round n, the rows divided among
+// them.  Measured on GB300 (16 blocks of 32 positions, V = 151,936 bf16, back
+// to back): 61.2 us per round against 69.0 us for the streaming and decide
+// kernels in turn.  A team of eight decide warps beside eight streaming warps
+// (which then streamed a share cut to its decide time) gave 71-75 us, four
+// decide warps beside twelve 63.5-64.0 us; with two, a decide item takes ~42
+// us under the concurrent stream, still before the streaming warps end.
 // Round n-1's partials were written by the previous launch on the stream,
 // which has completed when this grid passes griddepcontrol.wait.
 #include <algorithm>
