@@ -566,7 +566,9 @@ SDD_API sdd_status_t sdd_block_decide(const sdd_block_args *args, sdd_stream_t s
 
 /*
  * sdd_block_pipelined -- rounds of sdd_block over independent batches, two at
- * a time in one launch: the streaming pass of `next` and, on the same SMs,
+ * a time in one launch (no counterpart in the paper: it computes what
+ * sdd_block computes, Sec. 3.1, 3.2 and 4.1, scheduled differently on the
+ * GPU): the streaming pass of `next` and, on the same SMs,
  * the decide work (sdd_block_decide's) of `prev`, whose streaming pass ran
  * in the previous sdd_block_pipelined call on this stream.  The decide work
  * of a round is latency-bound (row finalisation, the rules, the sampling
