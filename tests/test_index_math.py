@@ -150,3 +150,38 @@ def test_partition_cost_against_its_definition():
                 # the owner of v: the warp whose cost interval holds cost(v)
                 w = owner(v)
                 assert (w * C) // w_ <= cost(v) < ((w + 1) * C) // w_, (RV, R, v)
+
+
+def _scan_warps(W_max, T, rows, per_row=16):
+    """scan_warps of csrc/internal.h."""
+    w = min(W_max, T // 2, rows * per_row)
+    return max(w, 1)
+
+
+def test_pipelined_pass_partitions():
+    """The pipelined round streams on fourteen (or, after a small round,
+    twelve) warps per CTA with drafter : target weights 21 : 18 and a
+    row-start cost of 400 drafter vectors: every warp's range is non-empty
+    and the owner of every vector agrees with the starts (the decide merges
+    the partials of warps first_owner .. last_owner of each row)."""
+    rng = np.random.default_rng(12)
+    RV = 18992                                      # 151,936 bf16 entries per row
+    cases = []
+    for B, gamma, wpc in ((16, 32, 14), (24, 32, 14), (1, 32, 12), (5, 8, 12), (16, 64, 14)):
+        rows0, rows1 = B * gamma, B * (gamma + 1)
+        T = (rows0 + rows1) * RV
+        W = _scan_warps(152 * wpc, T, rows0 + rows1)
+        R = 400 * 21
+        if RV < 32 or 18 * RV + R < 16 * (R + 2 * 21):   # set_divisors keeps no row-start cost
+            R = 0
+        cases.append((rows0 * RV, rows1 * RV, W, RV, R))
+    cases.append((1 * 8 * 2000, 1 * 9 * 2000, _scan_warps(152 * 12, 17 * 2000, 17), 2000, 0))
+    for T0, T1, W, rv, R in cases:
+        T, start, owner, _, C = _weighted(T0, T1, W, 21, 18, rv, R)
+        s = [start(w) for w in range(W + 1)]
+        assert s[0] == 0 and s[W] == T
+        assert all(s[w + 1] > s[w] for w in range(W)), ("empty warp", T0, T1, W, rv, R)
+        probe = set(rng.integers(0, T, 3000).tolist()) | set(s[:-1]) | {x - 1 for x in s[1:]}
+        for v in probe:
+            w = owner(int(v))
+            assert s[w] <= v < s[w + 1], (T0, T1, W, v, w)
